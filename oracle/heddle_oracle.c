@@ -1,0 +1,564 @@
+/*
+ * heddle_oracle.c -- CPU oracle for Heddle's batched candidate-plan pricing.
+ *
+ * TEST INFRASTRUCTURE ONLY (see heddle_oracle.h).  Every step is written as
+ * the plain definition it restates, in the order the paper describes it:
+ *
+ *   cost table   §5.2 "Throughput estimation": one entry per (GPU type, TP
+ *                degree) gives the per-layer computation and communication
+ *                cost.  Quantised here to whole nanoseconds.
+ *   DP degree    §5.3 "Layer split and DP degree" and §5.1 "Non-uniform GPU
+ *                composition support": pack each stage's TP group into nodes
+ *                of its type, a group never crossing a node; take the largest
+ *                replication count the packing admits.  Computed here by
+ *                explicit first-fit-decreasing placement.
+ *   partition    §3.1 listing, PartitionLayers: split the layers into S
+ *                contiguous non-empty stages minimising the largest stage
+ *                time, with the memory validation of §5.2.  Computed here by
+ *                the textbook O(S L^2) dynamic programme.
+ *   evaluate     §5.3 iteration time of a 1F1B pipeline,
+ *                (M-1) max_s t_s + sum_s t_s + max_s g_s.
+ *   rank, top-k  §5 overview: plans are ranked by predicted throughput.
+ *
+ * Readings of points the paper leaves open (quantisation, P2P, memory and
+ * gradient-sync formulas, tie-breaks) are the ones listed in the design
+ * notes; each is restated beside the code that applies it.
+ *
+ * Build: gcc -std=c11 -O2 -ffp-contract=off (no fused multiply-add, so the
+ * double arithmetic of the quantiser is the plain IEEE sequence written).
+ */
+#include "heddle_oracle.h"
+
+#include <math.h>
+#include <pthread.h>
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define MAXT 8
+#define MAXS 32
+#define MAXL 255
+#define INF INT64_MAX
+
+typedef unsigned __int128 u128;
+
+struct orc_ctx {
+    int n_types, L, moe;
+    int64_t gpus[MAXT];      /* GPUs of each type */
+    int32_t maxnode[MAXT];   /* largest node of each type */
+    int64_t inter_bw[MAXT];  /* slowest NIC among the nodes of each type */
+    int64_t intra_bw[MAXT];
+    int64_t mem[MAXT];
+    int n_nodes;
+    int32_t* node_type;
+    int32_t* node_gpus;
+    int64_t* q;      /* [n_types][4][L] quantised per-layer ns */
+    int64_t* P;      /* [n_types][4][L+1] prefix sums of q */
+    int64_t* state;  /* [L+1] prefix of state bytes */
+    int64_t* act;    /* [L+1] prefix of stored activation bytes */
+    int64_t* param;  /* [L+1] prefix of gradient (parameter) bytes */
+    int64_t p2p[MAXT][MAXT][2];
+};
+
+/* ---------------------------------------------------------------- tables */
+
+/* Nearest nanosecond, halves away from zero (C99 llround). */
+static int64_t to_ns(double seconds) { return (int64_t)llround(seconds * 1e9); }
+
+/* ceil(a / b) for a >= 0, b > 0 in 128-bit arithmetic. */
+static int64_t ceil_div128(u128 a, u128 b) { return (int64_t)((a + b - 1) / b); }
+
+/* Per-layer time in seconds of layer l on one GPU group of type g and degree
+ * k = 2^j (§5.2: computation plus communication of one layer).  Synthetic
+ * stand-in for a profile entry:
+ *   compute  flops / (k * TFLOPS * 1e12)
+ *   TP       k > 1: four ring all-reduces (two forward, two backward) of
+ *            ar_bytes, each moving 2(k-1)/k of the message
+ *   EP       k > 1: four all-to-alls (dispatch and combine, forward and
+ *            backward) of a2a_bytes, each moving (k-1)/k of the message
+ * Both collectives use the type's intra-node bandwidth when the group fits
+ * in one node, else the node NIC bandwidth (an EP group may leave a node,
+ * §5.3 "Expert tiling"). */
+static double layer_seconds(const orc_ctx* x, int g, int j, double flops, int64_t ar,
+                            int64_t a2a, double tflops) {
+    double k = (double)(1 << j);
+    double s = flops / (k * tflops * 1e12);
+    if (j > 0) {
+        double bw = (1 << j) <= x->maxnode[g] ? (double)x->intra_bw[g] : (double)x->inter_bw[g];
+        double ring = (2.0 * (k - 1.0)) / k;
+        double t = 4.0 * ring;
+        t = t * (double)ar;
+        t = t / bw;
+        s = s + t;
+        double part = (k - 1.0) / k;
+        t = 4.0 * part;
+        t = t * (double)a2a;
+        t = t / bw;
+        s = s + t;
+    }
+    return s;
+}
+
+orc_ctx* orc_create(int n_types, const double* tflops, const int64_t* mem_bytes,
+                    const int64_t* intra_bw, int n_nodes, const int32_t* node_type,
+                    const int32_t* node_gpus, const int64_t* node_nic, int n_layers,
+                    const double* flops, const int64_t* param_bytes,
+                    const int64_t* state_bytes, const int64_t* act_bytes,
+                    const int64_t* ar_bytes, const int64_t* a2a_bytes,
+                    int64_t boundary_bytes, int moe, const double* profile_s, char* err) {
+    if (n_types < 1 || n_types > MAXT || n_layers < 1 || n_layers > MAXL || n_nodes < 1) {
+        if (err) snprintf(err, 256, "size out of range");
+        return NULL;
+    }
+    orc_ctx* x = (orc_ctx*)calloc(1, sizeof(orc_ctx));
+    int L = n_layers;
+    x->n_types = n_types;
+    x->L = L;
+    x->moe = moe != 0;
+    x->n_nodes = n_nodes;
+    x->node_type = (int32_t*)malloc(sizeof(int32_t) * n_nodes);
+    x->node_gpus = (int32_t*)malloc(sizeof(int32_t) * n_nodes);
+    memcpy(x->node_type, node_type, sizeof(int32_t) * n_nodes);
+    memcpy(x->node_gpus, node_gpus, sizeof(int32_t) * n_nodes);
+    for (int g = 0; g < n_types; ++g) {
+        x->gpus[g] = 0;
+        x->maxnode[g] = 0;
+        x->inter_bw[g] = INT64_MAX;
+        x->intra_bw[g] = intra_bw[g];
+        x->mem[g] = mem_bytes[g];
+    }
+    for (int b = 0; b < n_nodes; ++b) {
+        int g = node_type[b];
+        if (g < 0 || g >= n_types || node_gpus[b] < 1) {
+            if (err) snprintf(err, 256, "bad node %d", b);
+            orc_destroy(x);
+            return NULL;
+        }
+        x->gpus[g] += node_gpus[b];
+        if (node_gpus[b] > x->maxnode[g]) x->maxnode[g] = node_gpus[b];
+        if (node_nic[b] < x->inter_bw[g]) x->inter_bw[g] = node_nic[b];
+    }
+    for (int g = 0; g < n_types; ++g)
+        if (x->gpus[g] == 0) x->inter_bw[g] = 0; /* absent type: never priced */
+
+    size_t nq = (size_t)n_types * 4 * L;
+    x->q = (int64_t*)calloc(nq, sizeof(int64_t));
+    x->P = (int64_t*)calloc((size_t)n_types * 4 * (L + 1), sizeof(int64_t));
+    for (int g = 0; g < n_types; ++g) {
+        if (x->gpus[g] == 0) continue; /* tables of absent types stay zero */
+        for (int j = 0; j < 4; ++j) {
+            int64_t* q = x->q + ((size_t)g * 4 + j) * L;
+            int64_t* P = x->P + ((size_t)g * 4 + j) * (L + 1);
+            P[0] = 0;
+            for (int l = 0; l < L; ++l) {
+                double sec = profile_s
+                                 ? profile_s[((size_t)g * 4 + j) * L + l]
+                                 : layer_seconds(x, g, j, flops[l], ar_bytes[l], a2a_bytes[l],
+                                                 tflops[g]);
+                q[l] = to_ns(sec);
+                P[l + 1] = P[l] + q[l];
+            }
+        }
+    }
+    x->state = (int64_t*)calloc(L + 1, sizeof(int64_t));
+    x->act = (int64_t*)calloc(L + 1, sizeof(int64_t));
+    x->param = (int64_t*)calloc(L + 1, sizeof(int64_t));
+    for (int l = 0; l < L; ++l) {
+        x->state[l + 1] = x->state[l] + state_bytes[l];
+        x->act[l + 1] = x->act[l] + act_bytes[l];
+        x->param[l + 1] = x->param[l] + param_bytes[l];
+    }
+    /* Inter-stage P2P (reading): forward activation plus backward gradient,
+     * 2 * boundary bytes, over the intra-node link when both stages are the
+     * same type and the two groups fit in one node, else over the slower of
+     * the two types' NICs. */
+    for (int g = 0; g < MAXT; ++g)
+        for (int h = 0; h < MAXT; ++h)
+            for (int same = 0; same < 2; ++same) {
+                int64_t bw = 0;
+                if (g < n_types && h < n_types && x->gpus[g] && x->gpus[h]) {
+                    if (same)
+                        bw = x->intra_bw[g];
+                    else
+                        bw = x->inter_bw[g] < x->inter_bw[h] ? x->inter_bw[g] : x->inter_bw[h];
+                }
+                x->p2p[g][h][same] =
+                    bw > 0 ? ceil_div128((u128)2 * (u128)boundary_bytes * 1000000000u, (u128)bw)
+                           : 0;
+            }
+    return x;
+}
+
+void orc_destroy(orc_ctx* x) {
+    if (!x) return;
+    free(x->node_type);
+    free(x->node_gpus);
+    free(x->q);
+    free(x->P);
+    free(x->state);
+    free(x->act);
+    free(x->param);
+    free(x);
+}
+
+void orc_tables(const orc_ctx* x, int64_t* q, int64_t* p2p, int32_t* maxnode,
+                int64_t* inter_bw) {
+    if (q) memcpy(q, x->q, sizeof(int64_t) * (size_t)x->n_types * 4 * x->L);
+    if (p2p) memcpy(p2p, x->p2p, sizeof(x->p2p));
+    for (int g = 0; g < x->n_types; ++g) {
+        if (maxnode) maxnode[g] = x->maxnode[g];
+        if (inter_bw) inter_bw[g] = x->inter_bw[g];
+    }
+}
+
+/* ------------------------------------------------------------- DP degree */
+
+/* Can n replicas of the groups be placed?  First-fit decreasing: groups are
+ * taken from the largest size down, each into the first node (in list order)
+ * with enough free GPUs.  Equal-size groups are placed as a batch, which is
+ * what placing them one at a time first-fit does. */
+static int ffd_fits(int n_nodes, const int32_t* node_gpus, const int64_t* count_by_size,
+                    int64_t n) {
+    int64_t* rem = (int64_t*)malloc(sizeof(int64_t) * (n_nodes > 0 ? n_nodes : 1));
+    for (int b = 0; b < n_nodes; ++b) rem[b] = node_gpus[b];
+    int ok = 1;
+    for (int e = 3; e >= 0 && ok; --e) {
+        int64_t w = (int64_t)1 << e;
+        int64_t left = count_by_size[e] * n;
+        for (int b = 0; b < n_nodes && left > 0; ++b) {
+            int64_t take = rem[b] / w;
+            if (take > left) take = left;
+            rem[b] -= take * w;
+            left -= take;
+        }
+        if (left > 0) ok = 0;
+    }
+    free(rem);
+    return ok;
+}
+
+/* Largest n such that n replicas fit (0 if not even one does). */
+static int64_t replicas(int n_nodes, const int32_t* node_gpus, const int64_t* count_by_size) {
+    int64_t any = 0, total = 0;
+    for (int e = 0; e < 4; ++e) any += count_by_size[e];
+    for (int b = 0; b < n_nodes; ++b) total += node_gpus[b];
+    if (any == 0) return INT64_MAX; /* this type hosts no stage */
+    int64_t n = 0;
+    while (n < total && ffd_fits(n_nodes, node_gpus, count_by_size, n + 1)) ++n;
+    return n;
+}
+
+int orc_replicas(int n_nodes, const int32_t* node_gpus, int n_groups,
+                 const int32_t* group_gpus) {
+    int64_t cnt[4] = {0, 0, 0, 0};
+    for (int i = 0; i < n_groups; ++i) {
+        int e = 0;
+        while (e < 3 && (1 << e) < group_gpus[i]) ++e;
+        cnt[e] += 1;
+    }
+    int64_t n = replicas(n_nodes, node_gpus, cnt);
+    return n == INT64_MAX ? 0 : (int)n;
+}
+
+/* DP degree of a candidate: the replication count every GPU type admits.
+ * A stage group of degree k larger than the largest node of its type (only
+ * possible for an EP degree, §5.3) is placed as k/p blocks of p GPUs, p the
+ * largest power of two not above that node size (reading). */
+static int64_t dp_degree(const orc_ctx* x, int S, const int* g, const int* j) {
+    int64_t best = INT64_MAX;
+    int32_t* ng = (int32_t*)malloc(sizeof(int32_t) * x->n_nodes);
+    for (int t = 0; t < x->n_types; ++t) {
+        int64_t cnt[4] = {0, 0, 0, 0};
+        int used = 0;
+        for (int s = 0; s < S; ++s) {
+            if (g[s] != t) continue;
+            used = 1;
+            int k = 1 << j[s];
+            int e = j[s];
+            while ((1 << e) > x->maxnode[t]) --e;
+            cnt[e] += k >> e;
+        }
+        if (!used) continue;
+        int nn = 0;
+        for (int b = 0; b < x->n_nodes; ++b)
+            if (x->node_type[b] == t) ng[nn++] = x->node_gpus[b];
+        int64_t r = replicas(nn, ng, cnt);
+        if (r < best) best = r;
+    }
+    free(ng);
+    return best == INT64_MAX ? 0 : best;
+}
+
+/* --------------------------------------------------------- PartitionLayers */
+
+/* f[s][i]: smallest achievable largest stage time of stages s..S-1 covering
+ * layers [i, L), INF if they cannot.  B* = f[0][0].  The canonical optimum is
+ * the lexicographically smallest boundary vector: walk s = 0..S-1 taking the
+ * smallest next boundary j whose stage fits, costs at most B*, and whose
+ * remainder can still finish within B*. */
+static int partition(int S, int L, const int64_t* const* P, const int64_t* c,
+                     const int64_t* const* W, const int64_t* cap, int64_t* f,
+                     int64_t* Bstar, int32_t* a) {
+#define F(s, i) f[(size_t)(s) * (L + 1) + (i)]
+    for (int i = 0; i <= L; ++i) F(S, i) = (i == L) ? 0 : INF;
+    for (int s = S - 1; s >= 0; --s) {
+        for (int i = 0; i <= L; ++i) {
+            int64_t best = INF;
+            for (int j = i + 1; j <= L; ++j) {
+                if (F(s + 1, j) == INF) continue;
+                if (W[s][j] - W[s][i] > cap[s]) continue;
+                int64_t t = P[s][j] - P[s][i] + c[s];
+                int64_t v = t > F(s + 1, j) ? t : F(s + 1, j);
+                if (v < best) best = v;
+            }
+            F(s, i) = best;
+        }
+    }
+    int64_t B = F(0, 0);
+    if (B == INF) return 0;
+    *Bstar = B;
+    a[0] = 0;
+    for (int s = 0; s < S; ++s) {
+        int i = a[s], chosen = -1;
+        for (int j = i + 1; j <= L; ++j) {
+            if (F(s + 1, j) > B) continue;
+            if (W[s][j] - W[s][i] > cap[s]) continue;
+            if (P[s][j] - P[s][i] + c[s] > B) continue;
+            chosen = j;
+            break;
+        }
+        a[s + 1] = chosen; /* exists because f[s][a_s] <= B */
+    }
+    return 1;
+#undef F
+}
+
+int orc_partition_raw(int S, int L, const int64_t* P, const int64_t* c, const int64_t* W,
+                      const int64_t* cap, int64_t* Bstar, int32_t* a) {
+    if (S < 1 || L < 1) return 0;
+    const int64_t** Pp = (const int64_t**)malloc(sizeof(int64_t*) * S);
+    const int64_t** Wp = (const int64_t**)malloc(sizeof(int64_t*) * S);
+    for (int s = 0; s < S; ++s) {
+        Pp[s] = P + (size_t)s * (L + 1);
+        Wp[s] = W + (size_t)s * (L + 1);
+    }
+    int64_t* f = (int64_t*)malloc(sizeof(int64_t) * (size_t)(S + 1) * (L + 1));
+    int ok = partition(S, L, Pp, c, Wp, cap, f, Bstar, a);
+    free(f);
+    free(Pp);
+    free(Wp);
+    return ok;
+}
+
+/* ------------------------------------------------------ price one candidate */
+
+typedef struct {
+    int64_t T, B;
+    int64_t n;
+    int status;
+    int32_t a[MAXS + 1];
+} priced;
+
+static void price_one(const orc_ctx* x, int S, int M, const uint8_t* codes, int64_t* f,
+                      int64_t* Wbuf, priced* out) {
+    int L = x->L;
+    memset(out, 0, sizeof(*out));
+    out->T = -1;
+    out->B = -1;
+    /* decode and validate the structural template (§5.1 masks) */
+    int g[MAXS], j[MAXS];
+    if (S < 1 || S > MAXS || S > L || M < 1) {
+        out->status = ORC_INVALID;
+        return;
+    }
+    for (int s = 0; s < S; ++s) {
+        int b = codes[s];
+        g[s] = b & 7;
+        j[s] = (b >> 3) & 3;
+        if ((b >> 5) != 0 || g[s] >= x->n_types || x->gpus[g[s]] == 0 ||
+            (!x->moe && (1 << j[s]) > x->maxnode[g[s]])) {
+            out->status = ORC_INVALID;
+            return;
+        }
+    }
+    /* DP degree (§5.3) */
+    int64_t n = dp_degree(x, S, g, j);
+    if (n == 0) {
+        out->status = ORC_NO_FIT;
+        return;
+    }
+    out->n = n;
+    /* stage views for PartitionLayers */
+    const int64_t* P[MAXS];
+    const int64_t* W[MAXS];
+    int64_t c[MAXS], cap[MAXS];
+    for (int s = 0; s < S; ++s) {
+        P[s] = x->P + ((size_t)g[s] * 4 + j[s]) * (L + 1);
+        if (s + 1 < S) {
+            int same = g[s] == g[s + 1] && (1 << j[s]) + (1 << j[s + 1]) <= x->maxnode[g[s]];
+            c[s] = x->p2p[g[s]][g[s + 1]][same];
+        } else {
+            c[s] = 0;
+        }
+        /* memory (§5.2): parameters, gradients and optimizer state of the
+         * stage's layers plus the activations of its in-flight microbatches
+         * (1F1B keeps min(S - s, M) on stage s), all split over the k GPUs of
+         * the group; compared as total <= capacity * k */
+        int64_t inflight = (S - s) < M ? (S - s) : M;
+        int64_t* w = Wbuf + (size_t)s * (L + 1);
+        for (int i = 0; i <= L; ++i) w[i] = x->state[i] + inflight * x->act[i];
+        W[s] = w;
+        cap[s] = x->mem[g[s]] * (int64_t)(1 << j[s]);
+    }
+    int64_t B;
+    if (!partition(S, L, P, c, W, cap, f, &B, out->a)) {
+        out->status = ORC_OOM;
+        return;
+    }
+    /* Evaluate (§5.3): T = (M-1) max t_s + sum t_s + max g_s */
+    int64_t tmax = 0, tsum = 0, gmax = 0;
+    for (int s = 0; s < S; ++s) {
+        int64_t t = P[s][out->a[s + 1]] - P[s][out->a[s]] + c[s];
+        if (t > tmax) tmax = t;
+        tsum += t;
+        /* DP gradient synchronisation of stage s (reading): a ring all-reduce
+         * over the n replicas of the stage's gradient shard (G_s / k bytes),
+         * 2(n-1)/n of it over the slowest NIC of the type, in whole ns
+         * rounded up; zero without replication */
+        int64_t gs = 0;
+        if (n > 1) {
+            int64_t G = x->param[out->a[s + 1]] - x->param[out->a[s]];
+            u128 num = (u128)2 * (u128)(n - 1) * (u128)G * 1000000000u;
+            u128 den = (u128)n * (u128)(1 << j[s]) * (u128)x->inter_bw[g[s]];
+            gs = ceil_div128(num, den);
+        }
+        if (gs > gmax) gmax = gs;
+    }
+    out->B = B;
+    out->T = (int64_t)(M - 1) * tmax + tsum + gmax;
+    out->status = ORC_OK;
+}
+
+typedef struct {
+    const orc_ctx* x;
+    int64_t lo, hi;
+    const uint8_t* S;
+    const uint16_t* M;
+    const uint8_t* code;
+    int64_t stride;
+    int s_max;
+    int64_t *T, *B;
+    uint16_t* n_dp;
+    uint8_t *status, *bounds;
+    int64_t n_all;
+} job;
+
+static void* run_job(void* arg) {
+    job* jb = (job*)arg;
+    const orc_ctx* x = jb->x;
+    int L = x->L;
+    int64_t* f = (int64_t*)malloc(sizeof(int64_t) * (size_t)(MAXS + 1) * (L + 1));
+    int64_t* Wbuf = (int64_t*)malloc(sizeof(int64_t) * (size_t)MAXS * (L + 1));
+    uint8_t codes[MAXS];
+    for (int64_t c = jb->lo; c < jb->hi; ++c) {
+        int S = jb->S[c];
+        priced r;
+        if (S > jb->s_max) {
+            memset(&r, 0, sizeof(r));
+            r.T = r.B = -1;
+            r.status = ORC_INVALID;
+        } else {
+            for (int s = 0; s < S && s < MAXS; ++s) codes[s] = jb->code[(int64_t)s * jb->stride + c];
+            price_one(x, S, jb->M[c], codes, f, Wbuf, &r);
+        }
+        jb->T[c] = r.T;
+        jb->B[c] = r.B;
+        jb->n_dp[c] = (uint16_t)(r.status == ORC_OK || r.status == ORC_OOM ? r.n : 0);
+        jb->status[c] = (uint8_t)r.status;
+        if (jb->bounds) {
+            for (int s = 0; s <= MAXS; ++s)
+                jb->bounds[(int64_t)s * jb->n_all + c] =
+                    (r.status == ORC_OK && s <= S) ? (uint8_t)r.a[s] : 0;
+        }
+    }
+    free(f);
+    free(Wbuf);
+    return NULL;
+}
+
+int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
+              const uint8_t* code, int64_t plane_stride, int s_max, int64_t* T,
+              int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
+              int threads) {
+    if (threads < 1) threads = 1;
+    if (threads > n) threads = n > 0 ? (int)n : 1;
+    job* jobs = (job*)calloc(threads, sizeof(job));
+    pthread_t* tid = (pthread_t*)calloc(threads, sizeof(pthread_t));
+    for (int t = 0; t < threads; ++t) {
+        job* jb = &jobs[t];
+        jb->x = x;
+        jb->lo = n * t / threads;
+        jb->hi = n * (t + 1) / threads;
+        jb->S = S;
+        jb->M = M;
+        jb->code = code;
+        jb->stride = plane_stride;
+        jb->s_max = s_max;
+        jb->T = T;
+        jb->B = bottleneck;
+        jb->n_dp = n_dp;
+        jb->status = status;
+        jb->bounds = bounds;
+        jb->n_all = n;
+    }
+    if (threads == 1) {
+        run_job(&jobs[0]);
+    } else {
+        for (int t = 0; t < threads; ++t) pthread_create(&tid[t], NULL, run_job, &jobs[t]);
+        for (int t = 0; t < threads; ++t) pthread_join(tid[t], NULL);
+    }
+    free(jobs);
+    free(tid);
+    return threads;
+}
+
+/* ------------------------------------------------------------ rank, top-k */
+
+typedef struct {
+    int64_t idx, T;
+    uint32_t nM;
+} entry;
+
+/* a before b: higher throughput nM/T, compared exactly as nM_a*T_b vs
+ * nM_b*T_a; equal throughput goes to the smaller index. */
+static int better_first(const void* pa, const void* pb) {
+    const entry* a = (const entry*)pa;
+    const entry* b = (const entry*)pb;
+    u128 lhs = (u128)a->nM * (u128)b->T;
+    u128 rhs = (u128)b->nM * (u128)a->T;
+    if (lhs != rhs) return lhs > rhs ? -1 : 1;
+    return a->idx < b->idx ? -1 : (a->idx > b->idx ? 1 : 0);
+}
+
+int orc_topk(int64_t n, int64_t base_index, const int64_t* T, const uint16_t* n_dp,
+             const uint16_t* M, const uint8_t* status, int k, int64_t* out_idx,
+             int64_t* out_T, uint32_t* out_nM) {
+    entry* e = (entry*)malloc(sizeof(entry) * (size_t)(n > 0 ? n : 1));
+    int64_t m = 0;
+    for (int64_t c = 0; c < n; ++c) {
+        if (status[c] != ORC_OK) continue;
+        e[m].idx = base_index + c;
+        e[m].T = T[c];
+        e[m].nM = (uint32_t)n_dp[c] * (uint32_t)M[c];
+        ++m;
+    }
+    qsort(e, (size_t)m, sizeof(entry), better_first);
+    int cnt = (int)(m < k ? m : k);
+    for (int i = 0; i < cnt; ++i) {
+        out_idx[i] = e[i].idx;
+        out_T[i] = e[i].T;
+        out_nM[i] = e[i].nM;
+    }
+    free(e);
+    return cnt;
+}

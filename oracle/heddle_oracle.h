@@ -1,0 +1,80 @@
+/*
+ * heddle_oracle.h -- CPU oracle for Heddle's batched candidate-plan pricing.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This is a plain, slow, obviously-correct
+ * restatement of the cost model of the paper (arxiv 2609.34244, §3.1 nested
+ * search listing, §5.1 structural templates, §5.2 cost model, §5.3 auto-fill
+ * and the 1F1B iteration time).  Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline / reference arm may load it.  It shares no code,
+ * header, table or helper with the CUDA library; both only read the same
+ * seeded input arrays.
+ *
+ * All inputs are plain arrays (structure of arrays).  Times are int64
+ * nanoseconds after quantisation, bytes are int64, bandwidths int64 bytes/s.
+ */
+#ifndef HEDDLE_ORACLE_H
+#define HEDDLE_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ORC_OK 0
+#define ORC_OOM 1
+#define ORC_NO_FIT 2
+#define ORC_INVALID 3
+
+typedef struct orc_ctx orc_ctx;
+
+/* Build the oracle's cost model for one cluster and one model.
+ * profile_s: nullable [n_types][4][n_layers] seconds per layer at degree 2^j.
+ * Returns NULL on malformed input (a message is written to err, 256 bytes). */
+orc_ctx* orc_create(int n_types, const double* tflops, const int64_t* mem_bytes,
+                    const int64_t* intra_bw, int n_nodes, const int32_t* node_type,
+                    const int32_t* node_gpus, const int64_t* node_nic, int n_layers,
+                    const double* flops, const int64_t* param_bytes,
+                    const int64_t* state_bytes, const int64_t* act_bytes,
+                    const int64_t* ar_bytes, const int64_t* a2a_bytes,
+                    int64_t boundary_bytes, int moe, const double* profile_s, char* err);
+void orc_destroy(orc_ctx* x);
+
+/* Quantised tables: q[n_types][4][L] per-layer ns, p2p[8][8][2] ns
+ * (from type, to type, same-node flag), present/maxnode/inter_bw per type. */
+void orc_tables(const orc_ctx* x, int64_t* q, int64_t* p2p, int32_t* maxnode,
+                int64_t* inter_bw);
+
+/* Price candidates [0, n): S[n], M[n], code[s * plane_stride + c] for
+ * s < s_max.  Outputs T, bottleneck, n_dp, status and (nullable) bounds
+ * [33][n].  threads <= 0 means one thread.  Returns the threads used. */
+int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
+              const uint8_t* code, int64_t plane_stride, int s_max, int64_t* T,
+              int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
+              int threads);
+
+/* Top-k of the OK candidates by throughput n*M/T, ties to the smaller index.
+ * idx = base_index + c.  Writes up to k entries; returns how many. */
+int orc_topk(int64_t n, int64_t base_index, const int64_t* T, const uint16_t* n_dp,
+             const uint16_t* M, const uint8_t* status, int k, int64_t* out_idx,
+             int64_t* out_T, uint32_t* out_nM);
+
+/* Min-max contiguous partition of L layers into S non-empty stages, stated
+ * on raw integer inputs (test hook).  Stage s costs P[s][j] - P[s][i] + c[s]
+ * and fits iff W[s][j] - W[s][i] <= cap[s]; P and W are [S][L+1].
+ * Returns 1 and writes B* and the lexicographically smallest optimal
+ * boundary vector a[0..S] if a valid partition exists, else returns 0. */
+int orc_partition_raw(int S, int L, const int64_t* P, const int64_t* c, const int64_t* W,
+                      const int64_t* cap, int64_t* Bstar, int32_t* a);
+
+/* Largest replication count n for which n copies of every group (sizes
+ * group_gpus[0..n_groups)) can be placed on nodes of node_gpus[0..n_nodes)
+ * without a group crossing a node (one GPU type).  Group sizes must be
+ * powers of two. */
+int orc_replicas(int n_nodes, const int32_t* node_gpus, int n_groups,
+                 const int32_t* group_gpus);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,170 @@
+"""ctypes wrapper around the CPU oracle (``heddle_oracle.c``).
+
+TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline / reference arm are the only callers.  The product
+path never imports this module.
+
+The oracle takes the same seeded input dictionaries as the CUDA library (see
+``paper_2609_34244_gb300.workloads``) and returns numpy arrays.
+"""
+
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+SRC = os.path.join(HERE, "heddle_oracle.c")
+HDR = os.path.join(HERE, "heddle_oracle.h")
+LIB = os.path.join(HERE, "liboracle.so")
+
+OK, OOM, NO_FIT, INVALID = 0, 1, 2, 3
+
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile ``liboracle.so`` with gcc (no fused multiply-add)."""
+    newest = max(os.path.getmtime(SRC), os.path.getmtime(HDR))
+    if force or not os.path.exists(LIB) or os.path.getmtime(LIB) < newest:
+        tmp = LIB + ".tmp%d" % os.getpid()
+        subprocess.check_call(["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fPIC", "-shared",
+                               "-o", tmp, SRC, "-lpthread", "-lm"])
+        os.replace(tmp, LIB)
+    return LIB
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        build()
+        L = C.CDLL(LIB)
+        p = C.c_void_p
+        L.orc_create.restype = p
+        L.orc_create.argtypes = [C.c_int, p, p, p, C.c_int, p, p, p, C.c_int, p, p, p, p, p, p,
+                                 C.c_int64, C.c_int, p, C.c_char_p]
+        L.orc_destroy.argtypes = [p]
+        L.orc_tables.argtypes = [p, p, p, p, p]
+        L.orc_price.restype = C.c_int
+        L.orc_price.argtypes = [p, C.c_int64, p, p, p, C.c_int64, C.c_int, p, p, p, p, p, C.c_int]
+        L.orc_topk.restype = C.c_int
+        L.orc_topk.argtypes = [C.c_int64, C.c_int64, p, p, p, p, C.c_int, p, p, p]
+        L.orc_partition_raw.restype = C.c_int
+        L.orc_partition_raw.argtypes = [C.c_int, C.c_int, p, p, p, p, p, p]
+        L.orc_replicas.restype = C.c_int
+        L.orc_replicas.argtypes = [C.c_int, p, C.c_int, p]
+        _lib = L
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(C.c_void_p)
+
+
+class Oracle:
+    """The oracle's cost model for one cluster and one model."""
+
+    def __init__(self, cluster: dict, model: dict):
+        L = lib()
+        self._keep = []
+
+        def arr(v, dt):
+            a = np.ascontiguousarray(v, dtype=dt)
+            self._keep.append(a)
+            return a
+
+        cl = {k: arr(cluster[k], dt) for k, dt in
+              (("tflops", np.float64), ("mem_bytes", np.int64), ("intra_bw", np.int64),
+               ("node_type", np.int32), ("node_gpus", np.int32), ("node_nic", np.int64))}
+        md = {k: arr(model[k], dt) for k, dt in
+              (("flops", np.float64), ("param_bytes", np.int64), ("state_bytes", np.int64),
+               ("act_bytes", np.int64), ("ar_bytes", np.int64), ("a2a_bytes", np.int64))}
+        prof = None if model.get("profile_s") is None else arr(model["profile_s"], np.float64)
+        err = C.create_string_buffer(256)
+        self.n_types = int(cl["tflops"].shape[0])
+        self.L = int(md["flops"].shape[0])
+        self._h = L.orc_create(self.n_types, _ptr(cl["tflops"]), _ptr(cl["mem_bytes"]),
+                               _ptr(cl["intra_bw"]), int(cl["node_type"].shape[0]),
+                               _ptr(cl["node_type"]), _ptr(cl["node_gpus"]), _ptr(cl["node_nic"]),
+                               self.L, _ptr(md["flops"]), _ptr(md["param_bytes"]),
+                               _ptr(md["state_bytes"]), _ptr(md["act_bytes"]), _ptr(md["ar_bytes"]),
+                               _ptr(md["a2a_bytes"]), int(model["boundary_bytes"]),
+                               int(bool(model.get("moe", False))), _ptr(prof), err)
+        if not self._h:
+            raise ValueError("oracle rejected inputs: " + err.value.decode())
+
+    def __del__(self):
+        h = getattr(self, "_h", None)
+        if h:
+            lib().orc_destroy(h)
+            self._h = None
+
+    def tables(self) -> dict:
+        """Quantised per-layer costs ``q[g, j, l]`` (ns), P2P constants
+        ``p2p[g, h, same]`` (ns), largest node and slowest NIC per type."""
+        q = np.zeros((self.n_types, 4, self.L), dtype=np.int64)
+        p2p = np.zeros((8, 8, 2), dtype=np.int64)
+        mx = np.zeros(self.n_types, dtype=np.int32)
+        bw = np.zeros(self.n_types, dtype=np.int64)
+        lib().orc_tables(self._h, _ptr(q), _ptr(p2p), _ptr(mx), _ptr(bw))
+        return {"q": q, "P": np.concatenate([np.zeros((self.n_types, 4, 1), np.int64),
+                                             np.cumsum(q, axis=2)], axis=2),
+                "p2p": p2p, "maxnode": mx, "inter_bw": bw}
+
+    def price(self, cands: dict, threads: int = 1, bounds: bool = True) -> dict:
+        """Price every candidate; returns T, bottleneck, n_dp, status, bounds[33, n]."""
+        S = np.ascontiguousarray(cands["S"], dtype=np.uint8)
+        M = np.ascontiguousarray(cands["M"], dtype=np.uint16)
+        code = np.ascontiguousarray(cands["code"], dtype=np.uint8)
+        n = int(S.shape[0])
+        s_max = int(code.shape[0])
+        out = {"T": np.zeros(n, np.int64), "bottleneck": np.zeros(n, np.int64),
+               "n_dp": np.zeros(n, np.uint16), "status": np.zeros(n, np.uint8),
+               "bounds": np.zeros((33, n), np.uint8) if bounds else None}
+        used = lib().orc_price(self._h, n, _ptr(S), _ptr(M), _ptr(code), n, s_max,
+                               _ptr(out["T"]), _ptr(out["bottleneck"]), _ptr(out["n_dp"]),
+                               _ptr(out["status"]), _ptr(out["bounds"]), int(threads))
+        out["threads"] = used
+        return out
+
+
+def topk(res: dict, M, k: int, base_index: int = 0) -> dict:
+    """Top-``k`` OK candidates by throughput n*M/T (ties: smaller index)."""
+    n = int(res["T"].shape[0])
+    T = np.ascontiguousarray(res["T"], dtype=np.int64)
+    nd = np.ascontiguousarray(res["n_dp"], dtype=np.uint16)
+    st = np.ascontiguousarray(res["status"], dtype=np.uint8)
+    Mm = np.ascontiguousarray(M, dtype=np.uint16)
+    idx = np.zeros(k, np.int64)
+    tt = np.zeros(k, np.int64)
+    nm = np.zeros(k, np.uint32)
+    cnt = lib().orc_topk(n, int(base_index), _ptr(T), _ptr(nd), _ptr(Mm), _ptr(st), int(k),
+                         _ptr(idx), _ptr(tt), _ptr(nm))
+    return {"count": cnt, "idx": idx[:cnt], "T": tt[:cnt], "nM": nm[:cnt]}
+
+
+def partition_raw(P, c, W=None, cap=None):
+    """Min-max contiguous partition on raw integer stage tables (test hook).
+
+    ``P``: [S][L+1] int64 cost prefixes, ``c``: [S] per-stage constants,
+    ``W``/``cap``: [S][L+1] memory prefixes and [S] capacities (default: no
+    memory limit).  Returns ``(B*, bounds)`` or ``None`` when no split fits."""
+    P = np.ascontiguousarray(P, dtype=np.int64)
+    S, L1 = P.shape
+    c = np.ascontiguousarray(c, dtype=np.int64)
+    W = np.zeros_like(P) if W is None else np.ascontiguousarray(W, dtype=np.int64)
+    cap = np.zeros(S, np.int64) if cap is None else np.ascontiguousarray(cap, dtype=np.int64)
+    B = np.zeros(1, np.int64)
+    a = np.zeros(S + 1, np.int32)
+    ok = lib().orc_partition_raw(S, L1 - 1, _ptr(P), _ptr(c), _ptr(W), _ptr(cap), _ptr(B), _ptr(a))
+    return (int(B[0]), a.tolist()) if ok else None
+
+
+def replicas(node_gpus, group_gpus) -> int:
+    """Largest replication count of ``group_gpus`` on ``node_gpus`` (one type)."""
+    ng = np.ascontiguousarray(node_gpus, dtype=np.int32)
+    gg = np.ascontiguousarray(group_gpus, dtype=np.int32)
+    return int(lib().orc_replicas(len(ng), _ptr(ng), len(gg), _ptr(gg)))

@@ -1,0 +1,342 @@
+"""Pins for the CPU oracle: each check compares the oracle against something
+other than itself -- hand-worked values (``tests/golden``), brute-force
+enumeration, closed forms and invariants.  Every check raises
+AssertionError on a mismatch.  ``test_oracle_pins.py`` runs them; the
+mutation test runs them against deliberately broken copies of the oracle and
+requires each copy to fail at least one.
+"""
+
+from __future__ import annotations
+
+import itertools
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+UNIT = 10**6  # hand examples count costs in units scaled to nanoseconds
+
+
+def _load(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+def _workloads():
+    from paper_2609_34244_gb300 import workloads as W
+    return W
+
+
+# ---------------------------------------------------------------- helpers
+
+def tables_from_scales(layers, scales, c, mem_layers=None, mem_cap=None):
+    """Raw stage tables: stage s costs scale_s * sum(layers) + c_s; memory
+    prefix of ``mem_layers`` (same for every stage) against ``mem_cap``."""
+    base = np.concatenate([[0], np.cumsum(np.asarray(layers, dtype=np.int64))])
+    P = np.stack([base * int(k) for k in scales])
+    if mem_layers is None:
+        W = np.zeros_like(P)
+        cap = np.zeros(len(scales), np.int64)
+    else:
+        m = np.concatenate([[0], np.cumsum(np.asarray(mem_layers, dtype=np.int64))])
+        W = np.stack([m for _ in scales])
+        cap = np.asarray(mem_cap, dtype=np.int64)
+    return P, np.asarray(c, dtype=np.int64), W, cap
+
+
+def brute_partition(P, c, W, cap):
+    """Every contiguous split into S non-empty stages, in lexicographic order
+    of the boundary vector; returns (B*, first optimal boundaries) or None."""
+    S, L1 = P.shape
+    L = L1 - 1
+    best = None
+    for cut in itertools.combinations(range(1, L), S - 1):
+        a = (0,) + cut + (L,)
+        ok = True
+        worst = 0
+        for s in range(S):
+            i, j = a[s], a[s + 1]
+            if W[s][j] - W[s][i] > cap[s]:
+                ok = False
+                break
+            worst = max(worst, int(P[s][j] - P[s][i] + c[s]))
+        if ok and (best is None or worst < best[0]):
+            best = (worst, list(a))
+    return best
+
+
+def brute_replicas(node_gpus, groups, limit=64):
+    """Largest n such that n copies of ``groups`` can be assigned to nodes
+    (exhaustive backtracking over assignments)."""
+    def fits(items, caps):
+        items = sorted(items, reverse=True)
+        caps = list(caps)
+
+        def rec(t):
+            if t == len(items):
+                return True
+            seen = set()
+            for b in range(len(caps)):
+                if caps[b] >= items[t] and caps[b] not in seen:
+                    seen.add(caps[b])
+                    caps[b] -= items[t]
+                    if rec(t + 1):
+                        return True
+                    caps[b] += items[t]
+            return False
+        return rec(0)
+
+    n = 0
+    while n < limit and fits(list(groups) * (n + 1), node_gpus):
+        n += 1
+    return n
+
+
+def oracle_for(O, case):
+    W = _workloads()
+    cl = case["cluster"]
+    cluster = W.make_cluster(cl["tflops"], cl["mem_bytes"], cl["intra_bw"],
+                             [tuple(x) for x in cl["nodes"]])
+    m = case["model"]
+    L = len(m["flops"])
+    model = W.make_model(m["flops"], m["param_bytes"], m["state_bytes"], m["act_bytes"],
+                         m["ar_bytes"], m["a2a_bytes"], m["boundary_bytes"], moe=m["moe"])
+    cands = W.from_structures([[tuple(s) for s in cd["stages"]] for cd in case["cands"]],
+                              [cd["M"] for cd in case["cands"]])
+    return O.Oracle(cluster, model), cands, L
+
+
+# ------------------------------------------------------------------- pins
+
+def check_hand_partitions(O):
+    """Hand-worked PartitionLayers examples (golden/hand_partition.json)."""
+    for case in _load("hand_partition.json")["cases"]:
+        P, c, W, cap = tables_from_scales(case["layers"], case["scales"], case["c"],
+                                          case.get("mem_layers"), case.get("mem_cap"))
+        got = O.partition_raw(P * UNIT, c * UNIT, W, cap)
+        if case["Bstar"] is None:
+            assert got is None, case["name"]
+            continue
+        assert got is not None, case["name"]
+        assert got[0] == case["Bstar"] * UNIT, (case["name"], got)
+        assert got[1] == case["bounds"], (case["name"], got)
+
+
+def check_hand_pricing(O):
+    """Hand-worked end-to-end prices (golden/hand_pricing.json)."""
+    for case in _load("hand_pricing.json")["cases"]:
+        orc, cands, L = oracle_for(O, case)
+        r = orc.price(cands)
+        for c, exp in enumerate(case["expect"]):
+            name = "%s cand %d" % (case["name"], c)
+            assert int(r["status"][c]) == exp["status"], (name, r["status"][c])
+            assert int(r["n_dp"][c]) == exp["n_dp"], (name, r["n_dp"][c])
+            assert int(r["T"][c]) == exp["T"], (name, r["T"][c])
+            assert int(r["bottleneck"][c]) == exp["bottleneck"], (name, r["bottleneck"][c])
+            S = int(cands["S"][c])
+            if exp["bounds"] is not None:
+                assert r["bounds"][: S + 1, c].tolist() == exp["bounds"], (name, r["bounds"][:, c])
+        if "topk_order" in case:
+            tk = O.topk(r, cands["M"], len(case["expect"]))
+            assert tk["idx"].tolist() == case["topk_order"], (case["name"], tk)
+
+
+def check_brute_force_partition(O, trials=400, seed=1234):
+    """Oracle DP == exhaustive enumeration of every contiguous split on small
+    random heterogeneous instances (memory caps that sometimes bind)."""
+    rng = np.random.default_rng(seed)
+    for t in range(trials):
+        S = int(rng.integers(1, 6))
+        L = int(rng.integers(S, 13))
+        layers = rng.integers(0, 50, L)
+        scales = rng.integers(1, 6, S)
+        c = rng.integers(0, 30, S) if rng.random() < 0.7 else np.zeros(S, np.int64)
+        c[-1] = 0
+        P = np.stack([np.concatenate([[0], np.cumsum(layers * k)]) for k in scales]).astype(np.int64)
+        # per-stage memory tables (different weights per stage, as in-flight counts differ)
+        mw = rng.integers(0, 10, L)
+        W = np.stack([np.concatenate([[0], np.cumsum(mw * (1 + (S - s) % 3))]) for s in range(S)])
+        tot = W[:, -1]
+        cap = (tot * rng.uniform(0.2, 1.2, S)).astype(np.int64) if rng.random() < 0.6 else tot
+        exp = brute_partition(P, c, W, cap)
+        got = O.partition_raw(P, c, W, cap)
+        if exp is None:
+            assert got is None, (t, got)
+        else:
+            assert got is not None, (t, exp)
+            assert got[0] == exp[0] and got[1] == exp[1], (t, S, L, got, exp)
+
+
+def check_closed_forms(O, seed=7):
+    """S = 1 is the serial sum; uniform unit costs give B* = ceil(L/S) with the
+    leftmost optimal split; identical stages with no P2P and no memory limit
+    are the textbook linear-partition problem: B* >= ceil(P[L]/S) and B* does
+    not increase when a stage is added."""
+    rng = np.random.default_rng(seed)
+    for L in range(1, 20):
+        layers = rng.integers(1, 100, L)
+        P, c, W, cap = tables_from_scales(layers, [1], [0])
+        assert O.partition_raw(P, c, W, cap) == (int(layers.sum()), [0, L])
+        for S in range(1, L + 1):
+            P, c, W, cap = tables_from_scales(np.ones(L, np.int64), [1] * S, [0] * S)
+            B, a = O.partition_raw(P, c, W, cap)
+            assert B == math.ceil(L / S), (L, S, B)
+            # leftmost: every boundary as small as the remainder allows
+            for s in range(1, S):
+                assert a[s] == max(s, L - (S - s) * B), (L, S, a)
+    for trial in range(60):
+        L = int(rng.integers(2, 30))
+        layers = rng.integers(0, 1000, L)
+        prev = None
+        for S in range(1, min(L, 8) + 1):
+            P, c, W, cap = tables_from_scales(layers, [1] * S, [0] * S)
+            B, a = O.partition_raw(P, c, W, cap)
+            assert B >= math.ceil(layers.sum() / S)
+            assert B >= layers.max()
+            if prev is not None:
+                assert B <= prev, (layers, S, B, prev)
+            prev = B
+
+
+def check_replicas(O, trials=150, seed=99):
+    """First-fit-decreasing replication count == exhaustive placement search
+    on small clusters; plus hand cases."""
+    assert O.replicas([8, 4], [4, 2, 2]) == 1
+    assert O.replicas([3, 3], [2, 1]) == 2
+    assert O.replicas([3, 3], [2, 2]) == 1
+    assert O.replicas([3, 3], [2, 2, 2]) == 0
+    assert O.replicas([8], [1]) == 8
+    assert O.replicas([4, 4, 4, 4], [4, 4]) == 2
+    assert O.replicas([2, 2], [4]) == 0
+    rng = np.random.default_rng(seed)
+    for t in range(trials):
+        nodes = [int(x) for x in rng.integers(1, 6, int(rng.integers(1, 4)))]
+        mx = max(nodes)
+        opts = [g for g in (1, 2, 4) if g <= mx]
+        groups = [int(rng.choice(opts)) for _ in range(int(rng.integers(1, 4)))]
+        exp = brute_replicas(nodes, groups, limit=sum(nodes))
+        assert O.replicas(nodes, groups) == exp, (nodes, groups, exp)
+
+
+def check_quantiser(O):
+    """Nearest-nanosecond rounding with halves away from zero, via an explicit
+    profile (the per-(type, degree, layer) cost entry of the paper's cost
+    model, §5.2)."""
+    W = _workloads()
+    vals = [(2.0e-3, 2_000_000), (0.0, 0), (2.0**-12, 244_141), (2.0**-11, 488_281)]
+    # j * 2^-10 s is exactly j * 976562.5 ns: for odd j an exact tie, rounded
+    # away from zero; one ulp below the tie rounds down
+    for j in (1, 3, 5, 1001):
+        x = j * 2.0**-10
+        assert x * 1e9 == j * 976562.5
+        vals.append((x, j * 976562 + (j + 1) // 2))
+        vals.append((math.nextafter(x, 0.0), j * 976562 + (j - 1) // 2))
+    L = len(vals)
+    prof = np.zeros((1, 4, L))
+    prof[0, :, :] = [v for v, _ in vals]
+    cluster = W.make_cluster([1000.0], [10**12], [10**11], [(0, 8, 10**10)])
+    model = W.make_model(np.ones(L), 1, 1, 1, 0, 0, 0, profile_s=prof)
+    q = O.Oracle(cluster, model).tables()["q"]
+    for l, (v, exp) in enumerate(vals):
+        assert (q[0, :, l] == exp).all(), (l, v, q[0, :, l], exp)
+
+
+def check_layer_cost_formula(O):
+    """Per-layer cost entries of the synthetic profile: compute, TP all-reduce
+    and EP all-to-all terms on round numbers worked out by hand."""
+    W = _workloads()
+    # type 0: 1000 TFLOPS, intra 300 GB/s, two 4-GPU nodes with 12.5 GB/s NICs
+    cluster = W.make_cluster([1000.0], [10**12], [300 * 10**9],
+                             [(0, 4, 12_500_000_000), (0, 4, 12_500_000_000)])
+    # layer 0: 1e12 FLOPs, 75 MB all-reduce; layer 1: 2e12 FLOPs, 100 MB all-to-all
+    model = W.make_model([1e12, 2e12], 1, 1, 1, [75_000_000, 0], [0, 100_000_000], 0, moe=True)
+    q = O.Oracle(cluster, model).tables()["q"][0]
+    # k=1: 1 ms, 2 ms
+    assert q[0].tolist() == [1_000_000, 2_000_000]
+    # k=2: 0.5 ms + 4*(2*1/2)*75e6/3e11 s = 0.5 + 1 = 1.5 ms; 1 ms + 4*(1/2)*1e8/3e11 s = 1 + 0.6667 ms
+    assert q[1].tolist() == [1_500_000, 1_666_667]
+    # k=4: 0.25 + 4*(2*3/4)*75e6/3e11 = 0.25 + 1.5 = 1.75 ms; 0.5 + 4*(3/4)*1e8/3e11 = 0.5 + 1 = 1.5 ms
+    assert q[2].tolist() == [1_750_000, 1_500_000]
+    # k=8 exceeds the 4-GPU node: NIC 12.5 GB/s.  0.125 + 4*(2*7/8)*75e6/1.25e10 = 0.125 + 42 ms;
+    # 0.25 + 4*(7/8)*1e8/1.25e10 = 0.25 + 28 ms
+    assert q[3].tolist() == [42_125_000, 28_250_000]
+
+
+def check_invariants(O, seed=3):
+    """On random workloads: T >= M * B*; T = M*P[L] + g for S = 1; bounds
+    strictly increasing from 0 to L; outputs follow a permutation of the
+    candidates; the top-k of shards merged equals the top-k of the whole."""
+    W = _workloads()
+    for name, n in (("dense32", 600), ("moe48", 600), ("dense80", 150)):
+        w = W.make_workload(name, seed=seed, n=n)
+        orc = O.Oracle(w.cluster, w.model)
+        r = orc.price(w.cands)
+        tab = orc.tables()
+        ok = r["status"] == 0
+        M = w.cands["M"].astype(np.int64)
+        assert (r["T"][ok] >= M[ok] * r["bottleneck"][ok]).all()
+        assert (r["T"][~ok] == -1).all() and (r["bottleneck"][~ok] == -1).all()
+        L = w.meta["L"]
+        for c in np.nonzero(ok)[0]:
+            S = int(w.cands["S"][c])
+            a = r["bounds"][: S + 1, c].astype(int)
+            assert a[0] == 0 and a[-1] == L and (np.diff(a) > 0).all()
+            if S == 1:
+                code = int(w.cands["code"][0, c])
+                PL = int(tab["P"][code & 7, (code >> 3) & 3, L])
+                assert r["bottleneck"][c] == PL
+                if r["n_dp"][c] == 1:
+                    assert r["T"][c] == int(M[c]) * PL
+        assert (np.diff(tab["P"], axis=2) >= 0).all()
+        perm = np.random.default_rng(seed).permutation(w.n)
+        pc = {"S": w.cands["S"][perm], "M": w.cands["M"][perm],
+              "code": np.ascontiguousarray(w.cands["code"][:, perm])}
+        rp = orc.price(pc)
+        for key in ("T", "bottleneck", "n_dp", "status"):
+            assert (rp[key] == r[key][perm]).all(), key
+        full = O.topk(r, w.cands["M"], 16)
+        pool = []
+        for lo in range(0, w.n, 97):
+            hi = min(w.n, lo + 97)
+            sub = {k: r[k][lo:hi] for k in ("T", "n_dp", "status")}
+            part = O.topk(sub, w.cands["M"][lo:hi], 16, base_index=lo)
+            pool += zip(part["idx"].tolist(), part["T"].tolist(), part["nM"].tolist())
+        # merge the shard lists by exact throughput n*M/T, then smaller index
+        pool.sort(key=lambda e: (-Fraction(e[2], e[1]), e[0]))
+        assert [e[0] for e in pool[:16]] == full["idx"].tolist()
+        pk = O.topk(rp, pc["M"], 16)
+        assert [int(perm[i]) for i in pk["idx"]] == full["idx"].tolist()
+
+
+def check_status_rules(O):
+    """Masked structures are INVALID (§5.1 masks): reserved bits, unknown type,
+    S > L, S = 0, M = 0, TP degree above the largest node of a dense type."""
+    W = _workloads()
+    cluster = W.make_cluster([1000.0, 500.0], [10**12, 10**12], [10**11, 10**11],
+                             [(0, 4, 10**10), (1, 2, 10**10)])
+    model = W.make_model([1e12] * 3, 1, 1, 1, 0, 0, 0)
+    orc = O.Oracle(cluster, model)
+    S = np.array([1, 1, 1, 4, 0, 1, 1, 1, 2], np.uint8)
+    M = np.array([1, 1, 1, 1, 1, 0, 1, 1, 1], np.uint16)
+    code = np.zeros((4, 9), np.uint8)
+    code[0] = [0x20, 2, 0, 0, 0, 0, int(W.encode(1, 2)), int(W.encode(0, 2)), 0]
+    code[1, 8] = int(W.encode(1, 1))
+    code[:, 3] = 0
+    r = orc.price({"S": S, "M": M, "code": code})
+    assert r["status"].tolist() == [3, 3, 0, 3, 3, 3, 3, 0, 0], r["status"]
+
+
+ALL_CHECKS = [
+    check_hand_partitions,
+    check_hand_pricing,
+    check_brute_force_partition,
+    check_closed_forms,
+    check_replicas,
+    check_quantiser,
+    check_layer_cost_formula,
+    check_invariants,
+    check_status_rules,
+]

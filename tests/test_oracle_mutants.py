@@ -1,0 +1,114 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each mutant is a temporary copy of ``oracle/heddle_oracle.c`` with one
+planted mistake (a dropped term, a wrong comparison, index or operand); it is
+compiled on the CPU into a temporary directory and the full pin suite of
+``pin_checks.py`` runs against it in a child process.  Every mutant must fail
+at least one pin.  The committed oracle is never modified.
+"""
+
+import json
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "heddle_oracle.c")
+
+MUTANTS = [
+    ("drop_p2p_in_dp", "int64_t t = P[s][j] - P[s][i] + c[s];", "int64_t t = P[s][j] - P[s][i];"),
+    ("memory_strict", "if (W[s][j] - W[s][i] > cap[s]) continue;\n                int64_t t",
+     "if (W[s][j] - W[s][i] >= cap[s]) continue;\n                int64_t t"),
+    ("iteration_M_not_M_minus_1", "(int64_t)(M - 1) * tmax", "(int64_t)M * tmax"),
+    ("drop_grad_sync", "+ tsum + gmax;", "+ tsum;"),
+    ("drop_sum_term", "out->T = (int64_t)(M - 1) * tmax + tsum + gmax;",
+     "out->T = (int64_t)(M - 1) * tmax + tmax + gmax;"),
+    ("inflight_reversed", "int64_t inflight = (S - s) < M ? (S - s) : M;",
+     "int64_t inflight = (s + 1) < M ? (s + 1) : M;"),
+    ("inflight_ignores_M", "int64_t inflight = (S - s) < M ? (S - s) : M;",
+     "int64_t inflight = (S - s);"),
+    ("tp_ring_factor", "double ring = (2.0 * (k - 1.0)) / k;", "double ring = (k - 1.0) / k;"),
+    ("ep_factor", "t = 4.0 * part;", "t = 2.0 * part;"),
+    ("collective_bw_rule", "(1 << j) <= x->maxnode[g] ? (double)x->intra_bw[g]",
+     "(1 << j) < x->maxnode[g] ? (double)x->intra_bw[g]"),
+    ("p2p_same_node_rule", "(1 << j[s]) + (1 << j[s + 1]) <= x->maxnode[g[s]]",
+     "(1 << j[s]) + (1 << j[s + 1]) < x->maxnode[g[s]]"),
+    ("p2p_direction", "c[s] = x->p2p[g[s]][g[s + 1]][same];", "c[s] = x->p2p[g[s]][g[s]][same];"),
+    ("dp_ring_factor", "u128 num = (u128)2 * (u128)(n - 1)", "u128 num = (u128)(n - 1)"),
+    ("dp_shard_not_divided", "u128 den = (u128)n * (u128)(1 << j[s]) *", "u128 den = (u128)n *"),
+    ("walk_ignores_remainder", "if (F(s + 1, j) > B) continue;", ""),
+    ("round_truncates", "return (int64_t)llround(seconds * 1e9);", "return (int64_t)(seconds * 1e9);"),
+    ("ffd_increasing", "for (int e = 3; e >= 0 && ok; --e)", "for (int e = 0; e <= 3 && ok; ++e)"),
+    ("topk_tie_larger_index", "return a->idx < b->idx ? -1 : (a->idx > b->idx ? 1 : 0);",
+     "return a->idx > b->idx ? -1 : (a->idx < b->idx ? 1 : 0);"),
+    ("rank_operand_transposed", "u128 lhs = (u128)a->nM * (u128)b->T;", "u128 lhs = (u128)a->nM * (u128)a->T;"),
+    ("mem_cap_not_times_k", "cap[s] = x->mem[g[s]] * (int64_t)(1 << j[s]);", "cap[s] = x->mem[g[s]];"),
+    ("nic_max_not_min", "if (node_nic[b] < x->inter_bw[g]) x->inter_bw[g] = node_nic[b];",
+     "if (x->inter_bw[g] == INT64_MAX || node_nic[b] > x->inter_bw[g]) x->inter_bw[g] = node_nic[b];"),
+    ("ceil_is_floor", "return (int64_t)((a + b - 1) / b);", "return (int64_t)(a / b);"),
+    ("tp_mask_off_by_one", "(!x->moe && (1 << j[s]) > x->maxnode[g[s]])",
+     "(!x->moe && (1 << j[s]) >= x->maxnode[g[s]])"),
+    ("empty_stage_allowed", "for (int j = i + 1; j <= L; ++j) {\n                if (F(s + 1, j) == INF) continue;",
+     "for (int j = i; j <= L; ++j) {\n                if (F(s + 1, j) == INF) continue;"),
+    ("max_not_min_in_dp", "if (v < best) best = v;", "if (best == INF || v > best) best = v;"),
+    ("ep_group_not_split", "while ((1 << e) > x->maxnode[t]) --e;", ""),
+    ("ep_blocks_of_one", "while ((1 << e) > x->maxnode[t]) --e;", "if ((1 << e) > x->maxnode[t]) e = 0;"),
+    ("compute_ignores_degree", "double s = flops / (k * tflops * 1e12);", "double s = flops / (tflops * 1e12);"),
+]
+
+CHILD = r"""
+import json, sys, traceback
+sys.path[:0] = [sys.argv[1], sys.argv[1] + "/tests"]
+from oracle import oracle as O
+O.LIB = sys.argv[2]
+O.build = lambda force=False: O.LIB
+import pin_checks as P
+failed = []
+for chk in P.ALL_CHECKS:
+    try:
+        chk(O)
+    except Exception as e:
+        failed.append(chk.__name__)
+print("FAILED=" + json.dumps(failed))
+"""
+
+
+def _compile(dirpath, text):
+    src = os.path.join(dirpath, "heddle_oracle.c")
+    with open(src, "w") as f:
+        f.write(text)
+    shutil.copy(os.path.join(ROOT, "oracle", "heddle_oracle.h"), dirpath)
+    lib = os.path.join(dirpath, "libmutant.so")
+    subprocess.check_call(["gcc", "-std=c11", "-O2", "-ffp-contract=off", "-fPIC", "-shared",
+                           "-o", lib, src, "-lpthread", "-lm"])
+    return lib
+
+
+def _run_pins(lib):
+    try:
+        p = subprocess.run([sys.executable, "-c", CHILD, ROOT, lib], capture_output=True,
+                           text=True, timeout=300)
+    except subprocess.TimeoutExpired:
+        return ["<timeout>"]
+    for line in p.stdout.splitlines():
+        if line.startswith("FAILED="):
+            return json.loads(line[len("FAILED="):])
+    return ["<crash rc=%d>" % p.returncode]
+
+
+def test_unmutated_copy_passes(tmp_path):
+    with open(SRC) as f:
+        text = f.read()
+    assert _run_pins(_compile(str(tmp_path), text)) == []
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_is_caught(tmp_path, name, old, new):
+    with open(SRC) as f:
+        text = f.read()
+    assert text.count(old) == 1, "mutation site not unique: " + name
+    failed = _run_pins(_compile(str(tmp_path), text.replace(old, new)))
+    assert failed, "no pin catches mutant " + name
