@@ -1,0 +1,300 @@
+"""Benchmark: candidate plans priced per second on one GB300.
+
+A step prices the whole 128-layer stress workload -- 1e7 candidate pipeline
+structures for a 1024-GPU cluster of 8 types (S <= 32, TP in {1,2,4,8},
+M = 256) -- as ten device-resident batches of 1e6 (PartitionLayers +
+Evaluate kernel, then the block/grid top-k merge into one top-16 state).
+Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+
+N > 1 runs under torchrun, one rank per GPU; every rank prices its own 1e7
+candidates (weak scaling) and the per-rank top-16 lists are merged on the
+host.  ``--impl reference`` times the CPU oracle on the host cores instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "candidate plans priced/sec on 1 GB300 (and % of ALU/HBM roofline)"
+UNIT = "candidates/s"
+WORKLOAD = "stress128"
+WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 1024 GPUs of 8 types in "
+                 "nodes of 2/4/8, 1e7 candidates streamed as 10 device batches of 1e6, S<=32, "
+                 "TP in {1,2,4,8}, M=256, global top-16")
+# Algorithmic integer work of one interval check of PartitionLayers: stage
+# cost P[j]-P[i]+c compared with B (int64 subtract, add, compare) and stage
+# memory (S[j]-S[i]) + f*(A[j]-A[i]) compared with the capacity (two int64
+# subtracts, one multiply by a 32-bit count, one add, one compare): eight
+# int64 operations, 16 32-bit ALU lane operations.
+OPS_PER_CHECK = 16
+SMS, LANES_PER_SM = 152, 128  # 4 SM sub-partitions x 32 lanes issue per clock
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        if self.path and os.path.exists(self.path):
+            for line in open(self.path):
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+            os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def oracle_rate(w, seconds, threads, max_n=None):
+    """Oracle candidates/s on a bounded sample sized for about ``seconds``."""
+    from oracle import oracle as O
+    from paper_2609_34244_gb300 import workloads as W
+    orc = O.Oracle(w.cluster, w.model)
+    probe_n = min(w.n, 4 * threads * 8)
+    sub = W.slice_cands(w.cands, 0, probe_n)
+    t0 = time.perf_counter()
+    orc.price(sub, threads=threads, bounds=False)
+    dt = max(time.perf_counter() - t0, 1e-6)
+    n = int(min(w.n, max(probe_n, probe_n * seconds / dt)))
+    if max_n:
+        n = min(n, max_n)
+    sub = W.slice_cands(w.cands, 0, n)
+    t0 = time.perf_counter()
+    used = orc.price(sub, threads=threads, bounds=False)["threads"]
+    dt = time.perf_counter() - t0
+    return n / dt, n, used, dt
+
+
+def run_reference(args, w):
+    """The CPU oracle as the reference arm: each step prices a bounded sample."""
+    threads = os.cpu_count() or 1
+    _, n, used, _ = oracle_rate(w, 4.0, threads)
+    from oracle import oracle as O
+    from paper_2609_34244_gb300 import workloads as W
+    orc = O.Oracle(w.cluster, w.model)
+    sub = W.slice_cands(w.cands, 0, n)
+    for _ in range(args.warmup):
+        orc.price(sub, threads=threads, bounds=False)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        orc.price(sub, threads=threads, bounds=False)
+    dt = time.perf_counter() - t0
+    value = n * args.steps / dt
+    sample = "first %d candidates of %s seed 0 per step, %d host threads" % (n, WORKLOAD, used)
+    return {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": 0,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD_DESC, "candidates_per_step": n, "sample": sample},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": used, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--n", type=int, default=10_000_000)
+    ap.add_argument("--batch", type=int, default=1_000_000)
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    from paper_2609_34244_gb300 import workloads as W
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        w = W.make_workload(WORKLOAD, seed=0, n=min(args.n, 400_000))
+        print(json.dumps(run_reference(args, w)), flush=True)
+        return
+
+    import torch
+    from paper_2609_34244_gb300 import _build
+    _build.build()
+    from paper_2609_34244_gb300 import heddle as h
+    from paper_2609_34244_gb300 import shard
+
+    torch.cuda.set_device(local)
+    group = shard.init(world)
+    n, batch = args.n, min(args.batch, args.n)
+    # weak scaling: rank r prices its own n candidates (seed r), global indices r*n + c
+    w = W.make_workload(WORKLOAD, seed=rank, n=n)
+    base = rank * n
+    ctx = h.heddle_create(local)
+    h.heddle_load_cluster(ctx, w.cluster)
+    h.heddle_load_model(ctx, w.model)
+    dc = h.cands_to_device(w.cands)
+    res = h.alloc_results(n)
+    state = h.alloc_topk_state()
+    stream = torch.cuda.current_stream()
+    cbatches = [(h.make_candidates(dc, lo, min(n, lo + batch), base_index=base),
+                 h.make_results(res, lo, min(n, lo + batch))) for lo in range(0, n, batch)]
+    n_batches = len(cbatches)
+
+    def step(events=None):
+        h.heddle_topk_reset(ctx, state, 16, stream)
+        for i, (c, r) in enumerate(cbatches):
+            if events is not None:
+                events[i][0].record(stream)
+            h.heddle_price_candidates(ctx, c, r, stream)
+            if events is not None:
+                events[i][1].record(stream)
+            h.heddle_topk(ctx, c, r, state, stream)
+
+    # algorithmic work of one step (counting variant, untimed)
+    work = {"checks": 0, "probes": 0, "priced": 0}
+    h.heddle_topk_reset(ctx, state, 16, stream)
+    for c, r in cbatches:
+        h.heddle_count_next(ctx, True)
+        h.heddle_price_candidates(ctx, c, r, stream)
+    for key, v in h.heddle_work_counters(ctx).items():
+        work[key] += v
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    shard.barrier(group)
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(n_batches)] for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        torch.cuda.synchronize()
+        t_start.record(stream)
+        for k in range(args.steps):
+            step(ev[k])
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    shard.barrier(group)
+    clocks = clk.summary()
+    ms = t_start.elapsed_time(t_end)
+    price_ms = sum(a.elapsed_time(b) for row in ev for a, b in row)
+    ms_all = shard.max_over_ranks(group, ms)
+    errors = h.heddle_device_errors(ctx)
+    local_topk = h.read_topk_state(state)
+    merged = shard.merge_topk_across_ranks(group, local_topk, 16)
+
+    # end to end through the public host-buffer call (pinned host memory)
+    pinned = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
+              for k, v in w.cands.items()}
+    h2d = int(sum(v.numel() * v.element_size() for v in pinned.values()))
+    st = h.new_topk_state(16)
+    e2e_steps = max(1, args.e2e_steps)
+    h.heddle_price_topk_host(ctx, pinned, None, st, batch, stream)  # warm (allocates staging)
+    shard.barrier(group)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        st = h.new_topk_state(16)
+        h.heddle_price_topk_host(ctx, pinned, None, st, batch, stream)
+    e2e_s = (time.perf_counter() - t0) / e2e_steps
+    e2e_s = shard.max_over_ranks(group, e2e_s)
+    e2e_topk = h.topk_state_to_dict(st)
+    h.heddle_destroy(ctx)
+
+    if rank != 0:
+        return
+    peaks, peak_kind = load_peaks()
+    value = n * world * args.steps / (ms_all / 1e3)
+    ops_step = work["checks"] * OPS_PER_CHECK
+    peak_tops = SMS * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+    achieved_tops = ops_step * args.steps / (price_ms / 1e3) / 1e12
+    cpu = None
+    if not args.no_cpu_baseline:
+        rate, ncpu, used, dt = oracle_rate(w, args.cpu_seconds, os.cpu_count() or 1)
+        cpu = {"value": rate, "unit": UNIT, "cores": used, "kind": "oracle",
+               "sample": "first %d candidates of %s seed 0 (%.1f s, %d host threads)" % (ncpu, WORKLOAD, dt, used)}
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_all / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": WORKLOAD_DESC, "candidates_per_gpu": n, "batch": batch,
+                   "parallelism": "candidate shards, dp%d" % world,
+                   "l2": "inputs larger than L2 (%.0f MB of candidates per step per GPU)" % (h2d / 1e6),
+                   "seed": "rank"},
+        "gpu_launches": args.steps * (1 + 3 * n_batches) * world,
+        "per_candidate_ns": 1e6 * ms_all / args.steps / n,
+        "roofline": {"bound": "alu", "achieved": achieved_tops, "peak": peak_tops, "unit": "Tops/s",
+                     "frac": achieved_tops / peak_tops, "traffic": None,
+                     "kernel": "price_kernel", "ops_per_check": OPS_PER_CHECK,
+                     "checks_per_candidate": work["checks"] / n, "probes_per_priced": work["probes"] / max(1, work["priced"]),
+                     "price_ms_per_step": price_ms / args.steps,
+                     "peak_basis": "%s: %d SMs x %d lanes x %.0f MHz (%s sm_max)" % (
+                         "issue slots", SMS, LANES_PER_SM, float(peaks.get("sm_max_mhz", 2070.0)), peak_kind)},
+        "clocks": clocks,
+        "e2e": {"value": n * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d * world,
+                "d2h_bytes_per_step": h.TOPK_STATE_BYTES * world},
+        "device_errors": errors,
+        "topk_head": merged["idx"][:4].tolist() if merged["count"] else [],
+        "e2e_topk_matches": e2e_topk["idx"].tolist() == local_topk["idx"].tolist(),
+    }
+    if cpu:
+        out["cpu_baseline"] = cpu
+    print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

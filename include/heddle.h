@@ -1,0 +1,261 @@
+/*
+ * heddle.h -- C ABI of the GB300 (sm_103a) batched candidate-plan pricer.
+ *
+ * The operation is the inner loop of a parallelism planner (paper
+ * arxiv 2609.34244): for every candidate pipeline structure -- a depth S and,
+ * per stage, a GPU type and a TP degree (the "structural template" of §5.1) --
+ * find the DP replication count the node packing admits (§5.3), split the
+ * model's layers into S contiguous stages minimising the slowest stage under
+ * per-GPU memory limits (PartitionLayers of the §3.1 search listing, memory
+ * validation of §5.2), price the 1F1B iteration time
+ *     T = (M - 1) * max_s t_s + sum_s t_s + max_s g_s         (§5.3)
+ * with inter-stage P2P inside t_s and the DP gradient synchronisation g_s,
+ * and rank the candidates by throughput n * M / T (§5 overview).
+ *
+ * All pricing arithmetic after the cost-table build is integer: times in
+ * int64 nanoseconds, sizes in int64 bytes, bandwidths in int64 bytes/s.
+ * Results are bit-exact and independent of launch configuration.
+ *
+ * Conventions for every entry point:
+ *   - returns heddle_status; never aborts the process;
+ *   - a context is not thread-safe: one host thread uses it at a time;
+ *   - "device" pointers are CUDA device (or managed) memory on the context's
+ *     device, owned by the caller; the library keeps no reference after the
+ *     call returns (asynchronous calls read and write them on the stream);
+ *   - "stream" is a cudaStream_t (NULL = legacy default stream);
+ *   - per-candidate problems are data, reported in the status plane, not
+ *     call errors.
+ */
+#ifndef HEDDLE_H
+#define HEDDLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define HEDDLE_MAX_TYPES 8      /* GPU types per cluster */
+#define HEDDLE_MAX_STAGES 32    /* pipeline depth S */
+#define HEDDLE_MAX_LAYERS 255   /* model layers L (boundaries fit in a byte) */
+#define HEDDLE_MAX_GPUS 65535   /* GPUs per cluster (DP degree fits in uint16) */
+#define HEDDLE_MAX_TOPK 64
+#define HEDDLE_BOUND_PLANES (HEDDLE_MAX_STAGES + 1)
+
+typedef enum {
+    HEDDLE_OK = 0,
+    HEDDLE_E_ARG = 1,    /* null pointer, negative size, malformed record */
+    HEDDLE_E_STATE = 2,  /* cluster or model not loaded, or mismatched */
+    HEDDLE_E_LIMIT = 3,  /* a size or value exceeds a documented limit */
+    HEDDLE_E_CUDA = 4,   /* a CUDA runtime call failed (message has details) */
+    HEDDLE_E_NOMEM = 5   /* device or host allocation failed */
+} heddle_status;
+
+/* Per-candidate status (uint8 plane). */
+enum {
+    HEDDLE_CAND_OK = 0,
+    HEDDLE_CAND_OOM = 1,     /* no layer split fits the GPUs' memory (§5.2) */
+    HEDDLE_CAND_NO_FIT = 2,  /* not one replica can be placed on the nodes */
+    HEDDLE_CAND_INVALID = 3  /* masked structure (§5.1): see heddle_price_candidates */
+};
+
+typedef struct heddle_ctx heddle_ctx;
+
+/* Create a context on CUDA device `device`.  Allocates a small amount of
+ * device memory (the top-k merge scratch) and queries the SM count.
+ * *out is NULL on failure. */
+heddle_status heddle_create(heddle_ctx** out, int32_t device);
+
+/* Free the context and all device memory it owns.  NULL is ignored. */
+void heddle_destroy(heddle_ctx* ctx);
+
+/* Message of the last failed call on ctx (never NULL; "" after success).
+ * The buffer belongs to ctx and is overwritten by the next call. */
+const char* heddle_last_error(const heddle_ctx* ctx);
+
+/* ------------------------------------------------------------- cluster */
+
+/* One GPU type (§5.1 "normalized hardware attributes"): peak dense TFLOPS,
+ * memory per GPU in bytes, intra-node link bandwidth in bytes/s. */
+typedef struct {
+    double tflops;
+    int64_t mem_bytes;
+    int64_t intra_bw;
+} heddle_gpu_type;
+
+/* One node (§5.1 "a node list per GPU type"): type index, GPU count,
+ * inter-node NIC bandwidth in bytes/s. */
+typedef struct {
+    int32_t type;
+    int32_t gpus;
+    int64_t nic_bw;
+} heddle_node;
+
+/* Load the GPU composition.  Host arrays, copied before return.
+ * Limits: 1 <= n_types <= 8; n_nodes >= 1; every node: 0 <= type < n_types,
+ * gpus >= 1, 1 <= nic_bw <= 2^40; total GPUs <= 65535; tflops finite > 0;
+ * 1 <= mem_bytes <= 2^50; 1 <= intra_bw <= 2^40.  Types without nodes are
+ * allowed (candidates using them are INVALID).  Rebuilds the cost tables if
+ * a model is loaded (synchronous: the call returns after the device tables
+ * are ready). */
+heddle_status heddle_load_cluster(heddle_ctx* ctx, const heddle_gpu_type* types,
+                                  int32_t n_types, const heddle_node* nodes,
+                                  int32_t n_nodes);
+
+/* --------------------------------------------------------------- model */
+
+/* One layer (§5.2 "one layer per repeated structure"):
+ *   flops        forward+backward FLOPs for one microbatch
+ *   param_bytes  gradient bytes the DP all-reduce synchronises
+ *   state_bytes  parameters + gradients + optimizer state held for the layer
+ *   act_bytes    activation bytes kept per in-flight microbatch
+ *   ar_bytes     message of each of the layer's four TP all-reduces
+ *   a2a_bytes    message of each of the layer's four EP all-to-alls (0: dense) */
+typedef struct {
+    double flops;
+    int64_t param_bytes;
+    int64_t state_bytes;
+    int64_t act_bytes;
+    int64_t ar_bytes;
+    int64_t a2a_bytes;
+} heddle_layer;
+
+#define HEDDLE_MODEL_MOE 1 /* stage degree is an EP degree; may exceed a node */
+
+/* Load the model.  Host arrays, copied before return.
+ * boundary_bytes: activation bytes crossing a stage boundary per microbatch.
+ * profile_s: nullable [n_types][4][n_layers] seconds per layer at degree
+ *   2^j (computation plus communication, §5.2 profile entries); replaces the
+ *   synthetic formula and requires the cluster to be loaded first.
+ * Per-layer cost in ns (synthetic profile, degree k = 2^j, type g):
+ *   s = flops / (k * tflops_g * 1e12)
+ *   k > 1: s += 4 * (2(k-1)/k) * ar_bytes / bw  and  s += 4 * ((k-1)/k) * a2a_bytes / bw
+ *   bw = intra_bw_g if k <= largest node of g, else the slowest NIC of g
+ *   q = nearest integer of s * 1e9, halves away from zero
+ * evaluated left to right in IEEE double without fused multiply-add.
+ * Limits: 1 <= n_layers <= 255; all byte counts in [0, 2^42]; flops finite
+ * >= 0; every per-(type, degree) total of q <= 2^40 ns; P2P and gradient
+ * terms must stay below 2^40 / 2^56 ns (E_LIMIT otherwise). */
+heddle_status heddle_load_model(heddle_ctx* ctx, const heddle_layer* layers, int32_t n_layers,
+                                int64_t boundary_bytes, int32_t flags,
+                                const double* profile_s);
+
+/* ---------------------------------------------------------- candidates */
+
+/* Candidate batch, structure of arrays in device memory.
+ *   S[n]       stage count (uint8)
+ *   M[n]       microbatches per iteration (uint16)
+ *   code       stage bytes, stage-major: stage s of candidate c at
+ *              code[s * plane_stride + c], for s < s_max; byte = type
+ *              (bits 0-2) | log2 degree (bits 3-4); bits 5-7 must be 0
+ *   base_index global index of candidate 0 (used by the top-k) */
+typedef struct {
+    const uint8_t* S;
+    const uint16_t* M;
+    const uint8_t* code;
+    int64_t n;
+    int64_t plane_stride;
+    int32_t s_max;
+    int32_t reserved;
+    int64_t base_index;
+} heddle_candidates;
+
+/* Per-candidate results in device memory (caller-owned, n entries each).
+ *   T           iteration time, ns (-1 unless status OK)
+ *   bottleneck  min-max stage time B* = max_s t_s, ns (-1 unless OK)
+ *   n_dp        DP replication count (0 for INVALID / NO_FIT)
+ *   status      HEDDLE_CAND_*
+ *   bounds      nullable, [33][n] uint8: stage boundaries a_0..a_S of the
+ *               canonical split (plane s at bounds[s * n + c]); all zero
+ *               unless OK.  Among all splits attaining B* the canonical one
+ *               is the lexicographically smallest boundary vector. */
+typedef struct {
+    int64_t* T;
+    int64_t* bottleneck;
+    uint16_t* n_dp;
+    uint8_t* status;
+    uint8_t* bounds;
+} heddle_results;
+
+/* Price a batch (PartitionLayers + Evaluate, §3.1, §5.2, §5.3).
+ * Asynchronous on `stream`; no host round-trip; allocates nothing.
+ * A candidate is INVALID if S = 0, S > 32, S > s_max, S > L, M = 0, a stage
+ * byte has bits 5-7 set, names a type >= n_types or a type without GPUs, or
+ * (dense models) asks a degree above the largest node of its type (the TP
+ * mask of §5.1).  NO_FIT: DP degree 0.  OOM: no split fits in memory.
+ * Errors: E_ARG (null ctx/struct/pointers, n < 0, plane_stride < n,
+ * s_max outside [1, 32]), E_STATE (cluster or model missing), E_CUDA (launch
+ * failure).  n = 0 is a no-op. */
+heddle_status heddle_price_candidates(heddle_ctx* ctx, const heddle_candidates* cands,
+                                      const heddle_results* results, void* stream);
+
+/* ----------------------------------------------------------------- top-k */
+
+/* Running top-k of OK candidates, best first, caller-owned device memory.
+ * Order: higher throughput nM / T first (exact integer comparison
+ * nM_a * T_b > nM_b * T_a), equal throughput -> smaller idx first.
+ * nM = n_dp * M.  Each candidate index may be merged at most once. */
+typedef struct {
+    int32_t k;      /* 1..64 */
+    int32_t count;  /* entries in use, <= k */
+    int64_t idx[HEDDLE_MAX_TOPK];
+    int64_t T[HEDDLE_MAX_TOPK];
+    uint32_t nM[HEDDLE_MAX_TOPK];
+} heddle_topk_state;
+
+/* Set *state (device) to empty with capacity k (1..64).  Asynchronous. */
+heddle_status heddle_topk_reset(heddle_ctx* ctx, heddle_topk_state* state, int32_t k,
+                                void* stream);
+
+/* Merge the OK candidates of a priced batch into *state (device): a
+ * block-level top-k per CTA into context-owned scratch, then a one-CTA merge
+ * with the incoming state (two launches, no inter-CTA waiting).
+ * Asynchronous; reads cands->M, results->T/n_dp/status.  Errors: E_ARG,
+ * E_STATE, E_CUDA.  Calls on one context must not overlap on the GPU (they
+ * share the scratch): use one stream per context. */
+heddle_status heddle_topk(heddle_ctx* ctx, const heddle_candidates* cands,
+                          const heddle_results* results, heddle_topk_state* state,
+                          void* stream);
+
+/* -------------------------------------------------------- host buffers */
+
+/* End-to-end convenience for host (ideally pinned) buffers: streams the
+ * candidates in batches of `batch` through context-owned device staging
+ * buffers (two sets, copies overlapped with pricing), prices them, merges
+ * them into *state and copies back every non-NULL field of `results` (host
+ * arrays of cands->n entries; bounds uses plane stride cands->n).  *state is
+ * host memory, read on entry (k, and any entries already held) and written
+ * on return.  Synchronous: returns when all outputs are in host memory.
+ * Grows its staging buffers on first use (allocation).  Errors as above,
+ * plus E_NOMEM. */
+heddle_status heddle_price_topk_host(heddle_ctx* ctx, const heddle_candidates* cands,
+                                     const heddle_results* results, heddle_topk_state* state,
+                                     int64_t batch, void* stream);
+
+/* ------------------------------------------------------- introspection */
+
+/* Copy the quantised cost tables to host memory (synchronous):
+ * q[n_types][4][n_layers] per-layer ns at degree 2^j (zero for types
+ * without GPUs) and p2p[8][8][2] P2P ns (from type, to type, same-node).
+ * Either pointer may be NULL. */
+heddle_status heddle_get_tables(heddle_ctx* ctx, int64_t* q, int64_t* p2p);
+
+/* Device-side error flags raised since the last call (synchronises the
+ * device first, then clears them): bit 0 a table-staging wait timed out,
+ * bit 1 a search exceeded its iteration bound, bit 2 an internal
+ * consistency check failed.  0 in normal operation. */
+heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
+
+/* Work counters of the next heddle_price_candidates call on ctx, for the
+ * roofline report: when enabled, that call runs the counting variant of the
+ * pricing kernel and accumulates, in device memory owned by ctx,
+ * [0] interval checks evaluated, [1] feasibility probes, [2] candidates
+ * priced past validation.  heddle_work_counters(ctx, out) copies them out
+ * (synchronous) and resets them. */
+heddle_status heddle_count_next(heddle_ctx* ctx, int32_t enable);
+heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* HEDDLE_H */

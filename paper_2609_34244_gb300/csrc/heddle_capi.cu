@@ -1,0 +1,558 @@
+// heddle_capi.cu -- the C ABI (include/heddle.h): context, validated loads,
+// launches on the caller's stream, and the host-buffer streaming path.
+
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <vector>
+
+#include "heddle_internal.cuh"
+
+using hd::Layout;
+
+struct heddle_ctx {
+    int device = 0;
+    int num_sms = 0;
+    char msg[512] = {0};
+    // host copies of the descriptions
+    std::vector<heddle_gpu_type> types;
+    std::vector<heddle_node> nodes;
+    std::vector<heddle_layer> layers;
+    std::vector<double> profile;
+    bool have_cluster = false, have_model = false, have_profile = false;
+    int64_t boundary_bytes = 0;
+    int32_t moe = 0;
+    // device tables
+    Layout lay{};
+    bool tables_ready = false;
+    unsigned char* d_img = nullptr;
+    size_t img_cap = 0;
+    int64_t* d_q = nullptr;
+    size_t q_cap = 0;
+    uint32_t* d_flags = nullptr;            // [0] table build, [1] device errors
+    unsigned long long* d_counters = nullptr;  // [3]
+    bool count_next = false;
+    // top-k merge scratch
+    hd::TopkEntry* d_scratch = nullptr;
+    int32_t* d_scratch_count = nullptr;
+    int scratch_blocks = 0;
+    // host-buffer path
+    cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
+    cudaEvent_t ev_loaded[2] = {nullptr, nullptr}, ev_priced[2] = {nullptr, nullptr},
+                ev_free[2] = {nullptr, nullptr};
+    int64_t stage_cap = 0;
+    int32_t stage_smax = 0;
+    uint8_t* st_S[2] = {nullptr, nullptr};
+    uint16_t* st_M[2] = {nullptr, nullptr};
+    uint8_t* st_code[2] = {nullptr, nullptr};
+    int64_t* st_T[2] = {nullptr, nullptr};
+    int64_t* st_B[2] = {nullptr, nullptr};
+    uint16_t* st_n[2] = {nullptr, nullptr};
+    uint8_t* st_status[2] = {nullptr, nullptr};
+    uint8_t* st_bounds[2] = {nullptr, nullptr};
+    heddle_topk_state* d_state = nullptr;
+};
+
+namespace {
+
+heddle_status fail(heddle_ctx* x, heddle_status st, const char* fmt, ...) {
+    if (x) {
+        va_list ap;
+        va_start(ap, fmt);
+        vsnprintf(x->msg, sizeof(x->msg), fmt, ap);
+        va_end(ap);
+    }
+    return st;
+}
+
+heddle_status ok(heddle_ctx* x) {
+    x->msg[0] = 0;
+    return HEDDLE_OK;
+}
+
+#define CU(call)                                                                           \
+    do {                                                                                   \
+        cudaError_t e_ = (call);                                                           \
+        if (e_ != cudaSuccess)                                                             \
+            return fail(x, HEDDLE_E_CUDA, "%s: %s (%s:%d)", #call, cudaGetErrorString(e_), \
+                        __FILE__, __LINE__);                                               \
+    } while (0)
+
+// Makes the context's device current for the duration of a call.
+struct DeviceGuard {
+    int prev = -1;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) cudaSetDevice(dev);
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+template <class T>
+cudaError_t grow(T** p, size_t* cap, size_t need) {
+    if (*cap >= need && *p) return cudaSuccess;
+    if (*p) cudaFree(*p);
+    *p = nullptr;
+    *cap = 0;
+    cudaError_t e = cudaMalloc((void**)p, need);
+    if (e == cudaSuccess) *cap = need;
+    return e;
+}
+
+constexpr int64_t kByteLimit = (int64_t)1 << 42;
+constexpr int64_t kBwLimit = (int64_t)1 << 40;
+constexpr int64_t kMemLimit = (int64_t)1 << 50;
+
+heddle_status build_tables(heddle_ctx* x) {
+    x->tables_ready = false;
+    if (!x->have_cluster || !x->have_model) return ok(x);
+    const int NT = (int)x->types.size(), L = (int)x->layers.size();
+    if (x->have_profile && x->profile.size() != (size_t)NT * 4 * L)
+        return fail(x, HEDDLE_E_STATE,
+                    "model profile covers %zu entries, cluster needs %d types x 4 x %d layers",
+                    x->profile.size(), NT, L);
+    // the gradient term stays below 2^56 ns: 2 * sum(param) * 1e9 / slowest NIC
+    {
+        unsigned __int128 G = 0;
+        for (const auto& ly : x->layers) G += (unsigned __int128)ly.param_bytes;
+        for (int g = 0; g < NT; ++g) {
+            int64_t nic = INT64_MAX;
+            for (const auto& nd : x->nodes)
+                if (nd.type == g && nd.nic_bw < nic) nic = nd.nic_bw;
+            if (nic == INT64_MAX) continue;
+            const unsigned __int128 t = (2 * G * 1000000000u + nic - 1) / (unsigned __int128)nic;
+            if (t > ((unsigned __int128)1 << 56))
+                return fail(x, HEDDLE_E_LIMIT, "gradient synchronisation of type %d exceeds 2^56 ns", g);
+        }
+    }
+    x->lay = hd::make_layout(L, NT);
+    CU(grow(&x->d_img, &x->img_cap, x->lay.bytes));
+    CU(grow(&x->d_q, &x->q_cap, sizeof(int64_t) * (size_t)NT * 4 * L));
+    heddle_gpu_type* d_types = nullptr;
+    heddle_node* d_nodes = nullptr;
+    heddle_layer* d_layers = nullptr;
+    double* d_prof = nullptr;
+    cudaError_t e = cudaMalloc(&d_types, sizeof(heddle_gpu_type) * NT);
+    if (e == cudaSuccess) e = cudaMalloc(&d_nodes, sizeof(heddle_node) * x->nodes.size());
+    if (e == cudaSuccess) e = cudaMalloc(&d_layers, sizeof(heddle_layer) * L);
+    if (e == cudaSuccess && x->have_profile) e = cudaMalloc(&d_prof, sizeof(double) * x->profile.size());
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_types, x->types.data(), sizeof(heddle_gpu_type) * NT, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_nodes, x->nodes.data(), sizeof(heddle_node) * x->nodes.size(),
+                       cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_layers, x->layers.data(), sizeof(heddle_layer) * L, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && d_prof)
+        e = cudaMemcpy(d_prof, x->profile.data(), sizeof(double) * x->profile.size(),
+                       cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(x->d_img, 0, x->lay.bytes);
+    if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, sizeof(uint32_t));
+    if (e == cudaSuccess) {
+        hd::TableArgs a{};
+        a.lay = x->lay;
+        a.types = d_types;
+        a.nodes = d_nodes;
+        a.n_nodes = (int32_t)x->nodes.size();
+        a.layers = d_layers;
+        a.profile = d_prof;
+        a.boundary_bytes = x->boundary_bytes;
+        a.moe = x->moe;
+        a.img = x->d_img;
+        a.q = x->d_q;
+        a.flags = x->d_flags;
+        e = hd::launch_tables(a, 0);
+    }
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    uint32_t flags = 0;
+    if (e == cudaSuccess) e = cudaMemcpy(&flags, x->d_flags, sizeof(uint32_t), cudaMemcpyDeviceToHost);
+    cudaFree(d_types);
+    cudaFree(d_nodes);
+    cudaFree(d_layers);
+    if (d_prof) cudaFree(d_prof);
+    if (e != cudaSuccess) return fail(x, HEDDLE_E_CUDA, "cost-table build: %s", cudaGetErrorString(e));
+    if (flags & hd::kTabBadValue)
+        return fail(x, HEDDLE_E_ARG, "a per-layer cost is negative, not finite or above 4e18 ns");
+    if (flags & hd::kTabTooLarge)
+        return fail(x, HEDDLE_E_LIMIT, "a per-(type, degree) model time or a P2P term exceeds 2^40 ns");
+    x->tables_ready = true;
+    return ok(x);
+}
+
+heddle_status check_cands(heddle_ctx* x, const heddle_candidates* c, bool device) {
+    if (!c) return fail(x, HEDDLE_E_ARG, "candidates is NULL");
+    if (c->n < 0) return fail(x, HEDDLE_E_ARG, "negative candidate count");
+    if (c->n == 0) return HEDDLE_OK;
+    if (!c->S || !c->M || !c->code) return fail(x, HEDDLE_E_ARG, "null candidate array");
+    if (c->plane_stride < c->n) return fail(x, HEDDLE_E_ARG, "plane_stride below n");
+    if (c->s_max < 1 || c->s_max > HEDDLE_MAX_STAGES)
+        return fail(x, HEDDLE_E_ARG, "s_max must be in [1, %d]", HEDDLE_MAX_STAGES);
+    (void)device;
+    return HEDDLE_OK;
+}
+
+heddle_status check_ready(heddle_ctx* x) {
+    if (!x->have_cluster) return fail(x, HEDDLE_E_STATE, "no cluster loaded");
+    if (!x->have_model) return fail(x, HEDDLE_E_STATE, "no model loaded");
+    if (!x->tables_ready) return fail(x, HEDDLE_E_STATE, "cost tables are not built");
+    return HEDDLE_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+heddle_status heddle_create(heddle_ctx** out, int32_t device) {
+    if (!out) return HEDDLE_E_ARG;
+    *out = nullptr;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess || ndev == 0) return HEDDLE_E_CUDA;
+    if (device < 0 || device >= ndev) return HEDDLE_E_ARG;
+    heddle_ctx* x = new (std::nothrow) heddle_ctx();
+    if (!x) return HEDDLE_E_NOMEM;
+    x->device = device;
+    DeviceGuard dg(device);
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, device) != cudaSuccess) {
+        delete x;
+        return HEDDLE_E_CUDA;
+    }
+    x->num_sms = prop.multiProcessorCount;
+    x->scratch_blocks = 2 * x->num_sms;
+    cudaError_t e = cudaMalloc(&x->d_flags, 2 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, 2 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_counters, 3 * sizeof(unsigned long long));
+    if (e == cudaSuccess) e = cudaMemset(x->d_counters, 0, 3 * sizeof(unsigned long long));
+    if (e == cudaSuccess)
+        e = cudaMalloc(&x->d_scratch, sizeof(hd::TopkEntry) * hd::kMaxTopK * x->scratch_blocks);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch_count, sizeof(int32_t) * x->scratch_blocks);
+    if (e != cudaSuccess) {
+        heddle_destroy(x);
+        return HEDDLE_E_CUDA;
+    }
+    *out = x;
+    return HEDDLE_OK;
+}
+
+void heddle_destroy(heddle_ctx* x) {
+    if (!x) return;
+    DeviceGuard dg(x->device);
+    cudaFree(x->d_img);
+    cudaFree(x->d_q);
+    cudaFree(x->d_flags);
+    cudaFree(x->d_counters);
+    cudaFree(x->d_scratch);
+    cudaFree(x->d_scratch_count);
+    for (int b = 0; b < 2; ++b) {
+        cudaFree(x->st_S[b]);
+        cudaFree(x->st_M[b]);
+        cudaFree(x->st_code[b]);
+        cudaFree(x->st_T[b]);
+        cudaFree(x->st_B[b]);
+        cudaFree(x->st_n[b]);
+        cudaFree(x->st_status[b]);
+        cudaFree(x->st_bounds[b]);
+        if (x->ev_loaded[b]) cudaEventDestroy(x->ev_loaded[b]);
+        if (x->ev_priced[b]) cudaEventDestroy(x->ev_priced[b]);
+        if (x->ev_free[b]) cudaEventDestroy(x->ev_free[b]);
+    }
+    cudaFree(x->d_state);
+    if (x->s_h2d) cudaStreamDestroy(x->s_h2d);
+    if (x->s_d2h) cudaStreamDestroy(x->s_d2h);
+    delete x;
+}
+
+const char* heddle_last_error(const heddle_ctx* x) { return x ? x->msg : "null context"; }
+
+heddle_status heddle_load_cluster(heddle_ctx* x, const heddle_gpu_type* types, int32_t n_types,
+                                  const heddle_node* nodes, int32_t n_nodes) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!types || !nodes) return fail(x, HEDDLE_E_ARG, "null cluster array");
+    if (n_types < 1 || n_types > HEDDLE_MAX_TYPES)
+        return fail(x, HEDDLE_E_LIMIT, "n_types must be in [1, %d]", HEDDLE_MAX_TYPES);
+    if (n_nodes < 1) return fail(x, HEDDLE_E_ARG, "no nodes");
+    for (int g = 0; g < n_types; ++g) {
+        const heddle_gpu_type& t = types[g];
+        if (!(t.tflops > 0.0) || !isfinite(t.tflops))
+            return fail(x, HEDDLE_E_ARG, "type %d: tflops must be finite and positive", g);
+        if (t.mem_bytes < 1 || t.mem_bytes > kMemLimit)
+            return fail(x, HEDDLE_E_LIMIT, "type %d: mem_bytes outside [1, 2^50]", g);
+        if (t.intra_bw < 1 || t.intra_bw > kBwLimit)
+            return fail(x, HEDDLE_E_LIMIT, "type %d: intra_bw outside [1, 2^40]", g);
+    }
+    int64_t total = 0;
+    for (int b = 0; b < n_nodes; ++b) {
+        const heddle_node& nd = nodes[b];
+        if (nd.type < 0 || nd.type >= n_types) return fail(x, HEDDLE_E_ARG, "node %d: bad type", b);
+        if (nd.gpus < 1) return fail(x, HEDDLE_E_ARG, "node %d: gpus must be >= 1", b);
+        if (nd.nic_bw < 1 || nd.nic_bw > kBwLimit)
+            return fail(x, HEDDLE_E_LIMIT, "node %d: nic_bw outside [1, 2^40]", b);
+        total += nd.gpus;
+        if (total > HEDDLE_MAX_GPUS) return fail(x, HEDDLE_E_LIMIT, "more than %d GPUs", HEDDLE_MAX_GPUS);
+    }
+    DeviceGuard dg(x->device);
+    x->types.assign(types, types + n_types);
+    x->nodes.assign(nodes, nodes + n_nodes);
+    x->have_cluster = true;
+    return build_tables(x);
+}
+
+heddle_status heddle_load_model(heddle_ctx* x, const heddle_layer* layers, int32_t n_layers,
+                                int64_t boundary_bytes, int32_t flags, const double* profile_s) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!layers) return fail(x, HEDDLE_E_ARG, "layers is NULL");
+    if (n_layers < 1 || n_layers > HEDDLE_MAX_LAYERS)
+        return fail(x, HEDDLE_E_LIMIT, "n_layers must be in [1, %d]", HEDDLE_MAX_LAYERS);
+    if (boundary_bytes < 0 || boundary_bytes > kByteLimit)
+        return fail(x, HEDDLE_E_LIMIT, "boundary_bytes outside [0, 2^42]");
+    if (flags & ~HEDDLE_MODEL_MOE) return fail(x, HEDDLE_E_ARG, "unknown model flags");
+    for (int l = 0; l < n_layers; ++l) {
+        const heddle_layer& ly = layers[l];
+        if (!(ly.flops >= 0.0) || !isfinite(ly.flops))
+            return fail(x, HEDDLE_E_ARG, "layer %d: flops must be finite and >= 0", l);
+        const int64_t v[5] = {ly.param_bytes, ly.state_bytes, ly.act_bytes, ly.ar_bytes, ly.a2a_bytes};
+        for (int i = 0; i < 5; ++i)
+            if (v[i] < 0 || v[i] > kByteLimit)
+                return fail(x, HEDDLE_E_LIMIT, "layer %d: byte count outside [0, 2^42]", l);
+    }
+    if (profile_s && !x->have_cluster)
+        return fail(x, HEDDLE_E_STATE, "a profile needs the cluster loaded first");
+    DeviceGuard dg(x->device);
+    x->layers.assign(layers, layers + n_layers);
+    x->boundary_bytes = boundary_bytes;
+    x->moe = (flags & HEDDLE_MODEL_MOE) ? 1 : 0;
+    x->have_profile = profile_s != nullptr;
+    if (profile_s) {
+        const size_t n = (size_t)x->types.size() * 4 * n_layers;
+        x->profile.assign(profile_s, profile_s + n);
+    } else {
+        x->profile.clear();
+    }
+    x->have_model = true;
+    return build_tables(x);
+}
+
+heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
+                                      const heddle_results* r, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    heddle_status st = check_cands(x, c, true);
+    if (st != HEDDLE_OK) return st;
+    if (!r) return fail(x, HEDDLE_E_ARG, "results is NULL");
+    if ((st = check_ready(x)) != HEDDLE_OK) return st;
+    if (c->n == 0) return ok(x);
+    if (!r->T || !r->bottleneck || !r->n_dp || !r->status)
+        return fail(x, HEDDLE_E_ARG, "null result array");
+    DeviceGuard dg(x->device);
+    hd::PriceArgs a{};
+    a.lay = x->lay;
+    a.img = x->d_img;
+    a.moe = x->moe;
+    a.S = c->S;
+    a.M = c->M;
+    a.code = c->code;
+    a.n = c->n;
+    a.stride = c->plane_stride;
+    a.s_max = c->s_max;
+    a.T = r->T;
+    a.B = r->bottleneck;
+    a.ndp = r->n_dp;
+    a.status = r->status;
+    a.bounds = r->bounds;
+    a.err = x->d_flags + 1;
+    a.counters = x->count_next ? x->d_counters : nullptr;
+    x->count_next = false;
+    CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream));
+    return ok(x);
+}
+
+heddle_status heddle_topk_reset(heddle_ctx* x, heddle_topk_state* state, int32_t k, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!state) return fail(x, HEDDLE_E_ARG, "state is NULL");
+    if (k < 1 || k > HEDDLE_MAX_TOPK) return fail(x, HEDDLE_E_LIMIT, "k must be in [1, %d]", HEDDLE_MAX_TOPK);
+    DeviceGuard dg(x->device);
+    CU(hd::launch_topk_reset(state, k, (cudaStream_t)stream));
+    return ok(x);
+}
+
+heddle_status heddle_topk(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
+                          heddle_topk_state* state, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    heddle_status st = check_cands(x, c, true);
+    if (st != HEDDLE_OK) return st;
+    if (!r || !state) return fail(x, HEDDLE_E_ARG, "results or state is NULL");
+    if (c->n == 0) return ok(x);
+    if (!r->T || !r->n_dp || !r->status) return fail(x, HEDDLE_E_ARG, "null result array");
+    DeviceGuard dg(x->device);
+    hd::TopkArgs a{};
+    a.M = c->M;
+    a.T = r->T;
+    a.ndp = r->n_dp;
+    a.status = r->status;
+    a.n = c->n;
+    a.base_index = c->base_index;
+    a.state = state;
+    a.scratch = x->d_scratch;
+    a.scratch_count = x->d_scratch_count;
+    a.max_blocks = x->scratch_blocks;
+    CU(hd::launch_topk(a, x->num_sms, (cudaStream_t)stream));
+    return ok(x);
+}
+
+heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
+                                     const heddle_results* r, heddle_topk_state* state,
+                                     int64_t batch, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    heddle_status st = check_cands(x, c, false);
+    if (st != HEDDLE_OK) return st;
+    if (!state) return fail(x, HEDDLE_E_ARG, "state is NULL");
+    if (state->k < 1 || state->k > HEDDLE_MAX_TOPK)
+        return fail(x, HEDDLE_E_LIMIT, "state k must be in [1, %d]", HEDDLE_MAX_TOPK);
+    if (batch < 1) return fail(x, HEDDLE_E_ARG, "batch must be >= 1");
+    if ((st = check_ready(x)) != HEDDLE_OK) return st;
+    DeviceGuard dg(x->device);
+    cudaStream_t sc = (cudaStream_t)stream;
+    const int64_t n = c->n;
+    const int64_t nb_max = n < batch ? (n > 0 ? n : 1) : batch;
+    // staging buffers (grown on demand) and the copy streams / events
+    if (!x->s_h2d) {
+        CU(cudaStreamCreateWithFlags(&x->s_h2d, cudaStreamNonBlocking));
+        CU(cudaStreamCreateWithFlags(&x->s_d2h, cudaStreamNonBlocking));
+        for (int b = 0; b < 2; ++b) {
+            CU(cudaEventCreateWithFlags(&x->ev_loaded[b], cudaEventDisableTiming));
+            CU(cudaEventCreateWithFlags(&x->ev_priced[b], cudaEventDisableTiming));
+            CU(cudaEventCreateWithFlags(&x->ev_free[b], cudaEventDisableTiming));
+        }
+        CU(cudaMalloc(&x->d_state, sizeof(heddle_topk_state)));
+    }
+    if (x->stage_cap < nb_max || x->stage_smax < c->s_max) {
+        CU(cudaDeviceSynchronize());
+        const int64_t cap = nb_max > x->stage_cap ? nb_max : x->stage_cap;
+        const int32_t sm = c->s_max > x->stage_smax ? c->s_max : x->stage_smax;
+        for (int b = 0; b < 2; ++b) {
+            cudaFree(x->st_S[b]);
+            cudaFree(x->st_M[b]);
+            cudaFree(x->st_code[b]);
+            cudaFree(x->st_T[b]);
+            cudaFree(x->st_B[b]);
+            cudaFree(x->st_n[b]);
+            cudaFree(x->st_status[b]);
+            cudaFree(x->st_bounds[b]);
+            x->st_S[b] = nullptr;
+            x->st_M[b] = nullptr;
+            x->st_code[b] = nullptr;
+            x->st_T[b] = x->st_B[b] = nullptr;
+            x->st_n[b] = nullptr;
+            x->st_status[b] = x->st_bounds[b] = nullptr;
+            if (cudaMalloc(&x->st_S[b], cap) != cudaSuccess ||
+                cudaMalloc(&x->st_M[b], 2 * cap) != cudaSuccess ||
+                cudaMalloc(&x->st_code[b], (size_t)sm * cap) != cudaSuccess ||
+                cudaMalloc(&x->st_T[b], 8 * cap) != cudaSuccess ||
+                cudaMalloc(&x->st_B[b], 8 * cap) != cudaSuccess ||
+                cudaMalloc(&x->st_n[b], 2 * cap) != cudaSuccess ||
+                cudaMalloc(&x->st_status[b], cap) != cudaSuccess ||
+                cudaMalloc(&x->st_bounds[b], (size_t)HEDDLE_BOUND_PLANES * cap) != cudaSuccess) {
+                x->stage_cap = 0;
+                x->stage_smax = 0;
+                return fail(x, HEDDLE_E_NOMEM, "staging buffers for %lld candidates", (long long)cap);
+            }
+        }
+        x->stage_cap = cap;
+        x->stage_smax = sm;
+    }
+    CU(cudaMemcpyAsync(x->d_state, state, sizeof(heddle_topk_state), cudaMemcpyHostToDevice, sc));
+    CU(cudaEventRecord(x->ev_free[0], sc));
+    CU(cudaEventRecord(x->ev_free[1], sc));
+    const bool want_bounds = r && r->bounds;
+    for (int64_t lo = 0, it = 0; lo < n; lo += batch, ++it) {
+        const int b = (int)(it & 1);
+        const int64_t nb = (n - lo) < batch ? (n - lo) : batch;
+        // host -> device on the copy stream once the set is free
+        CU(cudaStreamWaitEvent(x->s_h2d, x->ev_free[b], 0));
+        CU(cudaMemcpyAsync(x->st_S[b], c->S + lo, nb, cudaMemcpyHostToDevice, x->s_h2d));
+        CU(cudaMemcpyAsync(x->st_M[b], c->M + lo, 2 * nb, cudaMemcpyHostToDevice, x->s_h2d));
+        CU(cudaMemcpy2DAsync(x->st_code[b], nb, c->code + lo, c->plane_stride, nb, c->s_max,
+                             cudaMemcpyHostToDevice, x->s_h2d));
+        CU(cudaEventRecord(x->ev_loaded[b], x->s_h2d));
+        // price and merge on the caller's stream
+        CU(cudaStreamWaitEvent(sc, x->ev_loaded[b], 0));
+        heddle_candidates cb{};
+        cb.S = x->st_S[b];
+        cb.M = x->st_M[b];
+        cb.code = x->st_code[b];
+        cb.n = nb;
+        cb.plane_stride = nb;
+        cb.s_max = c->s_max;
+        cb.base_index = c->base_index + lo;
+        heddle_results rb{};
+        rb.T = x->st_T[b];
+        rb.bottleneck = x->st_B[b];
+        rb.n_dp = x->st_n[b];
+        rb.status = x->st_status[b];
+        rb.bounds = want_bounds ? x->st_bounds[b] : nullptr;
+        if ((st = heddle_price_candidates(x, &cb, &rb, sc)) != HEDDLE_OK) return st;
+        if ((st = heddle_topk(x, &cb, &rb, x->d_state, sc)) != HEDDLE_OK) return st;
+        CU(cudaEventRecord(x->ev_priced[b], sc));
+        // device -> host of the requested result fields on the second copy stream
+        CU(cudaStreamWaitEvent(x->s_d2h, x->ev_priced[b], 0));
+        if (r && r->T) CU(cudaMemcpyAsync(r->T + lo, rb.T, 8 * nb, cudaMemcpyDeviceToHost, x->s_d2h));
+        if (r && r->bottleneck)
+            CU(cudaMemcpyAsync(r->bottleneck + lo, rb.bottleneck, 8 * nb, cudaMemcpyDeviceToHost, x->s_d2h));
+        if (r && r->n_dp) CU(cudaMemcpyAsync(r->n_dp + lo, rb.n_dp, 2 * nb, cudaMemcpyDeviceToHost, x->s_d2h));
+        if (r && r->status)
+            CU(cudaMemcpyAsync(r->status + lo, rb.status, nb, cudaMemcpyDeviceToHost, x->s_d2h));
+        if (want_bounds)
+            CU(cudaMemcpy2DAsync(r->bounds + lo, n, rb.bounds, nb, nb, HEDDLE_BOUND_PLANES,
+                                 cudaMemcpyDeviceToHost, x->s_d2h));
+        CU(cudaEventRecord(x->ev_free[b], x->s_d2h));
+    }
+    CU(cudaMemcpyAsync(state, x->d_state, sizeof(heddle_topk_state), cudaMemcpyDeviceToHost, sc));
+    CU(cudaStreamSynchronize(x->s_d2h));
+    CU(cudaStreamSynchronize(x->s_h2d));
+    CU(cudaStreamSynchronize(sc));
+    return ok(x);
+}
+
+heddle_status heddle_get_tables(heddle_ctx* x, int64_t* q, int64_t* p2p) {
+    if (!x) return HEDDLE_E_ARG;
+    heddle_status st = check_ready(x);
+    if (st != HEDDLE_OK) return st;
+    DeviceGuard dg(x->device);
+    if (q)
+        CU(cudaMemcpy(q, x->d_q, sizeof(int64_t) * (size_t)x->lay.NT * 4 * x->lay.L,
+                      cudaMemcpyDeviceToHost));
+    if (p2p) CU(cudaMemcpy(p2p, x->d_img + x->lay.offP2P, sizeof(int64_t) * 128, cudaMemcpyDeviceToHost));
+    return ok(x);
+}
+
+heddle_status heddle_device_errors(heddle_ctx* x, uint32_t* flags) {
+    if (!x || !flags) return x ? fail(x, HEDDLE_E_ARG, "flags is NULL") : HEDDLE_E_ARG;
+    DeviceGuard dg(x->device);
+    CU(cudaDeviceSynchronize());
+    CU(cudaMemcpy(flags, x->d_flags + 1, sizeof(uint32_t), cudaMemcpyDeviceToHost));
+    CU(cudaMemset(x->d_flags + 1, 0, sizeof(uint32_t)));
+    return ok(x);
+}
+
+heddle_status heddle_count_next(heddle_ctx* x, int32_t enable) {
+    if (!x) return HEDDLE_E_ARG;
+    x->count_next = enable != 0;
+    return ok(x);
+}
+
+heddle_status heddle_work_counters(heddle_ctx* x, uint64_t out[3]) {
+    if (!x || !out) return x ? fail(x, HEDDLE_E_ARG, "out is NULL") : HEDDLE_E_ARG;
+    DeviceGuard dg(x->device);
+    unsigned long long v[3];
+    CU(cudaDeviceSynchronize());
+    CU(cudaMemcpy(v, x->d_counters, sizeof(v), cudaMemcpyDeviceToHost));
+    CU(cudaMemset(x->d_counters, 0, sizeof(v)));
+    for (int i = 0; i < 3; ++i) out[i] = v[i];
+    return ok(x);
+}
+
+}  // extern "C"

@@ -1,0 +1,124 @@
+// heddle_internal.cuh -- definitions shared by the library's translation
+// units (never installed, never included by the oracle).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "heddle.h"
+
+namespace hd {
+
+constexpr int kMaxTypes = HEDDLE_MAX_TYPES;
+constexpr int kMaxStages = HEDDLE_MAX_STAGES;
+constexpr int kMaxLayers = HEDDLE_MAX_LAYERS;
+constexpr int kMaxTopK = HEDDLE_MAX_TOPK;
+constexpr int64_t kInf = INT64_MAX;
+
+// Device error flags (heddle_device_errors).
+constexpr uint32_t kErrStageWait = 1u;
+constexpr uint32_t kErrSearchBound = 2u;
+constexpr uint32_t kErrInternal = 4u;
+// Table-build flags (checked by the host at load time).
+constexpr uint32_t kTabBadValue = 1u;   // non-finite or negative per-layer cost
+constexpr uint32_t kTabTooLarge = 2u;   // a table total or P2P term above its limit
+
+// Byte layout of the cost-table image.  The pricing kernel copies the whole
+// image into shared memory with one bulk (TMA) copy per CTA, so every
+// section starts on a 16-byte boundary and the total is a multiple of 16.
+struct Layout {
+    int32_t L, NT;
+    uint32_t offP;      // int64 [NT][4][L+1]   prefix of per-layer ns per (type, degree)
+    uint32_t offSA;     // int64x2 [L+1]         prefix of (state bytes, activation bytes)
+    uint32_t offPB;     // int64 [L+1]           prefix of gradient bytes
+    uint32_t offP2P;    // int64 [8][8][2]       P2P ns (from, to, same-node)
+    uint32_t offMem;    // int64 [8]             memory per GPU
+    uint32_t offInter;  // int64 [8]             slowest NIC of the type
+    uint32_t offMinQ;   // int64 [NT][4]         cheapest single layer per (type, degree)
+    uint32_t offMaxN;   // int32 [8]             largest node of the type
+    uint32_t offPow2;   // int32 [8]             largest power of two <= largest node (<= 8)
+    uint32_t offGpus;   // int32 [8]             GPUs of the type
+    uint32_t offCap;    // int32 [8][4]          sum over nodes of floor(gpus / 2^e) * 2^e
+    uint32_t bytes;
+};
+
+inline uint32_t align16(uint32_t x) { return (x + 15u) & ~15u; }
+
+inline Layout make_layout(int L, int NT) {
+    Layout y{};
+    y.L = L;
+    y.NT = NT;
+    uint32_t o = 0;
+    y.offP = o;     o = align16(o + 8u * NT * 4 * (L + 1));
+    y.offSA = o;    o = align16(o + 16u * (L + 1));
+    y.offPB = o;    o = align16(o + 8u * (L + 1));
+    y.offP2P = o;   o = align16(o + 8u * 8 * 8 * 2);
+    y.offMem = o;   o = align16(o + 8u * 8);
+    y.offInter = o; o = align16(o + 8u * 8);
+    y.offMinQ = o;  o = align16(o + 8u * NT * 4);
+    y.offMaxN = o;  o = align16(o + 4u * 8);
+    y.offPow2 = o;  o = align16(o + 4u * 8);
+    y.offGpus = o;  o = align16(o + 4u * 8);
+    y.offCap = o;   o = align16(o + 4u * 8 * 4);
+    y.bytes = o;
+    return y;
+}
+
+struct TableArgs {
+    Layout lay;
+    const heddle_gpu_type* types;
+    const heddle_node* nodes;
+    int32_t n_nodes;
+    const heddle_layer* layers;
+    const double* profile;   // nullable
+    int64_t boundary_bytes;
+    int32_t moe;
+    unsigned char* img;      // out
+    int64_t* q;              // out [NT][4][L]
+    uint32_t* flags;         // out
+};
+cudaError_t launch_tables(const TableArgs& a, cudaStream_t st);
+
+struct PriceArgs {
+    Layout lay;
+    const unsigned char* img;
+    int32_t moe;
+    const uint8_t* S;
+    const uint16_t* M;
+    const uint8_t* code;
+    int64_t n;
+    int64_t stride;
+    int32_t s_max;
+    int64_t* T;
+    int64_t* B;
+    uint16_t* ndp;
+    uint8_t* status;
+    uint8_t* bounds;
+    uint32_t* err;
+    unsigned long long* counters;  // non-null selects the counting variant
+};
+cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st);
+
+struct TopkEntry {
+    int64_t idx;
+    int64_t T;
+    uint32_t nM;
+    uint32_t pad;
+};
+
+struct TopkArgs {
+    const uint16_t* M;
+    const int64_t* T;
+    const uint16_t* ndp;
+    const uint8_t* status;
+    int64_t n;
+    int64_t base_index;
+    heddle_topk_state* state;  // device, in/out
+    TopkEntry* scratch;        // [grid][kMaxTopK]
+    int32_t* scratch_count;    // [grid]
+    int32_t max_blocks;
+};
+cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st);
+
+}  // namespace hd

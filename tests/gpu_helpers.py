@@ -1,0 +1,87 @@
+"""Helpers for the GPU tests: run the CUDA path through the C ABI and the
+oracle on the same seeded inputs."""
+
+from __future__ import annotations
+
+import functools
+
+import numpy as np
+
+
+def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False):
+    """Price on the GPU through the C ABI; returns numpy results, the top-k
+    and (optionally) the work counters.  ``batch`` splits the candidates into
+    consecutive launches merged into one top-k state."""
+    import torch
+    ctx = h.heddle_create(0)
+    try:
+        h.heddle_load_cluster(ctx, w_cluster)
+        h.heddle_load_model(ctx, w_model)
+        n = int(cands["S"].shape[0])
+        dc = h.cands_to_device(cands)
+        res = h.alloc_results(n, bounds=False)
+        state = h.alloc_topk_state()
+        h.heddle_topk_reset(ctx, state, k)
+        batch = n if batch is None else batch
+        out_bounds = np.zeros((33, n), np.uint8) if bounds else None
+        if count:
+            h.heddle_count_next(ctx, True)
+        for lo in range(0, max(n, 1), max(batch, 1)):
+            hi = min(n, lo + batch)
+            if hi <= lo:
+                break
+            bb = torch.empty((33, hi - lo), dtype=torch.uint8, device="cuda") if bounds else None
+            c = h.make_candidates(dc, lo, hi)
+            r = h.heddle_results(res["T"].data_ptr() + 8 * lo, res["bottleneck"].data_ptr() + 8 * lo,
+                                 res["n_dp"].data_ptr() + 2 * lo, res["status"].data_ptr() + lo,
+                                 None if bb is None else bb.data_ptr())
+            h.heddle_price_candidates(ctx, c, r)
+            h.heddle_topk(ctx, c, r, state)
+            if bounds:
+                out_bounds[:, lo:hi] = bb.cpu().numpy()
+        torch.cuda.synchronize()
+        out = h.results_to_numpy(res)
+        out["bounds"] = out_bounds
+        out["topk"] = h.read_topk_state(state)
+        out["errors"] = h.heddle_device_errors(ctx)
+        if count:
+            out["counters"] = h.heddle_work_counters(ctx)
+        return out
+    finally:
+        h.heddle_destroy(ctx)
+
+
+def assert_same(gpu, orc, idx=None, what=""):
+    """Bit-exact comparison of every per-candidate field (optionally on the
+    sampled indices ``idx``; the oracle then holds results for idx only)."""
+    for key in ("status", "n_dp", "T", "bottleneck"):
+        g = gpu[key] if idx is None else gpu[key][idx]
+        o = orc[key]
+        bad = np.nonzero(g != o)[0]
+        assert bad.size == 0, "%s %s differs at %d candidates, first %s: gpu %s oracle %s" % (
+            what, key, bad.size, bad[:5], g[bad[:5]], o[bad[:5]])
+    if gpu.get("bounds") is not None and orc.get("bounds") is not None:
+        g = gpu["bounds"] if idx is None else gpu["bounds"][:, idx]
+        bad = np.nonzero((g != orc["bounds"]).any(axis=0))[0]
+        assert bad.size == 0, "%s bounds differ at %d candidates, first %s" % (what, bad.size, bad[:5])
+
+
+def exact_topk(idx_all, T, nM, k):
+    """Exact top-k of (idx, T, nM) triples by nM/T then smaller idx, using a
+    float64 pre-filter and integer cross-multiplication to finish."""
+    if len(idx_all) == 0:
+        return []
+    key = nM.astype(np.float64) / T.astype(np.float64)
+    m = min(len(key), max(4 * k, 1000))
+    thresh = np.partition(key, len(key) - m)[len(key) - m]
+    sel = np.nonzero(key >= thresh)[0]
+    items = [(int(idx_all[i]), int(T[i]), int(nM[i])) for i in sel]
+
+    def cmp(a, b):
+        l, r = a[2] * b[1], b[2] * a[1]
+        if l != r:
+            return -1 if l > r else 1
+        return -1 if a[0] < b[0] else (1 if a[0] > b[0] else 0)
+
+    items.sort(key=functools.cmp_to_key(cmp))
+    return items[:k]

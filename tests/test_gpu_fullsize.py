@@ -1,0 +1,48 @@
+"""Full-size workloads in the benchmark's launch configuration (device-resident
+batches of at most 1e6 candidates priced and merged into one top-k state):
+every sampled candidate bit-exact against the oracle, the top-k equal to an
+exact host top-k of the GPU's own per-candidate outputs, and every top-k
+entry re-priced by the oracle."""
+
+import numpy as np
+import pytest
+
+import gpu_helpers as G
+
+pytestmark = pytest.mark.gpu
+
+FULL = [("dense32", 100_000, None), ("dense80", 1_000_000, 4000), ("moe48", 1_000_000, 4000),
+        ("stress128", 10_000_000, 300)]
+
+
+@pytest.mark.parametrize("name,n,per_batch_sample", FULL)
+def test_full_size(heddle_lib, oracle_mod, name, n, per_batch_sample):
+    import torch
+    from paper_2609_34244_gb300 import workloads as W
+    assert torch.cuda.is_available()
+    h = heddle_lib
+    w = W.make_workload(name, seed=0, n=n)
+    batch = 1_000_000
+    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, bounds=False, batch=batch)
+    assert got["errors"] == 0
+    orc = oracle_mod.Oracle(w.cluster, w.model)
+    rng = np.random.default_rng(123)
+    if per_batch_sample is None:
+        idx = np.arange(n)
+    else:
+        idx = np.concatenate([lo + rng.choice(min(batch, n - lo), per_batch_sample, replace=False)
+                              for lo in range(0, n, batch)])
+    sub = W.make_cands(w.cands["S"][idx], w.cands["M"][idx], np.ascontiguousarray(w.cands["code"][:, idx]))
+    ref = orc.price(sub, threads=16, bounds=False)
+    G.assert_same(got, ref, idx=idx, what=name)
+    # top-k of the GPU outputs, computed exactly on the host
+    ok = np.nonzero(got["status"] == 0)[0]
+    nM = got["n_dp"][ok].astype(np.int64) * w.cands["M"][ok].astype(np.int64)
+    exp = G.exact_topk(ok, got["T"][ok], nM, 16)
+    assert got["topk"]["idx"].tolist() == [e[0] for e in exp]
+    # and every top-k entry priced again by the oracle
+    ti = got["topk"]["idx"]
+    tsub = W.make_cands(w.cands["S"][ti], w.cands["M"][ti], np.ascontiguousarray(w.cands["code"][:, ti]))
+    tref = orc.price(tsub, bounds=False)
+    assert (tref["T"] == got["topk"]["T"]).all()
+    assert (tref["n_dp"].astype(np.uint32) * w.cands["M"][ti].astype(np.uint32) == got["topk"]["nM"]).all()
