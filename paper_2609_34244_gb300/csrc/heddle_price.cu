@@ -20,10 +20,18 @@
 // smallest it rejected (lo): every B' in [hi, B] (feasible probe) or
 // [B, lo) (infeasible probe) takes the same decisions, so the search moves
 // its bracket to those values and ends on B* = the smallest feasible B,
-// itself a stage cost.  The C sets of that last probe give the canonical
+// itself a stage cost.  The C sets of the probe at B* give the canonical
 // split directly: a_{s+1} = min { j in C_{s+1} : j > a_s }, the smallest
 // boundary vector attaining B* (the feasible splits form a lattice under
 // componentwise min).
+//
+// Memory layout: the tables live in shared memory; per-thread state that is
+// indexed by a stage or a set word (stage codes, the forward bounds U, the
+// two position sets the backward pass reads and writes) lives in shared
+// memory interleaved by thread (element e of thread t at [e * kBlock + t]),
+// so each lane hits its own bank whatever index it uses.  A stage's
+// parameters are held in registers while that stage is swept.  Only the last
+// probe writes its sets to local memory, for the canonical split.
 
 #include <algorithm>
 
@@ -34,12 +42,11 @@ namespace {
 
 typedef unsigned __int128 u128;
 
-constexpr int kBlock = 128;
+constexpr int kBlock = 256;
 constexpr int kWords = 8;  // 256-bit position sets (L <= 255)
+constexpr int kCodeWords = kMaxStages / 4;
 constexpr int kMaxIters = 256;
 constexpr long long kStageWaitSpins = 1 << 22;
-
-enum { CHK_OK = 0, CHK_FAIL = 1, CHK_MEM = 2 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -89,7 +96,6 @@ struct Tabs {
     const int64_t* p2p;
     const int64_t* mem;
     const int64_t* inter;
-    const int64_t* minq;
     const int32_t* maxn;
     const int32_t* pow2;
     const int32_t* gpus;
@@ -97,45 +103,75 @@ struct Tabs {
     int L, NT;
 };
 
-// One candidate's per-stage view plus the position sets of the probes.
-struct Work {
-    int S, L;
-    uint16_t row[kMaxStages];      // offset of the stage's prefix row in P
-    int64_t c[kMaxStages];         // P2P to the next stage
-    int64_t capk[kMaxStages];      // memory per GPU x group size
-    int32_t f[kMaxStages];         // in-flight microbatches
-    uint8_t U[kMaxStages + 1];
-    int16_t cmin[kMaxStages + 1], cmax[kMaxStages + 1];
-    uint32_t C[kMaxStages + 1][kWords];
-    int64_t hi_c, lo_c;            // snapping values of the current probe
+// Per-thread views into the interleaved shared-memory arrays (already offset
+// by the thread index; element e at [e * kBlock]).
+struct Lane {
+    uint32_t* code4;  // [kCodeWords] four stage codes per word
+    uint8_t* U;       // [kMaxStages + 1]
+    uint32_t* C[2];   // [words] two position sets
+};
+
+__device__ __forceinline__ int stage_code(const Lane& ln, int s) {
+    return (ln.code4[(s >> 2) * kBlock] >> ((s & 3) * 8)) & 0xff;
+}
+
+// Parameters of one stage, held in registers while the stage is swept.
+struct Stage {
+    const int64_t* P;  // prefix row of the stage's (type, degree)
+    int64_t c;         // P2P to the next stage
+    int64_t capk;      // memory per GPU x group size
+    int32_t f;         // in-flight microbatches
+};
+
+__device__ __forceinline__ Stage load_stage(const Tabs& t, const Lane& ln, int s, int S, int M) {
+    const int code = stage_code(ln, s);
+    const int g = code & 7, j = (code >> 3) & 3;
+    Stage st;
+    st.P = t.P + (g * 4 + j) * (t.L + 1);
+    st.capk = t.mem[g] << j;
+    st.f = min(S - s, M);
+    st.c = 0;
+    if (s + 1 < S) {
+        const int cn = stage_code(ln, s + 1);
+        const int h = cn & 7, jn = (cn >> 3) & 3;
+        const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
+        st.c = t.p2p[(g * 8 + h) * 2 + same];
+    }
+    return st;
+}
+
+// Snapping values of the current probe.
+struct Snap {
+    int64_t hi, lo;
     unsigned long long checks;
 };
 
-__device__ __forceinline__ int check(const Tabs& t, Work& w, int s, int i, int j, int64_t B) {
-    const int64_t* P = t.P + w.row[s];
-    const longlong2 a = t.SA[i], b = t.SA[j];
-    const int64_t mem = (b.x - a.x) + (int64_t)w.f[s] * (b.y - a.y);
-    ++w.checks;
-    if (mem > w.capk[s]) return CHK_MEM;
-    const int64_t cost = P[j] - P[i] + w.c[s];
+// Interval [i, j) on stage st with cached prefix values of both ends:
+// 0 fits (cost <= B), 1 too slow, 2 out of memory.
+__device__ __forceinline__ int judge(const Stage& st, int64_t Pi, longlong2 Si, int64_t Pj, longlong2 Sj,
+                                     int64_t B, Snap& sn) {
+    ++sn.checks;
+    const int64_t mem = (Sj.x - Si.x) + (int64_t)st.f * (Sj.y - Si.y);
+    if (mem > st.capk) return 2;
+    const int64_t cost = Pj - Pi + st.c;
     if (cost <= B) {
-        if (cost > w.hi_c) w.hi_c = cost;
-        return CHK_OK;
+        sn.hi = max(sn.hi, cost);
+        return 0;
     }
-    if (cost < w.lo_c) w.lo_c = cost;
-    return CHK_FAIL;
+    sn.lo = min(sn.lo, cost);
+    return 1;
 }
 
-__device__ __forceinline__ bool bit_test(const uint32_t* C, int i) { return (C[i >> 5] >> (i & 31)) & 1u; }
+__device__ __forceinline__ uint32_t word(const uint32_t* C, int w) { return C[w * kBlock]; }
 
 // largest set position in [lo, i], -1 if none
 __device__ __forceinline__ int prev_set(const uint32_t* C, int i, int lo) {
     if (i < lo) return -1;
     int wd = i >> 5;
-    uint32_t m = C[wd] & (0xffffffffu >> (31 - (i & 31)));
+    uint32_t m = word(C, wd) & (0xffffffffu >> (31 - (i & 31)));
     while (m == 0) {
         if (--wd < (lo >> 5)) return -1;
-        m = C[wd];
+        m = word(C, wd);
     }
     const int x = (wd << 5) + 31 - __clz(m);
     return x >= lo ? x : -1;
@@ -145,67 +181,120 @@ __device__ __forceinline__ int prev_set(const uint32_t* C, int i, int lo) {
 __device__ __forceinline__ int next_set(const uint32_t* C, int i, int hi) {
     if (i > hi) return -1;
     int wd = i >> 5;
-    uint32_t m = C[wd] & (0xffffffffu << (i & 31));
+    uint32_t m = word(C, wd) & (0xffffffffu << (i & 31));
     while (m == 0) {
         if (++wd > (hi >> 5)) return -1;
-        m = C[wd];
+        m = word(C, wd);
     }
     const int x = (wd << 5) + __ffs(m) - 1;
     return x <= hi ? x : -1;
 }
 
-__device__ bool probe(const Tabs& t, Work& w, int64_t B) {
-    const int S = w.S, L = w.L;
-    w.hi_c = -1;
-    w.lo_c = kInf;
+// Sets of the probe at B*, kept for the canonical split (local memory).
+struct Final {
+    uint32_t w[kMaxStages + 1][kWords];
+    int16_t lo[kMaxStages + 1], hi[kMaxStages + 1];
+};
+
+template <bool kStore>
+__device__ bool probe(const Tabs& t, const Lane& ln, int S, int M, int64_t B, Snap& sn, Final* fin) {
+    const int L = t.L;
+    sn.hi = -1;
+    sn.lo = kInf;
     // forward upper bounds on the boundaries
-    w.U[0] = 0;
+    int u = 0;
+    ln.U[0] = 0;
     for (int s = 0; s + 1 < S; ++s) {
-        const int i = w.U[s];
+        const Stage st = load_stage(t, ln, s, S, M);
+        const int64_t Pi = st.P[u];
+        const longlong2 Si = t.SA[u];
         const int lim = L - (S - 1 - s);
-        int j = i;
-        while (j + 1 <= lim && check(t, w, s, i, j + 1, B) == CHK_OK) ++j;
+        int j = u;
+        while (j + 1 <= lim) {
+            if (judge(st, Pi, Si, st.P[j + 1], t.SA[j + 1], B, sn) != 0) break;
+            ++j;
+        }
         if (j < s + 1) return false;
-        w.U[s + 1] = (uint8_t)j;
+        u = j;
+        ln.U[(s + 1) * kBlock] = (uint8_t)j;
     }
-    // backward feasible-start sets
+    // backward feasible-start sets: C_S = {L}, then stages S-1 .. 1
+    int cur = 0;
     {
-        // C_S = {L}; clear every word a successor search of stage S-1 can
-        // read (positions S..L)
-        uint32_t* CS = w.C[S];
-        for (int wd = S >> 5; wd < (L >> 5); ++wd) CS[wd] = 0;
-        CS[L >> 5] = 1u << (L & 31);
-        w.cmin[S] = w.cmax[S] = (int16_t)L;
+        uint32_t* CS = ln.C[cur];
+        for (int wd = S >> 5; wd < (L >> 5); ++wd) CS[wd * kBlock] = 0;
+        CS[(L >> 5) * kBlock] = 1u << (L & 31);
     }
+    int nmin = L, nmax = L;
     for (int s = S - 1; s >= 1; --s) {
-        const uint32_t* Cn = w.C[s + 1];
-        const int nmin = w.cmin[s + 1], nmax = w.cmax[s + 1];
-        const int top = min((int)w.U[s], nmax - 1);
+        const uint32_t* Cn = ln.C[cur];
+        uint32_t* Cs = ln.C[cur ^ 1];
+        const int top = min((int)ln.U[s * kBlock], nmax - 1);
         if (top < s) return false;
-        uint32_t* Cs = w.C[s];
-        for (int wd = s >> 5; wd <= (top >> 5); ++wd) Cs[wd] = 0;
+        const Stage st = load_stage(t, ln, s, S, M);
+        for (int wd = s >> 5; wd <= (top >> 5); ++wd) Cs[wd * kBlock] = 0;
         int succ = next_set(Cn, top + 1, nmax);
+        int64_t Pj = st.P[succ];
+        longlong2 Sj = t.SA[succ];
         int i = top, hi = -1, lo = -1;
+        int accw = top >> 5;  // word of Cs being assembled
+        uint32_t acc = 0;
+        int cnw = -1;         // cached word of Cn
+        uint32_t cn = 0;
         while (i >= s) {
-            const int r = check(t, w, s, i, succ, B);
-            if (r == CHK_OK) {
-                Cs[i >> 5] |= 1u << (i & 31);
+            const int64_t Pi = st.P[i];
+            const longlong2 Si = t.SA[i];
+            if (judge(st, Pi, Si, Pj, Sj, B, sn) == 0) {
+                if ((i >> 5) != accw) {
+                    Cs[accw * kBlock] = acc;
+                    accw = i >> 5;
+                    acc = 0;
+                }
+                acc |= 1u << (i & 31);
                 if (hi < 0) hi = i;
                 lo = i;
-                if (i >= nmin && bit_test(Cn, i)) succ = i;
+                if (i >= nmin) {
+                    if ((i >> 5) != cnw) {
+                        cnw = i >> 5;
+                        cn = word(Cn, cnw);
+                    }
+                    if ((cn >> (i & 31)) & 1u) {
+                        succ = i;
+                        Pj = Pi;
+                        Sj = Si;
+                    }
+                }
                 --i;
             } else {
                 const int j2 = prev_set(Cn, i, nmin);
                 if (j2 < 0) break;
                 i = j2 - 1;
                 succ = j2;
+                Pj = st.P[j2];
+                Sj = t.SA[j2];
             }
         }
+        Cs[accw * kBlock] = acc;
         if (hi < 0) return false;
-        w.cmin[s] = (int16_t)lo;
-        w.cmax[s] = (int16_t)hi;
+        if (kStore) {
+            for (int wd = lo >> 5; wd <= (hi >> 5); ++wd) fin->w[s][wd] = Cs[wd * kBlock];
+            fin->lo[s] = (int16_t)lo;
+            fin->hi[s] = (int16_t)hi;
+        }
+        cur ^= 1;
+        nmin = lo;
+        nmax = hi;
     }
-    return check(t, w, 0, 0, w.cmin[1], B) == CHK_OK;
+    const Stage st0 = load_stage(t, ln, 0, S, M);
+    return judge(st0, st0.P[0], t.SA[0], st0.P[nmin], t.SA[nmin], B, sn) == 0;
+}
+
+// floor(a / b) for 0 <= a < 2^24, 1 <= b < 2^16: float estimate, integer fix-up
+__device__ __forceinline__ int64_t small_div(int64_t a, int64_t b) {
+    int64_t q = (int64_t)((float)a * __frcp_rn((float)b));
+    while (q > 0 && q * b > a) --q;
+    while ((q + 1) * b <= a) ++q;
+    return q;
 }
 
 template <bool kCount>
@@ -222,7 +311,6 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
     t.p2p = reinterpret_cast<const int64_t*>(smem + y.offP2P);
     t.mem = reinterpret_cast<const int64_t*>(smem + y.offMem);
     t.inter = reinterpret_cast<const int64_t*>(smem + y.offInter);
-    t.minq = reinterpret_cast<const int64_t*>(smem + y.offMinQ);
     t.maxn = reinterpret_cast<const int32_t*>(smem + y.offMaxN);
     t.pow2 = reinterpret_cast<const int32_t*>(smem + y.offPow2);
     t.gpus = reinterpret_cast<const int32_t*>(smem + y.offGpus);
@@ -230,11 +318,20 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
     t.L = y.L;
     t.NT = y.NT;
     const int L = y.L;
+    const int W = (L >> 5) + 1;
 
-    Work w;
-    w.L = L;
+    // per-thread interleaved arrays after the table image
+    uint32_t* lane_words = reinterpret_cast<uint32_t*>(smem + y.bytes);
+    Lane ln;
+    ln.code4 = lane_words + threadIdx.x;
+    ln.C[0] = lane_words + kCodeWords * kBlock + threadIdx.x;
+    ln.C[1] = ln.C[0] + W * kBlock;
+    ln.U = reinterpret_cast<uint8_t*>(lane_words + (kCodeWords + 2 * W) * kBlock) + threadIdx.x;
+
+    Snap sn;
+    sn.checks = 0;
     unsigned long long probes = 0, priced = 0;
-    w.checks = 0;
+    Final fin;
 
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < a.n; c += stride) {
@@ -242,80 +339,83 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
         const int M = a.M[c];
         int status = HEDDLE_CAND_OK;
         int64_t n = 0;
-        uint8_t codes[kMaxStages];
-        // ---- decode + validate (§5.1 depth / device / TP masks)
+        // ---- decode + validate (§5.1 depth / device / TP masks); DP demand
+        // per (type, size class) in 16-bit lanes: class e counts the GPUs of
+        // groups (or blocks) of at least 2^e GPUs, types 0-3 in lo, 4-7 in hi
+        uint64_t dlo[4] = {0, 0, 0, 0}, dhi[4] = {0, 0, 0, 0};
         if (S < 1 || S > kMaxStages || S > a.s_max || S > L || M < 1) {
             status = HEDDLE_CAND_INVALID;
         } else {
+            uint32_t packed = 0;
             for (int s = 0; s < S; ++s) {
                 const int b = a.code[(int64_t)s * a.stride + c];
-                codes[s] = (uint8_t)b;
+                packed |= (uint32_t)b << ((s & 3) * 8);
+                if ((s & 3) == 3 || s == S - 1) {
+                    ln.code4[(s >> 2) * kBlock] = packed;
+                    packed = 0;
+                }
                 const int g = b & 7, j = (b >> 3) & 3;
-                if ((b >> 5) != 0 || g >= t.NT || t.gpus[g] == 0 ||
-                    (!a.moe && (1 << j) > t.maxn[g]))
+                if ((b >> 5) != 0 || g >= t.NT || t.gpus[g] == 0 || (!a.moe && (1 << j) > t.maxn[g])) {
                     status = HEDDLE_CAND_INVALID;
+                } else {
+                    const int k = 1 << j;
+                    const int unit = k <= t.maxn[g] ? k : t.pow2[g];
+                    const uint64_t add = (uint64_t)k << (16 * (g & 3));
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        if ((1 << e) <= unit) {
+                            if (g < 4)
+                                dlo[e] += add;
+                            else
+                                dhi[e] += add;
+                        }
+                    }
+                }
             }
         }
         // ---- DP degree: n = min over (type, size class) of capacity / demand
         if (status == HEDDLE_CAND_OK) {
-            uint16_t dem[kMaxTypes][4];
-            for (int g = 0; g < kMaxTypes; ++g)
-                for (int e = 0; e < 4; ++e) dem[g][e] = 0;
-            for (int s = 0; s < S; ++s) {
-                const int g = codes[s] & 7, j = (codes[s] >> 3) & 3;
-                const int k = 1 << j;
-                const int unit = k <= t.maxn[g] ? k : t.pow2[g];
-                for (int e = 0; (1 << e) <= unit; ++e) dem[g][e] += (uint16_t)k;
-            }
             n = kInf;
-            for (int g = 0; g < t.NT; ++g)
-                for (int e = 0; e < 4; ++e)
-                    if (dem[g][e]) n = min(n, (int64_t)(t.cap[g * 4 + e] / dem[g][e]));
+#pragma unroll
+            for (int g = 0; g < kMaxTypes; ++g) {
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const uint64_t v = g < 4 ? dlo[e] : dhi[e];
+                    const int64_t d = (int64_t)((v >> (16 * (g & 3))) & 0xffff);
+                    if (d) n = min(n, small_div(t.cap[g * 4 + e], d));
+                }
+            }
             if (n == 0) status = HEDDLE_CAND_NO_FIT;
         }
         int64_t Bstar = -1, T = -1;
+        uint8_t bnd[kMaxStages + 1];
         if (status == HEDDLE_CAND_OK) {
             if (kCount) ++priced;
-            // ---- stage views
-            w.S = S;
-            for (int s = 0; s < S; ++s) {
-                const int g = codes[s] & 7, j = (codes[s] >> 3) & 3;
-                w.row[s] = (uint16_t)((g * 4 + j) * (L + 1));
-                if (s + 1 < S) {
-                    const int h = codes[s + 1] & 7, jn = (codes[s + 1] >> 3) & 3;
-                    const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
-                    w.c[s] = t.p2p[(g * 8 + h) * 2 + same];
-                } else {
-                    w.c[s] = 0;
-                }
-                w.capk[s] = t.mem[g] << j;
-                w.f[s] = min(S - s, M);
-            }
             // ---- PartitionLayers: memory-only probe, then the threshold search
             if (kCount) ++probes;
-            if (!probe(t, w, kInf)) {
+            if (!probe<false>(t, ln, S, M, kInf, sn, nullptr)) {
                 status = HEDDLE_CAND_OOM;
             } else {
-                int64_t hi = w.hi_c, lo = 0;
+                int64_t hi = sn.hi, lo = 0;
                 bool lo_known = false;
                 // first guess: the balanced bottleneck of a proportional split
                 float inv = 0.f, cw = 0.f;
                 for (int s = 0; s < S; ++s) {
-                    const float tot = (float)t.P[w.row[s] + L] + 1.0f;
+                    const Stage st = load_stage(t, ln, s, S, M);
+                    const float tot = (float)st.P[L] + 1.0f;
                     inv += 1.0f / tot;
-                    cw += (float)w.c[s] / tot;
+                    cw += (float)st.c / tot;
                 }
                 int64_t B = (int64_t)((1.0f + cw) / inv);
                 int64_t step = max((int64_t)1, (int64_t)((float)B * (float)S / (2.0f * (float)L)));
                 int it = 0;
                 while (lo < hi) {
-                    if (B < lo) B = lo;
-                    if (B > hi - 1) B = hi - 1;
+                    B = min(max(B, lo), hi - 1);
                     if (kCount) ++probes;
-                    if (probe(t, w, B)) {
-                        hi = w.hi_c;
+                    if (probe<false>(t, ln, S, M, B, sn, nullptr)) {
+                        hi = sn.hi;
                     } else {
-                        lo = w.lo_c;
+                        lo = sn.lo;
                         lo_known = true;
                     }
                     if (lo >= hi) break;
@@ -331,14 +431,16 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
                     }
                 }
                 Bstar = hi;
-                // sets of the optimum for the canonical split
+                // the sets of the optimum give the canonical split
                 if (kCount) ++probes;
-                if (!probe(t, w, Bstar)) atomicOr(a.err, kErrInternal);
-                uint8_t bnd[kMaxStages + 1];
+                if (!probe<true>(t, ln, S, M, Bstar, sn, &fin)) atomicOr(a.err, kErrInternal);
                 bnd[0] = 0;
                 for (int s = 0; s + 1 < S; ++s) {
-                    const int x = next_set(w.C[s + 1], bnd[s] + 1, w.cmax[s + 1]);
-                    bnd[s + 1] = (uint8_t)(x < 0 ? 0 : x);
+                    const int from = max((int)bnd[s] + 1, (int)fin.lo[s + 1]);
+                    int wd = from >> 5;
+                    uint32_t m = fin.w[s + 1][wd] & (0xffffffffu << (from & 31));
+                    while (m == 0 && wd < (fin.hi[s + 1] >> 5)) m = fin.w[s + 1][++wd];
+                    bnd[s + 1] = (uint8_t)(m ? (wd << 5) + __ffs(m) - 1 : 0);
                 }
                 bnd[S] = (uint8_t)L;
                 // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s
@@ -346,13 +448,14 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
                 int sg = -1;
                 u128 bestG = 0, bestD = 1;
                 for (int s = 0; s < S; ++s) {
-                    const int64_t* P = t.P + w.row[s];
-                    const int64_t ts = P[bnd[s + 1]] - P[bnd[s]] + w.c[s];
+                    const Stage st = load_stage(t, ln, s, S, M);
+                    const int64_t ts = st.P[bnd[s + 1]] - st.P[bnd[s]] + st.c;
                     tmax = max(tmax, ts);
                     tsum += ts;
                     if (n > 1) {
                         // stage with the largest G_s / (k_s bw_s), compared exactly
-                        const int g = codes[s] & 7, j = (codes[s] >> 3) & 3;
+                        const int code = stage_code(ln, s);
+                        const int g = code & 7, j = (code >> 3) & 3;
                         const u128 G = (u128)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
                         const u128 D = (u128)t.inter[g] << j;
                         if (sg < 0 || G * bestD > bestG * D) {
@@ -371,22 +474,20 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
                     gmax = (int64_t)((num + den - 1) / den);
                 }
                 T = (int64_t)(M - 1) * Bstar + tsum + gmax;
-                if (a.bounds) {
-                    for (int s = 0; s <= kMaxStages; ++s)
-                        a.bounds[(int64_t)s * a.n + c] = s <= S ? bnd[s] : 0;
-                }
             }
         }
-        a.T[c] = status == HEDDLE_CAND_OK ? T : -1;
-        a.B[c] = status == HEDDLE_CAND_OK ? Bstar : -1;
-        a.ndp[c] = (uint16_t)((status == HEDDLE_CAND_OK || status == HEDDLE_CAND_OOM) ? n : 0);
+        const bool ok = status == HEDDLE_CAND_OK;
+        a.T[c] = ok ? T : -1;
+        a.B[c] = ok ? Bstar : -1;
+        a.ndp[c] = (uint16_t)((ok || status == HEDDLE_CAND_OOM) ? n : 0);
         a.status[c] = (uint8_t)status;
-        if (a.bounds && status != HEDDLE_CAND_OK) {
-            for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.n + c] = 0;
+        if (a.bounds) {
+            for (int s = 0; s <= kMaxStages; ++s)
+                a.bounds[(int64_t)s * a.n + c] = (ok && s <= S) ? bnd[s] : 0;
         }
     }
     if (kCount) {
-        unsigned long long v0 = w.checks, v1 = probes, v2 = priced;
+        unsigned long long v0 = sn.checks, v1 = probes, v2 = priced;
         for (int o = 16; o > 0; o >>= 1) {
             v0 += __shfl_down_sync(0xffffffffu, v0, o);
             v1 += __shfl_down_sync(0xffffffffu, v1, o);
@@ -400,33 +501,33 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
     }
 }
 
+// shared memory of the per-thread interleaved arrays
+size_t lane_bytes(int L) {
+    const int W = (L >> 5) + 1;
+    return (size_t)kBlock * (4 * kCodeWords + 4 * 2 * W + (kMaxStages + 1));
+}
+
+template <bool kCount>
+cudaError_t launch_one(const PriceArgs& a, int num_sms, cudaStream_t st) {
+    const size_t smem = a.lay.bytes + lane_bytes(a.lay.L);
+    cudaError_t e = cudaFuncSetAttribute(price_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, price_kernel<kCount>, kBlock, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const int64_t need = (a.n + kBlock - 1) / kBlock;
+    const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
+    price_kernel<kCount><<<grid, kBlock, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
-    const size_t smem = a.lay.bytes;
-    cudaError_t e;
-    int per_sm = 0;
-    if (a.counters) {
-        e = cudaFuncSetAttribute(price_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
-        if (e != cudaSuccess) return e;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, price_kernel<true>, kBlock, smem);
-    } else {
-        e = cudaFuncSetAttribute(price_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem);
-        if (e != cudaSuccess) return e;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, price_kernel<false>, kBlock, smem);
-    }
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) per_sm = 1;
-    const int64_t need = (a.n + kBlock - 1) / kBlock;
-    const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
-    if (a.counters)
-        price_kernel<true><<<grid, kBlock, smem, st>>>(a);
-    else
-        price_kernel<false><<<grid, kBlock, smem, st>>>(a);
-    return cudaGetLastError();
+    return a.counters ? launch_one<true>(a, num_sms, st) : launch_one<false>(a, num_sms, st);
 }
 
 }  // namespace hd
