@@ -61,8 +61,9 @@ enum {
 
 typedef struct heddle_ctx heddle_ctx;
 
-/* Create a context on CUDA device `device`.  Allocates a small amount of
- * device memory (the top-k merge scratch) and queries the SM count.
+/* Create a context on CUDA device `device`.  Allocates its device scratch
+ * once (about 44 MB: the search worklist of 2^20 candidates and the top-k
+ * merge lists) and queries the SM count.
  * *out is NULL on failure. */
 heddle_status heddle_create(heddle_ctx** out, int32_t device);
 
@@ -178,7 +179,12 @@ typedef struct {
 } heddle_results;
 
 /* Price a batch (PartitionLayers + Evaluate, §3.1, §5.2, §5.3).
- * Asynchronous on `stream`; no host round-trip; allocates nothing.
+ * Asynchronous on `stream`; no host round-trip; allocates nothing.  Each
+ * chunk of up to 2^20 candidates takes two launches: a screen (masks, DP
+ * degree, memory) that compacts the candidates needing the threshold search
+ * into a worklist owned by the context, then the search over that worklist.
+ * Calls on one context must therefore not overlap on the GPU (use one
+ * stream per context, or one context per stream).
  * A candidate is INVALID if S = 0, S > 32, S > s_max, S > L, M = 0, a stage
  * byte has bits 5-7 set, names a type >= n_types or a type without GPUs, or
  * (dense models) asks a degree above the largest node of its type (the TP

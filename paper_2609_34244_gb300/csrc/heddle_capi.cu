@@ -34,6 +34,14 @@ struct heddle_ctx {
     uint32_t* d_flags = nullptr;            // [0] table build, [1] device errors
     unsigned long long* d_counters = nullptr;  // [3]
     bool count_next = false;
+    // search worklist scratch (hd::kWorklistCap candidates)
+    int32_t* d_wl_count = nullptr;
+    int32_t* d_wl_idx = nullptr;
+    uint16_t* d_wl_n = nullptr;
+    uint16_t* d_wl_M = nullptr;
+    uint8_t* d_wl_S = nullptr;
+    uint8_t* d_wl_memok = nullptr;
+    uint8_t* d_wl_code = nullptr;
     // top-k merge scratch
     hd::TopkEntry* d_scratch = nullptr;
     int32_t* d_scratch_count = nullptr;
@@ -231,6 +239,14 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     if (e == cudaSuccess)
         e = cudaMalloc(&x->d_scratch, sizeof(hd::TopkEntry) * hd::kMaxTopK * x->scratch_blocks);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch_count, sizeof(int32_t) * x->scratch_blocks);
+    const size_t cap = hd::kWorklistCap;
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_count, sizeof(int32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_idx, sizeof(int32_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_n, sizeof(uint16_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_M, sizeof(uint16_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_S, cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_memok, cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_code, (size_t)HEDDLE_MAX_STAGES * cap);
     if (e != cudaSuccess) {
         heddle_destroy(x);
         return HEDDLE_E_CUDA;
@@ -248,6 +264,13 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_counters);
     cudaFree(x->d_scratch);
     cudaFree(x->d_scratch_count);
+    cudaFree(x->d_wl_count);
+    cudaFree(x->d_wl_idx);
+    cudaFree(x->d_wl_n);
+    cudaFree(x->d_wl_M);
+    cudaFree(x->d_wl_S);
+    cudaFree(x->d_wl_memok);
+    cudaFree(x->d_wl_code);
     for (int b = 0; b < 2; ++b) {
         cudaFree(x->st_S[b]);
         cudaFree(x->st_M[b]);
@@ -352,21 +375,34 @@ heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
     a.lay = x->lay;
     a.img = x->d_img;
     a.moe = x->moe;
-    a.S = c->S;
-    a.M = c->M;
-    a.code = c->code;
-    a.n = c->n;
     a.stride = c->plane_stride;
     a.s_max = c->s_max;
-    a.T = r->T;
-    a.B = r->bottleneck;
-    a.ndp = r->n_dp;
-    a.status = r->status;
-    a.bounds = r->bounds;
+    a.bstride = c->n;
     a.err = x->d_flags + 1;
     a.counters = x->count_next ? x->d_counters : nullptr;
     x->count_next = false;
-    CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream));
+    a.wl_count = x->d_wl_count;
+    a.wl_idx = x->d_wl_idx;
+    a.wl_n = x->d_wl_n;
+    a.wl_M = x->d_wl_M;
+    a.wl_S = x->d_wl_S;
+    a.wl_memok = x->d_wl_memok;
+    a.wl_code = x->d_wl_code;
+    a.wl_cap = hd::kWorklistCap;
+    // chunks of at most the worklist capacity, in stream order
+    for (int64_t lo = 0; lo < c->n; lo += hd::kWorklistCap) {
+        const int64_t nb = c->n - lo < hd::kWorklistCap ? c->n - lo : hd::kWorklistCap;
+        a.S = c->S + lo;
+        a.M = c->M + lo;
+        a.code = c->code + lo;
+        a.n = nb;
+        a.T = r->T + lo;
+        a.B = r->bottleneck + lo;
+        a.ndp = r->n_dp + lo;
+        a.status = r->status + lo;
+        a.bounds = r->bounds ? r->bounds + lo : nullptr;
+        CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream));
+    }
     return ok(x);
 }
 

@@ -39,6 +39,11 @@ struct Layout {
     uint32_t offPow2;   // int32 [8]             largest power of two <= largest node (<= 8)
     uint32_t offGpus;   // int32 [8]             GPUs of the type
     uint32_t offCap;    // int32 [8][4]          sum over nodes of floor(gpus / 2^e) * 2^e
+    uint32_t offWin;    // uint8 [8][4][33]      longest run of layers that fits memory per
+                        //                       (type, degree, in-flight microbatches f)
+    uint32_t offModel;  // int32 [4]             [0] every layer has the same state and
+                        //                       activation bytes; [1] every layer has the
+                        //                       same quantised cost per (type, degree)
     uint32_t bytes;
 };
 
@@ -60,6 +65,8 @@ inline Layout make_layout(int L, int NT) {
     y.offPow2 = o;  o = align16(o + 4u * 8);
     y.offGpus = o;  o = align16(o + 4u * 8);
     y.offCap = o;   o = align16(o + 4u * 8 * 4);
+    y.offWin = o;   o = align16(o + 8u * 4 * 33);
+    y.offModel = o; o = align16(o + 4u * 4);
     y.bytes = o;
     return y;
 }
@@ -94,10 +101,24 @@ struct PriceArgs {
     uint16_t* ndp;
     uint8_t* status;
     uint8_t* bounds;
+    int64_t bstride;  // plane stride of bounds (>= n)
     uint32_t* err;
     unsigned long long* counters;  // non-null selects the counting variant
+    // worklist of the candidates that need the threshold search (device
+    // scratch owned by the context, capacity wl_cap candidates)
+    int32_t* wl_count;
+    int32_t* wl_idx;
+    uint16_t* wl_n;
+    uint16_t* wl_M;
+    uint8_t* wl_S;
+    uint8_t* wl_memok;   // 1: memory feasibility already decided by the screen
+    uint8_t* wl_code;    // [kMaxStages][wl_cap]
+    int32_t wl_cap;
+    int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
 };
+// Prices candidates [0, a.n) with a.n <= a.wl_cap: screen, then search.
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st);
+constexpr int32_t kWorklistCap = 1 << 20;
 
 struct TopkEntry {
     int64_t idx;

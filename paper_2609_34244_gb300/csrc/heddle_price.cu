@@ -2,9 +2,18 @@
 // degree (§5.3 packing), PartitionLayers (min-max split, §3.1 listing, with
 // the memory validation of §5.2) and Evaluate (1F1B iteration time, §5.3).
 //
-// One thread prices one candidate; a persistent grid strides over the batch.
-// Each CTA first copies the cost-table image into shared memory with one
-// bulk TMA copy (cp.async.bulk, completion on an mbarrier).
+// Two launches per batch.  The screen kernel (one thread per candidate,
+// coalesced) decodes and validates every candidate, computes its DP degree
+// and decides memory feasibility from a table of the longest run of layers
+// each (type, degree, in-flight count) can hold: if the runs of the stages
+// sum below L no split fits (OOM); when every layer has the same state and
+// activation bytes, runs summing to at least L (each at least one layer)
+// also guarantee a split that fits, so no memory-only probe is needed.
+// Candidates that still need PartitionLayers are compacted into a worklist;
+// the search kernel (one thread per worklist entry, persistent grid) runs the
+// threshold search on them, so cheap and expensive candidates do not share
+// warps.  Each search CTA first copies the cost-table image into shared
+// memory with one bulk TMA copy (cp.async.bulk, completion on an mbarrier).
 //
 // PartitionLayers is solved exactly by a threshold search on the bottleneck
 // value B.  probe(B) decides whether some split has every stage time <= B
@@ -100,6 +109,7 @@ struct Tabs {
     const int32_t* pow2;
     const int32_t* gpus;
     const int32_t* cap;
+    const uint8_t* win;
     int L, NT;
 };
 
@@ -297,26 +307,134 @@ __device__ __forceinline__ int64_t small_div(int64_t a, int64_t b) {
     return q;
 }
 
+__device__ void bind_tables(Tabs& t, const unsigned char* img, const Layout& y) {
+    t.P = reinterpret_cast<const int64_t*>(img + y.offP);
+    t.SA = reinterpret_cast<const longlong2*>(img + y.offSA);
+    t.PB = reinterpret_cast<const int64_t*>(img + y.offPB);
+    t.p2p = reinterpret_cast<const int64_t*>(img + y.offP2P);
+    t.mem = reinterpret_cast<const int64_t*>(img + y.offMem);
+    t.inter = reinterpret_cast<const int64_t*>(img + y.offInter);
+    t.maxn = reinterpret_cast<const int32_t*>(img + y.offMaxN);
+    t.pow2 = reinterpret_cast<const int32_t*>(img + y.offPow2);
+    t.gpus = reinterpret_cast<const int32_t*>(img + y.offGpus);
+    t.cap = reinterpret_cast<const int32_t*>(img + y.offCap);
+    t.win = img + y.offWin;
+    t.L = y.L;
+    t.NT = y.NT;
+}
+
+__device__ __forceinline__ void write_rejected(const PriceArgs& a, int64_t c, int status, int64_t n) {
+    a.T[c] = -1;
+    a.B[c] = -1;
+    a.ndp[c] = (uint16_t)(status == HEDDLE_CAND_OOM ? n : 0);
+    a.status[c] = (uint8_t)status;
+    if (a.bounds)
+        for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = 0;
+}
+
+constexpr int kScreenBlock = 256;
+
+// Steps 1-2 and the memory screen for every candidate of the batch.
+__global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
+    Tabs t;
+    bind_tables(t, a.img, a.lay);  // global image, L1-resident
+    const int L = t.L;
+    const bool memuni = reinterpret_cast<const int32_t*>(a.img + a.lay.offModel)[0] != 0;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t n_round = (a.n + 31) & ~(int64_t)31;  // whole warps iterate together
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < n_round; c += stride) {
+        const bool live = c < a.n;
+        int S = 0, M = 0, status = HEDDLE_CAND_INVALID;
+        int64_t n = 0;
+        if (live) {
+            S = a.S[c];
+            M = a.M[c];
+            status = HEDDLE_CAND_OK;
+            // DP demand per (type, size class) in 16-bit lanes: class e counts
+            // the GPUs of groups (or blocks) of at least 2^e GPUs, types 0-3 in
+            // lo, 4-7 in hi; memory: sum of the stages' longest fitting runs
+            uint64_t dlo[4] = {0, 0, 0, 0}, dhi[4] = {0, 0, 0, 0};
+            int run_sum = 0, run_min = 255;
+            if (S < 1 || S > kMaxStages || S > a.s_max || S > L || M < 1) {
+                status = HEDDLE_CAND_INVALID;
+            } else {
+                for (int s = 0; s < S; ++s) {
+                    const int b = __ldg(a.code + (int64_t)s * a.stride + c);
+                    const int g = b & 7, j = (b >> 3) & 3;
+                    if ((b >> 5) != 0 || g >= t.NT || t.gpus[g] == 0 || (!a.moe && (1 << j) > t.maxn[g])) {
+                        status = HEDDLE_CAND_INVALID;
+                        break;
+                    }
+                    const int k = 1 << j;
+                    const int unit = k <= t.maxn[g] ? k : t.pow2[g];
+                    const uint64_t add = (uint64_t)k << (16 * (g & 3));
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        if ((1 << e) <= unit) {
+                            if (g < 4)
+                                dlo[e] += add;
+                            else
+                                dhi[e] += add;
+                        }
+                    }
+                    const int w = t.win[(g * 4 + j) * 33 + min(S - s, M)];
+                    run_sum += w;
+                    run_min = min(run_min, w);
+                }
+            }
+            if (status == HEDDLE_CAND_OK) {
+                n = kInf;
+#pragma unroll
+                for (int g = 0; g < kMaxTypes; ++g) {
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const uint64_t v = g < 4 ? dlo[e] : dhi[e];
+                        const int64_t d = (int64_t)((v >> (16 * (g & 3))) & 0xffff);
+                        if (d) n = min(n, small_div(t.cap[g * 4 + e], d));
+                    }
+                }
+                if (n == 0)
+                    status = HEDDLE_CAND_NO_FIT;
+                else if (run_min < 1 || run_sum < L)
+                    status = HEDDLE_CAND_OOM;
+            }
+            if (status != HEDDLE_CAND_OK) write_rejected(a, c, status, n);
+        }
+        // compact the candidates that need the search (one atomic per warp)
+        const bool take = live && status == HEDDLE_CAND_OK;
+        const unsigned mask = __ballot_sync(0xffffffffu, take);
+        if (!mask) continue;
+        const int lane = threadIdx.x & 31;
+        int base = 0;
+        if (lane == 0) base = atomicAdd(a.wl_count, __popc(mask));
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (take) {
+            const int p = base + __popc(mask & ((1u << lane) - 1));
+            if (p < a.wl_cap) {
+                a.wl_idx[p] = (int32_t)c;
+                a.wl_n[p] = (uint16_t)n;
+                a.wl_M[p] = (uint16_t)M;
+                a.wl_S[p] = (uint8_t)S;
+                a.wl_memok[p] = memuni ? 1 : 0;
+                for (int s = 0; s < S; ++s)
+                    a.wl_code[(int64_t)s * a.wl_cap + p] = __ldg(a.code + (int64_t)s * a.stride + c);
+            } else {
+                atomicOr(a.err, kErrInternal);
+            }
+        }
+    }
+}
+
+// Steps 3-4 for every worklist entry.
 template <bool kCount>
-__global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
+__global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     if (!stage_tables(smem, a.img, a.lay.bytes, &bar, a.err)) return;
 
     const Layout& y = a.lay;
     Tabs t;
-    t.P = reinterpret_cast<const int64_t*>(smem + y.offP);
-    t.SA = reinterpret_cast<const longlong2*>(smem + y.offSA);
-    t.PB = reinterpret_cast<const int64_t*>(smem + y.offPB);
-    t.p2p = reinterpret_cast<const int64_t*>(smem + y.offP2P);
-    t.mem = reinterpret_cast<const int64_t*>(smem + y.offMem);
-    t.inter = reinterpret_cast<const int64_t*>(smem + y.offInter);
-    t.maxn = reinterpret_cast<const int32_t*>(smem + y.offMaxN);
-    t.pow2 = reinterpret_cast<const int32_t*>(smem + y.offPow2);
-    t.gpus = reinterpret_cast<const int32_t*>(smem + y.offGpus);
-    t.cap = reinterpret_cast<const int32_t*>(smem + y.offCap);
-    t.L = y.L;
-    t.NT = y.NT;
+    bind_tables(t, smem, y);
     const int L = y.L;
     const int W = (L >> 5) + 1;
 
@@ -333,157 +451,126 @@ __global__ void __launch_bounds__(kBlock) price_kernel(PriceArgs a) {
     unsigned long long probes = 0, priced = 0;
     Final fin;
 
+    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < a.n; c += stride) {
-        const int S = a.S[c];
-        const int M = a.M[c];
-        int status = HEDDLE_CAND_OK;
-        int64_t n = 0;
-        // ---- decode + validate (§5.1 depth / device / TP masks); DP demand
-        // per (type, size class) in 16-bit lanes: class e counts the GPUs of
-        // groups (or blocks) of at least 2^e GPUs, types 0-3 in lo, 4-7 in hi
-        uint64_t dlo[4] = {0, 0, 0, 0}, dhi[4] = {0, 0, 0, 0};
-        if (S < 1 || S > kMaxStages || S > a.s_max || S > L || M < 1) {
-            status = HEDDLE_CAND_INVALID;
-        } else {
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < count; p += stride) {
+        const int64_t c = a.wl_idx[p];
+        const int S = a.wl_S[p];
+        const int M = a.wl_M[p];
+        const int64_t n = a.wl_n[p];
+        const bool memok = a.wl_memok[p] != 0;
+        {
             uint32_t packed = 0;
             for (int s = 0; s < S; ++s) {
-                const int b = a.code[(int64_t)s * a.stride + c];
-                packed |= (uint32_t)b << ((s & 3) * 8);
+                packed |= (uint32_t)a.wl_code[(int64_t)s * a.wl_cap + p] << ((s & 3) * 8);
                 if ((s & 3) == 3 || s == S - 1) {
                     ln.code4[(s >> 2) * kBlock] = packed;
                     packed = 0;
                 }
-                const int g = b & 7, j = (b >> 3) & 3;
-                if ((b >> 5) != 0 || g >= t.NT || t.gpus[g] == 0 || (!a.moe && (1 << j) > t.maxn[g])) {
-                    status = HEDDLE_CAND_INVALID;
-                } else {
-                    const int k = 1 << j;
-                    const int unit = k <= t.maxn[g] ? k : t.pow2[g];
-                    const uint64_t add = (uint64_t)k << (16 * (g & 3));
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        if ((1 << e) <= unit) {
-                            if (g < 4)
-                                dlo[e] += add;
-                            else
-                                dhi[e] += add;
-                        }
-                    }
-                }
             }
         }
-        // ---- DP degree: n = min over (type, size class) of capacity / demand
-        if (status == HEDDLE_CAND_OK) {
-            n = kInf;
-#pragma unroll
-            for (int g = 0; g < kMaxTypes; ++g) {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const uint64_t v = g < 4 ? dlo[e] : dhi[e];
-                    const int64_t d = (int64_t)((v >> (16 * (g & 3))) & 0xffff);
-                    if (d) n = min(n, small_div(t.cap[g * 4 + e], d));
-                }
-            }
-            if (n == 0) status = HEDDLE_CAND_NO_FIT;
+        if (kCount) ++priced;
+        // an upper bound that is feasible whenever memory is: every stage
+        // cost of every interval is at most max_s (P_s[L] + c_s)
+        int64_t hi = 0;
+        float inv = 0.f, cw = 0.f;
+        for (int s = 0; s < S; ++s) {
+            const Stage st = load_stage(t, ln, s, S, M);
+            hi = max(hi, st.P[L] + st.c);
+            const float tot = (float)st.P[L] + 1.0f;
+            inv += 1.0f / tot;
+            cw += (float)st.c / tot;
         }
-        int64_t Bstar = -1, T = -1;
-        uint8_t bnd[kMaxStages + 1];
-        if (status == HEDDLE_CAND_OK) {
-            if (kCount) ++priced;
-            // ---- PartitionLayers: memory-only probe, then the threshold search
+        if (!memok) {
+            // memory-only probe decides OOM and gives a tighter upper bound
             if (kCount) ++probes;
             if (!probe<false>(t, ln, S, M, kInf, sn, nullptr)) {
-                status = HEDDLE_CAND_OOM;
+                write_rejected(a, c, HEDDLE_CAND_OOM, n);
+                continue;
+            }
+            hi = sn.hi;
+        }
+        // ---- PartitionLayers: threshold search from the balanced guess
+        int64_t lo = 0;
+        bool lo_known = false, hi_known = false;
+        int64_t B = (int64_t)((1.0f + cw) / inv);
+        int64_t step = max((int64_t)1, (int64_t)((float)B * (float)S / (2.0f * (float)L)));
+        int it = 0;
+        while (lo < hi) {
+            B = min(max(B, lo), hi - 1);
+            if (kCount) ++probes;
+            if (probe<false>(t, ln, S, M, B, sn, nullptr)) {
+                hi = sn.hi;
+                hi_known = true;
             } else {
-                int64_t hi = sn.hi, lo = 0;
-                bool lo_known = false;
-                // first guess: the balanced bottleneck of a proportional split
-                float inv = 0.f, cw = 0.f;
-                for (int s = 0; s < S; ++s) {
-                    const Stage st = load_stage(t, ln, s, S, M);
-                    const float tot = (float)st.P[L] + 1.0f;
-                    inv += 1.0f / tot;
-                    cw += (float)st.c / tot;
-                }
-                int64_t B = (int64_t)((1.0f + cw) / inv);
-                int64_t step = max((int64_t)1, (int64_t)((float)B * (float)S / (2.0f * (float)L)));
-                int it = 0;
-                while (lo < hi) {
-                    B = min(max(B, lo), hi - 1);
-                    if (kCount) ++probes;
-                    if (probe<false>(t, ln, S, M, B, sn, nullptr)) {
-                        hi = sn.hi;
-                    } else {
-                        lo = sn.lo;
-                        lo_known = true;
-                    }
-                    if (lo >= hi) break;
-                    if (!lo_known) {
-                        B = hi - step;
-                        step *= 2;
-                    } else {
-                        B = lo + (hi - lo) / 2;
-                    }
-                    if (++it > kMaxIters) {
-                        atomicOr(a.err, kErrSearchBound);
-                        break;
-                    }
-                }
-                Bstar = hi;
-                // the sets of the optimum give the canonical split
-                if (kCount) ++probes;
-                if (!probe<true>(t, ln, S, M, Bstar, sn, &fin)) atomicOr(a.err, kErrInternal);
-                bnd[0] = 0;
-                for (int s = 0; s + 1 < S; ++s) {
-                    const int from = max((int)bnd[s] + 1, (int)fin.lo[s + 1]);
-                    int wd = from >> 5;
-                    uint32_t m = fin.w[s + 1][wd] & (0xffffffffu << (from & 31));
-                    while (m == 0 && wd < (fin.hi[s + 1] >> 5)) m = fin.w[s + 1][++wd];
-                    bnd[s + 1] = (uint8_t)(m ? (wd << 5) + __ffs(m) - 1 : 0);
-                }
-                bnd[S] = (uint8_t)L;
-                // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s
-                int64_t tmax = 0, tsum = 0;
-                int sg = -1;
-                u128 bestG = 0, bestD = 1;
-                for (int s = 0; s < S; ++s) {
-                    const Stage st = load_stage(t, ln, s, S, M);
-                    const int64_t ts = st.P[bnd[s + 1]] - st.P[bnd[s]] + st.c;
-                    tmax = max(tmax, ts);
-                    tsum += ts;
-                    if (n > 1) {
-                        // stage with the largest G_s / (k_s bw_s), compared exactly
-                        const int code = stage_code(ln, s);
-                        const int g = code & 7, j = (code >> 3) & 3;
-                        const u128 G = (u128)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
-                        const u128 D = (u128)t.inter[g] << j;
-                        if (sg < 0 || G * bestD > bestG * D) {
-                            sg = s;
-                            bestG = G;
-                            bestD = D;
-                        }
-                    }
-                }
-                if (tmax != Bstar) atomicOr(a.err, kErrInternal);
-                int64_t gmax = 0;
-                if (n > 1) {
-                    // ring all-reduce over n replicas: ceil(2(n-1) G 1e9 / (n k bw))
-                    const u128 num = (u128)2 * (u128)(n - 1) * bestG * 1000000000u;
-                    const u128 den = (u128)n * bestD;
-                    gmax = (int64_t)((num + den - 1) / den);
-                }
-                T = (int64_t)(M - 1) * Bstar + tsum + gmax;
+                lo = sn.lo;
+                lo_known = true;
+            }
+            if (lo >= hi) break;
+            if (!lo_known) {
+                B = hi - step;  // gallop down from a feasible guess
+                step *= 2;
+            } else if (!hi_known) {
+                B = lo + step;  // gallop up from an infeasible guess
+                step *= 2;
+            } else {
+                B = lo + (hi - lo) / 2;
+            }
+            if (++it > kMaxIters) {
+                atomicOr(a.err, kErrSearchBound);
+                break;
             }
         }
-        const bool ok = status == HEDDLE_CAND_OK;
-        a.T[c] = ok ? T : -1;
-        a.B[c] = ok ? Bstar : -1;
-        a.ndp[c] = (uint16_t)((ok || status == HEDDLE_CAND_OOM) ? n : 0);
-        a.status[c] = (uint8_t)status;
+        const int64_t Bstar = hi;
+        // the sets of the optimum give the canonical split
+        if (kCount) ++probes;
+        if (!probe<true>(t, ln, S, M, Bstar, sn, &fin)) atomicOr(a.err, kErrInternal);
+        uint8_t bnd[kMaxStages + 1];
+        bnd[0] = 0;
+        for (int s = 0; s + 1 < S; ++s) {
+            const int from = max((int)bnd[s] + 1, (int)fin.lo[s + 1]);
+            int wd = from >> 5;
+            uint32_t m = fin.w[s + 1][wd] & (0xffffffffu << (from & 31));
+            while (m == 0 && wd < (fin.hi[s + 1] >> 5)) m = fin.w[s + 1][++wd];
+            bnd[s + 1] = (uint8_t)(m ? (wd << 5) + __ffs(m) - 1 : 0);
+        }
+        bnd[S] = (uint8_t)L;
+        // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s
+        int64_t tmax = 0, tsum = 0;
+        int sg = -1;
+        u128 bestG = 0, bestD = 1;
+        for (int s = 0; s < S; ++s) {
+            const Stage st = load_stage(t, ln, s, S, M);
+            const int64_t ts = st.P[bnd[s + 1]] - st.P[bnd[s]] + st.c;
+            tmax = max(tmax, ts);
+            tsum += ts;
+            if (n > 1) {
+                // stage with the largest G_s / (k_s bw_s), compared exactly
+                const int code = stage_code(ln, s);
+                const int g = code & 7, j = (code >> 3) & 3;
+                const u128 G = (u128)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
+                const u128 D = (u128)t.inter[g] << j;
+                if (sg < 0 || G * bestD > bestG * D) {
+                    sg = s;
+                    bestG = G;
+                    bestD = D;
+                }
+            }
+        }
+        if (tmax != Bstar) atomicOr(a.err, kErrInternal);
+        int64_t gmax = 0;
+        if (n > 1) {
+            // ring all-reduce over n replicas: ceil(2(n-1) G 1e9 / (n k bw))
+            const u128 num = (u128)2 * (u128)(n - 1) * bestG * 1000000000u;
+            const u128 den = (u128)n * bestD;
+            gmax = (int64_t)((num + den - 1) / den);
+        }
+        a.T[c] = (int64_t)(M - 1) * Bstar + tsum + gmax;
+        a.B[c] = Bstar;
+        a.ndp[c] = (uint16_t)n;
+        a.status[c] = HEDDLE_CAND_OK;
         if (a.bounds) {
-            for (int s = 0; s <= kMaxStages; ++s)
-                a.bounds[(int64_t)s * a.n + c] = (ok && s <= S) ? bnd[s] : 0;
+            for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = s <= S ? bnd[s] : 0;
         }
     }
     if (kCount) {
@@ -508,18 +595,19 @@ size_t lane_bytes(int L) {
 }
 
 template <bool kCount>
-cudaError_t launch_one(const PriceArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const size_t smem = a.lay.bytes + lane_bytes(a.lay.L);
-    cudaError_t e = cudaFuncSetAttribute(price_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(search_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, price_kernel<kCount>, kBlock, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, search_kernel<kCount>, kBlock, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    // the worklist length is only known on the device: size for the batch
     const int64_t need = (a.n + kBlock - 1) / kBlock;
     const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
-    price_kernel<kCount><<<grid, kBlock, smem, st>>>(a);
+    search_kernel<kCount><<<grid, kBlock, smem, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -527,7 +615,13 @@ cudaError_t launch_one(const PriceArgs& a, int num_sms, cudaStream_t st) {
 
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
-    return a.counters ? launch_one<true>(a, num_sms, st) : launch_one<false>(a, num_sms, st);
+    if (a.n > a.wl_cap) return cudaErrorInvalidValue;
+    cudaError_t e = cudaMemsetAsync(a.wl_count, 0, sizeof(int32_t), st);
+    if (e != cudaSuccess) return e;
+    const int grid = (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * 8);
+    screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    return a.counters ? launch_search<true>(a, num_sms, st) : launch_search<false>(a, num_sms, st);
 }
 
 }  // namespace hd

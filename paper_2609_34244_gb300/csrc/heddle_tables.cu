@@ -137,6 +137,16 @@ __global__ void __launch_bounds__(kThreads) build_tables_kernel(TableArgs a) {
         }
         minq[r] = mn;
     }
+    // equal per-layer cost for every (type, degree) of a present type
+    __shared__ int cost_uniform;
+    if (tid == 0) cost_uniform = 1;
+    __syncthreads();
+    for (int t = tid; t < NT * 4 * L; t += blockDim.x) {
+        const int l = t % L;
+        if (l > 0 && a.q[t] != a.q[t - l]) cost_uniform = 0;
+    }
+    __syncthreads();
+    if (tid == 0) reinterpret_cast<int32_t*>(a.img + y.offModel)[1] = cost_uniform;
 
     // byte prefixes
     if (tid == 0) {
@@ -152,6 +162,46 @@ __global__ void __launch_bounds__(kThreads) build_tables_kernel(TableArgs a) {
             SA[2 * (l + 1) + 1] = ac;
             PB[l + 1] = pb;
         }
+    }
+
+    // longest run of consecutive layers whose state plus f in-flight
+    // activations fit one group of (type g, degree 2^j): a two-pointer scan
+    // per (g, j, f); a candidate whose stages' runs sum below L cannot fit
+    if (tid == 0) {
+        bool uni = true;
+        for (int l = 1; l < L; ++l)
+            uni = uni && a.layers[l].state_bytes == a.layers[0].state_bytes &&
+                  a.layers[l].act_bytes == a.layers[0].act_bytes;
+        reinterpret_cast<int32_t*>(a.img + y.offModel)[0] = uni ? 1 : 0;
+    }
+    uint8_t* win = a.img + y.offWin;
+    for (int t = tid; t < 8 * 4 * 33; t += blockDim.x) {
+        const int f = t % 33;
+        const int j = (t / 33) % 4;
+        const int g = t / (33 * 4);
+        int best = 0;
+        if (g < NT && gpus[g] > 0 && f > 0) {
+            const int64_t capk = mem[g] << j;
+            int e = 0;
+            int64_t st = 0, ac = 0;  // bytes of layers [i, e)
+            for (int i = 0; i < L; ++i) {
+                if (e < i) {
+                    e = i;
+                    st = ac = 0;
+                }
+                while (e < L && (st + a.layers[e].state_bytes) + (int64_t)f * (ac + a.layers[e].act_bytes) <= capk) {
+                    st += a.layers[e].state_bytes;
+                    ac += a.layers[e].act_bytes;
+                    ++e;
+                }
+                best = max(best, e - i);
+                if (e > i) {
+                    st -= a.layers[i].state_bytes;
+                    ac -= a.layers[i].act_bytes;
+                }
+            }
+        }
+        win[t] = (uint8_t)best;
     }
 
     // P2P: forward activation plus backward gradient (2 x boundary bytes)

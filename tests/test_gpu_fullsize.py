@@ -46,3 +46,20 @@ def test_full_size(heddle_lib, oracle_mod, name, n, per_batch_sample):
     tref = orc.price(tsub, bounds=False)
     assert (tref["T"] == got["topk"]["T"]).all()
     assert (tref["n_dp"].astype(np.uint32) * w.cands["M"][ti].astype(np.uint32) == got["topk"]["nM"]).all()
+
+
+def test_one_call_larger_than_the_worklist(heddle_lib, oracle_mod):
+    """A single pricing call of 1.2e6 candidates (more than one 2^20-candidate
+    worklist chunk) with bounds, checked on a sample."""
+    import torch
+    from paper_2609_34244_gb300 import workloads as W
+    h = heddle_lib
+    n = 1_200_000
+    w = W.make_workload("dense32", seed=7, n=n)
+    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, bounds=True)
+    assert got["errors"] == 0
+    rng = np.random.default_rng(9)
+    idx = np.sort(np.concatenate([rng.choice(n, 3000, replace=False), np.arange((1 << 20) - 50, (1 << 20) + 50)]))
+    sub = W.make_cands(w.cands["S"][idx], w.cands["M"][idx], np.ascontiguousarray(w.cands["code"][:, idx]))
+    ref = oracle_mod.Oracle(w.cluster, w.model).price(sub, threads=16)
+    G.assert_same(got, ref, idx=idx, what="dense32 1.2e6")

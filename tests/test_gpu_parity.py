@@ -114,8 +114,9 @@ def test_raw_partitions_on_gpu(h, W, oracle_mod):
 
 
 def test_batching_and_launch_shape_do_not_change_results(h, W, oracle_mod):
-    w = W.make_workload("moe48", seed=3, n=5000)
+    w = W.make_workload("moe48", seed=0, n=5000)
     a = G.price_gpu(h, w.cluster, w.model, w.cands, k=64)
+    assert (a["status"] == 0).sum() > 20  # the search really runs
     b = G.price_gpu(h, w.cluster, w.model, w.cands, k=64, batch=777)
     for key in ("T", "bottleneck", "n_dp", "status", "bounds"):
         assert (a[key] == b[key]).all(), key
