@@ -35,12 +35,18 @@ WORKLOAD = "stress128"
 WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 1024 GPUs of 8 types in "
                  "nodes of 2/4/8, 1e7 candidates streamed as 10 device batches of 1e6, S<=32, "
                  "TP in {1,2,4,8}, M=256, global top-16")
-# Algorithmic integer work of one interval check of PartitionLayers: stage
-# cost P[j]-P[i]+c compared with B (int64 subtract, add, compare) and stage
-# memory (S[j]-S[i]) + f*(A[j]-A[i]) compared with the capacity (two int64
-# subtracts, one multiply by a 32-bit count, one add, one compare): eight
-# int64 operations, 16 32-bit ALU lane operations.
-OPS_PER_CHECK = 16
+# Algorithmic integer work per counted unit of the search, in 32-bit lane
+# operations.  General search, one interval check: stage cost P[j]-P[i]+c
+# against B (int64 subtract, add, compare) and stage memory
+# (S[j]-S[i]) + f*(A[j]-A[i]) against the capacity (two int64 subtracts, one
+# multiply by a 32-bit count, one add, one compare): 8 int64 ops = 16.
+# Equal-layer search, one stage capacity min(m, floor((B-c)/q)): B-c (2),
+# x >= m*q (multiply 2, compare 2), the quotient estimate and its two
+# multiply-compare corrections (10), the running sum (1), the two snapping
+# values c + k*q (multiply-add 4) and c + (k+1)*q (4) with their max / min
+# (4): 29.
+OPS_PER_UNIT = {1: 16, 2: 29}
+SEARCH_NAMES = {1: "general interval search", 2: "equal-layer closed form"}
 SMS, LANES_PER_SM = 152, 128  # 4 SM sub-partitions x 32 lanes issue per clock
 
 
@@ -206,14 +212,16 @@ def main():
                 events[i][1].record(stream)
             h.heddle_topk(ctx, c, r, state, stream)
 
-    # algorithmic work of one step (counting variant, untimed)
-    work = {"checks": 0, "probes": 0, "priced": 0}
-    h.heddle_topk_reset(ctx, state, 16, stream)
-    for c, r in cbatches:
-        h.heddle_count_next(ctx, True)
-        h.heddle_price_candidates(ctx, c, r, stream)
-    for key, v in h.heddle_work_counters(ctx).items():
-        work[key] += v
+    search = h.heddle_get_search(ctx)
+
+    def count_work():
+        """Algorithmic work of one step (counting variant, untimed)."""
+        for c, r in cbatches:
+            h.heddle_count_next(ctx, True)
+            h.heddle_price_candidates(ctx, c, r, stream)
+        return h.heddle_work_counters(ctx)
+
+    work = count_work()
 
     for _ in range(args.warmup):
         step()
@@ -238,6 +246,33 @@ def main():
     local_topk = h.read_topk_state(state)
     merged = shard.merge_topk_across_ranks(group, local_topk, 16)
 
+    # the general interval search on the same workload (secondary figure)
+    general = None
+    if search != h.SEARCH_GENERAL:
+        h.heddle_set_search(ctx, h.SEARCH_GENERAL)
+        gwork = count_work()
+        for _ in range(2):
+            step()
+        gev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(n_batches)] for _ in range(2)]
+        torch.cuda.synchronize()
+        g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        g0.record(stream)
+        for k in range(2):
+            step(gev[k])
+        g1.record(stream)
+        torch.cuda.synchronize()
+        gms = g0.elapsed_time(g1) / 2
+        gprice = sum(a.elapsed_time(b) for row in gev for a, b in row) / 2
+        gtopk = h.read_topk_state(state)
+        general = {"value": n / (gms / 1e3), "ms_per_step": gms, "price_ms_per_step": gprice,
+                   "checks_per_candidate": gwork["checks"] / n,
+                   "probes_per_searched": gwork["probes"] / max(1, gwork["priced"]),
+                   "alu_frac": gwork["checks"] * OPS_PER_UNIT[1] / (gprice / 1e3) / 1e12 /
+                   (SMS * LANES_PER_SM * 2070.0 * 1e6 / 1e12),
+                   "same_topk": gtopk["idx"].tolist() == local_topk["idx"].tolist()}
+        h.heddle_set_search(ctx, h.SEARCH_AUTO)
+
     # end to end through the public host-buffer call (pinned host memory)
     pinned = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
               for k, v in w.cands.items()}
@@ -259,7 +294,7 @@ def main():
         return
     peaks, peak_kind = load_peaks()
     value = n * world * args.steps / (ms_all / 1e3)
-    ops_step = work["checks"] * OPS_PER_CHECK
+    ops_step = work["checks"] * OPS_PER_UNIT[search]
     peak_tops = SMS * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
     achieved_tops = ops_step * args.steps / (price_ms / 1e3) / 1e12
     cpu = None
@@ -279,8 +314,11 @@ def main():
         "per_candidate_ns": 1e6 * ms_all / args.steps / n,
         "roofline": {"bound": "alu", "achieved": achieved_tops, "peak": peak_tops, "unit": "Tops/s",
                      "frac": achieved_tops / peak_tops, "traffic": None,
-                     "kernel": "price_kernel", "ops_per_check": OPS_PER_CHECK,
-                     "checks_per_candidate": work["checks"] / n, "probes_per_priced": work["probes"] / max(1, work["priced"]),
+                     "kernel": "heddle_price_candidates (screen + search)", "search": SEARCH_NAMES[search],
+                     "ops_per_unit": OPS_PER_UNIT[search],
+                     "units_per_candidate": work["checks"] / n,
+                     "probes_per_searched": work["probes"] / max(1, work["priced"]),
+                     "searched_fraction": work["priced"] / n,
                      "price_ms_per_step": price_ms / args.steps,
                      "peak_basis": "%s: %d SMs x %d lanes x %.0f MHz (%s sm_max)" % (
                          "issue slots", SMS, LANES_PER_SM, float(peaks.get("sm_max_mhz", 2070.0)), peak_kind)},
@@ -288,6 +326,7 @@ def main():
         "e2e": {"value": n * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d * world,
                 "d2h_bytes_per_step": h.TOPK_STATE_BYTES * world},
         "device_errors": errors,
+        "general_search": general,
         "topk_head": merged["idx"][:4].tolist() if merged["count"] else [],
         "e2e_topk_matches": e2e_topk["idx"].tolist() == local_topk["idx"].tolist(),
     }

@@ -252,11 +252,27 @@ heddle_status heddle_get_tables(heddle_ctx* ctx, int64_t* q, int64_t* p2p);
  * consistency check failed.  0 in normal operation. */
 heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
 
+/* PartitionLayers search.  AUTO (default) uses the equal-layer closed form
+ * when every layer of the loaded model has the same quantised cost for each
+ * (type, degree) and the same state and activation bytes -- then a stage of
+ * per-layer cost q and memory capacity m holds min(m, floor((B - c) / q))
+ * layers at bound B and a probe costs O(S) -- and the general interval
+ * search otherwise.  GENERAL forces the general search.  Both are exact and
+ * return identical results.  heddle_get_search reports the search the next
+ * pricing call will run (GENERAL or EQUAL_LAYERS); E_STATE if the cost
+ * tables are not built. */
+#define HEDDLE_SEARCH_AUTO 0
+#define HEDDLE_SEARCH_GENERAL 1
+#define HEDDLE_SEARCH_EQUAL_LAYERS 2
+heddle_status heddle_set_search(heddle_ctx* ctx, int32_t mode);
+heddle_status heddle_get_search(heddle_ctx* ctx, int32_t* in_use);
+
 /* Work counters of the next heddle_price_candidates call on ctx, for the
  * roofline report: when enabled, that call runs the counting variant of the
  * pricing kernel and accumulates, in device memory owned by ctx,
- * [0] interval checks evaluated, [1] feasibility probes, [2] candidates
- * priced past validation.  heddle_work_counters(ctx, out) copies them out
+ * [0] interval checks evaluated (general search) or stage capacities
+ * evaluated (equal-layer search), [1] feasibility probes, [2] candidates
+ * that reached the search.  heddle_work_counters(ctx, out) copies them out
  * (synchronous) and resets them. */
 heddle_status heddle_count_next(heddle_ctx* ctx, int32_t enable);
 heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);

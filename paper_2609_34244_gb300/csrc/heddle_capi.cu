@@ -27,6 +27,8 @@ struct heddle_ctx {
     // device tables
     Layout lay{};
     bool tables_ready = false;
+    int32_t model_flags[4] = {0, 0, 0, 0};  // copy of the image's model flags
+    int32_t search_mode = HEDDLE_SEARCH_AUTO;
     unsigned char* d_img = nullptr;
     size_t img_cap = 0;
     int64_t* d_q = nullptr;
@@ -179,6 +181,9 @@ heddle_status build_tables(heddle_ctx* x) {
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     uint32_t flags = 0;
     if (e == cudaSuccess) e = cudaMemcpy(&flags, x->d_flags, sizeof(uint32_t), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(x->model_flags, x->d_img + x->lay.offModel, sizeof(x->model_flags),
+                       cudaMemcpyDeviceToHost);
     cudaFree(d_types);
     cudaFree(d_nodes);
     cudaFree(d_layers);
@@ -202,6 +207,12 @@ heddle_status check_cands(heddle_ctx* x, const heddle_candidates* c, bool device
         return fail(x, HEDDLE_E_ARG, "s_max must be in [1, %d]", HEDDLE_MAX_STAGES);
     (void)device;
     return HEDDLE_OK;
+}
+
+// the equal-layer closed form applies when every layer has the same cost per
+// (type, degree) and the same memory, unless the general search is forced
+bool equal_layer_search(const heddle_ctx* x) {
+    return x->search_mode == HEDDLE_SEARCH_AUTO && x->model_flags[0] && x->model_flags[1];
 }
 
 heddle_status check_ready(heddle_ctx* x) {
@@ -389,6 +400,7 @@ heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
     a.wl_memok = x->d_wl_memok;
     a.wl_code = x->d_wl_code;
     a.wl_cap = hd::kWorklistCap;
+    a.uniform = equal_layer_search(x) ? 1 : 0;
     // chunks of at most the worklist capacity, in stream order
     for (int64_t lo = 0; lo < c->n; lo += hd::kWorklistCap) {
         const int64_t nb = c->n - lo < hd::kWorklistCap ? c->n - lo : hd::kWorklistCap;
@@ -571,6 +583,22 @@ heddle_status heddle_device_errors(heddle_ctx* x, uint32_t* flags) {
     CU(cudaDeviceSynchronize());
     CU(cudaMemcpy(flags, x->d_flags + 1, sizeof(uint32_t), cudaMemcpyDeviceToHost));
     CU(cudaMemset(x->d_flags + 1, 0, sizeof(uint32_t)));
+    return ok(x);
+}
+
+heddle_status heddle_set_search(heddle_ctx* x, int32_t mode) {
+    if (!x) return HEDDLE_E_ARG;
+    if (mode != HEDDLE_SEARCH_AUTO && mode != HEDDLE_SEARCH_GENERAL)
+        return fail(x, HEDDLE_E_ARG, "unknown search mode %d", mode);
+    x->search_mode = mode;
+    return ok(x);
+}
+
+heddle_status heddle_get_search(heddle_ctx* x, int32_t* in_use) {
+    if (!x || !in_use) return x ? fail(x, HEDDLE_E_ARG, "in_use is NULL") : HEDDLE_E_ARG;
+    heddle_status st = check_ready(x);
+    if (st != HEDDLE_OK) return st;
+    *in_use = equal_layer_search(x) ? HEDDLE_SEARCH_EQUAL_LAYERS : HEDDLE_SEARCH_GENERAL;
     return ok(x);
 }
 

@@ -588,6 +588,234 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// Equal-layer search.  When every layer has the same quantised cost q_s on
+// the stage's (type, degree) and the same state and activation bytes, stage
+// s holds at bound B exactly cap_s(B) = min(m_s, floor((B - c_s) / q_s))
+// layers (m_s: the longest run that fits its memory), a split with every
+// stage time <= B exists iff every cap_s >= 1 and sum_s cap_s >= L, and the
+// smallest boundary vector is a_{s+1} = max(a_s + 1, L - sum_{t>s} cap_t).
+// A probe is O(S).  Snapping: a feasible probe keeps the same caps down to
+// max_s (c_s + cap_s q_s); an infeasible one up to the smallest
+// c_s + (cap_s + 1) q_s of a stage that can still grow.
+
+struct EqStage {
+    int64_t q, c;
+    int m;
+};
+
+__device__ __forceinline__ EqStage eq_stage(const Tabs& t, const Lane& ln, int s, int S, int M) {
+    const int code = stage_code(ln, s);
+    const int g = code & 7, j = (code >> 3) & 3;
+    EqStage e;
+    const int64_t* P = t.P + (g * 4 + j) * (t.L + 1);
+    e.q = P[1] - P[0];
+    e.m = t.win[(g * 4 + j) * 33 + min(S - s, M)];
+    e.c = 0;
+    if (s + 1 < S) {
+        const int cn = stage_code(ln, s + 1);
+        const int h = cn & 7, jn = (cn >> 3) & 3;
+        const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
+        e.c = t.p2p[(g * 8 + h) * 2 + same];
+    }
+    return e;
+}
+
+// layers the stage holds at bound B (-1: not even one)
+__device__ __forceinline__ int eq_cap(const EqStage& e, int64_t B) {
+    if (B < e.c + e.q || e.m < 1) return -1;
+    const int64_t x = B - e.c;
+    if (e.q == 0 || x >= (int64_t)e.m * e.q) return e.m;
+    // x < m q with m <= 255: a float estimate is off by at most one
+    int k = (int)((float)x / (float)e.q);
+    if ((int64_t)k * e.q > x) --k;
+    if ((int64_t)(k + 1) * e.q <= x) ++k;
+    return k;
+}
+
+__device__ bool eq_probe(const Tabs& t, const Lane& ln, int S, int M, int64_t B, Snap& sn) {
+    sn.hi = -1;
+    sn.lo = kInf;
+    int sum = 0;
+    bool ok = true;
+    for (int s = 0; s < S; ++s) {
+        const EqStage e = eq_stage(t, ln, s, S, M);
+        ++sn.checks;
+        const int k = eq_cap(e, B);
+        if (k < 1) {
+            ok = false;
+            if (e.m >= 1) sn.lo = min(sn.lo, e.c + e.q);
+            continue;
+        }
+        sum += k;
+        sn.hi = max(sn.hi, e.c + (int64_t)k * e.q);
+        if (k < e.m) sn.lo = min(sn.lo, e.c + (int64_t)(k + 1) * e.q);
+    }
+    return ok && sum >= t.L;
+}
+
+template <bool kCount>
+__global__ void __launch_bounds__(kBlock) eq_search_kernel(PriceArgs a) {
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ uint64_t bar;
+    if (!stage_tables(smem, a.img, a.lay.bytes, &bar, a.err)) return;
+    const Layout& y = a.lay;
+    Tabs t;
+    bind_tables(t, smem, y);
+    const int L = y.L;
+    uint32_t* lane_words = reinterpret_cast<uint32_t*>(smem + y.bytes);
+    Lane ln;
+    ln.code4 = lane_words + threadIdx.x;
+    ln.U = reinterpret_cast<uint8_t*>(lane_words + kCodeWords * kBlock) + threadIdx.x;
+    ln.C[0] = ln.C[1] = nullptr;
+
+    Snap sn;
+    sn.checks = 0;
+    unsigned long long probes = 0, priced = 0;
+    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < count; p += stride) {
+        const int64_t c = a.wl_idx[p];
+        const int S = a.wl_S[p];
+        const int M = a.wl_M[p];
+        const int64_t n = a.wl_n[p];
+        {
+            uint32_t packed = 0;
+            for (int s = 0; s < S; ++s) {
+                packed |= (uint32_t)a.wl_code[(int64_t)s * a.wl_cap + p] << ((s & 3) * 8);
+                if ((s & 3) == 3 || s == S - 1) {
+                    ln.code4[(s >> 2) * kBlock] = packed;
+                    packed = 0;
+                }
+            }
+        }
+        if (kCount) ++priced;
+        // feasible upper bound (every stage at its memory cap; the screen
+        // guarantees the caps cover L) and the continuous balanced guess
+        int64_t hi = 0;
+        float inv = 0.f, cw = 0.f;
+        for (int s = 0; s < S; ++s) {
+            const EqStage e = eq_stage(t, ln, s, S, M);
+            hi = max(hi, e.c + (int64_t)e.m * e.q);
+            const float qf = (float)e.q + 1e-3f;
+            inv += 1.0f / qf;
+            cw += (float)e.c / qf;
+        }
+        int64_t lo = 0;
+        bool lo_known = false, hi_known = false;
+        int64_t B = (int64_t)(((float)L + cw) / inv);
+        int64_t step = max((int64_t)1, B / (2 * (int64_t)L / S + 1));
+        int it = 0;
+        while (lo < hi) {
+            B = min(max(B, lo), hi - 1);
+            if (kCount) ++probes;
+            if (eq_probe(t, ln, S, M, B, sn)) {
+                hi = sn.hi;
+                hi_known = true;
+            } else {
+                lo = sn.lo;
+                lo_known = true;
+            }
+            if (lo >= hi) break;
+            if (!lo_known) {
+                B = hi - step;
+                step *= 2;
+            } else if (!hi_known) {
+                B = lo + step;
+                step *= 2;
+            } else {
+                B = lo + (hi - lo) / 2;
+            }
+            if (++it > kMaxIters) {
+                atomicOr(a.err, kErrSearchBound);
+                break;
+            }
+        }
+        const int64_t Bstar = hi;
+        // caps at B*, then the smallest boundaries
+        int total = 0;
+        for (int s = 0; s < S; ++s) {
+            const int k = eq_cap(eq_stage(t, ln, s, S, M), Bstar);
+            if (k < 1) atomicOr(a.err, kErrInternal);
+            ln.U[s * kBlock] = (uint8_t)max(k, 0);
+            total += k;
+        }
+        uint8_t bnd[kMaxStages + 1];
+        bnd[0] = 0;
+        int pre = 0, at = 0;
+        for (int s = 0; s + 1 < S; ++s) {
+            pre += ln.U[s * kBlock];
+            at = max(at + 1, L - (total - pre));
+            bnd[s + 1] = (uint8_t)at;
+        }
+        bnd[S] = (uint8_t)L;
+        // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s
+        int64_t tmax = 0, tsum = 0;
+        int sg = -1;
+        u128 bestG = 0, bestD = 1;
+        for (int s = 0; s < S; ++s) {
+            const Stage st = load_stage(t, ln, s, S, M);
+            const int64_t ts = st.P[bnd[s + 1]] - st.P[bnd[s]] + st.c;
+            tmax = max(tmax, ts);
+            tsum += ts;
+            if (n > 1) {
+                const int code = stage_code(ln, s);
+                const int g = code & 7, j = (code >> 3) & 3;
+                const u128 G = (u128)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
+                const u128 D = (u128)t.inter[g] << j;
+                if (sg < 0 || G * bestD > bestG * D) {
+                    sg = s;
+                    bestG = G;
+                    bestD = D;
+                }
+            }
+        }
+        if (tmax != Bstar) atomicOr(a.err, kErrInternal);
+        int64_t gmax = 0;
+        if (n > 1) {
+            const u128 num = (u128)2 * (u128)(n - 1) * bestG * 1000000000u;
+            const u128 den = (u128)n * bestD;
+            gmax = (int64_t)((num + den - 1) / den);
+        }
+        a.T[c] = (int64_t)(M - 1) * Bstar + tsum + gmax;
+        a.B[c] = Bstar;
+        a.ndp[c] = (uint16_t)n;
+        a.status[c] = HEDDLE_CAND_OK;
+        if (a.bounds) {
+            for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = s <= S ? bnd[s] : 0;
+        }
+    }
+    if (kCount) {
+        unsigned long long v0 = sn.checks, v1 = probes, v2 = priced;
+        for (int o = 16; o > 0; o >>= 1) {
+            v0 += __shfl_down_sync(0xffffffffu, v0, o);
+            v1 += __shfl_down_sync(0xffffffffu, v1, o);
+            v2 += __shfl_down_sync(0xffffffffu, v2, o);
+        }
+        if ((threadIdx.x & 31) == 0) {
+            atomicAdd(&a.counters[0], v0);
+            atomicAdd(&a.counters[1], v1);
+            atomicAdd(&a.counters[2], v2);
+        }
+    }
+}
+
+template <bool kCount>
+cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
+    const size_t smem = a.lay.bytes + (size_t)kBlock * (4 * kCodeWords + (kMaxStages + 1));
+    cudaError_t e = cudaFuncSetAttribute(eq_search_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, eq_search_kernel<kCount>, kBlock, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const int64_t need = (a.n + kBlock - 1) / kBlock;
+    const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
+    eq_search_kernel<kCount><<<grid, kBlock, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
 // shared memory of the per-thread interleaved arrays
 size_t lane_bytes(int L) {
     const int W = (L >> 5) + 1;
@@ -621,6 +849,8 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const int grid = (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * 8);
     screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (a.uniform)
+        return a.counters ? launch_eq_search<true>(a, num_sms, st) : launch_eq_search<false>(a, num_sms, st);
     return a.counters ? launch_search<true>(a, num_sms, st) : launch_search<false>(a, num_sms, st);
 }
 

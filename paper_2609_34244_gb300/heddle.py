@@ -63,7 +63,8 @@ TOPK_STATE_BYTES = C.sizeof(heddle_topk_state)
 EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_cluster",
            "heddle_load_model", "heddle_price_candidates", "heddle_topk_reset", "heddle_topk",
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
-           "heddle_count_next", "heddle_work_counters"]
+           "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search"]
+SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS = 0, 1, 2
 
 _lib = None
 
@@ -91,6 +92,8 @@ def load_library(path: str = LIB_PATH):
         "heddle_device_errors": (i32, [p, C.POINTER(C.c_uint32)]),
         "heddle_count_next": (i32, [p, i32]),
         "heddle_work_counters": (i32, [p, C.POINTER(C.c_uint64)]),
+        "heddle_set_search": (i32, [p, i32]),
+        "heddle_get_search": (i32, [p, C.POINTER(C.c_int32)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -241,6 +244,16 @@ def heddle_work_counters(ctx):
     out = (C.c_uint64 * 3)()
     _check(ctx, load_library().heddle_work_counters(ctx, out))
     return {"checks": int(out[0]), "probes": int(out[1]), "priced": int(out[2])}
+
+
+def heddle_set_search(ctx, mode: int):
+    _check(ctx, load_library().heddle_set_search(ctx, int(mode)))
+
+
+def heddle_get_search(ctx) -> int:
+    m = C.c_int32(0)
+    _check(ctx, load_library().heddle_get_search(ctx, C.byref(m)))
+    return int(m.value)
 
 
 # ------------------------------------------------------------- marshalling helpers

@@ -8,7 +8,7 @@ import functools
 import numpy as np
 
 
-def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False):
+def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False, search=None):
     """Price on the GPU through the C ABI; returns numpy results, the top-k
     and (optionally) the work counters.  ``batch`` splits the candidates into
     consecutive launches merged into one top-k state."""
@@ -17,6 +17,8 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
     try:
         h.heddle_load_cluster(ctx, w_cluster)
         h.heddle_load_model(ctx, w_model)
+        if search is not None:
+            h.heddle_set_search(ctx, search)
         n = int(cands["S"].shape[0])
         dc = h.cands_to_device(cands)
         res = h.alloc_results(n, bounds=False)
@@ -44,6 +46,7 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
         out["bounds"] = out_bounds
         out["topk"] = h.read_topk_state(state)
         out["errors"] = h.heddle_device_errors(ctx)
+        out["search"] = h.heddle_get_search(ctx)
         if count:
             out["counters"] = h.heddle_work_counters(ctx)
         return out

@@ -15,15 +15,16 @@ FULL = [("dense32", 100_000, None), ("dense80", 1_000_000, 4000), ("moe48", 1_00
         ("stress128", 10_000_000, 300)]
 
 
+@pytest.mark.parametrize("search", [0, 1], ids=["auto", "general"])
 @pytest.mark.parametrize("name,n,per_batch_sample", FULL)
-def test_full_size(heddle_lib, oracle_mod, name, n, per_batch_sample):
+def test_full_size(heddle_lib, oracle_mod, name, n, per_batch_sample, search):
     import torch
     from paper_2609_34244_gb300 import workloads as W
     assert torch.cuda.is_available()
     h = heddle_lib
     w = W.make_workload(name, seed=0, n=n)
     batch = 1_000_000
-    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, bounds=False, batch=batch)
+    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, bounds=False, batch=batch, search=search)
     assert got["errors"] == 0
     orc = oracle_mod.Oracle(w.cluster, w.model)
     rng = np.random.default_rng(123)

@@ -31,14 +31,20 @@ SMALL = [("tiny", None), ("tiny_ext", None), ("dense32", 6007), ("dense80", 1531
          ("moe48", 6011), ("stress128", 613)]
 
 
+# the equal-layer search runs on models whose layers all cost the same
+EQUAL = {"dense32", "dense80", "stress128"}
+
+
 @pytest.mark.parametrize("name,n", SMALL)
 @pytest.mark.parametrize("seed", [0, 1])
-def test_parity_small(h, W, oracle_mod, name, n, seed):
+@pytest.mark.parametrize("search", [0, 1], ids=["auto", "general"])
+def test_parity_small(h, W, oracle_mod, name, n, seed, search):
     w = W.make_workload(name, seed=seed, n=n)
     orc = oracle_mod.Oracle(w.cluster, w.model)
     ref = orc.price(w.cands, threads=8)
-    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16)
+    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, search=search)
     assert got["errors"] == 0
+    assert got["search"] == (2 if (search == 0 and name in EQUAL) else 1)
     G.assert_same(got, ref, what=name)
     tk = oracle_mod.topk(ref, w.cands["M"], 16)
     assert got["topk"]["count"] == tk["count"]
@@ -111,6 +117,35 @@ def test_raw_partitions_on_gpu(h, W, oracle_mod):
         got = G.price_gpu(h, cluster, model, cands)
         assert got["errors"] == 0
         G.assert_same(got, ref, what="trial %d" % trial)
+
+
+def test_equal_layer_random_instances(h, W, oracle_mod):
+    """Random equal-layer models (one layer repeated, so the closed-form
+    search runs), memory often binding, P2P and replication on: GPU in both
+    search modes vs the oracle DP."""
+    rng = np.random.default_rng(17)
+    for trial in range(40):
+        L = int(rng.integers(1, 64))
+        nt = int(rng.integers(1, 5))
+        cluster = W.make_cluster(rng.uniform(50, 1000, nt), rng.integers(1, 12, nt) * 10**9,
+                                 rng.integers(1, 10, nt) * 10**11,
+                                 [(g % nt, int(rng.choice([1, 2, 3, 4, 8])), int(rng.integers(1, 50)) * 10**9)
+                                  for g in range(nt + int(rng.integers(0, 6)))])
+        flops = float(rng.uniform(0, 5e12)) if rng.random() < 0.9 else 0.0
+        model = W.make_model(np.full(L, flops), int(rng.integers(0, 10**9)), int(rng.integers(0, 2 * 10**9)),
+                             int(rng.integers(0, 10**9)), int(rng.integers(0, 10**8)), 0,
+                             int(rng.integers(0, 10**8)), moe=bool(rng.random() < 0.3))
+        n = 700
+        S = rng.integers(1, min(L, 32) + 1, n)
+        code = W.encode(rng.integers(0, nt, (32, n)), rng.integers(0, 4, (32, n)))
+        code[np.arange(32)[:, None] >= S[None, :]] = 0
+        cands = W.make_cands(S, rng.integers(1, 300, n), code)
+        ref = oracle_mod.Oracle(cluster, model).price(cands)
+        for search in (0, 1):
+            got = G.price_gpu(h, cluster, model, cands, search=search)
+            assert got["errors"] == 0
+            assert got["search"] == (2 if search == 0 else 1)
+            G.assert_same(got, ref, what="trial %d search %d" % (trial, search))
 
 
 def test_batching_and_launch_shape_do_not_change_results(h, W, oracle_mod):
