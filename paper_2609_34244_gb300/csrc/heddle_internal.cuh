@@ -118,6 +118,8 @@ struct PriceArgs {
 };
 // Prices candidates [0, a.n) with a.n <= a.wl_cap: screen, then search.
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st);
+// The equal-layer search over the worklist the screen produced.
+cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
 
 struct TopkEntry {

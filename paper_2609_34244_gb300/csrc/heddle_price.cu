@@ -334,12 +334,44 @@ __device__ __forceinline__ void write_rejected(const PriceArgs& a, int64_t c, in
 
 constexpr int kScreenBlock = 256;
 
+// floor(a / d) for 0 <= a < 2^16 and 1 <= d <= 256 as a * ceil(2^32 / d) / 2^32:
+// the error a (ceil(2^32/d) - 2^32/d) / 2^32 < 2^-16 never reaches 1/d, the
+// smallest distance from a / d up to the next integer
+__device__ __forceinline__ uint32_t div_small(uint32_t a, uint32_t d, const uint32_t* magic) {
+    return d == 1 ? a : __umulhi(a, magic[d]);
+}
+
 // Steps 1-2 and the memory screen for every candidate of the batch.
 __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
-    Tabs t;
-    bind_tables(t, a.img, a.lay);  // global image, L1-resident
-    const int L = t.L;
-    const bool memuni = reinterpret_cast<const int32_t*>(a.img + a.lay.offModel)[0] != 0;
+    // stage byte -> 0x10 | unit class when the stage is admissible, else 0
+    __shared__ uint8_t unit_of[32];
+    __shared__ uint8_t win[8 * 4 * 33];
+    __shared__ uint32_t cap[8 * 4];
+    __shared__ uint32_t magic[257];
+    __shared__ uint64_t dem[8 * kScreenBlock];  // per-thread GPUs per unit class, 4 x 16 bits per type
+    const Layout& y = a.lay;
+    const int L = y.L;
+    {
+        const int32_t* gmaxn = reinterpret_cast<const int32_t*>(a.img + y.offMaxN);
+        const int32_t* gpow2 = reinterpret_cast<const int32_t*>(a.img + y.offPow2);
+        const int32_t* ggpus = reinterpret_cast<const int32_t*>(a.img + y.offGpus);
+        const int32_t* gcap = reinterpret_cast<const int32_t*>(a.img + y.offCap);
+        for (int i = threadIdx.x; i < 32; i += blockDim.x) {
+            const int g = i & 7, j = i >> 3;
+            uint8_t u = 0;
+            if (g < y.NT && ggpus[g] > 0 && (a.moe || (1 << j) <= gmaxn[g])) {
+                const int unit = (1 << j) <= gmaxn[g] ? (1 << j) : gpow2[g];
+                u = (uint8_t)(0x10 | (31 - __clz(unit)));
+            }
+            unit_of[i] = u;
+            cap[i] = (uint32_t)gcap[i];
+        }
+        for (int i = threadIdx.x; i < 8 * 4 * 33; i += blockDim.x) win[i] = a.img[y.offWin + i];
+        for (int i = threadIdx.x; i < 257; i += blockDim.x) magic[i] = i >= 2 ? 0xffffffffu / i + 1 : 0;
+    }
+    __syncthreads();
+    const bool memuni = reinterpret_cast<const int32_t*>(a.img + y.offModel)[0] != 0;
+    uint64_t* mydem = dem + threadIdx.x;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t n_round = (a.n + 31) & ~(int64_t)31;  // whole warps iterate together
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < n_round; c += stride) {
@@ -349,54 +381,47 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
         if (live) {
             S = a.S[c];
             M = a.M[c];
-            status = HEDDLE_CAND_OK;
-            // DP demand per (type, size class) in 16-bit lanes: class e counts
-            // the GPUs of groups (or blocks) of at least 2^e GPUs, types 0-3 in
-            // lo, 4-7 in hi; memory: sum of the stages' longest fitting runs
-            uint64_t dlo[4] = {0, 0, 0, 0}, dhi[4] = {0, 0, 0, 0};
-            int run_sum = 0, run_min = 255;
-            if (S < 1 || S > kMaxStages || S > a.s_max || S > L || M < 1) {
-                status = HEDDLE_CAND_INVALID;
-            } else {
+            if (S >= 1 && S <= kMaxStages && S <= a.s_max && S <= L && M >= 1) {
+#pragma unroll
+                for (int g = 0; g < 8; ++g) mydem[g * kScreenBlock] = 0;
+                uint32_t bad = 0, present = 0;
+                int run_sum = 0, run_min = 255;
                 for (int s = 0; s < S; ++s) {
                     const int b = __ldg(a.code + (int64_t)s * a.stride + c);
+                    const int u = unit_of[b & 31];
+                    bad |= (uint32_t)(b >> 5) | (uint32_t)(u == 0);
                     const int g = b & 7, j = (b >> 3) & 3;
-                    if ((b >> 5) != 0 || g >= t.NT || t.gpus[g] == 0 || (!a.moe && (1 << j) > t.maxn[g])) {
-                        status = HEDDLE_CAND_INVALID;
-                        break;
-                    }
-                    const int k = 1 << j;
-                    const int unit = k <= t.maxn[g] ? k : t.pow2[g];
-                    const uint64_t add = (uint64_t)k << (16 * (g & 3));
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        if ((1 << e) <= unit) {
-                            if (g < 4)
-                                dlo[e] += add;
-                            else
-                                dhi[e] += add;
-                        }
-                    }
-                    const int w = t.win[(g * 4 + j) * 33 + min(S - s, M)];
+                    present |= 1u << g;
+                    // k GPUs in units of 2^(u & 3)
+                    mydem[g * kScreenBlock] += (uint64_t)(1u << j) << (16 * (u & 3));
+                    const int w = win[(g * 4 + j) * 33 + min(S - s, M)];
                     run_sum += w;
                     run_min = min(run_min, w);
                 }
-            }
-            if (status == HEDDLE_CAND_OK) {
-                n = kInf;
+                if (bad) {
+                    status = HEDDLE_CAND_INVALID;
+                } else {
+                    // n = min over (type, class e) of capacity / GPUs in units >= 2^e
+                    uint32_t nn = 0xffffffffu;
+                    while (present) {
+                        const int g = __ffs(present) - 1;
+                        present &= present - 1;
+                        const uint64_t v = mydem[g * kScreenBlock];
+                        uint32_t d = 0;
 #pragma unroll
-                for (int g = 0; g < kMaxTypes; ++g) {
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const uint64_t v = g < 4 ? dlo[e] : dhi[e];
-                        const int64_t d = (int64_t)((v >> (16 * (g & 3))) & 0xffff);
-                        if (d) n = min(n, small_div(t.cap[g * 4 + e], d));
+                        for (int e = 3; e >= 0; --e) {
+                            d += (uint32_t)(v >> (16 * e)) & 0xffffu;
+                            if (d) nn = min(nn, div_small(cap[g * 4 + e], d, magic));
+                        }
                     }
+                    n = nn;
+                    if (n == 0)
+                        status = HEDDLE_CAND_NO_FIT;
+                    else if (run_min < 1 || run_sum < L)
+                        status = HEDDLE_CAND_OOM;
+                    else
+                        status = HEDDLE_CAND_OK;
                 }
-                if (n == 0)
-                    status = HEDDLE_CAND_NO_FIT;
-                else if (run_min < 1 || run_sum < L)
-                    status = HEDDLE_CAND_OOM;
             }
             if (status != HEDDLE_CAND_OK) write_rejected(a, c, status, n);
         }
@@ -588,234 +613,6 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
     }
 }
 
-// ---------------------------------------------------------------------------
-// Equal-layer search.  When every layer has the same quantised cost q_s on
-// the stage's (type, degree) and the same state and activation bytes, stage
-// s holds at bound B exactly cap_s(B) = min(m_s, floor((B - c_s) / q_s))
-// layers (m_s: the longest run that fits its memory), a split with every
-// stage time <= B exists iff every cap_s >= 1 and sum_s cap_s >= L, and the
-// smallest boundary vector is a_{s+1} = max(a_s + 1, L - sum_{t>s} cap_t).
-// A probe is O(S).  Snapping: a feasible probe keeps the same caps down to
-// max_s (c_s + cap_s q_s); an infeasible one up to the smallest
-// c_s + (cap_s + 1) q_s of a stage that can still grow.
-
-struct EqStage {
-    int64_t q, c;
-    int m;
-};
-
-__device__ __forceinline__ EqStage eq_stage(const Tabs& t, const Lane& ln, int s, int S, int M) {
-    const int code = stage_code(ln, s);
-    const int g = code & 7, j = (code >> 3) & 3;
-    EqStage e;
-    const int64_t* P = t.P + (g * 4 + j) * (t.L + 1);
-    e.q = P[1] - P[0];
-    e.m = t.win[(g * 4 + j) * 33 + min(S - s, M)];
-    e.c = 0;
-    if (s + 1 < S) {
-        const int cn = stage_code(ln, s + 1);
-        const int h = cn & 7, jn = (cn >> 3) & 3;
-        const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
-        e.c = t.p2p[(g * 8 + h) * 2 + same];
-    }
-    return e;
-}
-
-// layers the stage holds at bound B (-1: not even one)
-__device__ __forceinline__ int eq_cap(const EqStage& e, int64_t B) {
-    if (B < e.c + e.q || e.m < 1) return -1;
-    const int64_t x = B - e.c;
-    if (e.q == 0 || x >= (int64_t)e.m * e.q) return e.m;
-    // x < m q with m <= 255: a float estimate is off by at most one
-    int k = (int)((float)x / (float)e.q);
-    if ((int64_t)k * e.q > x) --k;
-    if ((int64_t)(k + 1) * e.q <= x) ++k;
-    return k;
-}
-
-__device__ bool eq_probe(const Tabs& t, const Lane& ln, int S, int M, int64_t B, Snap& sn) {
-    sn.hi = -1;
-    sn.lo = kInf;
-    int sum = 0;
-    bool ok = true;
-    for (int s = 0; s < S; ++s) {
-        const EqStage e = eq_stage(t, ln, s, S, M);
-        ++sn.checks;
-        const int k = eq_cap(e, B);
-        if (k < 1) {
-            ok = false;
-            if (e.m >= 1) sn.lo = min(sn.lo, e.c + e.q);
-            continue;
-        }
-        sum += k;
-        sn.hi = max(sn.hi, e.c + (int64_t)k * e.q);
-        if (k < e.m) sn.lo = min(sn.lo, e.c + (int64_t)(k + 1) * e.q);
-    }
-    return ok && sum >= t.L;
-}
-
-template <bool kCount>
-__global__ void __launch_bounds__(kBlock) eq_search_kernel(PriceArgs a) {
-    extern __shared__ __align__(128) unsigned char smem[];
-    __shared__ uint64_t bar;
-    if (!stage_tables(smem, a.img, a.lay.bytes, &bar, a.err)) return;
-    const Layout& y = a.lay;
-    Tabs t;
-    bind_tables(t, smem, y);
-    const int L = y.L;
-    uint32_t* lane_words = reinterpret_cast<uint32_t*>(smem + y.bytes);
-    Lane ln;
-    ln.code4 = lane_words + threadIdx.x;
-    ln.U = reinterpret_cast<uint8_t*>(lane_words + kCodeWords * kBlock) + threadIdx.x;
-    ln.C[0] = ln.C[1] = nullptr;
-
-    Snap sn;
-    sn.checks = 0;
-    unsigned long long probes = 0, priced = 0;
-    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < count; p += stride) {
-        const int64_t c = a.wl_idx[p];
-        const int S = a.wl_S[p];
-        const int M = a.wl_M[p];
-        const int64_t n = a.wl_n[p];
-        {
-            uint32_t packed = 0;
-            for (int s = 0; s < S; ++s) {
-                packed |= (uint32_t)a.wl_code[(int64_t)s * a.wl_cap + p] << ((s & 3) * 8);
-                if ((s & 3) == 3 || s == S - 1) {
-                    ln.code4[(s >> 2) * kBlock] = packed;
-                    packed = 0;
-                }
-            }
-        }
-        if (kCount) ++priced;
-        // feasible upper bound (every stage at its memory cap; the screen
-        // guarantees the caps cover L) and the continuous balanced guess
-        int64_t hi = 0;
-        float inv = 0.f, cw = 0.f;
-        for (int s = 0; s < S; ++s) {
-            const EqStage e = eq_stage(t, ln, s, S, M);
-            hi = max(hi, e.c + (int64_t)e.m * e.q);
-            const float qf = (float)e.q + 1e-3f;
-            inv += 1.0f / qf;
-            cw += (float)e.c / qf;
-        }
-        int64_t lo = 0;
-        bool lo_known = false, hi_known = false;
-        int64_t B = (int64_t)(((float)L + cw) / inv);
-        int64_t step = max((int64_t)1, B / (2 * (int64_t)L / S + 1));
-        int it = 0;
-        while (lo < hi) {
-            B = min(max(B, lo), hi - 1);
-            if (kCount) ++probes;
-            if (eq_probe(t, ln, S, M, B, sn)) {
-                hi = sn.hi;
-                hi_known = true;
-            } else {
-                lo = sn.lo;
-                lo_known = true;
-            }
-            if (lo >= hi) break;
-            if (!lo_known) {
-                B = hi - step;
-                step *= 2;
-            } else if (!hi_known) {
-                B = lo + step;
-                step *= 2;
-            } else {
-                B = lo + (hi - lo) / 2;
-            }
-            if (++it > kMaxIters) {
-                atomicOr(a.err, kErrSearchBound);
-                break;
-            }
-        }
-        const int64_t Bstar = hi;
-        // caps at B*, then the smallest boundaries
-        int total = 0;
-        for (int s = 0; s < S; ++s) {
-            const int k = eq_cap(eq_stage(t, ln, s, S, M), Bstar);
-            if (k < 1) atomicOr(a.err, kErrInternal);
-            ln.U[s * kBlock] = (uint8_t)max(k, 0);
-            total += k;
-        }
-        uint8_t bnd[kMaxStages + 1];
-        bnd[0] = 0;
-        int pre = 0, at = 0;
-        for (int s = 0; s + 1 < S; ++s) {
-            pre += ln.U[s * kBlock];
-            at = max(at + 1, L - (total - pre));
-            bnd[s + 1] = (uint8_t)at;
-        }
-        bnd[S] = (uint8_t)L;
-        // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s
-        int64_t tmax = 0, tsum = 0;
-        int sg = -1;
-        u128 bestG = 0, bestD = 1;
-        for (int s = 0; s < S; ++s) {
-            const Stage st = load_stage(t, ln, s, S, M);
-            const int64_t ts = st.P[bnd[s + 1]] - st.P[bnd[s]] + st.c;
-            tmax = max(tmax, ts);
-            tsum += ts;
-            if (n > 1) {
-                const int code = stage_code(ln, s);
-                const int g = code & 7, j = (code >> 3) & 3;
-                const u128 G = (u128)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
-                const u128 D = (u128)t.inter[g] << j;
-                if (sg < 0 || G * bestD > bestG * D) {
-                    sg = s;
-                    bestG = G;
-                    bestD = D;
-                }
-            }
-        }
-        if (tmax != Bstar) atomicOr(a.err, kErrInternal);
-        int64_t gmax = 0;
-        if (n > 1) {
-            const u128 num = (u128)2 * (u128)(n - 1) * bestG * 1000000000u;
-            const u128 den = (u128)n * bestD;
-            gmax = (int64_t)((num + den - 1) / den);
-        }
-        a.T[c] = (int64_t)(M - 1) * Bstar + tsum + gmax;
-        a.B[c] = Bstar;
-        a.ndp[c] = (uint16_t)n;
-        a.status[c] = HEDDLE_CAND_OK;
-        if (a.bounds) {
-            for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = s <= S ? bnd[s] : 0;
-        }
-    }
-    if (kCount) {
-        unsigned long long v0 = sn.checks, v1 = probes, v2 = priced;
-        for (int o = 16; o > 0; o >>= 1) {
-            v0 += __shfl_down_sync(0xffffffffu, v0, o);
-            v1 += __shfl_down_sync(0xffffffffu, v1, o);
-            v2 += __shfl_down_sync(0xffffffffu, v2, o);
-        }
-        if ((threadIdx.x & 31) == 0) {
-            atomicAdd(&a.counters[0], v0);
-            atomicAdd(&a.counters[1], v1);
-            atomicAdd(&a.counters[2], v2);
-        }
-    }
-}
-
-template <bool kCount>
-cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
-    const size_t smem = a.lay.bytes + (size_t)kBlock * (4 * kCodeWords + (kMaxStages + 1));
-    cudaError_t e = cudaFuncSetAttribute(eq_search_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
-    int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, eq_search_kernel<kCount>, kBlock, smem);
-    if (e != cudaSuccess) return e;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    const int64_t need = (a.n + kBlock - 1) / kBlock;
-    const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
-    eq_search_kernel<kCount><<<grid, kBlock, smem, st>>>(a);
-    return cudaGetLastError();
-}
-
 // shared memory of the per-thread interleaved arrays
 size_t lane_bytes(int L) {
     const int W = (L >> 5) + 1;
@@ -849,8 +646,7 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const int grid = (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * 8);
     screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if (a.uniform)
-        return a.counters ? launch_eq_search<true>(a, num_sms, st) : launch_eq_search<false>(a, num_sms, st);
+    if (a.uniform) return launch_eq_search(a, num_sms, st);
     return a.counters ? launch_search<true>(a, num_sms, st) : launch_search<false>(a, num_sms, st);
 }
 
