@@ -203,14 +203,16 @@ def main():
     n_batches = len(cbatches)
 
     def step(events=None):
+        """One pass of the hot path: every batch priced and merged into the
+        running top-16 (heddle_price_topk: screen, search with the fused
+        block-level top-k, merge)."""
         h.heddle_topk_reset(ctx, state, 16, stream)
         for i, (c, r) in enumerate(cbatches):
             if events is not None:
                 events[i][0].record(stream)
-            h.heddle_price_candidates(ctx, c, r, stream)
+            h.heddle_price_topk(ctx, c, r, state, stream)
             if events is not None:
                 events[i][1].record(stream)
-            h.heddle_topk(ctx, c, r, state, stream)
 
     search = h.heddle_get_search(ctx)
 
@@ -310,11 +312,13 @@ def main():
                    "parallelism": "candidate shards, dp%d" % world,
                    "l2": "inputs larger than L2 (%.0f MB of candidates per step per GPU)" % (h2d / 1e6),
                    "seed": "rank"},
+        # per step: the top-k reset kernel, then per batch the screen, the
+        # search and the merge (the two cudaMemsetAsync calls are not kernels)
         "gpu_launches": args.steps * (1 + 3 * n_batches) * world,
         "per_candidate_ns": 1e6 * ms_all / args.steps / n,
         "roofline": {"bound": "alu", "achieved": achieved_tops, "peak": peak_tops, "unit": "Tops/s",
                      "frac": achieved_tops / peak_tops, "traffic": None,
-                     "kernel": "heddle_price_candidates (screen + search)", "search": SEARCH_NAMES[search],
+                     "kernel": "heddle_price_topk (screen + search + merge)", "search": SEARCH_NAMES[search],
                      "ops_per_unit": OPS_PER_UNIT[search],
                      "units_per_candidate": work["checks"] / n,
                      "probes_per_searched": work["probes"] / max(1, work["priced"]),

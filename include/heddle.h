@@ -223,6 +223,16 @@ heddle_status heddle_topk(heddle_ctx* ctx, const heddle_candidates* cands,
                           const heddle_results* results, heddle_topk_state* state,
                           void* stream);
 
+/* Price a batch and merge its OK candidates into *state (device): after each
+ * chunk's search, the block-level top-k runs over that chunk's worklist of
+ * searched candidates only (the screen already rejected the rest), then the
+ * per-CTA lists are merged into the state -- no pass over the full results.
+ * Same results and the same state as heddle_price_candidates followed by
+ * heddle_topk.  Errors as for both. */
+heddle_status heddle_price_topk(heddle_ctx* ctx, const heddle_candidates* cands,
+                                const heddle_results* results, heddle_topk_state* state,
+                                void* stream);
+
 /* -------------------------------------------------------- host buffers */
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the

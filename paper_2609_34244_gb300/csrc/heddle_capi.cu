@@ -44,10 +44,14 @@ struct heddle_ctx {
     uint8_t* d_wl_S = nullptr;
     uint8_t* d_wl_memok = nullptr;
     uint8_t* d_wl_code = nullptr;
+    int64_t* d_wl_T = nullptr;
+    uint32_t* d_wl_nM = nullptr;
     // top-k merge scratch
     hd::TopkEntry* d_scratch = nullptr;
     int32_t* d_scratch_count = nullptr;
     int scratch_blocks = 0;
+    hd::TopkEntry* d_scratch2 = nullptr;
+    int32_t* d_scratch2_count = nullptr;
     // host-buffer path
     cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
     cudaEvent_t ev_loaded[2] = {nullptr, nullptr}, ev_priced[2] = {nullptr, nullptr},
@@ -242,7 +246,7 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
         return HEDDLE_E_CUDA;
     }
     x->num_sms = prop.multiProcessorCount;
-    x->scratch_blocks = 2 * x->num_sms;
+    x->scratch_blocks = 8 * x->num_sms;  // per-CTA lists of the top-k and of the fused search
     cudaError_t e = cudaMalloc(&x->d_flags, 2 * sizeof(uint32_t));
     if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, 2 * sizeof(uint32_t));
     if (e == cudaSuccess) e = cudaMalloc(&x->d_counters, 3 * sizeof(unsigned long long));
@@ -258,6 +262,11 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_S, cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_memok, cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_code, (size_t)HEDDLE_MAX_STAGES * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_T, sizeof(int64_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_nM, sizeof(uint32_t) * cap);
+    const int l2 = (x->scratch_blocks + 31) / 32;
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2, sizeof(hd::TopkEntry) * hd::kMaxTopK * l2);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2_count, sizeof(int32_t) * l2);
     if (e != cudaSuccess) {
         heddle_destroy(x);
         return HEDDLE_E_CUDA;
@@ -282,6 +291,10 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_wl_S);
     cudaFree(x->d_wl_memok);
     cudaFree(x->d_wl_code);
+    cudaFree(x->d_wl_T);
+    cudaFree(x->d_wl_nM);
+    cudaFree(x->d_scratch2);
+    cudaFree(x->d_scratch2_count);
     for (int b = 0; b < 2; ++b) {
         cudaFree(x->st_S[b]);
         cudaFree(x->st_M[b]);
@@ -371,9 +384,25 @@ heddle_status heddle_load_model(heddle_ctx* x, const heddle_layer* layers, int32
     return build_tables(x);
 }
 
-heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
-                                      const heddle_results* r, void* stream) {
-    if (!x) return HEDDLE_E_ARG;
+}  // extern "C"
+
+namespace {
+
+hd::TopkArgs topk_args(heddle_ctx* x, heddle_topk_state* state) {
+    hd::TopkArgs a{};
+    a.state = state;
+    a.scratch = x->d_scratch;
+    a.scratch_count = x->d_scratch_count;
+    a.max_blocks = x->scratch_blocks;
+    a.scratch2 = x->d_scratch2;
+    a.scratch2_count = x->d_scratch2_count;
+    return a;
+}
+
+// Price cands into r; with a state, run the top-k over each chunk's searched
+// candidates (the only ones that can be OK) and merge them into *state.
+heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
+                         heddle_topk_state* state, void* stream) {
     heddle_status st = check_cands(x, c, true);
     if (st != HEDDLE_OK) return st;
     if (!r) return fail(x, HEDDLE_E_ARG, "results is NULL");
@@ -401,6 +430,8 @@ heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
     a.wl_code = x->d_wl_code;
     a.wl_cap = hd::kWorklistCap;
     a.uniform = equal_layer_search(x) ? 1 : 0;
+    a.wl_T = x->d_wl_T;
+    a.wl_nM = x->d_wl_nM;
     // chunks of at most the worklist capacity, in stream order
     for (int64_t lo = 0; lo < c->n; lo += hd::kWorklistCap) {
         const int64_t nb = c->n - lo < hd::kWorklistCap ? c->n - lo : hd::kWorklistCap;
@@ -414,8 +445,36 @@ heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
         a.status = r->status + lo;
         a.bounds = r->bounds ? r->bounds + lo : nullptr;
         CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream));
+        if (state) {
+            // top-k over the searched candidates of this chunk only
+            hd::TopkArgs m = topk_args(x, state);
+            m.base_index = c->base_index + lo;
+            m.wl_count = x->d_wl_count;
+            m.wl_idx = x->d_wl_idx;
+            m.wl_T = x->d_wl_T;
+            m.wl_nM = x->d_wl_nM;
+            m.wl_cap = hd::kWorklistCap;
+            CU(hd::launch_topk_worklist(m, nb, x->num_sms, (cudaStream_t)stream));
+        }
     }
     return ok(x);
+}
+
+}  // namespace
+
+extern "C" {
+
+heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
+                                      const heddle_results* r, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    return price_impl(x, c, r, nullptr, stream);
+}
+
+heddle_status heddle_price_topk(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
+                                heddle_topk_state* state, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!state) return fail(x, HEDDLE_E_ARG, "state is NULL");
+    return price_impl(x, c, r, state, stream);
 }
 
 heddle_status heddle_topk_reset(heddle_ctx* x, heddle_topk_state* state, int32_t k, void* stream) {
@@ -436,17 +495,13 @@ heddle_status heddle_topk(heddle_ctx* x, const heddle_candidates* c, const heddl
     if (c->n == 0) return ok(x);
     if (!r->T || !r->n_dp || !r->status) return fail(x, HEDDLE_E_ARG, "null result array");
     DeviceGuard dg(x->device);
-    hd::TopkArgs a{};
+    hd::TopkArgs a = topk_args(x, state);
     a.M = c->M;
     a.T = r->T;
     a.ndp = r->n_dp;
     a.status = r->status;
     a.n = c->n;
     a.base_index = c->base_index;
-    a.state = state;
-    a.scratch = x->d_scratch;
-    a.scratch_count = x->d_scratch_count;
-    a.max_blocks = x->scratch_blocks;
     CU(hd::launch_topk(a, x->num_sms, (cudaStream_t)stream));
     return ok(x);
 }
@@ -542,8 +597,7 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         rb.n_dp = x->st_n[b];
         rb.status = x->st_status[b];
         rb.bounds = want_bounds ? x->st_bounds[b] : nullptr;
-        if ((st = heddle_price_candidates(x, &cb, &rb, sc)) != HEDDLE_OK) return st;
-        if ((st = heddle_topk(x, &cb, &rb, x->d_state, sc)) != HEDDLE_OK) return st;
+        if ((st = price_impl(x, &cb, &rb, x->d_state, sc)) != HEDDLE_OK) return st;
         CU(cudaEventRecord(x->ev_priced[b], sc));
         // device -> host of the requested result fields on the second copy stream
         CU(cudaStreamWaitEvent(x->s_d2h, x->ev_priced[b], 0));

@@ -282,6 +282,8 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             gmax = (int64_t)((num + den - 1) / den);
         }
         a.T[c] = (int64_t)(M - 1) * Bstar + tsum + gmax;
+        a.wl_T[p] = a.T[c];
+        a.wl_nM[p] = (uint32_t)n * (uint32_t)M;
         a.B[c] = Bstar;
         a.ndp[c] = (uint16_t)n;
         a.status[c] = HEDDLE_CAND_OK;

@@ -71,6 +71,13 @@ inline Layout make_layout(int L, int NT) {
     return y;
 }
 
+struct TopkEntry {
+    int64_t idx;
+    int64_t T;
+    uint32_t nM;
+    uint32_t pad;
+};
+
 struct TableArgs {
     Layout lay;
     const heddle_gpu_type* types;
@@ -115,6 +122,10 @@ struct PriceArgs {
     uint8_t* wl_code;    // [kMaxStages][wl_cap]
     int32_t wl_cap;
     int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
+    // per worklist entry, written by the search: T (-1 unless OK) and n * M,
+    // so a top-k can run over the searched candidates only
+    int64_t* wl_T;
+    uint32_t* wl_nM;
 };
 // Prices candidates [0, a.n) with a.n <= a.wl_cap: screen, then search.
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st);
@@ -122,14 +133,9 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
 
-struct TopkEntry {
-    int64_t idx;
-    int64_t T;
-    uint32_t nM;
-    uint32_t pad;
-};
 
 struct TopkArgs {
+    // results of a batch (heddle_topk) ...
     const uint16_t* M;
     const int64_t* T;
     const uint16_t* ndp;
@@ -140,8 +146,20 @@ struct TopkArgs {
     TopkEntry* scratch;        // [grid][kMaxTopK]
     int32_t* scratch_count;    // [grid]
     int32_t max_blocks;
+    // ... or the worklist of a priced chunk (heddle_price_topk)
+    const int32_t* wl_count;
+    const int32_t* wl_idx;
+    const int64_t* wl_T;
+    const uint32_t* wl_nM;
+    int32_t wl_cap;
+    // second-level lists of the two-level merge
+    TopkEntry* scratch2;
+    int32_t* scratch2_count;
 };
 cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st);
+// Top-k of the searched candidates of a priced chunk (a.wl_*), merged into
+// *a.state; `n` bounds the worklist length (the chunk size).
+cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st);
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st);
 
 }  // namespace hd

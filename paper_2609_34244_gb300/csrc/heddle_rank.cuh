@@ -1,0 +1,92 @@
+// heddle_rank.cuh -- the rank order of priced plans and warp-level top-k
+// lists, shared by the top-k kernels and the search kernels that fuse the
+// block-level top-k.
+//
+// Plans are ranked by predicted throughput (§5 overview); with n replicas of
+// M microbatches per iteration time T a plan processes n*M microbatches per
+// T, so a ranks before b iff nM_a * T_b > nM_b * T_a (exact, 128-bit), and
+// equal throughput goes to the smaller global index.  The order is strict, so
+// the top-k is unique and does not depend on the launch shape.
+#pragma once
+
+#include "heddle_internal.cuh"
+
+namespace hd {
+
+typedef unsigned __int128 u128;
+
+__device__ __forceinline__ bool better(const TopkEntry& a, const TopkEntry& b) {
+    const u128 l = (u128)a.nM * (u128)(uint64_t)b.T;
+    const u128 r = (u128)b.nM * (u128)(uint64_t)a.T;
+    if (l != r) return l > r;
+    return a.idx < b.idx;
+}
+
+// Warp-cooperative insertion into a sorted list of `cnt` entries (capacity
+// k <= 64; lane l owns slots l and l + 32).  All lanes pass the same e.
+__device__ inline void warp_insert(TopkEntry* list, int& cnt, int k, const TopkEntry& e) {
+    const int lane = threadIdx.x & 31;
+    const int p0 = lane, p1 = lane + 32;
+    const bool b0 = p0 < cnt && better(list[p0], e);
+    const bool b1 = p1 < cnt && better(list[p1], e);
+    const int pos = __popc(__ballot_sync(0xffffffffu, b0)) + __popc(__ballot_sync(0xffffffffu, b1));
+    if (pos >= k) return;
+    const int ncnt = min(cnt + 1, k);
+    TopkEntry v0, v1;
+    if (p0 < ncnt) v0 = p0 == pos ? e : (p0 > pos ? list[p0 - 1] : list[p0]);
+    if (p1 < ncnt) v1 = p1 == pos ? e : (p1 > pos ? list[p1 - 1] : list[p1]);
+    __syncwarp();
+    if (p0 < ncnt) list[p0] = v0;
+    if (p1 < ncnt) list[p1] = v1;
+    __syncwarp();
+    cnt = ncnt;
+}
+
+// Offer one entry per lane (valid lanes only) to the warp's list.
+__device__ inline void warp_offer(TopkEntry* list, int& cnt, int k, bool valid, const TopkEntry& e) {
+    const bool full = cnt >= k;
+    bool want = valid;
+    if (valid && full) want = better(e, list[k - 1]);
+    unsigned m = __ballot_sync(0xffffffffu, want);
+    while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        TopkEntry x;
+        x.idx = __shfl_sync(0xffffffffu, e.idx, src);
+        x.T = __shfl_sync(0xffffffffu, e.T, src);
+        x.nM = __shfl_sync(0xffffffffu, e.nM, src);
+        x.pad = 0;
+        // re-check against the list as it is now (earlier lanes may have raised the bar)
+        if (cnt < k || better(x, list[k - 1])) warp_insert(list, cnt, k, x);
+    }
+}
+
+// Merge the sorted lists of the CTA's warps (lists[w], counts[w]) into
+// lists[0] with warp 0, then write it and its length to out / out_count.
+// Every thread of the CTA must call it (it synchronises the CTA).
+__device__ inline void cta_merge_lists(TopkEntry* lists, int* counts, int k, int warps, int cnt0,
+                                       TopkEntry* out, int32_t* out_count) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    __syncthreads();
+    if (warp == 0) {
+        int cnt = cnt0;
+        for (int w2 = 1; w2 < warps; ++w2) {
+            const int c2 = counts[w2];
+            for (int b = 0; b < c2; b += 32) {
+                const bool valid = b + lane < c2;
+                TopkEntry e;
+                if (valid) e = lists[w2 * kMaxTopK + b + lane];
+                warp_offer(lists, cnt, k, valid, e);
+            }
+        }
+        for (int p = lane; p < cnt; p += 32) out[p] = lists[p];
+        if (lane == 0) *out_count = cnt;
+    }
+}
+
+// capacity of a top-k state, clamped to the list size
+__device__ __forceinline__ int state_k(const heddle_topk_state* s) {
+    return min(max(s->k, 1), kMaxTopK);
+}
+
+}  // namespace hd

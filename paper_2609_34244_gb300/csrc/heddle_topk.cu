@@ -1,80 +1,48 @@
 // heddle_topk.cu -- rank and top-k of priced candidates.
 //
-// Plans are ranked by predicted throughput (§5 overview); with n replicas of
-// M microbatches per iteration time T a plan processes n*M microbatches per
-// T, so a ranks before b iff nM_a * T_b > nM_b * T_a (exact, 128-bit), and
-// equal throughput goes to the smaller global index.  The order is strict, so
-// the top-k is unique and the result does not depend on the launch shape.
+// The rank order and the warp-level lists are in heddle_rank.cuh.
 //
-// Launch 1: every CTA scans a slice of the batch; each warp keeps its own
+// Launch 1: every CTA scans a slice of the batch (or, after a pricing call,
+// of the worklist of searched candidates only); each warp keeps its own
 // sorted list in shared memory (an entry is inserted only if it beats the
 // current k-th, which after warm-up is rare), the CTA merges its warps'
-// lists and writes one list to scratch.  Launch 2: one CTA merges the
-// per-CTA lists with the incoming state.  No CTA waits on another.
+// lists and writes one list to scratch.  Then the per-CTA lists are folded
+// into the state: one CTA directly for up to 32 lists, else a reduction
+// launch of 32 lists per CTA first.  No CTA waits on another.
 
 #include <algorithm>
 
-#include "heddle_internal.cuh"
+#include "heddle_rank.cuh"
 
 namespace hd {
 namespace {
 
-typedef unsigned __int128 u128;
-
 constexpr int kTopkBlock = 256;
 constexpr int kWarps = kTopkBlock / 32;
+constexpr int kMergeBlock = 512;
+constexpr int kMergeWarps = kMergeBlock / 32;
 
-__device__ __forceinline__ bool better(const TopkEntry& a, const TopkEntry& b) {
-    const u128 l = (u128)a.nM * (u128)(uint64_t)b.T;
-    const u128 r = (u128)b.nM * (u128)(uint64_t)a.T;
-    if (l != r) return l > r;
-    return a.idx < b.idx;
-}
-
-// Warp-cooperative insertion into a sorted list of `cnt` entries (capacity
-// k <= 64; lane l owns slots l and l + 32).  All lanes pass the same e.
-__device__ void warp_insert(TopkEntry* list, int& cnt, int k, const TopkEntry& e) {
-    const int lane = threadIdx.x & 31;
-    const int p0 = lane, p1 = lane + 32;
-    const bool b0 = p0 < cnt && better(list[p0], e);
-    const bool b1 = p1 < cnt && better(list[p1], e);
-    const int pos = __popc(__ballot_sync(0xffffffffu, b0)) + __popc(__ballot_sync(0xffffffffu, b1));
-    if (pos >= k) return;
-    const int ncnt = min(cnt + 1, k);
-    TopkEntry v0, v1;
-    if (p0 < ncnt) v0 = p0 == pos ? e : (p0 > pos ? list[p0 - 1] : list[p0]);
-    if (p1 < ncnt) v1 = p1 == pos ? e : (p1 > pos ? list[p1 - 1] : list[p1]);
-    __syncwarp();
-    if (p0 < ncnt) list[p0] = v0;
-    if (p1 < ncnt) list[p1] = v1;
-    __syncwarp();
-    cnt = ncnt;
-}
-
-// Offer one entry per lane (valid lanes only) to the warp's list.
-__device__ void warp_offer(TopkEntry* list, int& cnt, int k, bool valid, const TopkEntry& e) {
-    const bool full = cnt >= k;
-    bool want = valid;
-    if (valid && full) want = better(e, list[k - 1]);
-    unsigned m = __ballot_sync(0xffffffffu, want);
-    while (m) {
-        const int src = __ffs(m) - 1;
-        m &= m - 1;
-        TopkEntry x;
-        x.idx = __shfl_sync(0xffffffffu, e.idx, src);
-        x.T = __shfl_sync(0xffffffffu, e.T, src);
-        x.nM = __shfl_sync(0xffffffffu, e.nM, src);
-        x.pad = 0;
-        // re-check against the list as it is now (earlier lanes may have raised the bar)
-        if (cnt < k || better(x, list[k - 1])) warp_insert(list, cnt, k, x);
+// One candidate entry: from a batch's results, or from the worklist of a
+// priced chunk (only the searched candidates, T = -1 unless OK).
+template <bool kWorklist>
+__device__ __forceinline__ bool fetch(const TopkArgs& a, int64_t i, TopkEntry& e) {
+    e.pad = 0;
+    if (kWorklist) {
+        const int64_t T = a.wl_T[i];
+        if (T < 0) return false;
+        e.idx = a.base_index + a.wl_idx[i];
+        e.T = T;
+        e.nM = a.wl_nM[i];
+        return true;
     }
+    if (a.status[i] != HEDDLE_CAND_OK) return false;
+    e.idx = a.base_index + i;
+    e.T = a.T[i];
+    e.nM = (uint32_t)a.ndp[i] * (uint32_t)a.M[i];
+    return true;
 }
 
-// capacity of the state, clamped to the list size
-__device__ __forceinline__ int state_k(const heddle_topk_state* s) {
-    return min(max(s->k, 1), kMaxTopK);
-}
-
+template <bool kWorklist>
 __global__ void __launch_bounds__(kTopkBlock) topk_block_kernel(TopkArgs a) {
     const int k = state_k(a.state);
     __shared__ TopkEntry lists[kWarps][kMaxTopK];
@@ -82,47 +50,63 @@ __global__ void __launch_bounds__(kTopkBlock) topk_block_kernel(TopkArgs a) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int cnt = 0;
     TopkEntry* list = lists[warp];
+    const int64_t n = kWorklist ? min((int64_t)*a.wl_count, (int64_t)a.wl_cap) : a.n;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
-    for (int64_t base = gw * 32; base < a.n; base += nwarps * 32) {
-        const int64_t c = base + lane;
+    for (int64_t base = gw * 32; base < n; base += nwarps * 32) {
+        const int64_t i = base + lane;
         TopkEntry e;
-        bool valid = false;
-        if (c < a.n && a.status[c] == HEDDLE_CAND_OK) {
-            e.idx = a.base_index + c;
-            e.T = a.T[c];
-            e.nM = (uint32_t)a.ndp[c] * (uint32_t)a.M[c];
-            e.pad = 0;
-            valid = true;
-        }
+        const bool valid = i < n && fetch<kWorklist>(a, i, e);
         warp_offer(list, cnt, k, valid, e);
     }
     if (lane == 0) counts[warp] = cnt;
-    __syncthreads();
-    if (warp == 0) {
-        for (int w2 = 1; w2 < kWarps; ++w2) {
-            const int c2 = counts[w2];
-            for (int b = 0; b < c2; b += 32) {
-                const bool valid = b + lane < c2;
-                TopkEntry e;
-                if (valid) e = lists[w2][b + lane];
-                warp_offer(list, cnt, k, valid, e);
-            }
-        }
-        for (int p = lane; p < cnt; p += 32) a.scratch[(size_t)blockIdx.x * kMaxTopK + p] = list[p];
-        if (lane == 0) a.scratch_count[blockIdx.x] = cnt;
+    cta_merge_lists(&lists[0][0], counts, k, kWarps, cnt, a.scratch + (size_t)blockIdx.x * kMaxTopK,
+                    a.scratch_count + blockIdx.x);
+}
+
+// Offer the entries of list `l` (count `c`) to this warp's list.
+__device__ __forceinline__ void offer_list(const TopkEntry* l, int c, TopkEntry* list, int& cnt, int k) {
+    const int lane = threadIdx.x & 31;
+    for (int b = 0; b < c; b += 32) {
+        const bool valid = b + lane < c;
+        TopkEntry e;
+        if (valid) e = l[b + lane];
+        warp_offer(list, cnt, k, valid, e);
     }
 }
 
-__global__ void __launch_bounds__(kTopkBlock) topk_merge_kernel(TopkArgs a, int blocks) {
-    __shared__ TopkEntry lists[kWarps][kMaxTopK];
-    __shared__ int counts[kWarps];
+// First merge level: CTA b folds lists [32 b, 32 b + 32) into out[b]; each
+// warp takes two lists, whose counts it loads together.
+__global__ void __launch_bounds__(kMergeBlock) topk_reduce_kernel(TopkArgs a, int blocks) {
+    __shared__ TopkEntry lists[kMergeWarps * kMaxTopK];
+    __shared__ int counts[kMergeWarps];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int k = state_k(a.state);
     int cnt = 0;
-    TopkEntry* list = lists[warp];
-    // warp 0 starts from the incoming state; every warp takes a share of the CTA lists
+    TopkEntry* list = lists + warp * kMaxTopK;
+    const int l0 = blockIdx.x * 32 + warp, l1 = l0 + kMergeWarps;
+    const int c0 = l0 < blocks ? a.scratch_count[l0] : 0;
+    const int c1 = l1 < blocks ? a.scratch_count[l1] : 0;
+    offer_list(a.scratch + (size_t)l0 * kMaxTopK, c0, list, cnt, k);
+    offer_list(a.scratch + (size_t)l1 * kMaxTopK, c1, list, cnt, k);
+    if (lane == 0) counts[warp] = cnt;
+    cta_merge_lists(lists, counts, k, kMergeWarps, cnt, a.scratch2 + (size_t)blockIdx.x * kMaxTopK,
+                    a.scratch2_count + blockIdx.x);
+}
+
+// Last merge level: one CTA folds `blocks` lists and the incoming state.
+__global__ void __launch_bounds__(kMergeBlock) topk_merge_kernel(TopkArgs a, const TopkEntry* src,
+                                                                 const int32_t* src_count, int blocks) {
+    __shared__ TopkEntry lists[kMergeWarps * kMaxTopK];
+    __shared__ int counts[kMergeWarps];
+    __shared__ TopkEntry merged[kMaxTopK];
+    __shared__ int32_t merged_count;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int k = state_k(a.state);
+    int cnt = 0;
+    TopkEntry* list = lists + warp * kMaxTopK;
     if (warp == 0) {
+        // the incoming state
         const int c0 = min(max(a.state->count, 0), k);
         for (int b = 0; b < c0; b += 32) {
             const bool valid = b + lane < c0;
@@ -136,40 +120,32 @@ __global__ void __launch_bounds__(kTopkBlock) topk_merge_kernel(TopkArgs a, int 
             warp_offer(list, cnt, k, valid, e);
         }
     }
-    for (int blk = warp; blk < blocks; blk += kWarps) {
-        const int cb = a.scratch_count[blk];
-        for (int b = 0; b < cb; b += 32) {
-            const bool valid = b + lane < cb;
-            TopkEntry e;
-            if (valid) e = a.scratch[(size_t)blk * kMaxTopK + b + lane];
-            warp_offer(list, cnt, k, valid, e);
-        }
-    }
+    for (int l = warp; l < blocks; l += kMergeWarps) offer_list(src + (size_t)l * kMaxTopK, src_count[l], list, cnt, k);
     if (lane == 0) counts[warp] = cnt;
+    cta_merge_lists(lists, counts, k, kMergeWarps, cnt, merged, &merged_count);
     __syncthreads();
-    if (warp == 0) {
-        for (int w2 = 1; w2 < kWarps; ++w2) {
-            const int c2 = counts[w2];
-            for (int b = 0; b < c2; b += 32) {
-                const bool valid = b + lane < c2;
-                TopkEntry e;
-                if (valid) e = lists[w2][b + lane];
-                warp_offer(list, cnt, k, valid, e);
-            }
-        }
-        for (int p = lane; p < kMaxTopK; p += 32) {
-            if (p < cnt) {
-                a.state->idx[p] = list[p].idx;
-                a.state->T[p] = list[p].T;
-                a.state->nM[p] = list[p].nM;
-            } else {
-                a.state->idx[p] = -1;
-                a.state->T[p] = -1;
-                a.state->nM[p] = 0;
-            }
-        }
-        if (lane == 0) a.state->count = cnt;
+    for (int p = threadIdx.x; p < kMaxTopK; p += blockDim.x) {
+        const bool live = p < merged_count;
+        a.state->idx[p] = live ? merged[p].idx : -1;
+        a.state->T[p] = live ? merged[p].T : -1;
+        a.state->nM[p] = live ? merged[p].nM : 0;
     }
+    if (threadIdx.x == 0) a.state->count = merged_count;
+}
+
+// Merge `blocks` per-CTA lists of a.scratch into *a.state: directly, or
+// through one reduction level of 32 lists per CTA when there are many.
+cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st) {
+    if (blocks <= 2 * kMergeWarps) {
+        topk_merge_kernel<<<1, kMergeBlock, 0, st>>>(a, a.scratch, a.scratch_count, blocks);
+        return cudaGetLastError();
+    }
+    const int m1 = (blocks + 31) / 32;
+    topk_reduce_kernel<<<m1, kMergeBlock, 0, st>>>(a, blocks);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    topk_merge_kernel<<<1, kMergeBlock, 0, st>>>(a, a.scratch2, a.scratch2_count, m1);
+    return cudaGetLastError();
 }
 
 __global__ void topk_reset_kernel(heddle_topk_state* s, int k) {
@@ -191,11 +167,21 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st) {
     const int64_t per_block = (int64_t)kTopkBlock * 8;  // at least 8 candidates per thread
     int grid = (int)std::min<int64_t>((a.n + per_block - 1) / per_block, (int64_t)2 * num_sms);
     grid = std::max(1, std::min(grid, a.max_blocks));
-    topk_block_kernel<<<grid, kTopkBlock, 0, st>>>(a);
+    topk_block_kernel<false><<<grid, kTopkBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    topk_merge_kernel<<<1, kTopkBlock, 0, st>>>(a, grid);
-    return cudaGetLastError();
+    return merge_lists(a, grid, st);
+}
+
+cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    const int64_t per_block = (int64_t)kTopkBlock * 8;
+    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)2 * num_sms);
+    grid = std::max(1, std::min(grid, a.max_blocks));
+    topk_block_kernel<true><<<grid, kTopkBlock, 0, st>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return merge_lists(a, grid, st);
 }
 
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st) {

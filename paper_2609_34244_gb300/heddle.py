@@ -63,7 +63,8 @@ TOPK_STATE_BYTES = C.sizeof(heddle_topk_state)
 EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_cluster",
            "heddle_load_model", "heddle_price_candidates", "heddle_topk_reset", "heddle_topk",
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
-           "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search"]
+           "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
+           "heddle_price_topk"]
 SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS = 0, 1, 2
 
 _lib = None
@@ -87,6 +88,7 @@ def load_library(path: str = LIB_PATH):
         "heddle_price_candidates": (i32, [p, p, p, p]),
         "heddle_topk_reset": (i32, [p, p, i32, p]),
         "heddle_topk": (i32, [p, p, p, p, p]),
+        "heddle_price_topk": (i32, [p, p, p, p, p]),
         "heddle_price_topk_host": (i32, [p, p, p, p, i64, p]),
         "heddle_get_tables": (i32, [p, p, p]),
         "heddle_device_errors": (i32, [p, C.POINTER(C.c_uint32)]),
@@ -210,6 +212,13 @@ def heddle_topk(ctx, cands, results, state, stream=None):
     c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
     r = results if isinstance(results, heddle_results) else make_results(results)
     _check(ctx, load_library().heddle_topk(ctx, C.byref(c), C.byref(r), _ptr(state), _stream(stream)))
+
+
+def heddle_price_topk(ctx, cands, results, state, stream=None):
+    """Price device candidates and merge their OK ones into the device state."""
+    c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
+    r = results if isinstance(results, heddle_results) else make_results(results)
+    _check(ctx, load_library().heddle_price_topk(ctx, C.byref(c), C.byref(r), _ptr(state), _stream(stream)))
 
 
 def heddle_price_topk_host(ctx, cands: dict, results: dict | None, state: heddle_topk_state,

@@ -8,10 +8,12 @@ import functools
 import numpy as np
 
 
-def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False, search=None):
+def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False, search=None,
+              fused=False):
     """Price on the GPU through the C ABI; returns numpy results, the top-k
     and (optionally) the work counters.  ``batch`` splits the candidates into
-    consecutive launches merged into one top-k state."""
+    consecutive launches merged into one top-k state; ``fused`` prices and
+    merges in one call (heddle_price_topk)."""
     import torch
     ctx = h.heddle_create(0)
     try:
@@ -37,8 +39,11 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
             r = h.heddle_results(res["T"].data_ptr() + 8 * lo, res["bottleneck"].data_ptr() + 8 * lo,
                                  res["n_dp"].data_ptr() + 2 * lo, res["status"].data_ptr() + lo,
                                  None if bb is None else bb.data_ptr())
-            h.heddle_price_candidates(ctx, c, r)
-            h.heddle_topk(ctx, c, r, state)
+            if fused:
+                h.heddle_price_topk(ctx, c, r, state)
+            else:
+                h.heddle_price_candidates(ctx, c, r)
+                h.heddle_topk(ctx, c, r, state)
             if bounds:
                 out_bounds[:, lo:hi] = bb.cpu().numpy()
         torch.cuda.synchronize()

@@ -163,6 +163,26 @@ def test_batching_and_launch_shape_do_not_change_results(h, W, oracle_mod):
     assert c["counters"]["checks"] > 0 and c["counters"]["priced"] > 0
 
 
+@pytest.mark.parametrize("name,n,seed", [("dense32", 20011, 0), ("moe48", 20011, 0), ("tiny_ext", None, 0),
+                                         ("stress128", 30011, 1), ("dense80", 9001, 2)])
+@pytest.mark.parametrize("k", [1, 16, 64])
+def test_fused_price_topk(h, W, oracle_mod, name, n, seed, k):
+    """heddle_price_topk (top-k fused into the search) == price then topk ==
+    the oracle's top-k, for several k, batch splits and both searches."""
+    w = W.make_workload(name, seed=seed, n=n)
+    ref = oracle_mod.Oracle(w.cluster, w.model).price(w.cands, threads=8)
+    tk = oracle_mod.topk(ref, w.cands["M"], k)
+    for search in (0, 1):
+        for batch in (None, 7001):
+            got = G.price_gpu(h, w.cluster, w.model, w.cands, k=k, bounds=False, batch=batch, search=search,
+                              fused=True)
+            assert got["errors"] == 0
+            G.assert_same(got, ref, what="%s fused" % name)
+            assert got["topk"]["idx"].tolist() == tk["idx"].tolist(), (name, k, search, batch)
+            assert got["topk"]["T"].tolist() == tk["T"].tolist()
+            assert got["topk"]["nM"].tolist() == tk["nM"].tolist()
+
+
 def test_edge_cases(h, W, oracle_mod):
     # n = 0 is a no-op; n = 1
     w = W.make_workload("dense32", n=1)
