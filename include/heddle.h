@@ -233,6 +233,36 @@ heddle_status heddle_price_topk(heddle_ctx* ctx, const heddle_candidates* cands,
                                 const heddle_results* results, heddle_topk_state* state,
                                 void* stream);
 
+/* ------------------------------------------------- allocation-free top-k */
+
+/* The top-k merge of heddle_topk for callers that cannot allocate device
+ * memory at all -- for example code running inside another framework's
+ * memory pool, where every device allocation must go through that pool, or
+ * code that must not allocate after start-up -- and therefore cannot create
+ * a heddle context either.  The paper has no counterpart: this is a
+ * property of the library, not of the method.
+ *
+ * No context: runs on the calling thread's current device and allocates
+ * nothing (no cudaMalloc, no library allocation).  Its scratch is a
+ * file-scope device array of 96.25 KB that every device holds from the time
+ * the library's device code is loaded until the process exits: 64 lists of
+ * 64 entries, one per slice of 65,536 candidates, so a call handles at most
+ * HEDDLE_TOPK_NOALLOC_MAX_N = 4,194,304 candidates (E_LIMIT beyond).
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * Every call on a device shares the array and overwrites it, so calls whose
+ * kernels overlap on the GPU race: serialise them (one stream).
+ *
+ * Arguments as heddle_topk: merges the OK candidates of a priced batch
+ * (cands->M, base_index; results->T, n_dp, status; device memory) into
+ * *state (device, as set up by heddle_topk_reset or copied in by the
+ * caller).  Same resulting state as heddle_topk.  Asynchronous on `stream`.
+ * Errors: E_ARG (null pointers, n < 0), E_LIMIT (n above the maximum),
+ * E_CUDA (symbol lookup or launch failed); there is no message buffer. */
+#define HEDDLE_TOPK_NOALLOC_MAX_N 4194304
+heddle_status heddle_topk_noalloc(const heddle_candidates* cands, const heddle_results* results,
+                                  heddle_topk_state* state, void* stream);
+
 /* -------------------------------------------------------- host buffers */
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the

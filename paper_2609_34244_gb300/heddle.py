@@ -64,7 +64,8 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
            "heddle_load_model", "heddle_price_candidates", "heddle_topk_reset", "heddle_topk",
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
            "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
-           "heddle_price_topk"]
+           "heddle_price_topk", "heddle_topk_noalloc"]
+TOPK_NOALLOC_MAX_N = 4194304
 SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS = 0, 1, 2
 
 _lib = None
@@ -89,6 +90,7 @@ def load_library(path: str = LIB_PATH):
         "heddle_topk_reset": (i32, [p, p, i32, p]),
         "heddle_topk": (i32, [p, p, p, p, p]),
         "heddle_price_topk": (i32, [p, p, p, p, p]),
+        "heddle_topk_noalloc": (i32, [p, p, p, p]),
         "heddle_price_topk_host": (i32, [p, p, p, p, i64, p]),
         "heddle_get_tables": (i32, [p, p, p]),
         "heddle_device_errors": (i32, [p, C.POINTER(C.c_uint32)]),
@@ -219,6 +221,15 @@ def heddle_price_topk(ctx, cands, results, state, stream=None):
     c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
     r = results if isinstance(results, heddle_results) else make_results(results)
     _check(ctx, load_library().heddle_price_topk(ctx, C.byref(c), C.byref(r), _ptr(state), _stream(stream)))
+
+
+def heddle_topk_noalloc(cands, results, state, stream=None):
+    """Allocation-free top-k merge (no context; current device); see the header."""
+    c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
+    r = results if isinstance(results, heddle_results) else make_results(results)
+    st = load_library().heddle_topk_noalloc(C.byref(c), C.byref(r), _ptr(state), _stream(stream))
+    if st != 0:
+        raise HeddleError(st, "heddle_topk_noalloc failed")
 
 
 def heddle_price_topk_host(ctx, cands: dict, results: dict | None, state: heddle_topk_state,
