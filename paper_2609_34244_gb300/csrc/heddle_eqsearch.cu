@@ -7,19 +7,27 @@
 //     cap_s(B) = min(m_s, floor((B - c_s) / q_s))
 // layers within bound B (m_s: the longest run of layers that fits the
 // stage's memory, c_s: its P2P).  A split with every stage time <= B exists
-// iff every cap_s >= 1 and sum_s cap_s >= L, so a probe costs O(S).  The
-// search snaps to exact breakpoints: a feasible probe keeps the same caps
-// down to max_s (c_s + cap_s q_s), an infeasible one up to the smallest
-// c_s + (cap_s + 1) q_s of a stage that can still grow; it starts from the
-// continuous balance sum_s (B - c_s) / q_s = L and brackets by the largest q.
-// At B* the componentwise smallest split -- hence the lexicographically
-// smallest -- is a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
+// iff every cap_s >= 1 and sum_s cap_s >= L, so a probe costs O(S).
+// B* >= max_s (c_s + q_s) (every stage holds a layer), which starts the
+// bracket; the first probe is the continuous balance
+// sum_s (B - c_s) / q_s = L, later ones interpolate the cap count between
+// the bracket's probes (a Newton step on the count while one side is
+// missing), falling back to bisection.  Every probe snaps the bracket to
+// exact breakpoints: a feasible probe keeps the same caps down to
+// max_s (c_s + cap_s q_s), an infeasible one up to the smallest
+// c_s + (cap_s + 1) q_s of a stage that can still grow, so the search ends
+// on B* itself with the caps of its last feasible probe, which hold at B*.
+// The componentwise smallest split -- hence the lexicographically smallest
+// -- is then a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
 //
-// Layout: a few small tables (per-layer cost per (type, degree), P2P,
-// gradient-byte prefix, NIC, memory runs) are copied to shared memory once
-// per CTA; every candidate's stages are packed once into 32-bit words
-// (cost index | P2P index | memory run) held in shared memory interleaved by
-// thread, so probes read one conflict-free word per stage.
+// Layout: a few small tables (per-layer cost and its reciprocal per (type,
+// degree), P2P, gradient-byte prefix, NIC, memory runs) are copied to shared
+// memory once per CTA; every candidate's stages are packed once into 32-bit
+// words (cost index | P2P index | memory run) held in shared memory
+// interleaved by thread, so probes read one conflict-free word per stage.
+// Each CTA takes 256 worklist entries at a time and sorts them by S
+// (counting sort) so that the lanes of a warp run stage loops of equal
+// length.
 
 #include <algorithm>
 
@@ -35,7 +43,7 @@ constexpr int kZeroP2P = 128;  // a zero entry after the 8 x 8 x 2 P2P table
 constexpr int kMaxIters = 256;
 
 struct EqLayout {
-    uint32_t q, p2p, inter, maxn, PB, win, sw, caps, bytes;
+    uint32_t q, rq, p2p, inter, maxn, PB, win, sw, caps, bytes;
 };
 
 __host__ __device__ inline uint32_t al16(uint32_t x) { return (x + 15u) & ~15u; }
@@ -44,26 +52,28 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
     EqLayout e;
     uint32_t o = 0;
     e.q = o;     o = al16(o + 8 * 32);             // int64 [j * 8 + g]
+    e.rq = o;    o = al16(o + 4 * 32);             // float 1 / q
     e.p2p = o;   o = al16(o + 8 * 129);            // int64 [(g * 8 + h) * 2 + same], [128] = 0
     e.inter = o; o = al16(o + 8 * 8);              // int64 [g]
     e.maxn = o;  o = al16(o + 4 * 8);              // int32 [g]
     e.PB = o;    o = al16(o + 8 * (L + 1));        // int64 gradient-byte prefix
     e.win = o;   o = al16(o + 8 * 4 * 33);         // uint8 [(g * 4 + j) * 33 + f]
     e.sw = o;    o = al16(o + 4 * kMaxStages * kEqBlock);  // uint32 [s][thread]
-    e.caps = o;  o = al16(o + (kMaxStages + 1) * kEqBlock); // uint8 [s][thread]
+    e.caps = o;  o = al16(o + 2 * (kMaxStages + 1) * kEqBlock);  // uint8 [2][s][thread]
     e.bytes = o;
     return e;
 }
 
 struct EqTabs {
     const int64_t* q;
+    const float* rq;
     const int64_t* p2p;
     const int64_t* inter;
     const int32_t* maxn;
     const int64_t* PB;
     const uint8_t* win;
     uint32_t* sw;   // this thread's stage words, element s at [s * kEqBlock]
-    uint8_t* caps;  // this thread's caps, element s at [s * kEqBlock]
+    uint8_t* caps;  // this thread's caps, two sets, set b element s at [(b * 33 + s) * kEqBlock]
     int L;
 };
 
@@ -102,7 +112,7 @@ __device__ __forceinline__ Cap stage_cap(const EqTabs& t, uint32_t w, int64_t B)
         return r;
     }
     // x < m q with m <= 255: the float estimate is off by at most one
-    int k = (int)((float)x / (float)r.q);
+    int k = (int)((float)x * t.rq[w & 31]);
     if ((int64_t)k * r.q > x) --k;
     if ((int64_t)(k + 1) * r.q <= x) ++k;
     r.k = k;
@@ -110,17 +120,25 @@ __device__ __forceinline__ Cap stage_cap(const EqTabs& t, uint32_t w, int64_t B)
 }
 
 struct Snap {
-    int64_t hi, lo;
+    int64_t hi, lo;  // snapping values
+    int tot;         // layers the stages hold (stages holding one or more)
+    float slope;     // growth of tot per unit of B: sum of 1/q over stages below their run
     unsigned long long units;
 };
 
-__device__ bool eq_probe(const EqTabs& t, int S, int64_t B, Snap& sn) {
+// Probe bound B; the caps go to cap set `set`.
+__device__ bool eq_probe(const EqTabs& t, int S, int64_t B, int set, Snap& sn) {
     sn.hi = -1;
     sn.lo = kInf;
+    sn.slope = 0.f;
     int sum = 0;
     bool ok = true;
+    uint8_t* caps = t.caps + set * (kMaxStages + 1) * kEqBlock;
     for (int s = 0; s < S; ++s) {
-        const Cap r = stage_cap(t, t.sw[s * kEqBlock], B);
+        const uint32_t w = t.sw[s * kEqBlock];
+        const Cap r = stage_cap(t, w, B);
+        caps[s * kEqBlock] = (uint8_t)max(r.k, 0);
+        if (r.k < r.m) sn.slope += t.rq[w & 31];
         if (r.k < 1) {
             ok = false;
             if (r.m >= 1) sn.lo = min(sn.lo, r.c + r.q);
@@ -131,18 +149,22 @@ __device__ bool eq_probe(const EqTabs& t, int S, int64_t B, Snap& sn) {
         if (r.k < r.m) sn.lo = min(sn.lo, r.c + (int64_t)(r.k + 1) * r.q);
     }
     sn.units += S;
+    sn.tot = sum;
     return ok && sum >= t.L;
 }
 
 template <bool kCount>
 __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ int bins[kMaxStages + 2];
+    __shared__ uint16_t order[kEqBlock];
     const Layout& y = a.lay;
     const int L = y.L;
     const EqLayout el = eq_layout(L);
     // small tables, copied once per CTA
     {
         int64_t* q = reinterpret_cast<int64_t*>(smem + el.q);
+        float* rq = reinterpret_cast<float*>(smem + el.rq);
         int64_t* p2p = reinterpret_cast<int64_t*>(smem + el.p2p);
         int64_t* inter = reinterpret_cast<int64_t*>(smem + el.inter);
         int32_t* maxn = reinterpret_cast<int32_t*>(smem + el.maxn);
@@ -151,7 +173,9 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
         const int64_t* gP = reinterpret_cast<const int64_t*>(a.img + y.offP);
         for (int i = threadIdx.x; i < 32; i += blockDim.x) {
             const int g = i & 7, j = i >> 3;
-            q[i] = g < y.NT ? gP[(g * 4 + j) * (L + 1) + 1] - gP[(g * 4 + j) * (L + 1)] : 0;
+            const int64_t v = g < y.NT ? gP[(g * 4 + j) * (L + 1) + 1] - gP[(g * 4 + j) * (L + 1)] : 0;
+            q[i] = v;
+            rq[i] = v > 0 ? 1.0f / (float)v : 0.0f;
         }
         for (int i = threadIdx.x; i < 129; i += blockDim.x)
             p2p[i] = i < 128 ? reinterpret_cast<const int64_t*>(a.img + y.offP2P)[i] : 0;
@@ -166,6 +190,7 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     __syncthreads();
     EqTabs t;
     t.q = reinterpret_cast<const int64_t*>(smem + el.q);
+    t.rq = reinterpret_cast<const float*>(smem + el.rq);
     t.p2p = reinterpret_cast<const int64_t*>(smem + el.p2p);
     t.inter = reinterpret_cast<const int64_t*>(smem + el.inter);
     t.maxn = reinterpret_cast<const int32_t*>(smem + el.maxn);
@@ -179,17 +204,40 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     sn.units = 0;
     unsigned long long probes = 0, searched = 0;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < count; p += stride) {
+    const int64_t count_r = (count + kEqBlock - 1) / kEqBlock * kEqBlock;
+    const int64_t stride = (int64_t)gridDim.x * kEqBlock;
+    for (int64_t base = (int64_t)blockIdx.x * kEqBlock; base < count_r; base += stride) {
+        // ---- this CTA's 256 entries, counting-sorted by S (0: no entry)
+        const int64_t p0 = base + threadIdx.x;
+        const int s0 = p0 < count ? a.wl_S[p0] : 0;
+        if (threadIdx.x < kMaxStages + 2) bins[threadIdx.x] = 0;
+        __syncthreads();
+        atomicAdd(&bins[s0], 1);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            int run = 0;
+            for (int b = 0; b <= kMaxStages; ++b) {
+                const int v = bins[b];
+                bins[b] = run;
+                run += v;
+            }
+        }
+        __syncthreads();
+        order[atomicAdd(&bins[s0], 1)] = (uint16_t)threadIdx.x;
+        __syncthreads();
+        const int64_t p = base + order[threadIdx.x];
+        __syncthreads();  // bins and order are reused by the next slice
+        if (p >= count) continue;
+
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
         const int M = a.wl_M[p];
         const int64_t n = a.wl_n[p];
         if (kCount) ++searched;
         // pack the stages; feasible upper bound (every stage at its memory
-        // run, which the screen guarantees covers L) and the continuous
-        // balance sum_s (B - c_s) / q_s = L as the first probe
-        int64_t hi = 0, qmax = 1;
+        // run, which the screen guarantees covers L), lower bound (every
+        // stage holds one layer) and the continuous balance as first probe
+        int64_t hi = 0, lo = 0;
         float inv = 0.f, cw = 0.f;
         int code = a.wl_code[p];
         for (int s = 0; s < S; ++s) {
@@ -200,52 +248,63 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             const int64_t q = t.q[w & 31], cc = t.p2p[(w >> 5) & 255];
             const int m = (int)(w >> 13) & 255;
             hi = max(hi, cc + (int64_t)m * q);
-            qmax = max(qmax, q);
+            lo = max(lo, cc + q);
             const float qf = (float)q + 0.5f;
             inv += 1.0f / qf;
             cw += (float)cc / qf;
             code = next;
         }
-        int64_t lo = 0;
-        bool lo_known = false, hi_known = false;
         int64_t B = (int64_t)(((float)L + cw) / inv);
-        int64_t step = qmax;
+        // bracket probes (bound, cap count) for the interpolation
+        int64_t Blo = -1, Bhi = -1;
+        int clo = 0, chi = 0;
+        int wset = 0, fset = -1;  // cap set written next / of the last feasible probe
         int it = 0;
         while (lo < hi) {
             B = min(max(B, lo), hi - 1);
             if (kCount) ++probes;
-            if (eq_probe(t, S, B, sn)) {
+            const bool feas = eq_probe(t, S, B, wset, sn);
+            if (feas) {
                 hi = sn.hi;
-                hi_known = true;
+                Bhi = B;
+                chi = sn.tot;
+                fset = wset;
+                wset ^= 1;
             } else {
-                lo = sn.lo;
-                lo_known = true;
+                lo = max(lo, sn.lo);
+                Blo = B;
+                clo = sn.tot;
             }
             if (lo >= hi) break;
-            if (!lo_known) {
-                B = hi - step;
-                step *= 2;
-            } else if (!hi_known) {
-                B = lo + step;
-                step *= 2;
+            // next bound: interpolate the cap count between the bracket's
+            // probes, else a Newton step, else bisect
+            float target;
+            if (Blo >= 0 && Bhi >= 0 && chi > clo) {
+                target = (float)Blo + ((float)L - 0.5f - (float)clo) / (float)(chi - clo) * (float)(Bhi - Blo);
+            } else if (sn.slope > 0.f) {
+                target = feas ? (float)B - ceilf(((float)sn.tot - (float)L + 0.5f) / sn.slope)
+                              : (float)B + ceilf(((float)L - (float)sn.tot) / sn.slope);
             } else {
-                B = lo + (hi - lo) / 2;
+                target = -1.f;
             }
+            B = (target >= (float)lo && target <= (float)(hi - 1)) ? (int64_t)target : lo + (hi - lo) / 2;
             if (++it > kMaxIters) {
                 atomicOr(a.err, kErrSearchBound);
                 break;
             }
         }
         const int64_t Bstar = hi;
-        // caps at B*, then the smallest boundaries from suffix sums
-        int total = 0;
-        for (int s = 0; s < S; ++s) {
-            const Cap r = stage_cap(t, t.sw[s * kEqBlock], Bstar);
-            if (r.k < 1) atomicOr(a.err, kErrInternal);
-            t.caps[s * kEqBlock] = (uint8_t)max(r.k, 0);
-            total += r.k;
+        if (fset < 0) {
+            // B* is the initial bound, never probed: its caps
+            if (kCount) ++probes;
+            if (!eq_probe(t, S, Bstar, 0, sn)) atomicOr(a.err, kErrInternal);
+            fset = 0;
         }
-        // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s, stage by stage
+        const uint8_t* caps = t.caps + fset * (kMaxStages + 1) * kEqBlock;
+        int total = 0;
+        for (int s = 0; s < S; ++s) total += caps[s * kEqBlock];
+        // ---- the smallest boundaries, then Evaluate:
+        //      T = (M-1) max t_s + sum t_s + max g_s, stage by stage
         int64_t tmax = 0, tsum = 0;
         int sg = -1;
         u128 bestG = 0, bestD = 1;
@@ -254,7 +313,9 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
         bnd[0] = 0;
         for (int s = 0; s < S; ++s) {
             const uint32_t w = t.sw[s * kEqBlock];
-            pre += t.caps[s * kEqBlock];
+            const int k = caps[s * kEqBlock];
+            if (k < 1) atomicOr(a.err, kErrInternal);
+            pre += k;
             const int nxt = s + 1 == S ? L : max(at + 1, L - (total - pre));
             bnd[s + 1] = (uint8_t)nxt;
             const int64_t ts = (int64_t)(nxt - at) * t.q[w & 31] + t.p2p[(w >> 5) & 255];
