@@ -84,6 +84,60 @@ __device__ inline void cta_merge_lists(TopkEntry* lists, int* counts, int k, int
     }
 }
 
+// Merge two sorted lists A (na) and B (nb) into out (the first min(na + nb,
+// k) entries), one warp, all lanes in parallel: an entry's place in the
+// merged list is its place in its own list plus the number of entries of
+// the other list that rank before it (a binary search); the order is strict,
+// so the places are distinct.  out must not overlap A or B.
+__device__ inline int warp_merge(const TopkEntry* A, int na, const TopkEntry* B, int nb, TopkEntry* out,
+                                 int k) {
+    const int lane = threadIdx.x & 31;
+    for (int i = lane; i < na && i < k; i += 32) {
+        const TopkEntry x = A[i];
+        int lo = 0, hi = nb;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (better(B[mid], x)) lo = mid + 1; else hi = mid;
+        }
+        if (i + lo < k) out[i + lo] = x;
+    }
+    for (int i = lane; i < nb && i < k; i += 32) {
+        const TopkEntry x = B[i];
+        int lo = 0, hi = na;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (better(A[mid], x)) lo = mid + 1; else hi = mid;
+        }
+        if (i + lo < k) out[i + lo] = x;
+    }
+    __syncwarp();
+    return min(na + nb, k);
+}
+
+// Tree merge of W sorted lists (lists[w * kMaxTopK], counts[w]) held in
+// shared memory, using tmp (ceil(W / 2) lists); the result ends in lists[0]
+// with length counts[0].  Every thread of the CTA must call it, with at
+// least W / 2 warps.
+__device__ inline void cta_tree_merge(TopkEntry* lists, int* counts, TopkEntry* tmp, int* tmp_counts, int W,
+                                      int k) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int width = W; width > 1; width = (width + 1) / 2) {
+        const int half = (width + 1) / 2;
+        __syncthreads();
+        if (warp < width - half) {
+            const int c = warp_merge(lists + warp * kMaxTopK, counts[warp], lists + (warp + half) * kMaxTopK,
+                                     counts[warp + half], tmp + warp * kMaxTopK, k);
+            if (lane == 0) tmp_counts[warp] = c;
+        }
+        __syncthreads();
+        if (warp < width - half) {
+            for (int i = lane; i < tmp_counts[warp]; i += 32) lists[warp * kMaxTopK + i] = tmp[warp * kMaxTopK + i];
+            if (lane == 0) counts[warp] = tmp_counts[warp];
+        }
+    }
+    __syncthreads();
+}
+
 // capacity of a top-k state, clamped to the list size
 __device__ __forceinline__ int state_k(const heddle_topk_state* s) {
     return min(max(s->k, 1), kMaxTopK);

@@ -6,9 +6,10 @@
 // of the worklist of searched candidates only); each warp keeps its own
 // sorted list in shared memory (an entry is inserted only if it beats the
 // current k-th, which after warm-up is rare), the CTA merges its warps'
-// lists and writes one list to scratch.  Then the per-CTA lists are folded
-// into the state: one CTA directly for up to 32 lists, else a reduction
-// launch of 32 lists per CTA first.  No CTA waits on another.
+// lists (a tree of parallel two-list merges) and writes one list to
+// scratch.  Then the per-CTA lists are folded into the state by merge
+// levels of 16 lists per CTA: one level for up to 16 lists, else two.  No
+// CTA waits on another.
 
 #include <algorithm>
 
@@ -19,7 +20,7 @@ namespace {
 
 constexpr int kTopkBlock = 256;
 constexpr int kWarps = kTopkBlock / 32;
-constexpr int kMergeBlock = 512;
+constexpr int kMergeBlock = 1024;  // warps 0-15 stage lists, warp 16 the state
 constexpr int kMergeWarps = kMergeBlock / 32;
 
 // One candidate entry: from a batch's results, or from the worklist of a
@@ -45,11 +46,12 @@ __device__ __forceinline__ bool fetch(const TopkArgs& a, int64_t i, TopkEntry& e
 template <bool kWorklist>
 __global__ void __launch_bounds__(kTopkBlock) topk_block_kernel(TopkArgs a) {
     const int k = state_k(a.state);
-    __shared__ TopkEntry lists[kWarps][kMaxTopK];
-    __shared__ int counts[kWarps];
+    __shared__ TopkEntry lists[kWarps * kMaxTopK];
+    __shared__ TopkEntry tmp[(kWarps / 2) * kMaxTopK];
+    __shared__ int counts[kWarps], tmp_counts[kWarps / 2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int cnt = 0;
-    TopkEntry* list = lists[warp];
+    TopkEntry* list = lists + warp * kMaxTopK;
     const int64_t n = kWorklist ? min((int64_t)*a.wl_count, (int64_t)a.wl_cap) : a.n;
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
@@ -60,91 +62,75 @@ __global__ void __launch_bounds__(kTopkBlock) topk_block_kernel(TopkArgs a) {
         warp_offer(list, cnt, k, valid, e);
     }
     if (lane == 0) counts[warp] = cnt;
-    cta_merge_lists(&lists[0][0], counts, k, kWarps, cnt, a.scratch + (size_t)blockIdx.x * kMaxTopK,
-                    a.scratch_count + blockIdx.x);
+    cta_tree_merge(lists, counts, tmp, tmp_counts, kWarps, k);
+    for (int p = threadIdx.x; p < counts[0]; p += blockDim.x)
+        a.scratch[(size_t)blockIdx.x * kMaxTopK + p] = lists[p];
+    if (threadIdx.x == 0) a.scratch_count[blockIdx.x] = counts[0];
 }
 
-// Offer the entries of list `l` (count `c`) to this warp's list.
-__device__ __forceinline__ void offer_list(const TopkEntry* l, int c, TopkEntry* list, int& cnt, int k) {
-    const int lane = threadIdx.x & 31;
-    for (int b = 0; b < c; b += 32) {
-        const bool valid = b + lane < c;
-        TopkEntry e;
-        if (valid) e = l[b + lane];
-        warp_offer(list, cnt, k, valid, e);
-    }
-}
-
-// First merge level: CTA b folds lists [32 b, 32 b + 32) into out[b]; each
-// warp takes two lists, whose counts it loads together.
-__global__ void __launch_bounds__(kMergeBlock) topk_reduce_kernel(TopkArgs a, int blocks) {
-    __shared__ TopkEntry lists[kMergeWarps * kMaxTopK];
-    __shared__ int counts[kMergeWarps];
+// One merge level: CTA b folds lists [kFan b, kFan b + kFan) of src into
+// dst[b]; with `final` (one CTA) the incoming state joins as one more list
+// and the result is written to the state.
+constexpr int kFan = 16;
+__global__ void __launch_bounds__(kMergeBlock) topk_level_kernel(TopkArgs a, const TopkEntry* src,
+                                                                 const int32_t* src_count, int nsrc,
+                                                                 TopkEntry* dst, int32_t* dst_count,
+                                                                 int final_level) {
+    static_assert(kMergeWarps > kFan, "one warp per list plus one for the state");
+    __shared__ TopkEntry lists[(kFan + 1) * kMaxTopK];
+    __shared__ TopkEntry tmp[((kFan + 2) / 2) * kMaxTopK];
+    __shared__ int counts[kFan + 1], tmp_counts[(kFan + 2) / 2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int k = state_k(a.state);
-    int cnt = 0;
-    TopkEntry* list = lists + warp * kMaxTopK;
-    const int l0 = blockIdx.x * 32 + warp, l1 = l0 + kMergeWarps;
-    const int c0 = l0 < blocks ? a.scratch_count[l0] : 0;
-    const int c1 = l1 < blocks ? a.scratch_count[l1] : 0;
-    offer_list(a.scratch + (size_t)l0 * kMaxTopK, c0, list, cnt, k);
-    offer_list(a.scratch + (size_t)l1 * kMaxTopK, c1, list, cnt, k);
-    if (lane == 0) counts[warp] = cnt;
-    cta_merge_lists(lists, counts, k, kMergeWarps, cnt, a.scratch2 + (size_t)blockIdx.x * kMaxTopK,
-                    a.scratch2_count + blockIdx.x);
-}
-
-// Last merge level: one CTA folds `blocks` lists and the incoming state.
-__global__ void __launch_bounds__(kMergeBlock) topk_merge_kernel(TopkArgs a, const TopkEntry* src,
-                                                                 const int32_t* src_count, int blocks) {
-    __shared__ TopkEntry lists[kMergeWarps * kMaxTopK];
-    __shared__ int counts[kMergeWarps];
-    __shared__ TopkEntry merged[kMaxTopK];
-    __shared__ int32_t merged_count;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int k = state_k(a.state);
-    int cnt = 0;
-    TopkEntry* list = lists + warp * kMaxTopK;
-    if (warp == 0) {
-        // the incoming state
-        const int c0 = min(max(a.state->count, 0), k);
-        for (int b = 0; b < c0; b += 32) {
-            const bool valid = b + lane < c0;
+    // warp w stages list kFan b + w (and warp kFan the state, on the last level)
+    if (warp < kFan) {
+        const int l = blockIdx.x * kFan + warp;
+        const int c = l < nsrc ? min(src_count[l], k) : 0;
+        for (int i = lane; i < c; i += 32) lists[warp * kMaxTopK + i] = src[(size_t)l * kMaxTopK + i];
+        if (lane == 0) counts[warp] = c;
+    } else if (warp == kFan) {
+        const int c = final_level ? min(max(a.state->count, 0), k) : 0;
+        for (int i = lane; i < c; i += 32) {
             TopkEntry e;
-            if (valid) {
-                e.idx = a.state->idx[b + lane];
-                e.T = a.state->T[b + lane];
-                e.nM = a.state->nM[b + lane];
-                e.pad = 0;
-            }
-            warp_offer(list, cnt, k, valid, e);
+            e.idx = a.state->idx[i];
+            e.T = a.state->T[i];
+            e.nM = a.state->nM[i];
+            e.pad = 0;
+            lists[kFan * kMaxTopK + i] = e;
         }
+        if (lane == 0) counts[kFan] = c;
     }
-    for (int l = warp; l < blocks; l += kMergeWarps) offer_list(src + (size_t)l * kMaxTopK, src_count[l], list, cnt, k);
-    if (lane == 0) counts[warp] = cnt;
-    cta_merge_lists(lists, counts, k, kMergeWarps, cnt, merged, &merged_count);
-    __syncthreads();
-    for (int p = threadIdx.x; p < kMaxTopK; p += blockDim.x) {
-        const bool live = p < merged_count;
-        a.state->idx[p] = live ? merged[p].idx : -1;
-        a.state->T[p] = live ? merged[p].T : -1;
-        a.state->nM[p] = live ? merged[p].nM : 0;
+    cta_tree_merge(lists, counts, tmp, tmp_counts, kFan + 1, k);
+    const int cnt = counts[0];
+    if (final_level) {
+        for (int p = threadIdx.x; p < kMaxTopK; p += blockDim.x) {
+            const bool live = p < cnt;
+            a.state->idx[p] = live ? lists[p].idx : -1;
+            a.state->T[p] = live ? lists[p].T : -1;
+            a.state->nM[p] = live ? lists[p].nM : 0;
+        }
+        if (threadIdx.x == 0) a.state->count = cnt;
+    } else {
+        for (int p = threadIdx.x; p < cnt; p += blockDim.x) dst[(size_t)blockIdx.x * kMaxTopK + p] = lists[p];
+        if (threadIdx.x == 0) dst_count[blockIdx.x] = cnt;
     }
-    if (threadIdx.x == 0) a.state->count = merged_count;
 }
 
-// Merge `blocks` per-CTA lists of a.scratch into *a.state: directly, or
-// through one reduction level of 32 lists per CTA when there are many.
+// Fold `blocks` per-CTA lists of a.scratch (at most kFan * kFan) into
+// *a.state: directly when there are few, else through one level into
+// a.scratch2 first.
 cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st) {
-    if (blocks <= 2 * kMergeWarps) {
-        topk_merge_kernel<<<1, kMergeBlock, 0, st>>>(a, a.scratch, a.scratch_count, blocks);
+    if (blocks > kFan * kFan) return cudaErrorInvalidValue;
+    if (blocks > kFan) {
+        const int m1 = (blocks + kFan - 1) / kFan;
+        topk_level_kernel<<<m1, kMergeBlock, 0, st>>>(a, a.scratch, a.scratch_count, blocks, a.scratch2,
+                                                      a.scratch2_count, 0);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        topk_level_kernel<<<1, kMergeBlock, 0, st>>>(a, a.scratch2, a.scratch2_count, m1, nullptr, nullptr, 1);
         return cudaGetLastError();
     }
-    const int m1 = (blocks + 31) / 32;
-    topk_reduce_kernel<<<m1, kMergeBlock, 0, st>>>(a, blocks);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    topk_merge_kernel<<<1, kMergeBlock, 0, st>>>(a, a.scratch2, a.scratch2_count, m1);
+    topk_level_kernel<<<1, kMergeBlock, 0, st>>>(a, a.scratch, a.scratch_count, blocks, nullptr, nullptr, 1);
     return cudaGetLastError();
 }
 
@@ -164,9 +150,10 @@ __global__ void topk_reset_kernel(heddle_topk_state* s, int k) {
 
 cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
-    const int64_t per_block = (int64_t)kTopkBlock * 8;  // at least 8 candidates per thread
-    int grid = (int)std::min<int64_t>((a.n + per_block - 1) / per_block, (int64_t)2 * num_sms);
+    const int64_t per_block = (int64_t)kTopkBlock * 16;  // at least 16 candidates per thread
+    int grid = (int)std::min<int64_t>((a.n + per_block - 1) / per_block, (int64_t)kFan * kFan);
     grid = std::max(1, std::min(grid, a.max_blocks));
+    (void)num_sms;
     topk_block_kernel<false><<<grid, kTopkBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
@@ -175,9 +162,10 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st) {
 
 cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st) {
     if (n <= 0) return cudaSuccess;
-    const int64_t per_block = (int64_t)kTopkBlock * 8;
-    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)2 * num_sms);
+    const int64_t per_block = (int64_t)kTopkBlock * 16;
+    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)kFan * kFan);
     grid = std::max(1, std::min(grid, a.max_blocks));
+    (void)num_sms;
     topk_block_kernel<true><<<grid, kTopkBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
