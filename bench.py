@@ -47,7 +47,28 @@ WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 10
 # (4): 29.
 OPS_PER_UNIT = {1: 16, 2: 29}
 SEARCH_NAMES = {1: "general interval search", 2: "equal-layer closed form"}
+SEARCH_KERNELS = {1: "search_kernel (general interval search)",
+                  2: "eq_search_kernel (equal-layer closed form)"}
 SMS, LANES_PER_SM = 152, 128  # 4 SM sub-partitions x 32 lanes issue per clock
+
+# DRAM bytes (read + write) of one search launch on a 1e6-candidate batch of
+# the stress workload, from an ncu capture, with the SHA-256 of the kernel
+# sources it was taken on; reported as null once those sources change.
+TRAFFIC = {}
+TRAFFIC_SOURCES = {1: ["heddle_price.cu", "heddle_internal.cuh"],
+                   2: ["heddle_eqsearch.cu", "heddle_internal.cuh"]}
+
+
+def traffic_per_launch(search, batch):
+    import hashlib
+    rec = TRAFFIC.get(search)
+    if rec is None or batch != rec["batch"]:
+        return None
+    hs = hashlib.sha256()
+    for f in TRAFFIC_SOURCES[search]:
+        with open(os.path.join(ROOT, "paper_2609_34244_gb300", "csrc", f), "rb") as fh:
+            hs.update(fh.read())
+    return rec["bytes"] if hs.hexdigest() == rec["sha256"] else None
 
 
 def load_peaks():
@@ -202,17 +223,12 @@ def main():
                  h.make_results(res, lo, min(n, lo + batch))) for lo in range(0, n, batch)]
     n_batches = len(cbatches)
 
-    def step(events=None):
+    def step():
         """One pass of the hot path: every batch priced and merged into the
-        running top-16 (heddle_price_topk: screen, search with the fused
-        block-level top-k, merge)."""
+        running top-16 (heddle_price_topk: screen, search, top-k merge)."""
         h.heddle_topk_reset(ctx, state, 16, stream)
-        for i, (c, r) in enumerate(cbatches):
-            if events is not None:
-                events[i][0].record(stream)
+        for c, r in cbatches:
             h.heddle_price_topk(ctx, c, r, state, stream)
-            if events is not None:
-                events[i][1].record(stream)
 
     search = h.heddle_get_search(ctx)
 
@@ -229,20 +245,22 @@ def main():
         step()
     torch.cuda.synchronize()
     shard.barrier(group)
-    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(n_batches)] for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # per-kernel device time: the library records events on `stream` around
+    # its screen, search and top-k launches of every batch
+    h.heddle_time_phases(ctx, True)
     with ClockSampler(local) as clk:
         torch.cuda.synchronize()
         t_start.record(stream)
-        for k in range(args.steps):
-            step(ev[k])
+        for _ in range(args.steps):
+            step()
         t_end.record(stream)
         torch.cuda.synchronize()
+    h.heddle_time_phases(ctx, False)
     shard.barrier(group)
     clocks = clk.summary()
     ms = t_start.elapsed_time(t_end)
-    price_ms = sum(a.elapsed_time(b) for row in ev for a, b in row)
+    phases = h.heddle_phase_times(ctx)
     ms_all = shard.max_over_ranks(group, ms)
     errors = h.heddle_device_errors(ctx)
     local_topk = h.read_topk_state(state)
@@ -255,22 +273,23 @@ def main():
         gwork = count_work()
         for _ in range(2):
             step()
-        gev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                for _ in range(n_batches)] for _ in range(2)]
         torch.cuda.synchronize()
         g0, g1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        h.heddle_time_phases(ctx, True)
         g0.record(stream)
-        for k in range(2):
-            step(gev[k])
+        for _ in range(2):
+            step()
         g1.record(stream)
         torch.cuda.synchronize()
+        h.heddle_time_phases(ctx, False)
         gms = g0.elapsed_time(g1) / 2
-        gprice = sum(a.elapsed_time(b) for row in gev for a, b in row) / 2
+        gph = h.heddle_phase_times(ctx)
+        gsearch_ms = gph["search"][0] / 2
         gtopk = h.read_topk_state(state)
-        general = {"value": n / (gms / 1e3), "ms_per_step": gms, "price_ms_per_step": gprice,
+        general = {"value": n / (gms / 1e3), "ms_per_step": gms, "search_ms_per_step": gsearch_ms,
                    "checks_per_candidate": gwork["checks"] / n,
                    "probes_per_searched": gwork["probes"] / max(1, gwork["priced"]),
-                   "alu_frac": gwork["checks"] * OPS_PER_UNIT[1] / (gprice / 1e3) / 1e12 /
+                   "alu_frac": gwork["checks"] * OPS_PER_UNIT[1] / (gsearch_ms / 1e3) / 1e12 /
                    (SMS * LANES_PER_SM * 2070.0 * 1e6 / 1e12),
                    "same_topk": gtopk["idx"].tolist() == local_topk["idx"].tolist()}
         h.heddle_set_search(ctx, h.SEARCH_AUTO)
@@ -298,7 +317,12 @@ def main():
     value = n * world * args.steps / (ms_all / 1e3)
     ops_step = work["checks"] * OPS_PER_UNIT[search]
     peak_tops = SMS * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
-    achieved_tops = ops_step * args.steps / (price_ms / 1e3) / 1e12
+    # the dominant kernel is the search: its average launch duration from
+    # the events around it, its algorithmic ops per launch from the counters
+    search_ms, search_launches = phases["search"]
+    search_us = 1e3 * search_ms / max(1, search_launches)
+    achieved_tops = ops_step * args.steps / (search_ms / 1e3) / 1e12
+    total_phase_ms = sum(v[0] for v in phases.values())
     cpu = None
     if not args.no_cpu_baseline:
         rate, ncpu, used, dt = oracle_rate(w, args.cpu_seconds, os.cpu_count() or 1)
@@ -312,18 +336,22 @@ def main():
                    "parallelism": "candidate shards, dp%d" % world,
                    "l2": "inputs larger than L2 (%.0f MB of candidates per step per GPU)" % (h2d / 1e6),
                    "seed": "rank"},
-        # per step: the top-k reset kernel, then per batch the screen, the
-        # search and the merge (the two cudaMemsetAsync calls are not kernels)
-        "gpu_launches": args.steps * (1 + 3 * n_batches) * world,
+        # per step the top-k reset kernel, plus the kernels the library
+        # counted in the timed steps (screen, search, top-k block and levels)
+        "gpu_launches": (args.steps + sum(v[1] for v in phases.values())) * world,
         "per_candidate_ns": 1e6 * ms_all / args.steps / n,
         "roofline": {"bound": "alu", "achieved": achieved_tops, "peak": peak_tops, "unit": "Tops/s",
-                     "frac": achieved_tops / peak_tops, "traffic": None,
-                     "kernel": "heddle_price_topk (screen + search + merge)", "search": SEARCH_NAMES[search],
+                     "frac": achieved_tops / peak_tops,
+                     "traffic": traffic_per_launch(search, batch),
+                     "kernel": SEARCH_KERNELS[search], "search": SEARCH_NAMES[search],
+                     "launch_us": search_us, "launches_timed": search_launches,
                      "ops_per_unit": OPS_PER_UNIT[search],
+                     "ops_per_launch": ops_step / n_batches,
                      "units_per_candidate": work["checks"] / n,
                      "probes_per_searched": work["probes"] / max(1, work["priced"]),
                      "searched_fraction": work["priced"] / n,
-                     "price_ms_per_step": price_ms / args.steps,
+                     "phases_us_per_launch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in phases.items()},
+                     "phase_share": {k: v[0] / total_phase_ms for k, v in phases.items()},
                      "peak_basis": "%s: %d SMs x %d lanes x %.0f MHz (%s sm_max)" % (
                          "issue slots", SMS, LANES_PER_SM, float(peaks.get("sm_max_mhz", 2070.0)), peak_kind)},
         "clocks": clocks,

@@ -317,6 +317,28 @@ heddle_status heddle_get_search(heddle_ctx* ctx, int32_t* in_use);
 heddle_status heddle_count_next(heddle_ctx* ctx, int32_t enable);
 heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);
 
+/* Device time of each phase of the pricing calls, measured with CUDA events
+ * on the caller's stream.  The paper has no counterpart: it is how the
+ * roofline report times its kernels without a profiler.  While enabled
+ * (heddle_time_phases(ctx, 1); no stream capture meanwhile, the events are
+ * created on demand), every chunk that heddle_price_candidates,
+ * heddle_price_topk or heddle_price_topk_host prices records four events:
+ * before the screen kernel, between the screen and the search kernel,
+ * after the search kernel and, when the call merges a top-k, after the
+ * top-k kernels.  heddle_phase_times synchronises on them and returns, per
+ * phase (SCREEN, SEARCH, TOPK), the summed elapsed milliseconds and the
+ * number of kernels launched in it (one screen and one search kernel per
+ * chunk; two or three top-k kernels), then forgets them.  The events add no work to the
+ * kernels; enabling or disabling changes no result.  Errors: E_ARG,
+ * E_CUDA. */
+#define HEDDLE_PHASE_SCREEN 0
+#define HEDDLE_PHASE_SEARCH 1
+#define HEDDLE_PHASE_TOPK 2
+#define HEDDLE_N_PHASES 3
+heddle_status heddle_time_phases(heddle_ctx* ctx, int32_t enable);
+heddle_status heddle_phase_times(heddle_ctx* ctx, double ms[HEDDLE_N_PHASES],
+                                 int64_t launches[HEDDLE_N_PHASES]);
+
 #ifdef __cplusplus
 }
 #endif

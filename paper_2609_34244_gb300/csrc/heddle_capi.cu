@@ -67,6 +67,16 @@ struct heddle_ctx {
     uint8_t* st_status[2] = {nullptr, nullptr};
     uint8_t* st_bounds[2] = {nullptr, nullptr};
     heddle_topk_state* d_state = nullptr;
+    // phase timing: four events per priced chunk (start, after the screen,
+    // after the search, after the top-k), recorded while time_phases is set
+    bool time_phases = false;
+    std::vector<cudaEvent_t> ev_pool;
+    struct PhaseRec {
+        cudaEvent_t e[4];
+        bool topk;
+        int64_t launches[3];
+    };
+    std::vector<PhaseRec> phase_recs;
 };
 
 namespace {
@@ -309,6 +319,9 @@ void heddle_destroy(heddle_ctx* x) {
         if (x->ev_free[b]) cudaEventDestroy(x->ev_free[b]);
     }
     cudaFree(x->d_state);
+    for (auto& r : x->phase_recs)
+        for (cudaEvent_t ev : r.e) x->ev_pool.push_back(ev);
+    for (cudaEvent_t ev : x->ev_pool) cudaEventDestroy(ev);
     if (x->s_h2d) cudaStreamDestroy(x->s_h2d);
     if (x->s_d2h) cudaStreamDestroy(x->s_d2h);
     delete x;
@@ -399,6 +412,20 @@ hd::TopkArgs topk_args(heddle_ctx* x, heddle_topk_state* state) {
     return a;
 }
 
+// Four timing events for one chunk, from the pool (created on demand).
+heddle_status take_phase_rec(heddle_ctx* x, heddle_ctx::PhaseRec* rec) {
+    for (int i = 0; i < 4; ++i) {
+        if (x->ev_pool.empty()) {
+            cudaEvent_t ev;
+            CU(cudaEventCreate(&ev));
+            x->ev_pool.push_back(ev);
+        }
+        rec->e[i] = x->ev_pool.back();
+        x->ev_pool.pop_back();
+    }
+    return HEDDLE_OK;
+}
+
 // Price cands into r; with a state, run the top-k over each chunk's searched
 // candidates (the only ones that can be OK) and merge them into *state.
 heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
@@ -444,7 +471,17 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
         a.ndp = r->n_dp + lo;
         a.status = r->status + lo;
         a.bounds = r->bounds ? r->bounds + lo : nullptr;
-        CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream));
+        heddle_ctx::PhaseRec rec{};
+        if (x->time_phases) {
+            if ((st = take_phase_rec(x, &rec)) != HEDDLE_OK) return st;
+            rec.topk = state != nullptr;
+            x->phase_recs.push_back(rec);
+            CU(cudaEventRecord(rec.e[0], (cudaStream_t)stream));
+        }
+        int64_t* nl = x->time_phases ? x->phase_recs.back().launches : nullptr;
+        CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream, x->time_phases ? rec.e[1] : nullptr,
+                            nl));
+        if (x->time_phases) CU(cudaEventRecord(rec.e[2], (cudaStream_t)stream));
         if (state) {
             // top-k over the searched candidates of this chunk only
             hd::TopkArgs m = topk_args(x, state);
@@ -454,7 +491,9 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
             m.wl_T = x->d_wl_T;
             m.wl_nM = x->d_wl_nM;
             m.wl_cap = hd::kWorklistCap;
-            CU(hd::launch_topk_worklist(m, nb, x->num_sms, (cudaStream_t)stream));
+            CU(hd::launch_topk_worklist(m, nb, x->num_sms, (cudaStream_t)stream,
+                                        nl ? nl + 2 : nullptr));
+            if (x->time_phases) CU(cudaEventRecord(rec.e[3], (cudaStream_t)stream));
         }
     }
     return ok(x);
@@ -660,6 +699,37 @@ heddle_status heddle_count_next(heddle_ctx* x, int32_t enable) {
     if (!x) return HEDDLE_E_ARG;
     x->count_next = enable != 0;
     return ok(x);
+}
+
+heddle_status heddle_time_phases(heddle_ctx* x, int32_t enable) {
+    if (!x) return HEDDLE_E_ARG;
+    x->time_phases = enable != 0;
+    return ok(x);
+}
+
+heddle_status heddle_phase_times(heddle_ctx* x, double ms[HEDDLE_N_PHASES], int64_t launches[HEDDLE_N_PHASES]) {
+    if (!x || !ms || !launches) return x ? fail(x, HEDDLE_E_ARG, "null output") : HEDDLE_E_ARG;
+    DeviceGuard dg(x->device);
+    for (int p = 0; p < HEDDLE_N_PHASES; ++p) {
+        ms[p] = 0.0;
+        launches[p] = 0;
+    }
+    heddle_status st = HEDDLE_OK;
+    for (auto& r : x->phase_recs) {
+        const int last = r.topk ? 3 : 2;
+        cudaError_t e = cudaEventSynchronize(r.e[last]);
+        for (int p = 0; p < last && e == cudaSuccess; ++p) {
+            float t = 0.f;
+            e = cudaEventElapsedTime(&t, r.e[p], r.e[p + 1]);
+            ms[p] += t;
+            launches[p] += r.launches[p];
+        }
+        if (e != cudaSuccess && st == HEDDLE_OK)
+            st = fail(x, HEDDLE_E_CUDA, "phase timing: %s", cudaGetErrorString(e));
+        for (cudaEvent_t ev : r.e) x->ev_pool.push_back(ev);
+    }
+    x->phase_recs.clear();
+    return st == HEDDLE_OK ? ok(x) : st;
 }
 
 heddle_status heddle_work_counters(heddle_ctx* x, uint64_t out[3]) {

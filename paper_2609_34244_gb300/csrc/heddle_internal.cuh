@@ -128,7 +128,10 @@ struct PriceArgs {
     uint32_t* wl_nM;
 };
 // Prices candidates [0, a.n) with a.n <= a.wl_cap: screen, then search.
-cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st);
+// `mid` (nullable) is recorded on st between the two; `launches` (nullable)
+// gains the kernels launched: [0] screen, [1] search.
+cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid = nullptr,
+                         int64_t* launches = nullptr);
 // The equal-layer search over the worklist the screen produced.
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
@@ -156,10 +159,12 @@ struct TopkArgs {
     TopkEntry* scratch2;
     int32_t* scratch2_count;
 };
-cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st);
+// `launches` (nullable) gains the number of kernels launched.
+cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t* launches = nullptr);
 // Top-k of the searched candidates of a priced chunk (a.wl_*), merged into
 // *a.state; `n` bounds the worklist length (the chunk size).
-cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st);
+cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st,
+                                 int64_t* launches = nullptr);
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st);
 
 }  // namespace hd

@@ -641,7 +641,7 @@ cudaError_t launch_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
 
 }  // namespace
 
-cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid, int64_t* launches) {
     if (a.n <= 0) return cudaSuccess;
     if (a.n > a.wl_cap) return cudaErrorInvalidValue;
     cudaError_t e = cudaMemsetAsync(a.wl_count, 0, sizeof(int32_t), st);
@@ -649,6 +649,11 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const int grid = (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * 8);
     screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (launches) {
+        launches[0] += 1;  // the screen now, the search below
+        launches[1] += 1;
+    }
+    if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
     if (a.uniform) return launch_eq_search(a, num_sms, st);
     return a.counters ? launch_search<true>(a, num_sms, st) : launch_search<false>(a, num_sms, st);
 }

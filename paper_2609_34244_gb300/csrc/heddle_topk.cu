@@ -119,8 +119,9 @@ __global__ void __launch_bounds__(kMergeBlock) topk_level_kernel(TopkArgs a, con
 // Fold `blocks` per-CTA lists of a.scratch (at most kFan * kFan) into
 // *a.state: directly when there are few, else through one level into
 // a.scratch2 first.
-cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st) {
+cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st, int64_t* launches) {
     if (blocks > kFan * kFan) return cudaErrorInvalidValue;
+    if (launches) *launches += blocks > kFan ? 2 : 1;
     if (blocks > kFan) {
         const int m1 = (blocks + kFan - 1) / kFan;
         topk_level_kernel<<<m1, kMergeBlock, 0, st>>>(a, a.scratch, a.scratch_count, blocks, a.scratch2,
@@ -148,7 +149,7 @@ __global__ void topk_reset_kernel(heddle_topk_state* s, int k) {
 
 }  // namespace
 
-cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t* launches) {
     if (a.n <= 0) return cudaSuccess;
     const int64_t per_block = (int64_t)kTopkBlock * 16;  // at least 16 candidates per thread
     int grid = (int)std::min<int64_t>((a.n + per_block - 1) / per_block, (int64_t)kFan * kFan);
@@ -157,10 +158,12 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st) {
     topk_block_kernel<false><<<grid, kTopkBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    return merge_lists(a, grid, st);
+    if (launches) *launches += 1;
+    return merge_lists(a, grid, st, launches);
 }
 
-cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st) {
+cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st,
+                                 int64_t* launches) {
     if (n <= 0) return cudaSuccess;
     const int64_t per_block = (int64_t)kTopkBlock * 16;
     int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)kFan * kFan);
@@ -169,7 +172,8 @@ cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cuda
     topk_block_kernel<true><<<grid, kTopkBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    return merge_lists(a, grid, st);
+    if (launches) *launches += 1;
+    return merge_lists(a, grid, st, launches);
 }
 
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st) {

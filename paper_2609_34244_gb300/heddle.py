@@ -64,7 +64,8 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
            "heddle_load_model", "heddle_price_candidates", "heddle_topk_reset", "heddle_topk",
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
            "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
-           "heddle_price_topk", "heddle_topk_noalloc"]
+           "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times"]
+PHASES = ("screen", "search", "topk")
 TOPK_NOALLOC_MAX_N = 4194304
 SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS = 0, 1, 2
 
@@ -98,6 +99,8 @@ def load_library(path: str = LIB_PATH):
         "heddle_work_counters": (i32, [p, C.POINTER(C.c_uint64)]),
         "heddle_set_search": (i32, [p, i32]),
         "heddle_get_search": (i32, [p, C.POINTER(C.c_int32)]),
+        "heddle_time_phases": (i32, [p, i32]),
+        "heddle_phase_times": (i32, [p, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(L, name)
@@ -264,6 +267,19 @@ def heddle_work_counters(ctx):
     out = (C.c_uint64 * 3)()
     _check(ctx, load_library().heddle_work_counters(ctx, out))
     return {"checks": int(out[0]), "probes": int(out[1]), "priced": int(out[2])}
+
+
+def heddle_time_phases(ctx, enable: bool = True):
+    _check(ctx, load_library().heddle_time_phases(ctx, int(bool(enable))))
+
+
+def heddle_phase_times(ctx):
+    """Summed device milliseconds and kernel launches per pricing phase
+    since the last read: {"screen": (ms, launches), "search": ..., "topk": ...}."""
+    ms = (C.c_double * len(PHASES))()
+    n = (C.c_int64 * len(PHASES))()
+    _check(ctx, load_library().heddle_phase_times(ctx, ms, n))
+    return {name: (float(ms[i]), int(n[i])) for i, name in enumerate(PHASES)}
 
 
 def heddle_set_search(ctx, mode: int):

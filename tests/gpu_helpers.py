@@ -9,11 +9,12 @@ import numpy as np
 
 
 def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False, search=None,
-              fused=False):
+              fused=False, phases=False):
     """Price on the GPU through the C ABI; returns numpy results, the top-k
     and (optionally) the work counters.  ``batch`` splits the candidates into
     consecutive launches merged into one top-k state; ``fused`` prices and
-    merges in one call (heddle_price_topk)."""
+    merges in one call (heddle_price_topk); ``phases`` times the pricing
+    phases with the library's events and returns them under "phases"."""
     import torch
     ctx = h.heddle_create(0)
     try:
@@ -30,6 +31,8 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
         out_bounds = np.zeros((33, n), np.uint8) if bounds else None
         if count:
             h.heddle_count_next(ctx, True)
+        if phases:
+            h.heddle_time_phases(ctx, True)
         for lo in range(0, max(n, 1), max(batch, 1)):
             hi = min(n, lo + batch)
             if hi <= lo:
@@ -54,6 +57,8 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
         out["search"] = h.heddle_get_search(ctx)
         if count:
             out["counters"] = h.heddle_work_counters(ctx)
+        if phases:
+            out["phases"] = h.heddle_phase_times(ctx)
         return out
     finally:
         h.heddle_destroy(ctx)
