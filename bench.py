@@ -35,17 +35,22 @@ WORKLOAD = "stress128"
 WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 1024 GPUs of 8 types in "
                  "nodes of 2/4/8, 1e7 candidates streamed as 10 device batches of 1e6, S<=32, "
                  "TP in {1,2,4,8}, M=256, global top-16")
-# Algorithmic integer work per counted unit of the search, in 32-bit lane
-# operations.  General search, one interval check: stage cost P[j]-P[i]+c
-# against B (int64 subtract, add, compare) and stage memory
-# (S[j]-S[i]) + f*(A[j]-A[i]) against the capacity (two int64 subtracts, one
-# multiply by a 32-bit count, one add, one compare): 8 int64 ops = 16.
-# Equal-layer search, one stage capacity min(m, floor((B-c)/q)): B-c (2),
+# Algorithmic integer work per counted unit, in 32-bit lane operations.
+# General search, unit = one interval check: stage cost P[j]-P[i]+c against
+# B (int64 subtract, add, compare) and stage memory (S[j]-S[i]) +
+# f*(A[j]-A[i]) against the capacity (two int64 subtracts, one multiply by a
+# 32-bit count, one add, one compare): 8 int64 ops = 16.
+# Equal-layer search, unit = one stage of a searched candidate, counted once
+# whatever the number of probes: the work of checking B* and evaluating the
+# plan.  One exact stage capacity min(m, floor((B-c)/q)) at B*: B-c (2),
 # x >= m*q (multiply 2, compare 2), the quotient estimate and its two
-# multiply-compare corrections (10), the running sum (1), the two snapping
-# values c + k*q (multiply-add 4) and c + (k+1)*q (4) with their max / min
-# (4): 29.
-OPS_PER_UNIT = {1: 16, 2: 29}
+# multiply-compare corrections (10), the running sum (1), the snapping
+# values c + k*q (4) and c + (k+1)*q (4) with their max / min (4): 29.
+# Evaluate: stage time (a_{s+1}-a_s)*q + c (4), its max and sum (4), the
+# boundary max(a_s + 1, L - suffix) with the running count (4), the
+# stage's gradient bytes (2) and bandwidth (2), the exact ratio comparison
+# of two 64x64->128-bit products (20): 36.  Together 65.
+OPS_PER_UNIT = {1: 16, 2: 65}
 SEARCH_NAMES = {1: "general interval search", 2: "equal-layer closed form"}
 SEARCH_KERNELS = {1: "search_kernel (general interval search)",
                   2: "eq_search_kernel (equal-layer closed form)"}

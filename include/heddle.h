@@ -310,9 +310,10 @@ heddle_status heddle_get_search(heddle_ctx* ctx, int32_t* in_use);
 /* Work counters of the next heddle_price_candidates call on ctx, for the
  * roofline report: when enabled, that call runs the counting variant of the
  * pricing kernel and accumulates, in device memory owned by ctx,
- * [0] interval checks evaluated (general search) or stage capacities
- * evaluated (equal-layer search), [1] feasibility probes, [2] candidates
- * that reached the search.  heddle_work_counters(ctx, out) copies them out
+ * [0] interval checks evaluated (general search) or stages of the
+ * candidates that reached the search, each counted once (equal-layer
+ * search), [1] exact feasibility probes, [2] candidates that reached the
+ * search.  heddle_work_counters(ctx, out) copies them out
  * (synchronous) and resets them. */
 heddle_status heddle_count_next(heddle_ctx* ctx, int32_t enable);
 heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);

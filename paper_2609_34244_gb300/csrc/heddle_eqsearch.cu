@@ -7,27 +7,35 @@
 //     cap_s(B) = min(m_s, floor((B - c_s) / q_s))
 // layers within bound B (m_s: the longest run of layers that fits the
 // stage's memory, c_s: its P2P).  A split with every stage time <= B exists
-// iff every cap_s >= 1 and sum_s cap_s >= L, so a probe costs O(S).
-// B* >= max_s (c_s + q_s) (every stage holds a layer), which starts the
-// bracket; the first probe is the continuous balance
-// sum_s (B - c_s) / q_s = L, later ones interpolate the cap count between
-// the bracket's probes (a Newton step on the count while one side is
-// missing), falling back to bisection.  Every probe snaps the bracket to
-// exact breakpoints: a feasible probe keeps the same caps down to
-// max_s (c_s + cap_s q_s), an infeasible one up to the smallest
-// c_s + (cap_s + 1) q_s of a stage that can still grow, so the search ends
-// on B* itself with the caps of its last feasible probe, which hold at B*.
-// The componentwise smallest split -- hence the lexicographically smallest
-// -- is then a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
+// iff every cap_s >= 1 and sum_s cap_s >= L, so a probe costs O(S), and
+// B* is the smallest such B -- a breakpoint c_s + k q_s of some stage.
 //
-// Layout: a few small tables (per-layer cost and its reciprocal per (type,
-// degree), P2P, gradient-byte prefix, NIC, memory runs) are copied to shared
-// memory once per CTA; every candidate's stages are packed once into 32-bit
-// words (cost index | P2P index | memory run) held in shared memory
-// interleaved by thread, so probes read one conflict-free word per stage.
-// Each CTA takes 256 worklist entries at a time and sorts them by S
-// (counting sort) so that the lanes of a warp run stage loops of equal
-// length.
+// First guess, in float only: the continuous balance
+// sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2 (the
+// floors lose half a layer per such stage on average), solved by Newton
+// steps from the unsaturated balance.  Exact probes then decide and snap
+// the bracket to breakpoints: a feasible probe keeps its caps down to
+// hi = max_s (c_s + cap_s q_s); an infeasible one keeps them up to the next
+// breakpoint lo = min_s c_s + (cap_s + 1) q_s.  Two exact stop rules end
+// most searches after one probe:
+//   feasible, and dropping the stages that attain hi (each loses one layer
+//   just below hi) leaves fewer than L layers or an empty stage -> B* = hi;
+//   infeasible, and at lo every stage holds a layer and the stages that
+//   attain lo (each gains exactly one) bring the total to L -> B* = lo.
+// Otherwise the next bound interpolates the cap count between the bracket's
+// probes (a Newton step while one side is missing), else bisects.  The caps
+// at B* give the componentwise smallest split -- hence the lexicographically
+// smallest -- a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
+//
+// Scheduling: each CTA takes 256 worklist entries at a time, counting-sorted
+// by S so that the lanes of a warp run stage loops of equal length.  Every
+// thread packs its candidate's stages once into 32-bit words (cost index |
+// P2P index | memory run) held in shared memory interleaved by thread, runs
+// the float guess and one exact probe; the few searches still open are
+// queued in shared memory and finished by the first threads of the CTA
+// (reading the owner's words), so that they fill whole warps instead of
+// holding every warp that has one; then every thread evaluates its own
+// candidate.
 
 #include <algorithm>
 
@@ -42,8 +50,22 @@ constexpr int kEqBlock = 256;
 constexpr int kZeroP2P = 128;  // a zero entry after the 8 x 8 x 2 P2P table
 constexpr int kMaxIters = 256;
 
+constexpr int kTailCap = 64;  // open searches queued per slice
+
+// State of one threshold search.
+struct Search {
+    int64_t lo, hi, B;  // B* lies in [lo, hi]; B is the next bound to probe
+    int64_t Blo, Bhi;   // last infeasible / feasible bound probed (-1: none)
+    int64_t fhi;        // hi of the last feasible probe: its caps hold at fhi
+    int32_t clo, chi;   // layer counts of those probes
+    int16_t fset, wset; // cap set of the last feasible probe (-1: none), set written next
+    int16_t owner, S;   // thread whose shared-memory columns hold the stages; depth
+    int32_t probes;
+    int32_t pad;
+};
+
 struct EqLayout {
-    uint32_t q, rq, p2p, inter, maxn, PB, win, sw, caps, bytes;
+    uint32_t q, rq, qf, p2p, cf, inter, maxn, PB, win, sw, caps, tail, bstar, bytes;
 };
 
 __host__ __device__ inline uint32_t al16(uint32_t x) { return (x + 15u) & ~15u; }
@@ -53,13 +75,17 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
     uint32_t o = 0;
     e.q = o;     o = al16(o + 8 * 32);             // int64 [j * 8 + g]
     e.rq = o;    o = al16(o + 4 * 32);             // float 1 / q
+    e.qf = o;    o = al16(o + 4 * 32);             // float q
     e.p2p = o;   o = al16(o + 8 * 129);            // int64 [(g * 8 + h) * 2 + same], [128] = 0
+    e.cf = o;    o = al16(o + 4 * 129);            // float P2P
     e.inter = o; o = al16(o + 8 * 8);              // int64 [g]
     e.maxn = o;  o = al16(o + 4 * 8);              // int32 [g]
     e.PB = o;    o = al16(o + 8 * (L + 1));        // int64 gradient-byte prefix
     e.win = o;   o = al16(o + 8 * 4 * 33);         // uint8 [(g * 4 + j) * 33 + f]
     e.sw = o;    o = al16(o + 4 * kMaxStages * kEqBlock);  // uint32 [s][thread]
     e.caps = o;  o = al16(o + 2 * (kMaxStages + 1) * kEqBlock);  // uint8 [2][s][thread]
+    e.tail = o;  o = al16(o + sizeof(struct Search) * kTailCap);    // open searches
+    e.bstar = o; o = al16(o + 8 * kEqBlock);                         // int64 B* per thread
     e.bytes = o;
     return e;
 }
@@ -67,13 +93,15 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
 struct EqTabs {
     const int64_t* q;
     const float* rq;
+    const float* qf;
     const int64_t* p2p;
+    const float* cf;
     const int64_t* inter;
     const int32_t* maxn;
     const int64_t* PB;
     const uint8_t* win;
-    uint32_t* sw;   // this thread's stage words, element s at [s * kEqBlock]
-    uint8_t* caps;  // this thread's caps, two sets, set b element s at [(b * 33 + s) * kEqBlock]
+    uint32_t* sw;   // stage words of thread 0; thread o's element s at [s * kEqBlock + o]
+    uint8_t* caps;  // caps of thread 0, two sets; thread o's set b element s at [(b * 33 + s) * kEqBlock + o]
     int L;
 };
 
@@ -119,38 +147,150 @@ __device__ __forceinline__ Cap stage_cap(const EqTabs& t, uint32_t w, int64_t B)
     return r;
 }
 
-struct Snap {
-    int64_t hi, lo;  // snapping values
-    int tot;         // layers the stages hold (stages holding one or more)
-    float slope;     // growth of tot per unit of B: sum of 1/q over stages below their run
-    unsigned long long units;
+// Continuous count at Bf (float): sum_s min(m_s, (Bf - c_s) / q_s), with
+// the slope sum 1/q_s and the number of stages below their run.
+__device__ float eq_count(const EqTabs& t, const uint32_t* sw, int S, float Bf, float& slope, int& below) {
+    float cnt = 0.f, sl = 0.f;
+    int nb = 0;
+    for (int s = 0; s < S; ++s) {
+        const uint32_t w = sw[s * kEqBlock];
+        const float rq = t.rq[w & 31];
+        const float m = (float)((w >> 13) & 255);
+        const float x = (Bf - t.cf[(w >> 5) & 255]) * rq;
+        if (rq == 0.f || x >= m) {
+            cnt += m;
+        } else {
+            cnt += x;
+            sl += rq;
+            ++nb;
+        }
+    }
+    slope = sl;
+    below = nb;
+    return cnt;
+}
+
+// Result of an exact probe at bound B.
+struct Probe {
+    int64_t hi;    // largest stage time c + k q over stages holding a layer
+    int64_t lo;    // next breakpoint above B: min c + (k + 1) q over stages below their run
+    int64_t zmax;  // largest c + q over stages holding no layer (-1: none)
+    int tot;       // layers the stages hold
+    int nhi, nlo;  // stages attaining hi / lo
+    bool hi1;      // a stage attaining hi holds a single layer
+    float slope;   // sum of 1/q over stages below their run
 };
 
-// Probe bound B; the caps go to cap set `set`.
-__device__ bool eq_probe(const EqTabs& t, int S, int64_t B, int set, Snap& sn) {
-    sn.hi = -1;
-    sn.lo = kInf;
-    sn.slope = 0.f;
-    int sum = 0;
-    bool ok = true;
-    uint8_t* caps = t.caps + set * (kMaxStages + 1) * kEqBlock;
+// Exact probe of bound B for the stages in column sw; caps to column caps.
+__device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, uint8_t* caps, int S, int64_t B, Probe& p) {
+    p.hi = -1;
+    p.lo = kInf;
+    p.zmax = -1;
+    p.tot = 0;
+    p.nhi = 0;
+    p.nlo = 0;
+    p.hi1 = false;
+    p.slope = 0.f;
     for (int s = 0; s < S; ++s) {
-        const uint32_t w = t.sw[s * kEqBlock];
+        const uint32_t w = sw[s * kEqBlock];
         const Cap r = stage_cap(t, w, B);
-        caps[s * kEqBlock] = (uint8_t)max(r.k, 0);
-        if (r.k < r.m) sn.slope += t.rq[w & 31];
-        if (r.k < 1) {
-            ok = false;
-            if (r.m >= 1) sn.lo = min(sn.lo, r.c + r.q);
+        const int k = max(r.k, 0);
+        caps[s * kEqBlock] = (uint8_t)k;
+        if (r.m < 1) {
+            p.zmax = kInf;  // never holds a layer
             continue;
         }
-        sum += r.k;
-        sn.hi = max(sn.hi, r.c + (int64_t)r.k * r.q);
-        if (r.k < r.m) sn.lo = min(sn.lo, r.c + (int64_t)(r.k + 1) * r.q);
+        if (k < r.m) {
+            p.slope += t.rq[w & 31];
+            const int64_t nb = r.c + (int64_t)(k + 1) * r.q;
+            if (nb < p.lo) {
+                p.lo = nb;
+                p.nlo = 1;
+            } else if (nb == p.lo) {
+                ++p.nlo;
+            }
+        }
+        if (k < 1) {
+            p.zmax = max(p.zmax, r.c + r.q);
+            continue;
+        }
+        p.tot += k;
+        const int64_t v = r.c + (int64_t)k * r.q;
+        if (v > p.hi) {
+            p.hi = v;
+            p.nhi = 1;
+            p.hi1 = k == 1;
+        } else if (v == p.hi) {
+            ++p.nhi;
+            p.hi1 |= k == 1;
+        }
     }
-    sn.units += S;
-    sn.tot = sum;
-    return ok && sum >= t.L;
+    return p.zmax < 0 && p.tot >= t.L;
+}
+
+__device__ __forceinline__ uint8_t* cap_set(const EqTabs& t, int owner, int set) {
+    return t.caps + set * (kMaxStages + 1) * kEqBlock + owner;
+}
+
+// One exact probe of search q at q.B and the bracket update; returns true
+// when B* = q.hi is known.
+__device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
+    const uint32_t* sw = t.sw + q.owner;
+    q.B = min(max(q.B, q.lo), q.hi - 1);
+    ++q.probes;
+    Probe p;
+    const bool feas = eq_probe(t, sw, cap_set(t, q.owner, q.wset), q.S, q.B, p);
+    if (feas) {
+        q.hi = p.hi;
+        q.Bhi = q.B;
+        q.chi = p.tot;
+        q.fset = q.wset;
+        q.fhi = p.hi;
+        q.wset ^= 1;
+        // just below hi every stage attaining hi loses a layer
+        if (p.tot - p.nhi < t.L || p.hi1) q.lo = q.hi;
+    } else {
+        q.lo = min(max(q.lo, p.lo), q.hi);
+        q.Blo = q.B;
+        q.clo = p.tot;
+        // at lo every stage attaining lo gains exactly one layer
+        if (p.zmax <= p.lo && p.tot + p.nlo >= t.L) q.hi = q.lo;
+    }
+    if (q.lo >= q.hi) return true;
+    // next bound: interpolate the cap count between the bracket's probes,
+    // else a Newton step, else bisect
+    float target;
+    if (q.Blo >= 0 && q.Bhi >= 0 && q.chi > q.clo) {
+        target = (float)q.Blo + ((float)t.L - 0.5f - (float)q.clo) / (float)(q.chi - q.clo) * (float)(q.Bhi - q.Blo);
+    } else if (p.slope > 0.f) {
+        target = feas ? (float)q.B - ceilf(((float)p.tot - (float)t.L + 0.5f) / p.slope)
+                      : (float)q.B + ceilf(((float)t.L - (float)p.tot) / p.slope);
+    } else {
+        target = -1.f;
+    }
+    q.B = (target >= (float)q.lo && target <= (float)(q.hi - 1)) ? (int64_t)target : q.lo + (q.hi - q.lo) / 2;
+    if (q.probes > kMaxIters) {
+        atomicOr(err, kErrSearchBound);
+        q.lo = q.hi;
+        return true;
+    }
+    return false;
+}
+
+// Finish search q: probe until B* is known, then make sure a cap set holds
+// the caps at B*.  Writes B* and the set to the owner's slots.
+__device__ void eq_finish(const EqTabs& t, Search& q, int64_t* bstar, uint8_t* bset, uint32_t* err) {
+    while (q.lo < q.hi)
+        if (eq_step(t, q, err)) break;
+    if (q.fset < 0 || q.fhi != q.hi) {
+        // B* was reached from below (or never probed): its caps
+        ++q.probes;
+        Probe p;
+        if (!eq_probe(t, t.sw + q.owner, cap_set(t, q.owner, q.wset), q.S, q.hi, p)) atomicOr(err, kErrInternal);
+        q.fset = q.wset;
+    }
+    bstar[q.owner] = q.hi;
+    bset[q.owner] = (uint8_t)q.fset;
 }
 
 template <bool kCount>
@@ -158,6 +298,8 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int bins[kMaxStages + 2];
     __shared__ uint16_t order[kEqBlock];
+    __shared__ uint8_t bset[kEqBlock];
+    __shared__ int tail_n;
     const Layout& y = a.lay;
     const int L = y.L;
     const EqLayout el = eq_layout(L);
@@ -165,7 +307,9 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     {
         int64_t* q = reinterpret_cast<int64_t*>(smem + el.q);
         float* rq = reinterpret_cast<float*>(smem + el.rq);
+        float* qf = reinterpret_cast<float*>(smem + el.qf);
         int64_t* p2p = reinterpret_cast<int64_t*>(smem + el.p2p);
+        float* cf = reinterpret_cast<float*>(smem + el.cf);
         int64_t* inter = reinterpret_cast<int64_t*>(smem + el.inter);
         int32_t* maxn = reinterpret_cast<int32_t*>(smem + el.maxn);
         int64_t* PB = reinterpret_cast<int64_t*>(smem + el.PB);
@@ -176,9 +320,13 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             const int64_t v = g < y.NT ? gP[(g * 4 + j) * (L + 1) + 1] - gP[(g * 4 + j) * (L + 1)] : 0;
             q[i] = v;
             rq[i] = v > 0 ? 1.0f / (float)v : 0.0f;
+            qf[i] = (float)v;
         }
-        for (int i = threadIdx.x; i < 129; i += blockDim.x)
-            p2p[i] = i < 128 ? reinterpret_cast<const int64_t*>(a.img + y.offP2P)[i] : 0;
+        for (int i = threadIdx.x; i < 129; i += blockDim.x) {
+            const int64_t v = i < 128 ? reinterpret_cast<const int64_t*>(a.img + y.offP2P)[i] : 0;
+            p2p[i] = v;
+            cf[i] = (float)v;
+        }
         for (int i = threadIdx.x; i < 8; i += blockDim.x) {
             inter[i] = reinterpret_cast<const int64_t*>(a.img + y.offInter)[i];
             maxn[i] = reinterpret_cast<const int32_t*>(a.img + y.offMaxN)[i];
@@ -191,18 +339,21 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     EqTabs t;
     t.q = reinterpret_cast<const int64_t*>(smem + el.q);
     t.rq = reinterpret_cast<const float*>(smem + el.rq);
+    t.qf = reinterpret_cast<const float*>(smem + el.qf);
     t.p2p = reinterpret_cast<const int64_t*>(smem + el.p2p);
+    t.cf = reinterpret_cast<const float*>(smem + el.cf);
     t.inter = reinterpret_cast<const int64_t*>(smem + el.inter);
     t.maxn = reinterpret_cast<const int32_t*>(smem + el.maxn);
     t.PB = reinterpret_cast<const int64_t*>(smem + el.PB);
     t.win = smem + el.win;
-    t.sw = reinterpret_cast<uint32_t*>(smem + el.sw) + threadIdx.x;
-    t.caps = smem + el.caps + threadIdx.x;
+    t.sw = reinterpret_cast<uint32_t*>(smem + el.sw);
+    t.caps = smem + el.caps;
     t.L = L;
+    Search* tail = reinterpret_cast<Search*>(smem + el.tail);
+    int64_t* bstar = reinterpret_cast<int64_t*>(smem + el.bstar);
+    uint32_t* mysw = t.sw + threadIdx.x;
 
-    Snap sn;
-    sn.units = 0;
-    unsigned long long probes = 0, searched = 0;
+    unsigned long long units = 0, probes = 0, searched = 0;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const int64_t count_r = (count + kEqBlock - 1) / kEqBlock * kEqBlock;
     const int64_t stride = (int64_t)gridDim.x * kEqBlock;
@@ -211,6 +362,7 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
         const int64_t p0 = base + threadIdx.x;
         const int s0 = p0 < count ? a.wl_S[p0] : 0;
         if (threadIdx.x < kMaxStages + 2) bins[threadIdx.x] = 0;
+        if (threadIdx.x == 0) tail_n = 0;
         __syncthreads();
         atomicAdd(&bins[s0], 1);
         __syncthreads();
@@ -226,93 +378,102 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
         order[atomicAdd(&bins[s0], 1)] = (uint16_t)threadIdx.x;
         __syncthreads();
         const int64_t p = base + order[threadIdx.x];
-        __syncthreads();  // bins and order are reused by the next slice
-        if (p >= count) continue;
+        const bool have = p < count;
 
-        const int64_t c = a.wl_idx[p];
-        const int S = a.wl_S[p];
-        const int M = a.wl_M[p];
-        const int64_t n = a.wl_n[p];
-        if (kCount) ++searched;
-        // pack the stages; feasible upper bound (every stage at its memory
-        // run, which the screen guarantees covers L), lower bound (every
-        // stage holds one layer) and the continuous balance as first probe
-        int64_t hi = 0, lo = 0;
-        float inv = 0.f, cw = 0.f;
-        int code = a.wl_code[p];
-        for (int s = 0; s < S; ++s) {
-            const bool last = s + 1 == S;
-            const int next = last ? 0 : a.wl_code[(int64_t)(s + 1) * a.wl_cap + p];
-            const uint32_t w = stage_word(code, next, last, min(S - s, M), t);
-            t.sw[s * kEqBlock] = w;
-            const int64_t q = t.q[w & 31], cc = t.p2p[(w >> 5) & 255];
-            const int m = (int)(w >> 13) & 255;
-            hi = max(hi, cc + (int64_t)m * q);
-            lo = max(lo, cc + q);
-            const float qf = (float)q + 0.5f;
-            inv += 1.0f / qf;
-            cw += (float)cc / qf;
-            code = next;
-        }
-        int64_t B = (int64_t)(((float)L + cw) / inv);
-        // bracket probes (bound, cap count) for the interpolation
-        int64_t Blo = -1, Bhi = -1;
-        int clo = 0, chi = 0;
-        int wset = 0, fset = -1;  // cap set written next / of the last feasible probe
-        int it = 0;
-        while (lo < hi) {
-            B = min(max(B, lo), hi - 1);
-            if (kCount) ++probes;
-            const bool feas = eq_probe(t, S, B, wset, sn);
-            if (feas) {
-                hi = sn.hi;
-                Bhi = B;
-                chi = sn.tot;
-                fset = wset;
-                wset ^= 1;
+        int S = 0, M = 0;
+        int64_t n = 0, c = 0;
+        if (have) {
+            c = a.wl_idx[p];
+            S = a.wl_S[p];
+            M = a.wl_M[p];
+            n = a.wl_n[p];
+            if (kCount) {
+                ++searched;
+                units += S;
+            }
+            // pack the stages; feasible upper bound (every stage at its
+            // memory run, which the screen guarantees covers L), lower bound
+            // (every stage holds one layer), unsaturated continuous balance
+            Search q;
+            q.lo = 0;
+            q.hi = 0;
+            float inv = 0.f, cw = 0.f;
+            int code = a.wl_code[p];
+            for (int s = 0; s < S; ++s) {
+                const bool last = s + 1 == S;
+                const int next = last ? 0 : a.wl_code[(int64_t)(s + 1) * a.wl_cap + p];
+                const uint32_t w = stage_word(code, next, last, min(S - s, M), t);
+                mysw[s * kEqBlock] = w;
+                const int64_t qq = t.q[w & 31], cc = t.p2p[(w >> 5) & 255];
+                const int m = (int)(w >> 13) & 255;
+                q.hi = max(q.hi, cc + (int64_t)m * qq);
+                q.lo = max(q.lo, cc + qq);
+                const float rq = t.rq[w & 31];
+                inv += rq;
+                cw += t.cf[(w >> 5) & 255] * rq;
+                code = next;
+            }
+            // first guess: Newton on the saturating continuous count
+            float Bf = fmaxf((float)q.lo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : (float)q.lo);
+            for (int it = 0; it < 8; ++it) {
+                float sl;
+                int below;
+                Bf = fminf(Bf, (float)q.hi);
+                const float cnt = eq_count(t, mysw, S, Bf, sl, below);
+                const float tgt = (float)L + 0.5f * (float)below;
+                if (cnt >= tgt - 0.25f || sl <= 0.f) break;
+                Bf += (tgt - cnt) / sl;
+            }
+            q.B = (int64_t)fminf(Bf, (float)q.hi);
+            q.Blo = q.Bhi = q.fhi = -1;
+            q.clo = q.chi = 0;
+            q.fset = -1;
+            q.wset = 0;
+            q.owner = (int16_t)threadIdx.x;
+            q.S = (int16_t)S;
+            q.probes = 0;
+            q.pad = 0;
+            // one exact probe here; open searches go to the CTA's queue
+            bool done = q.lo >= q.hi || eq_step(t, q, a.err);
+            if (done && q.fset >= 0 && q.fhi == q.hi) {
+                bstar[threadIdx.x] = q.hi;
+                bset[threadIdx.x] = (uint8_t)q.fset;
             } else {
-                lo = max(lo, sn.lo);
-                Blo = B;
-                clo = sn.tot;
+                const int slot = atomicAdd(&tail_n, 1);
+                if (slot < kTailCap) {
+                    tail[slot] = q;
+                    q.probes = 0;  // counted by the thread that finishes it
+                } else {
+                    eq_finish(t, q, bstar, bset, a.err);
+                }
             }
-            if (lo >= hi) break;
-            // next bound: interpolate the cap count between the bracket's
-            // probes, else a Newton step, else bisect
-            float target;
-            if (Blo >= 0 && Bhi >= 0 && chi > clo) {
-                target = (float)Blo + ((float)L - 0.5f - (float)clo) / (float)(chi - clo) * (float)(Bhi - Blo);
-            } else if (sn.slope > 0.f) {
-                target = feas ? (float)B - ceilf(((float)sn.tot - (float)L + 0.5f) / sn.slope)
-                              : (float)B + ceilf(((float)L - (float)sn.tot) / sn.slope);
-            } else {
-                target = -1.f;
-            }
-            B = (target >= (float)lo && target <= (float)(hi - 1)) ? (int64_t)target : lo + (hi - lo) / 2;
-            if (++it > kMaxIters) {
-                atomicOr(a.err, kErrSearchBound);
-                break;
-            }
+            if (kCount) probes += q.probes;
         }
-        const int64_t Bstar = hi;
-        if (fset < 0) {
-            // B* is the initial bound, never probed: its caps
-            if (kCount) ++probes;
-            if (!eq_probe(t, S, Bstar, 0, sn)) atomicOr(a.err, kErrInternal);
-            fset = 0;
+        __syncthreads();
+        // ---- the open searches, one per thread
+        const int nt = min(tail_n, kTailCap);
+        for (int i = threadIdx.x; i < nt; i += kEqBlock) {
+            Search q = tail[i];
+            eq_finish(t, q, bstar, bset, a.err);
+            if (kCount) probes += q.probes;
         }
-        const uint8_t* caps = t.caps + fset * (kMaxStages + 1) * kEqBlock;
-        int total = 0;
-        for (int s = 0; s < S; ++s) total += caps[s * kEqBlock];
+        __syncthreads();
+        if (!have) continue;
+
         // ---- the smallest boundaries, then Evaluate:
         //      T = (M-1) max t_s + sum t_s + max g_s, stage by stage
+        const int64_t Bstar = bstar[threadIdx.x];
+        const uint8_t* caps = cap_set(t, threadIdx.x, bset[threadIdx.x]);
+        int total = 0;
+        for (int s = 0; s < S; ++s) total += caps[s * kEqBlock];
         int64_t tmax = 0, tsum = 0;
         int sg = -1;
-        u128 bestG = 0, bestD = 1;
+        uint64_t bestG = 0, bestD = 1;
         int pre = 0, at = 0;
         uint8_t bnd[kMaxStages + 1];
         bnd[0] = 0;
         for (int s = 0; s < S; ++s) {
-            const uint32_t w = t.sw[s * kEqBlock];
+            const uint32_t w = mysw[s * kEqBlock];
             const int k = caps[s * kEqBlock];
             if (k < 1) atomicOr(a.err, kErrInternal);
             pre += k;
@@ -324,9 +485,9 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             if (n > 1) {
                 // stage with the largest G_s / (k_s bw_s), compared exactly
                 const int g = w & 7, j = (w >> 3) & 3;
-                const u128 G = (u128)(t.PB[nxt] - t.PB[at]);
-                const u128 D = (u128)t.inter[g] << j;
-                if (sg < 0 || G * bestD > bestG * D) {
+                const uint64_t G = (uint64_t)(t.PB[nxt] - t.PB[at]);
+                const uint64_t D = (uint64_t)t.inter[g] << j;
+                if (sg < 0 || (u128)G * bestD > (u128)bestG * D) {
                     sg = s;
                     bestG = G;
                     bestD = D;
@@ -353,7 +514,7 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
         }
     }
     if (kCount) {
-        unsigned long long v0 = sn.units, v1 = probes, v2 = searched;
+        unsigned long long v0 = units, v1 = probes, v2 = searched;
         for (int o = 16; o > 0; o >>= 1) {
             v0 += __shfl_down_sync(0xffffffffu, v0, o);
             v1 += __shfl_down_sync(0xffffffffu, v1, o);

@@ -334,84 +334,143 @@ __device__ __forceinline__ void write_rejected(const PriceArgs& a, int64_t c, in
 
 constexpr int kScreenBlock = 256;
 
-// floor(a / d) for 0 <= a < 2^16 and 1 <= d <= 256 as a * ceil(2^32 / d) / 2^32:
-// the error a (ceil(2^32/d) - 2^32/d) / 2^32 < 2^-16 never reaches 1/d, the
-// smallest distance from a / d up to the next integer
+// floor(a / d) for 0 <= a < 2^16 and 1 <= d <= 256 as (a 2^8) ceil(2^24 / d)
+// / 2^32: the error a (ceil(2^24/d) - 2^24/d) / 2^24 < 2^-8 stays below 1/d,
+// the smallest distance from a / d up to the next integer
 __device__ __forceinline__ uint32_t div_small(uint32_t a, uint32_t d, const uint32_t* magic) {
-    return d == 1 ? a : __umulhi(a, magic[d]);
+    return __umulhi(a << 8, magic[d]);
 }
 
-// Steps 1-2 and the memory screen for every candidate of the batch.
+// Per stage byte: bit 31 inadmissible; bits 24-26 type; bits 16-21 the bit
+// position of the stage's GPUs in the type's demand word (degree bits +
+// 16 * unit class); bits 0-10 the row (type, degree) of the run table.
+__device__ __forceinline__ uint32_t stage_desc(int b, const Layout& y, const unsigned char* img, int moe) {
+    const int32_t* gmaxn = reinterpret_cast<const int32_t*>(img + y.offMaxN);
+    const int32_t* gpow2 = reinterpret_cast<const int32_t*>(img + y.offPow2);
+    const int32_t* ggpus = reinterpret_cast<const int32_t*>(img + y.offGpus);
+    const int g = b & 7, j = (b >> 3) & 3;
+    if ((b >> 5) != 0 || g >= y.NT || ggpus[g] <= 0 || (!moe && (1 << j) > gmaxn[g])) return 1u << 31;
+    const int unit = (1 << j) <= gmaxn[g] ? (1 << j) : gpow2[g];
+    const int uc = 31 - __clz(unit);
+    return ((uint32_t)g << 24) | ((uint32_t)(j + 16 * uc) << 16) | (uint32_t)((g * 4 + j) * 33);
+}
+
+// Steps 1-2 and the memory screen for every candidate of the batch.  Each
+// CTA takes 256 consecutive candidates at a time: their S and M, and the
+// code planes up to the largest S among them, are copied to shared memory
+// (16-byte vector copies when the planes are aligned), the candidates are
+// counting-sorted by S, and thread i screens the i-th of that order, so the
+// lanes of a warp run stage loops of nearly equal length.
 __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
-    // stage byte -> 0x10 | unit class when the stage is admissible, else 0
-    __shared__ uint8_t unit_of[32];
+    __shared__ uint32_t desc[256];
     __shared__ uint8_t win[8 * 4 * 33];
     __shared__ uint32_t cap[8 * 4];
     __shared__ uint32_t magic[257];
     __shared__ uint64_t dem[8 * kScreenBlock];  // per-thread GPUs per unit class, 4 x 16 bits per type
+    __shared__ __align__(16) uint8_t tile[kMaxStages * kScreenBlock];  // [stage][candidate of the slice]
+    __shared__ uint8_t sS[kScreenBlock];
+    __shared__ uint16_t sM[kScreenBlock];
+    __shared__ uint8_t order[kScreenBlock];
+    __shared__ int bins[kMaxStages + 3];
+    __shared__ int smax;
     const Layout& y = a.lay;
     const int L = y.L;
     {
-        const int32_t* gmaxn = reinterpret_cast<const int32_t*>(a.img + y.offMaxN);
-        const int32_t* gpow2 = reinterpret_cast<const int32_t*>(a.img + y.offPow2);
-        const int32_t* ggpus = reinterpret_cast<const int32_t*>(a.img + y.offGpus);
         const int32_t* gcap = reinterpret_cast<const int32_t*>(a.img + y.offCap);
-        for (int i = threadIdx.x; i < 32; i += blockDim.x) {
-            const int g = i & 7, j = i >> 3;
-            uint8_t u = 0;
-            if (g < y.NT && ggpus[g] > 0 && (a.moe || (1 << j) <= gmaxn[g])) {
-                const int unit = (1 << j) <= gmaxn[g] ? (1 << j) : gpow2[g];
-                u = (uint8_t)(0x10 | (31 - __clz(unit)));
-            }
-            unit_of[i] = u;
-            cap[i] = (uint32_t)gcap[i];
-        }
+        for (int i = threadIdx.x; i < 256; i += blockDim.x) desc[i] = stage_desc(i, y, a.img, a.moe);
+        for (int i = threadIdx.x; i < 32; i += blockDim.x) cap[i] = (uint32_t)gcap[i];
         for (int i = threadIdx.x; i < 8 * 4 * 33; i += blockDim.x) win[i] = a.img[y.offWin + i];
-        for (int i = threadIdx.x; i < 257; i += blockDim.x) magic[i] = i >= 2 ? 0xffffffffu / i + 1 : 0;
+        for (int i = threadIdx.x; i < 257; i += blockDim.x) magic[i] = i >= 1 ? ((1u << 24) + i - 1) / i : 0;
     }
-    __syncthreads();
     const bool memuni = reinterpret_cast<const int32_t*>(a.img + y.offModel)[0] != 0;
+    const int s_lim = min(min(kMaxStages, a.s_max), L);
+    const bool vec16 = ((reinterpret_cast<uintptr_t>(a.code) | (uintptr_t)a.stride) & 15) == 0;
     uint64_t* mydem = dem + threadIdx.x;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    const int64_t n_round = (a.n + 31) & ~(int64_t)31;  // whole warps iterate together
-    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < n_round; c += stride) {
-        const bool live = c < a.n;
+    const int lane = threadIdx.x & 31;
+    for (int64_t c0 = (int64_t)blockIdx.x * kScreenBlock; c0 < a.n; c0 += (int64_t)gridDim.x * kScreenBlock) {
+        const int nloc = (int)min((int64_t)kScreenBlock, a.n - c0);
+        // ---- S and M of the slice; S = 0 marks a depth or M outside range,
+        //      bin kMaxStages + 1 the padding past the batch
+        int key = kMaxStages + 1;
+        if (threadIdx.x < nloc) {
+            const int S = a.S[c0 + threadIdx.x];
+            const int M = a.M[c0 + threadIdx.x];
+            key = (S >= 1 && S <= s_lim && M >= 1) ? S : 0;
+            sS[threadIdx.x] = (uint8_t)key;
+            sM[threadIdx.x] = (uint16_t)M;
+        }
+        if (threadIdx.x < kMaxStages + 3) bins[threadIdx.x] = 0;
+        if (threadIdx.x == 0) smax = 0;
+        __syncthreads();
+        atomicAdd(&bins[key], 1);
+        if (key <= kMaxStages && key > 0) atomicMax(&smax, key);
+        __syncthreads();
+        // ---- code planes 0 .. smax-1 of the slice into the tile
+        const int np = smax;
+        if (vec16 && nloc == kScreenBlock) {
+            for (int i = threadIdx.x; i < np * (kScreenBlock / 16); i += kScreenBlock) {
+                const int s = i / (kScreenBlock / 16), o = (i % (kScreenBlock / 16)) * 16;
+                *reinterpret_cast<uint4*>(tile + s * kScreenBlock + o) =
+                    __ldg(reinterpret_cast<const uint4*>(a.code + (int64_t)s * a.stride + c0 + o));
+            }
+        } else {
+            for (int i = threadIdx.x; i < np * kScreenBlock; i += kScreenBlock) {
+                const int s = i / kScreenBlock, o = i % kScreenBlock;
+                if (o < nloc) tile[i] = __ldg(a.code + (int64_t)s * a.stride + c0 + o);
+            }
+        }
+        if (threadIdx.x == 0) {
+            int run = 0;
+            for (int b = 0; b <= kMaxStages + 1; ++b) {
+                const int v = bins[b];
+                bins[b] = run;
+                run += v;
+            }
+        }
+        __syncthreads();
+        order[atomicAdd(&bins[key], 1)] = (uint8_t)threadIdx.x;
+        __syncthreads();
+        const int ci = order[threadIdx.x];
+        const bool live = threadIdx.x < nloc;  // padding sorts last
+        const int64_t c = c0 + ci;
         int S = 0, M = 0, status = HEDDLE_CAND_INVALID;
         int64_t n = 0;
         if (live) {
-            S = a.S[c];
-            M = a.M[c];
-            if (S >= 1 && S <= kMaxStages && S <= a.s_max && S <= L && M >= 1) {
+            S = sS[ci];
+            M = sM[ci];
+            if (S > 0) {
 #pragma unroll
                 for (int g = 0; g < 8; ++g) mydem[g * kScreenBlock] = 0;
                 uint32_t bad = 0, present = 0;
                 int run_sum = 0, run_min = 255;
+                const uint8_t* col = tile + ci;
                 for (int s = 0; s < S; ++s) {
-                    const int b = __ldg(a.code + (int64_t)s * a.stride + c);
-                    const int u = unit_of[b & 31];
-                    bad |= (uint32_t)(b >> 5) | (uint32_t)(u == 0);
-                    const int g = b & 7, j = (b >> 3) & 3;
+                    const uint32_t d = desc[col[s * kScreenBlock]];
+                    bad |= d;
+                    const int g = (d >> 24) & 7;
                     present |= 1u << g;
-                    // k GPUs in units of 2^(u & 3)
-                    mydem[g * kScreenBlock] += (uint64_t)(1u << j) << (16 * (u & 3));
-                    const int w = win[(g * 4 + j) * 33 + min(S - s, M)];
+                    mydem[g * kScreenBlock] += 1ull << ((d >> 16) & 63);
+                    const int w = win[(d & 0x7ff) + min(S - s, M)];
                     run_sum += w;
                     run_min = min(run_min, w);
                 }
-                if (bad) {
+                if (bad >> 31) {
                     status = HEDDLE_CAND_INVALID;
                 } else {
-                    // n = min over (type, class e) of capacity / GPUs in units >= 2^e
+                    // n = min over (type, class e) of capacity / GPUs in units
+                    // >= 2^e; a class with no group of its own size is
+                    // dominated by the class above it
                     uint32_t nn = 0xffffffffu;
                     while (present) {
                         const int g = __ffs(present) - 1;
                         present &= present - 1;
                         const uint64_t v = mydem[g * kScreenBlock];
-                        uint32_t d = 0;
+                        uint32_t dsum = 0;
 #pragma unroll
                         for (int e = 3; e >= 0; --e) {
-                            d += (uint32_t)(v >> (16 * e)) & 0xffffu;
-                            if (d) nn = min(nn, div_small(cap[g * 4 + e], d, magic));
+                            const uint32_t f = (uint32_t)(v >> (16 * e)) & 0xffffu;
+                            dsum += f;
+                            if (f) nn = min(nn, div_small(cap[g * 4 + e], dsum, magic));
                         }
                     }
                     n = nn;
@@ -428,25 +487,25 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
         // compact the candidates that need the search (one atomic per warp)
         const bool take = live && status == HEDDLE_CAND_OK;
         const unsigned mask = __ballot_sync(0xffffffffu, take);
-        if (!mask) continue;
-        const int lane = threadIdx.x & 31;
-        int base = 0;
-        if (lane == 0) base = atomicAdd(a.wl_count, __popc(mask));
-        base = __shfl_sync(0xffffffffu, base, 0);
-        if (take) {
-            const int p = base + __popc(mask & ((1u << lane) - 1));
-            if (p < a.wl_cap) {
-                a.wl_idx[p] = (int32_t)c;
-                a.wl_n[p] = (uint16_t)n;
-                a.wl_M[p] = (uint16_t)M;
-                a.wl_S[p] = (uint8_t)S;
-                a.wl_memok[p] = memuni ? 1 : 0;
-                for (int s = 0; s < S; ++s)
-                    a.wl_code[(int64_t)s * a.wl_cap + p] = __ldg(a.code + (int64_t)s * a.stride + c);
-            } else {
-                atomicOr(a.err, kErrInternal);
+        if (mask) {
+            int base = 0;
+            if (lane == 0) base = atomicAdd(a.wl_count, __popc(mask));
+            base = __shfl_sync(0xffffffffu, base, 0);
+            if (take) {
+                const int p = base + __popc(mask & ((1u << lane) - 1));
+                if (p < a.wl_cap) {
+                    a.wl_idx[p] = (int32_t)c;
+                    a.wl_n[p] = (uint16_t)n;
+                    a.wl_M[p] = (uint16_t)M;
+                    a.wl_S[p] = (uint8_t)S;
+                    a.wl_memok[p] = memuni ? 1 : 0;
+                    for (int s = 0; s < S; ++s) a.wl_code[(int64_t)s * a.wl_cap + p] = tile[s * kScreenBlock + ci];
+                } else {
+                    atomicOr(a.err, kErrInternal);
+                }
             }
         }
+        __syncthreads();  // the tile, S, M and order are reused by the next slice
     }
 }
 
