@@ -355,7 +355,7 @@ def main():
                      "units_per_candidate": work["checks"] / n,
                      "probes_per_searched": work["probes"] / max(1, work["priced"]),
                      "searched_fraction": work["priced"] / n,
-                     "phases_us_per_launch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in phases.items()},
+                     "phases_us_per_batch": {k: 1e3 * v[0] / max(1, search_launches) for k, v in phases.items()},
                      "phase_share": {k: v[0] / total_phase_ms for k, v in phases.items()},
                      "peak_basis": "%s: %d SMs x %d lanes x %.0f MHz (%s sm_max)" % (
                          "issue slots", SMS, LANES_PER_SM, float(peaks.get("sm_max_mhz", 2070.0)), peak_kind)},

@@ -62,8 +62,8 @@ enum {
 typedef struct heddle_ctx heddle_ctx;
 
 /* Create a context on CUDA device `device`.  Allocates its device scratch
- * once (about 44 MB: the search worklist of 2^20 candidates and the top-k
- * merge lists) and queries the SM count.
+ * once (about 60 MB: the search worklist of 2^20 candidates with their 32
+ * stage bytes, and the top-k merge lists) and queries the SM count.
  * *out is NULL on failure. */
 heddle_status heddle_create(heddle_ctx** out, int32_t device);
 
@@ -214,8 +214,9 @@ heddle_status heddle_topk_reset(heddle_ctx* ctx, heddle_topk_state* state, int32
                                 void* stream);
 
 /* Merge the OK candidates of a priced batch into *state (device): a
- * block-level top-k per CTA into context-owned scratch, then a one-CTA merge
- * with the incoming state (two launches, no inter-CTA waiting).
+ * block-level top-k per CTA into context-owned scratch, then merge levels of
+ * 16 lists per CTA, the last with the incoming state (two or three
+ * launches, no inter-CTA waiting).
  * Asynchronous; reads cands->M, results->T/n_dp/status.  Errors: E_ARG,
  * E_STATE, E_CUDA.  Calls on one context must not overlap on the GPU (they
  * share the scratch): use one stream per context. */
@@ -329,7 +330,9 @@ heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);
  * top-k kernels.  heddle_phase_times synchronises on them and returns, per
  * phase (SCREEN, SEARCH, TOPK), the summed elapsed milliseconds and the
  * number of kernels launched in it (one screen and one search kernel per
- * chunk; two or three top-k kernels), then forgets them.  The events add no work to the
+ * chunk, with the equal-layer search also the kernel that orders the
+ * worklist by depth in the screen phase; two or three top-k kernels), then
+ * forgets them.  The events add no work to the
  * kernels; enabling or disabling changes no result.  Errors: E_ARG,
  * E_CUDA. */
 #define HEDDLE_PHASE_SCREEN 0

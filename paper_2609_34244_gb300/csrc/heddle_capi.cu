@@ -37,7 +37,8 @@ struct heddle_ctx {
     unsigned long long* d_counters = nullptr;  // [3]
     bool count_next = false;
     // search worklist scratch (hd::kWorklistCap candidates)
-    int32_t* d_wl_count = nullptr;
+    int32_t* d_wl_count = nullptr;  // hd::kWlMeta ints
+    int32_t* d_wl_order = nullptr;
     int32_t* d_wl_idx = nullptr;
     uint16_t* d_wl_n = nullptr;
     uint16_t* d_wl_M = nullptr;
@@ -265,7 +266,8 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
         e = cudaMalloc(&x->d_scratch, sizeof(hd::TopkEntry) * hd::kMaxTopK * x->scratch_blocks);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch_count, sizeof(int32_t) * x->scratch_blocks);
     const size_t cap = hd::kWorklistCap;
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_count, sizeof(int32_t));
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_count, sizeof(int32_t) * hd::kWlMeta);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_order, sizeof(int32_t) * cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_idx, sizeof(int32_t) * cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_n, sizeof(uint16_t) * cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_M, sizeof(uint16_t) * cap);
@@ -277,6 +279,7 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     const int l2 = (x->scratch_blocks + 31) / 32;
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2, sizeof(hd::TopkEntry) * hd::kMaxTopK * l2);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2_count, sizeof(int32_t) * l2);
+
     if (e != cudaSuccess) {
         heddle_destroy(x);
         return HEDDLE_E_CUDA;
@@ -295,6 +298,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_scratch);
     cudaFree(x->d_scratch_count);
     cudaFree(x->d_wl_count);
+    cudaFree(x->d_wl_order);
     cudaFree(x->d_wl_idx);
     cudaFree(x->d_wl_n);
     cudaFree(x->d_wl_M);
@@ -455,6 +459,7 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     a.wl_S = x->d_wl_S;
     a.wl_memok = x->d_wl_memok;
     a.wl_code = x->d_wl_code;
+    a.wl_order = x->d_wl_order;
     a.wl_cap = hd::kWorklistCap;
     a.uniform = equal_layer_search(x) ? 1 : 0;
     a.wl_T = x->d_wl_T;

@@ -27,8 +27,10 @@
 // at B* give the componentwise smallest split -- hence the lexicographically
 // smallest -- a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
 //
-// Scheduling: each CTA takes 256 worklist entries at a time, counting-sorted
-// by S so that the lanes of a warp run stage loops of equal length.  Every
+// Scheduling: an order kernel first lists the worklist by decreasing S
+// (the screen counted the entries per depth); each CTA takes 256
+// consecutive entries of that order, so the lanes of a warp run stage loops
+// of equal length and the warps of a CTA carry equal work.  Every
 // thread packs its candidate's stages once into 32-bit words (cost index |
 // P2P index | memory run) held in shared memory interleaved by thread, runs
 // the float guess and one exact probe; the few searches still open are
@@ -44,13 +46,11 @@
 namespace hd {
 namespace {
 
-typedef unsigned __int128 u128;
-
 constexpr int kEqBlock = 256;
 constexpr int kZeroP2P = 128;  // a zero entry after the 8 x 8 x 2 P2P table
 constexpr int kMaxIters = 256;
 
-constexpr int kTailCap = 64;  // open searches queued per slice
+constexpr int kTailCap = 32;  // open searches queued per slice
 
 // State of one threshold search.
 struct Search {
@@ -61,11 +61,13 @@ struct Search {
     int16_t fset, wset; // cap set of the last feasible probe (-1: none), set written next
     int16_t owner, S;   // thread whose shared-memory columns hold the stages; depth
     int32_t probes;
+    int32_t p;          // worklist entry
+    uint16_t M, n;      // its microbatches and DP degree
     int32_t pad;
 };
 
 struct EqLayout {
-    uint32_t q, rq, qf, p2p, cf, inter, maxn, PB, win, sw, caps, tail, bstar, bytes;
+    uint32_t q, rq, p2p, cf, inter, maxn, PB, win, sw, caps, tail, bytes;
 };
 
 __host__ __device__ inline uint32_t al16(uint32_t x) { return (x + 15u) & ~15u; }
@@ -75,7 +77,6 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
     uint32_t o = 0;
     e.q = o;     o = al16(o + 8 * 32);             // int64 [j * 8 + g]
     e.rq = o;    o = al16(o + 4 * 32);             // float 1 / q
-    e.qf = o;    o = al16(o + 4 * 32);             // float q
     e.p2p = o;   o = al16(o + 8 * 129);            // int64 [(g * 8 + h) * 2 + same], [128] = 0
     e.cf = o;    o = al16(o + 4 * 129);            // float P2P
     e.inter = o; o = al16(o + 8 * 8);              // int64 [g]
@@ -83,9 +84,8 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
     e.PB = o;    o = al16(o + 8 * (L + 1));        // int64 gradient-byte prefix
     e.win = o;   o = al16(o + 8 * 4 * 33);         // uint8 [(g * 4 + j) * 33 + f]
     e.sw = o;    o = al16(o + 4 * kMaxStages * kEqBlock);  // uint32 [s][thread]
-    e.caps = o;  o = al16(o + 2 * (kMaxStages + 1) * kEqBlock);  // uint8 [2][s][thread]
-    e.tail = o;  o = al16(o + sizeof(struct Search) * kTailCap);    // open searches
-    e.bstar = o; o = al16(o + 8 * kEqBlock);                         // int64 B* per thread
+    e.caps = o;  o = al16(o + 2 * kMaxStages * kEqBlock);         // uint8 [2][s][thread]
+    e.tail = o;  o = al16(o + sizeof(struct Search) * kTailCap);  // open searches
     e.bytes = o;
     return e;
 }
@@ -93,15 +93,15 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
 struct EqTabs {
     const int64_t* q;
     const float* rq;
-    const float* qf;
     const int64_t* p2p;
     const float* cf;
     const int64_t* inter;
     const int32_t* maxn;
     const int64_t* PB;
     const uint8_t* win;
+    int64_t pbytes;  // gradient bytes of every layer when they are all equal, else -1
     uint32_t* sw;   // stage words of thread 0; thread o's element s at [s * kEqBlock + o]
-    uint8_t* caps;  // caps of thread 0, two sets; thread o's set b element s at [(b * 33 + s) * kEqBlock + o]
+    uint8_t* caps;  // caps of thread 0, two sets; thread o's set b element s at [(b * 32 + s) * kEqBlock + o]
     int L;
 };
 
@@ -229,7 +229,7 @@ __device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, uint8_t* caps, int
 }
 
 __device__ __forceinline__ uint8_t* cap_set(const EqTabs& t, int owner, int set) {
-    return t.caps + set * (kMaxStages + 1) * kEqBlock + owner;
+    return t.caps + set * kMaxStages * kEqBlock + owner;
 }
 
 // One exact probe of search q at q.B and the bracket update; returns true
@@ -277,9 +277,9 @@ __device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
     return false;
 }
 
-// Finish search q: probe until B* is known, then make sure a cap set holds
-// the caps at B*.  Writes B* and the set to the owner's slots.
-__device__ void eq_finish(const EqTabs& t, Search& q, int64_t* bstar, uint8_t* bset, uint32_t* err) {
+// Finish search q: probe until B* = q.hi is known, then make sure cap set
+// q.fset holds the caps at B*.
+__device__ void eq_finish(const EqTabs& t, Search& q, uint32_t* err) {
     while (q.lo < q.hi)
         if (eq_step(t, q, err)) break;
     if (q.fset < 0 || q.fhi != q.hi) {
@@ -288,17 +288,88 @@ __device__ void eq_finish(const EqTabs& t, Search& q, int64_t* bstar, uint8_t* b
         Probe p;
         if (!eq_probe(t, t.sw + q.owner, cap_set(t, q.owner, q.wset), q.S, q.hi, p)) atomicOr(err, kErrInternal);
         q.fset = q.wset;
+        q.fhi = q.hi;
+        q.chi = p.tot;
     }
-    bstar[q.owner] = q.hi;
-    bset[q.owner] = (uint8_t)q.fset;
+}
+
+// The smallest boundaries from the caps at B* (cap set `set` of column
+// `owner`, holding `total` layers), then Evaluate:
+// T = (M-1) max t_s + sum t_s + max g_s, stage by stage; writes entry p.
+__device__ void eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int64_t p, int S, int M, int64_t n,
+                            int64_t Bstar, int set, int total) {
+    const int L = t.L;
+    const int64_t c = a.wl_idx[p];
+    const uint32_t* sw = t.sw + owner;
+    const uint8_t* caps = cap_set(t, owner, set);
+    int64_t tmax = 0, tsum = 0;
+    int sg = -1;
+    // the stage with the largest G_s / (k_s bw_s), compared exactly: with
+    // equal gradient bytes per layer G_s = layers * bytes, and layers
+    // (< 2^8) times bandwidth (< 2^43) fits 64 bits
+    uint64_t bestG = 0, bestD = 1;
+    int pre = 0, at = 0;
+    int64_t pb_at = t.PB[0];
+    for (int s = 0; s < S; ++s) {
+        const uint32_t w = sw[s * kEqBlock];
+        const int k = caps[s * kEqBlock];
+        if (k < 1) atomicOr(a.err, kErrInternal);
+        pre += k;
+        const int nxt = s + 1 == S ? L : max(at + 1, L - (total - pre));
+        if (a.bounds) a.bounds[(int64_t)(s + 1) * a.bstride + c] = (uint8_t)nxt;
+        const int64_t ts = (int64_t)(nxt - at) * t.q[w & 31] + t.p2p[(w >> 5) & 255];
+        tmax = max(tmax, ts);
+        tsum += ts;
+        if (n > 1) {
+            const int g = w & 7, j = (w >> 3) & 3;
+            const uint64_t D = (uint64_t)t.inter[g] << j;
+            if (t.pbytes >= 0) {
+                const uint64_t len = (uint64_t)(nxt - at);
+                if (sg < 0 || len * bestD > bestG * D) {
+                    sg = s;
+                    bestG = len;
+                    bestD = D;
+                }
+            } else {
+                const int64_t pb_nxt = t.PB[nxt];
+                const uint64_t G = (uint64_t)(pb_nxt - pb_at);
+                pb_at = pb_nxt;
+                if (sg < 0 || (u128)G * bestD > (u128)bestG * D) {
+                    sg = s;
+                    bestG = G;
+                    bestD = D;
+                }
+            }
+        }
+        at = nxt;
+    }
+    if (t.pbytes >= 0) bestG *= (uint64_t)t.pbytes;
+    if (a.bounds) {
+        a.bounds[c] = 0;
+        for (int s = S + 1; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = 0;
+    }
+    if (tmax != Bstar || pre != total) atomicOr(a.err, kErrInternal);
+    int64_t gmax = 0;
+    if (n > 1) {
+        // ring all-reduce over n replicas: ceil(2(n-1) G 1e9 / (n k bw))
+        // (G < 2^50 and bandwidths < 2^40 keep n k bw below 2^64)
+        const u128 num = (u128)(2 * (uint64_t)(n - 1) * 1000000000ull) * bestG;
+        bool ok = true;
+        gmax = (int64_t)ceil_div_u128(num, (uint64_t)n * bestD, &ok);
+        if (!ok) atomicOr(a.err, kErrInternal);
+    }
+    const int64_t T = (int64_t)(M - 1) * Bstar + tsum + gmax;
+    a.T[c] = T;
+    a.wl_T[p] = T;
+    a.wl_nM[p] = (uint32_t)n * (uint32_t)M;
+    a.B[c] = Bstar;
+    a.ndp[c] = (uint16_t)n;
+    a.status[c] = HEDDLE_CAND_OK;
 }
 
 template <bool kCount>
-__global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
+__global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int bins[kMaxStages + 2];
-    __shared__ uint16_t order[kEqBlock];
-    __shared__ uint8_t bset[kEqBlock];
     __shared__ int tail_n;
     const Layout& y = a.lay;
     const int L = y.L;
@@ -307,7 +378,6 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     {
         int64_t* q = reinterpret_cast<int64_t*>(smem + el.q);
         float* rq = reinterpret_cast<float*>(smem + el.rq);
-        float* qf = reinterpret_cast<float*>(smem + el.qf);
         int64_t* p2p = reinterpret_cast<int64_t*>(smem + el.p2p);
         float* cf = reinterpret_cast<float*>(smem + el.cf);
         int64_t* inter = reinterpret_cast<int64_t*>(smem + el.inter);
@@ -320,7 +390,6 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             const int64_t v = g < y.NT ? gP[(g * 4 + j) * (L + 1) + 1] - gP[(g * 4 + j) * (L + 1)] : 0;
             q[i] = v;
             rq[i] = v > 0 ? 1.0f / (float)v : 0.0f;
-            qf[i] = (float)v;
         }
         for (int i = threadIdx.x; i < 129; i += blockDim.x) {
             const int64_t v = i < 128 ? reinterpret_cast<const int64_t*>(a.img + y.offP2P)[i] : 0;
@@ -331,26 +400,27 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             inter[i] = reinterpret_cast<const int64_t*>(a.img + y.offInter)[i];
             maxn[i] = reinterpret_cast<const int32_t*>(a.img + y.offMaxN)[i];
         }
+        for (int i = threadIdx.x; i < 8 * 4 * 33; i += blockDim.x) win[i] = a.img[y.offWin + i];
         for (int i = threadIdx.x; i <= L; i += blockDim.x)
             PB[i] = reinterpret_cast<const int64_t*>(a.img + y.offPB)[i];
-        for (int i = threadIdx.x; i < 8 * 4 * 33; i += blockDim.x) win[i] = a.img[y.offWin + i];
     }
     __syncthreads();
     EqTabs t;
     t.q = reinterpret_cast<const int64_t*>(smem + el.q);
     t.rq = reinterpret_cast<const float*>(smem + el.rq);
-    t.qf = reinterpret_cast<const float*>(smem + el.qf);
     t.p2p = reinterpret_cast<const int64_t*>(smem + el.p2p);
     t.cf = reinterpret_cast<const float*>(smem + el.cf);
     t.inter = reinterpret_cast<const int64_t*>(smem + el.inter);
     t.maxn = reinterpret_cast<const int32_t*>(smem + el.maxn);
     t.PB = reinterpret_cast<const int64_t*>(smem + el.PB);
     t.win = smem + el.win;
+    t.pbytes = reinterpret_cast<const int32_t*>(a.img + y.offModel)[2]
+                   ? t.PB[1] - t.PB[0]
+                   : -1;
     t.sw = reinterpret_cast<uint32_t*>(smem + el.sw);
     t.caps = smem + el.caps;
     t.L = L;
     Search* tail = reinterpret_cast<Search*>(smem + el.tail);
-    int64_t* bstar = reinterpret_cast<int64_t*>(smem + el.bstar);
     uint32_t* mysw = t.sw + threadIdx.x;
 
     unsigned long long units = 0, probes = 0, searched = 0;
@@ -358,32 +428,19 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
     const int64_t count_r = (count + kEqBlock - 1) / kEqBlock * kEqBlock;
     const int64_t stride = (int64_t)gridDim.x * kEqBlock;
     for (int64_t base = (int64_t)blockIdx.x * kEqBlock; base < count_r; base += stride) {
-        // ---- this CTA's 256 entries, counting-sorted by S (0: no entry)
-        const int64_t p0 = base + threadIdx.x;
-        const int s0 = p0 < count ? a.wl_S[p0] : 0;
-        if (threadIdx.x < kMaxStages + 2) bins[threadIdx.x] = 0;
+        // ---- this CTA's 256 entries of the order by decreasing S, so the
+        //      lanes of a warp (and the warps of a CTA) have nearly equal S
         if (threadIdx.x == 0) tail_n = 0;
         __syncthreads();
-        atomicAdd(&bins[s0], 1);
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            int run = 0;
-            for (int b = 0; b <= kMaxStages; ++b) {
-                const int v = bins[b];
-                bins[b] = run;
-                run += v;
-            }
-        }
-        __syncthreads();
-        order[atomicAdd(&bins[s0], 1)] = (uint16_t)threadIdx.x;
-        __syncthreads();
-        const int64_t p = base + order[threadIdx.x];
-        const bool have = p < count;
+        const bool have = base + threadIdx.x < count;
+        const int64_t p = have ? a.wl_order[base + threadIdx.x] : 0;
 
         int S = 0, M = 0;
-        int64_t n = 0, c = 0;
+        int64_t n = 0;
+        int64_t Bstar = 0;  // with its cap set and layer count, unless queued
+        int bset = 0, btot = 0, slot = -1;
+        bool queued = false;
         if (have) {
-            c = a.wl_idx[p];
             S = a.wl_S[p];
             M = a.wl_M[p];
             n = a.wl_n[p];
@@ -398,11 +455,21 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             q.lo = 0;
             q.hi = 0;
             float inv = 0.f, cw = 0.f;
-            int code = a.wl_code[p];
-            for (int s = 0; s < S; ++s) {
-                const bool last = s + 1 == S;
-                const int next = last ? 0 : a.wl_code[(int64_t)(s + 1) * a.wl_cap + p];
-                const uint32_t w = stage_word(code, next, last, min(S - s, M), t);
+            // the entry's row of stage bytes (zero past S), 16 at a time
+            uint32_t cw4[8];
+            {
+                const uint4* row = reinterpret_cast<const uint4*>(a.wl_code + p * kMaxStages);
+                const uint4 v0 = __ldg(row);
+                const uint4 v1 = S > 16 ? __ldg(row + 1) : make_uint4(0, 0, 0, 0);
+                cw4[0] = v0.x; cw4[1] = v0.y; cw4[2] = v0.z; cw4[3] = v0.w;
+                cw4[4] = v1.x; cw4[5] = v1.y; cw4[6] = v1.z; cw4[7] = v1.w;
+            }
+#pragma unroll
+            for (int s = 0; s < kMaxStages; ++s) {
+                if (s >= S) break;
+                const int code = (cw4[s >> 2] >> ((s & 3) * 8)) & 0xff;
+                const int next = s + 1 < kMaxStages ? (cw4[(s + 1) >> 2] >> (((s + 1) & 3) * 8)) & 0xff : 0;
+                const uint32_t w = stage_word(code, next, s + 1 == S, min(S - s, M), t);
                 mysw[s * kEqBlock] = w;
                 const int64_t qq = t.q[w & 31], cc = t.p2p[(w >> 5) & 255];
                 const int m = (int)(w >> 13) & 255;
@@ -411,7 +478,6 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
                 const float rq = t.rq[w & 31];
                 inv += rq;
                 cw += t.cf[(w >> 5) & 255] * rq;
-                code = next;
             }
             // first guess: Newton on the saturating continuous count
             float Bf = fmaxf((float)q.lo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : (float)q.lo);
@@ -432,21 +498,25 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             q.owner = (int16_t)threadIdx.x;
             q.S = (int16_t)S;
             q.probes = 0;
+            q.p = (int32_t)p;
+            q.M = (uint16_t)M;
+            q.n = (uint16_t)n;
             q.pad = 0;
             // one exact probe here; open searches go to the CTA's queue
-            bool done = q.lo >= q.hi || eq_step(t, q, a.err);
-            if (done && q.fset >= 0 && q.fhi == q.hi) {
-                bstar[threadIdx.x] = q.hi;
-                bset[threadIdx.x] = (uint8_t)q.fset;
-            } else {
-                const int slot = atomicAdd(&tail_n, 1);
+            const bool done = q.lo >= q.hi || eq_step(t, q, a.err);
+            if (!(done && q.fset >= 0 && q.fhi == q.hi)) {
+                slot = atomicAdd(&tail_n, 1);
                 if (slot < kTailCap) {
                     tail[slot] = q;
                     q.probes = 0;  // counted by the thread that finishes it
+                    queued = true;
                 } else {
-                    eq_finish(t, q, bstar, bset, a.err);
+                    eq_finish(t, q, a.err);
                 }
             }
+            Bstar = q.hi;
+            bset = q.fset;
+            btot = q.chi;
             if (kCount) probes += q.probes;
         }
         __syncthreads();
@@ -454,64 +524,21 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
         const int nt = min(tail_n, kTailCap);
         for (int i = threadIdx.x; i < nt; i += kEqBlock) {
             Search q = tail[i];
-            eq_finish(t, q, bstar, bset, a.err);
+            eq_finish(t, q, a.err);
+            tail[i].hi = q.hi;
+            tail[i].fset = q.fset;
+            tail[i].chi = q.chi;
             if (kCount) probes += q.probes;
         }
         __syncthreads();
-        if (!have) continue;
-
-        // ---- the smallest boundaries, then Evaluate:
-        //      T = (M-1) max t_s + sum t_s + max g_s, stage by stage
-        const int64_t Bstar = bstar[threadIdx.x];
-        const uint8_t* caps = cap_set(t, threadIdx.x, bset[threadIdx.x]);
-        int total = 0;
-        for (int s = 0; s < S; ++s) total += caps[s * kEqBlock];
-        int64_t tmax = 0, tsum = 0;
-        int sg = -1;
-        uint64_t bestG = 0, bestD = 1;
-        int pre = 0, at = 0;
-        uint8_t bnd[kMaxStages + 1];
-        bnd[0] = 0;
-        for (int s = 0; s < S; ++s) {
-            const uint32_t w = mysw[s * kEqBlock];
-            const int k = caps[s * kEqBlock];
-            if (k < 1) atomicOr(a.err, kErrInternal);
-            pre += k;
-            const int nxt = s + 1 == S ? L : max(at + 1, L - (total - pre));
-            bnd[s + 1] = (uint8_t)nxt;
-            const int64_t ts = (int64_t)(nxt - at) * t.q[w & 31] + t.p2p[(w >> 5) & 255];
-            tmax = max(tmax, ts);
-            tsum += ts;
-            if (n > 1) {
-                // stage with the largest G_s / (k_s bw_s), compared exactly
-                const int g = w & 7, j = (w >> 3) & 3;
-                const uint64_t G = (uint64_t)(t.PB[nxt] - t.PB[at]);
-                const uint64_t D = (uint64_t)t.inter[g] << j;
-                if (sg < 0 || (u128)G * bestD > (u128)bestG * D) {
-                    sg = s;
-                    bestG = G;
-                    bestD = D;
-                }
-            }
-            at = nxt;
+        if (queued) {
+            const Search& q = tail[slot];
+            Bstar = q.hi;
+            bset = q.fset;
+            btot = q.chi;
         }
-        if (tmax != Bstar) atomicOr(a.err, kErrInternal);
-        int64_t gmax = 0;
-        if (n > 1) {
-            // ring all-reduce over n replicas: ceil(2(n-1) G 1e9 / (n k bw))
-            const u128 num = (u128)2 * (u128)(n - 1) * bestG * 1000000000u;
-            const u128 den = (u128)n * bestD;
-            gmax = (int64_t)((num + den - 1) / den);
-        }
-        a.T[c] = (int64_t)(M - 1) * Bstar + tsum + gmax;
-        a.wl_T[p] = a.T[c];
-        a.wl_nM[p] = (uint32_t)n * (uint32_t)M;
-        a.B[c] = Bstar;
-        a.ndp[c] = (uint16_t)n;
-        a.status[c] = HEDDLE_CAND_OK;
-        if (a.bounds) {
-            for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = s <= S ? bnd[s] : 0;
-        }
+        if (have) eq_evaluate(a, t, threadIdx.x, p, S, M, n, Bstar, bset, btot);
+        __syncthreads();  // columns and queue are reused by the next slice
     }
     if (kCount) {
         unsigned long long v0 = units, v1 = probes, v2 = searched;
@@ -525,6 +552,46 @@ __global__ void __launch_bounds__(kEqBlock) eq_search_kernel(PriceArgs a) {
             atomicAdd(&a.counters[1], v1);
             atomicAdd(&a.counters[2], v2);
         }
+    }
+}
+
+// The worklist in order of decreasing S: entry p goes to the start of its
+// depth's range (the entries of larger depths come first) plus a cursor
+// (warp-aggregated atomics); the order within a depth is immaterial.
+__global__ void __launch_bounds__(256) order_kernel(PriceArgs a) {
+    __shared__ int start[kMaxStages + 1];
+    if (threadIdx.x < 32) {
+        // start of depth S = entries of depths above S: an inclusive scan
+        // of depths 32 .. 1 in lanes 0 .. 31 (depth 0 never enters)
+        const int lane = threadIdx.x;
+        const int v = a.wl_count[1 + (kMaxStages - lane)];
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        start[kMaxStages - lane] = x - v;
+        if (lane == 31) start[0] = x;
+    }
+    __syncthreads();
+    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    const int64_t n_round = (count + 31) & ~(int64_t)31;
+    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < n_round;
+         p += (int64_t)gridDim.x * blockDim.x) {
+        const bool live = p < count;
+        const int S = live ? a.wl_S[p] : -1;
+        const unsigned mask = __ballot_sync(0xffffffffu, live);
+        if (!live) continue;
+        const unsigned same = __match_any_sync(mask, S);
+        const int lane = threadIdx.x & 31;
+        const int leader = __ffs(same) - 1;
+        int pos = 0;
+        if (lane == leader) pos = atomicAdd(a.wl_count + 1 + (kMaxStages + 1) + S, __popc(same));
+        pos = __shfl_sync(same, pos, leader) + __popc(same & ((1u << lane) - 1));
+        const int64_t dst = (int64_t)start[S] + pos;
+        if (dst < count) a.wl_order[dst] = (int32_t)p;
+        else atomicOr(a.err, kErrInternal);
     }
 }
 
@@ -546,6 +613,12 @@ cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
 }
 
 }  // namespace
+
+cudaError_t launch_eq_order(const PriceArgs& a, int num_sms, cudaStream_t st) {
+    const int grid = (int)std::min<int64_t>((a.n + 255) / 256, (int64_t)num_sms * 8);
+    order_kernel<<<grid, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
     return a.counters ? launch<true>(a, num_sms, st) : launch<false>(a, num_sms, st);

@@ -15,6 +15,8 @@ constexpr int kMaxLayers = HEDDLE_MAX_LAYERS;
 constexpr int kMaxTopK = HEDDLE_MAX_TOPK;
 constexpr int64_t kInf = INT64_MAX;
 
+typedef unsigned __int128 u128;
+
 // Device error flags (heddle_device_errors).
 constexpr uint32_t kErrStageWait = 1u;
 constexpr uint32_t kErrSearchBound = 2u;
@@ -113,13 +115,15 @@ struct PriceArgs {
     unsigned long long* counters;  // non-null selects the counting variant
     // worklist of the candidates that need the threshold search (device
     // scratch owned by the context, capacity wl_cap candidates)
-    int32_t* wl_count;
+    int32_t* wl_count;   // [1 + 2 (kMaxStages + 1)]: entries, then per depth S the
+                         // entries of that depth and an order cursor (cleared per chunk)
     int32_t* wl_idx;
     uint16_t* wl_n;
     uint16_t* wl_M;
     uint8_t* wl_S;
     uint8_t* wl_memok;   // 1: memory feasibility already decided by the screen
-    uint8_t* wl_code;    // [kMaxStages][wl_cap]
+    uint8_t* wl_code;    // [wl_cap][kMaxStages] stage bytes, a 32-byte row per entry (zero past S)
+    int32_t* wl_order;   // [wl_cap] entries by decreasing S (equal-layer search)
     int32_t wl_cap;
     int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
     // per worklist entry, written by the search: T (-1 unless OK) and n * M,
@@ -133,8 +137,11 @@ struct PriceArgs {
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid = nullptr,
                          int64_t* launches = nullptr);
 // The equal-layer search over the worklist the screen produced.
+// (after launch_eq_order, which orders the worklist by decreasing S)
+cudaError_t launch_eq_order(const PriceArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
+constexpr int kWlMeta = 1 + 2 * (kMaxStages + 1);  // ints of a.wl_count
 
 
 struct TopkArgs {
@@ -166,5 +173,34 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t
 cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st,
                                  int64_t* launches = nullptr);
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st);
+
+// ceil(A / C) for a 128-bit A and 1 <= C < 2^64 whose quotient is below
+// 2^62: a float estimate of the quotient refined with exact 128-bit
+// remainders (each refinement leaves about 2^-22 of the error), then exact
+// unit steps.  *ok is cleared if the steps did not settle (never expected).
+__device__ __forceinline__ float u128_to_float(u128 v) {
+    return (float)(uint64_t)(v >> 64) * 18446744073709551616.0f + (float)(uint64_t)v;
+}
+
+__device__ inline uint64_t ceil_div_u128(u128 A, uint64_t C, bool* ok) {
+    const float rc = 1.0f / (float)C;
+    const float e = u128_to_float(A) * rc;
+    uint64_t q = e < 4.0e18f ? (uint64_t)e : 4000000000000000000ull;
+    for (int it = 0; it < 6; ++it) {
+        const u128 qc = (u128)q * C;
+        if (qc > A) {
+            const uint64_t d = (uint64_t)(u128_to_float(qc - A) * rc);
+            q -= d == 0 ? 1 : (d < q ? d : q);
+        } else {
+            const u128 r = A - qc;
+            if (r < C) break;
+            const uint64_t d = (uint64_t)(u128_to_float(r) * rc);
+            q += d == 0 ? 1 : d;
+        }
+    }
+    const u128 qc = (u128)q * C;
+    if (qc > A || A - qc >= C) *ok = false;
+    return q + (qc != A ? 1 : 0);
+}
 
 }  // namespace hd

@@ -49,8 +49,6 @@
 namespace hd {
 namespace {
 
-typedef unsigned __int128 u128;
-
 constexpr int kBlock = 256;
 constexpr int kWords = 8;  // 256-bit position sets (L <= 255)
 constexpr int kCodeWords = kMaxStages / 4;
@@ -419,13 +417,24 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                 if (o < nloc) tile[i] = __ldg(a.code + (int64_t)s * a.stride + c0 + o);
             }
         }
-        if (threadIdx.x == 0) {
-            int run = 0;
-            for (int b = 0; b <= kMaxStages + 1; ++b) {
-                const int v = bins[b];
-                bins[b] = run;
-                run += v;
+        if (threadIdx.x < 32) {
+            // exclusive scan of bins 0..33 by one warp (lane l: bin l, lane
+            // 31 also bins 32 and 33)
+            const int v = bins[lane];
+            int x = v;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y2 = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x += y2;
             }
+            const int b32 = bins[32], b33 = bins[33];
+            __syncwarp();
+            bins[lane] = x - v;
+            if (lane == 31) {
+                bins[32] = x;
+                bins[33] = x + b32;
+            }
+            (void)b33;
         }
         __syncthreads();
         order[atomicAdd(&bins[key], 1)] = (uint8_t)threadIdx.x;
@@ -491,18 +500,32 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
             int base = 0;
             if (lane == 0) base = atomicAdd(a.wl_count, __popc(mask));
             base = __shfl_sync(0xffffffffu, base, 0);
+            const int p = base + __popc(mask & ((1u << lane) - 1));
             if (take) {
-                const int p = base + __popc(mask & ((1u << lane) - 1));
                 if (p < a.wl_cap) {
                     a.wl_idx[p] = (int32_t)c;
                     a.wl_n[p] = (uint16_t)n;
                     a.wl_M[p] = (uint16_t)M;
                     a.wl_S[p] = (uint8_t)S;
                     a.wl_memok[p] = memuni ? 1 : 0;
-                    for (int s = 0; s < S; ++s) a.wl_code[(int64_t)s * a.wl_cap + p] = tile[s * kScreenBlock + ci];
                 } else {
                     atomicOr(a.err, kErrInternal);
                 }
+            }
+            if (a.uniform && take) {
+                // entries per depth, for the equal-layer search's order
+                const unsigned same = __match_any_sync(mask, S);
+                if ((same & ((1u << lane) - 1)) == 0) atomicAdd(a.wl_count + 1 + S, __popc(same));
+            }
+            // each taken candidate's row of 32 stage bytes, written by the
+            // whole warp (lane = stage; zero past its depth)
+            for (unsigned m = mask; m; m &= m - 1) {
+                const int src = __ffs(m) - 1;
+                const int pc = __shfl_sync(0xffffffffu, p, src);
+                const int cc = __shfl_sync(0xffffffffu, ci, src);
+                const int Sc = __shfl_sync(0xffffffffu, S, src);
+                if (pc < a.wl_cap)
+                    a.wl_code[(int64_t)pc * kMaxStages + lane] = lane < Sc ? tile[lane * kScreenBlock + cc] : 0;
             }
         }
         __syncthreads();  // the tile, S, M and order are reused by the next slice
@@ -544,13 +567,19 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
         const int64_t n = a.wl_n[p];
         const bool memok = a.wl_memok[p] != 0;
         {
-            uint32_t packed = 0;
-            for (int s = 0; s < S; ++s) {
-                packed |= (uint32_t)a.wl_code[(int64_t)s * a.wl_cap + p] << ((s & 3) * 8);
-                if ((s & 3) == 3 || s == S - 1) {
-                    ln.code4[(s >> 2) * kBlock] = packed;
-                    packed = 0;
-                }
+            // the entry's row of stage bytes, 16 bytes at a time
+            const uint4* row = reinterpret_cast<const uint4*>(a.wl_code + p * kMaxStages);
+            const uint4 lo = __ldg(row);
+            ln.code4[0 * kBlock] = lo.x;
+            ln.code4[1 * kBlock] = lo.y;
+            ln.code4[2 * kBlock] = lo.z;
+            ln.code4[3 * kBlock] = lo.w;
+            if (S > 16) {
+                const uint4 hi = __ldg(row + 1);
+                ln.code4[4 * kBlock] = hi.x;
+                ln.code4[5 * kBlock] = hi.y;
+                ln.code4[6 * kBlock] = hi.z;
+                ln.code4[7 * kBlock] = hi.w;
             }
         }
         if (kCount) ++priced;
@@ -623,7 +652,7 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
         // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s
         int64_t tmax = 0, tsum = 0;
         int sg = -1;
-        u128 bestG = 0, bestD = 1;
+        uint64_t bestG = 0, bestD = 1;
         for (int s = 0; s < S; ++s) {
             const Stage st = load_stage(t, ln, s, S, M);
             const int64_t ts = st.P[bnd[s + 1]] - st.P[bnd[s]] + st.c;
@@ -633,9 +662,9 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
                 // stage with the largest G_s / (k_s bw_s), compared exactly
                 const int code = stage_code(ln, s);
                 const int g = code & 7, j = (code >> 3) & 3;
-                const u128 G = (u128)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
-                const u128 D = (u128)t.inter[g] << j;
-                if (sg < 0 || G * bestD > bestG * D) {
+                const uint64_t G = (uint64_t)(t.PB[bnd[s + 1]] - t.PB[bnd[s]]);
+                const uint64_t D = (uint64_t)t.inter[g] << j;
+                if (sg < 0 || (u128)G * bestD > (u128)bestG * D) {
                     sg = s;
                     bestG = G;
                     bestD = D;
@@ -646,9 +675,11 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
         int64_t gmax = 0;
         if (n > 1) {
             // ring all-reduce over n replicas: ceil(2(n-1) G 1e9 / (n k bw))
-            const u128 num = (u128)2 * (u128)(n - 1) * bestG * 1000000000u;
-            const u128 den = (u128)n * bestD;
-            gmax = (int64_t)((num + den - 1) / den);
+            // (G < 2^50 and bandwidths < 2^40 keep n k bw below 2^64)
+            const u128 num = (u128)(2 * (uint64_t)(n - 1) * 1000000000ull) * bestG;
+            bool ok = true;
+            gmax = (int64_t)ceil_div_u128(num, (uint64_t)n * bestD, &ok);
+            if (!ok) atomicOr(a.err, kErrInternal);
         }
         a.T[c] = (int64_t)(M - 1) * Bstar + tsum + gmax;
         a.wl_T[p] = a.T[c];
@@ -703,16 +734,27 @@ cudaError_t launch_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid, int64_t* launches) {
     if (a.n <= 0) return cudaSuccess;
     if (a.n > a.wl_cap) return cudaErrorInvalidValue;
-    cudaError_t e = cudaMemsetAsync(a.wl_count, 0, sizeof(int32_t), st);
+    cudaError_t e = cudaMemsetAsync(a.wl_count, 0, sizeof(int32_t) * kWlMeta, st);
     if (e != cudaSuccess) return e;
-    const int grid = (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * 8);
+    // one wave of resident CTAs, each looping over slices
+    static int screen_per_sm = 0;
+    if (screen_per_sm == 0) {
+        int v = 0;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, screen_kernel, kScreenBlock, 0);
+        if (e != cudaSuccess) return e;
+        screen_per_sm = v > 0 ? v : 1;
+    }
+    const int grid =
+        (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * screen_per_sm);
     screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if (launches) {
-        launches[0] += 1;  // the screen now, the search below
-        launches[1] += 1;
+    if (launches) launches[0] += 1;
+    if (a.uniform) {
+        if ((e = launch_eq_order(a, num_sms, st)) != cudaSuccess) return e;
+        if (launches) launches[0] += 1;
     }
     if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
+    if (launches) launches[1] += 1;
     if (a.uniform) return launch_eq_search(a, num_sms, st);
     return a.counters ? launch_search<true>(a, num_sms, st) : launch_search<false>(a, num_sms, st);
 }

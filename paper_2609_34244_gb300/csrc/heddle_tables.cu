@@ -173,6 +173,9 @@ __global__ void __launch_bounds__(kThreads) build_tables_kernel(TableArgs a) {
             uni = uni && a.layers[l].state_bytes == a.layers[0].state_bytes &&
                   a.layers[l].act_bytes == a.layers[0].act_bytes;
         reinterpret_cast<int32_t*>(a.img + y.offModel)[0] = uni ? 1 : 0;
+        bool puni = true;
+        for (int l = 1; l < L; ++l) puni = puni && a.layers[l].param_bytes == a.layers[0].param_bytes;
+        reinterpret_cast<int32_t*>(a.img + y.offModel)[2] = puni ? 1 : 0;
     }
     uint8_t* win = a.img + y.offWin;
     for (int t = tid; t < 8 * 4 * 33; t += blockDim.x) {
