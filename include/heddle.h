@@ -62,8 +62,9 @@ enum {
 typedef struct heddle_ctx heddle_ctx;
 
 /* Create a context on CUDA device `device`.  Allocates its device scratch
- * once (about 60 MB: the search worklist of 2^20 candidates with their 32
- * stage bytes, and the top-k merge lists) and queries the SM count.
+ * once (about 190 MB: the search worklist of 2^20 candidates with their 32
+ * stage bytes, its per-depth index lists and the top-k merge lists) and
+ * queries the SM count.
  * *out is NULL on failure. */
 heddle_status heddle_create(heddle_ctx** out, int32_t device);
 

@@ -38,7 +38,7 @@ struct heddle_ctx {
     bool count_next = false;
     // search worklist scratch (hd::kWorklistCap candidates)
     int32_t* d_wl_count = nullptr;  // hd::kWlMeta ints
-    int32_t* d_wl_order = nullptr;
+    int32_t* d_wl_bucket = nullptr;  // [32][2^20]
     int32_t* d_wl_idx = nullptr;
     uint16_t* d_wl_n = nullptr;
     uint16_t* d_wl_M = nullptr;
@@ -267,7 +267,7 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch_count, sizeof(int32_t) * x->scratch_blocks);
     const size_t cap = hd::kWorklistCap;
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_count, sizeof(int32_t) * hd::kWlMeta);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_order, sizeof(int32_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_bucket, sizeof(int32_t) * HEDDLE_MAX_STAGES * cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_idx, sizeof(int32_t) * cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_n, sizeof(uint16_t) * cap);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_M, sizeof(uint16_t) * cap);
@@ -298,7 +298,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_scratch);
     cudaFree(x->d_scratch_count);
     cudaFree(x->d_wl_count);
-    cudaFree(x->d_wl_order);
+    cudaFree(x->d_wl_bucket);
     cudaFree(x->d_wl_idx);
     cudaFree(x->d_wl_n);
     cudaFree(x->d_wl_M);
@@ -459,7 +459,7 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     a.wl_S = x->d_wl_S;
     a.wl_memok = x->d_wl_memok;
     a.wl_code = x->d_wl_code;
-    a.wl_order = x->d_wl_order;
+    a.wl_bucket = x->d_wl_bucket;
     a.wl_cap = hd::kWorklistCap;
     a.uniform = equal_layer_search(x) ? 1 : 0;
     a.wl_T = x->d_wl_T;

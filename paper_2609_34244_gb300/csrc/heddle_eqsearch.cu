@@ -27,10 +27,11 @@
 // at B* give the componentwise smallest split -- hence the lexicographically
 // smallest -- a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
 //
-// Scheduling: an order kernel first lists the worklist by decreasing S
-// (the screen counted the entries per depth); each CTA takes 256
-// consecutive entries of that order, so the lanes of a warp run stage loops
-// of equal length and the warps of a CTA carry equal work.  Every
+// Scheduling: the screen files every entry in a bucket per depth S; CTA b
+// takes entries [256 b, 256 b + 256) of the buckets read in order of
+// decreasing S, so the lanes of a warp run stage loops of equal length and
+// the warps of a CTA carry equal work (the search runs in one wave: a deep
+// warp would otherwise hold its whole CTA at the barrier).  Every
 // thread packs its candidate's stages once into 32-bit words (cost index |
 // P2P index | memory run) held in shared memory interleaved by thread, runs
 // the float guess and one exact probe; the few searches still open are
@@ -140,7 +141,7 @@ __device__ __forceinline__ Cap stage_cap(const EqTabs& t, uint32_t w, int64_t B)
         return r;
     }
     // x < m q with m <= 255: the float estimate is off by at most one
-    int k = (int)((float)x * t.rq[w & 31]);
+    int k = (int)(u64_to_float((uint64_t)x) * t.rq[w & 31]);
     if ((int64_t)k * r.q > x) --k;
     if ((int64_t)(k + 1) * r.q <= x) ++k;
     r.k = k;
@@ -261,14 +262,17 @@ __device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
     // else a Newton step, else bisect
     float target;
     if (q.Blo >= 0 && q.Bhi >= 0 && q.chi > q.clo) {
-        target = (float)q.Blo + ((float)t.L - 0.5f - (float)q.clo) / (float)(q.chi - q.clo) * (float)(q.Bhi - q.Blo);
+        target = u64_to_float(q.Blo) +
+                 ((float)t.L - 0.5f - (float)q.clo) / (float)(q.chi - q.clo) * u64_to_float(q.Bhi - q.Blo);
     } else if (p.slope > 0.f) {
-        target = feas ? (float)q.B - ceilf(((float)p.tot - (float)t.L + 0.5f) / p.slope)
-                      : (float)q.B + ceilf(((float)t.L - (float)p.tot) / p.slope);
+        const float Bf = u64_to_float(q.B);
+        target = feas ? Bf - ceilf(((float)p.tot - (float)t.L + 0.5f) / p.slope)
+                      : Bf + ceilf(((float)t.L - (float)p.tot) / p.slope);
     } else {
         target = -1.f;
     }
-    q.B = (target >= (float)q.lo && target <= (float)(q.hi - 1)) ? (int64_t)target : q.lo + (q.hi - q.lo) / 2;
+    q.B = (target >= u64_to_float(q.lo) && target <= u64_to_float(q.hi - 1)) ? (int64_t)float_to_u64(target)
+                                                                                : q.lo + (q.hi - q.lo) / 2;
     if (q.probes > kMaxIters) {
         atomicOr(err, kErrSearchBound);
         q.lo = q.hi;
@@ -371,6 +375,7 @@ template <bool kCount>
 __global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int tail_n;
+    __shared__ int end_of[kMaxStages + 2];  // entries of depths >= S, [S]
     const Layout& y = a.lay;
     const int L = y.L;
     const EqLayout el = eq_layout(L);
@@ -423,6 +428,20 @@ __global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
     Search* tail = reinterpret_cast<Search*>(smem + el.tail);
     uint32_t* mysw = t.sw + threadIdx.x;
 
+    if (threadIdx.x < 32) {
+        // end_of[S] = entries of depths >= S: an inclusive scan of depths
+        // 32 .. 1 in lanes 0 .. 31
+        const int lane = threadIdx.x;
+        int x = a.wl_count[1 + (kMaxStages - lane)];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y2 = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y2;
+        }
+        end_of[kMaxStages - lane] = x;
+        if (lane == 0) end_of[kMaxStages + 1] = 0;
+    }
+    __syncthreads();
     unsigned long long units = 0, probes = 0, searched = 0;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const int64_t count_r = (count + kEqBlock - 1) / kEqBlock * kEqBlock;
@@ -432,8 +451,18 @@ __global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
         //      lanes of a warp (and the warps of a CTA) have nearly equal S
         if (threadIdx.x == 0) tail_n = 0;
         __syncthreads();
-        const bool have = base + threadIdx.x < count;
-        const int64_t p = have ? a.wl_order[base + threadIdx.x] : 0;
+        const int64_t g = base + threadIdx.x;
+        const bool have = g < count;
+        int64_t p = 0;
+        if (have) {
+            // its depth: the largest S with end_of[S] > g (end_of falls with S)
+            int lo = 1, hi = kMaxStages;
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (end_of[mid] > g) lo = mid; else hi = mid - 1;
+            }
+            p = a.wl_bucket[(int64_t)(lo - 1) * a.wl_cap + (g - end_of[lo + 1])];
+        }
 
         int S = 0, M = 0;
         int64_t n = 0;
@@ -480,17 +509,18 @@ __global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
                 cw += t.cf[(w >> 5) & 255] * rq;
             }
             // first guess: Newton on the saturating continuous count
-            float Bf = fmaxf((float)q.lo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : (float)q.lo);
+            const float flo = u64_to_float(q.lo), fhi = u64_to_float(q.hi);
+            float Bf = fmaxf(flo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : flo);
             for (int it = 0; it < 8; ++it) {
                 float sl;
                 int below;
-                Bf = fminf(Bf, (float)q.hi);
+                Bf = fminf(Bf, fhi);
                 const float cnt = eq_count(t, mysw, S, Bf, sl, below);
                 const float tgt = (float)L + 0.5f * (float)below;
                 if (cnt >= tgt - 0.25f || sl <= 0.f) break;
                 Bf += (tgt - cnt) / sl;
             }
-            q.B = (int64_t)fminf(Bf, (float)q.hi);
+            q.B = (int64_t)float_to_u64(fminf(Bf, fhi));
             q.Blo = q.Bhi = q.fhi = -1;
             q.clo = q.chi = 0;
             q.fset = -1;
@@ -555,46 +585,6 @@ __global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
     }
 }
 
-// The worklist in order of decreasing S: entry p goes to the start of its
-// depth's range (the entries of larger depths come first) plus a cursor
-// (warp-aggregated atomics); the order within a depth is immaterial.
-__global__ void __launch_bounds__(256) order_kernel(PriceArgs a) {
-    __shared__ int start[kMaxStages + 1];
-    if (threadIdx.x < 32) {
-        // start of depth S = entries of depths above S: an inclusive scan
-        // of depths 32 .. 1 in lanes 0 .. 31 (depth 0 never enters)
-        const int lane = threadIdx.x;
-        const int v = a.wl_count[1 + (kMaxStages - lane)];
-        int x = v;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(0xffffffffu, x, o);
-            if (lane >= o) x += y;
-        }
-        start[kMaxStages - lane] = x - v;
-        if (lane == 31) start[0] = x;
-    }
-    __syncthreads();
-    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t n_round = (count + 31) & ~(int64_t)31;
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < n_round;
-         p += (int64_t)gridDim.x * blockDim.x) {
-        const bool live = p < count;
-        const int S = live ? a.wl_S[p] : -1;
-        const unsigned mask = __ballot_sync(0xffffffffu, live);
-        if (!live) continue;
-        const unsigned same = __match_any_sync(mask, S);
-        const int lane = threadIdx.x & 31;
-        const int leader = __ffs(same) - 1;
-        int pos = 0;
-        if (lane == leader) pos = atomicAdd(a.wl_count + 1 + (kMaxStages + 1) + S, __popc(same));
-        pos = __shfl_sync(same, pos, leader) + __popc(same & ((1u << lane) - 1));
-        const int64_t dst = (int64_t)start[S] + pos;
-        if (dst < count) a.wl_order[dst] = (int32_t)p;
-        else atomicOr(a.err, kErrInternal);
-    }
-}
-
 template <bool kCount>
 cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const size_t smem = eq_layout(a.lay.L).bytes;
@@ -613,12 +603,6 @@ cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
 }
 
 }  // namespace
-
-cudaError_t launch_eq_order(const PriceArgs& a, int num_sms, cudaStream_t st) {
-    const int grid = (int)std::min<int64_t>((a.n + 255) / 256, (int64_t)num_sms * 8);
-    order_kernel<<<grid, 256, 0, st>>>(a);
-    return cudaGetLastError();
-}
 
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
     return a.counters ? launch<true>(a, num_sms, st) : launch<false>(a, num_sms, st);

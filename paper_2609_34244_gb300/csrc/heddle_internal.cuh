@@ -115,15 +115,16 @@ struct PriceArgs {
     unsigned long long* counters;  // non-null selects the counting variant
     // worklist of the candidates that need the threshold search (device
     // scratch owned by the context, capacity wl_cap candidates)
-    int32_t* wl_count;   // [1 + 2 (kMaxStages + 1)]: entries, then per depth S the
-                         // entries of that depth and an order cursor (cleared per chunk)
+    int32_t* wl_count;   // [1 + kMaxStages + 1]: entries, then per depth S the entries of
+                         // that depth (equal-layer search; cleared per chunk)
     int32_t* wl_idx;
     uint16_t* wl_n;
     uint16_t* wl_M;
     uint8_t* wl_S;
     uint8_t* wl_memok;   // 1: memory feasibility already decided by the screen
     uint8_t* wl_code;    // [wl_cap][kMaxStages] stage bytes, a 32-byte row per entry (zero past S)
-    int32_t* wl_order;   // [wl_cap] entries by decreasing S (equal-layer search)
+    int32_t* wl_bucket;  // [kMaxStages][wl_cap]: per depth S (row S - 1) the entries of
+                         // that depth, in any order (equal-layer search)
     int32_t wl_cap;
     int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
     // per worklist entry, written by the search: T (-1 unless OK) and n * M,
@@ -137,11 +138,9 @@ struct PriceArgs {
 cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid = nullptr,
                          int64_t* launches = nullptr);
 // The equal-layer search over the worklist the screen produced.
-// (after launch_eq_order, which orders the worklist by decreasing S)
-cudaError_t launch_eq_order(const PriceArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
-constexpr int kWlMeta = 1 + 2 * (kMaxStages + 1);  // ints of a.wl_count
+constexpr int kWlMeta = 1 + kMaxStages + 1;  // ints of a.wl_count
 
 
 struct TopkArgs {
@@ -174,27 +173,43 @@ cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cuda
                                  int64_t* launches = nullptr);
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st);
 
+// Conversions between non-negative 64-bit integers and float through their
+// 32-bit halves: the 32-bit conversions run on the fast pipes, while a
+// 64-bit conversion instruction runs on the (narrow) FP64 pipe.
+// u64_to_float: relative error below 2^-23.
+__device__ __forceinline__ float u64_to_float(uint64_t x) {
+    return __fmaf_rn((float)(uint32_t)(x >> 32), 4294967296.0f, (float)(uint32_t)x);
+}
+
+// Truncation of a float in [0, 2^63) to an integer (exact: the low part
+// f - hi 2^32 is representable).
+__device__ __forceinline__ uint64_t float_to_u64(float f) {
+    const float hi = floorf(f * 2.3283064365386963e-10f);
+    const float lo = __fmaf_rn(-hi, 4294967296.0f, f);
+    return ((uint64_t)(uint32_t)hi << 32) + (uint64_t)(uint32_t)fmaxf(lo, 0.f);
+}
+
 // ceil(A / C) for a 128-bit A and 1 <= C < 2^64 whose quotient is below
 // 2^62: a float estimate of the quotient refined with exact 128-bit
 // remainders (each refinement leaves about 2^-22 of the error), then exact
 // unit steps.  *ok is cleared if the steps did not settle (never expected).
 __device__ __forceinline__ float u128_to_float(u128 v) {
-    return (float)(uint64_t)(v >> 64) * 18446744073709551616.0f + (float)(uint64_t)v;
+    return __fmaf_rn(u64_to_float((uint64_t)(v >> 64)), 18446744073709551616.0f, u64_to_float((uint64_t)v));
 }
 
 __device__ inline uint64_t ceil_div_u128(u128 A, uint64_t C, bool* ok) {
-    const float rc = 1.0f / (float)C;
+    const float rc = 1.0f / u64_to_float(C);
     const float e = u128_to_float(A) * rc;
-    uint64_t q = e < 4.0e18f ? (uint64_t)e : 4000000000000000000ull;
+    uint64_t q = e < 4.0e18f ? float_to_u64(e) : 4000000000000000000ull;
     for (int it = 0; it < 6; ++it) {
         const u128 qc = (u128)q * C;
         if (qc > A) {
-            const uint64_t d = (uint64_t)(u128_to_float(qc - A) * rc);
+            const uint64_t d = float_to_u64(u128_to_float(qc - A) * rc);
             q -= d == 0 ? 1 : (d < q ? d : q);
         } else {
             const u128 r = A - qc;
             if (r < C) break;
-            const uint64_t d = (uint64_t)(u128_to_float(r) * rc);
+            const uint64_t d = float_to_u64(u128_to_float(r) * rc);
             q += d == 0 ? 1 : d;
         }
     }

@@ -513,9 +513,14 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                 }
             }
             if (a.uniform && take) {
-                // entries per depth, for the equal-layer search's order
+                // the entry in its depth's bucket, for the equal-layer
+                // search's order by decreasing depth
                 const unsigned same = __match_any_sync(mask, S);
-                if ((same & ((1u << lane) - 1)) == 0) atomicAdd(a.wl_count + 1 + S, __popc(same));
+                const int leader = __ffs(same) - 1;
+                int b0 = 0;
+                if (lane == leader) b0 = atomicAdd(a.wl_count + 1 + S, __popc(same));
+                const int bpos = __shfl_sync(same, b0, leader) + __popc(same & ((1u << lane) - 1));
+                if (p < a.wl_cap && bpos < a.wl_cap) a.wl_bucket[(int64_t)(S - 1) * a.wl_cap + bpos] = p;
             }
             // each taken candidate's row of 32 stage bytes, written by the
             // whole warp (lane = stage; zero past its depth)
@@ -749,10 +754,6 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
     screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (launches) launches[0] += 1;
-    if (a.uniform) {
-        if ((e = launch_eq_order(a, num_sms, st)) != cudaSuccess) return e;
-        if (launches) launches[0] += 1;
-    }
     if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
     if (launches) launches[1] += 1;
     if (a.uniform) return launch_eq_search(a, num_sms, st);

@@ -3,11 +3,11 @@
 // The rank order and the warp-level lists are in heddle_rank.cuh.
 //
 // Launch 1: every CTA scans a slice of the batch (or, after a pricing call,
-// of the worklist of searched candidates only); each warp keeps its own
-// sorted list in shared memory (an entry is inserted only if it beats the
-// current k-th, which after warm-up is rare), the CTA merges its warps'
-// lists (a tree of parallel two-list merges) and writes one list to
-// scratch.  Then the per-CTA lists are folded into the state by merge
+// of the worklist of searched candidates only); an entry that does not beat
+// the incoming state's k-th is dropped at once, the others are offered to
+// the warp's sorted list in shared memory (inserted only if they beat its
+// current k-th), the CTA merges its warps' lists (a tree of parallel
+// two-list merges) and writes one list to scratch.  Then the per-CTA lists are folded into the state by merge
 // levels of 16 lists per CTA: one level for up to 16 lists, else two.  No
 // CTA waits on another.
 
@@ -43,26 +43,36 @@ __device__ __forceinline__ bool fetch(const TopkArgs& a, int64_t i, TopkEntry& e
     return true;
 }
 
-template <bool kWorklist>
-__global__ void __launch_bounds__(kTopkBlock) topk_block_kernel(TopkArgs a) {
+// Entries that do not beat the incoming state's k-th entry (when it holds
+// k) cannot enter the merged top-k, so they are not offered: after the
+// first batches almost every entry stops at this one comparison.
+template <bool kWorklist, int kBlock>
+__global__ void __launch_bounds__(kBlock) topk_block_kernel(TopkArgs a) {
+    constexpr int W = kBlock / 32;
     const int k = state_k(a.state);
-    __shared__ TopkEntry lists[kWarps * kMaxTopK];
-    __shared__ TopkEntry tmp[(kWarps / 2) * kMaxTopK];
-    __shared__ int counts[kWarps], tmp_counts[kWarps / 2];
+    __shared__ TopkEntry lists[W * kMaxTopK];
+    __shared__ TopkEntry tmp[(W / 2) * kMaxTopK];
+    __shared__ int counts[W], tmp_counts[W / 2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool full = a.state->count >= k;
+    TopkEntry bar;
+    bar.idx = full ? a.state->idx[k - 1] : 0;
+    bar.T = full ? a.state->T[k - 1] : 0;
+    bar.nM = full ? a.state->nM[k - 1] : 0;
+    bar.pad = 0;
     int cnt = 0;
     TopkEntry* list = lists + warp * kMaxTopK;
     const int64_t n = kWorklist ? min((int64_t)*a.wl_count, (int64_t)a.wl_cap) : a.n;
-    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
+    const int64_t nwarps = (int64_t)gridDim.x * W;
+    const int64_t gw = (int64_t)blockIdx.x * W + warp;
     for (int64_t base = gw * 32; base < n; base += nwarps * 32) {
         const int64_t i = base + lane;
         TopkEntry e;
-        const bool valid = i < n && fetch<kWorklist>(a, i, e);
+        const bool valid = i < n && fetch<kWorklist>(a, i, e) && (!full || better(e, bar));
         warp_offer(list, cnt, k, valid, e);
     }
     if (lane == 0) counts[warp] = cnt;
-    cta_tree_merge(lists, counts, tmp, tmp_counts, kWarps, k);
+    cta_tree_merge(lists, counts, tmp, tmp_counts, W, k);
     for (int p = threadIdx.x; p < counts[0]; p += blockDim.x)
         a.scratch[(size_t)blockIdx.x * kMaxTopK + p] = lists[p];
     if (threadIdx.x == 0) a.scratch_count[blockIdx.x] = counts[0];
@@ -155,7 +165,7 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t
     int grid = (int)std::min<int64_t>((a.n + per_block - 1) / per_block, (int64_t)kFan * kFan);
     grid = std::max(1, std::min(grid, a.max_blocks));
     (void)num_sms;
-    topk_block_kernel<false><<<grid, kTopkBlock, 0, st>>>(a);
+    topk_block_kernel<false, kTopkBlock><<<grid, kTopkBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (launches) *launches += 1;
@@ -165,11 +175,14 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t
 cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st,
                                  int64_t* launches) {
     if (n <= 0) return cudaSuccess;
-    const int64_t per_block = (int64_t)kTopkBlock * 16;
-    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)kFan * kFan);
+    // at most kFan CTAs of 512 threads: one merge level (the worklist holds
+    // only the searched candidates, mostly rejected by the state's k-th)
+    constexpr int kWlBlock = 512;
+    const int64_t per_block = (int64_t)kWlBlock * 16;
+    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)kFan);
     grid = std::max(1, std::min(grid, a.max_blocks));
     (void)num_sms;
-    topk_block_kernel<true><<<grid, kTopkBlock, 0, st>>>(a);
+    topk_block_kernel<true, kWlBlock><<<grid, kWlBlock, 0, st>>>(a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (launches) *launches += 1;
