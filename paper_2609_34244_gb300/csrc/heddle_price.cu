@@ -297,14 +297,6 @@ __device__ bool probe(const Tabs& t, const Lane& ln, int S, int M, int64_t B, Sn
     return judge(st0, st0.P[0], t.SA[0], st0.P[nmin], t.SA[nmin], B, sn) == 0;
 }
 
-// floor(a / b) for 0 <= a < 2^24, 1 <= b < 2^16: float estimate, integer fix-up
-__device__ __forceinline__ int64_t small_div(int64_t a, int64_t b) {
-    int64_t q = (int64_t)((float)a * __frcp_rn((float)b));
-    while (q > 0 && q * b > a) --q;
-    while ((q + 1) * b <= a) ++q;
-    return q;
-}
-
 __device__ void bind_tables(Tabs& t, const unsigned char* img, const Layout& y) {
     t.P = reinterpret_cast<const int64_t*>(img + y.offP);
     t.SA = reinterpret_cast<const longlong2*>(img + y.offSA);
@@ -595,9 +587,9 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
         for (int s = 0; s < S; ++s) {
             const Stage st = load_stage(t, ln, s, S, M);
             hi = max(hi, st.P[L] + st.c);
-            const float tot = (float)st.P[L] + 1.0f;
+            const float tot = u64_to_float(st.P[L]) + 1.0f;
             inv += 1.0f / tot;
-            cw += (float)st.c / tot;
+            cw += u64_to_float(st.c) / tot;
         }
         if (!memok) {
             // memory-only probe decides OOM and gives a tighter upper bound
@@ -612,8 +604,8 @@ __global__ void __launch_bounds__(kBlock) search_kernel(PriceArgs a) {
         // ---- PartitionLayers: threshold search from the balanced guess
         int64_t lo = 0;
         bool lo_known = false, hi_known = false;
-        int64_t B = (int64_t)((1.0f + cw) / inv);
-        int64_t step = max((int64_t)1, (int64_t)((float)B * (float)S / (2.0f * (float)L)));
+        int64_t B = (int64_t)float_to_u64((1.0f + cw) / inv);
+        int64_t step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
         int it = 0;
         while (lo < hi) {
             B = min(max(B, lo), hi - 1);
