@@ -168,3 +168,56 @@ def replicas(node_gpus, group_gpus) -> int:
     ng = np.ascontiguousarray(node_gpus, dtype=np.int32)
     gg = np.ascontiguousarray(group_gpus, dtype=np.int32)
     return int(lib().orc_replicas(len(ng), _ptr(ng), len(gg), _ptr(gg)))
+
+
+# ------------------------------------------------------- micro-batch fill
+
+def level_model(model: dict, level: int, profile_s=None) -> dict:
+    """The model at micro-batch size 2**level times the base size (§5.3
+    "Micro-batch size"): every quantity that grows with the tokens of a
+    micro-batch -- FLOPs, stored activations, the TP all-reduce and EP
+    all-to-all messages, the stage-boundary activation -- scales by
+    2**level; parameter, gradient and optimizer-state bytes do not.
+    ``profile_s`` (seconds per layer at this size, [types][4][L]) replaces
+    the synthetic compute formula when given."""
+    f = 1 << level
+    out = dict(model)
+    out["flops"] = np.asarray(model["flops"], np.float64) * float(f)
+    for k in ("act_bytes", "ar_bytes", "a2a_bytes"):
+        out[k] = np.asarray(model[k], np.int64) * f
+    out["boundary_bytes"] = int(model["boundary_bytes"]) * f
+    out["profile_s"] = None if profile_s is None else np.ascontiguousarray(profile_s, np.float64)
+    return out
+
+
+def price_mbs(cluster: dict, model: dict, cands: dict, levels: int, profiles=None, threads: int = 1,
+              bounds: bool = True) -> dict:
+    """Micro-batch-size fill (§5.3): price every candidate at micro-batch
+    sizes 2**i times the base size, i = 0 .. levels-1, and keep the size
+    with the shortest iteration time (ties: the smaller size).  A replica
+    still processes M base micro-batches per iteration, so at size 2**i it
+    runs M / 2**i micro-batches; a size that does not divide M is not
+    priced for that candidate.  The size that fits nowhere makes no
+    difference: a candidate that fits at no size keeps the base size's
+    status.  Returns the fields of ``Oracle.price`` plus ``mbs`` (the chosen
+    i; 0 for candidates that are not OK)."""
+    M = np.asarray(cands["M"], dtype=np.int64)
+    best = None
+    for i in range(levels):
+        prof = None if profiles is None else profiles[i]
+        orc = Oracle(cluster, level_model(model, i, prof))
+        div = (M % (1 << i)) == 0
+        ci = dict(cands)
+        ci["M"] = np.where(div, M >> i, 0).astype(np.uint16)  # M = 0 is INVALID
+        r = orc.price(ci, threads=threads, bounds=bounds)
+        if best is None:
+            best = {k: (v.copy() if isinstance(v, np.ndarray) else v) for k, v in r.items()}
+            best["mbs"] = np.zeros(len(M), np.uint8)
+            continue
+        take = (r["status"] == OK) & ((best["status"] != OK) | (r["T"] < best["T"]))
+        for k in ("T", "bottleneck", "n_dp", "status"):
+            best[k][take] = r[k][take]
+        if bounds:
+            best["bounds"][:, take] = r["bounds"][:, take]
+        best["mbs"][take] = i
+    return best

@@ -330,6 +330,30 @@ CONFIGS = {
 }
 
 
+def mbs_profiles(w, levels: int, seed: int = 0):
+    """Seeded per-size layer profiles for the micro-batch-size fill: a list
+    of ``levels`` arrays [types][4][L] of seconds per layer at micro-batch
+    2**i times the base size and TP degree 2**j.  The paper profiles every
+    size on real GPUs (§5.3, "the profiled powers of two"); this stand-in
+    draws per type a base time tau_g ~ U(0.5, 2) ms and a per-doubling
+    efficiency rho_g ~ U(0.6, 0.95) (a larger micro-batch uses the GPU
+    better), weights layer l by its share of the model's FLOPs, and sets
+    t = tau_g * w_l * (1 + 0.15 j) / 2**j * (2 rho_g)**i."""
+    rng = np.random.default_rng(0x5EED0 + seed)
+    NT = int(w.cluster["tflops"].shape[0])
+    fl = np.asarray(w.model["flops"], np.float64)
+    wl = fl / fl.mean() if fl.mean() > 0 else np.ones_like(fl)
+    tau = rng.uniform(0.5e-3, 2e-3, NT)
+    rho = rng.uniform(0.6, 0.95, NT)
+    j = np.arange(4, dtype=np.float64)
+    out = []
+    for i in range(levels):
+        t = (tau[:, None, None] * (1.0 + 0.15 * j)[None, :, None] / (2.0 ** j)[None, :, None]
+             * wl[None, None, :] * ((2.0 * rho) ** i)[:, None, None])
+        out.append(np.ascontiguousarray(t))
+    return out
+
+
 def make_workload(name: str, seed: int = 0, n: int | None = None) -> Workload:
     """Build the named workload; ``n`` overrides the candidate count (same
     cluster, model and candidate distribution)."""

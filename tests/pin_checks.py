@@ -329,6 +329,58 @@ def check_status_rules(O):
     assert r["status"].tolist() == [3, 3, 0, 3, 3, 3, 3, 0, 0], r["status"]
 
 
+def check_mbs_hand(O):
+    """Hand-worked micro-batch-size fill (golden/hand_mbs.json, §5.3)."""
+    W = _workloads()
+    d = _load("hand_mbs.json")
+    cl, m = d["cluster"], d["model"]
+    L = m["L"]
+    for case in d["cases"]:
+        cluster = W.make_cluster(cl["tflops"], [case["mem_bytes"]], cl["intra_bw"],
+                                 [tuple(x) for x in cl["nodes"]])
+        model = W.make_model([m["flops"]] * L, m["param_bytes"], m["state_bytes"], m["act_bytes"],
+                             m["ar_bytes"], m["a2a_bytes"], case.get("boundary_bytes", m["boundary_bytes"]))
+        if case["level_ms"] is None:
+            levels, profiles = case["levels"], None
+        else:
+            levels = len(case["level_ms"])
+            profiles = [np.full((1, 4, L), ms / 1000.0) for ms in case["level_ms"]]
+        cands = W.from_structures([[(0, 0), (0, 0)]], [case["M"]])
+        r = O.price_mbs(cluster, model, cands, levels, profiles)
+        e = case["expect"]
+        name = case["name"]
+        assert int(r["status"][0]) == e["status"], (name, r["status"][0])
+        assert int(r["mbs"][0]) == e["mbs"], (name, r["mbs"][0])
+        assert int(r["T"][0]) == e["T"], (name, r["T"][0])
+        assert int(r["bottleneck"][0]) == e["bottleneck"], (name, r["bottleneck"][0])
+        if e["bounds"] is not None:
+            assert r["bounds"][:3, 0].tolist() == e["bounds"], (name, r["bounds"][:3, 0])
+
+
+def check_mbs_properties(O, seed=11):
+    """Properties of the fill on seeded workloads with per-size profiles:
+    stored activations grow with the size at fixed micro-batches per
+    iteration, so a candidate that does not fit at the base size fits at no
+    size; a one-size fill is the plain price; the chosen size divides M."""
+    W = _workloads()
+    for name, n in (("dense32", 3000), ("moe48", 3000)):
+        w = W.make_workload(name, seed=seed, n=n)
+        prof = W.mbs_profiles(w, 3, seed=seed)
+        plain = O.Oracle(w.cluster, O.level_model(w.model, 0, prof[0])).price(w.cands)
+        one = O.price_mbs(w.cluster, w.model, w.cands, 1, prof[:1])
+        for k in ("T", "bottleneck", "n_dp", "status"):
+            assert (one[k] == plain[k]).all(), (name, k)
+        r = O.price_mbs(w.cluster, w.model, w.cands, 3, prof)
+        assert not ((plain["status"] == O.OOM) & (r["status"] == O.OK)).any(), name
+        assert ((r["status"] == O.OK) | (r["status"] == plain["status"])).all(), name
+        M = np.asarray(w.cands["M"], np.int64)
+        assert ((M % (1 << r["mbs"].astype(np.int64))) == 0).all(), name
+        ok = r["status"] == O.OK
+        assert (r["T"][ok & (plain["status"] == O.OK)] <= plain["T"][ok & (plain["status"] == O.OK)]).all(), name
+        if name == "dense32":  # 11% OK: some candidate gains from a larger size
+            assert (r["mbs"] > 0).any(), (name, "a larger size wins somewhere")
+
+
 ALL_CHECKS = [
     check_hand_partitions,
     check_hand_pricing,
@@ -339,4 +391,6 @@ ALL_CHECKS = [
     check_layer_cost_formula,
     check_invariants,
     check_status_rules,
+    check_mbs_hand,
+    check_mbs_properties,
 ]

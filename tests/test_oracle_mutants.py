@@ -59,10 +59,30 @@ MUTANTS = [
     ("compute_ignores_degree", "double s = flops / (k * tflops * 1e12);", "double s = flops / (tflops * 1e12);"),
 ]
 
+# planted mistakes in the Python part of the oracle (the micro-batch fill)
+PY_SRC = os.path.join(ROOT, "oracle", "oracle.py")
+PY_MUTANTS = [
+    ("mbs_flops_not_scaled", 'out["flops"] = np.asarray(model["flops"], np.float64) * float(f)',
+     'out["flops"] = np.asarray(model["flops"], np.float64)'),
+    ("mbs_act_not_scaled", 'for k in ("act_bytes", "ar_bytes", "a2a_bytes"):', 'for k in ("ar_bytes", "a2a_bytes"):'),
+    ("mbs_boundary_not_scaled", 'out["boundary_bytes"] = int(model["boundary_bytes"]) * f',
+     'out["boundary_bytes"] = int(model["boundary_bytes"])'),
+    ("mbs_tie_to_larger", '(r["T"] < best["T"])', '(r["T"] <= best["T"])'),
+    ("mbs_no_divisibility", 'ci["M"] = np.where(div, M >> i, 0).astype(np.uint16)',
+     'ci["M"] = np.maximum(M >> i, 1).astype(np.uint16)'),
+    ("mbs_M_not_divided", "np.where(div, M >> i, 0)", "np.where(div, M, 0)"),
+]
+
 CHILD = r"""
-import json, sys, traceback
+import json, sys, traceback, types
 sys.path[:0] = [sys.argv[1], sys.argv[1] + "/tests"]
 from oracle import oracle as O
+if len(sys.argv) > 3:
+    # a planted mistake in oracle.py: run the mutated source as the module
+    M = types.ModuleType("oracle_mutant")
+    M.__dict__["__file__"] = O.__file__
+    exec(compile(open(sys.argv[3]).read(), O.__file__, "exec"), M.__dict__)
+    O = M
 O.LIB = sys.argv[2]
 O.build = lambda force=False: O.LIB
 import pin_checks as P
@@ -87,10 +107,10 @@ def _compile(dirpath, text):
     return lib
 
 
-def _run_pins(lib):
+def _run_pins(lib, py_src=None):
     try:
-        p = subprocess.run([sys.executable, "-c", CHILD, ROOT, lib], capture_output=True,
-                           text=True, timeout=300)
+        p = subprocess.run([sys.executable, "-c", CHILD, ROOT, lib] + ([py_src] if py_src else []),
+                           capture_output=True, text=True, timeout=300)
     except subprocess.TimeoutExpired:
         return ["<timeout>"]
     for line in p.stdout.splitlines():
@@ -111,4 +131,18 @@ def test_mutant_is_caught(tmp_path, name, old, new):
         text = f.read()
     assert text.count(old) == 1, "mutation site not unique: " + name
     failed = _run_pins(_compile(str(tmp_path), text.replace(old, new)))
+    assert failed, "no pin catches mutant " + name
+
+
+@pytest.mark.parametrize("name,old,new", PY_MUTANTS, ids=[m[0] for m in PY_MUTANTS])
+def test_python_mutant_is_caught(tmp_path, name, old, new):
+    with open(SRC) as f:
+        lib = _compile(str(tmp_path), f.read())
+    with open(PY_SRC) as f:
+        text = f.read()
+    assert text.count(old) == 1, "mutation site not unique: " + name
+    py = os.path.join(str(tmp_path), "oracle_mutant.py")
+    with open(py, "w") as f:
+        f.write(text.replace(old, new))
+    failed = _run_pins(lib, py)
     assert failed, "no pin catches mutant " + name
