@@ -265,6 +265,45 @@ heddle_status heddle_price_topk(heddle_ctx* ctx, const heddle_candidates* cands,
 heddle_status heddle_topk_noalloc(const heddle_candidates* cands, const heddle_results* results,
                                   heddle_topk_state* state, void* stream);
 
+/* --------------------------------------------- micro-batch-size fill */
+
+/* §5.3 "Micro-batch size": the micro-batch size comes from the profiled
+ * powers of two; every size that fits memory is priced and the one with the
+ * shortest iteration time is kept.  The loaded model describes one
+ * micro-batch of the base size b0; level i is the size 2^i b0.
+ *
+ * heddle_load_mbs(ctx, levels, profile_s) prepares levels 0 .. levels-1
+ * (1 <= levels <= HEDDLE_MAX_MBS_LEVELS; 0 forgets them) and builds their
+ * cost tables (synchronous).  At level i the per-layer FLOPs, stored
+ * activations, TP all-reduce and EP all-to-all messages and the boundary
+ * activation are 2^i times the model's; parameter, gradient and state
+ * bytes are unchanged.  profile_s (nullable, host, copied) gives seconds
+ * per layer for every level: [levels][n_types][4][n_layers], degree 2^j, as
+ * the profile of heddle_load_model; without it the synthetic formula runs
+ * on the scaled FLOPs and messages (E_STATE if the model itself was loaded
+ * with a profile).  The levels are rebuilt when the cluster or model is
+ * reloaded (their profile must still match the sizes).  Errors: E_ARG
+ * (non-finite or negative profile entry), E_STATE, E_LIMIT (a scaled byte
+ * count above 2^42, a table total above its limit), E_CUDA.
+ *
+ * heddle_price_mbs(ctx, cands, results, mbs, stream) prices every candidate
+ * at every level: at level i a replica still processes M base micro-batches
+ * per iteration, as M / 2^i micro-batches of size 2^i b0, and a level whose
+ * size does not divide M is not priced for that candidate.  Each result row
+ * holds the level with the smallest T among the levels where the candidate
+ * is OK (equal T: the smaller level); a candidate OK at no level keeps the
+ * base level's status (memory grows with the size, so a candidate that does
+ * not fit at the base size fits at none).  mbs (nullable, device u8[n])
+ * receives the chosen level (0 when not OK).  The throughput key of
+ * heddle_topk stays n * M / T: M base micro-batches per iteration at any
+ * size.  Asynchronous on `stream`; device buffers as heddle_price_candidates
+ * (which keeps pricing the base size only).  Errors: E_ARG, E_STATE (no
+ * levels loaded), E_CUDA. */
+#define HEDDLE_MAX_MBS_LEVELS 4
+heddle_status heddle_load_mbs(heddle_ctx* ctx, int32_t levels, const double* profile_s);
+heddle_status heddle_price_mbs(heddle_ctx* ctx, const heddle_candidates* cands,
+                               const heddle_results* results, uint8_t* mbs, void* stream);
+
 /* -------------------------------------------------------- host buffers */
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the

@@ -6,6 +6,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <vector>
 
 #include "heddle_internal.cuh"
@@ -78,6 +79,26 @@ struct heddle_ctx {
         int64_t launches[3];
     };
     std::vector<PhaseRec> phase_recs;
+    // micro-batch-size fill: one cost-table image per size 2^i (level i),
+    // and the results of one level for one chunk
+    struct Level {
+        Layout lay{};
+        unsigned char* img = nullptr;
+        size_t img_cap = 0;
+        int64_t* q = nullptr;
+        size_t q_cap = 0;
+        int32_t flags[4] = {0, 0, 0, 0};
+    };
+    int32_t mbs_levels = 0;
+    std::vector<double> mbs_profile;  // [levels][types][4][L] seconds, or empty
+    bool mbs_ready = false;
+    Level lv[HEDDLE_MAX_MBS_LEVELS];
+    int64_t* lv_T = nullptr;
+    int64_t* lv_B = nullptr;
+    uint16_t* lv_n = nullptr;
+    uint8_t* lv_status = nullptr;
+    uint8_t* lv_bounds = nullptr;
+    size_t lv_T_cap = 0, lv_B_cap = 0, lv_n_cap = 0, lv_status_cap = 0, lv_bounds_cap = 0;
 };
 
 namespace {
@@ -133,18 +154,16 @@ constexpr int64_t kByteLimit = (int64_t)1 << 42;
 constexpr int64_t kBwLimit = (int64_t)1 << 40;
 constexpr int64_t kMemLimit = (int64_t)1 << 50;
 
-heddle_status build_tables(heddle_ctx* x) {
-    x->tables_ready = false;
-    if (!x->have_cluster || !x->have_model) return ok(x);
-    const int NT = (int)x->types.size(), L = (int)x->layers.size();
-    if (x->have_profile && x->profile.size() != (size_t)NT * 4 * L)
-        return fail(x, HEDDLE_E_STATE,
-                    "model profile covers %zu entries, cluster needs %d types x 4 x %d layers",
-                    x->profile.size(), NT, L);
+// Build one cost-table image (and its per-layer cost table) for the given
+// layers, profile (nullable: the synthetic formula) and boundary bytes.
+heddle_status build_image(heddle_ctx* x, const std::vector<heddle_layer>& layers, const double* profile,
+                          int64_t boundary_bytes, Layout& lay, unsigned char** img, size_t* img_cap,
+                          int64_t** qtab, size_t* q_cap, int32_t model_flags[4]) {
+    const int NT = (int)x->types.size(), L = (int)layers.size();
     // the gradient term stays below 2^56 ns: 2 * sum(param) * 1e9 / slowest NIC
     {
         unsigned __int128 G = 0;
-        for (const auto& ly : x->layers) G += (unsigned __int128)ly.param_bytes;
+        for (const auto& ly : layers) G += (unsigned __int128)ly.param_bytes;
         for (int g = 0; g < NT; ++g) {
             int64_t nic = INT64_MAX;
             for (const auto& nd : x->nodes)
@@ -155,9 +174,9 @@ heddle_status build_tables(heddle_ctx* x) {
                 return fail(x, HEDDLE_E_LIMIT, "gradient synchronisation of type %d exceeds 2^56 ns", g);
         }
     }
-    x->lay = hd::make_layout(L, NT);
-    CU(grow(&x->d_img, &x->img_cap, x->lay.bytes));
-    CU(grow(&x->d_q, &x->q_cap, sizeof(int64_t) * (size_t)NT * 4 * L));
+    lay = hd::make_layout(L, NT);
+    CU(grow(img, img_cap, lay.bytes));
+    CU(grow(qtab, q_cap, sizeof(int64_t) * (size_t)NT * 4 * L));
     heddle_gpu_type* d_types = nullptr;
     heddle_node* d_nodes = nullptr;
     heddle_layer* d_layers = nullptr;
@@ -165,31 +184,30 @@ heddle_status build_tables(heddle_ctx* x) {
     cudaError_t e = cudaMalloc(&d_types, sizeof(heddle_gpu_type) * NT);
     if (e == cudaSuccess) e = cudaMalloc(&d_nodes, sizeof(heddle_node) * x->nodes.size());
     if (e == cudaSuccess) e = cudaMalloc(&d_layers, sizeof(heddle_layer) * L);
-    if (e == cudaSuccess && x->have_profile) e = cudaMalloc(&d_prof, sizeof(double) * x->profile.size());
+    const size_t nprof = (size_t)NT * 4 * L;
+    if (e == cudaSuccess && profile) e = cudaMalloc(&d_prof, sizeof(double) * nprof);
     if (e == cudaSuccess)
         e = cudaMemcpy(d_types, x->types.data(), sizeof(heddle_gpu_type) * NT, cudaMemcpyHostToDevice);
     if (e == cudaSuccess)
         e = cudaMemcpy(d_nodes, x->nodes.data(), sizeof(heddle_node) * x->nodes.size(),
                        cudaMemcpyHostToDevice);
     if (e == cudaSuccess)
-        e = cudaMemcpy(d_layers, x->layers.data(), sizeof(heddle_layer) * L, cudaMemcpyHostToDevice);
-    if (e == cudaSuccess && d_prof)
-        e = cudaMemcpy(d_prof, x->profile.data(), sizeof(double) * x->profile.size(),
-                       cudaMemcpyHostToDevice);
-    if (e == cudaSuccess) e = cudaMemset(x->d_img, 0, x->lay.bytes);
+        e = cudaMemcpy(d_layers, layers.data(), sizeof(heddle_layer) * L, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && d_prof) e = cudaMemcpy(d_prof, profile, sizeof(double) * nprof, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(*img, 0, lay.bytes);
     if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, sizeof(uint32_t));
     if (e == cudaSuccess) {
         hd::TableArgs a{};
-        a.lay = x->lay;
+        a.lay = lay;
         a.types = d_types;
         a.nodes = d_nodes;
         a.n_nodes = (int32_t)x->nodes.size();
         a.layers = d_layers;
         a.profile = d_prof;
-        a.boundary_bytes = x->boundary_bytes;
+        a.boundary_bytes = boundary_bytes;
         a.moe = x->moe;
-        a.img = x->d_img;
-        a.q = x->d_q;
+        a.img = *img;
+        a.q = *qtab;
         a.flags = x->d_flags;
         e = hd::launch_tables(a, 0);
     }
@@ -197,8 +215,7 @@ heddle_status build_tables(heddle_ctx* x) {
     uint32_t flags = 0;
     if (e == cudaSuccess) e = cudaMemcpy(&flags, x->d_flags, sizeof(uint32_t), cudaMemcpyDeviceToHost);
     if (e == cudaSuccess)
-        e = cudaMemcpy(x->model_flags, x->d_img + x->lay.offModel, sizeof(x->model_flags),
-                       cudaMemcpyDeviceToHost);
+        e = cudaMemcpy(model_flags, *img + lay.offModel, sizeof(int32_t) * 4, cudaMemcpyDeviceToHost);
     cudaFree(d_types);
     cudaFree(d_nodes);
     cudaFree(d_layers);
@@ -208,7 +225,62 @@ heddle_status build_tables(heddle_ctx* x) {
         return fail(x, HEDDLE_E_ARG, "a per-layer cost is negative, not finite or above 4e18 ns");
     if (flags & hd::kTabTooLarge)
         return fail(x, HEDDLE_E_LIMIT, "a per-(type, degree) model time or a P2P term exceeds 2^40 ns");
+    return ok(x);
+}
+
+// The tables of the micro-batch-size fill: level i is the model at
+// micro-batch 2^i times the base size -- FLOPs, stored activations, the TP
+// all-reduce and EP all-to-all messages and the boundary activation scale
+// by 2^i; parameter, gradient and state bytes do not -- with its profile
+// slice when per-size profiles were given.
+heddle_status build_levels(heddle_ctx* x) {
+    x->mbs_ready = false;
+    if (x->mbs_levels < 1 || !x->have_cluster || !x->have_model) return ok(x);
+    const int NT = (int)x->types.size(), L = (int)x->layers.size();
+    const bool prof = !x->mbs_profile.empty();
+    if (prof && x->mbs_profile.size() != (size_t)x->mbs_levels * NT * 4 * L)
+        return fail(x, HEDDLE_E_STATE, "size profiles cover %zu entries, need %d levels x %d types x 4 x %d layers",
+                    x->mbs_profile.size(), x->mbs_levels, NT, L);
+    if (!prof && x->have_profile)
+        return fail(x, HEDDLE_E_STATE, "the model was loaded with a profile: the fill needs per-size profiles");
+    for (int i = 0; i < x->mbs_levels; ++i) {
+        const int64_t f = (int64_t)1 << i;
+        std::vector<heddle_layer> ly = x->layers;
+        for (auto& y : ly) {
+            y.flops *= (double)f;
+            if (y.act_bytes > kByteLimit / f || y.ar_bytes > kByteLimit / f || y.a2a_bytes > kByteLimit / f)
+                return fail(x, HEDDLE_E_LIMIT, "size 2^%d: a byte count exceeds 2^42", i);
+            y.act_bytes *= f;
+            y.ar_bytes *= f;
+            y.a2a_bytes *= f;
+        }
+        if (x->boundary_bytes > kByteLimit / f)
+            return fail(x, HEDDLE_E_LIMIT, "size 2^%d: boundary_bytes exceeds 2^42", i);
+        heddle_ctx::Level& v = x->lv[i];
+        const double* pr = prof ? x->mbs_profile.data() + (size_t)i * NT * 4 * L : nullptr;
+        const heddle_status st =
+            build_image(x, ly, pr, x->boundary_bytes * f, v.lay, &v.img, &v.img_cap, &v.q, &v.q_cap, v.flags);
+        if (st != HEDDLE_OK) return st;
+    }
+    x->mbs_ready = true;
+    return ok(x);
+}
+
+heddle_status build_tables(heddle_ctx* x) {
+    x->tables_ready = false;
+    x->mbs_ready = false;
+    if (!x->have_cluster || !x->have_model) return ok(x);
+    const int NT = (int)x->types.size(), L = (int)x->layers.size();
+    if (x->have_profile && x->profile.size() != (size_t)NT * 4 * L)
+        return fail(x, HEDDLE_E_STATE,
+                    "model profile covers %zu entries, cluster needs %d types x 4 x %d layers",
+                    x->profile.size(), NT, L);
+    heddle_status st = build_image(x, x->layers, x->have_profile ? x->profile.data() : nullptr,
+                                   x->boundary_bytes, x->lay, &x->d_img, &x->img_cap, &x->d_q, &x->q_cap,
+                                   x->model_flags);
+    if (st != HEDDLE_OK) return st;
     x->tables_ready = true;
+    if (x->mbs_levels > 0) return build_levels(x);
     return ok(x);
 }
 
@@ -226,9 +298,10 @@ heddle_status check_cands(heddle_ctx* x, const heddle_candidates* c, bool device
 
 // the equal-layer closed form applies when every layer has the same cost per
 // (type, degree) and the same memory, unless the general search is forced
-bool equal_layer_search(const heddle_ctx* x) {
-    return x->search_mode == HEDDLE_SEARCH_AUTO && x->model_flags[0] && x->model_flags[1];
+bool equal_layer_search(const heddle_ctx* x, const int32_t* model_flags) {
+    return x->search_mode == HEDDLE_SEARCH_AUTO && model_flags[0] && model_flags[1];
 }
+bool equal_layer_search(const heddle_ctx* x) { return equal_layer_search(x, x->model_flags); }
 
 heddle_status check_ready(heddle_ctx* x) {
     if (!x->have_cluster) return fail(x, HEDDLE_E_STATE, "no cluster loaded");
@@ -323,6 +396,15 @@ void heddle_destroy(heddle_ctx* x) {
         if (x->ev_free[b]) cudaEventDestroy(x->ev_free[b]);
     }
     cudaFree(x->d_state);
+    for (auto& v : x->lv) {
+        cudaFree(v.img);
+        cudaFree(v.q);
+    }
+    cudaFree(x->lv_T);
+    cudaFree(x->lv_B);
+    cudaFree(x->lv_n);
+    cudaFree(x->lv_status);
+    cudaFree(x->lv_bounds);
     for (auto& r : x->phase_recs)
         for (cudaEvent_t ev : r.e) x->ev_pool.push_back(ev);
     for (cudaEvent_t ev : x->ev_pool) cudaEventDestroy(ev);
@@ -432,8 +514,12 @@ heddle_status take_phase_rec(heddle_ctx* x, heddle_ctx::PhaseRec* rec) {
 
 // Price cands into r; with a state, run the top-k over each chunk's searched
 // candidates (the only ones that can be OK) and merge them into *state.
+// `lvl` (nullable) selects the tables of one micro-batch size and `shift`
+// its log2: the screen then prices each candidate with M >> shift
+// micro-batches (invalid where 2^shift does not divide M).
 heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
-                         heddle_topk_state* state, void* stream) {
+                         heddle_topk_state* state, void* stream, const heddle_ctx::Level* lvl = nullptr,
+                         int shift = 0) {
     heddle_status st = check_cands(x, c, true);
     if (st != HEDDLE_OK) return st;
     if (!r) return fail(x, HEDDLE_E_ARG, "results is NULL");
@@ -443,8 +529,9 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
         return fail(x, HEDDLE_E_ARG, "null result array");
     DeviceGuard dg(x->device);
     hd::PriceArgs a{};
-    a.lay = x->lay;
-    a.img = x->d_img;
+    a.lay = lvl ? lvl->lay : x->lay;
+    a.img = lvl ? lvl->img : x->d_img;
+    a.mbs_shift = shift;
     a.moe = x->moe;
     a.stride = c->plane_stride;
     a.s_max = c->s_max;
@@ -461,7 +548,7 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     a.wl_code = x->d_wl_code;
     a.wl_bucket = x->d_wl_bucket;
     a.wl_cap = hd::kWorklistCap;
-    a.uniform = equal_layer_search(x) ? 1 : 0;
+    a.uniform = equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
     a.wl_T = x->d_wl_T;
     a.wl_nM = x->d_wl_nM;
     // chunks of at most the worklist capacity, in stream order
@@ -703,6 +790,82 @@ heddle_status heddle_get_search(heddle_ctx* x, int32_t* in_use) {
 heddle_status heddle_count_next(heddle_ctx* x, int32_t enable) {
     if (!x) return HEDDLE_E_ARG;
     x->count_next = enable != 0;
+    return ok(x);
+}
+
+heddle_status heddle_load_mbs(heddle_ctx* x, int32_t levels, const double* profile_s) {
+    if (!x) return HEDDLE_E_ARG;
+    if (levels < 0 || levels > HEDDLE_MAX_MBS_LEVELS)
+        return fail(x, HEDDLE_E_LIMIT, "levels must be in [0, %d]", HEDDLE_MAX_MBS_LEVELS);
+    if (profile_s && (!x->have_cluster || !x->have_model))
+        return fail(x, HEDDLE_E_STATE, "size profiles need the cluster and the model loaded first");
+    DeviceGuard dg(x->device);
+    x->mbs_levels = levels;
+    if (profile_s && levels > 0) {
+        const size_t n = (size_t)levels * x->types.size() * 4 * x->layers.size();
+        for (size_t i = 0; i < n; ++i)
+            if (!(profile_s[i] >= 0.0) || !isfinite(profile_s[i]))
+                return fail(x, HEDDLE_E_ARG, "size profile entry %zu is negative or not finite", i);
+        x->mbs_profile.assign(profile_s, profile_s + n);
+    } else {
+        x->mbs_profile.clear();
+    }
+    return build_levels(x);
+}
+
+heddle_status heddle_price_mbs(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r, uint8_t* mbs,
+                               void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    heddle_status st = check_cands(x, c, true);
+    if (st != HEDDLE_OK) return st;
+    if (!r) return fail(x, HEDDLE_E_ARG, "results is NULL");
+    if ((st = check_ready(x)) != HEDDLE_OK) return st;
+    if (x->mbs_levels < 1 || !x->mbs_ready) return fail(x, HEDDLE_E_STATE, "no micro-batch sizes loaded");
+    if (c->n == 0) return ok(x);
+    if (!r->T || !r->bottleneck || !r->n_dp || !r->status) return fail(x, HEDDLE_E_ARG, "null result array");
+    DeviceGuard dg(x->device);
+    cudaStream_t sm = (cudaStream_t)stream;
+    // the base size straight into the caller's results
+    if ((st = price_impl(x, c, r, nullptr, stream, &x->lv[0], 0)) != HEDDLE_OK) return st;
+    if (mbs) CU(cudaMemsetAsync(mbs, 0, (size_t)c->n, sm));
+    if (x->mbs_levels == 1) return ok(x);
+    const size_t cap = (size_t)std::min<int64_t>(c->n, hd::kWorklistCap);
+    CU(grow(&x->lv_T, &x->lv_T_cap, sizeof(int64_t) * cap));
+    CU(grow(&x->lv_B, &x->lv_B_cap, sizeof(int64_t) * cap));
+    CU(grow(&x->lv_n, &x->lv_n_cap, sizeof(uint16_t) * cap));
+    CU(grow(&x->lv_status, &x->lv_status_cap, cap));
+    if (r->bounds) CU(grow(&x->lv_bounds, &x->lv_bounds_cap, (size_t)(HEDDLE_MAX_STAGES + 1) * cap));
+    // every larger size, one chunk at a time, folded into the results
+    for (int64_t lo = 0; lo < c->n; lo += hd::kWorklistCap) {
+        const int64_t nb = std::min<int64_t>(c->n - lo, hd::kWorklistCap);
+        heddle_candidates cc = *c;
+        cc.S = c->S + lo;
+        cc.M = c->M + lo;
+        cc.code = c->code + lo;
+        cc.n = nb;
+        cc.base_index = c->base_index + lo;
+        heddle_results rr{x->lv_T, x->lv_B, x->lv_n, x->lv_status, r->bounds ? x->lv_bounds : nullptr};
+        for (int i = 1; i < x->mbs_levels; ++i) {
+            if ((st = price_impl(x, &cc, &rr, nullptr, stream, &x->lv[i], i)) != HEDDLE_OK) return st;
+            hd::MbsMergeArgs m{};
+            m.n = nb;
+            m.T_l = x->lv_T;
+            m.B_l = x->lv_B;
+            m.n_l = x->lv_n;
+            m.status_l = x->lv_status;
+            m.bounds_l = r->bounds ? x->lv_bounds : nullptr;
+            m.bstride_l = nb;
+            m.T = r->T + lo;
+            m.B = r->bottleneck + lo;
+            m.ndp = r->n_dp + lo;
+            m.status = r->status + lo;
+            m.bounds = r->bounds ? r->bounds + lo : nullptr;
+            m.bstride = c->n;
+            m.mbs = mbs ? mbs + lo : nullptr;
+            m.level = i;
+            CU(hd::launch_mbs_merge(m, x->num_sms, sm));
+        }
+    }
     return ok(x);
 }
 

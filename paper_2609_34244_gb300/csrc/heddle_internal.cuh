@@ -127,6 +127,7 @@ struct PriceArgs {
                          // that depth, in any order (equal-layer search)
     int32_t wl_cap;
     int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
+    int32_t mbs_shift;   // micro-batch size 2^shift: M >> shift micro-batches (invalid unless 2^shift | M)
     // per worklist entry, written by the search: T (-1 unless OK) and n * M,
     // so a top-k can run over the searched candidates only
     int64_t* wl_T;
@@ -172,6 +173,27 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t
 cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st,
                                  int64_t* launches = nullptr);
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st);
+
+// Micro-batch-size fill: fold the results of one size (level) into the
+// running best (smaller T wins, ties keep the earlier, smaller size).
+struct MbsMergeArgs {
+    int64_t n;
+    const int64_t* T_l;
+    const int64_t* B_l;
+    const uint16_t* n_l;
+    const uint8_t* status_l;
+    const uint8_t* bounds_l;  // nullable, plane stride bstride_l
+    int64_t bstride_l;
+    int64_t* T;
+    int64_t* B;
+    uint16_t* ndp;
+    uint8_t* status;
+    uint8_t* bounds;  // nullable, plane stride bstride
+    int64_t bstride;
+    uint8_t* mbs;     // nullable
+    int32_t level;
+};
+cudaError_t launch_mbs_merge(const MbsMergeArgs& a, int num_sms, cudaStream_t st);
 
 // Conversions between non-negative 64-bit integers and float through their
 // 32-bit halves: the 32-bit conversions run on the fast pipes, while a

@@ -384,8 +384,12 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
         int key = kMaxStages + 1;
         if (threadIdx.x < nloc) {
             const int S = a.S[c0 + threadIdx.x];
-            const int M = a.M[c0 + threadIdx.x];
-            key = (S >= 1 && S <= s_lim && M >= 1) ? S : 0;
+            // at micro-batch size 2^shift a replica runs M / 2^shift
+            // micro-batches; a size that does not divide M is not priced
+            const int Mraw = a.M[c0 + threadIdx.x];
+            const int M = Mraw >> a.mbs_shift;
+            const bool whole = (Mraw & ((1 << a.mbs_shift) - 1)) == 0;
+            key = (S >= 1 && S <= s_lim && M >= 1 && whole) ? S : 0;
             sS[threadIdx.x] = (uint8_t)key;
             sM[threadIdx.x] = (uint16_t)M;
         }

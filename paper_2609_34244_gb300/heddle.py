@@ -64,7 +64,9 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
            "heddle_load_model", "heddle_price_candidates", "heddle_topk_reset", "heddle_topk",
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
            "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
-           "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times"]
+           "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times",
+           "heddle_load_mbs", "heddle_price_mbs"]
+MAX_MBS_LEVELS = 4
 PHASES = ("screen", "search", "topk")
 TOPK_NOALLOC_MAX_N = 4194304
 SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS = 0, 1, 2
@@ -100,6 +102,8 @@ def load_library(path: str = LIB_PATH):
         "heddle_set_search": (i32, [p, i32]),
         "heddle_get_search": (i32, [p, C.POINTER(C.c_int32)]),
         "heddle_time_phases": (i32, [p, i32]),
+        "heddle_load_mbs": (i32, [p, i32, p]),
+        "heddle_price_mbs": (i32, [p, p, p, p, p]),
         "heddle_phase_times": (i32, [p, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
     }
     for name, (res, args) in sig.items():
@@ -207,6 +211,26 @@ def heddle_price_candidates(ctx, cands, results, stream=None):
     c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
     r = results if isinstance(results, heddle_results) else make_results(results)
     _check(ctx, load_library().heddle_price_candidates(ctx, C.byref(c), C.byref(r), _stream(stream)))
+
+
+def heddle_load_mbs(ctx, levels: int, profiles=None):
+    """Prepare the micro-batch-size fill for sizes 2**i, i < ``levels``;
+    ``profiles``: optional per-size seconds per layer, a sequence of
+    ``levels`` arrays [types][4][L] (host)."""
+    prof = None
+    if profiles is not None:
+        prof = np.ascontiguousarray(np.stack([np.asarray(x, np.float64) for x in profiles]), dtype=np.float64)
+    _check(ctx, load_library().heddle_load_mbs(ctx, int(levels), None if prof is None else prof.ctypes.data))
+
+
+def heddle_price_mbs(ctx, cands, results, mbs=None, stream=None):
+    """Price device candidates at every loaded micro-batch size and keep the
+    fastest per candidate; ``mbs`` (optional device uint8 tensor) receives
+    the chosen size's log2."""
+    c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
+    r = results if isinstance(results, heddle_results) else make_results(results)
+    _check(ctx, load_library().heddle_price_mbs(ctx, C.byref(c), C.byref(r),
+                                                None if mbs is None else _ptr(mbs), _stream(stream)))
 
 
 def heddle_topk_reset(ctx, state, k: int, stream=None):

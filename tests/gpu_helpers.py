@@ -98,3 +98,34 @@ def exact_topk(idx_all, T, nM, k):
 
     items.sort(key=functools.cmp_to_key(cmp))
     return items[:k]
+
+
+def price_mbs_gpu(h, w_cluster, w_model, cands, levels, profiles=None, bounds=True, search=None):
+    """Micro-batch-size fill on the GPU through the C ABI; numpy results
+    plus the chosen level ``mbs``."""
+    import torch
+    ctx = h.heddle_create(0)
+    try:
+        h.heddle_load_cluster(ctx, w_cluster)
+        h.heddle_load_model(ctx, w_model)
+        if search is not None:
+            h.heddle_set_search(ctx, search)
+        h.heddle_load_mbs(ctx, levels, profiles)
+        n = int(cands["S"].shape[0])
+        dc = h.cands_to_device(cands)
+        res = h.alloc_results(n, bounds=bounds)
+        mbs = torch.full((max(n, 1),), 255, dtype=torch.uint8, device="cuda")
+        h.heddle_price_mbs(ctx, h.make_candidates(dc), h.make_results(res), mbs)
+        torch.cuda.synchronize()
+        out = h.results_to_numpy(res)
+        out["mbs"] = mbs[:n].cpu().numpy()
+        out["errors"] = h.heddle_device_errors(ctx)
+        return out
+    finally:
+        h.heddle_destroy(ctx)
+
+
+def take(cands, idx):
+    """The candidates at indices ``idx`` (a host SoA copy)."""
+    return {"S": cands["S"][idx].copy(), "M": cands["M"][idx].copy(),
+            "code": np.ascontiguousarray(cands["code"][:, idx])}
