@@ -190,6 +190,7 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mbs-levels", type=int, default=4, help="micro-batch sizes of the fill figure (0: skip)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -300,6 +301,41 @@ def main():
                    "same_topk": gtopk["idx"].tolist() == local_topk["idx"].tolist()}
         h.heddle_set_search(ctx, h.SEARCH_AUTO)
 
+    # micro-batch-size fill (§5.3) on the same candidates: four sizes with
+    # seeded per-size profiles, device-resident, timed like the main step
+    mbs_fig = None
+    if args.mbs_levels > 0:
+        levels = args.mbs_levels
+        h.heddle_load_mbs(ctx, levels, W.mbs_profiles(w, levels, seed=rank))
+        mbs_out = torch.empty(n, dtype=torch.uint8, device="cuda")
+
+        def mbs_step():
+            for lo in range(0, n, batch):
+                hi = min(n, lo + batch)
+                h.heddle_price_mbs(ctx, h.make_candidates(dc, lo, hi, base_index=base),
+                                   h.make_results(res, lo, hi), mbs_out[lo:hi], stream)
+
+        for _ in range(2):
+            mbs_step()
+        torch.cuda.synchronize()
+        m0, m1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        h.heddle_time_phases(ctx, True)
+        m0.record(stream)
+        for _ in range(3):
+            mbs_step()
+        m1.record(stream)
+        torch.cuda.synchronize()
+        h.heddle_time_phases(ctx, False)
+        mph = h.heddle_phase_times(ctx)
+        mms = m0.elapsed_time(m1) / 3
+        ok = res["status"] == 0
+        chosen = torch.bincount(mbs_out[ok].long(), minlength=levels).tolist()
+        mbs_fig = {"value": n / (mms / 1e3), "unit": UNIT, "levels": levels, "ms_per_step": mms,
+                   "phases_ms_per_step": {k: v[0] / 3 for k, v in mph.items()},
+                   "ok_candidates_by_chosen_level": chosen,
+                   "profiles": "seeded per-size profiles (workloads.mbs_profiles)"}
+        h.heddle_load_mbs(ctx, 0)
+
     # end to end through the public host-buffer call (pinned host memory)
     pinned = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
               for k, v in w.cands.items()}
@@ -365,6 +401,7 @@ def main():
                 "d2h_bytes_per_step": h.TOPK_STATE_BYTES * world},
         "device_errors": errors,
         "general_search": general,
+        "mbs_fill": mbs_fig,
         "topk_head": merged["idx"][:4].tolist() if merged["count"] else [],
         "e2e_topk_matches": e2e_topk["idx"].tolist() == local_topk["idx"].tolist(),
     }

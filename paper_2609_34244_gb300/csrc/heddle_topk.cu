@@ -24,23 +24,23 @@ constexpr int kMergeBlock = 1024;  // warps 0-15 stage lists, warp 16 the state
 constexpr int kMergeWarps = kMergeBlock / 32;
 
 // One candidate entry: from a batch's results, or from the worklist of a
-// priced chunk (only the searched candidates, T = -1 unless OK).
+// priced chunk (only the searched candidates, T = -1 unless OK).  Every
+// field is loaded whether or not the entry turns out valid, so the loads of
+// several entries are independent and can be in flight together.
 template <bool kWorklist>
 __device__ __forceinline__ bool fetch(const TopkArgs& a, int64_t i, TopkEntry& e) {
     e.pad = 0;
     if (kWorklist) {
-        const int64_t T = a.wl_T[i];
-        if (T < 0) return false;
+        e.T = a.wl_T[i];
         e.idx = a.base_index + a.wl_idx[i];
-        e.T = T;
         e.nM = a.wl_nM[i];
-        return true;
+        return e.T >= 0;
     }
-    if (a.status[i] != HEDDLE_CAND_OK) return false;
+    const bool ok = a.status[i] == HEDDLE_CAND_OK;
     e.idx = a.base_index + i;
     e.T = a.T[i];
     e.nM = (uint32_t)a.ndp[i] * (uint32_t)a.M[i];
-    return true;
+    return ok;
 }
 
 // Entries that do not beat the incoming state's k-th entry (when it holds
@@ -65,11 +65,24 @@ __global__ void __launch_bounds__(kBlock) topk_block_kernel(TopkArgs a) {
     const int64_t n = kWorklist ? min((int64_t)*a.wl_count, (int64_t)a.wl_cap) : a.n;
     const int64_t nwarps = (int64_t)gridDim.x * W;
     const int64_t gw = (int64_t)blockIdx.x * W + warp;
-    for (int64_t base = gw * 32; base < n; base += nwarps * 32) {
-        const int64_t i = base + lane;
-        TopkEntry e;
-        const bool valid = i < n && fetch<kWorklist>(a, i, e) && (!full || better(e, bar));
-        warp_offer(list, cnt, k, valid, e);
+    // four rounds of 32 entries per warp are loaded before any is offered
+    constexpr int U = 4;
+    const int64_t step = nwarps * 32;
+    for (int64_t base = gw * 32; base < n; base += step * U) {
+        TopkEntry e[U];
+        bool valid[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t i = base + u * step + lane;
+            valid[u] = false;
+            e[u].idx = 0;
+            e[u].T = 0;
+            e[u].nM = 0;
+            e[u].pad = 0;
+            if (i < n) valid[u] = fetch<kWorklist>(a, i, e[u]);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) warp_offer(list, cnt, k, valid[u] && (!full || better(e[u], bar)), e[u]);
     }
     if (lane == 0) counts[warp] = cnt;
     cta_tree_merge(lists, counts, tmp, tmp_counts, W, k);
