@@ -226,9 +226,11 @@ heddle_status heddle_topk(heddle_ctx* ctx, const heddle_candidates* cands,
                           void* stream);
 
 /* Price a batch and merge its OK candidates into *state (device): after each
- * chunk's search, the block-level top-k runs over that chunk's worklist of
- * searched candidates only (the screen already rejected the rest), then the
- * per-CTA lists are merged into the state -- no pass over the full results.
+ * chunk's search, one top-k launch runs over that chunk's worklist of
+ * searched candidates only (the screen already rejected the rest): per-CTA
+ * lists, the last CTA of each group of 16 merges its group and the last
+ * group merges the group lists into the state (tickets, no waiting) -- no
+ * pass over the full results.
  * Same results and the same state as heddle_price_candidates followed by
  * heddle_topk.  Errors as for both. */
 heddle_status heddle_price_topk(heddle_ctx* ctx, const heddle_candidates* cands,
@@ -369,10 +371,8 @@ heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);
  * after the search kernel and, when the call merges a top-k, after the
  * top-k kernels.  heddle_phase_times synchronises on them and returns, per
  * phase (SCREEN, SEARCH, TOPK), the summed elapsed milliseconds and the
- * number of kernels launched in it (one screen and one search kernel per
- * chunk, with the equal-layer search also the kernel that orders the
- * worklist by depth in the screen phase; two or three top-k kernels), then
- * forgets them.  The events add no work to the
+ * number of kernels launched in it (one screen, one search and one top-k
+ * kernel per chunk), then forgets them.  The events add no work to the
  * kernels; enabling or disabling changes no result.  Errors: E_ARG,
  * E_CUDA. */
 #define HEDDLE_PHASE_SCREEN 0

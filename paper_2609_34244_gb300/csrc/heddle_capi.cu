@@ -54,6 +54,7 @@ struct heddle_ctx {
     int scratch_blocks = 0;
     hd::TopkEntry* d_scratch2 = nullptr;
     int32_t* d_scratch2_count = nullptr;
+    int32_t* d_tickets = nullptr;  // [17], zero between top-k launches
     // host-buffer path
     cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
     cudaEvent_t ev_loaded[2] = {nullptr, nullptr}, ev_priced[2] = {nullptr, nullptr},
@@ -352,6 +353,8 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     const int l2 = (x->scratch_blocks + 31) / 32;
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2, sizeof(hd::TopkEntry) * hd::kMaxTopK * l2);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2_count, sizeof(int32_t) * l2);
+    if (e == cudaSuccess) e = cudaMalloc(&x->d_tickets, sizeof(int32_t) * 17);
+    if (e == cudaSuccess) e = cudaMemset(x->d_tickets, 0, sizeof(int32_t) * 17);
 
     if (e != cudaSuccess) {
         heddle_destroy(x);
@@ -382,6 +385,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_wl_nM);
     cudaFree(x->d_scratch2);
     cudaFree(x->d_scratch2_count);
+    cudaFree(x->d_tickets);
     for (int b = 0; b < 2; ++b) {
         cudaFree(x->st_S[b]);
         cudaFree(x->st_M[b]);
@@ -495,6 +499,7 @@ hd::TopkArgs topk_args(heddle_ctx* x, heddle_topk_state* state) {
     a.max_blocks = x->scratch_blocks;
     a.scratch2 = x->d_scratch2;
     a.scratch2_count = x->d_scratch2_count;
+    a.tickets = x->d_tickets;
     return a;
 }
 

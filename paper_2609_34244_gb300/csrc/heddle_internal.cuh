@@ -162,9 +162,12 @@ struct TopkArgs {
     const int64_t* wl_T;
     const uint32_t* wl_nM;
     int32_t wl_cap;
-    // second-level lists of the two-level merge
+    // second-level lists of the two-level merge (group lists of the
+    // one-launch worklist top-k), and that kernel's tickets: [16] per group,
+    // then one for the final merge; zero between launches
     TopkEntry* scratch2;
     int32_t* scratch2_count;
+    int32_t* tickets;
 };
 // `launches` (nullable) gains the number of kernels launched.
 cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t* launches = nullptr);

@@ -158,6 +158,134 @@ cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st, int64_t*
     return cudaGetLastError();
 }
 
+// ---- one-launch top-k of a priced chunk's worklist.  Up to 64 CTAs scan
+// the worklist as topk_block_kernel does; CTAs form groups of kFan: the last
+// CTA of a group to finish (a ticket counter after a memory fence, no
+// waiting) merges the group's lists, and the last group to finish folds
+// the group lists and the incoming state into the state, then clears the
+// tickets for the next launch.
+constexpr int kFusedBlock = 256;
+constexpr int kFusedGroups = 4;
+
+// Stage lists [first, first + nl) of src into lists[0 ..), one warp per
+// list; the entries were written by other CTAs, so they are read past L1.
+template <int W>
+__device__ void stage_lists(TopkEntry* lists, int* counts, const TopkEntry* src, const int32_t* src_count,
+                            int first, int nl, int k) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int w = warp; w < nl; w += W) {
+        const int l = first + w;
+        const int c = min(__ldcg(src_count + l), k);
+        const TopkEntry* from = src + (size_t)l * kMaxTopK;
+        for (int i = lane; i < c; i += 32) {
+            TopkEntry e;
+            e.idx = __ldcg(&from[i].idx);
+            e.T = __ldcg(&from[i].T);
+            e.nM = __ldcg(&from[i].nM);
+            e.pad = 0;
+            lists[w * kMaxTopK + i] = e;
+        }
+        if (lane == 0) counts[w] = c;
+    }
+}
+
+// Write list 0 (counts[0] entries) to dst / dst_count and draw a ticket:
+// the barrier gathers the CTA's stores, thread 0 fences them (fences are
+// cumulative) before its atomic, and the CTA that draws the last of
+// `expected` tickets fences again before it reads the others' lists.
+__device__ bool publish(const TopkEntry* list, const int* counts, TopkEntry* dst, int32_t* dst_count,
+                        int32_t* ticket, int expected, int* last_flag) {
+    for (int p = threadIdx.x; p < counts[0]; p += blockDim.x) dst[p] = list[p];
+    if (threadIdx.x == 0) *dst_count = counts[0];
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const bool last = atomicAdd(ticket, 1) == expected - 1;
+        if (last) __threadfence();
+        *last_flag = last;
+    }
+    __syncthreads();
+    return *last_flag != 0;
+}
+
+__global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
+    constexpr int W = kFusedBlock / 32;
+    static_assert(W >= (kFan + 1) / 2, "a tree merge of W lists runs W / 2 warps at once");
+    static_assert(kFusedGroups + 1 <= kFan + 1, "the final merge holds the group lists and the state");
+    const int k = state_k(a.state);
+    __shared__ TopkEntry lists[(kFan + 1) * kMaxTopK];
+    __shared__ TopkEntry tmp[((kFan + 2) / 2) * kMaxTopK];
+    __shared__ int counts[kFan + 1], tmp_counts[(kFan + 2) / 2];
+    __shared__ int last_flag;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool full = a.state->count >= k;
+    TopkEntry bar;
+    bar.idx = full ? a.state->idx[k - 1] : 0;
+    bar.T = full ? a.state->T[k - 1] : 0;
+    bar.nM = full ? a.state->nM[k - 1] : 0;
+    bar.pad = 0;
+    // ---- this CTA's share of the worklist
+    int cnt = 0;
+    TopkEntry* list = lists + warp * kMaxTopK;
+    const int64_t n = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    const int64_t step = (int64_t)gridDim.x * W * 32;
+    constexpr int U = 4;
+    for (int64_t base = ((int64_t)blockIdx.x * W + warp) * 32; base < n; base += step * U) {
+        TopkEntry e[U];
+        bool valid[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t i = base + u * step + lane;
+            valid[u] = false;
+            e[u].idx = 0;
+            e[u].T = 0;
+            e[u].nM = 0;
+            e[u].pad = 0;
+            if (i < n) valid[u] = fetch<true>(a, i, e[u]);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) warp_offer(list, cnt, k, valid[u] && (!full || better(e[u], bar)), e[u]);
+    }
+    if (lane == 0) counts[warp] = cnt;
+    cta_tree_merge(lists, counts, tmp, tmp_counts, W, k);
+    // ---- the last CTA of its group merges the group's lists
+    const int group = blockIdx.x / kFan, ngroups = (gridDim.x + kFan - 1) / kFan;
+    const int first = group * kFan, gsize = min(kFan, (int)gridDim.x - first);
+    if (!publish(lists, counts, a.scratch + (size_t)blockIdx.x * kMaxTopK, a.scratch_count + blockIdx.x,
+                 a.tickets + group, gsize, &last_flag))
+        return;
+    stage_lists<W>(lists, counts, a.scratch, a.scratch_count, first, gsize, k);
+    cta_tree_merge(lists, counts, tmp, tmp_counts, gsize, k);
+    // ---- the last group folds the group lists and the incoming state
+    if (!publish(lists, counts, a.scratch2 + (size_t)group * kMaxTopK, a.scratch2_count + group,
+                 a.tickets + kFan, ngroups, &last_flag))
+        return;
+    stage_lists<W>(lists, counts, a.scratch2, a.scratch2_count, 0, ngroups, k);
+    if (warp == W - 1) {
+        const int c = min(max(a.state->count, 0), k);
+        for (int i = lane; i < c; i += 32) {
+            TopkEntry e;
+            e.idx = a.state->idx[i];
+            e.T = a.state->T[i];
+            e.nM = a.state->nM[i];
+            e.pad = 0;
+            lists[ngroups * kMaxTopK + i] = e;
+        }
+        if (lane == 0) counts[ngroups] = c;
+    }
+    cta_tree_merge(lists, counts, tmp, tmp_counts, ngroups + 1, k);
+    const int total = counts[0];
+    for (int p = threadIdx.x; p < kMaxTopK; p += blockDim.x) {
+        const bool live = p < total;
+        a.state->idx[p] = live ? lists[p].idx : -1;
+        a.state->T[p] = live ? lists[p].T : -1;
+        a.state->nM[p] = live ? lists[p].nM : 0;
+    }
+    if (threadIdx.x == 0) a.state->count = total;
+    // every other CTA has drawn its tickets: clear them for the next launch
+    for (int i = threadIdx.x; i <= kFan; i += blockDim.x) a.tickets[i] = 0;
+}
+
 __global__ void topk_reset_kernel(heddle_topk_state* s, int k) {
     for (int p = threadIdx.x; p < kMaxTopK; p += blockDim.x) {
         s->idx[p] = -1;
@@ -188,18 +316,15 @@ cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t
 cudaError_t launch_topk_worklist(const TopkArgs& a, int64_t n, int num_sms, cudaStream_t st,
                                  int64_t* launches) {
     if (n <= 0) return cudaSuccess;
-    // at most kFan CTAs of 512 threads: one merge level (the worklist holds
-    // only the searched candidates, mostly rejected by the state's k-th)
-    constexpr int kWlBlock = 512;
-    const int64_t per_block = (int64_t)kWlBlock * 16;
-    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)kFan);
+    // one launch: the worklist holds only the searched candidates, most of
+    // them rejected by the state's k-th
+    const int64_t per_block = (int64_t)kFusedBlock * 16;
+    int grid = (int)std::min<int64_t>((n + per_block - 1) / per_block, (int64_t)kFan * kFusedGroups);
     grid = std::max(1, std::min(grid, a.max_blocks));
     (void)num_sms;
-    topk_block_kernel<true, kWlBlock><<<grid, kWlBlock, 0, st>>>(a);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    topk_fused_kernel<<<grid, kFusedBlock, 0, st>>>(a);
     if (launches) *launches += 1;
-    return merge_lists(a, grid, st, launches);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_topk_reset(heddle_topk_state* state, int32_t k, cudaStream_t st) {

@@ -162,7 +162,7 @@ def test_batching_and_launch_shape_do_not_change_results(h, W, oracle_mod):
         assert (a[key] == c[key]).all(), key
     assert c["counters"]["checks"] > 0 and c["counters"]["priced"] > 0
     # phase timing: same results, one screen and one search launch per
-    # chunk, two or three top-k launches per fused chunk
+    # chunk, one top-k launch per fused chunk
     chunks = -(-5000 // 777)
     for fused in (False, True):
         d = G.price_gpu(h, w.cluster, w.model, w.cands, k=64, batch=777, fused=fused, phases=True)
@@ -173,7 +173,7 @@ def test_batching_and_launch_shape_do_not_change_results(h, W, oracle_mod):
         assert ph["screen"][1] == chunks and ph["search"][1] == chunks, ph
         assert ph["screen"][0] > 0 and ph["search"][0] > 0, ph
         if fused:
-            assert 2 * chunks <= ph["topk"][1] <= 3 * chunks and ph["topk"][0] > 0, ph
+            assert ph["topk"][1] == chunks and ph["topk"][0] > 0, ph
         else:
             assert ph["topk"] == (0.0, 0), ph
 
