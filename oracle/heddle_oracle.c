@@ -58,6 +58,7 @@ struct orc_ctx {
     int64_t* act;    /* [L+1] prefix of stored activation bytes */
     int64_t* param;  /* [L+1] prefix of gradient (parameter) bytes */
     int64_t p2p[MAXT][MAXT][2];
+    int split_mode;  /* 0: min-max PartitionLayers, 1: the paper's Distribute rule */
 };
 
 /* ---------------------------------------------------------------- tables */
@@ -359,6 +360,124 @@ typedef struct {
     int32_t a[MAXS + 1];
 } priced;
 
+/* Evaluate (§5.3): T = (M-1) max t_s + sum t_s + max g_s for the split a;
+ * writes max t_s to *tmax_out. */
+static int64_t evaluate(const orc_ctx* x, int S, int M, int64_t n, const int64_t* const* P, const int64_t* c,
+                        const int* j, const int* g, const int32_t* a, int64_t* tmax_out) {
+    int64_t tmax = 0, tsum = 0, gmax = 0;
+    for (int s = 0; s < S; ++s) {
+        int64_t t = P[s][a[s + 1]] - P[s][a[s]] + c[s];
+        if (t > tmax) tmax = t;
+        tsum += t;
+        /* DP gradient synchronisation of stage s (reading): a ring all-reduce
+         * over the n replicas of the stage's gradient shard (G_s / k bytes),
+         * 2(n-1)/n of it over the slowest NIC of the type, in whole ns
+         * rounded up; zero without replication */
+        int64_t gs = 0;
+        if (n > 1) {
+            int64_t G = x->param[a[s + 1]] - x->param[a[s]];
+            u128 num = (u128)2 * (u128)(n - 1) * (u128)G * 1000000000u;
+            u128 den = (u128)n * (u128)(1 << j[s]) * (u128)x->inter_bw[g[s]];
+            gs = ceil_div128(num, den);
+        }
+        if (gs > gmax) gmax = gs;
+    }
+    *tmax_out = tmax;
+    return (int64_t)(M - 1) * tmax + tsum + gmax;
+}
+
+/* ---------------------------------------------- the paper's split rule */
+
+/* §5.3 "Layer split and DP degree": the paper's planner gives each stage
+ * layers in proportion to its profiled speed; if that split exceeds a
+ * stage's memory it prices a fixed list of alternative splits and keeps the
+ * fastest that fits.  Readings: the speed of stage s is 2^40 divided by the
+ * time of all L layers on its type and degree, rounded down; the list is
+ * (1) in proportion to speed, (2) equal layer counts, (3) in proportion to
+ * the longest run of consecutive layers each stage's memory holds; the
+ * fastest is the smallest T, the earlier alternative on ties. */
+
+/* L layers over S stages in proportion to weights w >= 0 (sum > 0): floor
+ * of the exact share, at least one layer per stage; missing layers go one
+ * each to the largest remainders (the earlier stage on ties); surplus
+ * layers (the one-layer minimum can overshoot) come one at a time off the
+ * stage holding the most (the later stage on ties).  Boundaries to a. */
+static void proportional_split(int S, int L, const int64_t* w, int32_t* a) {
+    int64_t V = 0;
+    for (int s = 0; s < S; ++s) V += w[s];
+    int64_t cnt[MAXS], rem[MAXS];
+    int64_t total = 0;
+    for (int s = 0; s < S; ++s) {
+        int64_t share = (int64_t)L * w[s];
+        cnt[s] = share / V;
+        rem[s] = share % V;
+        if (cnt[s] < 1) cnt[s] = 1;
+        total += cnt[s];
+    }
+    int given[MAXS] = {0};
+    while (total < L) {
+        int best = -1;
+        for (int s = 0; s < S; ++s)
+            if (!given[s] && (best < 0 || rem[s] > rem[best])) best = s;
+        given[best] = 1;
+        cnt[best] += 1;
+        total += 1;
+    }
+    while (total > L) {
+        int best = -1;
+        for (int s = 0; s < S; ++s)
+            if (cnt[s] > 1 && (best < 0 || cnt[s] >= cnt[best])) best = s;
+        cnt[best] -= 1;
+        total -= 1;
+    }
+    a[0] = 0;
+    for (int s = 0; s < S; ++s) a[s + 1] = a[s] + (int32_t)cnt[s];
+}
+
+/* Longest run of consecutive layers [i, j) with W[j] - W[i] <= cap. */
+static int64_t longest_run(const int64_t* W, int L, int64_t cap) {
+    int64_t best = 0;
+    for (int i = 0; i < L; ++i)
+        for (int j = i + 1; j <= L && W[j] - W[i] <= cap; ++j)
+            if (j - i > best) best = j - i;
+    return best;
+}
+
+/* The paper's rule: returns 1 and the chosen split in a (with its T and
+ * max t_s) if one of the alternatives fits, else 0. */
+static int distribute(const orc_ctx* x, int S, int L, int M, int64_t n, const int64_t* const* P,
+                      const int64_t* c, const int64_t* const* W, const int64_t* cap, const int* g,
+                      const int* j, int32_t* a, int64_t* T_out, int64_t* B_out) {
+    int64_t w[3][MAXS];
+    for (int s = 0; s < S; ++s) {
+        int64_t all = P[s][L];
+        w[0][s] = all > 0 ? ((int64_t)1 << 40) / all : ((int64_t)1 << 40);
+        w[1][s] = 1;
+        w[2][s] = longest_run(W[s], L, cap[s]);
+    }
+    int found = 0;
+    for (int alt = 0; alt < 3; ++alt) {
+        int64_t V = 0;
+        for (int s = 0; s < S; ++s) V += w[alt][s];
+        if (V <= 0) continue;
+        int32_t b[MAXS + 1];
+        proportional_split(S, L, w[alt], b);
+        int fits = 1;
+        for (int s = 0; s < S && fits; ++s)
+            if (W[s][b[s + 1]] - W[s][b[s]] > cap[s]) fits = 0;
+        if (!fits) continue;
+        int64_t tmax;
+        int64_t T = evaluate(x, S, M, n, P, c, j, g, b, &tmax);
+        if (!found || T < *T_out) {
+            found = 1;
+            *T_out = T;
+            *B_out = tmax;
+            for (int s = 0; s <= S; ++s) a[s] = b[s];
+        }
+    }
+    return found;
+}
+
 static void price_one(const orc_ctx* x, int S, int M, const uint8_t* codes, int64_t* f,
                       int64_t* Wbuf, priced* out) {
     int L = x->L;
@@ -410,34 +529,28 @@ static void price_one(const orc_ctx* x, int S, int M, const uint8_t* codes, int6
         W[s] = w;
         cap[s] = x->mem[g[s]] * (int64_t)(1 << j[s]);
     }
+    if (x->split_mode == 1) {
+        /* the paper's split rule instead of PartitionLayers */
+        if (!distribute(x, S, L, M, n, P, c, W, cap, g, j, out->a, &out->T, &out->B)) {
+            out->status = ORC_OOM;
+            out->T = out->B = -1;
+            return;
+        }
+        out->status = ORC_OK;
+        return;
+    }
     int64_t B;
     if (!partition(S, L, P, c, W, cap, f, &B, out->a)) {
         out->status = ORC_OOM;
         return;
     }
-    /* Evaluate (§5.3): T = (M-1) max t_s + sum t_s + max g_s */
-    int64_t tmax = 0, tsum = 0, gmax = 0;
-    for (int s = 0; s < S; ++s) {
-        int64_t t = P[s][out->a[s + 1]] - P[s][out->a[s]] + c[s];
-        if (t > tmax) tmax = t;
-        tsum += t;
-        /* DP gradient synchronisation of stage s (reading): a ring all-reduce
-         * over the n replicas of the stage's gradient shard (G_s / k bytes),
-         * 2(n-1)/n of it over the slowest NIC of the type, in whole ns
-         * rounded up; zero without replication */
-        int64_t gs = 0;
-        if (n > 1) {
-            int64_t G = x->param[out->a[s + 1]] - x->param[out->a[s]];
-            u128 num = (u128)2 * (u128)(n - 1) * (u128)G * 1000000000u;
-            u128 den = (u128)n * (u128)(1 << j[s]) * (u128)x->inter_bw[g[s]];
-            gs = ceil_div128(num, den);
-        }
-        if (gs > gmax) gmax = gs;
-    }
+    int64_t tmax;
     out->B = B;
-    out->T = (int64_t)(M - 1) * tmax + tsum + gmax;
+    out->T = evaluate(x, S, M, n, P, c, j, g, out->a, &tmax);
     out->status = ORC_OK;
 }
+
+void orc_set_split(orc_ctx* x, int mode) { x->split_mode = mode; }
 
 typedef struct {
     const orc_ctx* x;

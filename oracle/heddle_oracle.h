@@ -53,6 +53,14 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
               int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
               int threads);
 
+/* Layer split used by orc_price: 0 (default) the min-max PartitionLayers of
+ * the hot path; 1 the paper's own rule (§5.3 "Layer split and DP degree"):
+ * layers in proportion to each stage's speed (2^40 / time of all layers on
+ * its type and degree, rounded down), else the fastest fitting split of a
+ * fixed list -- equal layer counts, layers in proportion to each stage's
+ * longest memory-fitting run -- else OOM. */
+void orc_set_split(orc_ctx* x, int mode);
+
 /* Top-k of the OK candidates by throughput n*M/T, ties to the smaller index.
  * idx = base_index + c.  Writes up to k entries; returns how many. */
 int orc_topk(int64_t n, int64_t base_index, const int64_t* T, const uint16_t* n_dp,

@@ -56,6 +56,7 @@ def lib():
         L.orc_partition_raw.argtypes = [C.c_int, C.c_int, p, p, p, p, p, p]
         L.orc_replicas.restype = C.c_int
         L.orc_replicas.argtypes = [C.c_int, p, C.c_int, p]
+        L.orc_set_split.argtypes = [p, C.c_int]
         _lib = L
     return _lib
 
@@ -95,6 +96,12 @@ class Oracle:
                                int(bool(model.get("moe", False))), _ptr(prof), err)
         if not self._h:
             raise ValueError("oracle rejected inputs: " + err.value.decode())
+
+    def set_split(self, mode: str):
+        """``"minmax"`` (PartitionLayers, the default) or ``"distribute"``
+        (the paper's own proportional rule with its fixed alternatives)."""
+        lib().orc_set_split(self._h, {"minmax": 0, "distribute": 1}[mode])
+        return self
 
     def __del__(self):
         h = getattr(self, "_h", None)

@@ -381,6 +381,55 @@ def check_mbs_properties(O, seed=11):
             assert (r["mbs"] > 0).any(), (name, "a larger size wins somewhere")
 
 
+def check_distribute_hand(O):
+    """Hand-worked prices under the paper's own split rule
+    (golden/hand_distribute.json, §5.3)."""
+    W = _workloads()
+    for case in _load("hand_distribute.json")["cases"]:
+        nt = len(case["tflops"])
+        cluster = W.make_cluster(case["tflops"], case["mem_bytes"], [300 * 10**9] * nt,
+                                 [tuple(x) for x in case["nodes"]])
+        L = len(case["flops"])
+        model = W.make_model(case["flops"], 0, case["state_bytes"], case["act_bytes"], 0, 0, 0)
+        cands = W.from_structures([[tuple(s) for s in case["stages"]]], [4])
+        S = len(case["stages"])
+        for mode, e in (("distribute", case["expect"]), ("minmax", case.get("minmax"))):
+            if e is None:
+                continue
+            r = O.Oracle(cluster, model).set_split(mode).price(cands)
+            name = "%s (%s)" % (case["name"], mode)
+            assert int(r["status"][0]) == e["status"], (name, r["status"][0])
+            assert int(r["T"][0]) == e["T"], (name, r["T"][0])
+            assert int(r["bottleneck"][0]) == e["bottleneck"], (name, r["bottleneck"][0])
+            if e["bounds"] is not None and mode == "distribute":
+                assert r["bounds"][: S + 1, 0].tolist() == e["bounds"], (name, r["bounds"][:, 0])
+
+
+def check_distribute_properties(O, seed=5):
+    """The paper's rule against the exact split on seeded workloads: it
+    fits only where some split fits, and its bottleneck is never below the
+    min-max bottleneck B*; with equal layers, equal speeds and ample memory
+    it is the equal-count split."""
+    W = _workloads()
+    for name, n in (("dense32", 2000), ("moe48", 2000), ("stress128", 400)):
+        w = W.make_workload(name, seed=seed, n=n)
+        exact = O.Oracle(w.cluster, w.model).price(w.cands)
+        dist = O.Oracle(w.cluster, w.model).set_split("distribute").price(w.cands)
+        okd = dist["status"] == O.OK
+        assert (exact["status"][okd] == O.OK).all(), name
+        assert (dist["bottleneck"][okd] >= exact["bottleneck"][okd]).all(), name
+        same = dist["status"] != O.OK
+        assert (dist["status"][same & (exact["status"] != O.OK)] == exact["status"][same & (exact["status"] != O.OK)]).all()
+        if name != "moe48":  # moe48 is 1% OK even under the exact split
+            assert okd.sum() > 0, name
+    cluster = W.make_cluster([1000.0], [10**13], [10**11], [(0, 8, 10**10)])
+    model = W.make_model([1e12] * 10, 0, 0, 0, 0, 0, 0)
+    cands = W.from_structures([[(0, 0)] * 3, [(0, 0)] * 4], [8, 8])
+    r = O.Oracle(cluster, model).set_split("distribute").price(cands)
+    assert r["bounds"][:4, 0].tolist() == [0, 4, 7, 10], r["bounds"][:, 0]
+    assert r["bounds"][:5, 1].tolist() == [0, 3, 6, 8, 10], r["bounds"][:, 1]
+
+
 ALL_CHECKS = [
     check_hand_partitions,
     check_hand_pricing,
@@ -393,4 +442,6 @@ ALL_CHECKS = [
     check_status_rules,
     check_mbs_hand,
     check_mbs_properties,
+    check_distribute_hand,
+    check_distribute_properties,
 ]

@@ -57,6 +57,12 @@ MUTANTS = [
     ("ep_group_not_split", "while ((1 << e) > x->maxnode[t]) --e;", ""),
     ("ep_blocks_of_one", "while ((1 << e) > x->maxnode[t]) --e;", "if ((1 << e) > x->maxnode[t]) e = 0;"),
     ("compute_ignores_degree", "double s = flops / (k * tflops * 1e12);", "double s = flops / (tflops * 1e12);"),
+    ("distribute_tie_to_later", "if (!given[s] && (best < 0 || rem[s] > rem[best])) best = s;",
+     "if (!given[s] && (best < 0 || rem[s] >= rem[best])) best = s;"),
+    ("distribute_no_one_layer_minimum", "if (cnt[s] < 1) cnt[s] = 1;", "if (cnt[s] < 0) cnt[s] = 0;"),
+    ("distribute_time_not_speed", "w[0][s] = all > 0 ? ((int64_t)1 << 40) / all : ((int64_t)1 << 40);",
+     "w[0][s] = all;"),
+    ("distribute_memory_ignored", "if (W[s][b[s + 1]] - W[s][b[s]] > cap[s]) fits = 0;", "(void)cap;"),
 ]
 
 # planted mistakes in the Python part of the oracle (the micro-batch fill)
