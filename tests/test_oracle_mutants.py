@@ -24,8 +24,8 @@ MUTANTS = [
      "if (W[s][j] - W[s][i] >= cap[s]) continue;\n                int64_t t"),
     ("iteration_M_not_M_minus_1", "(int64_t)(M - 1) * tmax", "(int64_t)M * tmax"),
     ("drop_grad_sync", "+ tsum + gmax;", "+ tsum;"),
-    ("drop_sum_term", "out->T = (int64_t)(M - 1) * tmax + tsum + gmax;",
-     "out->T = (int64_t)(M - 1) * tmax + tmax + gmax;"),
+    ("drop_sum_term", "return (int64_t)(M - 1) * tmax + tsum + gmax;",
+     "return (int64_t)(M - 1) * tmax + tmax + gmax;"),
     ("inflight_reversed", "int64_t inflight = (S - s) < M ? (S - s) : M;",
      "int64_t inflight = (s + 1) < M ? (s + 1) : M;"),
     ("inflight_ignores_M", "int64_t inflight = (S - s) < M ? (S - s) : M;",
