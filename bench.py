@@ -191,6 +191,7 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--mbs-levels", type=int, default=4, help="micro-batch sizes of the fill figure (0: skip)")
+    ap.add_argument("--no-distribute", action="store_true", help="skip the paper's-split comparison figure")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -272,6 +273,43 @@ def main():
     errors = h.heddle_device_errors(ctx)
     local_topk = h.read_topk_state(state)
     merged = shard.merge_topk_across_ranks(group, local_topk, 16)
+
+    # the paper's own layer split (§5.3) on the same candidates: its speed
+    # and how much longer its iteration times are than the exact split's
+    distribute = None
+    if not args.no_distribute:
+        res2 = h.alloc_results(n)
+        dbatches = [(c, h.make_results(res2, lo, min(n, lo + batch)))
+                    for (c, _), lo in zip(cbatches, range(0, n, batch))]
+        h.heddle_set_search(ctx, h.SEARCH_DISTRIBUTE)
+        dstate = h.alloc_topk_state()
+
+        def dist_step():
+            h.heddle_topk_reset(ctx, dstate, 16, stream)
+            for c, r in dbatches:
+                h.heddle_price_topk(ctx, c, r, dstate, stream)
+
+        dist_step()
+        torch.cuda.synchronize()
+        d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        d0.record(stream)
+        for _ in range(2):
+            dist_step()
+        d1.record(stream)
+        torch.cuda.synchronize()
+        dms = d0.elapsed_time(d1) / 2
+        ex_ok = res["status"] == 0
+        di_ok = res2["status"] == 0
+        both = ex_ok & di_ok
+        gap = (res2["T"][both].double() - res["T"][both].double()) / res["T"][both].double()
+        distribute = {"value": n / (dms / 1e3), "unit": UNIT, "ms_per_step": dms,
+                      "exact_ok": int(ex_ok.sum()), "distribute_ok": int(di_ok.sum()),
+                      "mean_T_gap_where_both_ok": float(gap.mean()) if both.any() else None,
+                      "share_slower": float((gap > 0).double().mean()) if both.any() else None,
+                      "share_faster": float((gap < 0).double().mean()) if both.any() else None,
+                      "bottleneck_never_below_Bstar": bool((res2["bottleneck"][both] >= res["bottleneck"][both]).all())}
+        h.heddle_set_search(ctx, h.SEARCH_AUTO)
+        del res2
 
     # the general interval search on the same workload (secondary figure)
     general = None
@@ -401,6 +439,7 @@ def main():
                 "d2h_bytes_per_step": h.TOPK_STATE_BYTES * world},
         "device_errors": errors,
         "general_search": general,
+        "distribute_split": distribute,
         "mbs_fill": mbs_fig,
         "topk_head": merged["idx"][:4].tolist() if merged["count"] else [],
         "e2e_topk_matches": e2e_topk["idx"].tolist() == local_topk["idx"].tolist(),

@@ -343,10 +343,21 @@ heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
  * search otherwise.  GENERAL forces the general search.  Both are exact and
  * return identical results.  heddle_get_search reports the search the next
  * pricing call will run (GENERAL or EQUAL_LAYERS); E_STATE if the cost
- * tables are not built. */
+ * tables are not built.
+ *
+ * DISTRIBUTE replaces PartitionLayers by the paper's own layer split
+ * (§5.3 "Layer split and DP degree"), to measure what the exact min-max
+ * split gains: layers in proportion to each stage's speed (2^40 / time of
+ * all layers on its type and degree, rounded down; largest remainders, at
+ * least one layer per stage), else the fastest fitting split of a fixed
+ * list -- equal layer counts, layers in proportion to each stage's longest
+ * memory-fitting run -- else OOM; then the same Evaluate.  Results, status
+ * rules and the top-k are as for the other modes; bottleneck is the chosen
+ * split's largest stage time (not B*). */
 #define HEDDLE_SEARCH_AUTO 0
 #define HEDDLE_SEARCH_GENERAL 1
 #define HEDDLE_SEARCH_EQUAL_LAYERS 2
+#define HEDDLE_SEARCH_DISTRIBUTE 3
 heddle_status heddle_set_search(heddle_ctx* ctx, int32_t mode);
 heddle_status heddle_get_search(heddle_ctx* ctx, int32_t* in_use);
 

@@ -554,6 +554,7 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     a.wl_bucket = x->d_wl_bucket;
     a.wl_cap = hd::kWorklistCap;
     a.uniform = equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
+    a.split_mode = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? 1 : 0;
     a.wl_T = x->d_wl_T;
     a.wl_nM = x->d_wl_nM;
     // chunks of at most the worklist capacity, in stream order
@@ -778,7 +779,7 @@ heddle_status heddle_device_errors(heddle_ctx* x, uint32_t* flags) {
 
 heddle_status heddle_set_search(heddle_ctx* x, int32_t mode) {
     if (!x) return HEDDLE_E_ARG;
-    if (mode != HEDDLE_SEARCH_AUTO && mode != HEDDLE_SEARCH_GENERAL)
+    if (mode != HEDDLE_SEARCH_AUTO && mode != HEDDLE_SEARCH_GENERAL && mode != HEDDLE_SEARCH_DISTRIBUTE)
         return fail(x, HEDDLE_E_ARG, "unknown search mode %d", mode);
     x->search_mode = mode;
     return ok(x);
@@ -788,7 +789,9 @@ heddle_status heddle_get_search(heddle_ctx* x, int32_t* in_use) {
     if (!x || !in_use) return x ? fail(x, HEDDLE_E_ARG, "in_use is NULL") : HEDDLE_E_ARG;
     heddle_status st = check_ready(x);
     if (st != HEDDLE_OK) return st;
-    *in_use = equal_layer_search(x) ? HEDDLE_SEARCH_EQUAL_LAYERS : HEDDLE_SEARCH_GENERAL;
+    *in_use = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? HEDDLE_SEARCH_DISTRIBUTE
+              : equal_layer_search(x)                 ? HEDDLE_SEARCH_EQUAL_LAYERS
+                                                      : HEDDLE_SEARCH_GENERAL;
     return ok(x);
 }
 

@@ -128,6 +128,7 @@ struct PriceArgs {
     int32_t wl_cap;
     int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
     int32_t mbs_shift;   // micro-batch size 2^shift: M >> shift micro-batches (invalid unless 2^shift | M)
+    int32_t split_mode;  // 1: the paper's own split rule (distribute_kernel) instead of PartitionLayers
     // per worklist entry, written by the search: T (-1 unless OK) and n * M,
     // so a top-k can run over the searched candidates only
     int64_t* wl_T;
@@ -140,6 +141,8 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
                          int64_t* launches = nullptr);
 // The equal-layer search over the worklist the screen produced.
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
+// The paper's own layer split over the worklist (comparison mode).
+cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
 constexpr int kWlMeta = 1 + kMaxStages + 1;  // ints of a.wl_count
 

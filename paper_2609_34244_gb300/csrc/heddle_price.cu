@@ -752,6 +752,7 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
     if (launches) launches[0] += 1;
     if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
     if (launches) launches[1] += 1;
+    if (a.split_mode) return launch_distribute(a, num_sms, st);
     if (a.uniform) return launch_eq_search(a, num_sms, st);
     return a.counters ? launch_search<true>(a, num_sms, st) : launch_search<false>(a, num_sms, st);
 }

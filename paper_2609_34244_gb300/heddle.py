@@ -69,7 +69,7 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
 MAX_MBS_LEVELS = 4
 PHASES = ("screen", "search", "topk")
 TOPK_NOALLOC_MAX_N = 4194304
-SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS = 0, 1, 2
+SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS, SEARCH_DISTRIBUTE = 0, 1, 2, 3
 
 _lib = None
 
