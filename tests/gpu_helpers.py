@@ -100,9 +100,9 @@ def exact_topk(idx_all, T, nM, k):
     return items[:k]
 
 
-def price_mbs_gpu(h, w_cluster, w_model, cands, levels, profiles=None, bounds=True, search=None):
-    """Micro-batch-size fill on the GPU through the C ABI; numpy results
-    plus the chosen level ``mbs``."""
+def price_mbs_gpu(h, w_cluster, w_model, cands, levels, profiles=None, bounds=True, search=None, batch=None):
+    """Micro-batch-size fill on the GPU through the C ABI (one call, or one
+    per ``batch`` candidates); numpy results plus the chosen level ``mbs``."""
     import torch
     ctx = h.heddle_create(0)
     try:
@@ -115,7 +115,12 @@ def price_mbs_gpu(h, w_cluster, w_model, cands, levels, profiles=None, bounds=Tr
         dc = h.cands_to_device(cands)
         res = h.alloc_results(n, bounds=bounds)
         mbs = torch.full((max(n, 1),), 255, dtype=torch.uint8, device="cuda")
-        h.heddle_price_mbs(ctx, h.make_candidates(dc), h.make_results(res), mbs)
+        if batch is None:
+            h.heddle_price_mbs(ctx, h.make_candidates(dc), h.make_results(res), mbs)
+        else:
+            for lo in range(0, n, batch):
+                hi = min(n, lo + batch)
+                h.heddle_price_mbs(ctx, h.make_candidates(dc, lo, hi), h.make_results(res, lo, hi), mbs[lo:hi])
         torch.cuda.synchronize()
         out = h.results_to_numpy(res)
         out["mbs"] = mbs[:n].cpu().numpy()
