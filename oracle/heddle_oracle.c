@@ -265,7 +265,7 @@ int orc_replicas(int n_nodes, const int32_t* node_gpus, int n_groups,
  * A stage group of degree k larger than the largest node of its type (only
  * possible for an EP degree, §5.3) is placed as k/p blocks of p GPUs, p the
  * largest power of two not above that node size (reading). */
-static int64_t dp_degree(const orc_ctx* x, int S, const int* g, const int* j) {
+static int64_t dp_degree(const orc_ctx* x, int S, const int* g, const int* j, const int32_t* node_free) {
     int64_t best = INT64_MAX;
     int32_t* ng = (int32_t*)malloc(sizeof(int32_t) * x->n_nodes);
     for (int t = 0; t < x->n_types; ++t) {
@@ -282,7 +282,7 @@ static int64_t dp_degree(const orc_ctx* x, int S, const int* g, const int* j) {
         if (!used) continue;
         int nn = 0;
         for (int b = 0; b < x->n_nodes; ++b)
-            if (x->node_type[b] == t) ng[nn++] = x->node_gpus[b];
+            if (x->node_type[b] == t) ng[nn++] = node_free ? node_free[b] : x->node_gpus[b];
         int64_t r = replicas(nn, ng, cnt);
         if (r < best) best = r;
     }
@@ -478,8 +478,10 @@ static int distribute(const orc_ctx* x, int S, int L, int M, int64_t n, const in
     return found;
 }
 
+/* Price one candidate; node_free (nullable) replaces the cluster's GPUs per
+ * node for the DP degree (the GPUs a plan has left, Algorithm 1). */
 static void price_one(const orc_ctx* x, int S, int M, const uint8_t* codes, int64_t* f,
-                      int64_t* Wbuf, priced* out) {
+                      int64_t* Wbuf, priced* out, const int32_t* node_free) {
     int L = x->L;
     memset(out, 0, sizeof(*out));
     out->T = -1;
@@ -501,7 +503,7 @@ static void price_one(const orc_ctx* x, int S, int M, const uint8_t* codes, int6
         }
     }
     /* DP degree (§5.3) */
-    int64_t n = dp_degree(x, S, g, j);
+    int64_t n = dp_degree(x, S, g, j, node_free);
     if (n == 0) {
         out->status = ORC_NO_FIT;
         return;
@@ -582,7 +584,7 @@ static void* run_job(void* arg) {
             r.status = ORC_INVALID;
         } else {
             for (int s = 0; s < S && s < MAXS; ++s) codes[s] = jb->code[(int64_t)s * jb->stride + c];
-            price_one(x, S, jb->M[c], codes, f, Wbuf, &r);
+            price_one(x, S, jb->M[c], codes, f, Wbuf, &r, NULL);
         }
         jb->T[c] = r.T;
         jb->B[c] = r.B;
@@ -633,6 +635,107 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
     free(jobs);
     free(tid);
     return threads;
+}
+
+/* ------------------------------------------------- multi-template plans */
+
+/* Algorithm 1 builds a plan as a sequence of structural templates, each
+ * holding its own GPUs (§5 "Planning as autoregressive construction"); the
+ * reward of a step is the throughput the new template adds (§5.5,
+ * Eq. reward).  A plan is priced template by template against the GPUs the
+ * earlier templates left: the template's DP degree comes from the free
+ * GPUs per node, its groups are then placed -- largest first, each on a
+ * node of its type whose free GPUs equal the group size, else on the node
+ * with the fewest free GPUs above it (§5.1: a node whose size equals the
+ * requested degree first, else GPUs from a larger node; the earliest node
+ * on ties) -- and a template that does not fit (OOM, NO_FIT, INVALID) ends
+ * the plan at the templates placed so far.  Plan throughput (reading): the
+ * sum over placed templates of n M 1e9 / T base micro-batches per second,
+ * each term rounded in IEEE double, in template order. */
+static void place_groups(const orc_ctx* x, int S, const int* g, const int* j, int64_t n, int32_t* node_free) {
+    for (int e = 3; e >= 0; --e) {
+        int32_t w = 1 << e;
+        for (int s = 0; s < S; ++s) {
+            int k = 1 << j[s];
+            int eb = j[s];
+            while ((1 << eb) > x->maxnode[g[s]]) --eb;
+            if (eb != e) continue;
+            int64_t blocks = (int64_t)(k >> eb) * n;
+            for (int64_t b = 0; b < blocks; ++b) {
+                int pick = -1;
+                for (int d = 0; d < x->n_nodes; ++d)
+                    if (x->node_type[d] == g[s] && node_free[d] == w) {
+                        pick = d;
+                        break;
+                    }
+                if (pick < 0)
+                    for (int d = 0; d < x->n_nodes; ++d)
+                        if (x->node_type[d] == g[s] && node_free[d] > w &&
+                            (pick < 0 || node_free[d] < node_free[pick]))
+                            pick = d;
+                if (pick < 0) return; /* cannot happen: n came from these nodes */
+                node_free[pick] -= w;
+            }
+        }
+    }
+}
+
+int orc_price_plans(const orc_ctx* x, int64_t n_plans, int max_tmpl, const uint8_t* n_tmpl,
+                    const uint8_t* S, const uint16_t* M, const uint8_t* code, int s_max,
+                    int64_t* T, int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* placed,
+                    double* thr) {
+    int L = x->L;
+    int64_t* f = (int64_t*)malloc(sizeof(int64_t) * (size_t)(MAXS + 1) * (L + 1));
+    int64_t* Wbuf = (int64_t*)malloc(sizeof(int64_t) * (size_t)MAXS * (L + 1));
+    int32_t* node_free = (int32_t*)malloc(sizeof(int32_t) * (x->n_nodes > 0 ? x->n_nodes : 1));
+    for (int64_t c = 0; c < n_plans; ++c) {
+        for (int d = 0; d < x->n_nodes; ++d) node_free[d] = x->node_gpus[d];
+        int ended = 0, nt = n_tmpl[c] < max_tmpl ? n_tmpl[c] : max_tmpl;
+        double sum = 0.0;
+        placed[c] = 0;
+        for (int t = 0; t < max_tmpl; ++t) {
+            int64_t o = (int64_t)t * n_plans + c;
+            T[o] = -1;
+            bottleneck[o] = -1;
+            n_dp[o] = 0;
+            if (ended || t >= nt) {
+                status[o] = ORC_SKIPPED;
+                continue;
+            }
+            int St = S[o];
+            uint8_t codes[MAXS];
+            priced r;
+            if (St > s_max) {
+                memset(&r, 0, sizeof(r));
+                r.status = ORC_INVALID;
+            } else {
+                for (int s = 0; s < St && s < MAXS; ++s) codes[s] = code[((int64_t)t * s_max + s) * n_plans + c];
+                price_one(x, St, M[o], codes, f, Wbuf, &r, node_free);
+            }
+            status[o] = (uint8_t)r.status;
+            if (r.status != ORC_OK) {
+                n_dp[o] = (uint16_t)(r.status == ORC_OOM ? r.n : 0);
+                ended = 1;
+                continue;
+            }
+            T[o] = r.T;
+            bottleneck[o] = r.B;
+            n_dp[o] = (uint16_t)r.n;
+            sum = sum + ((double)(r.n * (int64_t)M[o]) * 1e9) / (double)r.T;
+            placed[c] = (uint8_t)(t + 1);
+            int g[MAXS], j[MAXS];
+            for (int s = 0; s < St; ++s) {
+                g[s] = codes[s] & 7;
+                j[s] = (codes[s] >> 3) & 3;
+            }
+            place_groups(x, St, g, j, r.n, node_free);
+        }
+        thr[c] = sum;
+    }
+    free(f);
+    free(Wbuf);
+    free(node_free);
+    return 0;
 }
 
 /* ------------------------------------------------------------ rank, top-k */

@@ -25,6 +25,7 @@ extern "C" {
 #define ORC_OOM 1
 #define ORC_NO_FIT 2
 #define ORC_INVALID 3
+#define ORC_SKIPPED 4 /* a plan's template after the plan ended */
 
 typedef struct orc_ctx orc_ctx;
 
@@ -60,6 +61,21 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
  * fixed list -- equal layer counts, layers in proportion to each stage's
  * longest memory-fitting run -- else OOM. */
 void orc_set_split(orc_ctx* x, int mode);
+
+/* Multi-template plans (Algorithm 1): n_plans plans of up to max_tmpl
+ * templates (n_tmpl[c] used); template t of plan c has depth S[t*n + c],
+ * micro-batches M[t*n + c] and stage codes code[(t*s_max + s)*n + c].
+ * Templates are priced in order against the GPUs the earlier ones left
+ * (DP degree from the free GPUs per node; groups placed largest first on a
+ * node whose free GPUs equal the group size, else the node with the fewest
+ * free GPUs above it); the first template that is not OK ends the plan.
+ * Per template [t*n + c]: T, bottleneck, n_dp, status (ORC_SKIPPED past
+ * the end); per plan: placed templates and throughput
+ * sum n*M*1e9/T (IEEE double, template order).  Single-threaded. */
+int orc_price_plans(const orc_ctx* x, int64_t n_plans, int max_tmpl, const uint8_t* n_tmpl,
+                    const uint8_t* S, const uint16_t* M, const uint8_t* code, int s_max,
+                    int64_t* T, int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* placed,
+                    double* thr);
 
 /* Top-k of the OK candidates by throughput n*M/T, ties to the smaller index.
  * idx = base_index + c.  Writes up to k entries; returns how many. */

@@ -21,7 +21,7 @@ SRC = os.path.join(HERE, "heddle_oracle.c")
 HDR = os.path.join(HERE, "heddle_oracle.h")
 LIB = os.path.join(HERE, "liboracle.so")
 
-OK, OOM, NO_FIT, INVALID = 0, 1, 2, 3
+OK, OOM, NO_FIT, INVALID, SKIPPED = 0, 1, 2, 3, 4
 
 _lib = None
 
@@ -57,6 +57,8 @@ def lib():
         L.orc_replicas.restype = C.c_int
         L.orc_replicas.argtypes = [C.c_int, p, C.c_int, p]
         L.orc_set_split.argtypes = [p, C.c_int]
+        L.orc_price_plans.restype = C.c_int
+        L.orc_price_plans.argtypes = [p, C.c_int64, C.c_int, p, p, p, p, C.c_int, p, p, p, p, p, p]
         _lib = L
     return _lib
 
@@ -96,6 +98,25 @@ class Oracle:
                                int(bool(model.get("moe", False))), _ptr(prof), err)
         if not self._h:
             raise ValueError("oracle rejected inputs: " + err.value.decode())
+
+    def price_plans(self, plans: dict) -> dict:
+        """Multi-template plans (Algorithm 1): ``plans`` holds ``n_tmpl[n]``,
+        ``S[t, n]``, ``M[t, n]`` and ``code[t, s, n]``.  Returns per template
+        ``T``, ``bottleneck``, ``n_dp``, ``status`` ([t, n]) and per plan
+        ``placed`` and ``thr`` (base micro-batches per second)."""
+        nt = np.ascontiguousarray(plans["n_tmpl"], dtype=np.uint8)
+        S = np.ascontiguousarray(plans["S"], dtype=np.uint8)
+        M = np.ascontiguousarray(plans["M"], dtype=np.uint16)
+        code = np.ascontiguousarray(plans["code"], dtype=np.uint8)
+        tmax, n = S.shape
+        s_max = int(code.shape[1])
+        out = {"T": np.zeros((tmax, n), np.int64), "bottleneck": np.zeros((tmax, n), np.int64),
+               "n_dp": np.zeros((tmax, n), np.uint16), "status": np.zeros((tmax, n), np.uint8),
+               "placed": np.zeros(n, np.uint8), "thr": np.zeros(n, np.float64)}
+        lib().orc_price_plans(self._h, n, tmax, _ptr(nt), _ptr(S), _ptr(M), _ptr(code), s_max, _ptr(out["T"]),
+                              _ptr(out["bottleneck"]), _ptr(out["n_dp"]), _ptr(out["status"]),
+                              _ptr(out["placed"]), _ptr(out["thr"]))
+        return out
 
     def set_split(self, mode: str):
         """``"minmax"`` (PartitionLayers, the default) or ``"distribute"``

@@ -354,6 +354,21 @@ def mbs_profiles(w, levels: int, seed: int = 0):
     return out
 
 
+def make_plans(w, n_plans: int, max_templates: int = 4, seed: int = 0) -> dict:
+    """Seeded multi-template plans for ``w`` (same cluster and model): plan
+    c holds n_tmpl[c] ~ U{1..max_templates} templates, each drawn from a pool
+    of the workload's own candidate recipe (depth, GPU types and degrees,
+    M).  Stage-major arrays per template slot: S[t, n], M[t, n],
+    code[t, s, n]."""
+    rng = np.random.default_rng(0xA11 + seed)
+    pool = make_workload(w.name, seed=w.seed, n=n_plans * max_templates).cands
+    pn = int(pool["S"].shape[0])
+    pick = rng.integers(0, pn, (max_templates, n_plans))
+    n_tmpl = rng.integers(1, max_templates + 1, n_plans).astype(np.uint8)
+    return {"n_tmpl": n_tmpl, "S": pool["S"][pick], "M": pool["M"][pick],
+            "code": np.ascontiguousarray(np.stack([pool["code"][:, pick[t]] for t in range(max_templates)]))}
+
+
 def make_workload(name: str, seed: int = 0, n: int | None = None) -> Workload:
     """Build the named workload; ``n`` overrides the candidate count (same
     cluster, model and candidate distribution)."""

@@ -430,6 +430,75 @@ def check_distribute_properties(O, seed=5):
     assert r["bounds"][:5, 1].tolist() == [0, 3, 6, 8, 10], r["bounds"][:, 1]
 
 
+def _plans_from(case_templates, n_tmpl, W):
+    """Plan arrays for one plan from per-template stage lists."""
+    tmax = len(case_templates)
+    S = np.zeros((tmax, 1), np.uint8)
+    M = np.full((tmax, 1), 4, np.uint16)
+    code = np.zeros((tmax, 32, 1), np.uint8)
+    for t, stages in enumerate(case_templates):
+        S[t, 0] = len(stages)
+        for s, (g, j) in enumerate(stages):
+            code[t, s, 0] = int(W.encode(g, j))
+    return {"n_tmpl": np.array([n_tmpl], np.uint8), "S": S, "M": M, "code": code}
+
+
+def check_plans_hand(O):
+    """Hand-worked multi-template plans (golden/hand_plans.json, Algorithm 1)."""
+    W = _workloads()
+    d = _load("hand_plans.json")
+    cl = d["cluster"]
+    cluster = W.make_cluster(cl["tflops"], cl["mem_bytes"], cl["intra_bw"], [tuple(x) for x in cl["nodes"]])
+    model = W.make_model(d["flops"], 0, 0, 0, 0, 0, 0)
+    orc = O.Oracle(cluster, model)
+    for case in d["cases"]:
+        r = orc.price_plans(_plans_from(case["templates"], case["n_tmpl"], W))
+        e = case["expect"]
+        name = case["name"]
+        assert r["status"][:, 0].tolist() == e["status"], (name, r["status"][:, 0])
+        assert r["n_dp"][:, 0].tolist() == e["n_dp"], (name, r["n_dp"][:, 0])
+        assert r["T"][:, 0].tolist() == e["T"], (name, r["T"][:, 0])
+        assert int(r["placed"][0]) == e["placed"], (name, r["placed"][0])
+        assert float(r["thr"][0]) == e["thr"], (name, r["thr"][0])
+
+
+def check_plans_properties(O, seed=2):
+    """Plans on seeded workloads: a template priced first equals the plain
+    price; ``placed`` counts the leading OK templates and later ones are
+    skipped; the throughput adds up the placed templates' terms; a later
+    template never has more replicas than it would on the whole cluster;
+    the GPUs of the placed templates fit the cluster."""
+    W = _workloads()
+    for name, n in (("dense32", 300), ("moe48", 300), ("tiny", 200)):
+        w = W.make_workload(name, seed=seed, n=n)
+        plans = W.make_plans(w, n, 4, seed=seed)
+        orc = O.Oracle(w.cluster, w.model)
+        r = orc.price_plans(plans)
+        first = orc.price({"S": plans["S"][0], "M": plans["M"][0], "code": plans["code"][0]})
+        for k in ("T", "bottleneck", "n_dp", "status"):
+            assert (r[k][0] == first[k]).all(), (name, k)
+        tmax = plans["S"].shape[0]
+        for c in range(n):
+            p = int(r["placed"][c])
+            st = r["status"][:, c]
+            assert (st[:p] == O.OK).all(), (name, c)
+            assert p == tmax or p == plans["n_tmpl"][c] or st[p] != O.OK, (name, c)
+            assert (st[p + 1:] == O.SKIPPED).all() or (p < plans["n_tmpl"][c] and (st[p + 1:] == O.SKIPPED).all())
+            acc = 0.0
+            used = np.zeros(8, np.int64)
+            for t in range(p):
+                acc = acc + (float(int(r["n_dp"][t, c]) * int(plans["M"][t, c])) * 1e9) / float(r["T"][t, c])
+                alone = orc.price({"S": plans["S"][t, c:c + 1], "M": plans["M"][t, c:c + 1],
+                                   "code": plans["code"][t, :, c:c + 1]})
+                assert int(r["n_dp"][t, c]) <= int(alone["n_dp"][0]), (name, c, t)
+                for s in range(int(plans["S"][t, c])):
+                    b = int(plans["code"][t, s, c])
+                    used[b & 7] += int(r["n_dp"][t, c]) << ((b >> 3) & 3)
+            assert acc == float(r["thr"][c]), (name, c)
+            for g in range(len(w.cluster["tflops"])):
+                assert used[g] <= int(w.cluster["node_gpus"][w.cluster["node_type"] == g].sum()), (name, c, g)
+
+
 ALL_CHECKS = [
     check_hand_partitions,
     check_hand_pricing,
@@ -444,4 +513,6 @@ ALL_CHECKS = [
     check_mbs_properties,
     check_distribute_hand,
     check_distribute_properties,
+    check_plans_hand,
+    check_plans_properties,
 ]

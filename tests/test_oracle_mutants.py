@@ -63,6 +63,14 @@ MUTANTS = [
     ("distribute_time_not_speed", "w[0][s] = all > 0 ? ((int64_t)1 << 40) / all : ((int64_t)1 << 40);",
      "w[0][s] = all;"),
     ("distribute_memory_ignored", "if (W[s][b[s + 1]] - W[s][b[s]] > cap[s]) fits = 0;", "(void)cap;"),
+    ("plans_first_fit_not_exact_size", "if (x->node_type[d] == g[s] && node_free[d] == w) {",
+     "if (x->node_type[d] == g[s] && node_free[d] >= w) {"),
+    ("plans_continue_after_failure", "                ended = 1;\n                continue;",
+     "                continue;"),
+    ("plans_degree_from_whole_cluster", "price_one(x, St, M[o], codes, f, Wbuf, &r, node_free);",
+     "price_one(x, St, M[o], codes, f, Wbuf, &r, NULL);"),
+    ("plans_throughput_per_ns", "sum = sum + ((double)(r.n * (int64_t)M[o]) * 1e9) / (double)r.T;",
+     "sum = sum + ((double)(r.n * (int64_t)M[o])) / (double)r.T;"),
 ]
 
 # planted mistakes in the Python part of the oracle (the micro-batch fill)
