@@ -56,7 +56,8 @@ enum {
     HEDDLE_CAND_OK = 0,
     HEDDLE_CAND_OOM = 1,     /* no layer split fits the GPUs' memory (§5.2) */
     HEDDLE_CAND_NO_FIT = 2,  /* not one replica can be placed on the nodes */
-    HEDDLE_CAND_INVALID = 3  /* masked structure (§5.1): see heddle_price_candidates */
+    HEDDLE_CAND_INVALID = 3, /* masked structure (§5.1): see heddle_price_candidates */
+    HEDDLE_CAND_SKIPPED = 4  /* a plan's template after the plan ended (heddle_price_plans) */
 };
 
 typedef struct heddle_ctx heddle_ctx;
@@ -306,6 +307,52 @@ heddle_status heddle_load_mbs(heddle_ctx* ctx, int32_t levels, const double* pro
 heddle_status heddle_price_mbs(heddle_ctx* ctx, const heddle_candidates* cands,
                                const heddle_results* results, uint8_t* mbs, void* stream);
 
+/* ----------------------------------------------- multi-template plans */
+
+/* Algorithm 1 builds a plan as a sequence of structural templates, each
+ * holding its own GPUs; the reward of a step is the throughput the new
+ * template adds (§5.5, Eq. reward).  heddle_price_plans prices a batch of
+ * such plans: template t of a plan is priced against the GPUs templates
+ * 0 .. t-1 left.  Its DP degree comes from the free GPUs per node (the
+ * closed form of heddle_price_candidates on the free counts); its groups are
+ * then placed largest first, each on a node of its type whose free GPUs
+ * equal the group size, else on the node with the fewest free GPUs above it
+ * (§5.1: a node whose size equals the degree first, else GPUs from a larger
+ * node).  The layer split, the bottleneck and OOM do not depend on the DP
+ * degree, so each slot is first priced as standalone candidates with the
+ * context's search mode, then re-evaluated with the plan's degree.  The
+ * first template that is not OK (INVALID, NO_FIT on the GPUs left, OOM)
+ * ends the plan; later templates are SKIPPED.  The plan's throughput is
+ * the sum over its placed templates of n * M * 1e9 / T base micro-batches
+ * per second, each term rounded in IEEE double, in template order (so the
+ * step rewards are those terms).
+ *
+ * plans: n plans (0 <= n <= 2^20 per call), slots (1..HEDDLE_MAX_TEMPLATES)
+ * template slots; n_templates[c] (device u8) the templates of plan c
+ * (values above slots count as slots); t[i] the candidates of slot i
+ * (device arrays as heddle_candidates, t[i].n == n).
+ * results: per slot device arrays as heddle_results (T, bottleneck, n_dp,
+ * status, optional bounds), overwritten with the plan's prices; placed[c]
+ * (device u8) the templates placed; thr[c] (device double) the throughput.
+ * Asynchronous on `stream`.  Errors: E_ARG, E_STATE, E_LIMIT (n above 2^20,
+ * a node of more than HEDDLE_PLAN_MAX_NODE GPUs), E_CUDA, E_NOMEM. */
+#define HEDDLE_MAX_TEMPLATES 4
+#define HEDDLE_PLAN_MAX_NODE 64
+typedef struct {
+    int64_t n;
+    int32_t slots;
+    int32_t reserved;
+    const uint8_t* n_templates;
+    heddle_candidates t[HEDDLE_MAX_TEMPLATES];
+} heddle_plans;
+typedef struct {
+    heddle_results t[HEDDLE_MAX_TEMPLATES];
+    uint8_t* placed;
+    double* thr;
+} heddle_plan_results;
+heddle_status heddle_price_plans(heddle_ctx* ctx, const heddle_plans* plans,
+                                 const heddle_plan_results* results, void* stream);
+
 /* -------------------------------------------------------- host buffers */
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the
@@ -351,7 +398,9 @@ heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
  * all layers on its type and degree, rounded down; largest remainders, at
  * least one layer per stage), else the fastest fitting split of a fixed
  * list -- equal layer counts, layers in proportion to each stage's longest
- * memory-fitting run -- else OOM; then the same Evaluate.  Results, status
+ * memory-fitting run -- else OOM; "fastest" is the smallest pipeline time
+ * (M-1) max t_s + sum t_s (Algorithm 1 splits before it picks the DP
+ * degree); then the same Evaluate.  Results, status
  * rules and the top-k are as for the other modes; bottleneck is the chosen
  * split's largest stage time (not B*). */
 #define HEDDLE_SEARCH_AUTO 0

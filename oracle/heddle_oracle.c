@@ -395,7 +395,9 @@ static int64_t evaluate(const orc_ctx* x, int S, int M, int64_t n, const int64_t
  * time of all L layers on its type and degree, rounded down; the list is
  * (1) in proportion to speed, (2) equal layer counts, (3) in proportion to
  * the longest run of consecutive layers each stage's memory holds; the
- * fastest is the smallest T, the earlier alternative on ties. */
+ * fastest is the smallest pipeline time (M-1) max t_s + sum t_s, the
+ * earlier alternative on ties -- Algorithm 1 splits the layers before the
+ * fill picks the DP degree, so the choice cannot see the gradient term. */
 
 /* L layers over S stages in proportion to weights w >= 0 (sum > 0): floor
  * of the exact share, at least one layer per stage; missing layers go one
@@ -456,6 +458,7 @@ static int distribute(const orc_ctx* x, int S, int L, int M, int64_t n, const in
         w[2][s] = longest_run(W[s], L, cap[s]);
     }
     int found = 0;
+    int64_t best_pipe = 0;
     for (int alt = 0; alt < 3; ++alt) {
         int64_t V = 0;
         for (int s = 0; s < S; ++s) V += w[alt][s];
@@ -466,15 +469,20 @@ static int distribute(const orc_ctx* x, int S, int L, int M, int64_t n, const in
         for (int s = 0; s < S && fits; ++s)
             if (W[s][b[s + 1]] - W[s][b[s]] > cap[s]) fits = 0;
         if (!fits) continue;
-        int64_t tmax;
-        int64_t T = evaluate(x, S, M, n, P, c, j, g, b, &tmax);
-        if (!found || T < *T_out) {
+        int64_t tmax = 0, tsum = 0;
+        for (int s = 0; s < S; ++s) {
+            int64_t t = P[s][b[s + 1]] - P[s][b[s]] + c[s];
+            if (t > tmax) tmax = t;
+            tsum += t;
+        }
+        int64_t pipe = (int64_t)(M - 1) * tmax + tsum;
+        if (!found || pipe < best_pipe) {
             found = 1;
-            *T_out = T;
-            *B_out = tmax;
+            best_pipe = pipe;
             for (int s = 0; s <= S; ++s) a[s] = b[s];
         }
     }
+    if (found) *T_out = evaluate(x, S, M, n, P, c, j, g, a, B_out);
     return found;
 }
 

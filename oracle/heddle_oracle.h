@@ -59,7 +59,9 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
  * layers in proportion to each stage's speed (2^40 / time of all layers on
  * its type and degree, rounded down), else the fastest fitting split of a
  * fixed list -- equal layer counts, layers in proportion to each stage's
- * longest memory-fitting run -- else OOM. */
+ * longest memory-fitting run -- else OOM; "fastest" is the smallest
+ * pipeline time (M-1) max t_s + sum t_s (the split precedes the DP degree
+ * in Algorithm 1). */
 void orc_set_split(orc_ctx* x, int mode);
 
 /* Multi-template plans (Algorithm 1): n_plans plans of up to max_tmpl

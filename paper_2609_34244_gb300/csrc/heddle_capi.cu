@@ -100,6 +100,13 @@ struct heddle_ctx {
     uint8_t* lv_status = nullptr;
     uint8_t* lv_bounds = nullptr;
     size_t lv_T_cap = 0, lv_B_cap = 0, lv_n_cap = 0, lv_status_cap = 0, lv_bounds_cap = 0;
+    // multi-template plans: the cluster's nodes on the device, split bounds
+    // of slots whose caller passed none
+    int32_t* d_node_type = nullptr;
+    int32_t* d_node_gpus = nullptr;
+    size_t node_cap = 0, node_cap2 = 0;
+    uint8_t* plan_bounds[HEDDLE_MAX_TEMPLATES] = {nullptr, nullptr, nullptr, nullptr};
+    size_t plan_bounds_cap[HEDDLE_MAX_TEMPLATES] = {0, 0, 0, 0};
 };
 
 namespace {
@@ -409,6 +416,9 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->lv_n);
     cudaFree(x->lv_status);
     cudaFree(x->lv_bounds);
+    cudaFree(x->d_node_type);
+    cudaFree(x->d_node_gpus);
+    for (auto* b : x->plan_bounds) cudaFree(b);
     for (auto& r : x->phase_recs)
         for (cudaEvent_t ev : r.e) x->ev_pool.push_back(ev);
     for (cudaEvent_t ev : x->ev_pool) cudaEventDestroy(ev);
@@ -874,6 +884,78 @@ heddle_status heddle_price_mbs(heddle_ctx* x, const heddle_candidates* c, const 
             CU(hd::launch_mbs_merge(m, x->num_sms, sm));
         }
     }
+    return ok(x);
+}
+
+heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const heddle_plan_results* pr,
+                                 void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!pl || !pr) return fail(x, HEDDLE_E_ARG, "plans or results is NULL");
+    heddle_status st = check_ready(x);
+    if (st != HEDDLE_OK) return st;
+    if (pl->n < 0) return fail(x, HEDDLE_E_ARG, "negative plan count");
+    if (pl->n > hd::kWorklistCap) return fail(x, HEDDLE_E_LIMIT, "more than 2^20 plans in one call");
+    if (pl->slots < 1 || pl->slots > HEDDLE_MAX_TEMPLATES)
+        return fail(x, HEDDLE_E_ARG, "slots must be in [1, %d]", HEDDLE_MAX_TEMPLATES);
+    if (pl->n == 0) return ok(x);
+    if (!pl->n_templates || !pr->placed || !pr->thr) return fail(x, HEDDLE_E_ARG, "null plan array");
+    for (int t = 0; t < pl->slots; ++t) {
+        if (pl->t[t].n != pl->n) return fail(x, HEDDLE_E_ARG, "slot %d holds %lld candidates, not n", t,
+                                             (long long)pl->t[t].n);
+        if ((st = check_cands(x, &pl->t[t], true)) != HEDDLE_OK) return st;
+        const heddle_results& r = pr->t[t];
+        if (!r.T || !r.bottleneck || !r.n_dp || !r.status) return fail(x, HEDDLE_E_ARG, "null result array, slot %d", t);
+    }
+    for (const auto& nd : x->nodes)
+        if (nd.gpus > HEDDLE_PLAN_MAX_NODE)
+            return fail(x, HEDDLE_E_LIMIT, "plans need nodes of at most %d GPUs", HEDDLE_PLAN_MAX_NODE);
+    DeviceGuard dg(x->device);
+    cudaStream_t sm = (cudaStream_t)stream;
+    const size_t nn = x->nodes.size();
+    CU(grow(&x->d_node_type, &x->node_cap, sizeof(int32_t) * nn));
+    CU(grow(&x->d_node_gpus, &x->node_cap2, sizeof(int32_t) * nn));
+    {
+        std::vector<int32_t> ty(nn), gp(nn);
+        for (size_t b = 0; b < nn; ++b) {
+            ty[b] = x->nodes[b].type;
+            gp[b] = x->nodes[b].gpus;
+        }
+        CU(cudaMemcpy(x->d_node_type, ty.data(), sizeof(int32_t) * nn, cudaMemcpyHostToDevice));
+        CU(cudaMemcpy(x->d_node_gpus, gp.data(), sizeof(int32_t) * nn, cudaMemcpyHostToDevice));
+    }
+    hd::PlanArgs a{};
+    a.lay = x->lay;
+    a.img = x->d_img;
+    a.n = pl->n;
+    a.slots = pl->slots;
+    a.n_tmpl = pl->n_templates;
+    a.node_type = x->d_node_type;
+    a.node_gpus = x->d_node_gpus;
+    a.n_nodes = (int32_t)nn;
+    a.placed = pr->placed;
+    a.thr = pr->thr;
+    a.err = x->d_flags + 1;
+    // every slot priced as standalone candidates (the split needs bounds)
+    for (int t = 0; t < pl->slots; ++t) {
+        heddle_results r = pr->t[t];
+        if (!r.bounds) {
+            CU(grow(&x->plan_bounds[t], &x->plan_bounds_cap[t], (size_t)(HEDDLE_MAX_STAGES + 1) * pl->n));
+            r.bounds = x->plan_bounds[t];
+        }
+        if ((st = price_impl(x, &pl->t[t], &r, nullptr, stream)) != HEDDLE_OK) return st;
+        hd::PlanSlot& s = a.slot[t];
+        s.S = pl->t[t].S;
+        s.M = pl->t[t].M;
+        s.code = pl->t[t].code;
+        s.stride = pl->t[t].plane_stride;
+        s.T = r.T;
+        s.B = r.bottleneck;
+        s.ndp = r.n_dp;
+        s.status = r.status;
+        s.bounds = r.bounds;
+        s.bstride = pl->n;
+    }
+    CU(hd::launch_plans(a, x->num_sms, sm));
     return ok(x);
 }
 

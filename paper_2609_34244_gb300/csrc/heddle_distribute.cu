@@ -13,8 +13,10 @@
 // each stage's memory holds; shares are floors of L w_s / sum w with at
 // least one layer per stage, missing layers to the largest remainders (the
 // earlier stage on ties), surplus layers off the stage holding the most
-// (the later stage on ties); the fastest is the smallest T, the earlier
-// alternative on ties.  No alternative fits: OOM.
+// (the later stage on ties); the fastest is the smallest pipeline time
+// (M-1) max t_s + sum t_s, the earlier alternative on ties (Algorithm 1
+// splits the layers before the fill picks the DP degree, so the choice
+// cannot see the gradient term).  No alternative fits: OOM.
 //
 // One thread per worklist entry (the screen has already rejected the
 // candidates no split fits); the small tables are read through the L1
@@ -113,7 +115,7 @@ __global__ void __launch_bounds__(kDistBlock) distribute_kernel(PriceArgs a) {
             for (int k = 0; k < 3; ++k) V[k] += w[k][s];
         }
         bool found = false;
-        int64_t bestT = 0, bestB = 0;
+        int64_t bestT = 0, bestB = 0, bestPipe = 0;
         uint8_t bestb[kMaxStages + 1];
         for (int alt = 0; alt < 3; ++alt) {
             if (V[alt] <= 0) continue;
@@ -125,37 +127,39 @@ __global__ void __launch_bounds__(kDistBlock) distribute_kernel(PriceArgs a) {
                 fits = (hi.x - lo.x) + (int64_t)fs[s] * (hi.y - lo.y) <= capk[s];
             }
             if (!fits) continue;
-            // Evaluate: T = (M-1) max t_s + sum t_s + max g_s
+            // the pipeline time of this split decides between alternatives
             int64_t tmax = 0, tsum = 0;
-            uint64_t bestG = 0, bestD = 1;
-            int sg = -1;
             for (int s = 0; s < S; ++s) {
                 const int64_t t = P[row[s] + b[s + 1]] - P[row[s] + b[s]] + cs[s];
                 tmax = max(tmax, t);
                 tsum += t;
-                if (n > 1) {
-                    const uint64_t G = (uint64_t)(PB[b[s + 1]] - PB[b[s]]);
-                    if (sg < 0 || (u128)G * bestD > (u128)bestG * D[s]) {
-                        sg = s;
-                        bestG = G;
-                        bestD = D[s];
-                    }
-                }
             }
-            int64_t gmax = 0;
-            if (n > 1) {
-                const u128 num = (u128)(2 * (uint64_t)(n - 1) * 1000000000ull) * bestG;
-                bool ok = true;
-                gmax = (int64_t)ceil_div_u128(num, (uint64_t)n * bestD, &ok);
-                if (!ok) atomicOr(a.err, kErrInternal);
-            }
-            const int64_t T = (int64_t)(M - 1) * tmax + tsum + gmax;
-            if (!found || T < bestT) {
+            const int64_t pipe = (int64_t)(M - 1) * tmax + tsum;
+            if (!found || pipe < bestPipe) {
                 found = true;
-                bestT = T;
+                bestPipe = pipe;
+                bestT = pipe;
                 bestB = tmax;
                 for (int s = 0; s <= S; ++s) bestb[s] = b[s];
             }
+        }
+        if (found && n > 1) {
+            // Evaluate adds the gradient term: the stage with the largest
+            // G_s / (k_s bw_s), compared exactly, then ceil(2(n-1) G 1e9 / (n k bw))
+            uint64_t bestG = 0, bestD = 1;
+            int sg = -1;
+            for (int s = 0; s < S; ++s) {
+                const uint64_t G = (uint64_t)(PB[bestb[s + 1]] - PB[bestb[s]]);
+                if (sg < 0 || (u128)G * bestD > (u128)bestG * D[s]) {
+                    sg = s;
+                    bestG = G;
+                    bestD = D[s];
+                }
+            }
+            const u128 num = (u128)(2 * (uint64_t)(n - 1) * 1000000000ull) * bestG;
+            bool ok = true;
+            bestT += (int64_t)ceil_div_u128(num, (uint64_t)n * bestD, &ok);
+            if (!ok) atomicOr(a.err, kErrInternal);
         }
         if (found) {
             a.T[c] = bestT;

@@ -141,6 +141,39 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
                          int64_t* launches = nullptr);
 // The equal-layer search over the worklist the screen produced.
 cudaError_t launch_eq_search(const PriceArgs& a, int num_sms, cudaStream_t st);
+// Multi-template plans (Algorithm 1): per template slot the plans' arrays,
+// already priced standalone (bounds required), overwritten with the plan's
+// prices; per plan the templates placed and the summed throughput.
+constexpr int kMaxTemplates = HEDDLE_MAX_TEMPLATES;
+constexpr int kPlanMaxNode = HEDDLE_PLAN_MAX_NODE;
+struct PlanSlot {
+    const uint8_t* S;
+    const uint16_t* M;
+    const uint8_t* code;  // [s][stride]
+    int64_t stride;
+    int64_t* T;
+    int64_t* B;
+    uint16_t* ndp;
+    uint8_t* status;
+    uint8_t* bounds;  // [33][bstride]
+    int64_t bstride;
+};
+struct PlanArgs {
+    Layout lay;
+    const unsigned char* img;
+    int64_t n;
+    int32_t slots;
+    const uint8_t* n_tmpl;
+    PlanSlot slot[kMaxTemplates];
+    const int32_t* node_type;
+    const int32_t* node_gpus;
+    int32_t n_nodes;
+    uint8_t* placed;
+    double* thr;
+    uint32_t* err;
+};
+cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st);
+
 // The paper's own layer split over the worklist (comparison mode).
 cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;

@@ -53,6 +53,19 @@ class heddle_results(C.Structure):
                 ("status", C.c_void_p), ("bounds", C.c_void_p)]
 
 
+MAX_TEMPLATES = 4
+CAND_SKIPPED = 4
+
+
+class heddle_plans(C.Structure):
+    _fields_ = [("n", C.c_int64), ("slots", C.c_int32), ("reserved", C.c_int32),
+                ("n_templates", C.c_void_p), ("t", heddle_candidates * MAX_TEMPLATES)]
+
+
+class heddle_plan_results(C.Structure):
+    _fields_ = [("t", heddle_results * MAX_TEMPLATES), ("placed", C.c_void_p), ("thr", C.c_void_p)]
+
+
 class heddle_topk_state(C.Structure):
     _fields_ = [("k", C.c_int32), ("count", C.c_int32), ("idx", C.c_int64 * MAX_TOPK),
                 ("T", C.c_int64 * MAX_TOPK), ("nM", C.c_uint32 * MAX_TOPK)]
@@ -65,7 +78,7 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
            "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
            "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times",
-           "heddle_load_mbs", "heddle_price_mbs"]
+           "heddle_load_mbs", "heddle_price_mbs", "heddle_price_plans"]
 MAX_MBS_LEVELS = 4
 PHASES = ("screen", "search", "topk")
 TOPK_NOALLOC_MAX_N = 4194304
@@ -103,6 +116,7 @@ def load_library(path: str = LIB_PATH):
         "heddle_get_search": (i32, [p, C.POINTER(C.c_int32)]),
         "heddle_time_phases": (i32, [p, i32]),
         "heddle_load_mbs": (i32, [p, i32, p]),
+        "heddle_price_plans": (i32, [p, p, p, p]),
         "heddle_price_mbs": (i32, [p, p, p, p, p]),
         "heddle_phase_times": (i32, [p, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
     }
@@ -231,6 +245,39 @@ def heddle_price_mbs(ctx, cands, results, mbs=None, stream=None):
     r = results if isinstance(results, heddle_results) else make_results(results)
     _check(ctx, load_library().heddle_price_mbs(ctx, C.byref(c), C.byref(r),
                                                 None if mbs is None else _ptr(mbs), _stream(stream)))
+
+
+def plans_to_device(plans: dict, device="cuda") -> dict:
+    """Copy host plan arrays (n_tmpl[n], S[t, n], M[t, n], code[t, s, n]) to
+    CUDA tensors, one candidate SoA per template slot."""
+    import torch
+    slots = [cands_to_device({"S": plans["S"][t], "M": plans["M"][t], "code": plans["code"][t]}, device)
+             for t in range(plans["S"].shape[0])]
+    return {"n_tmpl": torch.from_numpy(np.ascontiguousarray(plans["n_tmpl"])).to(device), "slots": slots}
+
+
+def alloc_plan_results(n: int, slots: int, bounds: bool = False, device="cuda") -> dict:
+    import torch
+    return {"slots": [alloc_results(n, bounds=bounds, device=device) for _ in range(slots)],
+            "placed": torch.empty(n, dtype=torch.uint8, device=device),
+            "thr": torch.empty(n, dtype=torch.float64, device=device)}
+
+
+def heddle_price_plans(ctx, dplans: dict, pres: dict, stream=None):
+    """Price device plans (``plans_to_device``) into ``alloc_plan_results``."""
+    slots = len(dplans["slots"])
+    n = int(dplans["n_tmpl"].shape[0])
+    pl = heddle_plans()
+    pl.n = n
+    pl.slots = slots
+    pl.n_templates = _ptr(dplans["n_tmpl"])
+    pr = heddle_plan_results()
+    for t in range(slots):
+        pl.t[t] = make_candidates(dplans["slots"][t])
+        pr.t[t] = make_results(pres["slots"][t])
+    pr.placed = _ptr(pres["placed"])
+    pr.thr = _ptr(pres["thr"])
+    _check(ctx, load_library().heddle_price_plans(ctx, C.byref(pl), C.byref(pr), _stream(stream)))
 
 
 def heddle_topk_reset(ctx, state, k: int, stream=None):

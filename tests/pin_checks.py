@@ -422,6 +422,14 @@ def check_distribute_properties(O, seed=5):
         assert (dist["status"][same & (exact["status"] != O.OK)] == exact["status"][same & (exact["status"] != O.OK)]).all()
         if name != "moe48":  # moe48 is 1% OK even under the exact split
             assert okd.sum() > 0, name
+        # the split precedes the DP degree (Algorithm 1): gradient bytes,
+        # which only the gradient term sees, cannot change it
+        m0 = dict(w.model)
+        m0["param_bytes"] = np.zeros_like(np.asarray(w.model["param_bytes"]))
+        d0 = O.Oracle(w.cluster, m0).set_split("distribute").price(w.cands)
+        assert (d0["status"] == dist["status"]).all(), name
+        assert (d0["bottleneck"] == dist["bottleneck"]).all(), name
+        assert (d0["bounds"] == dist["bounds"]).all(), name
     cluster = W.make_cluster([1000.0], [10**13], [10**11], [(0, 8, 10**10)])
     model = W.make_model([1e12] * 10, 0, 0, 0, 0, 0, 0)
     cands = W.from_structures([[(0, 0)] * 3, [(0, 0)] * 4], [8, 8])

@@ -22,7 +22,7 @@ MUTANTS = [
     ("drop_p2p_in_dp", "int64_t t = P[s][j] - P[s][i] + c[s];", "int64_t t = P[s][j] - P[s][i];"),
     ("memory_strict", "if (W[s][j] - W[s][i] > cap[s]) continue;\n                int64_t t",
      "if (W[s][j] - W[s][i] >= cap[s]) continue;\n                int64_t t"),
-    ("iteration_M_not_M_minus_1", "(int64_t)(M - 1) * tmax", "(int64_t)M * tmax"),
+    ("iteration_M_not_M_minus_1", "return (int64_t)(M - 1) * tmax", "return (int64_t)M * tmax"),
     ("drop_grad_sync", "+ tsum + gmax;", "+ tsum;"),
     ("drop_sum_term", "return (int64_t)(M - 1) * tmax + tsum + gmax;",
      "return (int64_t)(M - 1) * tmax + tmax + gmax;"),
@@ -71,6 +71,8 @@ MUTANTS = [
      "price_one(x, St, M[o], codes, f, Wbuf, &r, NULL);"),
     ("plans_throughput_per_ns", "sum = sum + ((double)(r.n * (int64_t)M[o]) * 1e9) / (double)r.T;",
      "sum = sum + ((double)(r.n * (int64_t)M[o])) / (double)r.T;"),
+    ("distribute_choice_sees_gradient", "int64_t pipe = (int64_t)(M - 1) * tmax + tsum;",
+     "int64_t tm2, pipe = evaluate(x, S, M, n, P, c, j, g, b, &tm2);"),
 ]
 
 # planted mistakes in the Python part of the oracle (the micro-batch fill)
