@@ -19,6 +19,11 @@
  *   evaluate     §5.3 iteration time of a 1F1B pipeline,
  *                (M-1) max_s t_s + sum_s t_s + max_s g_s.
  *   rank, top-k  §5 overview: plans are ranked by predicted throughput.
+ *   tiling       §5.3 "Expert tiling" (optional, orc_set_experts): a stage's
+ *                expert layers factor its devices into EP x ETP x EDP; every
+ *                factorisation that fits memory is priced, the stage keeps
+ *                the fastest, and the per-stage choices are re-selected
+ *                against the whole iteration time.
  *
  * Readings of points the paper leaves open (quantisation, P2P, memory and
  * gradient-sync formulas, tie-breaks) are the ones listed in the design
@@ -59,6 +64,17 @@ struct orc_ctx {
     int64_t* param;  /* [L+1] prefix of gradient (parameter) bytes */
     int64_t p2p[MAXT][MAXT][2];
     int split_mode;  /* 0: min-max PartitionLayers, 1: the paper's Distribute rule */
+    /* the layers' cost inputs, kept for the expert-tiling tables */
+    double tflops[MAXT];
+    double* flops;
+    int64_t *ar, *a2a;
+    int has_profile;
+    /* expert tiling (0: off) */
+    int tiled;
+    int64_t* estate;  /* [L+1] prefix of the expert part of state bytes */
+    int64_t* eparam;  /* [L+1] prefix of the expert part of gradient bytes */
+    int64_t* Pt;      /* [n_types][20][L+1] prefix of per-layer ns per tiling slot */
+    int tvalid[MAXT][20];
 };
 
 /* ---------------------------------------------------------------- tables */
@@ -116,6 +132,16 @@ orc_ctx* orc_create(int n_types, const double* tflops, const int64_t* mem_bytes,
     x->n_types = n_types;
     x->L = L;
     x->moe = moe != 0;
+    x->has_profile = profile_s != NULL;
+    x->flops = (double*)malloc(sizeof(double) * L);
+    x->ar = (int64_t*)malloc(sizeof(int64_t) * L);
+    x->a2a = (int64_t*)malloc(sizeof(int64_t) * L);
+    for (int l = 0; l < L; ++l) {
+        x->flops[l] = flops ? flops[l] : 0.0;
+        x->ar[l] = ar_bytes ? ar_bytes[l] : 0;
+        x->a2a[l] = a2a_bytes ? a2a_bytes[l] : 0;
+    }
+    for (int g = 0; g < n_types; ++g) x->tflops[g] = tflops[g];
     x->n_nodes = n_nodes;
     x->node_type = (int32_t*)malloc(sizeof(int32_t) * n_nodes);
     x->node_gpus = (int32_t*)malloc(sizeof(int32_t) * n_nodes);
@@ -199,6 +225,12 @@ void orc_destroy(orc_ctx* x) {
     free(x->state);
     free(x->act);
     free(x->param);
+    free(x->flops);
+    free(x->ar);
+    free(x->a2a);
+    free(x->estate);
+    free(x->eparam);
+    free(x->Pt);
     free(x);
 }
 
@@ -210,6 +242,116 @@ void orc_tables(const orc_ctx* x, int64_t* q, int64_t* p2p, int32_t* maxnode,
         if (maxnode) maxnode[g] = x->maxnode[g];
         if (inter_bw) inter_bw[g] = x->inter_bw[g];
     }
+}
+
+/* --------------------------------------------------------- expert tiling */
+
+/* §5.3 "Expert tiling": the 2^j devices of a stage factor as EP x ETP x EDP
+ * (e t d = 2^j).  With power-of-two degrees a tiling is the exponent pair
+ * (le, lt), ld = j - le - lt; the 1 + 3 + 6 + 10 tilings of 1, 2, 4 and 8
+ * devices take slots 0, 1-3, 4-9 and 10-19, in the order EDP exponent
+ * ascending, then ETP exponent ascending.  Slot 0 of every degree (EP over
+ * all devices, no ETP, no EDP) is the untiled stage. */
+static const int tile_base[4] = {0, 1, 4, 10};
+
+static void tiling_of(int j, int idx, int* le, int* lt, int* ld) {
+    int k = 0;
+    for (int d = 0; d <= j; ++d)
+        for (int t = 0; t + d <= j; ++t) {
+            if (k == idx) {
+                *ld = d;
+                *lt = t;
+                *le = j - d - t;
+                return;
+            }
+            ++k;
+        }
+}
+
+/* Per-layer seconds of layer l on a stage of type g with 2^j devices tiled
+ * as (2^le EP, 2^lt ETP, 2^(j-le-lt) EDP).  Readings (the paper names the
+ * collectives of each direction but prints no formula):
+ *   compute  flops / (k * TFLOPS * 1e12): every tiling spreads the layer's
+ *            work over all k devices
+ *   TP       k > 1: the dense part's four ring all-reduces of ar_bytes over
+ *            the k devices, as for an untiled stage
+ *   EP       e > 1: four all-to-alls of a2a_bytes, each moving (e-1)/e; ETP
+ *            is the innermost factor, so an EP group spans e * t
+ *            consecutive devices and uses the NIC once that leaves a node
+ *   ETP      t > 1: four ring all-reduces of a2a_bytes (the expert output),
+ *            2(t-1)/t each, inside a node (ETP carries TP's node bound)
+ *   EDP      no per-micro-batch traffic; it replicates the expert state
+ *            (memory) and synchronises expert gradients (evaluate)
+ * The untiled slot reproduces the untiled cost bit for bit. */
+static double tiled_seconds(const orc_ctx* x, int g, int j, int le, int lt, int l) {
+    double k = (double)(1 << j);
+    double sec = x->flops[l] / (k * x->tflops[g] * 1e12);
+    double near = (double)x->intra_bw[g], far = (double)x->inter_bw[g];
+    if (j > 0) {
+        double bw = (1 << j) <= x->maxnode[g] ? near : far;
+        double w = (2.0 * (k - 1.0)) / k;
+        sec = sec + ((4.0 * w) * (double)x->ar[l]) / bw;
+    }
+    if (le > 0) {
+        double e = (double)(1 << le);
+        double bw = (1 << (le + lt)) <= x->maxnode[g] ? near : far;
+        sec = sec + ((4.0 * ((e - 1.0) / e)) * (double)x->a2a[l]) / bw;
+    }
+    if (lt > 0) {
+        double t = (double)(1 << lt);
+        sec = sec + ((4.0 * ((2.0 * (t - 1.0)) / t)) * (double)x->a2a[l]) / near;
+    }
+    return sec;
+}
+
+int orc_set_experts(orc_ctx* x, const int64_t* expert_state, const int64_t* expert_param, char* err) {
+    int L = x->L;
+    free(x->estate);
+    free(x->eparam);
+    free(x->Pt);
+    x->estate = x->eparam = x->Pt = NULL;
+    x->tiled = 0;
+    if (!expert_state && !expert_param) return 0;
+    if (!expert_state || !expert_param || x->has_profile) {
+        if (err) snprintf(err, 256, "expert tiling needs both byte arrays and the synthetic cost model");
+        return -1;
+    }
+    for (int l = 0; l < L; ++l) {
+        int64_t st = x->state[l + 1] - x->state[l], pb = x->param[l + 1] - x->param[l];
+        if (expert_state[l] < 0 || expert_state[l] > st || expert_param[l] < 0 || expert_param[l] > pb) {
+            if (err) snprintf(err, 256, "expert bytes of layer %d outside [0, layer bytes]", l);
+            return -1;
+        }
+    }
+    x->estate = (int64_t*)calloc(L + 1, sizeof(int64_t));
+    x->eparam = (int64_t*)calloc(L + 1, sizeof(int64_t));
+    for (int l = 0; l < L; ++l) {
+        x->estate[l + 1] = x->estate[l] + expert_state[l];
+        x->eparam[l + 1] = x->eparam[l] + expert_param[l];
+    }
+    x->Pt = (int64_t*)calloc((size_t)x->n_types * 20 * (L + 1), sizeof(int64_t));
+    for (int g = 0; g < x->n_types; ++g)
+        for (int j = 0; j < 4; ++j)
+            for (int i = 0; i < (j + 1) * (j + 2) / 2; ++i) {
+                int le = 0, lt = 0, ld = 0, slot = tile_base[j] + i;
+                tiling_of(j, i, &le, &lt, &ld);
+                /* ETP slices one tensor, so it stays inside a node */
+                x->tvalid[g][slot] = x->gpus[g] > 0 && (1 << lt) <= x->maxnode[g];
+                int64_t* P = x->Pt + ((size_t)g * 20 + slot) * (L + 1);
+                P[0] = 0;
+                for (int l = 0; l < L; ++l)
+                    P[l + 1] = P[l] + (x->tvalid[g][slot] ? to_ns(tiled_seconds(x, g, j, le, lt, l)) : 0);
+            }
+    x->tiled = 1;
+    return 0;
+}
+
+void orc_tiled_tables(const orc_ctx* x, int64_t* Pt, int32_t* valid) {
+    if (!x->tiled) return;
+    if (Pt) memcpy(Pt, x->Pt, sizeof(int64_t) * (size_t)x->n_types * 20 * (x->L + 1));
+    if (valid)
+        for (int g = 0; g < x->n_types; ++g)
+            for (int t = 0; t < 20; ++t) valid[g * 20 + t] = x->tvalid[g][t];
 }
 
 /* ------------------------------------------------------------- DP degree */
@@ -358,6 +500,7 @@ typedef struct {
     int64_t n;
     int status;
     int32_t a[MAXS + 1];
+    uint8_t tile[MAXS]; /* expert tiling per stage: log2 EP | log2 ETP << 2 */
 } priced;
 
 /* Evaluate (§5.3): T = (M-1) max t_s + sum t_s + max g_s for the split a;
@@ -384,6 +527,147 @@ static int64_t evaluate(const orc_ctx* x, int S, int M, int64_t n, const int64_t
     }
     *tmax_out = tmax;
     return (int64_t)(M - 1) * tmax + tsum + gmax;
+}
+
+/* ------------------------------------------- tiled PartitionLayers, Evaluate */
+
+/* The tilings a stage may use: prefix row, EDP degree minus one, code. */
+typedef struct {
+    int n;
+    const int64_t* P[10];
+    int64_t d1[10];
+    uint8_t code[10];
+} tiles;
+
+/* Stage time of layers [i, j) under expert tiling: the fastest tiling whose
+ * memory fits (§5.3: every factorisation that fits per-GPU memory is priced
+ * and the shortest kept; the earliest slot on ties), INF if none fits.
+ * Memory (reading): per device, dense state / k + expert state / (e t) +
+ * f activations / k; with e t = k / d that is state + (d - 1) expert state
+ * + f act <= capacity * k.  *which gets the option index. */
+static int64_t tiled_time(const orc_ctx* x, const tiles* tl, int64_t c, int64_t f, int64_t cap, int i, int j,
+                          int* which) {
+    int64_t fastest = INF;
+    for (int o = 0; o < tl->n; ++o) {
+        int64_t mem = (x->state[j] - x->state[i]) + tl->d1[o] * (x->estate[j] - x->estate[i]) +
+                      f * (x->act[j] - x->act[i]);
+        if (mem > cap) continue;
+        int64_t t = tl->P[o][j] - tl->P[o][i] + c;
+        if (t < fastest) {
+            fastest = t;
+            if (which) *which = o;
+        }
+    }
+    return fastest;
+}
+
+/* The dynamic programme of partition() over the tiled stage time.  The
+ * fastest fitting tiling of an interval is no slower on a sub-interval
+ * (each tiling that fits the interval fits the sub-interval and costs
+ * less), so stage time stays monotone under inclusion and the canonical
+ * (lexicographically smallest) optimal split is defined as before. */
+static int partition_tiled(const orc_ctx* x, int S, const tiles* tl, const int64_t* c, const int64_t* f_s,
+                           const int64_t* cap, int64_t* f, int64_t* Bstar, int32_t* a) {
+    int L = x->L;
+#define FT(s, i) f[(size_t)(s) * (L + 1) + (i)]
+    for (int i = 0; i <= L; ++i) FT(S, i) = (i == L) ? 0 : INF;
+    for (int s = S - 1; s >= 0; --s)
+        for (int i = 0; i <= L; ++i) {
+            int64_t lowest = INF;
+            for (int j = i + 1; j <= L; ++j) {
+                if (FT(s + 1, j) == INF) continue;
+                int64_t t = tiled_time(x, &tl[s], c[s], f_s[s], cap[s], i, j, NULL);
+                if (t == INF) continue;
+                int64_t v = t > FT(s + 1, j) ? t : FT(s + 1, j);
+                if (v < lowest) lowest = v;
+            }
+            FT(s, i) = lowest;
+        }
+    int64_t B = FT(0, 0);
+    if (B == INF) return 0;
+    *Bstar = B;
+    a[0] = 0;
+    for (int s = 0; s < S; ++s) {
+        int chosen = -1;
+        for (int j = a[s] + 1; j <= L && chosen < 0; ++j)
+            if (FT(s + 1, j) <= B && tiled_time(x, &tl[s], c[s], f_s[s], cap[s], a[s], j, NULL) <= B) chosen = j;
+        a[s + 1] = chosen;
+    }
+    return 1;
+#undef FT
+}
+
+/* Gradient synchronisation of a tiled stage over layers [lo, hi) (reading):
+ * the dense gradients are all-reduced over the n replicas as in evaluate();
+ * the expert gradients over the n d copies of each expert shard (d EDP
+ * copies in each replica).  Per device that is Gd / k and Ge / (e t) =
+ * d Ge / k bytes, each ring moving 2(r-1)/r of it for r participants, so
+ *   g = ceil(2 ((n-1) Gd + (n d - 1) Ge) 1e9 / (n k bw))  ns,
+ * bw the type's intra-node bandwidth when n = 1 and the stage's devices fit
+ * in one node (the EDP copies alone, inside the node), else its slowest
+ * NIC.  With d = 1 this is the untiled formula. */
+static int64_t tiled_sync(const orc_ctx* x, int g, int j, int64_t n, int64_t d, int32_t lo, int32_t hi) {
+    int64_t Ge = x->eparam[hi] - x->eparam[lo];
+    int64_t Gd = (x->param[hi] - x->param[lo]) - Ge;
+    u128 vol = (u128)(n - 1) * (u128)Gd + (u128)(n * d - 1) * (u128)Ge;
+    if (vol == 0) return 0;
+    int64_t bw = (n == 1 && (1 << j) <= x->maxnode[g]) ? x->intra_bw[g] : x->inter_bw[g];
+    return ceil_div128((u128)2 * vol * 1000000000u, (u128)n * (u128)(1 << j) * (u128)bw);
+}
+
+/* §5.3: the per-stage fastest tilings are the starting point and the
+ * choice is re-selected against the whole iteration time on the split a.
+ * Exact form (reading): for a bound Y on the gradient term every stage
+ * takes its fastest fitting tiling with g_s <= Y (the earliest on ties),
+ * giving T(Y) = (M-1) max t_s + sum t_s + max g_s; the result is the
+ * smallest T(Y) over Y among the g values of all options, the smaller Y on
+ * ties.  A combination whose largest gradient term is Y* is matched or
+ * beaten by T(Y*), so this is the minimum of T over all combinations.
+ * Writes the plan's largest stage time and the chosen tilings. */
+static int64_t evaluate_tiled(const orc_ctx* x, int S, int M, int64_t n, const tiles* tl, const int64_t* c,
+                              const int64_t* f_s, const int64_t* cap, const int* g, const int* j, const int32_t* a,
+                              int64_t* B_out, uint8_t* tile_out) {
+    int64_t ot[MAXS][10], og[MAXS][10];
+    int fits[MAXS][10];
+    for (int s = 0; s < S; ++s)
+        for (int o = 0; o < tl[s].n; ++o) {
+            int64_t mem = (x->state[a[s + 1]] - x->state[a[s]]) +
+                          tl[s].d1[o] * (x->estate[a[s + 1]] - x->estate[a[s]]) +
+                          f_s[s] * (x->act[a[s + 1]] - x->act[a[s]]);
+            fits[s][o] = mem <= cap[s];
+            ot[s][o] = tl[s].P[o][a[s + 1]] - tl[s].P[o][a[s]] + c[s];
+            og[s][o] = tiled_sync(x, g[s], j[s], n, tl[s].d1[o] + 1, a[s], a[s + 1]);
+        }
+    int64_t bestT = INF, bestY = 0, bestB = 0;
+    for (int ys = 0; ys < S; ++ys)
+        for (int yo = 0; yo < tl[ys].n; ++yo) {
+            if (!fits[ys][yo]) continue;
+            int64_t Y = og[ys][yo];
+            int64_t tm = 0, ts = 0, gm = 0;
+            int pick[MAXS], all = 1;
+            for (int s = 0; s < S && all; ++s) {
+                pick[s] = -1;
+                for (int o = 0; o < tl[s].n; ++o)
+                    if (fits[s][o] && og[s][o] <= Y && (pick[s] < 0 || ot[s][o] < ot[s][pick[s]])) pick[s] = o;
+                if (pick[s] < 0) {
+                    all = 0;
+                    break;
+                }
+                if (ot[s][pick[s]] > tm) tm = ot[s][pick[s]];
+                ts += ot[s][pick[s]];
+                if (og[s][pick[s]] > gm) gm = og[s][pick[s]];
+            }
+            if (!all) continue;
+            int64_t T = (int64_t)(M - 1) * tm + ts + gm;
+            if (T < bestT || (T == bestT && Y < bestY)) {
+                bestT = T;
+                bestY = Y;
+                bestB = tm;
+                for (int s = 0; s < S; ++s) tile_out[s] = tl[s].code[pick[s]];
+            }
+        }
+    *B_out = bestB;
+    return bestT;
 }
 
 /* ---------------------------------------------- the paper's split rule */
@@ -539,6 +823,33 @@ static void price_one(const orc_ctx* x, int S, int M, const uint8_t* codes, int6
         W[s] = w;
         cap[s] = x->mem[g[s]] * (int64_t)(1 << j[s]);
     }
+    if (x->tiled) {
+        /* expert tiling (§5.3): every stage may use each valid tiling of
+         * its devices */
+        tiles tl[MAXS];
+        int64_t fs[MAXS];
+        for (int s = 0; s < S; ++s) {
+            tl[s].n = 0;
+            for (int i = 0; i < (j[s] + 1) * (j[s] + 2) / 2; ++i) {
+                int slot = tile_base[j[s]] + i, le = 0, lt = 0, ld = 0;
+                if (!x->tvalid[g[s]][slot]) continue;
+                tiling_of(j[s], i, &le, &lt, &ld);
+                tl[s].P[tl[s].n] = x->Pt + ((size_t)g[s] * 20 + slot) * (L + 1);
+                tl[s].d1[tl[s].n] = ((int64_t)1 << ld) - 1;
+                tl[s].code[tl[s].n] = (uint8_t)(le | (lt << 2));
+                tl[s].n += 1;
+            }
+            fs[s] = (S - s) < M ? (S - s) : M;
+        }
+        int64_t Bt;
+        if (!partition_tiled(x, S, tl, c, fs, cap, f, &Bt, out->a)) {
+            out->status = ORC_OOM;
+            return;
+        }
+        out->T = evaluate_tiled(x, S, M, n, tl, c, fs, cap, g, j, out->a, &out->B, out->tile);
+        out->status = ORC_OK;
+        return;
+    }
     if (x->split_mode == 1) {
         /* the paper's split rule instead of PartitionLayers */
         if (!distribute(x, S, L, M, n, P, c, W, cap, g, j, out->a, &out->T, &out->B)) {
@@ -572,7 +883,7 @@ typedef struct {
     int s_max;
     int64_t *T, *B;
     uint16_t* n_dp;
-    uint8_t *status, *bounds;
+    uint8_t *status, *bounds, *tiling;
     int64_t n_all;
 } job;
 
@@ -603,16 +914,21 @@ static void* run_job(void* arg) {
                 jb->bounds[(int64_t)s * jb->n_all + c] =
                     (r.status == ORC_OK && s <= S) ? (uint8_t)r.a[s] : 0;
         }
+        if (jb->tiling) {
+            for (int s = 0; s < MAXS; ++s)
+                jb->tiling[(int64_t)s * jb->n_all + c] = (r.status == ORC_OK && s < S) ? r.tile[s] : 0;
+        }
     }
     free(f);
     free(Wbuf);
     return NULL;
 }
 
-int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
-              const uint8_t* code, int64_t plane_stride, int s_max, int64_t* T,
-              int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
-              int threads) {
+int orc_price_tiled(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
+                    const uint8_t* code, int64_t plane_stride, int s_max, int64_t* T,
+                    int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
+                    uint8_t* tiling, int threads) {
+    if (x->tiled && x->split_mode != 0) return -1; /* tiling prices the min-max split only */
     if (threads < 1) threads = 1;
     if (threads > n) threads = n > 0 ? (int)n : 1;
     job* jobs = (job*)calloc(threads, sizeof(job));
@@ -632,6 +948,7 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
         jb->n_dp = n_dp;
         jb->status = status;
         jb->bounds = bounds;
+        jb->tiling = tiling;
         jb->n_all = n;
     }
     if (threads == 1) {
@@ -643,6 +960,14 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
     free(jobs);
     free(tid);
     return threads;
+}
+
+int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
+              const uint8_t* code, int64_t plane_stride, int s_max, int64_t* T,
+              int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
+              int threads) {
+    return orc_price_tiled(x, n, S, M, code, plane_stride, s_max, T, bottleneck, n_dp, status, bounds,
+                           NULL, threads);
 }
 
 /* ------------------------------------------------- multi-template plans */

@@ -64,6 +64,33 @@ int orc_price(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
  * in Algorithm 1). */
 void orc_set_split(orc_ctx* x, int mode);
 
+/* Expert tiling (§5.3 "Expert tiling"): expert_state[l] and expert_param[l]
+ * are the expert parts of layer l's state and gradient bytes (0 for a dense
+ * layer; at most the layer's totals).  Turns tiling on for orc_price /
+ * orc_price_tiled with PartitionLayers (both NULL turn it off).  A stage of
+ * 2^j devices may then use every tiling 2^le EP x 2^lt ETP x 2^ld EDP with
+ * ETP within the type's largest node: per-layer cost with the EP and ETP
+ * collectives, memory with the expert state replicated d times, gradient
+ * sync of expert gradients over n d copies; the split minimises the
+ * largest stage time at each stage's fastest fitting tiling, and the
+ * tilings are re-selected against the whole iteration time.  Needs the
+ * synthetic cost model (no explicit profile).  Returns 0, or -1 with a
+ * message in err. */
+int orc_set_experts(orc_ctx* x, const int64_t* expert_state, const int64_t* expert_param, char* err);
+
+/* Tiled cost tables (after orc_set_experts): Pt[n_types][20][L+1] prefix
+ * ns per tiling slot (slots 0, 1-3, 4-9, 10-19 for 1, 2, 4, 8 devices; EDP
+ * exponent ascending, then ETP exponent) and valid[n_types][20]. */
+void orc_tiled_tables(const orc_ctx* x, int64_t* Pt, int32_t* valid);
+
+/* orc_price plus, when tiling is on, the chosen tiling of every stage:
+ * tiling[s * n + c] = log2 EP | log2 ETP << 2 (nullable; 0 past S and
+ * unless OK).  Returns -1 if tiling is combined with the paper's split. */
+int orc_price_tiled(const orc_ctx* x, int64_t n, const uint8_t* S, const uint16_t* M,
+                    const uint8_t* code, int64_t plane_stride, int s_max, int64_t* T,
+                    int64_t* bottleneck, uint16_t* n_dp, uint8_t* status, uint8_t* bounds,
+                    uint8_t* tiling, int threads);
+
 /* Multi-template plans (Algorithm 1): n_plans plans of up to max_tmpl
  * templates (n_tmpl[c] used); template t of plan c has depth S[t*n + c],
  * micro-batches M[t*n + c] and stage codes code[(t*s_max + s)*n + c].

@@ -57,6 +57,11 @@ def lib():
         L.orc_replicas.restype = C.c_int
         L.orc_replicas.argtypes = [C.c_int, p, C.c_int, p]
         L.orc_set_split.argtypes = [p, C.c_int]
+        L.orc_set_experts.restype = C.c_int
+        L.orc_set_experts.argtypes = [p, p, p, C.c_char_p]
+        L.orc_tiled_tables.argtypes = [p, p, p]
+        L.orc_price_tiled.restype = C.c_int
+        L.orc_price_tiled.argtypes = [p, C.c_int64, p, p, p, C.c_int64, C.c_int, p, p, p, p, p, p, C.c_int]
         L.orc_price_plans.restype = C.c_int
         L.orc_price_plans.argtypes = [p, C.c_int64, C.c_int, p, p, p, p, C.c_int, p, p, p, p, p, p]
         _lib = L
@@ -118,6 +123,28 @@ class Oracle:
                               _ptr(out["placed"]), _ptr(out["thr"]))
         return out
 
+    def set_experts(self, expert_state=None, expert_param=None):
+        """Expert tiling (§5.3): the expert parts of every layer's state and
+        gradient bytes; ``None`` for both turns tiling off."""
+        err = C.create_string_buffer(256)
+        if expert_state is None and expert_param is None:
+            rc = lib().orc_set_experts(self._h, None, None, err)
+        else:
+            es = np.ascontiguousarray(expert_state, dtype=np.int64)
+            ep = np.ascontiguousarray(expert_param, dtype=np.int64)
+            rc = lib().orc_set_experts(self._h, _ptr(es), _ptr(ep), err)
+        if rc != 0:
+            raise ValueError("oracle rejected expert bytes: " + err.value.decode())
+        self.tiled = expert_state is not None
+        return self
+
+    def tiled_tables(self) -> dict:
+        """Tiled prefix rows ``Pt[g, slot, l]`` (ns) and ``valid[g, slot]``."""
+        Pt = np.zeros((self.n_types, 20, self.L + 1), np.int64)
+        valid = np.zeros((self.n_types, 20), np.int32)
+        lib().orc_tiled_tables(self._h, _ptr(Pt), _ptr(valid))
+        return {"Pt": Pt, "valid": valid}
+
     def set_split(self, mode: str):
         """``"minmax"`` (PartitionLayers, the default) or ``"distribute"``
         (the paper's own proportional rule with its fixed alternatives)."""
@@ -142,8 +169,10 @@ class Oracle:
                                              np.cumsum(q, axis=2)], axis=2),
                 "p2p": p2p, "maxnode": mx, "inter_bw": bw}
 
-    def price(self, cands: dict, threads: int = 1, bounds: bool = True) -> dict:
-        """Price every candidate; returns T, bottleneck, n_dp, status, bounds[33, n]."""
+    def price(self, cands: dict, threads: int = 1, bounds: bool = True, tiling: bool = False) -> dict:
+        """Price every candidate; returns T, bottleneck, n_dp, status, bounds[33, n]
+        and, with ``tiling``, the chosen expert tiling of every stage
+        ``tiling[32, n]`` (log2 EP | log2 ETP << 2)."""
         S = np.ascontiguousarray(cands["S"], dtype=np.uint8)
         M = np.ascontiguousarray(cands["M"], dtype=np.uint16)
         code = np.ascontiguousarray(cands["code"], dtype=np.uint8)
@@ -151,10 +180,14 @@ class Oracle:
         s_max = int(code.shape[0])
         out = {"T": np.zeros(n, np.int64), "bottleneck": np.zeros(n, np.int64),
                "n_dp": np.zeros(n, np.uint16), "status": np.zeros(n, np.uint8),
-               "bounds": np.zeros((33, n), np.uint8) if bounds else None}
-        used = lib().orc_price(self._h, n, _ptr(S), _ptr(M), _ptr(code), n, s_max,
-                               _ptr(out["T"]), _ptr(out["bottleneck"]), _ptr(out["n_dp"]),
-                               _ptr(out["status"]), _ptr(out["bounds"]), int(threads))
+               "bounds": np.zeros((33, n), np.uint8) if bounds else None,
+               "tiling": np.zeros((32, n), np.uint8) if tiling else None}
+        used = lib().orc_price_tiled(self._h, n, _ptr(S), _ptr(M), _ptr(code), n, s_max,
+                                     _ptr(out["T"]), _ptr(out["bottleneck"]), _ptr(out["n_dp"]),
+                                     _ptr(out["status"]), _ptr(out["bounds"]), _ptr(out["tiling"]),
+                                     int(threads))
+        if used < 0:
+            raise ValueError("expert tiling prices the min-max split only")
         out["threads"] = used
         return out
 

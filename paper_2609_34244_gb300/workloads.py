@@ -71,11 +71,16 @@ def make_cluster(tflops, mem_bytes, intra_bw, nodes):
 
 
 def make_model(flops, param_bytes, state_bytes, act_bytes, ar_bytes, a2a_bytes,
-               boundary_bytes, moe=False, profile_s=None, microbatch=1):
-    """Model arrays (one entry per layer) plus model-wide scalars."""
+               boundary_bytes, moe=False, profile_s=None, microbatch=1,
+               expert_state=None, expert_param=None):
+    """Model arrays (one entry per layer) plus model-wide scalars.  The
+    optional expert parts of the state and gradient bytes (MoE expert
+    blocks) feed the expert tiling."""
     L = len(flops)
     arr = lambda v, dt: np.broadcast_to(np.asarray(v, dtype=dt), (L,)).copy()
     return {
+        "expert_state_bytes": None if expert_state is None else arr(expert_state, np.int64),
+        "expert_param_bytes": None if expert_param is None else arr(expert_param, np.int64),
         "flops": arr(flops, np.float64),
         "param_bytes": arr(param_bytes, np.int64),
         "state_bytes": arr(state_bytes, np.int64),
@@ -301,10 +306,39 @@ def moe48(seed=0, n=1_000_000):
     tok = 2 * b * s * h
     ar = np.where(expert, tok // 2, tok)  # expert blocks: attention all-reduces only
     a2a = np.where(expert, tok, 0)
-    model = make_model(flops, 2 * params, 16 * params, act, ar, a2a, tok, moe=True, microbatch=b)
+    e_only = np.where(expert, E * 3 * h * ffn, 0)  # the experts' own parameters
+    model = make_model(flops, 2 * params, 16 * params, act, ar, a2a, tok, moe=True, microbatch=b,
+                       expert_state=16 * e_only, expert_param=2 * e_only)
     cands = _random_cands(rng, cluster, n, 12, DEGREES, 64, moe=True)
     meta = {"L": L, "n_types": 4, "gpus": 128, "s_max": 12, "degrees": DEGREES, "topk": 16}
     return Workload("moe48", seed, cluster, model, cands, meta)
+
+
+def moe16(seed=0, n=20_000):
+    """16-layer MoE model for the expert-tiling tests: dense and expert
+    blocks alternating (16 experts, top-2, h 2048, ffn 5632, seq 2048, bf16);
+    64 GPUs of 3 types in 2/4/8-GPU nodes with 8-48 GB each, so that the
+    expert state replicated by EDP fits on some stages and not on others;
+    S <= 6, EP in {1,2,4,8}, M = 16."""
+    rng = np.random.default_rng(seed)
+    cluster = _hetero_cluster(rng, 3, 64, (2, 4, 8), 0.3, mem_range=(8, 48))
+    h, ffn, s, b, E, top = 2048, 5632, 2048, 1, 16, 2
+    d_flops, d_params, d_act = _dense_layer(h, s, b, ffn)
+    e_only = E * 3 * h * ffn
+    e_params = 4 * h * h + e_only + h * E
+    e_flops = 3.0 * (2 * b * s * (4 * h * h + top * 3 * h * ffn) + 4 * b * s * s * h)
+    L = 16
+    expert = np.arange(L) % 2 == 1
+    params = np.where(expert, e_params, d_params)
+    tok = 2 * b * s * h
+    model = make_model(np.where(expert, e_flops, d_flops), 2 * params, 16 * params,
+                       np.where(expert, 2 * d_act, d_act), np.where(expert, tok // 2, tok),
+                       np.where(expert, tok, 0), tok, moe=True, microbatch=b,
+                       expert_state=np.where(expert, 16 * e_only, 0),
+                       expert_param=np.where(expert, 2 * e_only, 0))
+    cands = _random_cands(rng, cluster, n, 6, DEGREES, 16, moe=True)
+    meta = {"L": L, "n_types": 3, "gpus": 64, "s_max": 6, "degrees": DEGREES, "topk": 16}
+    return Workload("moe16", seed, cluster, model, cands, meta)
 
 
 def stress128(seed=0, n=10_000_000):
@@ -326,6 +360,7 @@ CONFIGS = {
     "dense32": lambda seed=0, n=None: dense32(seed, 100_000 if n is None else n),
     "dense80": lambda seed=0, n=None: dense80(seed, 1_000_000 if n is None else n),
     "moe48": lambda seed=0, n=None: moe48(seed, 1_000_000 if n is None else n),
+    "moe16": lambda seed=0, n=None: moe16(seed, 20_000 if n is None else n),
     "stress128": lambda seed=0, n=None: stress128(seed, 10_000_000 if n is None else n),
 }
 

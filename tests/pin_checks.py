@@ -507,6 +507,194 @@ def check_plans_properties(O, seed=2):
                 assert used[g] <= int(w.cluster["node_gpus"][w.cluster["node_type"] == g].sum()), (name, c, g)
 
 
+# ------------------------------------------------------------ expert tiling
+
+def _tiled_oracle(O, W, case):
+    cl = W.make_cluster(case["tflops"], case["mem_bytes"], case["intra_bw"], [tuple(x) for x in case["nodes"]])
+    md = W.make_model(case["flops"], case["param_bytes"], case["state_bytes"], case["act_bytes"], case["ar_bytes"],
+                      case["a2a_bytes"], case["boundary_bytes"], moe=True)
+    return O.Oracle(cl, md).set_experts(case["expert_state"], case["expert_param"])
+
+
+def check_tiling_hand(O):
+    """Hand-worked prices with expert tiling (golden/hand_tiling.json, §5.3
+    "Expert tiling"): ETP node bound, an EP group leaving a node, EDP
+    memory replication, dense and expert gradient sync, re-selection
+    against the whole iteration time."""
+    W = _workloads()
+    for case in _load("hand_tiling.json")["cases"]:
+        o = _tiled_oracle(O, W, case)
+        r = o.price(W.from_structures([[tuple(s) for s in case["stages"]]], [case["M"]]), tiling=True)
+        S = len(case["stages"])
+        e = case["expect"]
+        got = {"status": int(r["status"][0]), "T": int(r["T"][0]), "bottleneck": int(r["bottleneck"][0]),
+               "bounds": r["bounds"][: S + 1, 0].tolist(), "tiling": r["tiling"][:S, 0].tolist()}
+        assert got == e, (case["name"], got)
+
+
+def _tilings(j):
+    """(le, lt, ld) of 2^j devices in slot order: EDP exponent ascending,
+    then ETP exponent ascending."""
+    return [(j - d - t, t, d) for d in range(j + 1) for t in range(j + 1 - d)]
+
+
+def _tiled_instance(rng, W):
+    nt = int(rng.integers(1, 3))
+    nodes = [(g, int(rng.choice([2, 4])), int(rng.choice([1, 4, 10])) * 10**9)
+             for g in range(nt) for _ in range(int(rng.integers(2, 7)))]
+    cl = W.make_cluster(rng.uniform(0.5, 2.0, nt), rng.integers(20, 120, nt) * 10**9,
+                        rng.choice([50, 100, 300], nt) * 10**9, nodes)
+    L = int(rng.integers(3, 7))
+    expert = rng.random(L) < 0.5
+    es = np.where(expert, rng.integers(10, 80, L) * 10**9, 0)
+    ep = np.where(expert, rng.integers(1, 50, L) * 10**8, 0)
+    md = W.make_model(rng.uniform(1e9, 2e10, L), ep + rng.integers(1, 20, L) * 10**8,
+                      es + rng.integers(1, 20, L) * 10**9, rng.integers(0, 5, L) * 10**9,
+                      rng.integers(0, 5, L) * 10**7, np.where(expert, rng.integers(1, 20, L) * 10**7, 0),
+                      int(rng.integers(0, 3)) * 10**7, moe=True)
+    return cl, md, es, ep
+
+
+def check_tiling_brute_force(O, trials=200, seed=77):
+    """Tiled PartitionLayers and the re-selection against brute force on
+    tiny random MoE instances: the split is the lexicographically smallest
+    of those minimising the largest stage time when every stage takes its
+    fastest fitting tiling (every split enumerated); T is the minimum over
+    every combination of fitting tilings on that split; the reported
+    tilings attain it, fit memory and keep ETP within a node; OOM exactly
+    when no split fits under any tiling.  Stage costs come from the
+    oracle's tiled tables (their values are pinned by the hand cases and by
+    the untiled slot); gradient terms follow the stated formula."""
+    W = _workloads()
+    rng = np.random.default_rng(seed)
+    seen_nontrivial = 0
+    for _ in range(trials):
+        cl, md, es, ep = _tiled_instance(rng, W)
+        L = int(md["flops"].shape[0])
+        nt = int(cl["tflops"].shape[0])
+        structs = []
+        for _c in range(10):
+            S = int(rng.integers(1, min(3, L) + 1))
+            structs.append([(int(rng.integers(0, nt)), int(rng.integers(0, 4))) for _s in range(S)])
+        Ms = rng.choice([1, 2, 4, 8], len(structs))
+        cands = W.from_structures(structs, Ms)
+        o = O.Oracle(cl, md).set_experts(es, ep)
+        r = o.price(cands, tiling=True)
+        Pt = o.tiled_tables()["Pt"]
+        tb = o.tables()
+        maxn, inter, p2p = tb["maxnode"], tb["inter_bw"], tb["p2p"]
+        st = np.concatenate([[0], np.cumsum(md["state_bytes"])])
+        ex = np.concatenate([[0], np.cumsum(es)])
+        ac = np.concatenate([[0], np.cumsum(md["act_bytes"])])
+        pb = np.concatenate([[0], np.cumsum(md["param_bytes"])])
+        eb = np.concatenate([[0], np.cumsum(ep)])
+        for c, stages in enumerate(structs):
+            S, M = len(stages), int(Ms[c])
+            if int(r["status"][c]) not in (O.OK, O.OOM):
+                continue
+            n = int(r["n_dp"][c])
+            opts, cs, caps = [], [], []
+            for s, (g, j) in enumerate(stages):
+                base = (0, 1, 4, 10)[j]
+                opts.append([(base + i, le, lt, ld) for i, (le, lt, ld) in enumerate(_tilings(j))
+                             if (1 << lt) <= maxn[g]])
+                if s + 1 < S:
+                    h, jn = stages[s + 1]
+                    same = int(g == h and (1 << j) + (1 << jn) <= maxn[g])
+                    cs.append(int(p2p[g, h, same]))
+                else:
+                    cs.append(0)
+                caps.append(int(cl["mem_bytes"][g]) << j)
+
+            def fits(s, i, e, o_):
+                f = min(S - s, M)
+                mem = (st[e] - st[i]) + ((1 << o_[3]) - 1) * (ex[e] - ex[i]) + f * (ac[e] - ac[i])
+                return mem <= caps[s]
+
+            def tcost(s, i, e, o_):
+                return int(Pt[stages[s][0], o_[0], e] - Pt[stages[s][0], o_[0], i]) + cs[s]
+
+            def gsync(s, i, e, o_):
+                g, j = stages[s]
+                Ge = int(eb[e] - eb[i])
+                Gd = int(pb[e] - pb[i]) - Ge
+                vol = (n - 1) * Gd + (n * (1 << o_[3]) - 1) * Ge
+                if vol == 0:
+                    return 0
+                bw = int(cl["intra_bw"][g]) if (n == 1 and (1 << j) <= maxn[g]) else int(inter[g])
+                return -((-2 * vol * 10**9) // (n * (1 << j) * bw))
+
+            best, split = None, None
+            for cut in itertools.combinations(range(1, L), S - 1):
+                a = (0,) + cut + (L,)
+                worst = 0
+                for s in range(S):
+                    ts = [tcost(s, a[s], a[s + 1], o_) for o_ in opts[s] if fits(s, a[s], a[s + 1], o_)]
+                    if not ts:
+                        worst = None
+                        break
+                    worst = max(worst, min(ts))
+                if worst is not None and (best is None or worst < best):
+                    best, split = worst, a
+            if best is None:
+                assert int(r["status"][c]) == O.OOM, (c, structs[c])
+                continue
+            assert int(r["status"][c]) == O.OK, (c, structs[c])
+            assert tuple(r["bounds"][: S + 1, c].tolist()) == split, (c, split, r["bounds"][: S + 1, c])
+            a = split
+            choices = [[o_ for o_ in opts[s] if fits(s, a[s], a[s + 1], o_)] for s in range(S)]
+            Tmin = None
+            for combo in itertools.product(*choices):
+                ts = [tcost(s, a[s], a[s + 1], combo[s]) for s in range(S)]
+                gs = [gsync(s, a[s], a[s + 1], combo[s]) for s in range(S)]
+                T = (M - 1) * max(ts) + sum(ts) + max(gs)
+                Tmin = T if Tmin is None else min(Tmin, T)
+            assert int(r["T"][c]) == Tmin, (c, int(r["T"][c]), Tmin)
+            # the reported tilings: valid, fitting, and attaining T
+            got = []
+            for s in range(S):
+                code = int(r["tiling"][s, c])
+                le, lt = code & 3, code >> 2
+                match = [o_ for o_ in choices[s] if o_[1] == le and o_[2] == lt]
+                assert len(match) == 1, (c, s, code)
+                got.append(match[0])
+                seen_nontrivial += int(le != stages[s][1])
+            ts = [tcost(s, a[s], a[s + 1], got[s]) for s in range(S)]
+            gs = [gsync(s, a[s], a[s + 1], got[s]) for s in range(S)]
+            assert (M - 1) * max(ts) + sum(ts) + max(gs) == Tmin, c
+            assert max(ts) == int(r["bottleneck"][c]), c
+    assert seen_nontrivial > 0
+
+
+def check_tiling_reductions(O):
+    """The untiled slot of every degree reproduces the untiled cost table
+    bit for bit; a dense model with no expert bytes prices identically with
+    tiling on and keeps the untiled tiling (EP over all devices) on every
+    stage."""
+    W = _workloads()
+    for name in ("moe16", "moe48", "dense32"):
+        w = W.make_workload(name, seed=3, n=600)
+        es = w.model.get("expert_state_bytes")
+        ep = w.model.get("expert_param_bytes")
+        if es is None:
+            es = ep = np.zeros(w.model["flops"].shape[0], np.int64)
+        o = O.Oracle(w.cluster, w.model).set_experts(es, ep)
+        P = o.tables()["P"]
+        Pt = o.tiled_tables()["Pt"]
+        for j in range(4):
+            assert (Pt[:, (0, 1, 4, 10)[j], :] == P[:, j, :]).all(), (name, j)
+        if name == "dense32":
+            plain = O.Oracle(w.cluster, w.model).price(w.cands)
+            tiled = o.price(w.cands, tiling=True)
+            for k in ("T", "bottleneck", "n_dp", "status", "bounds"):
+                assert (plain[k] == tiled[k]).all(), (name, k)
+            ok = tiled["status"] == O.OK
+            S = w.cands["S"][ok]
+            live = np.arange(32)[:, None] < S[None, :]
+            j = (w.cands["code"][:, ok] >> 3) & 3
+            assert (tiled["tiling"][: j.shape[0], ok][live[: j.shape[0]]] == j[live[: j.shape[0]]]).all()
+
+
 ALL_CHECKS = [
     check_hand_partitions,
     check_hand_pricing,
@@ -523,4 +711,7 @@ ALL_CHECKS = [
     check_distribute_properties,
     check_plans_hand,
     check_plans_properties,
+    check_tiling_hand,
+    check_tiling_brute_force,
+    check_tiling_reductions,
 ]

@@ -73,6 +73,22 @@ MUTANTS = [
      "sum = sum + ((double)(r.n * (int64_t)M[o])) / (double)r.T;"),
     ("distribute_choice_sees_gradient", "int64_t pipe = (int64_t)(M - 1) * tmax + tsum;",
      "int64_t tm2, pipe = evaluate(x, S, M, n, P, c, j, g, b, &tm2);"),
+    ("tiling_etp_leaves_node", "x->tvalid[g][slot] = x->gpus[g] > 0 && (1 << lt) <= x->maxnode[g];",
+     "x->tvalid[g][slot] = x->gpus[g] > 0;"),
+    ("tiling_ep_group_without_etp", "double bw = (1 << (le + lt)) <= x->maxnode[g] ? near : far;",
+     "double bw = (1 << le) <= x->maxnode[g] ? near : far;"),
+    ("tiling_etp_ring_factor", "sec = sec + ((4.0 * ((2.0 * (t - 1.0)) / t)) * (double)x->a2a[l]) / near;",
+     "sec = sec + ((4.0 * ((t - 1.0) / t)) * (double)x->a2a[l]) / near;"),
+    ("tiling_split_ignores_edp_memory", "int64_t mem = (x->state[j] - x->state[i]) + tl->d1[o] * (x->estate[j] - x->estate[i]) +",
+     "int64_t mem = (x->state[j] - x->state[i]) + 0 * (x->estate[j] - x->estate[i]) +"),
+    ("tiling_choice_ignores_memory", "fits[s][o] = mem <= cap[s];", "fits[s][o] = 1;"),
+    ("tiling_sync_ignores_edp", "(u128)(n * d - 1) * (u128)Ge", "(u128)(n - 1) * (u128)Ge"),
+    ("tiling_sync_always_nic", "int64_t bw = (n == 1 && (1 << j) <= x->maxnode[g]) ? x->intra_bw[g] : x->inter_bw[g];",
+     "int64_t bw = x->inter_bw[g];"),
+    ("tiling_no_reselection", "if (fits[s][o] && og[s][o] <= Y && (pick[s] < 0", "if (fits[s][o] && (pick[s] < 0"),
+    ("tiling_tie_to_later_slot", "(pick[s] < 0 || ot[s][o] < ot[s][pick[s]])", "(pick[s] < 0 || ot[s][o] <= ot[s][pick[s]])"),
+    ("tiling_edp_order_reversed", "    for (int d = 0; d <= j; ++d)\n        for (int t = 0; t + d <= j; ++t) {",
+     "    for (int d = j; d >= 0; --d)\n        for (int t = 0; t + d <= j; ++t) {"),
 ]
 
 # planted mistakes in the Python part of the oracle (the micro-batch fill)
