@@ -193,6 +193,8 @@ def main():
     ap.add_argument("--mbs-levels", type=int, default=4, help="micro-batch sizes of the fill figure (0: skip)")
     ap.add_argument("--no-distribute", action="store_true", help="skip the paper's-split comparison figure")
     ap.add_argument("--plans", type=int, default=1_000_000, help="multi-template plans of the plan figure (0: skip)")
+    ap.add_argument("--tiling", type=int, default=1_000_000,
+                    help="moe48 candidates of the expert-tiling figure (0: skip)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -398,6 +400,64 @@ def main():
                      "best_plan_throughput": float(pr["thr"].max())}
         del dp, pr
 
+    # expert tiling (§5.3) on the MoE workload: the same candidates priced
+    # untiled and with every stage's EP x ETP x EDP choice, device-resident
+    tiling_fig = None
+    if args.tiling > 0:
+        nt_ = args.tiling
+        wt = W.make_workload("moe48", seed=rank, n=nt_)
+        ctx2 = h.heddle_create(0)
+        try:
+            h.heddle_load_cluster(ctx2, wt.cluster)
+            h.heddle_load_model(ctx2, wt.model)
+            dct = h.cands_to_device(wt.cands)
+            r_plain, r_tiled = h.alloc_results(nt_), h.alloc_results(nt_)
+            til = torch.empty((32, nt_), dtype=torch.uint8, device="cuda")
+
+            def timed(fn, reps=3):
+                fn()
+                torch.cuda.synchronize()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                for _ in range(reps):
+                    fn()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                return e0.elapsed_time(e1) / reps
+
+            plain_ms = timed(lambda: h.heddle_price_candidates(ctx2, h.make_candidates(dct),
+                                                               h.make_results(r_plain), stream))
+            h.heddle_load_experts(ctx2, wt.model["expert_state_bytes"], wt.model["expert_param_bytes"])
+            tiled_ms = timed(lambda: h.heddle_price_tiled(ctx2, h.make_candidates(dct), h.make_results(r_tiled),
+                                                          til, stream))
+            tiled_errors = h.heddle_device_errors(ctx2)
+            pT, tT = r_plain["T"].cpu().numpy(), r_tiled["T"].cpu().numpy()
+            pok, tok_ = r_plain["status"].cpu().numpy() == 0, r_tiled["status"].cpu().numpy() == 0
+            both = pok & tok_
+            codes = til.cpu().numpy()[:, tok_]
+            Sk = wt.cands["S"][tok_]
+            jk = (wt.cands["code"][:, tok_] >> 3) & 3
+            layouts = {}
+            for s_ in range(int(Sk.max()) if Sk.size else 0):
+                live = Sk > s_
+                le, lt = codes[s_, live] & 3, codes[s_, live] >> 2
+                ld = jk[s_, live] - le - lt
+                for a_, b_, c_ in zip(le, lt, ld):
+                    key = "%dx%dx%d" % (1 << a_, 1 << b_, 1 << c_)
+                    layouts[key] = layouts.get(key, 0) + 1
+            ratio = tT[both].astype(np.float64) / pT[both].astype(np.float64)
+            tiling_fig = {"value": nt_ / (tiled_ms / 1e3), "unit": UNIT, "workload": "moe48, %d candidates" % nt_,
+                          "ms_per_call": tiled_ms, "untiled_ms_per_call": plain_ms,
+                          "ok_untiled": int(pok.sum()), "ok_tiled": int(tok_.sum()),
+                          "mean_T_ratio_tiled_over_untiled": float(ratio.mean()) if ratio.size else None,
+                          "share_faster": float((ratio < 1).mean()) if ratio.size else None,
+                          "share_slower": float((ratio > 1).mean()) if ratio.size else None,
+                          "stage_layouts_EPxETPxEDP": dict(sorted(layouts.items(), key=lambda x: -x[1])),
+                          "device_errors": int(tiled_errors)}
+            del dct, r_plain, r_tiled, til
+        finally:
+            h.heddle_destroy(ctx2)
+
     # end to end through the public host-buffer call (pinned host memory)
     pinned = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
               for k, v in w.cands.items()}
@@ -466,6 +526,7 @@ def main():
         "distribute_split": distribute,
         "mbs_fill": mbs_fig,
         "plans": plans_fig,
+        "expert_tiling": tiling_fig,
         "topk_head": merged["idx"][:4].tolist() if merged["count"] else [],
         "e2e_topk_matches": e2e_topk["idx"].tolist() == local_topk["idx"].tolist(),
     }

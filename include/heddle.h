@@ -353,6 +353,51 @@ typedef struct {
 heddle_status heddle_price_plans(heddle_ctx* ctx, const heddle_plans* plans,
                                  const heddle_plan_results* results, void* stream);
 
+/* ------------------------------------------------------ expert tiling */
+
+/* §5.3 "Expert tiling": the 2^j devices of a stage factor into EP x ETP x
+ * EDP (2^le x 2^lt x 2^ld, le + lt + ld = j).  ETP slices one tensor, so it
+ * stays within the type's largest node; EP may leave a node; EDP is the
+ * rest.  heddle_load_experts(ctx, expert_state, expert_param, n_layers)
+ * gives, per layer of the loaded model, the experts' part of its state and
+ * gradient bytes (host arrays, copied; 0 for a dense layer, at most the
+ * layer's state_bytes / param_bytes) and turns tiling on for every later
+ * heddle_price_candidates, heddle_price_topk, heddle_price_topk_host and
+ * heddle_price_tiled call (both NULL turn it off; loading a model turns it
+ * off).  Synchronous; builds NT x 20 x (L+1) int64 tiled tables, which
+ * must fit 160 KB (E_LIMIT otherwise).  Needs the synthetic cost model
+ * (E_STATE with a profile).  Readings (the paper names each direction's
+ * collectives but prints no formula), per layer in seconds, IEEE double
+ * left to right, no fused multiply-add:
+ *   s = flops / (k * tflops * 1e12)
+ *   k > 1: s += (4 * 2(k-1)/k) * ar_bytes / bw_k     bw_k = intra if k <= largest node, else NIC
+ *   e > 1: s += (4 * (e-1)/e) * a2a_bytes / bw_et    ETP innermost: the EP group spans e*t devices
+ *   t > 1: s += (4 * 2(t-1)/t) * a2a_bytes / intra
+ * q = nearest ns; the tiling e = k, t = d = 1 is the untiled cost.  Memory
+ * with EDP d: state + (d-1) expert state + f act <= mem k.  Gradient sync
+ * of the stage: ceil(2((n-1) Gd + (n d - 1) Ge) 1e9 / (n k bw)) ns, Gd / Ge
+ * the dense / expert gradient bytes of its layers, bw = intra when n = 1
+ * and k <= largest node, else the slowest NIC.  PartitionLayers minimises
+ * the largest stage time with every stage on its fastest fitting tiling
+ * (the earliest slot on ties; slots order EDP exponent ascending, then ETP
+ * exponent); the tilings are then re-selected against the whole iteration
+ * time (M-1) max t + sum t + max g: for every bound Y among the gradient
+ * terms of the fitting tilings each stage takes its fastest fitting tiling
+ * with g <= Y, and the smallest T wins (the smaller Y on ties).
+ * `bottleneck` is then the plan's largest stage time under the chosen
+ * tilings.  Tiling prices the min-max split only: with search mode
+ * DISTRIBUTE pricing returns E_STATE, and so do heddle_price_mbs and
+ * heddle_price_plans while tiling is on.
+ *
+ * heddle_price_tiled prices like heddle_price_candidates and also writes
+ * the chosen tiling of every stage: tiling (device, nullable) [32][n]
+ * bytes, plane s at tiling[s * n + c] = log2 EP | log2 ETP << 2 (0 past S
+ * and unless OK).  E_STATE unless experts are loaded. */
+heddle_status heddle_load_experts(heddle_ctx* ctx, const int64_t* expert_state, const int64_t* expert_param,
+                                  int32_t n_layers);
+heddle_status heddle_price_tiled(heddle_ctx* ctx, const heddle_candidates* cands, const heddle_results* results,
+                                 uint8_t* tiling, void* stream);
+
 /* -------------------------------------------------------- host buffers */
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the
@@ -407,6 +452,7 @@ heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
 #define HEDDLE_SEARCH_GENERAL 1
 #define HEDDLE_SEARCH_EQUAL_LAYERS 2
 #define HEDDLE_SEARCH_DISTRIBUTE 3
+#define HEDDLE_SEARCH_TILED 4 /* reported by heddle_get_search while expert tiling is on */
 heddle_status heddle_set_search(heddle_ctx* ctx, int32_t mode);
 heddle_status heddle_get_search(heddle_ctx* ctx, int32_t* in_use);
 

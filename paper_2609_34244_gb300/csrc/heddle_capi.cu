@@ -9,7 +9,7 @@
 #include <algorithm>
 #include <vector>
 
-#include "heddle_internal.cuh"
+#include "heddle_tiled.cuh"
 
 using hd::Layout;
 
@@ -107,6 +107,12 @@ struct heddle_ctx {
     size_t node_cap = 0, node_cap2 = 0;
     uint8_t* plan_bounds[HEDDLE_MAX_TEMPLATES] = {nullptr, nullptr, nullptr, nullptr};
     size_t plan_bounds_cap[HEDDLE_MAX_TEMPLATES] = {0, 0, 0, 0};
+    // expert tiling: the experts' byte counts and the tiled image
+    bool have_experts = false, tiled_ready = false;
+    std::vector<int64_t> expert_state, expert_param;
+    hd::TiledLayout tlay{};
+    unsigned char* d_timg = nullptr;
+    size_t timg_cap = 0;
 };
 
 namespace {
@@ -274,8 +280,77 @@ heddle_status build_levels(heddle_ctx* x) {
     return ok(x);
 }
 
+// The tiled image (expert tiling) from the main image, the layers and the
+// experts' byte counts.
+heddle_status build_tiled(heddle_ctx* x) {
+    x->tiled_ready = false;
+    if (!x->have_experts || !x->tables_ready) return ok(x);
+    if (x->have_profile)
+        return fail(x, HEDDLE_E_STATE, "expert tiling needs the synthetic cost model (the model has a profile)");
+    const int NT = (int)x->types.size(), L = (int)x->layers.size();
+    const hd::TiledLayout tl = hd::make_tiled_layout(L, NT);
+    if (tl.bytes > hd::kTiledImageLimit)
+        return fail(x, HEDDLE_E_LIMIT, "tiled tables of %d types x %d layers take %u bytes (limit %u)", NT, L,
+                    tl.bytes, hd::kTiledImageLimit);
+    // gradient terms stay below 2^56 ns on the intra-node path as well
+    {
+        unsigned __int128 G = 0;
+        for (const auto& ly : x->layers) G += (unsigned __int128)ly.param_bytes;
+        for (int g = 0; g < NT; ++g) {
+            const unsigned __int128 t = (2 * G * 1000000000u + x->types[g].intra_bw - 1) /
+                                        (unsigned __int128)x->types[g].intra_bw;
+            if (t > ((unsigned __int128)1 << 56))
+                return fail(x, HEDDLE_E_LIMIT, "expert gradient synchronisation of type %d exceeds 2^56 ns", g);
+        }
+    }
+    CU(grow(&x->d_timg, &x->timg_cap, tl.bytes));
+    heddle_gpu_type* d_types = nullptr;
+    heddle_layer* d_layers = nullptr;
+    int64_t* d_ex = nullptr;
+    cudaError_t e = cudaMalloc(&d_types, sizeof(heddle_gpu_type) * NT);
+    if (e == cudaSuccess) e = cudaMalloc(&d_layers, sizeof(heddle_layer) * L);
+    if (e == cudaSuccess) e = cudaMalloc(&d_ex, sizeof(int64_t) * 2 * L);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_types, x->types.data(), sizeof(heddle_gpu_type) * NT, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_layers, x->layers.data(), sizeof(heddle_layer) * L, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_ex, x->expert_state.data(), sizeof(int64_t) * L, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+        e = cudaMemcpy(d_ex + L, x->expert_param.data(), sizeof(int64_t) * L, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemset(x->d_timg, 0, tl.bytes);
+    if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, sizeof(uint32_t));
+    if (e == cudaSuccess) {
+        hd::TiledTableArgs a{};
+        a.tl = tl;
+        a.lay = x->lay;
+        a.img = x->d_img;
+        a.types = d_types;
+        a.layers = d_layers;
+        a.expert_state = d_ex;
+        a.expert_param = d_ex + L;
+        a.timg = x->d_timg;
+        a.flags = x->d_flags;
+        e = hd::launch_tiled_tables(a, 0);
+    }
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    uint32_t flags = 0;
+    if (e == cudaSuccess) e = cudaMemcpy(&flags, x->d_flags, sizeof(uint32_t), cudaMemcpyDeviceToHost);
+    cudaFree(d_types);
+    cudaFree(d_layers);
+    cudaFree(d_ex);
+    if (e != cudaSuccess) return fail(x, HEDDLE_E_CUDA, "tiled table build: %s", cudaGetErrorString(e));
+    if (flags & hd::kTabBadValue)
+        return fail(x, HEDDLE_E_ARG, "a tiled per-layer cost is negative, not finite or above 4e18 ns");
+    if (flags & hd::kTabTooLarge) return fail(x, HEDDLE_E_LIMIT, "a tiled model time exceeds 2^40 ns");
+    x->tlay = tl;
+    x->tiled_ready = true;
+    return ok(x);
+}
+
 heddle_status build_tables(heddle_ctx* x) {
     x->tables_ready = false;
+    x->tiled_ready = false;
     x->mbs_ready = false;
     if (!x->have_cluster || !x->have_model) return ok(x);
     const int NT = (int)x->types.size(), L = (int)x->layers.size();
@@ -288,6 +363,7 @@ heddle_status build_tables(heddle_ctx* x) {
                                    x->model_flags);
     if (st != HEDDLE_OK) return st;
     x->tables_ready = true;
+    if (x->have_experts && (st = build_tiled(x)) != HEDDLE_OK) return st;
     if (x->mbs_levels > 0) return build_levels(x);
     return ok(x);
 }
@@ -416,6 +492,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->lv_n);
     cudaFree(x->lv_status);
     cudaFree(x->lv_bounds);
+    cudaFree(x->d_timg);
     cudaFree(x->d_node_type);
     cudaFree(x->d_node_gpus);
     for (auto* b : x->plan_bounds) cudaFree(b);
@@ -494,7 +571,45 @@ heddle_status heddle_load_model(heddle_ctx* x, const heddle_layer* layers, int32
         x->profile.clear();
     }
     x->have_model = true;
+    // the experts' byte counts describe the previous model's layers
+    x->have_experts = false;
+    x->expert_state.clear();
+    x->expert_param.clear();
     return build_tables(x);
+}
+
+heddle_status heddle_load_experts(heddle_ctx* x, const int64_t* expert_state, const int64_t* expert_param,
+                                  int32_t n_layers) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!expert_state && !expert_param) {
+        x->have_experts = x->tiled_ready = false;
+        x->expert_state.clear();
+        x->expert_param.clear();
+        return ok(x);
+    }
+    if (!expert_state || !expert_param) return fail(x, HEDDLE_E_ARG, "one of the expert arrays is NULL");
+    if (!x->have_model) return fail(x, HEDDLE_E_STATE, "no model loaded");
+    if (n_layers != (int32_t)x->layers.size())
+        return fail(x, HEDDLE_E_ARG, "n_layers %d differs from the model's %zu layers", n_layers, x->layers.size());
+    if (x->have_profile)
+        return fail(x, HEDDLE_E_STATE, "expert tiling needs the synthetic cost model (the model has a profile)");
+    for (int l = 0; l < n_layers; ++l) {
+        if (expert_state[l] < 0 || expert_state[l] > x->layers[l].state_bytes)
+            return fail(x, HEDDLE_E_ARG, "layer %d: expert_state outside [0, state_bytes]", l);
+        if (expert_param[l] < 0 || expert_param[l] > x->layers[l].param_bytes)
+            return fail(x, HEDDLE_E_ARG, "layer %d: expert_param outside [0, param_bytes]", l);
+    }
+    DeviceGuard dg(x->device);
+    x->expert_state.assign(expert_state, expert_state + n_layers);
+    x->expert_param.assign(expert_param, expert_param + n_layers);
+    x->have_experts = true;
+    const heddle_status st = build_tiled(x);
+    if (st != HEDDLE_OK) {
+        x->have_experts = false;
+        x->expert_state.clear();
+        x->expert_param.clear();
+    }
+    return st;
 }
 
 }  // extern "C"
@@ -534,7 +649,7 @@ heddle_status take_phase_rec(heddle_ctx* x, heddle_ctx::PhaseRec* rec) {
 // micro-batches (invalid where 2^shift does not divide M).
 heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
                          heddle_topk_state* state, void* stream, const heddle_ctx::Level* lvl = nullptr,
-                         int shift = 0) {
+                         int shift = 0, uint8_t* tiling = nullptr) {
     heddle_status st = check_cands(x, c, true);
     if (st != HEDDLE_OK) return st;
     if (!r) return fail(x, HEDDLE_E_ARG, "results is NULL");
@@ -542,7 +657,11 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     if (c->n == 0) return ok(x);
     if (!r->T || !r->bottleneck || !r->n_dp || !r->status)
         return fail(x, HEDDLE_E_ARG, "null result array");
+    const bool tiled = x->tiled_ready && !lvl;
+    if (tiled && x->search_mode == HEDDLE_SEARCH_DISTRIBUTE)
+        return fail(x, HEDDLE_E_STATE, "expert tiling prices the min-max split only (search mode DISTRIBUTE)");
     DeviceGuard dg(x->device);
+    if (tiled && tiling) CU(cudaMemsetAsync(tiling, 0, (size_t)HEDDLE_MAX_STAGES * c->n, (cudaStream_t)stream));
     hd::PriceArgs a{};
     a.lay = lvl ? lvl->lay : x->lay;
     a.img = lvl ? lvl->img : x->d_img;
@@ -563,7 +682,7 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     a.wl_code = x->d_wl_code;
     a.wl_bucket = x->d_wl_bucket;
     a.wl_cap = hd::kWorklistCap;
-    a.uniform = equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
+    a.uniform = !tiled && equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
     a.split_mode = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? 1 : 0;
     a.wl_T = x->d_wl_T;
     a.wl_nM = x->d_wl_nM;
@@ -587,8 +706,18 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
             CU(cudaEventRecord(rec.e[0], (cudaStream_t)stream));
         }
         int64_t* nl = x->time_phases ? x->phase_recs.back().launches : nullptr;
-        CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream, x->time_phases ? rec.e[1] : nullptr,
-                            nl));
+        if (tiled) {
+            hd::TiledArgs ta{};
+            ta.tl = x->tlay;
+            ta.timg = x->d_timg;
+            ta.tiling = tiling ? tiling + lo : nullptr;
+            ta.tstride = c->n;
+            CU(hd::launch_screen(a, x->num_sms, (cudaStream_t)stream, x->time_phases ? rec.e[1] : nullptr, nl));
+            if (nl) nl[1] += 1;
+            CU(hd::launch_tiled_search(a, ta, x->num_sms, (cudaStream_t)stream));
+        } else {
+            CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream, x->time_phases ? rec.e[1] : nullptr, nl));
+        }
         if (x->time_phases) CU(cudaEventRecord(rec.e[2], (cudaStream_t)stream));
         if (state) {
             // top-k over the searched candidates of this chunk only
@@ -615,6 +744,13 @@ heddle_status heddle_price_candidates(heddle_ctx* x, const heddle_candidates* c,
                                       const heddle_results* r, void* stream) {
     if (!x) return HEDDLE_E_ARG;
     return price_impl(x, c, r, nullptr, stream);
+}
+
+heddle_status heddle_price_tiled(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
+                                 uint8_t* tiling, void* stream) {
+    if (!x) return HEDDLE_E_ARG;
+    if (!x->tiled_ready) return fail(x, HEDDLE_E_STATE, "no experts loaded (heddle_load_experts)");
+    return price_impl(x, c, r, nullptr, stream, nullptr, 0, tiling);
 }
 
 heddle_status heddle_price_topk(heddle_ctx* x, const heddle_candidates* c, const heddle_results* r,
@@ -800,6 +936,7 @@ heddle_status heddle_get_search(heddle_ctx* x, int32_t* in_use) {
     heddle_status st = check_ready(x);
     if (st != HEDDLE_OK) return st;
     *in_use = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? HEDDLE_SEARCH_DISTRIBUTE
+              : x->tiled_ready                        ? HEDDLE_SEARCH_TILED
               : equal_layer_search(x)                 ? HEDDLE_SEARCH_EQUAL_LAYERS
                                                       : HEDDLE_SEARCH_GENERAL;
     return ok(x);
@@ -839,6 +976,7 @@ heddle_status heddle_price_mbs(heddle_ctx* x, const heddle_candidates* c, const 
     if (!r) return fail(x, HEDDLE_E_ARG, "results is NULL");
     if ((st = check_ready(x)) != HEDDLE_OK) return st;
     if (x->mbs_levels < 1 || !x->mbs_ready) return fail(x, HEDDLE_E_STATE, "no micro-batch sizes loaded");
+    if (x->tiled_ready) return fail(x, HEDDLE_E_STATE, "the micro-batch-size fill does not combine with expert tiling");
     if (c->n == 0) return ok(x);
     if (!r->T || !r->bottleneck || !r->n_dp || !r->status) return fail(x, HEDDLE_E_ARG, "null result array");
     DeviceGuard dg(x->device);
@@ -893,6 +1031,7 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     if (!pl || !pr) return fail(x, HEDDLE_E_ARG, "plans or results is NULL");
     heddle_status st = check_ready(x);
     if (st != HEDDLE_OK) return st;
+    if (x->tiled_ready) return fail(x, HEDDLE_E_STATE, "plan pricing does not combine with expert tiling");
     if (pl->n < 0) return fail(x, HEDDLE_E_ARG, "negative plan count");
     if (pl->n > hd::kWorklistCap) return fail(x, HEDDLE_E_LIMIT, "more than 2^20 plans in one call");
     if (pl->slots < 1 || pl->slots > HEDDLE_MAX_TEMPLATES)

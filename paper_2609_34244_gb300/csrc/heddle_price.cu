@@ -44,7 +44,7 @@
 
 #include <algorithm>
 
-#include "heddle_internal.cuh"
+#include "heddle_tiled.cuh"
 
 namespace hd {
 namespace {
@@ -732,7 +732,7 @@ cudaError_t launch_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
 
 }  // namespace
 
-cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid, int64_t* launches) {
+cudaError_t launch_screen(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid, int64_t* launches) {
     if (a.n <= 0) return cudaSuccess;
     if (a.n > a.wl_cap) return cudaErrorInvalidValue;
     cudaError_t e = cudaMemsetAsync(a.wl_count, 0, sizeof(int32_t) * kWlMeta, st);
@@ -751,6 +751,13 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (launches) launches[0] += 1;
     if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
+    return cudaSuccess;
+}
+
+cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid, int64_t* launches) {
+    if (a.n <= 0) return cudaSuccess;
+    cudaError_t e = launch_screen(a, num_sms, st, mid, launches);
+    if (e != cudaSuccess) return e;
     if (launches) launches[1] += 1;
     if (a.split_mode) return launch_distribute(a, num_sms, st);
     if (a.uniform) return launch_eq_search(a, num_sms, st);

@@ -21,6 +21,7 @@ BOUND_PLANES = MAX_STAGES + 1
 MODEL_MOE = 1
 CAND_OK, CAND_OOM, CAND_NO_FIT, CAND_INVALID = 0, 1, 2, 3
 STATUS_NAMES = {0: "OK", 1: "E_ARG", 2: "E_STATE", 3: "E_LIMIT", 4: "E_CUDA", 5: "E_NOMEM"}
+E_ARG, E_STATE, E_LIMIT, E_CUDA, E_NOMEM = 1, 2, 3, 4, 5
 
 
 class HeddleError(RuntimeError):
@@ -78,11 +79,12 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
            "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
            "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times",
-           "heddle_load_mbs", "heddle_price_mbs", "heddle_price_plans"]
+           "heddle_load_mbs", "heddle_price_mbs", "heddle_price_plans", "heddle_load_experts",
+           "heddle_price_tiled"]
 MAX_MBS_LEVELS = 4
 PHASES = ("screen", "search", "topk")
 TOPK_NOALLOC_MAX_N = 4194304
-SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS, SEARCH_DISTRIBUTE = 0, 1, 2, 3
+SEARCH_AUTO, SEARCH_GENERAL, SEARCH_EQUAL_LAYERS, SEARCH_DISTRIBUTE, SEARCH_TILED = 0, 1, 2, 3, 4
 
 _lib = None
 
@@ -118,6 +120,8 @@ def load_library(path: str = LIB_PATH):
         "heddle_load_mbs": (i32, [p, i32, p]),
         "heddle_price_plans": (i32, [p, p, p, p]),
         "heddle_price_mbs": (i32, [p, p, p, p, p]),
+        "heddle_load_experts": (i32, [p, p, p, i32]),
+        "heddle_price_tiled": (i32, [p, p, p, p, p]),
         "heddle_phase_times": (i32, [p, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
     }
     for name, (res, args) in sig.items():
@@ -245,6 +249,28 @@ def heddle_price_mbs(ctx, cands, results, mbs=None, stream=None):
     r = results if isinstance(results, heddle_results) else make_results(results)
     _check(ctx, load_library().heddle_price_mbs(ctx, C.byref(c), C.byref(r),
                                                 None if mbs is None else _ptr(mbs), _stream(stream)))
+
+
+def heddle_load_experts(ctx, expert_state=None, expert_param=None):
+    """Expert tiling (§5.3): the experts' part of every layer's state and
+    gradient bytes (host arrays); ``None`` for both turns tiling off."""
+    if expert_state is None and expert_param is None:
+        _check(ctx, load_library().heddle_load_experts(ctx, None, None, 0))
+        return
+    es = np.ascontiguousarray(expert_state, dtype=np.int64)
+    ep = np.ascontiguousarray(expert_param, dtype=np.int64)
+    if es.shape != ep.shape or es.ndim != 1:
+        raise ValueError("expert_state and expert_param must be 1-D arrays of one length")
+    _check(ctx, load_library().heddle_load_experts(ctx, es.ctypes.data, ep.ctypes.data, int(es.shape[0])))
+
+
+def heddle_price_tiled(ctx, cands, results, tiling=None, stream=None):
+    """Price device candidates with expert tiling; ``tiling`` (optional
+    device uint8 tensor [32, n]) receives each stage's log2 EP | log2 ETP << 2."""
+    c = cands if isinstance(cands, heddle_candidates) else make_candidates(cands)
+    r = results if isinstance(results, heddle_results) else make_results(results)
+    _check(ctx, load_library().heddle_price_tiled(ctx, C.byref(c), C.byref(r),
+                                                  None if tiling is None else _ptr(tiling), _stream(stream)))
 
 
 def plans_to_device(plans: dict, device="cuda") -> dict:

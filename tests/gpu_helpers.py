@@ -134,3 +134,47 @@ def take(cands, idx):
     """The candidates at indices ``idx`` (a host SoA copy)."""
     return {"S": cands["S"][idx].copy(), "M": cands["M"][idx].copy(),
             "code": np.ascontiguousarray(cands["code"][:, idx])}
+
+
+def price_tiled_gpu(h, w_cluster, w_model, cands, expert_state, expert_param, k=16, fused=False, batch=None):
+    """Expert tiling on the GPU through the C ABI: heddle_price_tiled (with
+    the tiling planes) and heddle_topk, or heddle_price_topk with ``fused``;
+    ``batch`` splits the candidates into consecutive calls."""
+    import torch
+    ctx = h.heddle_create(0)
+    try:
+        h.heddle_load_cluster(ctx, w_cluster)
+        h.heddle_load_model(ctx, w_model)
+        h.heddle_load_experts(ctx, expert_state, expert_param)
+        n = int(cands["S"].shape[0])
+        dc = h.cands_to_device(cands)
+        res = h.alloc_results(n, bounds=False)
+        state = h.alloc_topk_state()
+        h.heddle_topk_reset(ctx, state, k)
+        batch = n if batch is None else batch
+        out_bounds = np.zeros((33, n), np.uint8)
+        out_tiling = np.zeros((32, n), np.uint8)
+        for lo in range(0, n, max(batch, 1)):
+            hi = min(n, lo + batch)
+            bb = torch.empty((33, hi - lo), dtype=torch.uint8, device="cuda")
+            tt = torch.full((32, hi - lo), 0xEE, dtype=torch.uint8, device="cuda")
+            c = h.make_candidates(dc, lo, hi)
+            r = h.heddle_results(res["T"].data_ptr() + 8 * lo, res["bottleneck"].data_ptr() + 8 * lo,
+                                 res["n_dp"].data_ptr() + 2 * lo, res["status"].data_ptr() + lo, bb.data_ptr())
+            if fused:
+                h.heddle_price_topk(ctx, c, r, state)
+            else:
+                h.heddle_price_tiled(ctx, c, r, tt)
+                h.heddle_topk(ctx, c, r, state)
+            out_bounds[:, lo:hi] = bb.cpu().numpy()
+            out_tiling[:, lo:hi] = tt.cpu().numpy()
+        torch.cuda.synchronize()
+        out = h.results_to_numpy(res)
+        out["bounds"] = out_bounds
+        out["tiling"] = None if fused else out_tiling
+        out["topk"] = h.read_topk_state(state)
+        out["errors"] = h.heddle_device_errors(ctx)
+        out["search"] = h.heddle_get_search(ctx)
+        return out
+    finally:
+        h.heddle_destroy(ctx)
