@@ -105,6 +105,7 @@ struct heddle_ctx {
     int32_t* d_node_type = nullptr;
     int32_t* d_node_gpus = nullptr;
     size_t node_cap = 0, node_cap2 = 0;
+    bool nodes_on_device = false;  // d_node_* hold the loaded cluster's nodes
     uint8_t* plan_bounds[HEDDLE_MAX_TEMPLATES] = {nullptr, nullptr, nullptr, nullptr};
     size_t plan_bounds_cap[HEDDLE_MAX_TEMPLATES] = {0, 0, 0, 0};
     // expert tiling: the experts' byte counts and the tiled image
@@ -535,6 +536,7 @@ heddle_status heddle_load_cluster(heddle_ctx* x, const heddle_gpu_type* types, i
     DeviceGuard dg(x->device);
     x->types.assign(types, types + n_types);
     x->nodes.assign(nodes, nodes + n_nodes);
+    x->nodes_on_device = false;
     x->have_cluster = true;
     return build_tables(x);
 }
@@ -1051,9 +1053,12 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     DeviceGuard dg(x->device);
     cudaStream_t sm = (cudaStream_t)stream;
     const size_t nn = x->nodes.size();
-    CU(grow(&x->d_node_type, &x->node_cap, sizeof(int32_t) * nn));
-    CU(grow(&x->d_node_gpus, &x->node_cap2, sizeof(int32_t) * nn));
-    {
+    int32_t vmax = 1;
+    for (const auto& nd : x->nodes) vmax = std::max(vmax, nd.gpus);
+    if (!x->nodes_on_device) {
+        // once per loaded cluster (a synchronous copy)
+        CU(grow(&x->d_node_type, &x->node_cap, sizeof(int32_t) * nn));
+        CU(grow(&x->d_node_gpus, &x->node_cap2, sizeof(int32_t) * nn));
         std::vector<int32_t> ty(nn), gp(nn);
         for (size_t b = 0; b < nn; ++b) {
             ty[b] = x->nodes[b].type;
@@ -1061,6 +1066,7 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
         }
         CU(cudaMemcpy(x->d_node_type, ty.data(), sizeof(int32_t) * nn, cudaMemcpyHostToDevice));
         CU(cudaMemcpy(x->d_node_gpus, gp.data(), sizeof(int32_t) * nn, cudaMemcpyHostToDevice));
+        x->nodes_on_device = true;
     }
     hd::PlanArgs a{};
     a.lay = x->lay;
@@ -1071,6 +1077,7 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     a.node_type = x->d_node_type;
     a.node_gpus = x->d_node_gpus;
     a.n_nodes = (int32_t)nn;
+    a.vmax = vmax;
     a.placed = pr->placed;
     a.thr = pr->thr;
     a.err = x->d_flags + 1;

@@ -168,6 +168,7 @@ struct PlanArgs {
     const int32_t* node_type;
     const int32_t* node_gpus;
     int32_t n_nodes;
+    int32_t vmax;  // largest node (GPUs), <= kPlanMaxNode
     uint8_t* placed;
     double* thr;
     uint32_t* err;

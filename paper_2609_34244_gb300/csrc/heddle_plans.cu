@@ -14,7 +14,9 @@
 // groups are placed largest first on a node of its type whose free GPUs
 // equal the group size, else on the node with the fewest free GPUs above
 // it (§5.1).  Decisions depend on nodes only through their free counts, so
-// each thread keeps, per GPU type, a histogram of nodes by free GPUs.  The
+// each thread keeps, per GPU type, a histogram of nodes by free GPUs (in
+// shared memory, sized to the cluster's types and largest node, capacities
+// recomputed from it when a template's degree is needed).  The
 // first template that is not OK ends the plan; the plan's throughput is the
 // sum over placed templates of n M 1e9 / T, each term rounded in IEEE
 // double, in template order.
@@ -28,35 +30,48 @@ namespace {
 
 constexpr int kPlanBlock = 128;
 
+// Per-thread arrays in shared memory, interleaved by thread (element e of
+// thread t at [e * kPlanBlock + t]): the node histogram hist[g][v] (nodes of
+// type g with v free GPUs, v <= vmax) and the demand word dem[g] (GPUs of
+// groups per size class e in 16-bit field e).
+__host__ __device__ inline size_t plan_smem(int NT, int vmax) {
+    return (size_t)kPlanBlock * (2 * (size_t)NT * (vmax + 1) + 8 * kMaxTypes);
+}
+
 __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
     const Layout& y = a.lay;
-    const int L = y.L;
+    const int L = y.L, NT = y.NT, V = a.vmax;
     const int64_t* P = reinterpret_cast<const int64_t*>(a.img + y.offP);
     const int64_t* PB = reinterpret_cast<const int64_t*>(a.img + y.offPB);
     const int64_t* p2p = reinterpret_cast<const int64_t*>(a.img + y.offP2P);
     const int64_t* inter = reinterpret_cast<const int64_t*>(a.img + y.offInter);
     const int32_t* maxn = reinterpret_cast<const int32_t*>(a.img + y.offMaxN);
     const int32_t* pow2 = reinterpret_cast<const int32_t*>(a.img + y.offPow2);
+    extern __shared__ __align__(16) unsigned char psm[];
+    uint64_t* dem = reinterpret_cast<uint64_t*>(psm) + threadIdx.x;  // [g * kPlanBlock]
+    uint16_t* hist = reinterpret_cast<uint16_t*>(psm + (size_t)8 * kMaxTypes * kPlanBlock) + threadIdx.x;
     // the cluster's nodes per type and GPU count, shared by the CTA
-    __shared__ uint32_t init[kMaxTypes][kPlanMaxNode + 1];
+    __shared__ __align__(4) uint16_t init[kMaxTypes][kPlanMaxNode + 1];
     for (int i = threadIdx.x; i < kMaxTypes * (kPlanMaxNode + 1); i += blockDim.x) (&init[0][0])[i] = 0;
     __syncthreads();
-    for (int b = threadIdx.x; b < a.n_nodes; b += blockDim.x) atomicAdd(&init[a.node_type[b]][a.node_gpus[b]], 1u);
+    for (int b = threadIdx.x; b < a.n_nodes; b += blockDim.x) {
+        // 16-bit counts: at most 65535 nodes (the library's GPU limit)
+        unsigned int* w = reinterpret_cast<unsigned int*>(&init[0][0]) +
+                          ((a.node_type[b] * (kPlanMaxNode + 1) + a.node_gpus[b]) >> 1);
+        atomicAdd(w, ((a.node_type[b] * (kPlanMaxNode + 1) + a.node_gpus[b]) & 1) ? 0x10000u : 1u);
+    }
     __syncthreads();
+    auto H = [&](int g, int v) -> uint16_t& { return hist[(size_t)(g * (V + 1) + v) * kPlanBlock]; };
+    // whole warps step together (lanes past n idle), so the warp can
+    // reconverge before each slot's stores and every store covers whole
+    // 32-byte sectors (a partial sector costs a DRAM read-modify-write)
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < a.n; c += stride) {
-        // nodes per type by free GPUs, and per (type, class e) the GPUs
-        // groups of size >= 2^e can use: sum of floor(free / 2^e) 2^e
-        uint16_t hist[kMaxTypes][kPlanMaxNode + 1];
-        int64_t cap[kMaxTypes][4];
-        for (int g = 0; g < kMaxTypes; ++g) {
-            for (int e = 0; e < 4; ++e) cap[g][e] = 0;
-            for (int v = 0; v <= kPlanMaxNode; ++v) {
-                hist[g][v] = (uint16_t)init[g][v];
-                for (int e = 0; e < 4; ++e) cap[g][e] += (int64_t)init[g][v] * ((v >> e) << e);
-            }
-        }
-        const int nt = min((int)a.n_tmpl[c], a.slots);
+    for (int64_t c0 = (int64_t)blockIdx.x * blockDim.x; c0 < a.n; c0 += stride) {
+        const int64_t c = c0 + threadIdx.x;
+        const bool valid = c < a.n;
+        for (int g = 0; g < NT; ++g)
+            for (int v = 0; v <= V; ++v) H(g, v) = init[g][v];
+        const int nt = valid ? min((int)a.n_tmpl[c], a.slots) : 0;
         bool ended = false;
         int placed = 0;
         double thr = 0.0;
@@ -65,30 +80,45 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
             uint8_t st = HEDDLE_CAND_SKIPPED;
             int64_t T = -1, B = -1;
             int64_t n = 0;
-            const int S = sl.S[c];
-            const int M = sl.M[c];
+            const int S = valid ? sl.S[c] : 0;
+            const int M = valid ? sl.M[c] : 0;
             if (!ended && t < nt) {
                 const uint8_t st0 = sl.status[c];
                 if (st0 == HEDDLE_CAND_INVALID) {
                     st = HEDDLE_CAND_INVALID;
                 } else {
                     // demand per (type, size class) in GPUs of groups of that class
-                    uint32_t dem[kMaxTypes][4];
-                    for (int g = 0; g < kMaxTypes; ++g)
-                        for (int e = 0; e < 4; ++e) dem[g][e] = 0;
+                    for (int g = 0; g < NT; ++g) dem[g * kPlanBlock] = 0;
+                    uint32_t present = 0;
                     for (int s = 0; s < S; ++s) {
                         const int b = sl.code[(int64_t)s * sl.stride + c];
                         const int g = b & 7, j = (b >> 3) & 3;
                         const int unit = (1 << j) <= maxn[g] ? (1 << j) : pow2[g];
-                        dem[g][31 - __clz(unit)] += 1u << j;
+                        dem[g * kPlanBlock] += (uint64_t)(1u << j) << (16 * (31 - __clz(unit)));
+                        present |= 1u << g;
                     }
+                    // n = min over (type, class e) of floor(cap / demand),
+                    // cap = sum over nodes of floor(free / 2^e) 2^e
                     int64_t best = -1;
-                    for (int g = 0; g < kMaxTypes; ++g) {
+                    for (uint32_t pm = present; pm; pm &= pm - 1) {
+                        const int g = __ffs(pm) - 1;
+                        int64_t cap[4] = {0, 0, 0, 0};
+                        for (int v = 1; v <= V; ++v) {
+                            const int64_t h = H(g, v);
+                            if (!h) continue;
+                            cap[0] += h * v;
+                            cap[1] += h * ((v >> 1) << 1);
+                            cap[2] += h * ((v >> 2) << 2);
+                            cap[3] += h * ((v >> 3) << 3);
+                        }
+                        const uint64_t dw = dem[g * kPlanBlock];
                         uint32_t d = 0;
+#pragma unroll
                         for (int e = 3; e >= 0; --e) {
-                            d += dem[g][e];
-                            if (dem[g][e] == 0) continue;  // dominated by the class above
-                            const int64_t q = cap[g][e] / d;
+                            const uint32_t f = (uint32_t)(dw >> (16 * e)) & 0xffffu;
+                            d += f;
+                            if (f == 0) continue;  // dominated by the class above
+                            const int64_t q = cap[e] / d;
                             if (best < 0 || q < best) best = q;
                         }
                     }
@@ -140,29 +170,27 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
                         placed = t + 1;
                         // place n copies of the groups, largest first
                         for (int e = 3; e >= 0; --e) {
-                            const uint32_t w = 1u << e;
-                            for (int g = 0; g < kMaxTypes; ++g) {
-                                int64_t left = (int64_t)(dem[g][e] >> e) * n;
+                            const int w = 1 << e;
+                            for (uint32_t pm = present; pm; pm &= pm - 1) {
+                                const int g = __ffs(pm) - 1;
+                                int64_t left = (int64_t)(((dem[g * kPlanBlock] >> (16 * e)) & 0xffffu) >> e) * n;
                                 while (left > 0) {
-                                    if (hist[g][w] > 0) {
+                                    if (w <= V && H(g, w) > 0) {
                                         // nodes with exactly w free: m of them filled
-                                        const int64_t m = min(left, (int64_t)hist[g][w]);
-                                        hist[g][w] -= (uint16_t)m;
-                                        hist[g][0] += (uint16_t)m;
-                                        for (int e2 = 0; e2 < 4; ++e2) cap[g][e2] -= m * (((int64_t)w >> e2) << e2);
+                                        const int64_t m = min(left, (int64_t)H(g, w));
+                                        H(g, w) -= (uint16_t)m;
+                                        H(g, 0) += (uint16_t)m;
                                         left -= m;
                                         continue;
                                     }
                                     int v = w + 1;
-                                    while (v <= kPlanMaxNode && hist[g][v] == 0) ++v;
-                                    if (v > kPlanMaxNode) {
+                                    while (v <= V && H(g, v) == 0) ++v;
+                                    if (v > V) {
                                         atomicOr(a.err, kErrInternal);  // n came from these nodes
                                         break;
                                     }
-                                    hist[g][v] -= 1;
-                                    hist[g][v - w] += 1;
-                                    for (int e2 = 0; e2 < 4; ++e2)
-                                        cap[g][e2] -= (int64_t)(((v >> e2) << e2) - (((v - (int)w) >> e2) << e2));
+                                    H(g, v) -= 1;
+                                    H(g, v - w) += 1;
                                     left -= 1;
                                 }
                             }
@@ -171,15 +199,24 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
                 }
                 if (st != HEDDLE_CAND_OK) ended = true;
             }
-            sl.T[c] = T;
-            sl.B[c] = B;
-            sl.ndp[c] = (uint16_t)(st == HEDDLE_CAND_OK || st == HEDDLE_CAND_OOM ? n : 0);
-            sl.status[c] = st;
-            if (st != HEDDLE_CAND_OK)
-                for (int s = 0; s <= kMaxStages; ++s) sl.bounds[(int64_t)s * sl.bstride + c] = 0;
+            __syncwarp();
+            if (valid) {
+                sl.T[c] = T;
+                sl.B[c] = B;
+                sl.ndp[c] = (uint16_t)(st == HEDDLE_CAND_OK || st == HEDDLE_CAND_OOM ? n : 0);
+                sl.status[c] = st;
+                // every lane rewrites all planes (its split, or zeros unless OK)
+                for (int s = 0; s <= kMaxStages; ++s) {
+                    uint8_t* bp = sl.bounds + (int64_t)s * sl.bstride + c;
+                    *bp = st == HEDDLE_CAND_OK ? *bp : (uint8_t)0;
+                }
+            }
         }
-        a.placed[c] = (uint8_t)placed;
-        a.thr[c] = thr;
+        __syncwarp();
+        if (valid) {
+            a.placed[c] = (uint8_t)placed;
+            a.thr[c] = thr;
+        }
     }
 }
 
@@ -187,8 +224,16 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
 
 cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
-    const int grid = (int)std::min<int64_t>((a.n + kPlanBlock - 1) / kPlanBlock, (int64_t)num_sms * 16);
-    plan_kernel<<<grid, kPlanBlock, 0, st>>>(a);
+    if (a.vmax < 1 || a.vmax > kPlanMaxNode) return cudaErrorInvalidValue;
+    const size_t smem = plan_smem(a.lay.NT, a.vmax);
+    cudaError_t e = cudaFuncSetAttribute(plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, plan_kernel, kPlanBlock, smem);
+    if (e != cudaSuccess) return e;
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const int grid = (int)std::min<int64_t>((a.n + kPlanBlock - 1) / kPlanBlock, (int64_t)num_sms * per_sm);
+    plan_kernel<<<grid, kPlanBlock, smem, st>>>(a);
     return cudaGetLastError();
 }
 

@@ -245,9 +245,28 @@ __device__ __forceinline__ bool has(const uint32_t* C, int i) { return (C[i >> 5
 
 // smallest set position in [i, hi], -1 if none
 __device__ int next_in(const uint32_t* C, int i, int hi) {
-    for (int x = i; x <= hi; ++x)
-        if (has(C, x)) return x;
-    return -1;
+    if (i > hi) return -1;
+    int w = i >> 5;
+    uint32_t m = C[w] & (0xffffffffu << (i & 31));
+    while (m == 0) {
+        if (++w > (hi >> 5)) return -1;
+        m = C[w];
+    }
+    const int x = (w << 5) + __ffs(m) - 1;
+    return x <= hi ? x : -1;
+}
+
+// largest set position in [lo, i], -1 if none
+__device__ int prev_in(const uint32_t* C, int i, int lo) {
+    if (i < lo) return -1;
+    int w = i >> 5;
+    uint32_t m = C[w] & (0xffffffffu >> (31 - (i & 31)));
+    while (m == 0) {
+        if (--w < (lo >> 5)) return -1;
+        m = C[w];
+    }
+    const int x = (w << 5) + 31 - __clz(m);
+    return x >= lo ? x : -1;
 }
 
 // Exact probe of bound B: C[s] = feasible starts of stage s (C[S] = {L}).
@@ -265,18 +284,26 @@ __device__ bool tprobe(const TTabs& t, const uint8_t* codes, int S, int M, int64
         const int imax = L - (S - s);
         int succ = next_in(C[s + 1], imax + 1, L);
         bool any = false;
-        for (int i = imax; i >= s; --i) {
+        int i = imax;
+        while (i >= s) {
             if (has(C[s + 1], i + 1)) succ = i + 1;
-            if (succ < 0) continue;
-            const int64_t v = ttime(t, st, i, succ);
-            if (v == kInf) continue;
-            if (v <= B) {
+            // kInf: no successor, or no tiling of [i, succ) fits memory
+            const int64_t v = succ < 0 ? kInf : ttime(t, st, i, succ);
+            if (v != kInf && v <= B) {
                 C[s][i >> 5] |= 1u << (i & 31);
                 hi = max(hi, v);
                 any = true;
-            } else {
-                lo = min(lo, v);
+                --i;
+                continue;
             }
+            if (v != kInf) lo = min(lo, v);
+            // [i, succ) is rejected (too slow or out of memory), and so is
+            // every longer [i', succ): resume below the next smaller
+            // successor
+            const int j2 = prev_in(C[s + 1], i, s + 1);
+            if (j2 < 0) break;
+            succ = j2;
+            i = j2 - 1;
         }
         if (!any) return false;
     }
@@ -343,14 +370,44 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
             a.wl_T[p] = -1;
             continue;
         }
+        // first guess: the balanced bound with every stage at its fastest
+        // tiling over all layers, then gallop until the bracket closes
+        float inv = 0.f, cw = 0.f;
+        for (int s = 0; s < S; ++s) {
+            const TStage st = tstage(t, codes, s, S, M);
+            const int base = tile_base(st.j), cnt = (st.j + 1) * (st.j + 2) / 2;
+            int64_t all = kInf;
+            for (int o = 0; o < cnt; ++o)
+                if (t.code[st.g * kTileSlots + base + o] & 0x80)
+                    all = min(all, t.Pt[(size_t)(st.g * kTileSlots + base + o) * (L + 1) + L]);
+            const float tot = u64_to_float((uint64_t)all) + 1.0f;
+            inv += 1.0f / tot;
+            cw += u64_to_float((uint64_t)st.c) / tot;
+        }
         int64_t Bhi = hi, Blo = 0;
+        bool lo_known = false, hi_known = false;
+        int64_t B = (int64_t)float_to_u64((1.0f + cw) / inv);
+        int64_t step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
         int it = 0;
         while (Blo < Bhi) {
-            const int64_t B = Blo + (Bhi - Blo) / 2;
-            if (tprobe(t, codes, S, M, B, hi, lo, C))
+            B = min(max(B, Blo), Bhi - 1);
+            if (tprobe(t, codes, S, M, B, hi, lo, C)) {
                 Bhi = hi;
-            else
+                hi_known = true;
+            } else {
                 Blo = lo;
+                lo_known = true;
+            }
+            if (Blo >= Bhi) break;
+            if (!lo_known) {
+                B = Bhi - step;
+                step *= 2;
+            } else if (!hi_known) {
+                B = Blo + step;
+                step *= 2;
+            } else {
+                B = Blo + (Bhi - Blo) / 2;
+            }
             if (++it > kMaxIters) {
                 atomicOr(a.err, kErrSearchBound);
                 break;
