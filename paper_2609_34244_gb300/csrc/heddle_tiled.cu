@@ -123,13 +123,37 @@ __global__ void __launch_bounds__(kTabThreads) tiled_tables_kernel(TiledTableArg
         }
         Pt[(size_t)(g * kTileSlots + slot) * (L + 1) + l + 1] = q;
     }
+    __syncthreads();
+    // A tiling is dominated when another allowed tiling of the same degree
+    // and EDP degree (hence the same memory and gradient terms) comes first
+    // and is no slower on every layer, or is strictly faster on every layer:
+    // on every interval it is then never the fastest fitting tiling, nor the
+    // earliest among equally fast ones, so the search skips it (bit 6).
     for (int t = tid; t < 8 * kTileSlots; t += blockDim.x) {
         const int slot = t % kTileSlots, g = t / kTileSlots;
         const int j = degree_of_slot(slot);
         int le, lt, ld;
         tiling_of(j, slot - tile_base(j), le, lt, ld);
         const bool allowed = g < NT && ggpus[g] > 0 && (1 << lt) <= gmaxn[g];
-        code[t] = (uint8_t)(le | (lt << 2) | (ld << 4) | (allowed ? 0x80 : 0));
+        bool dominated = false;
+        if (allowed) {
+            const int64_t* me = Pt + (size_t)(g * kTileSlots + slot) * (L + 1);
+            const int cnt = (j + 1) * (j + 2) / 2;
+            for (int o = 0; o < cnt && !dominated; ++o) {
+                const int other = tile_base(j) + o;
+                int le2, lt2, ld2;
+                tiling_of(j, o, le2, lt2, ld2);
+                if (other == slot || ld2 != ld || (1 << lt2) > gmaxn[g]) continue;
+                const int64_t* ot = Pt + (size_t)(g * kTileSlots + other) * (L + 1);
+                bool le_all = true, lt_all = true;
+                for (int l = 1; l <= L && le_all; ++l) {
+                    le_all = ot[l] <= me[l];
+                    lt_all = lt_all && ot[l] < me[l];
+                }
+                dominated = le_all && (lt_all || other < slot);
+            }
+        }
+        code[t] = (uint8_t)(le | (lt << 2) | (ld << 4) | (dominated ? 0x40 : 0) | (allowed ? 0x80 : 0));
     }
     __syncthreads();
     for (int r = tid; r < NT * kTileSlots; r += blockDim.x) {
@@ -233,7 +257,7 @@ __device__ int64_t ttime(const TTabs& t, const TStage& st, int i, int e) {
     for (int o = 0; o < cnt; ++o) {
         const int slot = base + o;
         const uint8_t cd = t.code[st.g * kTileSlots + slot];
-        if (!(cd & 0x80)) continue;
+        if ((cd & 0xc0) != 0x80) continue;  // not allowed, or dominated
         if (!tfits(t, st, i, e, (cd >> 4) & 3)) continue;
         const int64_t* P = t.Pt + (size_t)(st.g * kTileSlots + slot) * (t.L + 1);
         best = min(best, P[e] - P[i] + st.c);
@@ -378,7 +402,7 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
             const int base = tile_base(st.j), cnt = (st.j + 1) * (st.j + 2) / 2;
             int64_t all = kInf;
             for (int o = 0; o < cnt; ++o)
-                if (t.code[st.g * kTileSlots + base + o] & 0x80)
+                if ((t.code[st.g * kTileSlots + base + o] & 0xc0) == 0x80)
                     all = min(all, t.Pt[(size_t)(st.g * kTileSlots + base + o) * (L + 1) + L]);
             const float tot = u64_to_float((uint64_t)all) + 1.0f;
             inv += 1.0f / tot;
@@ -451,7 +475,7 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
                 // the slots of EDP exponent m: ETP exponent 0 .. j - m
                 for (int lt = 0; lt <= st.j - m; ++lt, ++o) {
                     const uint8_t cd = t.code[st.g * kTileSlots + base + o];
-                    if (!(cd & 0x80) || !tfits(t, st, i0, i1, m)) continue;
+                    if ((cd & 0xc0) != 0x80 || !tfits(t, st, i0, i1, m)) continue;
                     hasld |= (uint8_t)(1 << m);
                     const int64_t* P = t.Pt + (size_t)(st.g * kTileSlots + base + o) * (L + 1);
                     const int64_t v = P[i1] - P[i0] + st.c;
