@@ -181,12 +181,21 @@ typedef struct {
 } heddle_results;
 
 /* Price a batch (PartitionLayers + Evaluate, §3.1, §5.2, §5.3).
- * Asynchronous on `stream`; no host round-trip; allocates nothing.  Each
- * chunk of up to 2^20 candidates takes two launches: a screen (masks, DP
- * degree, memory) that compacts the candidates needing the threshold search
- * into a worklist owned by the context, then the search over that worklist.
- * Calls on one context must therefore not overlap on the GPU (use one
- * stream per context, or one context per stream).
+ * Asynchronous on `stream`; no host round-trip.  Each chunk of the batch
+ * (heddle_set_chunk, default and at most 2^20 candidates) takes two
+ * launches: a screen (masks, DP degree, memory) that compacts the
+ * candidates needing the threshold search into a worklist owned by the
+ * context, then the search over that worklist.  A batch of one chunk runs
+ * on `stream` and allocates nothing.  A batch of several chunks
+ * alternates two worklist sets and two context-owned work streams, so
+ * chunk i + 1 is screened and searched while chunk i finishes: each work
+ * stream first waits for the work queued on `stream` before the call, any
+ * top-k merge runs on `stream` in chunk order, and `stream` waits for every
+ * chunk before work queued after the call runs (stream-ordered as a single
+ * launch would be).  The first such call allocates the second set
+ * (~190 MB) and the streams (E_NOMEM if that fails).  Calls on one context
+ * must not overlap on the GPU (use one stream per context, or one context
+ * per stream).
  * A candidate is INVALID if S = 0, S > 32, S > s_max, S > L, M = 0, a stage
  * byte has bits 5-7 set, names a type >= n_types or a type without GPUs, or
  * (dense models) asks a degree above the largest node of its type (the TP
@@ -196,6 +205,10 @@ typedef struct {
  * failure).  n = 0 is a no-op. */
 heddle_status heddle_price_candidates(heddle_ctx* ctx, const heddle_candidates* cands,
                                       const heddle_results* results, void* stream);
+
+/* Chunk size of the pricing calls: 1 <= chunk <= 2^20 (E_LIMIT otherwise).
+ * Results never depend on it. */
+heddle_status heddle_set_chunk(heddle_ctx* ctx, int64_t chunk);
 
 /* ----------------------------------------------------------------- top-k */
 
@@ -401,14 +414,18 @@ heddle_status heddle_price_tiled(heddle_ctx* ctx, const heddle_candidates* cands
 /* -------------------------------------------------------- host buffers */
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the
- * candidates in batches of `batch` through context-owned device staging
- * buffers (two sets, copies overlapped with pricing), prices them, merges
- * them into *state and copies back every non-NULL field of `results` (host
- * arrays of cands->n entries; bounds uses plane stride cands->n).  *state is
- * host memory, read on entry (k, and any entries already held) and written
- * on return.  Synchronous: returns when all outputs are in host memory.
- * Grows its staging buffers on first use (allocation).  Errors as above,
- * plus E_NOMEM. */
+ * candidates in batches of `batch` (1 <= batch <= 2^20, E_LIMIT above)
+ * through context-owned device staging buffers (two sets), prices them,
+ * merges them into *state and copies back every non-NULL field of
+ * `results` (host arrays of cands->n entries; bounds uses plane stride
+ * cands->n).  Batch k is copied in on a copy stream, screened and searched
+ * on work stream k % 2 with worklist set k % 2, merged on `stream` in batch
+ * order and copied out on a second copy stream, so copies, the search of
+ * one batch and the screen of the next overlap.  *state is host memory,
+ * read on entry (k, and any entries already held) and written on return.
+ * Synchronous: returns when all outputs are in host memory.  Grows its
+ * staging buffers and creates the second worklist set on first use
+ * (allocation).  Errors as above, plus E_NOMEM. */
 heddle_status heddle_price_topk_host(heddle_ctx* ctx, const heddle_candidates* cands,
                                      const heddle_results* results, heddle_topk_state* state,
                                      int64_t batch, void* stream);
@@ -472,10 +489,13 @@ heddle_status heddle_work_counters(heddle_ctx* ctx, uint64_t out[3]);
  * roofline report times its kernels without a profiler.  While enabled
  * (heddle_time_phases(ctx, 1); no stream capture meanwhile, the events are
  * created on demand), every chunk that heddle_price_candidates,
- * heddle_price_topk or heddle_price_topk_host prices records four events:
- * before the screen kernel, between the screen and the search kernel,
- * after the search kernel and, when the call merges a top-k, after the
- * top-k kernels.  heddle_phase_times synchronises on them and returns, per
+ * heddle_price_topk or heddle_price_topk_host prices records events
+ * before the screen kernel, between the screen and the search kernel and
+ * after the search kernel (on the stream that runs them) and, when the call
+ * merges a top-k, before and after the top-k kernels (on `stream`).  With
+ * several chunks in flight the phases of neighbouring chunks overlap, so
+ * each phase's time is its own kernels' elapsed time while they share the
+ * GPU.  heddle_phase_times synchronises on them and returns, per
  * phase (SCREEN, SEARCH, TOPK), the summed elapsed milliseconds and the
  * number of kernels launched in it (one screen, one search and one top-k
  * kernel per chunk), then forgets them.  The events add no work to the

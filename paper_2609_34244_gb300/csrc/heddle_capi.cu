@@ -37,17 +37,29 @@ struct heddle_ctx {
     uint32_t* d_flags = nullptr;            // [0] table build, [1] device errors
     unsigned long long* d_counters = nullptr;  // [3]
     bool count_next = false;
-    // search worklist scratch (hd::kWorklistCap candidates)
-    int32_t* d_wl_count = nullptr;  // hd::kWlMeta ints
-    int32_t* d_wl_bucket = nullptr;  // [32][2^20]
-    int32_t* d_wl_idx = nullptr;
-    uint16_t* d_wl_n = nullptr;
-    uint16_t* d_wl_M = nullptr;
-    uint8_t* d_wl_S = nullptr;
-    uint8_t* d_wl_memok = nullptr;
-    uint8_t* d_wl_code = nullptr;
-    int64_t* d_wl_T = nullptr;
-    uint32_t* d_wl_nM = nullptr;
+    // search worklist scratch (hd::kWorklistCap candidates); the second
+    // set, the two work streams and their events exist once a call has
+    // priced more than one chunk (consecutive chunks alternate sets and
+    // streams, so one chunk's screen and search overlap the previous
+    // chunk's search and top-k)
+    struct Worklist {
+        int32_t* count = nullptr;   // hd::kWlMeta ints
+        int32_t* bucket = nullptr;  // [32][2^20]
+        int32_t* idx = nullptr;
+        uint16_t* n = nullptr;
+        uint16_t* M = nullptr;
+        uint8_t* S = nullptr;
+        uint8_t* memok = nullptr;
+        uint8_t* code = nullptr;
+        int64_t* T = nullptr;
+        uint32_t* nM = nullptr;
+    };
+    Worklist wl[2];
+    bool pipe_ready = false;
+    cudaStream_t s_work[2] = {nullptr, nullptr};
+    cudaEvent_t ev_in = nullptr;
+    cudaEvent_t ev_searched[2] = {nullptr, nullptr}, ev_wl_free[2] = {nullptr, nullptr};
+    int64_t chunk = hd::kWorklistCap;
     // top-k merge scratch
     hd::TopkEntry* d_scratch = nullptr;
     int32_t* d_scratch_count = nullptr;
@@ -75,7 +87,7 @@ struct heddle_ctx {
     bool time_phases = false;
     std::vector<cudaEvent_t> ev_pool;
     struct PhaseRec {
-        cudaEvent_t e[4];
+        cudaEvent_t e[5];  // screen start, screen end, search end, top-k start, top-k end
         bool topk;
         int64_t launches[3];
     };
@@ -395,6 +407,35 @@ heddle_status check_ready(heddle_ctx* x) {
     return HEDDLE_OK;
 }
 
+cudaError_t alloc_worklist(heddle_ctx::Worklist& w) {
+    const size_t cap = hd::kWorklistCap;
+    cudaError_t e = cudaMalloc(&w.count, sizeof(int32_t) * hd::kWlMeta);
+    if (e == cudaSuccess) e = cudaMalloc(&w.bucket, sizeof(int32_t) * HEDDLE_MAX_STAGES * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.idx, sizeof(int32_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.n, sizeof(uint16_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.M, sizeof(uint16_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.S, cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.memok, cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.code, (size_t)HEDDLE_MAX_STAGES * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.T, sizeof(int64_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.nM, sizeof(uint32_t) * cap);
+    return e;
+}
+
+void free_worklist(heddle_ctx::Worklist& w) {
+    cudaFree(w.count);
+    cudaFree(w.bucket);
+    cudaFree(w.idx);
+    cudaFree(w.n);
+    cudaFree(w.M);
+    cudaFree(w.S);
+    cudaFree(w.memok);
+    cudaFree(w.code);
+    cudaFree(w.T);
+    cudaFree(w.nM);
+    w = heddle_ctx::Worklist{};
+}
+
 }  // namespace
 
 extern "C" {
@@ -423,17 +464,7 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     if (e == cudaSuccess)
         e = cudaMalloc(&x->d_scratch, sizeof(hd::TopkEntry) * hd::kMaxTopK * x->scratch_blocks);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch_count, sizeof(int32_t) * x->scratch_blocks);
-    const size_t cap = hd::kWorklistCap;
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_count, sizeof(int32_t) * hd::kWlMeta);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_bucket, sizeof(int32_t) * HEDDLE_MAX_STAGES * cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_idx, sizeof(int32_t) * cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_n, sizeof(uint16_t) * cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_M, sizeof(uint16_t) * cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_S, cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_memok, cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_code, (size_t)HEDDLE_MAX_STAGES * cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_T, sizeof(int64_t) * cap);
-    if (e == cudaSuccess) e = cudaMalloc(&x->d_wl_nM, sizeof(uint32_t) * cap);
+    if (e == cudaSuccess) e = alloc_worklist(x->wl[0]);
     const int l2 = (x->scratch_blocks + 31) / 32;
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2, sizeof(hd::TopkEntry) * hd::kMaxTopK * l2);
     if (e == cudaSuccess) e = cudaMalloc(&x->d_scratch2_count, sizeof(int32_t) * l2);
@@ -457,16 +488,14 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_counters);
     cudaFree(x->d_scratch);
     cudaFree(x->d_scratch_count);
-    cudaFree(x->d_wl_count);
-    cudaFree(x->d_wl_bucket);
-    cudaFree(x->d_wl_idx);
-    cudaFree(x->d_wl_n);
-    cudaFree(x->d_wl_M);
-    cudaFree(x->d_wl_S);
-    cudaFree(x->d_wl_memok);
-    cudaFree(x->d_wl_code);
-    cudaFree(x->d_wl_T);
-    cudaFree(x->d_wl_nM);
+    free_worklist(x->wl[0]);
+    free_worklist(x->wl[1]);
+    for (int b = 0; b < 2; ++b) {
+        if (x->s_work[b]) cudaStreamDestroy(x->s_work[b]);
+        if (x->ev_searched[b]) cudaEventDestroy(x->ev_searched[b]);
+        if (x->ev_wl_free[b]) cudaEventDestroy(x->ev_wl_free[b]);
+    }
+    if (x->ev_in) cudaEventDestroy(x->ev_in);
     cudaFree(x->d_scratch2);
     cudaFree(x->d_scratch2_count);
     cudaFree(x->d_tickets);
@@ -618,6 +647,27 @@ heddle_status heddle_load_experts(heddle_ctx* x, const int64_t* expert_state, co
 
 namespace {
 
+// The second worklist set, the work streams and their events (once).
+heddle_status ensure_pipeline(heddle_ctx* x) {
+    if (x->pipe_ready) return HEDDLE_OK;
+    cudaError_t e = alloc_worklist(x->wl[1]);
+    for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+        if (!x->s_work[b]) e = cudaStreamCreateWithFlags(&x->s_work[b], cudaStreamNonBlocking);
+        if (e == cudaSuccess && !x->ev_searched[b])
+            e = cudaEventCreateWithFlags(&x->ev_searched[b], cudaEventDisableTiming);
+        if (e == cudaSuccess && !x->ev_wl_free[b])
+            e = cudaEventCreateWithFlags(&x->ev_wl_free[b], cudaEventDisableTiming);
+    }
+    if (e == cudaSuccess && !x->ev_in) e = cudaEventCreateWithFlags(&x->ev_in, cudaEventDisableTiming);
+    if (e != cudaSuccess) {
+        free_worklist(x->wl[1]);
+        return fail(x, e == cudaErrorMemoryAllocation ? HEDDLE_E_NOMEM : HEDDLE_E_CUDA,
+                    "second worklist set: %s", cudaGetErrorString(e));
+    }
+    x->pipe_ready = true;
+    return HEDDLE_OK;
+}
+
 hd::TopkArgs topk_args(heddle_ctx* x, heddle_topk_state* state) {
     hd::TopkArgs a{};
     a.state = state;
@@ -630,9 +680,9 @@ hd::TopkArgs topk_args(heddle_ctx* x, heddle_topk_state* state) {
     return a;
 }
 
-// Four timing events for one chunk, from the pool (created on demand).
+// Five timing events for one chunk, from the pool (created on demand).
 heddle_status take_phase_rec(heddle_ctx* x, heddle_ctx::PhaseRec* rec) {
-    for (int i = 0; i < 4; ++i) {
+    for (int i = 0; i < 5; ++i) {
         if (x->ev_pool.empty()) {
             cudaEvent_t ev;
             CU(cudaEventCreate(&ev));
@@ -640,6 +690,93 @@ heddle_status take_phase_rec(heddle_ctx* x, heddle_ctx::PhaseRec* rec) {
         }
         rec->e[i] = x->ev_pool.back();
         x->ev_pool.pop_back();
+    }
+    return HEDDLE_OK;
+}
+
+// The call-wide fields of the pricing arguments (consumes count_next).
+void fill_price_args(heddle_ctx* x, const heddle_candidates* c, const heddle_ctx::Level* lvl, int shift, bool tiled,
+                     hd::PriceArgs& a) {
+    a.lay = lvl ? lvl->lay : x->lay;
+    a.img = lvl ? lvl->img : x->d_img;
+    a.mbs_shift = shift;
+    a.moe = x->moe;
+    a.stride = c->plane_stride;
+    a.s_max = c->s_max;
+    a.bstride = c->n;
+    a.err = x->d_flags + 1;
+    a.counters = x->count_next ? x->d_counters : nullptr;
+    x->count_next = false;
+    a.wl_cap = hd::kWorklistCap;
+    a.uniform = !tiled && equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
+    a.split_mode = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? 1 : 0;
+}
+
+// One chunk [lo, lo + nb) of cands into r: screen and search on `ws` with
+// worklist set W, then (with a state) the top-k over the chunk's searched
+// candidates on `cs`, after the search when ws != cs.  `a` holds the
+// call-wide fields; its chunk fields are set here.
+heddle_status price_chunk(heddle_ctx* x, hd::PriceArgs& a, const heddle_candidates* c, const heddle_results* r,
+                          int64_t lo, int64_t nb, int set, cudaStream_t ws, heddle_topk_state* state,
+                          cudaStream_t cs, bool tiled, uint8_t* tiling) {
+    heddle_status st;
+    const heddle_ctx::Worklist& W = x->wl[set];
+    a.wl_count = W.count;
+    a.wl_idx = W.idx;
+    a.wl_n = W.n;
+    a.wl_M = W.M;
+    a.wl_S = W.S;
+    a.wl_memok = W.memok;
+    a.wl_code = W.code;
+    a.wl_bucket = W.bucket;
+    a.wl_T = W.T;
+    a.wl_nM = W.nM;
+    a.S = c->S + lo;
+    a.M = c->M + lo;
+    a.code = c->code + lo;
+    a.n = nb;
+    a.T = r->T + lo;
+    a.B = r->bottleneck + lo;
+    a.ndp = r->n_dp + lo;
+    a.status = r->status + lo;
+    a.bounds = r->bounds ? r->bounds + lo : nullptr;
+    heddle_ctx::PhaseRec rec{};
+    if (x->time_phases) {
+        if ((st = take_phase_rec(x, &rec)) != HEDDLE_OK) return st;
+        rec.topk = state != nullptr;
+        x->phase_recs.push_back(rec);
+        CU(cudaEventRecord(rec.e[0], ws));
+    }
+    int64_t* nl = x->time_phases ? x->phase_recs.back().launches : nullptr;
+    if (tiled) {
+        hd::TiledArgs ta{};
+        ta.tl = x->tlay;
+        ta.timg = x->d_timg;
+        ta.tiling = tiling ? tiling + lo : nullptr;
+        ta.tstride = c->n;
+        CU(hd::launch_screen(a, x->num_sms, ws, x->time_phases ? rec.e[1] : nullptr, nl));
+        if (nl) nl[1] += 1;
+        CU(hd::launch_tiled_search(a, ta, x->num_sms, ws));
+    } else {
+        CU(hd::launch_price(a, x->num_sms, ws, x->time_phases ? rec.e[1] : nullptr, nl));
+    }
+    if (x->time_phases) CU(cudaEventRecord(rec.e[2], ws));
+    if (state) {
+        if (ws != cs) {
+            CU(cudaEventRecord(x->ev_searched[set], ws));
+            CU(cudaStreamWaitEvent(cs, x->ev_searched[set], 0));
+        }
+        if (x->time_phases) CU(cudaEventRecord(rec.e[3], cs));
+        // top-k over the searched candidates of this chunk only
+        hd::TopkArgs m = topk_args(x, state);
+        m.base_index = c->base_index + lo;
+        m.wl_count = W.count;
+        m.wl_idx = W.idx;
+        m.wl_T = W.T;
+        m.wl_nM = W.nM;
+        m.wl_cap = hd::kWorklistCap;
+        CU(hd::launch_topk_worklist(m, nb, x->num_sms, cs, nl ? nl + 2 : nullptr));
+        if (x->time_phases) CU(cudaEventRecord(rec.e[4], cs));
     }
     return HEDDLE_OK;
 }
@@ -665,76 +802,37 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     DeviceGuard dg(x->device);
     if (tiled && tiling) CU(cudaMemsetAsync(tiling, 0, (size_t)HEDDLE_MAX_STAGES * c->n, (cudaStream_t)stream));
     hd::PriceArgs a{};
-    a.lay = lvl ? lvl->lay : x->lay;
-    a.img = lvl ? lvl->img : x->d_img;
-    a.mbs_shift = shift;
-    a.moe = x->moe;
-    a.stride = c->plane_stride;
-    a.s_max = c->s_max;
-    a.bstride = c->n;
-    a.err = x->d_flags + 1;
-    a.counters = x->count_next ? x->d_counters : nullptr;
-    x->count_next = false;
-    a.wl_count = x->d_wl_count;
-    a.wl_idx = x->d_wl_idx;
-    a.wl_n = x->d_wl_n;
-    a.wl_M = x->d_wl_M;
-    a.wl_S = x->d_wl_S;
-    a.wl_memok = x->d_wl_memok;
-    a.wl_code = x->d_wl_code;
-    a.wl_bucket = x->d_wl_bucket;
-    a.wl_cap = hd::kWorklistCap;
-    a.uniform = !tiled && equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
-    a.split_mode = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? 1 : 0;
-    a.wl_T = x->d_wl_T;
-    a.wl_nM = x->d_wl_nM;
-    // chunks of at most the worklist capacity, in stream order
-    for (int64_t lo = 0; lo < c->n; lo += hd::kWorklistCap) {
-        const int64_t nb = c->n - lo < hd::kWorklistCap ? c->n - lo : hd::kWorklistCap;
-        a.S = c->S + lo;
-        a.M = c->M + lo;
-        a.code = c->code + lo;
-        a.n = nb;
-        a.T = r->T + lo;
-        a.B = r->bottleneck + lo;
-        a.ndp = r->n_dp + lo;
-        a.status = r->status + lo;
-        a.bounds = r->bounds ? r->bounds + lo : nullptr;
-        heddle_ctx::PhaseRec rec{};
-        if (x->time_phases) {
-            if ((st = take_phase_rec(x, &rec)) != HEDDLE_OK) return st;
-            rec.topk = state != nullptr;
-            x->phase_recs.push_back(rec);
-            CU(cudaEventRecord(rec.e[0], (cudaStream_t)stream));
-        }
-        int64_t* nl = x->time_phases ? x->phase_recs.back().launches : nullptr;
-        if (tiled) {
-            hd::TiledArgs ta{};
-            ta.tl = x->tlay;
-            ta.timg = x->d_timg;
-            ta.tiling = tiling ? tiling + lo : nullptr;
-            ta.tstride = c->n;
-            CU(hd::launch_screen(a, x->num_sms, (cudaStream_t)stream, x->time_phases ? rec.e[1] : nullptr, nl));
-            if (nl) nl[1] += 1;
-            CU(hd::launch_tiled_search(a, ta, x->num_sms, (cudaStream_t)stream));
-        } else {
-            CU(hd::launch_price(a, x->num_sms, (cudaStream_t)stream, x->time_phases ? rec.e[1] : nullptr, nl));
-        }
-        if (x->time_phases) CU(cudaEventRecord(rec.e[2], (cudaStream_t)stream));
-        if (state) {
-            // top-k over the searched candidates of this chunk only
-            hd::TopkArgs m = topk_args(x, state);
-            m.base_index = c->base_index + lo;
-            m.wl_count = x->d_wl_count;
-            m.wl_idx = x->d_wl_idx;
-            m.wl_T = x->d_wl_T;
-            m.wl_nM = x->d_wl_nM;
-            m.wl_cap = hd::kWorklistCap;
-            CU(hd::launch_topk_worklist(m, nb, x->num_sms, (cudaStream_t)stream,
-                                        nl ? nl + 2 : nullptr));
-            if (x->time_phases) CU(cudaEventRecord(rec.e[3], (cudaStream_t)stream));
-        }
+    fill_price_args(x, c, lvl, shift, tiled, a);
+    // chunks of at most x->chunk candidates.  With one chunk everything runs
+    // on the caller's stream.  With more, chunk i runs its screen and search
+    // on work stream i % 2 with worklist set i % 2 (after the caller's
+    // earlier work and after chunk i - 2 released that set), and its top-k
+    // on the caller's stream after its search, so the top-k merges stay in
+    // chunk order while chunk i + 1 is screened and searched meanwhile.
+    const cudaStream_t cs = (cudaStream_t)stream;
+    const int64_t chunk = x->chunk;
+    const bool pipe = c->n > chunk;
+    if (pipe) {
+        if ((st = ensure_pipeline(x)) != HEDDLE_OK) return st;
+        CU(cudaEventRecord(x->ev_in, cs));
     }
+    bool used[2] = {false, false};
+    int64_t i = 0;
+    for (int64_t lo = 0; lo < c->n; lo += chunk, ++i) {
+        const int64_t nb = c->n - lo < chunk ? c->n - lo : chunk;
+        const int b = pipe ? (int)(i & 1) : 0;
+        const cudaStream_t ws = pipe ? x->s_work[b] : cs;
+        if (pipe) {
+            CU(cudaStreamWaitEvent(ws, x->ev_in, 0));
+            if (used[b]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[b], 0));
+            used[b] = true;
+        }
+        if ((st = price_chunk(x, a, c, r, lo, nb, b, ws, state, cs, tiled, tiling)) != HEDDLE_OK) return st;
+        if (pipe) CU(cudaEventRecord(x->ev_wl_free[b], state ? cs : ws));
+    }
+    if (pipe && !state)
+        for (int b = 0; b < 2; ++b)
+            if (used[b]) CU(cudaStreamWaitEvent(cs, x->ev_wl_free[b], 0));
     return ok(x);
 }
 
@@ -801,8 +899,13 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
     if (state->k < 1 || state->k > HEDDLE_MAX_TOPK)
         return fail(x, HEDDLE_E_LIMIT, "state k must be in [1, %d]", HEDDLE_MAX_TOPK);
     if (batch < 1) return fail(x, HEDDLE_E_ARG, "batch must be >= 1");
+    if (batch > hd::kWorklistCap) return fail(x, HEDDLE_E_LIMIT, "batch must be at most %d", hd::kWorklistCap);
     if ((st = check_ready(x)) != HEDDLE_OK) return st;
+    const bool tiled = x->tiled_ready;
+    if (tiled && x->search_mode == HEDDLE_SEARCH_DISTRIBUTE)
+        return fail(x, HEDDLE_E_STATE, "expert tiling prices the min-max split only (search mode DISTRIBUTE)");
     DeviceGuard dg(x->device);
+    if ((st = ensure_pipeline(x)) != HEDDLE_OK) return st;
     cudaStream_t sc = (cudaStream_t)stream;
     const int64_t n = c->n;
     const int64_t nb_max = n < batch ? (n > 0 ? n : 1) : batch;
@@ -856,6 +959,10 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
     CU(cudaEventRecord(x->ev_free[0], sc));
     CU(cudaEventRecord(x->ev_free[1], sc));
     const bool want_bounds = r && r->bounds;
+    // batch k: copies in on s_h2d, screen and search on work stream k % 2
+    // (worklist set k % 2, released by batch k - 2's top-k), top-k merge on
+    // the caller's stream in batch order, copies out on s_d2h
+    bool used[2] = {false, false};
     for (int64_t lo = 0, it = 0; lo < n; lo += batch, ++it) {
         const int b = (int)(it & 1);
         const int64_t nb = (n - lo) < batch ? (n - lo) : batch;
@@ -866,8 +973,10 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         CU(cudaMemcpy2DAsync(x->st_code[b], nb, c->code + lo, c->plane_stride, nb, c->s_max,
                              cudaMemcpyHostToDevice, x->s_h2d));
         CU(cudaEventRecord(x->ev_loaded[b], x->s_h2d));
-        // price and merge on the caller's stream
-        CU(cudaStreamWaitEvent(sc, x->ev_loaded[b], 0));
+        const cudaStream_t ws = x->s_work[b];
+        CU(cudaStreamWaitEvent(ws, x->ev_loaded[b], 0));
+        if (used[b]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[b], 0));
+        used[b] = true;
         heddle_candidates cb{};
         cb.S = x->st_S[b];
         cb.M = x->st_M[b];
@@ -882,7 +991,13 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         rb.n_dp = x->st_n[b];
         rb.status = x->st_status[b];
         rb.bounds = want_bounds ? x->st_bounds[b] : nullptr;
-        if ((st = price_impl(x, &cb, &rb, x->d_state, sc)) != HEDDLE_OK) return st;
+        if (nb > 0) {
+            hd::PriceArgs a{};
+            fill_price_args(x, &cb, nullptr, 0, tiled, a);
+            if ((st = price_chunk(x, a, &cb, &rb, 0, nb, b, ws, x->d_state, sc, tiled, nullptr)) != HEDDLE_OK)
+                return st;
+        }
+        CU(cudaEventRecord(x->ev_wl_free[b], sc));
         CU(cudaEventRecord(x->ev_priced[b], sc));
         // device -> host of the requested result fields on the second copy stream
         CU(cudaStreamWaitEvent(x->s_d2h, x->ev_priced[b], 0));
@@ -1105,6 +1220,14 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     return ok(x);
 }
 
+heddle_status heddle_set_chunk(heddle_ctx* x, int64_t chunk) {
+    if (!x) return HEDDLE_E_ARG;
+    if (chunk < 1 || chunk > hd::kWorklistCap)
+        return fail(x, HEDDLE_E_LIMIT, "chunk must be in [1, %d]", hd::kWorklistCap);
+    x->chunk = chunk;
+    return ok(x);
+}
+
 heddle_status heddle_time_phases(heddle_ctx* x, int32_t enable) {
     if (!x) return HEDDLE_E_ARG;
     x->time_phases = enable != 0;
@@ -1119,12 +1242,15 @@ heddle_status heddle_phase_times(heddle_ctx* x, double ms[HEDDLE_N_PHASES], int6
         launches[p] = 0;
     }
     heddle_status st = HEDDLE_OK;
+    // screen e0 -> e1, search e1 -> e2, top-k e3 -> e4 (its own start: with
+    // several chunks the top-k runs on another stream than the search)
+    static const int from[HEDDLE_N_PHASES] = {0, 1, 3}, to[HEDDLE_N_PHASES] = {1, 2, 4};
     for (auto& r : x->phase_recs) {
-        const int last = r.topk ? 3 : 2;
-        cudaError_t e = cudaEventSynchronize(r.e[last]);
-        for (int p = 0; p < last && e == cudaSuccess; ++p) {
+        const int np = r.topk ? 3 : 2;
+        cudaError_t e = cudaEventSynchronize(r.e[r.topk ? 4 : 2]);
+        for (int p = 0; p < np && e == cudaSuccess; ++p) {
             float t = 0.f;
-            e = cudaEventElapsedTime(&t, r.e[p], r.e[p + 1]);
+            e = cudaEventElapsedTime(&t, r.e[from[p]], r.e[to[p]]);
             ms[p] += t;
             launches[p] += r.launches[p];
         }

@@ -80,7 +80,7 @@ EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_
            "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
            "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times",
            "heddle_load_mbs", "heddle_price_mbs", "heddle_price_plans", "heddle_load_experts",
-           "heddle_price_tiled"]
+           "heddle_price_tiled", "heddle_set_chunk"]
 MAX_MBS_LEVELS = 4
 PHASES = ("screen", "search", "topk")
 TOPK_NOALLOC_MAX_N = 4194304
@@ -122,6 +122,7 @@ def load_library(path: str = LIB_PATH):
         "heddle_price_mbs": (i32, [p, p, p, p, p]),
         "heddle_load_experts": (i32, [p, p, p, i32]),
         "heddle_price_tiled": (i32, [p, p, p, p, p]),
+        "heddle_set_chunk": (i32, [p, i64]),
         "heddle_phase_times": (i32, [p, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
     }
     for name, (res, args) in sig.items():
@@ -249,6 +250,12 @@ def heddle_price_mbs(ctx, cands, results, mbs=None, stream=None):
     r = results if isinstance(results, heddle_results) else make_results(results)
     _check(ctx, load_library().heddle_price_mbs(ctx, C.byref(c), C.byref(r),
                                                 None if mbs is None else _ptr(mbs), _stream(stream)))
+
+
+def heddle_set_chunk(ctx, chunk: int):
+    """Chunk size of the pricing calls (1 .. 2**20); a call of several
+    chunks pipelines them over two work streams."""
+    _check(ctx, load_library().heddle_set_chunk(ctx, int(chunk)))
 
 
 def heddle_load_experts(ctx, expert_state=None, expert_param=None):

@@ -9,12 +9,14 @@ import numpy as np
 
 
 def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False, search=None,
-              fused=False, phases=False):
+              fused=False, phases=False, chunk=None):
     """Price on the GPU through the C ABI; returns numpy results, the top-k
     and (optionally) the work counters.  ``batch`` splits the candidates into
     consecutive launches merged into one top-k state; ``fused`` prices and
     merges in one call (heddle_price_topk); ``phases`` times the pricing
-    phases with the library's events and returns them under "phases"."""
+    phases with the library's events and returns them under "phases";
+    ``chunk`` sets the library's chunk size (calls of several chunks are
+    pipelined over its work streams)."""
     import torch
     ctx = h.heddle_create(0)
     try:
@@ -22,6 +24,8 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
         h.heddle_load_model(ctx, w_model)
         if search is not None:
             h.heddle_set_search(ctx, search)
+        if chunk is not None:
+            h.heddle_set_chunk(ctx, chunk)
         n = int(cands["S"].shape[0])
         dc = h.cands_to_device(cands)
         res = h.alloc_results(n, bounds=False)
@@ -136,7 +140,8 @@ def take(cands, idx):
             "code": np.ascontiguousarray(cands["code"][:, idx])}
 
 
-def price_tiled_gpu(h, w_cluster, w_model, cands, expert_state, expert_param, k=16, fused=False, batch=None):
+def price_tiled_gpu(h, w_cluster, w_model, cands, expert_state, expert_param, k=16, fused=False, batch=None,
+                    chunk=None):
     """Expert tiling on the GPU through the C ABI: heddle_price_tiled (with
     the tiling planes) and heddle_topk, or heddle_price_topk with ``fused``;
     ``batch`` splits the candidates into consecutive calls."""
@@ -146,6 +151,8 @@ def price_tiled_gpu(h, w_cluster, w_model, cands, expert_state, expert_param, k=
         h.heddle_load_cluster(ctx, w_cluster)
         h.heddle_load_model(ctx, w_model)
         h.heddle_load_experts(ctx, expert_state, expert_param)
+        if chunk is not None:
+            h.heddle_set_chunk(ctx, chunk)
         n = int(cands["S"].shape[0])
         dc = h.cands_to_device(cands)
         res = h.alloc_results(n, bounds=False)
