@@ -37,7 +37,9 @@ WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 10
                  "work streams, S<=32, "
                  "TP in {1,2,4,8}, M=256, global top-16")
 # Algorithmic integer work per counted unit, in 32-bit lane operations.
-# General search, unit = one interval check: stage cost P[j]-P[i]+c against
+# General search, unit = one interval check (as the warp-per-entry kernel
+# performs them: whole 32-position words per round, so it counts the
+# positions a serial probe would skip as well): stage cost P[j]-P[i]+c against
 # B (int64 subtract, add, compare) and stage memory (S[j]-S[i]) +
 # f*(A[j]-A[i]) against the capacity (two int64 subtracts, one multiply by a
 # 32-bit count, one add, one compare): 8 int64 ops = 16.
@@ -53,7 +55,7 @@ WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 10
 # of two 64x64->128-bit products (20): 36.  Together 65.
 OPS_PER_UNIT = {1: 16, 2: 65}
 SEARCH_NAMES = {1: "general interval search", 2: "equal-layer closed form"}
-SEARCH_KERNELS = {1: "search_kernel (general interval search)",
+SEARCH_KERNELS = {1: "wsearch_kernel (general threshold search, one warp per entry)",
                   2: "eq_search_kernel (equal-layer closed form)"}
 SMS, LANES_PER_SM = 152, 128  # 4 SM sub-partitions x 32 lanes issue per clock
 
