@@ -16,35 +16,35 @@
 // node, else the slowest NIC.
 //
 // Two kernels: a one-CTA table build (after the main cost tables), and the
-// tiled search over the screen's worklist, one thread per entry with the
+// tiled search over the screen's worklist, one warp per entry with the
 // tiled image in shared memory:
 //   stage time     t_s(i, j) = min over allowed tilings whose memory fits of
 //                  P_tiling[j] - P_tiling[i] + c_s (the earliest slot on
 //                  ties); monotone under interval inclusion
-//   PartitionLayers  threshold search on B with an exact probe: backward
-//                  sets C_s of feasible stage-s starts (the smallest
-//                  successor in C_{s+1} dominates), snapping the bracket to
-//                  the largest accepted / smallest rejected stage time;
-//                  the canonical split walks the sets at B* taking the
-//                  smallest boundary each time
-//   re-selection   per stage and EDP exponent m, the fastest fitting tiling
-//                  with EDP exponent <= m; g grows with d, so for a bound Y
-//                  on the gradient term each stage's admissible tilings are
-//                  such a prefix; T(Y) is evaluated for every Y among the
-//                  stages' gradient terms of fitting tilings and the
-//                  smallest T wins (the smaller Y on ties).
+//   PartitionLayers  the exact threshold search of the general search, its
+//                  probe (heddle_wprobe.cuh) judging 32 positions per round
+//                  with this stage time; the canonical split from the sets
+//                  at B*
+//   re-selection   one lane per stage keeps, per EDP exponent m, the
+//                  fastest fitting tiling with EDP exponent <= m and the
+//                  gradient term of m; g grows with d, so for a bound Y on
+//                  the gradient term each stage's admissible tilings are
+//                  such a prefix; T(Y) (warp reductions) is evaluated for
+//                  every Y among the stages' gradient terms of fitting
+//                  tilings and the smallest T wins (the smaller Y on ties).
 
 #include <algorithm>
 
 #include "heddle_tiled.cuh"
+#include "heddle_wprobe.cuh"
 
 namespace hd {
 namespace {
 
 constexpr int kTabThreads = 256;
 constexpr int64_t kTableLimit = (int64_t)1 << 40;
-constexpr int kTBlock = 128;
-constexpr int kSetWords = 8;  // 256-bit position sets (L <= 255)
+constexpr int kTBlock = 256;
+constexpr int kTWarps = kTBlock / 32;
 constexpr int kMaxIters = 256;
 
 // Nearest integer of v >= 0, halves away from zero (v - trunc(v) is exact
@@ -212,145 +212,68 @@ struct TTabs {
     const int64_t* p2p;
     const int64_t* mem;
     const int64_t* inter;
-    const int64_t* intra;
     const int32_t* maxn;
+    const int64_t* intra;
     const uint8_t* code;
     int L;
 };
 
 // One stage's constants.
-struct TStage {
+struct TLane {
     int g, j;
-    int64_t c;     // P2P to the next stage
-    int64_t cap;   // memory per GPU x devices
-    int64_t f;     // in-flight micro-batches
+    int64_t c;    // P2P to the next stage
+    int64_t cap;  // memory per GPU x devices
+    int64_t f;    // in-flight micro-batches
 };
 
-__device__ __forceinline__ TStage tstage(const TTabs& t, const uint8_t* codes, int s, int S, int M) {
-    TStage st;
-    const int b = codes[s];
-    st.g = b & 7;
-    st.j = (b >> 3) & 3;
-    st.cap = t.mem[st.g] << st.j;
-    st.f = min(S - s, M);
-    st.c = 0;
-    if (s + 1 < S) {
-        const int bn = codes[s + 1];
-        const int h = bn & 7, jn = (bn >> 3) & 3;
-        const int same = (st.g == h) && ((1 << st.j) + (1 << jn) <= t.maxn[st.g]);
-        st.c = t.p2p[(st.g * 8 + h) * 2 + same];
-    }
-    return st;
-}
-
 // Memory of layers [i, e) with EDP exponent ld fits?
-__device__ __forceinline__ bool tfits(const TTabs& t, const TStage& st, int i, int e, int ld) {
+__device__ __forceinline__ bool tfits(const TTabs& t, const TLane& st, int i, int e, int ld) {
     const longlong2 a = t.SA[i], b = t.SA[e];
     const int64_t mem = (b.x - a.x) + (((int64_t)1 << ld) - 1) * (t.ES[e] - t.ES[i]) + st.f * (b.y - a.y);
     return mem <= st.cap;
 }
 
-// Fastest fitting tiling of layers [i, e) on stage st (kInf if none).
-__device__ int64_t ttime(const TTabs& t, const TStage& st, int i, int e) {
-    const int base = tile_base(st.j), cnt = (st.j + 1) * (st.j + 2) / 2;
-    int64_t best = kInf;
-    for (int o = 0; o < cnt; ++o) {
-        const int slot = base + o;
-        const uint8_t cd = t.code[st.g * kTileSlots + slot];
-        if ((cd & 0xc0) != 0x80) continue;  // not allowed, or dominated
-        if (!tfits(t, st, i, e, (cd >> 4) & 3)) continue;
-        const int64_t* P = t.Pt + (size_t)(st.g * kTileSlots + slot) * (t.L + 1);
-        best = min(best, P[e] - P[i] + st.c);
+// The interval test of the tiled search: the fastest allowed, undominated
+// tiling whose memory fits (2 if none fits).
+struct TiledJudge {
+    typedef TLane Stage;
+    const TTabs& t;
+    TLane mine;  // the stage this lane holds
+    __device__ TLane stage(int s) const {
+        TLane r;
+        r.g = __shfl_sync(wp::kFull, mine.g, s);
+        r.j = __shfl_sync(wp::kFull, mine.j, s);
+        r.c = __shfl_sync(wp::kFull, mine.c, s);
+        r.cap = __shfl_sync(wp::kFull, mine.cap, s);
+        r.f = __shfl_sync(wp::kFull, mine.f, s);
+        return r;
     }
-    return best;
-}
-
-__device__ __forceinline__ bool has(const uint32_t* C, int i) { return (C[i >> 5] >> (i & 31)) & 1u; }
-
-// smallest set position in [i, hi], -1 if none
-__device__ int next_in(const uint32_t* C, int i, int hi) {
-    if (i > hi) return -1;
-    int w = i >> 5;
-    uint32_t m = C[w] & (0xffffffffu << (i & 31));
-    while (m == 0) {
-        if (++w > (hi >> 5)) return -1;
-        m = C[w];
-    }
-    const int x = (w << 5) + __ffs(m) - 1;
-    return x <= hi ? x : -1;
-}
-
-// largest set position in [lo, i], -1 if none
-__device__ int prev_in(const uint32_t* C, int i, int lo) {
-    if (i < lo) return -1;
-    int w = i >> 5;
-    uint32_t m = C[w] & (0xffffffffu >> (31 - (i & 31)));
-    while (m == 0) {
-        if (--w < (lo >> 5)) return -1;
-        m = C[w];
-    }
-    const int x = (w << 5) + 31 - __clz(m);
-    return x >= lo ? x : -1;
-}
-
-// Exact probe of bound B: C[s] = feasible starts of stage s (C[S] = {L}).
-// hi / lo: largest accepted / smallest rejected stage time judged.
-__device__ bool tprobe(const TTabs& t, const uint8_t* codes, int S, int M, int64_t B, int64_t& hi, int64_t& lo,
-                       uint32_t (*C)[kSetWords]) {
-    const int L = t.L;
-    hi = -1;
-    lo = kInf;
-    for (int w = 0; w < kSetWords; ++w) C[S][w] = 0;
-    C[S][L >> 5] = 1u << (L & 31);
-    for (int s = S - 1; s >= 1; --s) {
-        for (int w = 0; w < kSetWords; ++w) C[s][w] = 0;
-        const TStage st = tstage(t, codes, s, S, M);
-        const int imax = L - (S - s);
-        int succ = next_in(C[s + 1], imax + 1, L);
-        bool any = false;
-        int i = imax;
-        while (i >= s) {
-            if (has(C[s + 1], i + 1)) succ = i + 1;
-            // kInf: no successor, or no tiling of [i, succ) fits memory
-            const int64_t v = succ < 0 ? kInf : ttime(t, st, i, succ);
-            if (v != kInf && v <= B) {
-                C[s][i >> 5] |= 1u << (i & 31);
-                hi = max(hi, v);
-                any = true;
-                --i;
-                continue;
-            }
-            if (v != kInf) lo = min(lo, v);
-            // [i, succ) is rejected (too slow or out of memory), and so is
-            // every longer [i', succ): resume below the next smaller
-            // successor
-            const int j2 = prev_in(C[s + 1], i, s + 1);
-            if (j2 < 0) break;
-            succ = j2;
-            i = j2 - 1;
+    __device__ __forceinline__ int eval(const TLane& st, int i, int e, int64_t B, int64_t* cost) const {
+        const int base = tile_base(st.j), cnt = (st.j + 1) * (st.j + 2) / 2;
+        int64_t best = kInf;
+        for (int o = 0; o < cnt; ++o) {
+            const uint8_t cd = t.code[st.g * kTileSlots + base + o];
+            if ((cd & 0xc0) != 0x80) continue;  // not allowed, or dominated
+            if (!tfits(t, st, i, e, (cd >> 4) & 3)) continue;
+            const int64_t* P = t.Pt + (size_t)(st.g * kTileSlots + base + o) * (t.L + 1);
+            best = min(best, P[e] - P[i] + st.c);
         }
-        if (!any) return false;
+        if (best == kInf) return 2;
+        *cost = best;
+        return best <= B ? 0 : 1;
     }
-    const int succ0 = S == 1 ? L : next_in(C[1], 1, L);
-    if (succ0 < 0) return false;
-    const int64_t v = ttime(t, tstage(t, codes, 0, S, M), 0, succ0);
-    if (v == kInf) return false;
-    if (v <= B) {
-        hi = max(hi, v);
-        return true;
-    }
-    lo = min(lo, v);
-    return false;
+};
+
+// element k of a 4-entry register array (k in [0, 3])
+template <class T>
+__device__ __forceinline__ T pick4(const T (&v)[4], int k) {
+    return k == 0 ? v[0] : k == 1 ? v[1] : k == 2 ? v[2] : v[3];
 }
 
 __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, TiledArgs ta) {
-    extern __shared__ __align__(16) unsigned char smem[];
-    {
-        const uint4* src = reinterpret_cast<const uint4*>(ta.timg);
-        uint4* dst = reinterpret_cast<uint4*>(smem);
-        for (uint32_t i = threadIdx.x; i < ta.tl.bytes / 16; i += blockDim.x) dst[i] = src[i];
-    }
-    __syncthreads();
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ uint64_t bar;
+    if (!wp::load_image(smem, ta.timg, ta.tl.bytes, &bar, a.err)) return;
     const TiledLayout& y = ta.tl;
     TTabs t;
     t.Pt = reinterpret_cast<const int64_t*>(smem + y.offPt);
@@ -366,47 +289,65 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
     t.code = smem + y.offCode;
     t.L = y.L;
     const int L = y.L;
-
-    uint32_t C[kMaxStages + 1][kSetWords];
-    uint8_t codes[kMaxStages];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    wp::WarpArea& wa = reinterpret_cast<wp::WarpArea*>(smem + ((y.bytes + 127u) & ~127u))[warp];
+    unsigned long long checks = 0;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < count;
-         p += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t nwarps = (int64_t)gridDim.x * kTWarps;
+    for (int64_t p = (int64_t)blockIdx.x * kTWarps + warp; p < count; p += nwarps) {
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
         const int M = a.wl_M[p];
         const int64_t n = a.wl_n[p];
-        {
-            const uint4* row = reinterpret_cast<const uint4*>(a.wl_code + p * kMaxStages);
-            const uint4 v0 = row[0], v1 = row[1];
-            const uint32_t w[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-            for (int s = 0; s < kMaxStages; ++s) codes[s] = (uint8_t)(w[s >> 2] >> ((s & 3) * 8));
+        const bool live = lane < S;
+        // this lane's stage (lane < S)
+        const int code = a.wl_code[p * kMaxStages + lane];
+        const int nxt = __shfl_down_sync(wp::kFull, code, 1);
+        TLane mine;
+        mine.g = code & 7;
+        mine.j = (code >> 3) & 3;
+        mine.cap = t.mem[mine.g] << mine.j;
+        mine.f = live ? min(S - lane, M) : 0;
+        mine.c = 0;
+        if (lane + 1 < S) {
+            const int h = nxt & 7, jn = (nxt >> 3) & 3;
+            const int same = (mine.g == h) && ((1 << mine.j) + (1 << jn) <= t.maxn[mine.g]);
+            mine.c = t.p2p[(mine.g * 8 + h) * 2 + same];
         }
+        const TiledJudge judge{t, mine};
         // memory-only probe: OOM, else a feasible upper bound
         int64_t hi, lo;
-        if (!tprobe(t, codes, S, M, kInf, hi, lo, C)) {
-            a.T[c] = -1;
-            a.B[c] = -1;
-            a.ndp[c] = (uint16_t)n;
-            a.status[c] = HEDDLE_CAND_OOM;
-            if (a.bounds)
-                for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = 0;
-            a.wl_T[p] = -1;
+        if (!wp::probe(judge, S, L, kInf, wa, hi, lo, checks)) {
+            if (lane == 0) {
+                a.T[c] = -1;
+                a.B[c] = -1;
+                a.ndp[c] = (uint16_t)n;
+                a.status[c] = HEDDLE_CAND_OOM;
+                a.wl_T[p] = -1;
+            }
+            if (a.bounds) {
+                a.bounds[(int64_t)(lane + 1) * a.bstride + c] = 0;
+                if (lane == 0) a.bounds[c] = 0;
+            }
             continue;
         }
         // first guess: the balanced bound with every stage at its fastest
         // tiling over all layers, then gallop until the bracket closes
         float inv = 0.f, cw = 0.f;
-        for (int s = 0; s < S; ++s) {
-            const TStage st = tstage(t, codes, s, S, M);
-            const int base = tile_base(st.j), cnt = (st.j + 1) * (st.j + 2) / 2;
+        if (live) {
+            const int base = tile_base(mine.j), cnt = (mine.j + 1) * (mine.j + 2) / 2;
             int64_t all = kInf;
             for (int o = 0; o < cnt; ++o)
-                if ((t.code[st.g * kTileSlots + base + o] & 0xc0) == 0x80)
-                    all = min(all, t.Pt[(size_t)(st.g * kTileSlots + base + o) * (L + 1) + L]);
+                if ((t.code[mine.g * kTileSlots + base + o] & 0xc0) == 0x80)
+                    all = min(all, t.Pt[(size_t)(mine.g * kTileSlots + base + o) * (L + 1) + L]);
             const float tot = u64_to_float((uint64_t)all) + 1.0f;
-            inv += 1.0f / tot;
-            cw += u64_to_float((uint64_t)st.c) / tot;
+            inv = 1.0f / tot;
+            cw = u64_to_float((uint64_t)mine.c) / tot;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            inv += __shfl_xor_sync(wp::kFull, inv, o);
+            cw += __shfl_xor_sync(wp::kFull, cw, o);
         }
         int64_t Bhi = hi, Blo = 0;
         bool lo_known = false, hi_known = false;
@@ -415,7 +356,7 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
         int it = 0;
         while (Blo < Bhi) {
             B = min(max(B, Blo), Bhi - 1);
-            if (tprobe(t, codes, S, M, B, hi, lo, C)) {
+            if (wp::probe(judge, S, L, B, wa, hi, lo, checks)) {
                 Bhi = hi;
                 hi_known = true;
             } else {
@@ -433,112 +374,107 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
                 B = Blo + (Bhi - Blo) / 2;
             }
             if (++it > kMaxIters) {
-                atomicOr(a.err, kErrSearchBound);
+                if (lane == 0) atomicOr(a.err, kErrSearchBound);
                 break;
             }
         }
         const int64_t Bstar = Bhi;
-        if (!tprobe(t, codes, S, M, Bstar, hi, lo, C)) atomicOr(a.err, kErrInternal);
-        uint8_t bnd[kMaxStages + 1];
-        bnd[0] = 0;
-        for (int s = 0; s + 1 < S; ++s) {
-            const int x = next_in(C[s + 1], bnd[s] + 1, L);
-            if (x < 0) atomicOr(a.err, kErrInternal);
-            bnd[s + 1] = (uint8_t)max(x, 0);
-        }
-        bnd[S] = (uint8_t)L;
+        if (!wp::probe(judge, S, L, Bstar, wa, hi, lo, checks) && lane == 0) atomicOr(a.err, kErrInternal);
+        if (!wp::walk(wa, S, L) && lane == 0) atomicOr(a.err, kErrInternal);
 
-        // ---- re-selection on the split: per stage and EDP exponent m the
-        //      fastest fitting tiling with EDP exponent <= m, and the
-        //      gradient term of each EDP exponent
-        int64_t bt[kMaxStages][4], gg[kMaxStages][4];
-        uint8_t bc[kMaxStages][4], bl[kMaxStages][4], hd_[kMaxStages];
-        for (int s = 0; s < S; ++s) {
-            const TStage st = tstage(t, codes, s, S, M);
-            const int i0 = bnd[s], i1 = bnd[s + 1];
+        // ---- re-selection on the split, one lane per stage: per EDP
+        //      exponent m the fastest fitting tiling with EDP exponent <= m
+        //      (bt, its code bc and exponent bl) and the gradient term gg
+        int64_t bt[4] = {kInf, kInf, kInf, kInf}, gg[4] = {0, 0, 0, 0};
+        int bc[4] = {0, 0, 0, 0}, bl[4] = {0, 0, 0, 0};
+        int hasld = 0, a1 = 0;
+        if (live) {
+            const int i0 = wa.A[lane], i1 = wa.A[lane + 1];
+            a1 = i1;
             const int64_t Ge = t.PE[i1] - t.PE[i0];
             const int64_t Gd = (t.PB[i1] - t.PB[i0]) - Ge;
-            const int64_t bw = (n == 1 && (1 << st.j) <= t.maxn[st.g]) ? t.intra[st.g] : t.inter[st.g];
-            const int base = tile_base(st.j);
+            const int64_t bw = (n == 1 && (1 << mine.j) <= t.maxn[mine.g]) ? t.intra[mine.g] : t.inter[mine.g];
+            const int base = tile_base(mine.j);
             int64_t best = kInf;
-            uint8_t bcode = 0, bld = 0, hasld = 0;
-            int o = 0;
-            for (int m = 0; m <= st.j; ++m) {
+            int bcode = 0, bld = 0, o = 0;
+#pragma unroll
+            for (int m = 0; m < 4; ++m) {
+                if (m > mine.j) break;
                 const u128 vol = (u128)(n - 1) * (u128)Gd + (u128)((n << m) - 1) * (u128)Ge;
                 int64_t gv = 0;
                 if (vol != 0) {
-                    bool ok = true;
-                    gv = (int64_t)ceil_div_u128((u128)2 * vol * 1000000000u, (uint64_t)(n << st.j) * (uint64_t)bw, &ok);
-                    if (!ok) atomicOr(a.err, kErrInternal);
+                    bool okd = true;
+                    gv = (int64_t)ceil_div_u128((u128)2 * vol * 1000000000u, (uint64_t)(n << mine.j) * (uint64_t)bw,
+                                                &okd);
+                    if (!okd) atomicOr(a.err, kErrInternal);
                 }
-                gg[s][m] = gv;
+                gg[m] = gv;
                 // the slots of EDP exponent m: ETP exponent 0 .. j - m
-                for (int lt = 0; lt <= st.j - m; ++lt, ++o) {
-                    const uint8_t cd = t.code[st.g * kTileSlots + base + o];
-                    if ((cd & 0xc0) != 0x80 || !tfits(t, st, i0, i1, m)) continue;
-                    hasld |= (uint8_t)(1 << m);
-                    const int64_t* P = t.Pt + (size_t)(st.g * kTileSlots + base + o) * (L + 1);
-                    const int64_t v = P[i1] - P[i0] + st.c;
+                for (int lt = 0; lt <= mine.j - m; ++lt, ++o) {
+                    const uint8_t cd = t.code[mine.g * kTileSlots + base + o];
+                    if ((cd & 0xc0) != 0x80 || !tfits(t, mine, i0, i1, m)) continue;
+                    hasld |= 1 << m;
+                    const int64_t* P = t.Pt + (size_t)(mine.g * kTileSlots + base + o) * (L + 1);
+                    const int64_t v = P[i1] - P[i0] + mine.c;
                     if (v < best) {
                         best = v;
                         bcode = cd & 15;
-                        bld = (uint8_t)m;
+                        bld = m;
                     }
                 }
-                bt[s][m] = best;
-                bc[s][m] = bcode;
-                bl[s][m] = bld;
+                bt[m] = best;
+                bc[m] = bcode;
+                bl[m] = bld;
             }
-            hd_[s] = hasld;
         }
         int64_t bestT = kInf, bestY = 0, bestB = 0;
-        int ys_best = -1;
-        uint8_t pick[kMaxStages];
+        int mycode = 0;
+        bool found = false;
         for (int ys = 0; ys < S; ++ys) {
-            const int jy = (codes[ys] >> 3) & 3;
-            for (int my = 0; my <= jy; ++my) {
-                if (!((hd_[ys] >> my) & 1)) continue;
-                const int64_t Y = gg[ys][my];
-                int64_t tm = 0, ts = 0, gm = 0;
-                bool all = true;
-                for (int s = 0; s < S && all; ++s) {
-                    const int js = (codes[s] >> 3) & 3;
-                    int mm = -1;
-                    while (mm + 1 <= js && gg[s][mm + 1] <= Y) ++mm;
-                    if (mm < 0 || bt[s][mm] == kInf) {
-                        all = false;
-                        break;
-                    }
-                    tm = max(tm, bt[s][mm]);
-                    ts += bt[s][mm];
-                    gm = max(gm, gg[s][bl[s][mm]]);
-                    pick[s] = (uint8_t)mm;
-                }
-                if (!all) continue;
-                const int64_t T = (int64_t)(M - 1) * tm + ts + gm;
-                if (T < bestT || (T == bestT && Y < bestY)) {
+            const int hy = __shfl_sync(wp::kFull, hasld, ys);
+#pragma unroll
+            for (int my = 0; my < 4; ++my) {
+                const int64_t Y = __shfl_sync(wp::kFull, gg[my], ys);
+                if (!((hy >> my) & 1)) continue;
+                // each stage: its fastest fitting tiling with g <= Y (the
+                // admissible EDP exponents are a prefix: g grows with d)
+                int mm = -1;
+#pragma unroll
+                for (int m = 0; m < 4; ++m)
+                    if (m <= mine.j && gg[m] <= Y) mm = m;
+                const int64_t tv = mm >= 0 ? pick4(bt, mm) : kInf;
+                const bool bad = live && tv == kInf;
+                if (__any_sync(wp::kFull, bad)) continue;
+                const int64_t gsel = live ? pick4(gg, pick4(bl, mm)) : 0;
+                const int64_t tm = wp::wmax64(live ? tv : 0), tsum = wp::wsum64(live ? tv : 0);
+                const int64_t gm = wp::wmax64(gsel);
+                const int64_t T = (int64_t)(M - 1) * tm + tsum + gm;
+                if (!found || T < bestT || (T == bestT && Y < bestY)) {
+                    found = true;
                     bestT = T;
                     bestY = Y;
                     bestB = tm;
-                    ys_best = ys;
-                    if (ta.tiling)
-                        for (int s = 0; s < S; ++s) ta.tiling[(int64_t)s * ta.tstride + c] = bc[s][pick[s]];
+                    mycode = live ? pick4(bc, mm) : 0;
                 }
             }
         }
-        if (ys_best < 0) {
-            atomicOr(a.err, kErrInternal);
-            bestT = -1;
+        if (lane == 0) {
+            if (!found) atomicOr(a.err, kErrInternal);
+            a.T[c] = found ? bestT : -1;
+            a.wl_T[p] = found ? bestT : -1;
+            a.wl_nM[p] = (uint32_t)n * (uint32_t)M;
+            a.B[c] = bestB;
+            a.ndp[c] = (uint16_t)n;
+            a.status[c] = HEDDLE_CAND_OK;
         }
-        a.T[c] = bestT;
-        a.wl_T[p] = bestT;
-        a.wl_nM[p] = (uint32_t)n * (uint32_t)M;
-        a.B[c] = bestB;
-        a.ndp[c] = (uint16_t)n;
-        a.status[c] = HEDDLE_CAND_OK;
-        if (a.bounds)
-            for (int s = 0; s <= kMaxStages; ++s) a.bounds[(int64_t)s * a.bstride + c] = s <= S ? bnd[s] : 0;
+        if (ta.tiling && live) ta.tiling[(int64_t)lane * ta.tstride + c] = (uint8_t)mycode;
+        if (a.bounds) {
+            a.bounds[(int64_t)(lane + 1) * a.bstride + c] = live ? (uint8_t)a1 : 0;
+            if (lane == 0) a.bounds[c] = 0;
+        }
+        __syncwarp();  // wa is reused by the next entry
     }
+    (void)checks;
 }
 
 }  // namespace
@@ -549,15 +485,16 @@ cudaError_t launch_tiled_tables(const TiledTableArgs& a, cudaStream_t st) {
 }
 
 cudaError_t launch_tiled_search(const PriceArgs& a, const TiledArgs& t, int num_sms, cudaStream_t st) {
-    const size_t smem = t.tl.bytes;
+    const size_t smem = ((t.tl.bytes + 127u) & ~127u) + sizeof(wp::WarpArea) * kTWarps;
     cudaError_t e = cudaFuncSetAttribute(tiled_search_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int per_sm = 0;
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, tiled_search_kernel, kTBlock, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    // the worklist length is only known on the device: size for the batch
-    const int64_t need = (a.n + kTBlock - 1) / kTBlock;
+    // the worklist length is only known on the device: one warp per entry,
+    // at most one wave
+    const int64_t need = (a.n + kTWarps - 1) / kTWarps;
     const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
     tiled_search_kernel<<<grid, kTBlock, smem, st>>>(a, t);
     return cudaGetLastError();

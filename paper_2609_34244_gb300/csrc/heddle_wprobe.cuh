@@ -1,0 +1,243 @@
+// heddle_wprobe.cuh -- the exact PartitionLayers probe run by one warp per
+// worklist entry, shared by the general search and the expert-tiling search.
+//
+// probe(B) decides whether a split with every stage time <= B and every
+// stage within memory exists:
+//   forward:  U_0 = 0, U_{s+1} = the furthest end stage s reaches from U_s
+//             (an upper bound on every feasible boundary a_{s+1});
+//   backward: C_S = {L}; C_s = { i in [s, U_s] : the smallest j in C_{s+1}
+//             above i gives a stage [i, j) that fits }; feasible iff stage 0
+//             fits [0, min C_1).
+// Stage time and memory grow with the interval, so the smallest successor
+// dominates and C_s is exactly the set of feasible stage-s starts below U_s.
+// The probe also returns the largest accepted and the smallest rejected
+// stage time: every B' in [hi, B] (feasible) or [B, lo) (infeasible) takes
+// the same decisions, so a search snaps its bracket to them and ends on B*;
+// the sets at B* give the canonical (lexicographically smallest) split.
+//
+// The 32 lanes judge 32 positions at once: a stage's forward reach is the
+// first rejection among 32 consecutive ends, and a backward set is built
+// one 32-bit word per round -- lane l judges start 32 w + l against its
+// smallest successor (a bit scan of the successor set) and the ballot is
+// the word.  A judge type J supplies the stages and the interval test:
+//   typename J::Stage J::stage(int s) const   -- every lane calls it
+//   int J::eval(const Stage&, int i, int j, int64_t B, int64_t* cost) const
+//       -- 0 fits (cost <= B), 1 too slow, 2 out of memory.
+
+#pragma once
+
+#include "heddle_internal.cuh"
+
+namespace hd {
+namespace wp {
+
+constexpr int kSetWords = 8;  // 256-bit position sets (L <= 255)
+constexpr unsigned kFull = 0xffffffffu;
+constexpr long long kWaitSpins = 1 << 22;
+
+// per-warp shared state: sets C[0..32], forward bounds U, the split A
+struct WarpArea {
+    uint32_t C[kMaxStages + 1][kSetWords];
+    uint8_t U[kMaxStages + 1];
+    uint8_t A[kMaxStages + 1];
+    uint8_t pad[30];
+};
+
+__device__ __forceinline__ uint32_t saddr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+// A table image into shared memory: one thread arms an mbarrier with the
+// byte count (a multiple of 16) and issues bulk asynchronous copies; all
+// wait on phase 0 with a bounded spin.  False (and the error flag) if the
+// wait gave up.
+__device__ inline bool load_image(unsigned char* dst, const unsigned char* src, uint32_t bytes, uint64_t* bar,
+                                  uint32_t* err) {
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(saddr(bar)));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(saddr(bar)), "r"(bytes)
+                     : "memory");
+        for (uint32_t o = 0; o < bytes; o += 32768) {
+            const uint32_t nb = bytes - o < 32768 ? bytes - o : 32768;
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    saddr(dst + o)),
+                "l"(src + o), "r"(nb), "r"(saddr(bar))
+                : "memory");
+        }
+    }
+    __syncthreads();
+    uint32_t done = 0;
+    for (long long spin = 0; spin < kWaitSpins; ++spin) {
+        asm volatile(
+            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0; selp.u32 %0, 1, 0, p; }"
+            : "=r"(done)
+            : "r"(saddr(bar))
+            : "memory");
+        if (done) break;
+    }
+    const int all = __syncthreads_and(done != 0);
+    if (!all && threadIdx.x == 0) atomicOr(err, kErrStageWait);
+    return all != 0;
+}
+
+__device__ __forceinline__ int64_t wmax64(int64_t v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = max(v, (int64_t)__shfl_xor_sync(kFull, v, o));
+    return v;
+}
+__device__ __forceinline__ int64_t wmin64(int64_t v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = min(v, (int64_t)__shfl_xor_sync(kFull, v, o));
+    return v;
+}
+__device__ __forceinline__ int64_t wsum64(int64_t v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+    return v;
+}
+
+// smallest set position of C in (i, L], -1 if none (warp-uniform inputs)
+__device__ __forceinline__ int next_above(const uint32_t* C, int i, int L) {
+    int w = (i + 1) >> 5;
+    if (w > (L >> 5)) return -1;
+    uint32_t m = C[w] & (0xffffffffu << ((i + 1) & 31));
+    while (m == 0) {
+        if (++w > (L >> 5)) return -1;
+        m = C[w];
+    }
+    return (w << 5) + __ffs(m) - 1;
+}
+
+// Exact probe of bound B by one warp (all lanes call it; uniform result).
+// The sets land in wa; hi / lo are the snap values; checks counts the
+// interval judgements of this lane.
+template <class J>
+__device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int64_t& hi_out, int64_t& lo_out,
+                      unsigned long long& checks) {
+    const int lane = threadIdx.x & 31;
+    int64_t hi = -1, lo = kInf;
+    bool ok = true;
+    // forward upper bounds on the boundaries
+    int u = 0;
+    if (lane == 0) wa.U[0] = 0;
+    for (int s = 0; s + 1 < S && ok; ++s) {
+        const typename J::Stage st = judge.stage(s);
+        const int lim = L - (S - 1 - s);
+        int reach = u;  // furthest accepted end (u: none yet)
+        for (int base = u + 1; base <= lim; base += 32) {
+            const int j = base + lane;
+            int r = 1;  // beyond lim: treated as a rejection
+            int64_t v = 0;
+            if (j <= lim) {
+                r = judge.eval(st, u, j, B, &v);
+                ++checks;
+                if (r == 0) hi = max(hi, v);
+                else if (r == 1) lo = min(lo, v);
+            }
+            const unsigned rej = __ballot_sync(kFull, r != 0);
+            if (rej) {
+                reach = base + __ffs(rej) - 2;
+                break;
+            }
+            reach = base + 31;
+        }
+        if (reach < s + 1) ok = false;
+        u = reach;
+        if (lane == 0) wa.U[s + 1] = (uint8_t)reach;
+    }
+    __syncwarp();
+    // backward feasible-start sets: C_S = {L}, then stages S-1 .. 1
+    if (ok) {
+        if (lane < kSetWords) wa.C[S][lane] = lane == (L >> 5) ? 1u << (L & 31) : 0u;
+        __syncwarp();
+        int nmax = L;
+        for (int s = S - 1; s >= 1 && ok; --s) {
+            const uint32_t* Cn = wa.C[s + 1];
+            if (lane < kSetWords) wa.C[s][lane] = 0;
+            __syncwarp();
+            const int top = min((int)wa.U[s], nmax - 1);
+            if (top < s) {
+                ok = false;
+                break;
+            }
+            const typename J::Stage st = judge.stage(s);
+            int any = 0, newmax = -1;
+            for (int w = top >> 5; w >= (s >> 5); --w) {
+                const int i = (w << 5) + lane;
+                // smallest successor above i: in this word, else beyond it
+                const uint32_t cw = Cn[w];
+                const uint32_t above = lane == 31 ? 0u : (cw >> (lane + 1)) << (lane + 1);
+                int beyond = -1;
+                for (int w2 = w + 1; w2 <= (L >> 5); ++w2)
+                    if (Cn[w2]) {
+                        beyond = (w2 << 5) + __ffs(Cn[w2]) - 1;
+                        break;
+                    }
+                const int succ = above ? (w << 5) + __ffs(above) - 1 : beyond;
+                int r = 3;
+                int64_t v = 0;
+                if (i >= s && i <= top && succ >= 0) {
+                    r = judge.eval(st, i, succ, B, &v);
+                    ++checks;
+                    if (r == 0) hi = max(hi, v);
+                    else if (r == 1) lo = min(lo, v);
+                }
+                const unsigned acc = __ballot_sync(kFull, r == 0);
+                if (lane == 0) wa.C[s][w] = acc;
+                if (acc) {
+                    any = 1;
+                    if (newmax < 0) newmax = (w << 5) + 31 - __clz(acc);
+                }
+            }
+            __syncwarp();
+            if (!any) ok = false;
+            nmax = newmax;
+        }
+    }
+    bool feasible = false;
+    if (ok) {
+        const int succ0 = S == 1 ? L : next_above(wa.C[1], 0, L);
+        const typename J::Stage st0 = judge.stage(0);
+        if (succ0 >= 0 && lane == 0) {
+            int64_t v = 0;
+            const int r = judge.eval(st0, 0, succ0, B, &v);
+            ++checks;
+            if (r == 0) {
+                hi = max(hi, v);
+                feasible = true;
+            } else if (r == 1) {
+                lo = min(lo, v);
+            }
+        }
+        feasible = __shfl_sync(kFull, feasible, 0);
+    }
+    hi_out = wmax64(hi);
+    lo_out = wmin64(lo);
+    return feasible;
+}
+
+// The canonical split from the sets of a feasible probe at B*, by lane 0
+// into wa.A (a_{s+1} = the smallest element of C_{s+1} above a_s); false if
+// a set ran out (never expected after a feasible probe).
+__device__ inline bool walk(WarpArea& wa, int S, int L) {
+    bool ok = true;
+    if ((threadIdx.x & 31) == 0) {
+        int at = 0;
+        wa.A[0] = 0;
+        for (int s = 0; s + 1 < S; ++s) {
+            const int x = next_above(wa.C[s + 1], at, L);
+            if (x < 0) ok = false;
+            at = max(x, at + 1);
+            wa.A[s + 1] = (uint8_t)at;
+        }
+        wa.A[S] = (uint8_t)L;
+    }
+    __syncwarp();
+    return __shfl_sync(kFull, ok, 0);
+}
+
+}  // namespace wp
+}  // namespace hd

@@ -2,89 +2,29 @@
 // §5.2 memory validation, §5.3 iteration time) for models whose layers
 // differ, one warp per worklist entry.
 //
-// The search is the exact threshold search of the thread-per-entry kernel:
-// probe(B) decides whether a split with every stage time <= B and every
-// stage within memory exists,
-//   forward:  U_0 = 0, U_{s+1} = the furthest end stage s reaches from U_s
-//             (an upper bound on every feasible boundary a_{s+1});
-//   backward: C_S = {L}; C_s = { i in [s, U_s] : the smallest j in C_{s+1}
-//             above i gives a stage [i, j) that fits }; feasible iff stage 0
-//             fits [0, min C_1);
-// the probe also returns the largest accepted and the smallest rejected
-// stage time, the bracket snaps to them, and the sets at B* give the
-// canonical (lexicographically smallest) split.
-//
-// Here the 32 lanes of a warp judge 32 positions at once: the forward reach
-// of a stage is the first rejection among 32 consecutive ends (stage time
-// and memory grow with the end), and a backward set is built one 32-bit
-// word per round -- lane l judges start 32 w + l against its smallest
-// successor (a bit scan in the successor set) and the ballot is the word.
-// Stage parameters come from the lane that holds the stage; the snap values
-// are warp reductions; Evaluate runs with one lane per stage.  The table
-// image is staged into shared memory with bulk asynchronous copies
-// (cp.async.bulk, completion on an mbarrier, bounded wait); each warp keeps
-// its sets and split in shared memory.
+// The exact threshold search: a memory-only probe decides OOM (unless the
+// screen already knows a split fits) and bounds B*; a balanced first guess
+// gallops until the bracket closes, each probe snapping it to the largest
+// accepted or the smallest rejected stage time; the sets of the probe at B*
+// give the canonical split.  The probe (heddle_wprobe.cuh) judges 32
+// positions per round with the interval test of this file: stage time
+// P[j] - P[i] + c and memory against k times the GPU memory.  Evaluate runs
+// one lane per stage: the stage times' maximum and sum, the stage with the
+// largest G / (k bw) by exact cross-multiplication, and one 128/64-bit
+// ceiling division for the gradient term.  The table image is staged into
+// shared memory with bulk asynchronous copies.
 
-#include <algorithm>
-
-#include "heddle_internal.cuh"
+#include "heddle_wprobe.cuh"
 
 namespace hd {
 namespace {
 
+using wp::kFull;
+using wp::WarpArea;
+
 constexpr int kWBlock = 256;
 constexpr int kWarps = kWBlock / 32;
-constexpr int kSetWords = 8;  // 256-bit position sets (L <= 255)
 constexpr int kMaxIters = 256;
-constexpr long long kWaitSpins = 1 << 22;
-constexpr unsigned kFull = 0xffffffffu;
-
-// per-warp shared state: sets C[0..32], forward bounds U, the split A
-struct WarpArea {
-    uint32_t C[kMaxStages + 1][kSetWords];
-    uint8_t U[kMaxStages + 1];
-    uint8_t A[kMaxStages + 1];
-    uint8_t pad[30];
-};
-
-__device__ __forceinline__ uint32_t saddr(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-// The table image into shared memory: one thread arms an mbarrier with the
-// byte count and issues the bulk copies; all wait on phase 0 with a bounded
-// spin.  False (and the error flag) if the wait gave up.
-__device__ bool load_image(unsigned char* dst, const unsigned char* src, uint32_t bytes, uint64_t* bar,
-                           uint32_t* err) {
-    if (threadIdx.x == 0) {
-        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(saddr(bar)));
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(saddr(bar)), "r"(bytes)
-                     : "memory");
-        for (uint32_t o = 0; o < bytes; o += 32768) {
-            const uint32_t nb = bytes - o < 32768 ? bytes - o : 32768;
-            asm volatile(
-                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                    saddr(dst + o)),
-                "l"(src + o), "r"(nb), "r"(saddr(bar))
-                : "memory");
-        }
-    }
-    __syncthreads();
-    uint32_t done = 0;
-    for (long long spin = 0; spin < kWaitSpins; ++spin) {
-        asm volatile(
-            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0; selp.u32 %0, 1, 0, p; }"
-            : "=r"(done)
-            : "r"(saddr(bar))
-            : "memory");
-        if (done) break;
-    }
-    const int all = __syncthreads_and(done != 0);
-    if (!all && threadIdx.x == 0) atomicOr(err, kErrStageWait);
-    return all != 0;
-}
 
 struct WTabs {
     const int64_t* P;
@@ -105,160 +45,34 @@ struct WStage {
     int64_t f;     // in-flight micro-batches
 };
 
-__device__ __forceinline__ WStage bcast(const WStage& mine, int s) {
-    WStage r;
-    r.row = __shfl_sync(kFull, mine.row, s);
-    r.c = __shfl_sync(kFull, mine.c, s);
-    r.capk = __shfl_sync(kFull, mine.capk, s);
-    r.f = __shfl_sync(kFull, mine.f, s);
-    return r;
-}
-
-// Interval [i, j) on stage st: 0 fits (cost <= B), 1 too slow, 2 out of
-// memory; the cost in *cost.
-__device__ __forceinline__ int wjudge(const WTabs& t, const WStage& st, int i, int j, int64_t B, int64_t* cost) {
-    const longlong2 si = t.SA[i], sj = t.SA[j];
-    if ((sj.x - si.x) + st.f * (sj.y - si.y) > st.capk) return 2;
-    const int64_t v = t.P[st.row + j] - t.P[st.row + i] + st.c;
-    *cost = v;
-    return v <= B ? 0 : 1;
-}
-
-__device__ __forceinline__ int64_t wmax64(int64_t v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = max(v, (int64_t)__shfl_xor_sync(kFull, v, o));
-    return v;
-}
-__device__ __forceinline__ int64_t wmin64(int64_t v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = min(v, (int64_t)__shfl_xor_sync(kFull, v, o));
-    return v;
-}
-
-// smallest set position of C in (i, L], -1 if none (warp-uniform inputs)
-__device__ __forceinline__ int next_above(const uint32_t* C, int i, int L) {
-    int w = (i + 1) >> 5;
-    if (w > (L >> 5)) return -1;
-    uint32_t m = C[w] & (0xffffffffu << ((i + 1) & 31));
-    while (m == 0) {
-        if (++w > (L >> 5)) return -1;
-        m = C[w];
+// The interval test of the general search: stage time P[j] - P[i] + c and
+// memory (S[j] - S[i]) + f (A[j] - A[i]) against k times the GPU memory.
+struct PlainJudge {
+    typedef WStage Stage;
+    const WTabs& t;
+    WStage mine;  // the stage this lane holds
+    __device__ WStage stage(int s) const {
+        WStage r;
+        r.row = __shfl_sync(kFull, mine.row, s);
+        r.c = __shfl_sync(kFull, mine.c, s);
+        r.capk = __shfl_sync(kFull, mine.capk, s);
+        r.f = __shfl_sync(kFull, mine.f, s);
+        return r;
     }
-    return (w << 5) + __ffs(m) - 1;
-}
-
-// Exact probe of bound B by one warp (all lanes, uniform result).  mine:
-// the stage this lane holds (lane < S).  The sets land in wa.
-__device__ bool wprobe(const WTabs& t, const WStage& mine, int S, int64_t B, WarpArea& wa, int64_t& hi_out,
-                       int64_t& lo_out, unsigned long long& checks) {
-    const int L = t.L;
-    const int lane = threadIdx.x & 31;
-    int64_t hi = -1, lo = kInf;
-    bool ok = true;
-    // forward upper bounds on the boundaries
-    int u = 0;
-    if (lane == 0) wa.U[0] = 0;
-    for (int s = 0; s + 1 < S && ok; ++s) {
-        const WStage st = bcast(mine, s);
-        const int lim = L - (S - 1 - s);
-        int reach = u;  // furthest accepted end (u: none yet)
-        for (int base = u + 1; base <= lim; base += 32) {
-            const int j = base + lane;
-            int r = 1;  // beyond lim: treated as a rejection
-            int64_t v = 0;
-            if (j <= lim) {
-                r = wjudge(t, st, u, j, B, &v);
-                ++checks;
-                if (r == 0) hi = max(hi, v);
-                else if (r == 1) lo = min(lo, v);
-            }
-            const unsigned rej = __ballot_sync(kFull, r != 0);
-            if (rej) {
-                reach = base + __ffs(rej) - 2;
-                break;
-            }
-            reach = base + 31;
-        }
-        if (reach < s + 1) ok = false;
-        u = reach;
-        if (lane == 0) wa.U[s + 1] = (uint8_t)reach;
+    __device__ __forceinline__ int eval(const WStage& st, int i, int j, int64_t B, int64_t* cost) const {
+        const longlong2 si = t.SA[i], sj = t.SA[j];
+        if ((sj.x - si.x) + st.f * (sj.y - si.y) > st.capk) return 2;
+        const int64_t v = t.P[st.row + j] - t.P[st.row + i] + st.c;
+        *cost = v;
+        return v <= B ? 0 : 1;
     }
-    __syncwarp();
-    // backward feasible-start sets: C_S = {L}, then stages S-1 .. 1
-    if (ok) {
-        if (lane < kSetWords) wa.C[S][lane] = lane == (L >> 5) ? 1u << (L & 31) : 0u;
-        __syncwarp();
-        int nmax = L;
-        for (int s = S - 1; s >= 1 && ok; --s) {
-            const uint32_t* Cn = wa.C[s + 1];
-            if (lane < kSetWords) wa.C[s][lane] = 0;
-            __syncwarp();
-            const int top = min((int)wa.U[s], nmax - 1);
-            if (top < s) {
-                ok = false;
-                break;
-            }
-            const WStage st = bcast(mine, s);
-            int any = 0, newmax = -1;
-            for (int w = top >> 5; w >= (s >> 5); --w) {
-                const int i = (w << 5) + lane;
-                // smallest successor above i: in this word, else beyond it
-                const uint32_t cw = Cn[w];
-                const uint32_t above = lane == 31 ? 0u : (cw >> (lane + 1)) << (lane + 1);
-                int beyond = -1;
-                for (int w2 = w + 1; w2 <= (L >> 5); ++w2)
-                    if (Cn[w2]) {
-                        beyond = (w2 << 5) + __ffs(Cn[w2]) - 1;
-                        break;
-                    }
-                const int succ = above ? (w << 5) + __ffs(above) - 1 : beyond;
-                int r = 3;
-                int64_t v = 0;
-                if (i >= s && i <= top && succ >= 0) {
-                    r = wjudge(t, st, i, succ, B, &v);
-                    ++checks;
-                    if (r == 0) hi = max(hi, v);
-                    else if (r == 1) lo = min(lo, v);
-                }
-                const unsigned acc = __ballot_sync(kFull, r == 0);
-                if (lane == 0) wa.C[s][w] = acc;
-                if (acc) {
-                    any = 1;
-                    if (newmax < 0) newmax = (w << 5) + 31 - __clz(acc);
-                }
-            }
-            __syncwarp();
-            if (!any) ok = false;
-            nmax = newmax;
-        }
-    }
-    bool feasible = false;
-    if (ok) {
-        const int succ0 = S == 1 ? L : next_above(wa.C[1], 0, L);
-        const WStage st0 = bcast(mine, 0);
-        if (succ0 >= 0 && lane == 0) {
-            int64_t v = 0;
-            const int r = wjudge(t, st0, 0, succ0, B, &v);
-            ++checks;
-            if (r == 0) {
-                hi = max(hi, v);
-                feasible = true;
-            } else if (r == 1) {
-                lo = min(lo, v);
-            }
-        }
-        feasible = __shfl_sync(kFull, feasible, 0);
-    }
-    hi_out = wmax64(hi);
-    lo_out = wmin64(lo);
-    return feasible;
-}
+};
 
 template <bool kCount>
 __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
-    if (!load_image(smem, a.img, a.lay.bytes, &bar, a.err)) return;
+    if (!wp::load_image(smem, a.img, a.lay.bytes, &bar, a.err)) return;
     const Layout& y = a.lay;
     WTabs t;
     t.P = reinterpret_cast<const int64_t*>(smem + y.offP);
@@ -308,17 +122,18 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
             inv = 1.0f / tot;
             cw = u64_to_float((uint64_t)mine.c) / tot;
         }
-        hi = wmax64(hi);
+        hi = wp::wmax64(hi);
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             inv += __shfl_xor_sync(kFull, inv, o);
             cw += __shfl_xor_sync(kFull, cw, o);
         }
+        const PlainJudge judge{t, mine};
         int64_t shi, slo;
         if (!memok) {
             // memory-only probe decides OOM and gives a tighter upper bound
             if (kCount && lane == 0) ++probes;
-            if (!wprobe(t, mine, S, kInf, wa, shi, slo, checks)) {
+            if (!wp::probe(judge, S, L, kInf, wa, shi, slo, checks)) {
                 if (lane == 0) {
                     a.T[c] = -1;
                     a.B[c] = -1;
@@ -343,7 +158,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         while (lo < hi) {
             B = min(max(B, lo), hi - 1);
             if (kCount && lane == 0) ++probes;
-            if (wprobe(t, mine, S, B, wa, shi, slo, checks)) {
+            if (wp::probe(judge, S, L, B, wa, shi, slo, checks)) {
                 hi = shi;
                 hi_known = true;
             } else {
@@ -368,19 +183,8 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         const int64_t Bstar = hi;
         // the sets of the optimum give the canonical split
         if (kCount && lane == 0) ++probes;
-        if (!wprobe(t, mine, S, Bstar, wa, shi, slo, checks) && lane == 0) atomicOr(a.err, kErrInternal);
-        if (lane == 0) {
-            int at = 0;
-            wa.A[0] = 0;
-            for (int s = 0; s + 1 < S; ++s) {
-                const int x = next_above(wa.C[s + 1], at, L);
-                if (x < 0) atomicOr(a.err, kErrInternal);
-                at = max(x, at + 1);
-                wa.A[s + 1] = (uint8_t)at;
-            }
-            wa.A[S] = (uint8_t)L;
-        }
-        __syncwarp();
+        if (!wp::probe(judge, S, L, Bstar, wa, shi, slo, checks) && lane == 0) atomicOr(a.err, kErrInternal);
+        if (!wp::walk(wa, S, L) && lane == 0) atomicOr(a.err, kErrInternal);
         // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s, lane per stage
         int64_t ts = 0;
         uint64_t G = 0, D = 1;
@@ -392,10 +196,8 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
             G = (uint64_t)(t.PB[a1] - t.PB[a0]);
             D = (uint64_t)t.inter[g] << j;
         }
-        const int64_t tmax = wmax64(ts);
-        int64_t tsum = ts;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) tsum += __shfl_xor_sync(kFull, tsum, o);
+        const int64_t tmax = wp::wmax64(ts);
+        const int64_t tsum = wp::wsum64(ts);
         // the stage with the largest G / (k bw), compared exactly
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
