@@ -270,7 +270,7 @@ __device__ __forceinline__ T pick4(const T (&v)[4], int k) {
     return k == 0 ? v[0] : k == 1 ? v[1] : k == 2 ? v[2] : v[3];
 }
 
-__global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, TiledArgs ta) {
+__global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, TiledArgs ta) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     if (!wp::load_image(smem, ta.timg, ta.tl.bytes, &bar, a.err)) return;
@@ -315,24 +315,8 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
             mine.c = t.p2p[(mine.g * 8 + h) * 2 + same];
         }
         const TiledJudge judge{t, mine};
-        // memory-only probe: OOM, else a feasible upper bound
-        int64_t hi, lo;
-        if (!wp::probe(judge, S, L, kInf, wa, hi, lo, checks)) {
-            if (lane == 0) {
-                a.T[c] = -1;
-                a.B[c] = -1;
-                a.ndp[c] = (uint16_t)n;
-                a.status[c] = HEDDLE_CAND_OOM;
-                a.wl_T[p] = -1;
-            }
-            if (a.bounds) {
-                a.bounds[(int64_t)(lane + 1) * a.bstride + c] = 0;
-                if (lane == 0) a.bounds[c] = 0;
-            }
-            continue;
-        }
         // first guess: the balanced bound with every stage at its fastest
-        // tiling over all layers, then gallop until the bracket closes
+        // tiling over all layers
         float inv = 0.f, cw = 0.f;
         if (live) {
             const int base = tile_base(mine.j), cnt = (mine.j + 1) * (mine.j + 2) / 2;
@@ -349,37 +333,71 @@ __global__ void __launch_bounds__(kTBlock) tiled_search_kernel(PriceArgs a, Tile
             inv += __shfl_xor_sync(wp::kFull, inv, o);
             cw += __shfl_xor_sync(wp::kFull, cw, o);
         }
-        int64_t Bhi = hi, Blo = 0;
-        bool lo_known = false, hi_known = false;
-        int64_t B = (int64_t)float_to_u64((1.0f + cw) / inv);
-        int64_t step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
-        int it = 0;
-        while (Blo < Bhi) {
-            B = min(max(B, Blo), Bhi - 1);
-            if (wp::probe(judge, S, L, B, wa, hi, lo, checks)) {
+        // one probe call site (the probe is large): phase 0 the memory-only
+        // probe (OOM, else a feasible upper bound), phase 1 the threshold
+        // search galloping from the guess, phase 2 the probe at B* whose
+        // sets give the split
+        int64_t Bhi = 0, Blo = 0, B = kInf, step = 1;
+        bool lo_known = false, hi_known = false, oom = false;
+        int phase = 0, it = 0;
+        while (true) {
+            int64_t hi, lo;
+            const bool feas = wp::probe(judge, S, L, B, wa, hi, lo, checks);
+            if (phase == 0) {
+                if (!feas) {
+                    oom = true;
+                    break;
+                }
                 Bhi = hi;
-                hi_known = true;
+                B = (int64_t)float_to_u64((1.0f + cw) / inv);
+                step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
+                phase = 1;
+            } else if (phase == 1) {
+                if (feas) {
+                    Bhi = hi;
+                    hi_known = true;
+                } else {
+                    Blo = lo;
+                    lo_known = true;
+                }
+                if (!lo_known) {
+                    B = Bhi - step;
+                    step *= 2;
+                } else if (!hi_known) {
+                    B = Blo + step;
+                    step *= 2;
+                } else {
+                    B = Blo + (Bhi - Blo) / 2;
+                }
+                if (++it > kMaxIters) {
+                    if (lane == 0) atomicOr(a.err, kErrSearchBound);
+                    Blo = Bhi;
+                }
             } else {
-                Blo = lo;
-                lo_known = true;
-            }
-            if (Blo >= Bhi) break;
-            if (!lo_known) {
-                B = Bhi - step;
-                step *= 2;
-            } else if (!hi_known) {
-                B = Blo + step;
-                step *= 2;
-            } else {
-                B = Blo + (Bhi - Blo) / 2;
-            }
-            if (++it > kMaxIters) {
-                if (lane == 0) atomicOr(a.err, kErrSearchBound);
+                if (!feas && lane == 0) atomicOr(a.err, kErrInternal);
                 break;
             }
+            if (phase == 1 && Blo >= Bhi) {
+                phase = 2;
+                B = Bhi;
+            } else if (phase == 1) {
+                B = min(max(B, Blo), Bhi - 1);
+            }
         }
-        const int64_t Bstar = Bhi;
-        if (!wp::probe(judge, S, L, Bstar, wa, hi, lo, checks) && lane == 0) atomicOr(a.err, kErrInternal);
+        if (oom) {
+            if (lane == 0) {
+                a.T[c] = -1;
+                a.B[c] = -1;
+                a.ndp[c] = (uint16_t)n;
+                a.status[c] = HEDDLE_CAND_OOM;
+                a.wl_T[p] = -1;
+            }
+            if (a.bounds) {
+                a.bounds[(int64_t)(lane + 1) * a.bstride + c] = 0;
+                if (lane == 0) a.bounds[c] = 0;
+            }
+            continue;
+        }
         if (!wp::walk(wa, S, L) && lane == 0) atomicOr(a.err, kErrInternal);
 
         // ---- re-selection on the split, one lane per stage: per EDP

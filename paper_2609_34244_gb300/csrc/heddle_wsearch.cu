@@ -129,61 +129,84 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
             cw += __shfl_xor_sync(kFull, cw, o);
         }
         const PlainJudge judge{t, mine};
-        int64_t shi, slo;
-        if (!memok) {
-            // memory-only probe decides OOM and gives a tighter upper bound
-            if (kCount && lane == 0) ++probes;
-            if (!wp::probe(judge, S, L, kInf, wa, shi, slo, checks)) {
-                if (lane == 0) {
-                    a.T[c] = -1;
-                    a.B[c] = -1;
-                    a.ndp[c] = (uint16_t)n;
-                    a.status[c] = HEDDLE_CAND_OOM;
-                    a.wl_T[p] = -1;
-                }
-                if (a.bounds) {
-                    a.bounds[(int64_t)(lane + 1) * a.bstride + c] = 0;
-                    if (lane == 0) a.bounds[c] = 0;
-                }
-                continue;
+        // one probe call site (the probe is large): phase 0 the memory-only
+        // probe (OOM, else a tighter upper bound; skipped when the screen
+        // knows a split fits), phase 1 the threshold search galloping from
+        // the balanced guess, phase 2 the probe at B* whose sets give the
+        // split
+        int64_t lo = 0, B = kInf, step = 1;
+        bool lo_known = false, hi_known = false, oom = false;
+        int phase = memok ? 1 : 0, it = 0;
+        if (memok) {
+            B = (int64_t)float_to_u64((1.0f + cw) / inv);
+            step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
+            if (lo >= hi) {
+                phase = 2;
+                B = hi;
+            } else {
+                B = min(max(B, lo), hi - 1);
             }
-            hi = shi;
         }
-        // ---- PartitionLayers: threshold search from the balanced guess
-        int64_t lo = 0;
-        bool lo_known = false, hi_known = false;
-        int64_t B = (int64_t)float_to_u64((1.0f + cw) / inv);
-        int64_t step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
-        int it = 0;
-        while (lo < hi) {
-            B = min(max(B, lo), hi - 1);
+        while (true) {
+            int64_t shi, slo;
             if (kCount && lane == 0) ++probes;
-            if (wp::probe(judge, S, L, B, wa, shi, slo, checks)) {
+            const bool feas = wp::probe(judge, S, L, B, wa, shi, slo, checks);
+            if (phase == 0) {
+                if (!feas) {
+                    oom = true;
+                    break;
+                }
                 hi = shi;
-                hi_known = true;
+                B = (int64_t)float_to_u64((1.0f + cw) / inv);
+                step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
+                phase = 1;
+            } else if (phase == 1) {
+                if (feas) {
+                    hi = shi;
+                    hi_known = true;
+                } else {
+                    lo = slo;
+                    lo_known = true;
+                }
+                if (!lo_known) {
+                    B = hi - step;
+                    step *= 2;
+                } else if (!hi_known) {
+                    B = lo + step;
+                    step *= 2;
+                } else {
+                    B = lo + (hi - lo) / 2;
+                }
+                if (++it > kMaxIters) {
+                    if (lane == 0) atomicOr(a.err, kErrSearchBound);
+                    lo = hi;
+                }
             } else {
-                lo = slo;
-                lo_known = true;
-            }
-            if (lo >= hi) break;
-            if (!lo_known) {
-                B = hi - step;
-                step *= 2;
-            } else if (!hi_known) {
-                B = lo + step;
-                step *= 2;
-            } else {
-                B = lo + (hi - lo) / 2;
-            }
-            if (++it > kMaxIters) {
-                if (lane == 0) atomicOr(a.err, kErrSearchBound);
+                if (!feas && lane == 0) atomicOr(a.err, kErrInternal);
                 break;
             }
+            if (phase == 1 && lo >= hi) {
+                phase = 2;
+                B = hi;
+            } else if (phase == 1) {
+                B = min(max(B, lo), hi - 1);
+            }
+        }
+        if (oom) {
+            if (lane == 0) {
+                a.T[c] = -1;
+                a.B[c] = -1;
+                a.ndp[c] = (uint16_t)n;
+                a.status[c] = HEDDLE_CAND_OOM;
+                a.wl_T[p] = -1;
+            }
+            if (a.bounds) {
+                a.bounds[(int64_t)(lane + 1) * a.bstride + c] = 0;
+                if (lane == 0) a.bounds[c] = 0;
+            }
+            continue;
         }
         const int64_t Bstar = hi;
-        // the sets of the optimum give the canonical split
-        if (kCount && lane == 0) ++probes;
-        if (!wp::probe(judge, S, L, Bstar, wa, shi, slo, checks) && lane == 0) atomicOr(a.err, kErrInternal);
         if (!wp::walk(wa, S, L) && lane == 0) atomicOr(a.err, kErrInternal);
         // ---- Evaluate: T = (M-1) max t_s + sum t_s + max g_s, lane per stage
         int64_t ts = 0;
