@@ -415,10 +415,11 @@ heddle_status heddle_price_tiled(heddle_ctx* ctx, const heddle_candidates* cands
 
 /* End-to-end convenience for host (ideally pinned) buffers: streams the
  * candidates in batches of `batch` (1 <= batch <= 2^20, E_LIMIT above)
- * through context-owned device staging buffers (two sets), prices them,
+ * through context-owned device staging buffers (three sets), prices them,
  * merges them into *state and copies back every non-NULL field of
  * `results` (host arrays of cands->n entries; bounds uses plane stride
- * cands->n).  Batch k is copied in on a copy stream, screened and searched
+ * cands->n).  Batch k is copied in on a copy stream into staging set k % 3
+ * (free once batch k - 3 is copied out), screened and searched
  * on work stream k % 2 with worklist set k % 2, merged on `stream` in batch
  * order and copied out on a second copy stream, so copies, the search of
  * one batch and the screen of the next overlap.  *state is host memory,

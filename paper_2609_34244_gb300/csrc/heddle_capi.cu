@@ -69,18 +69,21 @@ struct heddle_ctx {
     int32_t* d_tickets = nullptr;  // [17], zero between top-k launches
     // host-buffer path
     cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
-    cudaEvent_t ev_loaded[2] = {nullptr, nullptr}, ev_priced[2] = {nullptr, nullptr},
-                ev_free[2] = {nullptr, nullptr};
+    // kStageSets staging sets: a batch's copies in wait only for the batch
+    // kStageSets earlier to be merged, so the copy stream keeps running while
+    // the two batches before it are still being searched
+    static constexpr int kStageSets = 3;
+    cudaEvent_t ev_loaded[kStageSets] = {}, ev_priced[kStageSets] = {}, ev_free[kStageSets] = {};
     int64_t stage_cap = 0;
     int32_t stage_smax = 0;
-    uint8_t* st_S[2] = {nullptr, nullptr};
-    uint16_t* st_M[2] = {nullptr, nullptr};
-    uint8_t* st_code[2] = {nullptr, nullptr};
-    int64_t* st_T[2] = {nullptr, nullptr};
-    int64_t* st_B[2] = {nullptr, nullptr};
-    uint16_t* st_n[2] = {nullptr, nullptr};
-    uint8_t* st_status[2] = {nullptr, nullptr};
-    uint8_t* st_bounds[2] = {nullptr, nullptr};
+    uint8_t* st_S[kStageSets] = {};
+    uint16_t* st_M[kStageSets] = {};
+    uint8_t* st_code[kStageSets] = {};
+    int64_t* st_T[kStageSets] = {};
+    int64_t* st_B[kStageSets] = {};
+    uint16_t* st_n[kStageSets] = {};
+    uint8_t* st_status[kStageSets] = {};
+    uint8_t* st_bounds[kStageSets] = {};
     heddle_topk_state* d_state = nullptr;
     // phase timing: four events per priced chunk (start, after the screen,
     // after the search, after the top-k), recorded while time_phases is set
@@ -499,7 +502,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_scratch2);
     cudaFree(x->d_scratch2_count);
     cudaFree(x->d_tickets);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < heddle_ctx::kStageSets; ++b) {
         cudaFree(x->st_S[b]);
         cudaFree(x->st_M[b]);
         cudaFree(x->st_code[b]);
@@ -913,7 +916,7 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
     if (!x->s_h2d) {
         CU(cudaStreamCreateWithFlags(&x->s_h2d, cudaStreamNonBlocking));
         CU(cudaStreamCreateWithFlags(&x->s_d2h, cudaStreamNonBlocking));
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < heddle_ctx::kStageSets; ++b) {
             CU(cudaEventCreateWithFlags(&x->ev_loaded[b], cudaEventDisableTiming));
             CU(cudaEventCreateWithFlags(&x->ev_priced[b], cudaEventDisableTiming));
             CU(cudaEventCreateWithFlags(&x->ev_free[b], cudaEventDisableTiming));
@@ -924,7 +927,7 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         CU(cudaDeviceSynchronize());
         const int64_t cap = nb_max > x->stage_cap ? nb_max : x->stage_cap;
         const int32_t sm = c->s_max > x->stage_smax ? c->s_max : x->stage_smax;
-        for (int b = 0; b < 2; ++b) {
+        for (int b = 0; b < heddle_ctx::kStageSets; ++b) {
             cudaFree(x->st_S[b]);
             cudaFree(x->st_M[b]);
             cudaFree(x->st_code[b]);
@@ -956,15 +959,16 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         x->stage_smax = sm;
     }
     CU(cudaMemcpyAsync(x->d_state, state, sizeof(heddle_topk_state), cudaMemcpyHostToDevice, sc));
-    CU(cudaEventRecord(x->ev_free[0], sc));
-    CU(cudaEventRecord(x->ev_free[1], sc));
+    for (int b = 0; b < heddle_ctx::kStageSets; ++b) CU(cudaEventRecord(x->ev_free[b], sc));
     const bool want_bounds = r && r->bounds;
-    // batch k: copies in on s_h2d, screen and search on work stream k % 2
-    // (worklist set k % 2, released by batch k - 2's top-k), top-k merge on
-    // the caller's stream in batch order, copies out on s_d2h
+    // batch k: copies in on s_h2d into staging set k % 3 (free once batch
+    // k - 3 is copied out), screen and search on work stream k % 2 (worklist
+    // set k % 2, released by batch k - 2's top-k), top-k merge on the
+    // caller's stream in batch order, copies out on s_d2h
     bool used[2] = {false, false};
     for (int64_t lo = 0, it = 0; lo < n; lo += batch, ++it) {
-        const int b = (int)(it & 1);
+        const int b = (int)(it % heddle_ctx::kStageSets);
+        const int wb = (int)(it & 1);
         const int64_t nb = (n - lo) < batch ? (n - lo) : batch;
         // host -> device on the copy stream once the set is free
         CU(cudaStreamWaitEvent(x->s_h2d, x->ev_free[b], 0));
@@ -973,10 +977,10 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         CU(cudaMemcpy2DAsync(x->st_code[b], nb, c->code + lo, c->plane_stride, nb, c->s_max,
                              cudaMemcpyHostToDevice, x->s_h2d));
         CU(cudaEventRecord(x->ev_loaded[b], x->s_h2d));
-        const cudaStream_t ws = x->s_work[b];
+        const cudaStream_t ws = x->s_work[wb];
         CU(cudaStreamWaitEvent(ws, x->ev_loaded[b], 0));
-        if (used[b]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[b], 0));
-        used[b] = true;
+        if (used[wb]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[wb], 0));
+        used[wb] = true;
         heddle_candidates cb{};
         cb.S = x->st_S[b];
         cb.M = x->st_M[b];
@@ -994,10 +998,10 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         if (nb > 0) {
             hd::PriceArgs a{};
             fill_price_args(x, &cb, nullptr, 0, tiled, a);
-            if ((st = price_chunk(x, a, &cb, &rb, 0, nb, b, ws, x->d_state, sc, tiled, nullptr)) != HEDDLE_OK)
+            if ((st = price_chunk(x, a, &cb, &rb, 0, nb, wb, ws, x->d_state, sc, tiled, nullptr)) != HEDDLE_OK)
                 return st;
         }
-        CU(cudaEventRecord(x->ev_wl_free[b], sc));
+        CU(cudaEventRecord(x->ev_wl_free[wb], sc));
         CU(cudaEventRecord(x->ev_priced[b], sc));
         // device -> host of the requested result fields on the second copy stream
         CU(cudaStreamWaitEvent(x->s_d2h, x->ev_priced[b], 0));
