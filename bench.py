@@ -62,8 +62,8 @@ SMS, LANES_PER_SM = 152, 128  # 4 SM sub-partitions x 32 lanes issue per clock
 # DRAM bytes (read + write) of one search launch on a 1e6-candidate batch of
 # the stress workload, from an ncu capture, with the SHA-256 of the kernel
 # sources it was taken on; reported as null once those sources change.
-TRAFFIC = {2: {"bytes": 15872768, "batch": 1000000,
-              "sha256": "db339698d9a6370d2be7b954b24e60f33d6034f6349d4a7bad9bc26422e82582"}}
+TRAFFIC = {2: {"bytes": 16187136, "batch": 1000000,
+              "sha256": "d6b7b201d6c9c78d0500ec240d6f994e48501f877b20eaf68beb6711066eea93"}}
 TRAFFIC_SOURCES = {1: ["heddle_price.cu", "heddle_internal.cuh"],
                    2: ["heddle_eqsearch.cu", "heddle_internal.cuh"]}
 
@@ -270,11 +270,17 @@ def main():
     with ClockSampler(local) as clk:
         torch.cuda.synchronize()
         t_start.record(stream)
+        step_ev = []
         for _ in range(args.steps):
             step()
+            ev = torch.cuda.Event(enable_timing=True)
+            ev.record(stream)
+            step_ev.append(ev)
         t_end.record(stream)
         torch.cuda.synchronize()
     h.heddle_time_phases(ctx, False)
+    # per-step device times (consecutive events on the stream)
+    step_ms = [t_start.elapsed_time(step_ev[0])] + [a.elapsed_time(b) for a, b in zip(step_ev, step_ev[1:])]
     shard.barrier(group)
     clocks = clk.summary()
     ms = t_start.elapsed_time(t_end)
@@ -283,6 +289,20 @@ def main():
     errors = h.heddle_device_errors(ctx)
     local_topk = h.read_topk_state(state)
     merged = shard.merge_topk_across_ranks(group, local_topk, 16)
+
+    # single-batch wall latency: one call on one batch of `batch` candidates,
+    # host call to results ready (synchronised), after a warm call
+    one_c, one_r = cbatches[0]
+    h.heddle_topk_reset(ctx, state, 16, stream)
+    h.heddle_price_topk(ctx, one_c, one_r, state, stream)
+    torch.cuda.synchronize()
+    lat = []
+    for _ in range(20):
+        t0 = time.perf_counter()
+        h.heddle_topk_reset(ctx, state, 16, stream)
+        h.heddle_price_topk(ctx, one_c, one_r, state, stream)
+        torch.cuda.synchronize()
+        lat.append((time.perf_counter() - t0) * 1e3)
 
     # the same kernels without overlap (one call per batch, so each chunk's
     # screen, search and top-k run alone): the search's isolated duration
@@ -522,6 +542,11 @@ def main():
         # counted in the timed steps (screen, search, top-k block and levels)
         "gpu_launches": (args.steps + sum(v[1] for v in phases.values())) * world,
         "per_candidate_ns": 1e6 * ms_all / args.steps / n,
+        "step_ms": {"median": float(np.median(step_ms)), "best": float(np.min(step_ms)),
+                    "worst": float(np.max(step_ms)), "runs": len(step_ms)},
+        "single_batch_latency_ms": {"median": float(np.median(lat)), "best": float(np.min(lat)),
+                                    "batch": batch, "how": "wall time of one heddle_price_topk call on one batch, "
+                                                           "synchronised, 20 runs after a warm call"},
         "roofline": {"bound": "alu", "achieved": achieved_tops, "peak": peak_tops, "unit": "Tops/s",
                      "frac": achieved_tops / peak_tops,
                      "traffic": traffic_per_launch(search, batch),

@@ -12,8 +12,8 @@
 //
 // First guess, in float only: the continuous balance
 // sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2 (the
-// floors lose half a layer per such stage on average), solved by Newton
-// steps from the unsaturated balance.  Exact probes then decide and snap
+// floors lose half a layer per such stage on average), solved by at most
+// three Newton steps from the unsaturated balance.  Exact probes then decide and snap
 // the bracket to breakpoints: a feasible probe keeps its caps down to
 // hi = max_s (c_s + cap_s q_s); an infeasible one keeps them up to the next
 // breakpoint lo = min_s c_s + (cap_s + 1) q_s.  Two exact stop rules end
@@ -511,7 +511,7 @@ __global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
             // first guess: Newton on the saturating continuous count
             const float flo = u64_to_float(q.lo), fhi = u64_to_float(q.hi);
             float Bf = fmaxf(flo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : flo);
-            for (int it = 0; it < 8; ++it) {
+            for (int it = 0; it < 3; ++it) {  // the exact probes finish the job
                 float sl;
                 int below;
                 Bf = fminf(Bf, fhi);
