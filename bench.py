@@ -173,7 +173,9 @@ def run_reference(args, w):
     dt = time.perf_counter() - t0
     value = n * args.steps / dt
     sample = "first %d candidates of %s seed 0 per step, %d host threads" % (n, WORKLOAD, used)
-    return {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": 0,
+    # n_gpus: the N of the run this arm is paired with (the oracle itself
+    # runs on rank 0's host cores; `cpu_baseline.cores` says how many)
+    return {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
             "data": "synthetic",
