@@ -109,12 +109,16 @@ struct heddle_ctx {
     std::vector<double> mbs_profile;  // [levels][types][4][L] seconds, or empty
     bool mbs_ready = false;
     Level lv[HEDDLE_MAX_MBS_LEVELS];
-    int64_t* lv_T = nullptr;
-    int64_t* lv_B = nullptr;
-    uint16_t* lv_n = nullptr;
-    uint8_t* lv_status = nullptr;
-    uint8_t* lv_bounds = nullptr;
-    size_t lv_T_cap = 0, lv_B_cap = 0, lv_n_cap = 0, lv_status_cap = 0, lv_bounds_cap = 0;
+    // one result set per size above the base (their pricings run as a
+    // pipeline, their merges after)
+    int64_t* lv_T[HEDDLE_MAX_MBS_LEVELS] = {};
+    int64_t* lv_B[HEDDLE_MAX_MBS_LEVELS] = {};
+    uint16_t* lv_n[HEDDLE_MAX_MBS_LEVELS] = {};
+    uint8_t* lv_status[HEDDLE_MAX_MBS_LEVELS] = {};
+    uint8_t* lv_bounds[HEDDLE_MAX_MBS_LEVELS] = {};
+    size_t lv_T_cap[HEDDLE_MAX_MBS_LEVELS] = {}, lv_B_cap[HEDDLE_MAX_MBS_LEVELS] = {},
+           lv_n_cap[HEDDLE_MAX_MBS_LEVELS] = {}, lv_status_cap[HEDDLE_MAX_MBS_LEVELS] = {},
+           lv_bounds_cap[HEDDLE_MAX_MBS_LEVELS] = {};
     // multi-template plans: the cluster's nodes on the device, split bounds
     // of slots whose caller passed none
     int32_t* d_node_type = nullptr;
@@ -520,11 +524,13 @@ void heddle_destroy(heddle_ctx* x) {
         cudaFree(v.img);
         cudaFree(v.q);
     }
-    cudaFree(x->lv_T);
-    cudaFree(x->lv_B);
-    cudaFree(x->lv_n);
-    cudaFree(x->lv_status);
-    cudaFree(x->lv_bounds);
+    for (int i = 0; i < HEDDLE_MAX_MBS_LEVELS; ++i) {
+        cudaFree(x->lv_T[i]);
+        cudaFree(x->lv_B[i]);
+        cudaFree(x->lv_n[i]);
+        cudaFree(x->lv_status[i]);
+        cudaFree(x->lv_bounds[i]);
+    }
     cudaFree(x->d_timg);
     cudaFree(x->d_node_type);
     cudaFree(x->d_node_gpus);
@@ -839,6 +845,56 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     return ok(x);
 }
 
+// One chunk of a pricing: candidates [lo, lo + nb) of c into r (offsets
+// and the bounds plane stride c->n as for a call on c), with the tables of
+// lvl (nullable: the main tables) at micro-batch shift `shift`.
+struct PriceUnit {
+    const heddle_candidates* c;
+    const heddle_results* r;
+    const heddle_ctx::Level* lvl;
+    int shift;
+    int64_t lo, nb;
+};
+
+// Independent chunk pricings (no top-k, no tiling output) as one pipeline:
+// they alternate the two work streams and worklist sets like the chunks of
+// one call, and `stream` waits for all of them.  The units are validated
+// by the caller.
+heddle_status price_units(heddle_ctx* x, const PriceUnit* u, int nu, void* stream) {
+    heddle_status st;
+    const cudaStream_t cs = (cudaStream_t)stream;
+    const bool tiled = x->tiled_ready;
+    if (tiled && x->search_mode == HEDDLE_SEARCH_DISTRIBUTE)
+        return fail(x, HEDDLE_E_STATE, "expert tiling prices the min-max split only (search mode DISTRIBUTE)");
+    DeviceGuard dg(x->device);
+    const bool pipe = nu > 1;
+    if (pipe) {
+        if ((st = ensure_pipeline(x)) != HEDDLE_OK) return st;
+        CU(cudaEventRecord(x->ev_in, cs));
+    }
+    bool used[2] = {false, false};
+    for (int k = 0; k < nu; ++k) {
+        if (u[k].nb <= 0) continue;
+        const int b = pipe ? (k & 1) : 0;
+        const cudaStream_t ws = pipe ? x->s_work[b] : cs;
+        if (pipe) {
+            CU(cudaStreamWaitEvent(ws, x->ev_in, 0));
+            if (used[b]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[b], 0));
+            used[b] = true;
+        }
+        const bool t = tiled && !u[k].lvl;
+        hd::PriceArgs a{};
+        fill_price_args(x, u[k].c, u[k].lvl, u[k].shift, t, a);
+        if ((st = price_chunk(x, a, u[k].c, u[k].r, u[k].lo, u[k].nb, b, ws, nullptr, cs, t, nullptr)) != HEDDLE_OK)
+            return st;
+        if (pipe) CU(cudaEventRecord(x->ev_wl_free[b], ws));
+    }
+    if (pipe)
+        for (int b = 0; b < 2; ++b)
+            if (used[b]) CU(cudaStreamWaitEvent(cs, x->ev_wl_free[b], 0));
+    return ok(x);
+}
+
 }  // namespace
 
 extern "C" {
@@ -1102,35 +1158,49 @@ heddle_status heddle_price_mbs(heddle_ctx* x, const heddle_candidates* c, const 
     if (!r->T || !r->bottleneck || !r->n_dp || !r->status) return fail(x, HEDDLE_E_ARG, "null result array");
     DeviceGuard dg(x->device);
     cudaStream_t sm = (cudaStream_t)stream;
-    // the base size straight into the caller's results
-    if ((st = price_impl(x, c, r, nullptr, stream, &x->lv[0], 0)) != HEDDLE_OK) return st;
     if (mbs) CU(cudaMemsetAsync(mbs, 0, (size_t)c->n, sm));
-    if (x->mbs_levels == 1) return ok(x);
-    const size_t cap = (size_t)std::min<int64_t>(c->n, hd::kWorklistCap);
-    CU(grow(&x->lv_T, &x->lv_T_cap, sizeof(int64_t) * cap));
-    CU(grow(&x->lv_B, &x->lv_B_cap, sizeof(int64_t) * cap));
-    CU(grow(&x->lv_n, &x->lv_n_cap, sizeof(uint16_t) * cap));
-    CU(grow(&x->lv_status, &x->lv_status_cap, cap));
-    if (r->bounds) CU(grow(&x->lv_bounds, &x->lv_bounds_cap, (size_t)(HEDDLE_MAX_STAGES + 1) * cap));
-    // every larger size, one chunk at a time, folded into the results
-    for (int64_t lo = 0; lo < c->n; lo += hd::kWorklistCap) {
-        const int64_t nb = std::min<int64_t>(c->n - lo, hd::kWorklistCap);
+    const int nl = x->mbs_levels;
+    const size_t cap = (size_t)std::min<int64_t>(c->n, x->chunk);
+    for (int i = 1; i < nl; ++i) {
+        CU(grow(&x->lv_T[i], &x->lv_T_cap[i], sizeof(int64_t) * cap));
+        CU(grow(&x->lv_B[i], &x->lv_B_cap[i], sizeof(int64_t) * cap));
+        CU(grow(&x->lv_n[i], &x->lv_n_cap[i], sizeof(uint16_t) * cap));
+        CU(grow(&x->lv_status[i], &x->lv_status_cap[i], cap));
+        if (r->bounds) CU(grow(&x->lv_bounds[i], &x->lv_bounds_cap[i], (size_t)(HEDDLE_MAX_STAGES + 1) * cap));
+    }
+    // per chunk: every size priced as one pipeline (the base size straight
+    // into the caller's results, each larger size into its own set), then
+    // the larger sizes folded into the results in order
+    for (int64_t lo = 0; lo < c->n; lo += x->chunk) {
+        const int64_t nb = std::min<int64_t>(c->n - lo, x->chunk);
         heddle_candidates cc = *c;
         cc.S = c->S + lo;
         cc.M = c->M + lo;
         cc.code = c->code + lo;
         cc.n = nb;
         cc.base_index = c->base_index + lo;
-        heddle_results rr{x->lv_T, x->lv_B, x->lv_n, x->lv_status, r->bounds ? x->lv_bounds : nullptr};
-        for (int i = 1; i < x->mbs_levels; ++i) {
-            if ((st = price_impl(x, &cc, &rr, nullptr, stream, &x->lv[i], i)) != HEDDLE_OK) return st;
+        heddle_results rs[HEDDLE_MAX_MBS_LEVELS];
+        PriceUnit units[HEDDLE_MAX_MBS_LEVELS];
+        for (int i = 0; i < nl; ++i) {
+            if (i == 0) {
+                // the base size straight into the caller's results
+                units[0] = PriceUnit{c, r, &x->lv[0], 0, lo, nb};
+            } else {
+                // a larger size into its own set, laid out for this chunk
+                rs[i] = heddle_results{x->lv_T[i], x->lv_B[i], x->lv_n[i], x->lv_status[i],
+                                       r->bounds ? x->lv_bounds[i] : nullptr};
+                units[i] = PriceUnit{&cc, &rs[i], &x->lv[i], i, 0, nb};
+            }
+        }
+        if ((st = price_units(x, units, nl, stream)) != HEDDLE_OK) return st;
+        for (int i = 1; i < nl; ++i) {
             hd::MbsMergeArgs m{};
             m.n = nb;
-            m.T_l = x->lv_T;
-            m.B_l = x->lv_B;
-            m.n_l = x->lv_n;
-            m.status_l = x->lv_status;
-            m.bounds_l = r->bounds ? x->lv_bounds : nullptr;
+            m.T_l = x->lv_T[i];
+            m.B_l = x->lv_B[i];
+            m.n_l = x->lv_n[i];
+            m.status_l = x->lv_status[i];
+            m.bounds_l = r->bounds ? x->lv_bounds[i] : nullptr;
             m.bstride_l = nb;
             m.T = r->T + lo;
             m.B = r->bottleneck + lo;
@@ -1200,14 +1270,27 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     a.placed = pr->placed;
     a.thr = pr->thr;
     a.err = x->d_flags + 1;
-    // every slot priced as standalone candidates (the split needs bounds)
+    // every slot priced as standalone candidates (the split needs bounds),
+    // the slots pipelined over the work streams
+    heddle_results rs[HEDDLE_MAX_TEMPLATES];
+    const heddle_candidates* cs_[HEDDLE_MAX_TEMPLATES];
     for (int t = 0; t < pl->slots; ++t) {
-        heddle_results r = pr->t[t];
-        if (!r.bounds) {
+        rs[t] = pr->t[t];
+        if (!rs[t].bounds) {
             CU(grow(&x->plan_bounds[t], &x->plan_bounds_cap[t], (size_t)(HEDDLE_MAX_STAGES + 1) * pl->n));
-            r.bounds = x->plan_bounds[t];
+            rs[t].bounds = x->plan_bounds[t];
         }
-        if ((st = price_impl(x, &pl->t[t], &r, nullptr, stream)) != HEDDLE_OK) return st;
+        cs_[t] = &pl->t[t];
+    }
+    {
+        std::vector<PriceUnit> units;
+        for (int t = 0; t < pl->slots; ++t)
+            for (int64_t lo = 0; lo < pl->n; lo += x->chunk)
+                units.push_back(PriceUnit{cs_[t], &rs[t], nullptr, 0, lo, std::min<int64_t>(x->chunk, pl->n - lo)});
+        if ((st = price_units(x, units.data(), (int)units.size(), stream)) != HEDDLE_OK) return st;
+    }
+    for (int t = 0; t < pl->slots; ++t) {
+        const heddle_results& r = rs[t];
         hd::PlanSlot& s = a.slot[t];
         s.S = pl->t[t].S;
         s.M = pl->t[t].M;
