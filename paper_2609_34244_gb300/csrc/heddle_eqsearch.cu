@@ -28,10 +28,11 @@
 // smallest -- a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
 //
 // Scheduling: the screen files every entry in a bucket per depth S; CTA b
-// takes entries [256 b, 256 b + 256) of the buckets read in order of
+// takes entries [128 b, 128 b + 128) of the buckets read in order of
 // decreasing S, so the lanes of a warp run stage loops of equal length and
 // the warps of a CTA carry equal work (the search runs in one wave: a deep
-// warp would otherwise hold its whole CTA at the barrier).  Every
+// warp would otherwise hold its whole CTA at the barrier).  Small CTAs
+// (eight per SM) spread the deep slices over more SMs.  Every
 // thread packs its candidate's stages once into 32-bit words (cost index |
 // P2P index | memory run) held in shared memory interleaved by thread, runs
 // the float guess and one exact probe; the few searches still open are
@@ -47,7 +48,7 @@
 namespace hd {
 namespace {
 
-constexpr int kEqBlock = 256;
+constexpr int kEqBlock = 128;
 constexpr int kZeroP2P = 128;  // a zero entry after the 8 x 8 x 2 P2P table
 constexpr int kMaxIters = 256;
 
@@ -372,7 +373,7 @@ __device__ void eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int6
 }
 
 template <bool kCount>
-__global__ void __launch_bounds__(kEqBlock, 4) eq_search_kernel(PriceArgs a) {
+__global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(PriceArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
     __shared__ int tail_n;
     __shared__ int end_of[kMaxStages + 2];  // entries of depths >= S, [S]

@@ -63,7 +63,7 @@ __device__ __forceinline__ uint32_t stage_desc(int b, const Layout& y, const uns
 __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
     __shared__ uint32_t desc[256];
     __shared__ uint8_t win[8 * 4 * 33];
-    __shared__ uint32_t cap[8 * 4];
+    __shared__ __align__(16) uint32_t cap[8 * 4];
     __shared__ uint32_t magic[257];
     __shared__ uint64_t dem[8 * kScreenBlock];  // per-thread GPUs per unit class, 4 x 16 bits per type
     __shared__ __align__(16) uint8_t tile[kMaxStages * kScreenBlock];  // [stage][candidate of the slice]
@@ -155,14 +155,13 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
             if (S > 0) {
 #pragma unroll
                 for (int g = 0; g < 8; ++g) mydem[g * kScreenBlock] = 0;
-                uint32_t bad = 0, present = 0;
+                uint32_t bad = 0;
                 int run_sum = 0, run_min = 255;
                 const uint8_t* col = tile + ci;
                 for (int s = 0; s < S; ++s) {
                     const uint32_t d = desc[col[s * kScreenBlock]];
                     bad |= d;
                     const int g = (d >> 24) & 7;
-                    present |= 1u << g;
                     mydem[g * kScreenBlock] += 1ull << ((d >> 16) & 63);
                     const int w = win[(d & 0x7ff) + min(S - s, M)];
                     run_sum += w;
@@ -173,19 +172,21 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                 } else {
                     // n = min over (type, class e) of capacity / GPUs in units
                     // >= 2^e; a class with no group of its own size is
-                    // dominated by the class above it
+                    // dominated by the class above it.  Every type is
+                    // visited (an absent type's demand word is zero), so the
+                    // eight chains of loads are independent
                     uint32_t nn = 0xffffffffu;
-                    while (present) {
-                        const int g = __ffs(present) - 1;
-                        present &= present - 1;
-                        const uint64_t v = mydem[g * kScreenBlock];
-                        uint32_t dsum = 0;
 #pragma unroll
-                        for (int e = 3; e >= 0; --e) {
-                            const uint32_t f = (uint32_t)(v >> (16 * e)) & 0xffffu;
-                            dsum += f;
-                            if (f) nn = min(nn, div_small(cap[g * 4 + e], dsum, magic));
-                        }
+                    for (int g = 0; g < 8; ++g) {
+                        const uint64_t v = mydem[g * kScreenBlock];
+                        const uint4 cg = *reinterpret_cast<const uint4*>(cap + g * 4);
+                        const uint32_t f3 = (uint32_t)(v >> 48), f2 = (uint32_t)(v >> 32) & 0xffffu;
+                        const uint32_t f1 = (uint32_t)(v >> 16) & 0xffffu, f0 = (uint32_t)v & 0xffffu;
+                        const uint32_t d3 = f3, d2 = d3 + f2, d1 = d2 + f1, d0 = d1 + f0;
+                        const uint32_t q3 = div_small(cg.w, d3, magic), q2 = div_small(cg.z, d2, magic);
+                        const uint32_t q1 = div_small(cg.y, d1, magic), q0 = div_small(cg.x, d0, magic);
+                        nn = min(nn, min(min(f3 ? q3 : 0xffffffffu, f2 ? q2 : 0xffffffffu),
+                                         min(f1 ? q1 : 0xffffffffu, f0 ? q0 : 0xffffffffu)));
                     }
                     n = nn;
                     if (n == 0)
