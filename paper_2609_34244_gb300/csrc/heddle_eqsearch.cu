@@ -58,18 +58,16 @@ constexpr int kTailCap = 32;  // open searches queued per slice
 struct Search {
     int64_t lo, hi, B;  // B* lies in [lo, hi]; B is the next bound to probe
     int64_t Blo, Bhi;   // last infeasible / feasible bound probed (-1: none)
-    int64_t fhi;        // hi of the last feasible probe: its caps hold at fhi
+    int64_t fhi;        // hi of the last feasible probe (-1: none); chi is its layer count
     int32_t clo, chi;   // layer counts of those probes
-    int16_t fset, wset; // cap set of the last feasible probe (-1: none), set written next
-    int16_t owner, S;   // thread whose shared-memory columns hold the stages; depth
+    int16_t owner, S;   // thread whose shared-memory column holds the stages; depth
     int32_t probes;
     int32_t p;          // worklist entry
     uint16_t M, n;      // its microbatches and DP degree
-    int32_t pad;
 };
 
 struct EqLayout {
-    uint32_t q, rq, p2p, cf, inter, maxn, PB, win, sw, caps, tail, bytes;
+    uint32_t q, rq, p2p, cf, inter, maxn, PB, win, sw, tail, bytes;
 };
 
 __host__ __device__ inline uint32_t al16(uint32_t x) { return (x + 15u) & ~15u; }
@@ -86,7 +84,6 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
     e.PB = o;    o = al16(o + 8 * (L + 1));        // int64 gradient-byte prefix
     e.win = o;   o = al16(o + 8 * 4 * 33);         // uint8 [(g * 4 + j) * 33 + f]
     e.sw = o;    o = al16(o + 4 * kMaxStages * kEqBlock);  // uint32 [s][thread]
-    e.caps = o;  o = al16(o + 2 * kMaxStages * kEqBlock);         // uint8 [2][s][thread]
     e.tail = o;  o = al16(o + sizeof(struct Search) * kTailCap);  // open searches
     e.bytes = o;
     return e;
@@ -103,7 +100,6 @@ struct EqTabs {
     const uint8_t* win;
     int64_t pbytes;  // gradient bytes of every layer when they are all equal, else -1
     uint32_t* sw;   // stage words of thread 0; thread o's element s at [s * kEqBlock + o]
-    uint8_t* caps;  // caps of thread 0, two sets; thread o's set b element s at [(b * 32 + s) * kEqBlock + o]
     int L;
 };
 
@@ -183,8 +179,8 @@ struct Probe {
     float slope;   // sum of 1/q over stages below their run
 };
 
-// Exact probe of bound B for the stages in column sw; caps to column caps.
-__device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, uint8_t* caps, int S, int64_t B, Probe& p) {
+// Exact probe of bound B for the stages in column sw.
+__device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, int S, int64_t B, Probe& p) {
     p.hi = -1;
     p.lo = kInf;
     p.zmax = -1;
@@ -197,7 +193,6 @@ __device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, uint8_t* caps, int
         const uint32_t w = sw[s * kEqBlock];
         const Cap r = stage_cap(t, w, B);
         const int k = max(r.k, 0);
-        caps[s * kEqBlock] = (uint8_t)k;
         if (r.m < 1) {
             p.zmax = kInf;  // never holds a layer
             continue;
@@ -230,10 +225,6 @@ __device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, uint8_t* caps, int
     return p.zmax < 0 && p.tot >= t.L;
 }
 
-__device__ __forceinline__ uint8_t* cap_set(const EqTabs& t, int owner, int set) {
-    return t.caps + set * kMaxStages * kEqBlock + owner;
-}
-
 // One exact probe of search q at q.B and the bracket update; returns true
 // when B* = q.hi is known.
 __device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
@@ -241,14 +232,12 @@ __device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
     q.B = min(max(q.B, q.lo), q.hi - 1);
     ++q.probes;
     Probe p;
-    const bool feas = eq_probe(t, sw, cap_set(t, q.owner, q.wset), q.S, q.B, p);
+    const bool feas = eq_probe(t, sw, q.S, q.B, p);
     if (feas) {
         q.hi = p.hi;
         q.Bhi = q.B;
         q.chi = p.tot;
-        q.fset = q.wset;
         q.fhi = p.hi;
-        q.wset ^= 1;
         // just below hi every stage attaining hi loses a layer
         if (p.tot - p.nhi < t.L || p.hi1) q.lo = q.hi;
     } else {
@@ -282,31 +271,30 @@ __device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
     return false;
 }
 
-// Finish search q: probe until B* = q.hi is known, then make sure cap set
-// q.fset holds the caps at B*.
+// Finish search q: probe until B* = q.hi is known, then make sure q.chi is
+// the layer count at B*.  (A feasible probe at B keeps every cap of its hi:
+// no stage time lies in (hi, B].)
 __device__ void eq_finish(const EqTabs& t, Search& q, uint32_t* err) {
     while (q.lo < q.hi)
         if (eq_step(t, q, err)) break;
-    if (q.fset < 0 || q.fhi != q.hi) {
-        // B* was reached from below (or never probed): its caps
+    if (q.fhi != q.hi) {
+        // B* was reached from below (or never probed): its layer count
         ++q.probes;
         Probe p;
-        if (!eq_probe(t, t.sw + q.owner, cap_set(t, q.owner, q.wset), q.S, q.hi, p)) atomicOr(err, kErrInternal);
-        q.fset = q.wset;
+        if (!eq_probe(t, t.sw + q.owner, q.S, q.hi, p)) atomicOr(err, kErrInternal);
         q.fhi = q.hi;
         q.chi = p.tot;
     }
 }
 
-// The smallest boundaries from the caps at B* (cap set `set` of column
-// `owner`, holding `total` layers), then Evaluate:
-// T = (M-1) max t_s + sum t_s + max g_s, stage by stage; writes entry p.
+// The smallest boundaries from the caps at B* (recomputed stage by stage
+// from the stage words of column `owner`; `total` layers in all), then
+// Evaluate: T = (M-1) max t_s + sum t_s + max g_s; writes entry p.
 __device__ void eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int64_t p, int S, int M, int64_t n,
-                            int64_t Bstar, int set, int total) {
+                            int64_t Bstar, int total) {
     const int L = t.L;
     const int64_t c = a.wl_idx[p];
     const uint32_t* sw = t.sw + owner;
-    const uint8_t* caps = cap_set(t, owner, set);
     int64_t tmax = 0, tsum = 0;
     int sg = -1;
     // the stage with the largest G_s / (k_s bw_s), compared exactly: with
@@ -317,12 +305,13 @@ __device__ void eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int6
     int64_t pb_at = t.PB[0];
     for (int s = 0; s < S; ++s) {
         const uint32_t w = sw[s * kEqBlock];
-        const int k = caps[s * kEqBlock];
+        const Cap r = stage_cap(t, w, Bstar);
+        const int k = r.k;
         if (k < 1) atomicOr(a.err, kErrInternal);
         pre += k;
         const int nxt = s + 1 == S ? L : max(at + 1, L - (total - pre));
         if (a.bounds) a.bounds[(int64_t)(s + 1) * a.bstride + c] = (uint8_t)nxt;
-        const int64_t ts = (int64_t)(nxt - at) * t.q[w & 31] + t.p2p[(w >> 5) & 255];
+        const int64_t ts = (int64_t)(nxt - at) * r.q + r.c;
         tmax = max(tmax, ts);
         tsum += ts;
         if (n > 1) {
@@ -424,7 +413,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                    ? t.PB[1] - t.PB[0]
                    : -1;
     t.sw = reinterpret_cast<uint32_t*>(smem + el.sw);
-    t.caps = smem + el.caps;
     t.L = L;
     Search* tail = reinterpret_cast<Search*>(smem + el.tail);
     uint32_t* mysw = t.sw + threadIdx.x;
@@ -467,8 +455,8 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
 
         int S = 0, M = 0;
         int64_t n = 0;
-        int64_t Bstar = 0;  // with its cap set and layer count, unless queued
-        int bset = 0, btot = 0, slot = -1;
+        int64_t Bstar = 0;  // with its layer count, unless queued
+        int btot = 0, slot = -1;
         bool queued = false;
         if (have) {
             S = a.wl_S[p];
@@ -524,18 +512,15 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
             q.B = (int64_t)float_to_u64(fminf(Bf, fhi));
             q.Blo = q.Bhi = q.fhi = -1;
             q.clo = q.chi = 0;
-            q.fset = -1;
-            q.wset = 0;
             q.owner = (int16_t)threadIdx.x;
             q.S = (int16_t)S;
             q.probes = 0;
             q.p = (int32_t)p;
             q.M = (uint16_t)M;
             q.n = (uint16_t)n;
-            q.pad = 0;
             // one exact probe here; open searches go to the CTA's queue
             const bool done = q.lo >= q.hi || eq_step(t, q, a.err);
-            if (!(done && q.fset >= 0 && q.fhi == q.hi)) {
+            if (!(done && q.fhi == q.hi)) {
                 slot = atomicAdd(&tail_n, 1);
                 if (slot < kTailCap) {
                     tail[slot] = q;
@@ -546,7 +531,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                 }
             }
             Bstar = q.hi;
-            bset = q.fset;
             btot = q.chi;
             if (kCount) probes += q.probes;
         }
@@ -557,7 +541,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
             Search q = tail[i];
             eq_finish(t, q, a.err);
             tail[i].hi = q.hi;
-            tail[i].fset = q.fset;
             tail[i].chi = q.chi;
             if (kCount) probes += q.probes;
         }
@@ -565,10 +548,9 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
         if (queued) {
             const Search& q = tail[slot];
             Bstar = q.hi;
-            bset = q.fset;
             btot = q.chi;
         }
-        if (have) eq_evaluate(a, t, threadIdx.x, p, S, M, n, Bstar, bset, btot);
+        if (have) eq_evaluate(a, t, threadIdx.x, p, S, M, n, Bstar, btot);
         __syncthreads();  // columns and queue are reused by the next slice
     }
     if (kCount) {
