@@ -3,10 +3,15 @@
 // differ, one warp per worklist entry.
 //
 // The exact threshold search: a memory-only probe decides OOM (unless the
-// screen already knows a split fits) and bounds B*; a balanced first guess
-// gallops until the bracket closes, each probe snapping it to the largest
-// accepted or the smallest rejected stage time; the sets of the probe at B*
-// give the canonical split.  The probe (heddle_wprobe.cuh) judges 32
+// screen already knows a split fits) and bounds B*; the first guess solves
+// the saturating continuous balance of the equal-layer search with each
+// stage's average layer cost and its memory run from layer 0 (a few Newton
+// steps), then each probe snaps the bracket to the largest accepted or the
+// smallest rejected stage time and the next bound gallops from that value
+// (1, 2, 4, ... away) until both sides are known, then bisects.  The sets
+// of the probe at B* give the canonical split; a feasible probe that closes
+// the bracket already holds them (every bound in [hi, B] takes the same
+// decisions), so only a bracket closed from below costs a final probe.  The probe (heddle_wprobe.cuh) judges 32
 // positions per round with the interval test of this file: stage time
 // P[j] - P[i] + c and memory against k times the GPU memory.  Evaluate runs
 // one lane per stage: the stage times' maximum and sum, the stage with the
@@ -68,6 +73,40 @@ struct PlainJudge {
     }
 };
 
+// The first guess of B* (warp-uniform): the saturating continuous balance
+// sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2, with
+// each lane's stage given by 1 / q_s (rq, its average layer cost), c_s (cf)
+// and its memory run m_s (mr); at most three Newton steps from the
+// unsaturated balance, clamped to [max_s c_s + q_s, hi].
+__device__ int64_t first_guess(float rq, float cf, float mr, int S, int L, int64_t hi) {
+    const bool st = rq > 0.f;
+    float inv = rq, cw = cf * rq, flo = st ? cf + 1.0f / rq : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        inv += __shfl_xor_sync(kFull, inv, o);
+        cw += __shfl_xor_sync(kFull, cw, o);
+        flo = fmaxf(flo, __shfl_xor_sync(kFull, flo, o));
+    }
+    const float fhi = u64_to_float((uint64_t)hi);
+    float Bf = fmaxf(flo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : flo);
+    for (int it = 0; it < 3; ++it) {
+        Bf = fminf(Bf, fhi);
+        const float x = (Bf - cf) * rq;
+        const bool sat = !st || x >= mr;
+        float cnt = sat ? mr : x, sl = sat ? 0.f : rq, nb = sat ? 0.f : 1.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            cnt += __shfl_xor_sync(kFull, cnt, o);
+            sl += __shfl_xor_sync(kFull, sl, o);
+            nb += __shfl_xor_sync(kFull, nb, o);
+        }
+        const float tgt = (float)L + 0.5f * nb;
+        if (cnt >= tgt - 0.25f || sl <= 0.f) break;
+        Bf += (tgt - cnt) / sl;
+    }
+    return (int64_t)float_to_u64(fmaxf(fminf(Bf, fhi), 0.f));
+}
+
 template <bool kCount>
 __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -112,22 +151,25 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
             const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
             mine.c = t.p2p[(g * 8 + h) * 2 + same];
         }
-        // a bound feasible whenever memory is, and the balanced guess
+        // a bound feasible whenever memory is; the stage's average layer
+        // cost, P2P and memory run from layer 0 for the first guess
         int64_t hi = 0;
-        float inv = 0.f, cw = 0.f;
+        float rq = 0.f, cf = 0.f, mr = 0.f;
         if (live) {
             const int64_t all = t.P[mine.row + L];
             hi = all + mine.c;
-            const float tot = u64_to_float((uint64_t)all) + 1.0f;
-            inv = 1.0f / tot;
-            cw = u64_to_float((uint64_t)mine.c) / tot;
+            rq = all > 0 ? (float)L / u64_to_float((uint64_t)all) : 0.f;
+            cf = u64_to_float((uint64_t)mine.c);
+            int r0 = 0, r1 = L;  // the largest run [0, r) within memory
+            while (r0 < r1) {
+                const int mid = (r0 + r1 + 1) >> 1;
+                const longlong2 sm = t.SA[mid];
+                if ((sm.x - t.SA[0].x) + mine.f * (sm.y - t.SA[0].y) <= mine.capk) r0 = mid;
+                else r1 = mid - 1;
+            }
+            mr = (float)r0;
         }
         hi = wp::wmax64(hi);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            inv += __shfl_xor_sync(kFull, inv, o);
-            cw += __shfl_xor_sync(kFull, cw, o);
-        }
         const PlainJudge judge{t, mine};
         // one probe call site (the probe is large): phase 0 the memory-only
         // probe (OOM, else a tighter upper bound; skipped when the screen
@@ -138,13 +180,10 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         bool lo_known = false, hi_known = false, oom = false;
         int phase = memok ? 1 : 0, it = 0;
         if (memok) {
-            B = (int64_t)float_to_u64((1.0f + cw) / inv);
-            step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
+            B = min(max(first_guess(rq, cf, mr, S, L, hi), lo), hi - 1);
             if (lo >= hi) {
                 phase = 2;
                 B = hi;
-            } else {
-                B = min(max(B, lo), hi - 1);
             }
         }
         while (true) {
@@ -157,8 +196,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
                     break;
                 }
                 hi = shi;
-                B = (int64_t)float_to_u64((1.0f + cw) / inv);
-                step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
+                B = first_guess(rq, cf, mr, S, L, hi);
                 phase = 1;
             } else if (phase == 1) {
                 if (feas) {
@@ -172,7 +210,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
                     B = hi - step;
                     step *= 2;
                 } else if (!hi_known) {
-                    B = lo + step;
+                    B = lo + step - 1;
                     step *= 2;
                 } else {
                     B = lo + (hi - lo) / 2;
@@ -181,6 +219,8 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
                     if (lane == 0) atomicOr(a.err, kErrSearchBound);
                     lo = hi;
                 }
+                // closed by a feasible probe: its sets are those of B* = hi
+                if (lo >= hi && feas && it <= kMaxIters) break;
             } else {
                 if (!feas && lane == 0) atomicOr(a.err, kErrInternal);
                 break;
