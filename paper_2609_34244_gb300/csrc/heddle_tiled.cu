@@ -264,6 +264,34 @@ struct TiledJudge {
     }
 };
 
+// The first guess of B* (warp-collective, after the memory probe found a
+// split): each stage at its fastest allowed tiling's average layer cost,
+// with its P2P and its memory run from layer 0 without EDP copies (the
+// longest any tiling allows); not inlined, so the probe loop around it
+// keeps its registers.
+__device__ __noinline__ int64_t tiled_guess(const uint8_t* code, const int64_t* Pt, const longlong2* SA, int g, int j,
+                                            int64_t c, int64_t cap, int64_t f, bool live, int S, int L, int64_t hi) {
+    float rq = 0.f, cf = 0.f, mr = 0.f;
+    if (live) {
+        const int base = tile_base(j), cnt = (j + 1) * (j + 2) / 2;
+        int64_t all = kInf;
+        for (int o = 0; o < cnt; ++o)
+            if ((code[g * kTileSlots + base + o] & 0xc0) == 0x80)
+                all = min(all, Pt[(size_t)(g * kTileSlots + base + o) * (L + 1) + L]);
+        rq = all > 0 && all < kInf ? (float)L / u64_to_float((uint64_t)all) : 0.f;
+        cf = u64_to_float((uint64_t)c);
+        int r0 = 0, r1 = L;  // the largest run [0, r) within memory, no EDP copies
+        while (r0 < r1) {
+            const int mid = (r0 + r1 + 1) >> 1;
+            const longlong2 sm = SA[mid];
+            if ((sm.x - SA[0].x) + f * (sm.y - SA[0].y) <= cap) r0 = mid;
+            else r1 = mid - 1;
+        }
+        mr = (float)r0;
+    }
+    return wp::first_guess(rq, cf, mr, S, L, hi);
+}
+
 // element k of a 4-entry register array (k in [0, 3])
 template <class T>
 __device__ __forceinline__ T pick4(const T (&v)[4], int k) {
@@ -315,28 +343,10 @@ __global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, T
             mine.c = t.p2p[(mine.g * 8 + h) * 2 + same];
         }
         const TiledJudge judge{t, mine};
-        // first guess: the balanced bound with every stage at its fastest
-        // tiling over all layers
-        float inv = 0.f, cw = 0.f;
-        if (live) {
-            const int base = tile_base(mine.j), cnt = (mine.j + 1) * (mine.j + 2) / 2;
-            int64_t all = kInf;
-            for (int o = 0; o < cnt; ++o)
-                if ((t.code[mine.g * kTileSlots + base + o] & 0xc0) == 0x80)
-                    all = min(all, t.Pt[(size_t)(mine.g * kTileSlots + base + o) * (L + 1) + L]);
-            const float tot = u64_to_float((uint64_t)all) + 1.0f;
-            inv = 1.0f / tot;
-            cw = u64_to_float((uint64_t)mine.c) / tot;
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            inv += __shfl_xor_sync(wp::kFull, inv, o);
-            cw += __shfl_xor_sync(wp::kFull, cw, o);
-        }
         // one probe call site (the probe is large): phase 0 the memory-only
         // probe (OOM, else a feasible upper bound), phase 1 the threshold
-        // search galloping from the guess, phase 2 the probe at B* whose
-        // sets give the split
+        // search galloping from the snapped bounds, phase 2 the probe at B*
+        // whose sets give the split
         int64_t Bhi = 0, Blo = 0, B = kInf, step = 1;
         bool lo_known = false, hi_known = false, oom = false;
         int phase = 0, it = 0;
@@ -349,8 +359,7 @@ __global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, T
                     break;
                 }
                 Bhi = hi;
-                B = (int64_t)float_to_u64((1.0f + cw) / inv);
-                step = max((int64_t)1, (int64_t)float_to_u64(u64_to_float(B) * (float)S / (2.0f * (float)L)));
+                B = tiled_guess(t.code, t.Pt, t.SA, mine.g, mine.j, mine.c, mine.cap, mine.f, lane < S, S, L, Bhi);
                 phase = 1;
             } else if (phase == 1) {
                 if (feas) {
@@ -364,7 +373,7 @@ __global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, T
                     B = Bhi - step;
                     step *= 2;
                 } else if (!hi_known) {
-                    B = Blo + step;
+                    B = Blo + step - 1;
                     step *= 2;
                 } else {
                     B = Blo + (Bhi - Blo) / 2;

@@ -219,6 +219,40 @@ __device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int
     return feasible;
 }
 
+// The first guess of B* (warp-uniform): the saturating continuous balance
+// sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2, with
+// each lane's stage given by 1 / q_s (rq, its average layer cost), c_s (cf)
+// and its memory run m_s (mr); at most three Newton steps from the
+// unsaturated balance, clamped to [max_s c_s + q_s, hi].
+__device__ inline int64_t first_guess(float rq, float cf, float mr, int S, int L, int64_t hi) {
+    const bool st = rq > 0.f;
+    float inv = rq, cw = cf * rq, flo = st ? cf + 1.0f / rq : 0.f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        inv += __shfl_xor_sync(kFull, inv, o);
+        cw += __shfl_xor_sync(kFull, cw, o);
+        flo = fmaxf(flo, __shfl_xor_sync(kFull, flo, o));
+    }
+    const float fhi = u64_to_float((uint64_t)hi);
+    float Bf = fmaxf(flo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : flo);
+    for (int it = 0; it < 3; ++it) {
+        Bf = fminf(Bf, fhi);
+        const float x = (Bf - cf) * rq;
+        const bool sat = !st || x >= mr;
+        float cnt = sat ? mr : x, sl = sat ? 0.f : rq, nb = sat ? 0.f : 1.f;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            cnt += __shfl_xor_sync(kFull, cnt, o);
+            sl += __shfl_xor_sync(kFull, sl, o);
+            nb += __shfl_xor_sync(kFull, nb, o);
+        }
+        const float tgt = (float)L + 0.5f * nb;
+        if (cnt >= tgt - 0.25f || sl <= 0.f) break;
+        Bf += (tgt - cnt) / sl;
+    }
+    return (int64_t)float_to_u64(fmaxf(fminf(Bf, fhi), 0.f));
+}
+
 // The canonical split from the sets of a feasible probe at B*, by lane 0
 // into wa.A (a_{s+1} = the smallest element of C_{s+1} above a_s); false if
 // a set ran out (never expected after a feasible probe).

@@ -73,38 +73,26 @@ struct PlainJudge {
     }
 };
 
-// The first guess of B* (warp-uniform): the saturating continuous balance
-// sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2, with
-// each lane's stage given by 1 / q_s (rq, its average layer cost), c_s (cf)
-// and its memory run m_s (mr); at most three Newton steps from the
-// unsaturated balance, clamped to [max_s c_s + q_s, hi].
-__device__ int64_t first_guess(float rq, float cf, float mr, int S, int L, int64_t hi) {
-    const bool st = rq > 0.f;
-    float inv = rq, cw = cf * rq, flo = st ? cf + 1.0f / rq : 0.f;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        inv += __shfl_xor_sync(kFull, inv, o);
-        cw += __shfl_xor_sync(kFull, cw, o);
-        flo = fmaxf(flo, __shfl_xor_sync(kFull, flo, o));
-    }
-    const float fhi = u64_to_float((uint64_t)hi);
-    float Bf = fmaxf(flo, inv > 0.f ? ((float)L + 0.5f * (float)S + cw) / inv : flo);
-    for (int it = 0; it < 3; ++it) {
-        Bf = fminf(Bf, fhi);
-        const float x = (Bf - cf) * rq;
-        const bool sat = !st || x >= mr;
-        float cnt = sat ? mr : x, sl = sat ? 0.f : rq, nb = sat ? 0.f : 1.f;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            cnt += __shfl_xor_sync(kFull, cnt, o);
-            sl += __shfl_xor_sync(kFull, sl, o);
-            nb += __shfl_xor_sync(kFull, nb, o);
+// The first guess of B* (warp-collective): each stage's average layer cost,
+// P2P and memory run from layer 0 into the saturating balance; not
+// inlined, so the probe loop around it keeps its registers.
+__device__ __noinline__ int64_t plain_guess(const int64_t* P, const longlong2* SA, int row, int64_t c, int64_t capk,
+                                            int64_t f, bool live, int S, int L, int64_t hi) {
+    float rq = 0.f, cf = 0.f, mr = 0.f;
+    if (live) {
+        const int64_t all = P[row + L];
+        rq = all > 0 ? (float)L / u64_to_float((uint64_t)all) : 0.f;
+        cf = u64_to_float((uint64_t)c);
+        int r0 = 0, r1 = L;  // the largest run [0, r) within memory
+        while (r0 < r1) {
+            const int mid = (r0 + r1 + 1) >> 1;
+            const longlong2 sm = SA[mid];
+            if ((sm.x - SA[0].x) + f * (sm.y - SA[0].y) <= capk) r0 = mid;
+            else r1 = mid - 1;
         }
-        const float tgt = (float)L + 0.5f * nb;
-        if (cnt >= tgt - 0.25f || sl <= 0.f) break;
-        Bf += (tgt - cnt) / sl;
+        mr = (float)r0;
     }
-    return (int64_t)float_to_u64(fmaxf(fminf(Bf, fhi), 0.f));
+    return wp::first_guess(rq, cf, mr, S, L, hi);
 }
 
 template <bool kCount>
@@ -151,24 +139,8 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
             const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
             mine.c = t.p2p[(g * 8 + h) * 2 + same];
         }
-        // a bound feasible whenever memory is; the stage's average layer
-        // cost, P2P and memory run from layer 0 for the first guess
-        int64_t hi = 0;
-        float rq = 0.f, cf = 0.f, mr = 0.f;
-        if (live) {
-            const int64_t all = t.P[mine.row + L];
-            hi = all + mine.c;
-            rq = all > 0 ? (float)L / u64_to_float((uint64_t)all) : 0.f;
-            cf = u64_to_float((uint64_t)mine.c);
-            int r0 = 0, r1 = L;  // the largest run [0, r) within memory
-            while (r0 < r1) {
-                const int mid = (r0 + r1 + 1) >> 1;
-                const longlong2 sm = t.SA[mid];
-                if ((sm.x - t.SA[0].x) + mine.f * (sm.y - t.SA[0].y) <= mine.capk) r0 = mid;
-                else r1 = mid - 1;
-            }
-            mr = (float)r0;
-        }
+        // a bound feasible whenever memory is
+        int64_t hi = live ? t.P[mine.row + L] + mine.c : 0;
         hi = wp::wmax64(hi);
         const PlainJudge judge{t, mine};
         // one probe call site (the probe is large): phase 0 the memory-only
@@ -180,7 +152,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         bool lo_known = false, hi_known = false, oom = false;
         int phase = memok ? 1 : 0, it = 0;
         if (memok) {
-            B = min(max(first_guess(rq, cf, mr, S, L, hi), lo), hi - 1);
+            B = min(max(plain_guess(t.P, t.SA, mine.row, mine.c, mine.capk, mine.f, live, S, L, hi), lo), hi - 1);
             if (lo >= hi) {
                 phase = 2;
                 B = hi;
@@ -196,7 +168,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
                     break;
                 }
                 hi = shi;
-                B = first_guess(rq, cf, mr, S, L, hi);
+                B = plain_guess(t.P, t.SA, mine.row, mine.c, mine.capk, mine.f, live, S, L, hi);
                 phase = 1;
             } else if (phase == 1) {
                 if (feas) {
