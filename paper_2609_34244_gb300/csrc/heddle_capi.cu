@@ -34,7 +34,7 @@ struct heddle_ctx {
     size_t img_cap = 0;
     int64_t* d_q = nullptr;
     size_t q_cap = 0;
-    uint32_t* d_flags = nullptr;            // [0] table build, [1] device errors
+    uint32_t* d_flags = nullptr;            // [0] table build, [1] device errors, [2] top-k threshold
     unsigned long long* d_counters = nullptr;  // [3]
     bool count_next = false;
     // search worklist scratch (hd::kWorklistCap candidates); the second
@@ -53,6 +53,10 @@ struct heddle_ctx {
         uint8_t* code = nullptr;
         int64_t* T = nullptr;
         uint32_t* nM = nullptr;
+        // survivors of the top-k threshold (equal-layer search in a top-k pricing)
+        int32_t* sv_idx = nullptr;
+        int64_t* sv_T = nullptr;
+        uint32_t* sv_nM = nullptr;
     };
     Worklist wl[2];
     bool pipe_ready = false;
@@ -426,6 +430,9 @@ cudaError_t alloc_worklist(heddle_ctx::Worklist& w) {
     if (e == cudaSuccess) e = cudaMalloc(&w.code, (size_t)HEDDLE_MAX_STAGES * cap);
     if (e == cudaSuccess) e = cudaMalloc(&w.T, sizeof(int64_t) * cap);
     if (e == cudaSuccess) e = cudaMalloc(&w.nM, sizeof(uint32_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.sv_idx, sizeof(int32_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.sv_T, sizeof(int64_t) * cap);
+    if (e == cudaSuccess) e = cudaMalloc(&w.sv_nM, sizeof(uint32_t) * cap);
     return e;
 }
 
@@ -440,6 +447,9 @@ void free_worklist(heddle_ctx::Worklist& w) {
     cudaFree(w.code);
     cudaFree(w.T);
     cudaFree(w.nM);
+    cudaFree(w.sv_idx);
+    cudaFree(w.sv_T);
+    cudaFree(w.sv_nM);
     w = heddle_ctx::Worklist{};
 }
 
@@ -464,8 +474,8 @@ heddle_status heddle_create(heddle_ctx** out, int32_t device) {
     }
     x->num_sms = prop.multiProcessorCount;
     x->scratch_blocks = 8 * x->num_sms;  // per-CTA lists of the top-k and of the fused search
-    cudaError_t e = cudaMalloc(&x->d_flags, 2 * sizeof(uint32_t));
-    if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, 2 * sizeof(uint32_t));
+    cudaError_t e = cudaMalloc(&x->d_flags, 4 * sizeof(uint32_t));
+    if (e == cudaSuccess) e = cudaMemset(x->d_flags, 0, 4 * sizeof(uint32_t));
     if (e == cudaSuccess) e = cudaMalloc(&x->d_counters, 3 * sizeof(unsigned long long));
     if (e == cudaSuccess) e = cudaMemset(x->d_counters, 0, 3 * sizeof(unsigned long long));
     if (e == cudaSuccess)
@@ -740,6 +750,14 @@ heddle_status price_chunk(heddle_ctx* x, hd::PriceArgs& a, const heddle_candidat
     a.wl_bucket = W.bucket;
     a.wl_T = W.T;
     a.wl_nM = W.nM;
+    // inside a top-k pricing the equal-layer search hands the top-k only the
+    // entries that reach the running threshold
+    const bool survivors = state && a.uniform && !a.split_mode && !tiled;
+    a.sv_count = survivors ? W.count + hd::kWlSurv : nullptr;
+    a.sv_idx = W.sv_idx;
+    a.sv_T = W.sv_T;
+    a.sv_nM = W.sv_nM;
+    a.thr = x->d_flags + 2;
     a.S = c->S + lo;
     a.M = c->M + lo;
     a.code = c->code + lo;
@@ -779,11 +797,12 @@ heddle_status price_chunk(heddle_ctx* x, hd::PriceArgs& a, const heddle_candidat
         // top-k over the searched candidates of this chunk only
         hd::TopkArgs m = topk_args(x, state);
         m.base_index = c->base_index + lo;
-        m.wl_count = W.count;
-        m.wl_idx = W.idx;
-        m.wl_T = W.T;
-        m.wl_nM = W.nM;
+        m.wl_count = survivors ? W.count + hd::kWlSurv : W.count;
+        m.wl_idx = survivors ? W.sv_idx : W.idx;
+        m.wl_T = survivors ? W.sv_T : W.T;
+        m.wl_nM = survivors ? W.sv_nM : W.nM;
         m.wl_cap = hd::kWorklistCap;
+        m.thr = x->d_flags + 2;
         CU(hd::launch_topk_worklist(m, nb, x->num_sms, cs, nl ? nl + 2 : nullptr));
         if (x->time_phases) CU(cudaEventRecord(rec.e[4], cs));
     }
@@ -821,6 +840,9 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     const cudaStream_t cs = (cudaStream_t)stream;
     const int64_t chunk = x->chunk;
     const bool pipe = c->n > chunk;
+    // the threshold starts at zero for each call: the state may have been
+    // reset or replaced since the last one
+    if (state) CU(cudaMemsetAsync(x->d_flags + 2, 0, sizeof(uint32_t), cs));
     if (pipe) {
         if ((st = ensure_pipeline(x)) != HEDDLE_OK) return st;
         CU(cudaEventRecord(x->ev_in, cs));
@@ -1015,6 +1037,7 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         x->stage_smax = sm;
     }
     CU(cudaMemcpyAsync(x->d_state, state, sizeof(heddle_topk_state), cudaMemcpyHostToDevice, sc));
+    CU(cudaMemsetAsync(x->d_flags + 2, 0, sizeof(uint32_t), sc));
     for (int b = 0; b < heddle_ctx::kStageSets; ++b) CU(cudaEventRecord(x->ev_free[b], sc));
     const bool want_bounds = r && r->bounds;
     // batch k: copies in on s_h2d into staging set k % 3 (free once batch

@@ -289,9 +289,10 @@ __device__ void eq_finish(const EqTabs& t, Search& q, uint32_t* err) {
 
 // The smallest boundaries from the caps at B* (recomputed stage by stage
 // from the stage words of column `owner`; `total` layers in all), then
-// Evaluate: T = (M-1) max t_s + sum t_s + max g_s; writes entry p.
-__device__ void eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int64_t p, int S, int M, int64_t n,
-                            int64_t Bstar, int total) {
+// Evaluate: T = (M-1) max t_s + sum t_s + max g_s; writes entry p and
+// returns T.
+__device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int64_t p, int S, int M, int64_t n,
+                               int64_t Bstar, int total) {
     const int L = t.L;
     const int64_t c = a.wl_idx[p];
     const uint32_t* sw = t.sw + owner;
@@ -359,6 +360,7 @@ __device__ void eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int6
     a.B[c] = Bstar;
     a.ndp[c] = (uint16_t)n;
     a.status[c] = HEDDLE_CAND_OK;
+    return T;
 }
 
 template <bool kCount>
@@ -550,7 +552,28 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
             Bstar = q.hi;
             btot = q.chi;
         }
-        if (have) eq_evaluate(a, t, threadIdx.x, p, S, M, n, Bstar, btot);
+        int64_t T = -1;
+        if (have) T = eq_evaluate(a, t, threadIdx.x, p, S, M, n, Bstar, btot);
+        if (a.sv_count) {
+            // inside a top-k pricing: the entries whose n*M / T reaches the
+            // running threshold (float, below the k-th key by a margin that
+            // covers the rounding) go to the top-k's survivor list
+            const uint32_t nM = (uint32_t)n * (uint32_t)M;
+            const float thr = __uint_as_float(__ldcg(a.thr));
+            const bool keep = have && T > 0 && (float)nM / (float)T >= thr;
+            const unsigned mask = __ballot_sync(0xffffffffu, keep);
+            if (mask) {
+                const int lane = threadIdx.x & 31;
+                int base0 = 0;
+                if (lane == __ffs(mask) - 1) base0 = atomicAdd(a.sv_count, __popc(mask));
+                const int pos = __shfl_sync(0xffffffffu, base0, __ffs(mask) - 1) + __popc(mask & ((1u << lane) - 1));
+                if (keep && pos < a.wl_cap) {
+                    a.sv_idx[pos] = a.wl_idx[p];
+                    a.sv_T[pos] = T;
+                    a.sv_nM[pos] = nM;
+                }
+            }
+        }
         __syncthreads();  // columns and queue are reused by the next slice
     }
     if (kCount) {

@@ -133,6 +133,16 @@ struct PriceArgs {
     // so a top-k can run over the searched candidates only
     int64_t* wl_T;
     uint32_t* wl_nM;
+    // survivors of the top-k threshold (equal-layer search inside a top-k
+    // pricing; sv_count null otherwise): OK entries whose n*M / T, in
+    // float, is at least the float threshold *thr are appended as (chunk
+    // index, T, n*M).  *thr never exceeds the running top-k's k-th key
+    // (see TopkArgs::thr), so no entry that can enter the top-k is left out.
+    int32_t* sv_count;
+    int32_t* sv_idx;
+    int64_t* sv_T;
+    uint32_t* sv_nM;
+    const uint32_t* thr;
 };
 // Prices candidates [0, a.n) with a.n <= a.wl_cap: screen, then search.
 // `mid` (nullable) is recorded on st between the two; `launches` (nullable)
@@ -178,7 +188,8 @@ cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st);
 // The paper's own layer split over the worklist (comparison mode).
 cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
-constexpr int kWlMeta = 1 + kMaxStages + 1;  // ints of a.wl_count
+constexpr int kWlMeta = 1 + kMaxStages + 1 + 1;  // ints of a.wl_count
+constexpr int kWlSurv = kWlMeta - 1;             // the survivor count (see PriceArgs::sv_count)
 
 
 struct TopkArgs {
@@ -205,6 +216,13 @@ struct TopkArgs {
     TopkEntry* scratch2;
     int32_t* scratch2_count;
     int32_t* tickets;
+    // nullable: raised (atomicMax on the bits of a positive float) to the
+    // new state's k-th key n*M / T in float times (1 - 2^-16) once the state
+    // holds k entries.  Float conversions and the division are each within
+    // 2^-24 relative, so the stored value stays below every key at least
+    // the k-th's, exactly compared, by more than the rounding of a key
+    // computed the same way.
+    uint32_t* thr;
 };
 // `launches` (nullable) gains the number of kernels launched.
 cudaError_t launch_topk(const TopkArgs& a, int num_sms, cudaStream_t st, int64_t* launches = nullptr);

@@ -166,6 +166,10 @@ cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st, int64_t*
 // tickets for the next launch.
 constexpr int kFusedBlock = 256;
 constexpr int kFusedGroups = 4;
+// at most this many entries (typically the survivors of the threshold once
+// a pricing's first chunks have filled the state): CTA 0 alone merges them
+// with the state and the other CTAs leave at once
+constexpr int kFewEntries = 4096;
 
 // Stage lists [first, first + nl) of src into lists[0 ..), one warp per
 // list; the entries were written by other CTAs, so they are read past L1.
@@ -224,13 +228,16 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     bar.T = full ? a.state->T[k - 1] : 0;
     bar.nM = full ? a.state->nM[k - 1] : 0;
     bar.pad = 0;
-    // ---- this CTA's share of the worklist
+    // ---- this CTA's share of the worklist (all of it when it is short)
     int cnt = 0;
     TopkEntry* list = lists + warp * kMaxTopK;
     const int64_t n = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t step = (int64_t)gridDim.x * W * 32;
+    const bool few = n <= kFewEntries;
+    if (few && blockIdx.x != 0) return;
+    const int64_t step = few ? (int64_t)W * 32 : (int64_t)gridDim.x * W * 32;
+    const int64_t start = few ? (int64_t)warp * 32 : ((int64_t)blockIdx.x * W + warp) * 32;
     constexpr int U = 4;
-    for (int64_t base = ((int64_t)blockIdx.x * W + warp) * 32; base < n; base += step * U) {
+    for (int64_t base = start; base < n; base += step * U) {
         TopkEntry e[U];
         bool valid[U];
 #pragma unroll
@@ -248,19 +255,24 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     }
     if (lane == 0) counts[warp] = cnt;
     cta_tree_merge(lists, counts, tmp, tmp_counts, W, k);
-    // ---- the last CTA of its group merges the group's lists
-    const int group = blockIdx.x / kFan, ngroups = (gridDim.x + kFan - 1) / kFan;
-    const int first = group * kFan, gsize = min(kFan, (int)gridDim.x - first);
-    if (!publish(lists, counts, a.scratch + (size_t)blockIdx.x * kMaxTopK, a.scratch_count + blockIdx.x,
-                 a.tickets + group, gsize, &last_flag))
-        return;
-    stage_lists<W>(lists, counts, a.scratch, a.scratch_count, first, gsize, k);
-    cta_tree_merge(lists, counts, tmp, tmp_counts, gsize, k);
-    // ---- the last group folds the group lists and the incoming state
-    if (!publish(lists, counts, a.scratch2 + (size_t)group * kMaxTopK, a.scratch2_count + group,
-                 a.tickets + kFan, ngroups, &last_flag))
-        return;
-    stage_lists<W>(lists, counts, a.scratch2, a.scratch2_count, 0, ngroups, k);
+    int nl = 1;  // lists to fold with the incoming state
+    if (!few) {
+        // ---- the last CTA of its group merges the group's lists
+        const int group = blockIdx.x / kFan, ngroups = (gridDim.x + kFan - 1) / kFan;
+        const int first = group * kFan, gsize = min(kFan, (int)gridDim.x - first);
+        if (!publish(lists, counts, a.scratch + (size_t)blockIdx.x * kMaxTopK, a.scratch_count + blockIdx.x,
+                     a.tickets + group, gsize, &last_flag))
+            return;
+        stage_lists<W>(lists, counts, a.scratch, a.scratch_count, first, gsize, k);
+        cta_tree_merge(lists, counts, tmp, tmp_counts, gsize, k);
+        // ---- the last group folds the group lists and the incoming state
+        if (!publish(lists, counts, a.scratch2 + (size_t)group * kMaxTopK, a.scratch2_count + group,
+                     a.tickets + kFan, ngroups, &last_flag))
+            return;
+        stage_lists<W>(lists, counts, a.scratch2, a.scratch2_count, 0, ngroups, k);
+        nl = ngroups;
+    }
+    const int ngroups = nl;
     if (warp == W - 1) {
         const int c = min(max(a.state->count, 0), k);
         for (int i = lane; i < c; i += 32) {
@@ -281,9 +293,19 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
         a.state->T[p] = live ? lists[p].T : -1;
         a.state->nM[p] = live ? lists[p].nM : 0;
     }
-    if (threadIdx.x == 0) a.state->count = total;
-    // every other CTA has drawn its tickets: clear them for the next launch
-    for (int i = threadIdx.x; i <= kFan; i += blockDim.x) a.tickets[i] = 0;
+    if (threadIdx.x == 0) {
+        a.state->count = total;
+        if (a.thr && total >= k) {
+            // the new k-th key, rounded and lowered by 2^-16 (see TopkArgs::thr)
+            const TopkEntry e = lists[k - 1];
+            const float r = (float)e.nM / (float)e.T * (1.0f - 1.0f / 65536.0f);
+            atomicMax(a.thr, __float_as_uint(r));
+        }
+    }
+    // every other CTA has drawn its tickets (none did on the short path):
+    // clear them for the next launch
+    if (!few)
+        for (int i = threadIdx.x; i <= kFan; i += blockDim.x) a.tickets[i] = 0;
 }
 
 __global__ void topk_reset_kernel(heddle_topk_state* s, int k) {

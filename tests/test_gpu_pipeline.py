@@ -156,3 +156,54 @@ def test_host_path_batch_limit(h, W):
         assert e.value.status == h.E_LIMIT
     finally:
         h.heddle_destroy(ctx)
+
+
+def test_threshold_restarts_each_call(h, W, oracle_mod):
+    """Inside a top-k pricing the equal-layer search hands the top-k only the
+    entries that reach a running threshold below the state's k-th key.  The
+    threshold restarts with every call: after a reset, a call whose entries
+    are all worse than the previous call's k-th still finds its own exact
+    top-k, and calls continuing a full state (two halves) merge exactly,
+    through device buffers and through host buffers."""
+    import torch
+    w = W.make_workload("stress128", seed=7, n=120011)
+    ref = oracle_mod.Oracle(w.cluster, w.model).price(w.cands, threads=8)
+    nM = ref["n_dp"].astype(np.int64) * w.cands["M"].astype(np.int64)
+    ok = np.nonzero(ref["status"] == 0)[0]
+    key = nM[ok].astype(np.float64) / ref["T"][ok].astype(np.float64)
+    best = ok[np.argsort(-key, kind="stable")[:3000]]
+    worse = {k2: v.copy() for k2, v in w.cands.items()}
+    worse["S"][best] = 0  # invalid: every remaining entry is below the first call's k-th
+    rest = np.setdiff1d(ok, best)
+    expect = [e[0] for e in G.exact_topk(rest, ref["T"][rest], nM[rest], 16)]
+    full = [e[0] for e in G.exact_topk(ok, ref["T"][ok], nM[ok], 16)]
+    n = w.n
+    ctx = h.heddle_create(0)
+    try:
+        h.heddle_load_cluster(ctx, w.cluster)
+        h.heddle_load_model(ctx, w.model)
+        h.heddle_set_chunk(ctx, 16411)
+        res = h.alloc_results(n, bounds=False)
+        state = h.alloc_topk_state()
+        for cands, want in ((w.cands, full), (worse, expect)):
+            dc = h.cands_to_device(cands)
+            h.heddle_topk_reset(ctx, state, 16)
+            h.heddle_price_topk(ctx, h.make_candidates(dc), h.make_results(res), state)
+            torch.cuda.synchronize()
+            assert h.read_topk_state(state)["idx"].tolist() == want
+        # two calls on halves of the worse set continue one state
+        h.heddle_topk_reset(ctx, state, 16)
+        for lo, hi in ((0, n // 2), (n // 2, n)):
+            h.heddle_price_topk(ctx, h.make_candidates(dc, lo, hi), h.make_results(res, lo, hi), state)
+        torch.cuda.synchronize()
+        assert h.read_topk_state(state)["idx"].tolist() == expect
+        # host buffers: the same sequence
+        for cands, want in ((w.cands, full), (worse, expect)):
+            pinned = {k2: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
+                      for k2, v in cands.items()}
+            st = h.new_topk_state(16)
+            h.heddle_price_topk_host(ctx, pinned, None, st, batch=16411)
+            assert h.topk_state_to_dict(st)["idx"].tolist() == want
+        assert h.heddle_device_errors(ctx) == 0
+    finally:
+        h.heddle_destroy(ctx)
