@@ -58,11 +58,15 @@ struct heddle_ctx {
         int64_t* sv_T = nullptr;
         uint32_t* sv_nM = nullptr;
     };
-    Worklist wl[2];
+    // three worklist sets: chunk i uses set i % 3, so it waits for the top-k
+    // of chunk i - 3 (the first chunk's, which fills an empty state, is the
+    // longest), not of chunk i - 2
+    static constexpr int kWlSets = 3;
+    Worklist wl[kWlSets];
     bool pipe_ready = false;
     cudaStream_t s_work[2] = {nullptr, nullptr};
     cudaEvent_t ev_in = nullptr;
-    cudaEvent_t ev_searched[2] = {nullptr, nullptr}, ev_wl_free[2] = {nullptr, nullptr};
+    cudaEvent_t ev_searched[kWlSets] = {}, ev_wl_free[kWlSets] = {};
     int64_t chunk = hd::kWorklistCap;
     // top-k merge scratch
     hd::TopkEntry* d_scratch = nullptr;
@@ -505,13 +509,13 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_counters);
     cudaFree(x->d_scratch);
     cudaFree(x->d_scratch_count);
-    free_worklist(x->wl[0]);
-    free_worklist(x->wl[1]);
-    for (int b = 0; b < 2; ++b) {
-        if (x->s_work[b]) cudaStreamDestroy(x->s_work[b]);
+    for (int b = 0; b < heddle_ctx::kWlSets; ++b) {
+        free_worklist(x->wl[b]);
         if (x->ev_searched[b]) cudaEventDestroy(x->ev_searched[b]);
         if (x->ev_wl_free[b]) cudaEventDestroy(x->ev_wl_free[b]);
     }
+    for (int b = 0; b < 2; ++b)
+        if (x->s_work[b]) cudaStreamDestroy(x->s_work[b]);
     if (x->ev_in) cudaEventDestroy(x->ev_in);
     cudaFree(x->d_scratch2);
     cudaFree(x->d_scratch2_count);
@@ -666,22 +670,23 @@ heddle_status heddle_load_experts(heddle_ctx* x, const int64_t* expert_state, co
 
 namespace {
 
-// The second worklist set, the work streams and their events (once).
+// The other worklist sets, the work streams and their events (once).
 heddle_status ensure_pipeline(heddle_ctx* x) {
     if (x->pipe_ready) return HEDDLE_OK;
-    cudaError_t e = alloc_worklist(x->wl[1]);
-    for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+    cudaError_t e = cudaSuccess;
+    for (int b = 1; b < heddle_ctx::kWlSets && e == cudaSuccess; ++b) e = alloc_worklist(x->wl[b]);
+    for (int b = 0; b < 2 && e == cudaSuccess; ++b)
         if (!x->s_work[b]) e = cudaStreamCreateWithFlags(&x->s_work[b], cudaStreamNonBlocking);
-        if (e == cudaSuccess && !x->ev_searched[b])
-            e = cudaEventCreateWithFlags(&x->ev_searched[b], cudaEventDisableTiming);
+    for (int b = 0; b < heddle_ctx::kWlSets && e == cudaSuccess; ++b) {
+        if (!x->ev_searched[b]) e = cudaEventCreateWithFlags(&x->ev_searched[b], cudaEventDisableTiming);
         if (e == cudaSuccess && !x->ev_wl_free[b])
             e = cudaEventCreateWithFlags(&x->ev_wl_free[b], cudaEventDisableTiming);
     }
     if (e == cudaSuccess && !x->ev_in) e = cudaEventCreateWithFlags(&x->ev_in, cudaEventDisableTiming);
     if (e != cudaSuccess) {
-        free_worklist(x->wl[1]);
+        for (int b = 1; b < heddle_ctx::kWlSets; ++b) free_worklist(x->wl[b]);
         return fail(x, e == cudaErrorMemoryAllocation ? HEDDLE_E_NOMEM : HEDDLE_E_CUDA,
-                    "second worklist set: %s", cudaGetErrorString(e));
+                    "pipeline worklist sets: %s", cudaGetErrorString(e));
     }
     x->pipe_ready = true;
     return HEDDLE_OK;
@@ -833,8 +838,8 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
     fill_price_args(x, c, lvl, shift, tiled, a);
     // chunks of at most x->chunk candidates.  With one chunk everything runs
     // on the caller's stream.  With more, chunk i runs its screen and search
-    // on work stream i % 2 with worklist set i % 2 (after the caller's
-    // earlier work and after chunk i - 2 released that set), and its top-k
+    // on work stream i % 2 with worklist set i % 3 (after the caller's
+    // earlier work and after chunk i - 3 released that set), and its top-k
     // on the caller's stream after its search, so the top-k merges stay in
     // chunk order while chunk i + 1 is screened and searched meanwhile.
     const cudaStream_t cs = (cudaStream_t)stream;
@@ -847,12 +852,12 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
         if ((st = ensure_pipeline(x)) != HEDDLE_OK) return st;
         CU(cudaEventRecord(x->ev_in, cs));
     }
-    bool used[2] = {false, false};
+    bool used[heddle_ctx::kWlSets] = {};
     int64_t i = 0;
     for (int64_t lo = 0; lo < c->n; lo += chunk, ++i) {
         const int64_t nb = c->n - lo < chunk ? c->n - lo : chunk;
-        const int b = pipe ? (int)(i & 1) : 0;
-        const cudaStream_t ws = pipe ? x->s_work[b] : cs;
+        const int b = pipe ? (int)(i % heddle_ctx::kWlSets) : 0;
+        const cudaStream_t ws = pipe ? x->s_work[i & 1] : cs;
         if (pipe) {
             CU(cudaStreamWaitEvent(ws, x->ev_in, 0));
             if (used[b]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[b], 0));
@@ -862,7 +867,7 @@ heddle_status price_impl(heddle_ctx* x, const heddle_candidates* c, const heddle
         if (pipe) CU(cudaEventRecord(x->ev_wl_free[b], state ? cs : ws));
     }
     if (pipe && !state)
-        for (int b = 0; b < 2; ++b)
+        for (int b = 0; b < heddle_ctx::kWlSets; ++b)
             if (used[b]) CU(cudaStreamWaitEvent(cs, x->ev_wl_free[b], 0));
     return ok(x);
 }
@@ -894,11 +899,11 @@ heddle_status price_units(heddle_ctx* x, const PriceUnit* u, int nu, void* strea
         if ((st = ensure_pipeline(x)) != HEDDLE_OK) return st;
         CU(cudaEventRecord(x->ev_in, cs));
     }
-    bool used[2] = {false, false};
+    bool used[heddle_ctx::kWlSets] = {};
     for (int k = 0; k < nu; ++k) {
         if (u[k].nb <= 0) continue;
-        const int b = pipe ? (k & 1) : 0;
-        const cudaStream_t ws = pipe ? x->s_work[b] : cs;
+        const int b = pipe ? (k % heddle_ctx::kWlSets) : 0;
+        const cudaStream_t ws = pipe ? x->s_work[k & 1] : cs;
         if (pipe) {
             CU(cudaStreamWaitEvent(ws, x->ev_in, 0));
             if (used[b]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[b], 0));
@@ -912,7 +917,7 @@ heddle_status price_units(heddle_ctx* x, const PriceUnit* u, int nu, void* strea
         if (pipe) CU(cudaEventRecord(x->ev_wl_free[b], ws));
     }
     if (pipe)
-        for (int b = 0; b < 2; ++b)
+        for (int b = 0; b < heddle_ctx::kWlSets; ++b)
             if (used[b]) CU(cudaStreamWaitEvent(cs, x->ev_wl_free[b], 0));
     return ok(x);
 }
@@ -1042,12 +1047,12 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
     const bool want_bounds = r && r->bounds;
     // batch k: copies in on s_h2d into staging set k % 3 (free once batch
     // k - 3 is copied out), screen and search on work stream k % 2 (worklist
-    // set k % 2, released by batch k - 2's top-k), top-k merge on the
+    // set k % 3, released by batch k - 3's top-k), top-k merge on the
     // caller's stream in batch order, copies out on s_d2h
-    bool used[2] = {false, false};
+    bool used[heddle_ctx::kWlSets] = {};
     for (int64_t lo = 0, it = 0; lo < n; lo += batch, ++it) {
         const int b = (int)(it % heddle_ctx::kStageSets);
-        const int wb = (int)(it & 1);
+        const int wb = (int)(it % heddle_ctx::kWlSets);
         const int64_t nb = (n - lo) < batch ? (n - lo) : batch;
         // host -> device on the copy stream once the set is free
         CU(cudaStreamWaitEvent(x->s_h2d, x->ev_free[b], 0));
@@ -1056,7 +1061,7 @@ heddle_status heddle_price_topk_host(heddle_ctx* x, const heddle_candidates* c,
         CU(cudaMemcpy2DAsync(x->st_code[b], nb, c->code + lo, c->plane_stride, nb, c->s_max,
                              cudaMemcpyHostToDevice, x->s_h2d));
         CU(cudaEventRecord(x->ev_loaded[b], x->s_h2d));
-        const cudaStream_t ws = x->s_work[wb];
+        const cudaStream_t ws = x->s_work[it & 1];
         CU(cudaStreamWaitEvent(ws, x->ev_loaded[b], 0));
         if (used[wb]) CU(cudaStreamWaitEvent(ws, x->ev_wl_free[wb], 0));
         used[wb] = true;
