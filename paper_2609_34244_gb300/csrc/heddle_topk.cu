@@ -19,7 +19,6 @@ namespace hd {
 namespace {
 
 constexpr int kTopkBlock = 256;
-constexpr int kWarps = kTopkBlock / 32;
 constexpr int kMergeBlock = 1024;  // warps 0-15 stage lists, warp 16 the state
 constexpr int kMergeWarps = kMergeBlock / 32;
 
