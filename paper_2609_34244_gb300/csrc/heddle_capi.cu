@@ -763,6 +763,7 @@ heddle_status price_chunk(heddle_ctx* x, hd::PriceArgs& a, const heddle_candidat
     a.sv_T = W.sv_T;
     a.sv_nM = W.sv_nM;
     a.thr = x->d_flags + 2;
+    a.topk_k = state ? &state->k : nullptr;
     a.S = c->S + lo;
     a.M = c->M + lo;
     a.code = c->code + lo;

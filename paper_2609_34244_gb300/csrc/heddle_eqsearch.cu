@@ -557,10 +557,33 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
         if (a.sv_count) {
             // inside a top-k pricing: the entries whose n*M / T reaches the
             // running threshold (float, below the k-th key by a margin that
-            // covers the rounding) go to the top-k's survivor list
+            // covers the rounding) go to the top-k's survivor list.  The
+            // warp first raises the threshold to its own k-th best key (for
+            // k <= 32): any k entries' smallest key is at most the call's
+            // final k-th, so the raised value keeps the filter exact
             const uint32_t nM = (uint32_t)n * (uint32_t)M;
-            const float thr = __uint_as_float(__ldcg(a.thr));
-            const bool keep = have && T > 0 && (float)nM / (float)T >= thr;
+            const float key = have && T > 0 ? (float)nM / (float)T : -1.0f;
+            const int lane = threadIdx.x & 31;
+            const int kk = min(max(__ldg(a.topk_k), 1), kMaxTopK);
+            float own = 0.f;
+            if (kk <= 32) {
+                float v = key;  // bitonic sort of the warp's keys, descending
+#pragma unroll
+                for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+                    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+                        const float o = __shfl_xor_sync(0xffffffffu, v, stride);
+                        const bool desc = (lane & size) == 0 || size == 32;
+                        v = (((lane & stride) == 0) == desc) ? fmaxf(v, o) : fminf(v, o);
+                    }
+                const float kth = __shfl_sync(0xffffffffu, v, kk - 1);
+                if (kth > 0.f) {
+                    own = kth * (1.0f - 1.0f / 65536.0f);
+                    if (lane == 0) atomicMax(a.thr, __float_as_uint(own));
+                }
+            }
+            const float thr = fmaxf(__uint_as_float(__ldcg(a.thr)), own);
+            const bool keep = key > 0.f && key >= thr;
             const unsigned mask = __ballot_sync(0xffffffffu, keep);
             if (mask) {
                 const int lane = threadIdx.x & 31;

@@ -142,7 +142,8 @@ struct PriceArgs {
     int32_t* sv_idx;
     int64_t* sv_T;
     uint32_t* sv_nM;
-    const uint32_t* thr;
+    uint32_t* thr;
+    const int32_t* topk_k;  // the state's k (device)
 };
 // Prices candidates [0, a.n) with a.n <= a.wl_cap: screen, then search.
 // `mid` (nullable) is recorded on st between the two; `launches` (nullable)
