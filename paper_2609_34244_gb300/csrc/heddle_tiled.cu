@@ -22,7 +22,7 @@
 //                  P_tiling[j] - P_tiling[i] + c_s (the earliest slot on
 //                  ties); monotone under interval inclusion
 //   PartitionLayers  the exact threshold search of the general search, its
-//                  probe (heddle_wprobe.cuh) judging 32 positions per round
+//                  probe (heddle_wprobe.cuh) checking 32 positions per round
 //                  with this stage time; the canonical split from the sets
 //                  at B*
 //   re-selection   one lane per stage keeps, per EDP exponent m, the
@@ -235,7 +235,7 @@ __device__ __forceinline__ bool tfits(const TTabs& t, const TLane& st, int i, in
 
 // The interval test of the tiled search: the fastest allowed, undominated
 // tiling whose memory fits (2 if none fits).
-struct TiledJudge {
+struct TiledCheck {
     typedef TLane Stage;
     const TTabs& t;
     TLane mine;  // the stage this lane holds
@@ -342,7 +342,7 @@ __global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, T
             const int same = (mine.g == h) && ((1 << mine.j) + (1 << jn) <= t.maxn[mine.g]);
             mine.c = t.p2p[(mine.g * 8 + h) * 2 + same];
         }
-        const TiledJudge judge{t, mine};
+        const TiledCheck check{t, mine};
         // one probe call site (the probe is large): phase 0 the memory-only
         // probe (OOM, else a feasible upper bound), phase 1 the threshold
         // search galloping from the snapped bounds, phase 2 the probe at B*
@@ -352,7 +352,7 @@ __global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, T
         int phase = 0, it = 0;
         while (true) {
             int64_t hi, lo;
-            const bool feas = wp::probe(judge, S, L, B, wa, hi, lo, checks);
+            const bool feas = wp::probe(check, S, L, B, wa, hi, lo, checks);
             if (phase == 0) {
                 if (!feas) {
                     oom = true;

@@ -15,11 +15,11 @@
 // the same decisions, so a search snaps its bracket to them and ends on B*;
 // the sets at B* give the canonical (lexicographically smallest) split.
 //
-// The 32 lanes judge 32 positions at once: a stage's forward reach is the
+// The 32 lanes check 32 positions at once: a stage's forward reach is the
 // first rejection among 32 consecutive ends, and a backward set is built
-// one 32-bit word per round -- lane l judges start 32 w + l against its
+// one 32-bit word per round -- lane l checks start 32 w + l against its
 // smallest successor (a bit scan of the successor set) and the ballot is
-// the word.  A judge type J supplies the stages and the interval test:
+// the word.  A check type J supplies the stages and the interval test:
 //   typename J::Stage J::stage(int s) const   -- every lane calls it
 //   int J::eval(const Stage&, int i, int j, int64_t B, int64_t* cost) const
 //       -- 0 fits (cost <= B), 1 too slow, 2 out of memory.
@@ -113,9 +113,9 @@ __device__ __forceinline__ int next_above(const uint32_t* C, int i, int L) {
 
 // Exact probe of bound B by one warp (all lanes call it; uniform result).
 // The sets land in wa; hi / lo are the snap values; checks counts the
-// interval judgements of this lane.
+// interval checks of this lane.
 template <class J>
-__device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int64_t& hi_out, int64_t& lo_out,
+__device__ bool probe(const J& check, int S, int L, int64_t B, WarpArea& wa, int64_t& hi_out, int64_t& lo_out,
                       unsigned long long& checks) {
     const int lane = threadIdx.x & 31;
     int64_t hi = -1, lo = kInf;
@@ -124,7 +124,7 @@ __device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int
     int u = 0;
     if (lane == 0) wa.U[0] = 0;
     for (int s = 0; s + 1 < S && ok; ++s) {
-        const typename J::Stage st = judge.stage(s);
+        const typename J::Stage st = check.stage(s);
         const int lim = L - (S - 1 - s);
         int reach = u;  // furthest accepted end (u: none yet)
         for (int base = u + 1; base <= lim; base += 32) {
@@ -132,7 +132,7 @@ __device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int
             int r = 1;  // beyond lim: treated as a rejection
             int64_t v = 0;
             if (j <= lim) {
-                r = judge.eval(st, u, j, B, &v);
+                r = check.eval(st, u, j, B, &v);
                 ++checks;
                 if (r == 0) hi = max(hi, v);
                 else if (r == 1) lo = min(lo, v);
@@ -163,7 +163,7 @@ __device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int
                 ok = false;
                 break;
             }
-            const typename J::Stage st = judge.stage(s);
+            const typename J::Stage st = check.stage(s);
             int any = 0, newmax = -1;
             for (int w = top >> 5; w >= (s >> 5); --w) {
                 const int i = (w << 5) + lane;
@@ -180,7 +180,7 @@ __device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int
                 int r = 3;
                 int64_t v = 0;
                 if (i >= s && i <= top && succ >= 0) {
-                    r = judge.eval(st, i, succ, B, &v);
+                    r = check.eval(st, i, succ, B, &v);
                     ++checks;
                     if (r == 0) hi = max(hi, v);
                     else if (r == 1) lo = min(lo, v);
@@ -200,10 +200,10 @@ __device__ bool probe(const J& judge, int S, int L, int64_t B, WarpArea& wa, int
     bool feasible = false;
     if (ok) {
         const int succ0 = S == 1 ? L : next_above(wa.C[1], 0, L);
-        const typename J::Stage st0 = judge.stage(0);
+        const typename J::Stage st0 = check.stage(0);
         if (succ0 >= 0 && lane == 0) {
             int64_t v = 0;
-            const int r = judge.eval(st0, 0, succ0, B, &v);
+            const int r = check.eval(st0, 0, succ0, B, &v);
             ++checks;
             if (r == 0) {
                 hi = max(hi, v);

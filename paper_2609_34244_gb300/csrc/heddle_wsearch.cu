@@ -11,7 +11,7 @@
 // (1, 2, 4, ... away) until both sides are known, then bisects.  The sets
 // of the probe at B* give the canonical split; a feasible probe that closes
 // the bracket already holds them (every bound in [hi, B] takes the same
-// decisions), so only a bracket closed from below costs a final probe.  The probe (heddle_wprobe.cuh) judges 32
+// decisions), so only a bracket closed from below costs a final probe.  The probe (heddle_wprobe.cuh) checks 32
 // positions per round with the interval test of this file: stage time
 // P[j] - P[i] + c and memory against k times the GPU memory.  Evaluate runs
 // one lane per stage: the stage times' maximum and sum, the stage with the
@@ -52,7 +52,7 @@ struct WStage {
 
 // The interval test of the general search: stage time P[j] - P[i] + c and
 // memory (S[j] - S[i]) + f (A[j] - A[i]) against k times the GPU memory.
-struct PlainJudge {
+struct PlainCheck {
     typedef WStage Stage;
     const WTabs& t;
     WStage mine;  // the stage this lane holds
@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         // a bound feasible whenever memory is
         int64_t hi = live ? t.P[mine.row + L] + mine.c : 0;
         hi = wp::wmax64(hi);
-        const PlainJudge judge{t, mine};
+        const PlainCheck check{t, mine};
         // one probe call site (the probe is large): phase 0 the memory-only
         // probe (OOM, else a tighter upper bound; skipped when the screen
         // knows a split fits), phase 1 the threshold search galloping from
@@ -161,7 +161,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         while (true) {
             int64_t shi, slo;
             if (kCount && lane == 0) ++probes;
-            const bool feas = wp::probe(judge, S, L, B, wa, shi, slo, checks);
+            const bool feas = wp::probe(check, S, L, B, wa, shi, slo, checks);
             if (phase == 0) {
                 if (!feas) {
                     oom = true;
