@@ -52,7 +52,7 @@ constexpr int kEqBlock = 128;
 constexpr int kZeroP2P = 128;  // a zero entry after the 8 x 8 x 2 P2P table
 constexpr int kMaxIters = 256;
 
-constexpr int kTailCap = 32;  // open searches queued per slice
+constexpr int kTailCap = 48;  // open searches queued per slice
 
 // State of one threshold search.
 struct Search {
