@@ -40,9 +40,9 @@ __device__ __forceinline__ uint32_t div_small(uint32_t a, uint32_t d, const uint
     return __umulhi(a << 8, magic[d]);
 }
 
-// Per stage byte: bit 31 inadmissible; bits 24-26 type; bits 16-21 the bit
-// position of the stage's GPUs in the type's demand word (degree bits +
-// 16 * unit class); bits 0-10 the row (type, degree) of the run table.
+// Per stage byte: bit 31 inadmissible; bits 24-26 type; bits 16-20 the bit
+// that adds the stage's units to its type's demand word; bits 0-10 the row
+// (type, degree) of the run table.
 __device__ __forceinline__ uint32_t stage_desc(int b, const Layout& y, const unsigned char* img, int moe) {
     const int32_t* gmaxn = reinterpret_cast<const int32_t*>(img + y.offMaxN);
     const int32_t* gpow2 = reinterpret_cast<const int32_t*>(img + y.offPow2);
@@ -51,7 +51,11 @@ __device__ __forceinline__ uint32_t stage_desc(int b, const Layout& y, const uns
     if ((b >> 5) != 0 || g >= y.NT || ggpus[g] <= 0 || (!moe && (1 << j) > gmaxn[g])) return 1u << 31;
     const int unit = (1 << j) <= gmaxn[g] ? (1 << j) : gpow2[g];
     const int uc = 31 - __clz(unit);
-    return ((uint32_t)g << 24) | ((uint32_t)(j + 16 * uc) << 16) | (uint32_t)((g * 4 + j) * 33);
+    // the stage adds 2^(j - uc) units of 2^uc GPUs to field uc of its type's
+    // demand word (fields of 9, 8, 7 and 6 bits at bits 0, 9, 17, 24: at
+    // most 32 stages x 8 / 2^uc units)
+    const int off = uc == 0 ? 0 : uc == 1 ? 9 : uc == 2 ? 17 : 24;
+    return ((uint32_t)g << 24) | ((uint32_t)(j - uc + off) << 16) | (uint32_t)((g * 4 + j) * 33);
 }
 
 // Steps 1-2 and the memory screen for every candidate of the batch.  Each
@@ -65,7 +69,7 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
     __shared__ uint8_t win[8 * 4 * 33];
     __shared__ __align__(16) uint32_t cap[8 * 4];
     __shared__ uint32_t magic[257];
-    __shared__ uint64_t dem[8 * kScreenBlock];  // per-thread GPUs per unit class, 4 x 16 bits per type
+    __shared__ uint32_t dem[8 * kScreenBlock];  // per-thread units per class (see stage_desc), per type
     __shared__ __align__(16) uint8_t tile[kMaxStages * kScreenBlock];  // [stage][candidate of the slice]
     __shared__ uint8_t sS[kScreenBlock];
     __shared__ uint16_t sM[kScreenBlock];
@@ -84,7 +88,7 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
     const bool memuni = reinterpret_cast<const int32_t*>(a.img + y.offModel)[0] != 0;
     const int s_lim = min(min(kMaxStages, a.s_max), L);
     const bool vec16 = ((reinterpret_cast<uintptr_t>(a.code) | (uintptr_t)a.stride) & 15) == 0;
-    uint64_t* mydem = dem + threadIdx.x;
+    uint32_t* mydem = dem + threadIdx.x;
     const int lane = threadIdx.x & 31;
     for (int64_t c0 = (int64_t)blockIdx.x * kScreenBlock; c0 < a.n; c0 += (int64_t)gridDim.x * kScreenBlock) {
         const int nloc = (int)min((int64_t)kScreenBlock, a.n - c0);
@@ -162,7 +166,7 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                     const uint32_t d = desc[col[s * kScreenBlock]];
                     bad |= d;
                     const int g = (d >> 24) & 7;
-                    mydem[g * kScreenBlock] += 1ull << ((d >> 16) & 63);
+                    mydem[g * kScreenBlock] += 1u << ((d >> 16) & 31);
                     const int w = win[(d & 0x7ff) + min(S - s, M)];
                     run_sum += w;
                     run_min = min(run_min, w);
@@ -178,10 +182,11 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                     uint32_t nn = 0xffffffffu;
 #pragma unroll
                     for (int g = 0; g < 8; ++g) {
-                        const uint64_t v = mydem[g * kScreenBlock];
+                        const uint32_t v = mydem[g * kScreenBlock];
                         const uint4 cg = *reinterpret_cast<const uint4*>(cap + g * 4);
-                        const uint32_t f3 = (uint32_t)(v >> 48), f2 = (uint32_t)(v >> 32) & 0xffffu;
-                        const uint32_t f1 = (uint32_t)(v >> 16) & 0xffffu, f0 = (uint32_t)v & 0xffffu;
+                        // GPUs per class from the unit counts
+                        const uint32_t f3 = (v >> 24) << 3, f2 = ((v >> 17) & 0x7fu) << 2;
+                        const uint32_t f1 = ((v >> 9) & 0xffu) << 1, f0 = v & 0x1ffu;
                         const uint32_t d3 = f3, d2 = d3 + f2, d1 = d2 + f1, d0 = d1 + f0;
                         const uint32_t q3 = div_small(cg.w, d3, magic), q2 = div_small(cg.z, d2, magic);
                         const uint32_t q1 = div_small(cg.y, d1, magic), q0 = div_small(cg.x, d0, magic);
