@@ -1,52 +1,79 @@
-"""Full-size workloads in the benchmark's launch configuration (device-resident
-batches of at most 1e6 candidates priced and merged into one top-k state):
-every sampled candidate bit-exact against the oracle, the top-k equal to an
-exact host top-k of the GPU's own per-candidate outputs, and every top-k
-entry re-priced by the oracle."""
+"""Full-size workloads in the benchmark's launch configuration, compared with
+the oracle on every candidate.
+
+The oracle prices every candidate of each full-size workload here (all host
+threads; the 1e7-candidate stress workload takes a minute or two on 16
+cores), once per session.  Its results must also reproduce the digests in
+``golden/fullsize_oracle.json`` (written by the oracle alone), which pins the
+seeded inputs and the oracle's own output on this host to the ones stored.
+The GPU path -- one pricing call over all candidates in chunks of 1e6, as
+the benchmark times it, and separately one price + top-k call per 1e6 batch
+-- must then match the oracle on every field of every candidate and its
+top-16 must equal the oracle's top-16 over the whole set, for the
+equal-layer search (auto) and the general search."""
+
+import json
+import os
 
 import numpy as np
 import pytest
 
+import fullsize_common as F
 import gpu_helpers as G
 
 pytestmark = pytest.mark.gpu
 
-FULL = [("dense32", 100_000, None), ("dense80", 1_000_000, 4000), ("moe48", 1_000_000, 4000),
-        ("stress128", 10_000_000, 300)]
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "fullsize_oracle.json")
+_ORACLE = {}
 
 
+def _golden():
+    with open(GOLDEN) as f:
+        return json.load(f)
+
+
+def _oracle_full(oracle_mod, name, n):
+    """The workload and the oracle's results over all of it (cached)."""
+    if name not in _ORACLE:
+        from paper_2609_34244_gb300 import workloads as W
+        w = W.make_workload(name, seed=F.SEED, n=n)
+        ref = oracle_mod.Oracle(w.cluster, w.model).price(w.cands, threads=os.cpu_count() or 1, bounds=False)
+        top = oracle_mod.topk(ref, w.cands["M"], F.TOPK)
+        _ORACLE.clear()  # one full-size workload held at a time
+        _ORACLE[name] = (w, ref, top)
+    return _ORACLE[name]
+
+
+@pytest.mark.parametrize("path", ["bench", "batched"])
 @pytest.mark.parametrize("search", [0, 1], ids=["auto", "general"])
-@pytest.mark.parametrize("name,n,per_batch_sample", FULL)
-def test_full_size(heddle_lib, oracle_mod, name, n, per_batch_sample, search):
+@pytest.mark.parametrize("name,n", F.FULL_SIZES)
+def test_full_size(heddle_lib, oracle_mod, name, n, search, path):
     import torch
-    from paper_2609_34244_gb300 import workloads as W
     assert torch.cuda.is_available()
     h = heddle_lib
-    w = W.make_workload(name, seed=0, n=n)
-    batch = 1_000_000
-    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, bounds=False, batch=batch, search=search)
-    assert got["errors"] == 0
-    orc = oracle_mod.Oracle(w.cluster, w.model)
-    rng = np.random.default_rng(123)
-    if per_batch_sample is None:
-        idx = np.arange(n)
+    w, ref, top = _oracle_full(oracle_mod, name, n)
+    gold = _golden()[F.key(name, n)]
+    assert F.input_digest(w.cands) == gold["inputs_sha256"], "seeded inputs differ from the stored ones"
+    assert F.field_digests(ref) == gold["fields_sha256"], "the oracle on this host differs from the stored run"
+    assert [int(x) for x in top["idx"]] == gold["topk"]["idx"]
+    if path == "bench":
+        # one call over every candidate, priced in 1e6 chunks pipelined over
+        # the work streams and merged in order (the benchmark's step)
+        got = G.price_gpu(h, w.cluster, w.model, w.cands, k=F.TOPK, bounds=False, search=search, fused=True,
+                          chunk=1_000_000)
     else:
-        idx = np.concatenate([lo + rng.choice(min(batch, n - lo), per_batch_sample, replace=False)
-                              for lo in range(0, n, batch)])
-    sub = W.make_cands(w.cands["S"][idx], w.cands["M"][idx], np.ascontiguousarray(w.cands["code"][:, idx]))
-    ref = orc.price(sub, threads=16, bounds=False)
-    G.assert_same(got, ref, idx=idx, what=name)
-    # top-k of the GPU outputs, computed exactly on the host
-    ok = np.nonzero(got["status"] == 0)[0]
-    nM = got["n_dp"][ok].astype(np.int64) * w.cands["M"][ok].astype(np.int64)
-    exp = G.exact_topk(ok, got["T"][ok], nM, 16)
-    assert got["topk"]["idx"].tolist() == [e[0] for e in exp]
-    # and every top-k entry priced again by the oracle
-    ti = got["topk"]["idx"]
-    tsub = W.make_cands(w.cands["S"][ti], w.cands["M"][ti], np.ascontiguousarray(w.cands["code"][:, ti]))
-    tref = orc.price(tsub, bounds=False)
-    assert (tref["T"] == got["topk"]["T"]).all()
-    assert (tref["n_dp"].astype(np.uint32) * w.cands["M"][ti].astype(np.uint32) == got["topk"]["nM"]).all()
+        got = G.price_gpu(h, w.cluster, w.model, w.cands, k=F.TOPK, bounds=False, batch=1_000_000,
+                          search=search)
+    assert got["errors"] == 0
+    if search == 1:
+        assert got["search"] == h.SEARCH_GENERAL
+    G.assert_same(got, ref, what="%s %s" % (name, path))
+    assert F.field_digests(got) == gold["fields_sha256"]
+    tk = got["topk"]
+    assert tk["count"] == top["count"]
+    assert tk["idx"].tolist() == top["idx"].tolist()
+    assert tk["T"].tolist() == top["T"].tolist()
+    assert tk["nM"].tolist() == top["nM"].tolist()
 
 
 def test_one_call_larger_than_the_worklist(heddle_lib, oracle_mod):
