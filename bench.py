@@ -54,10 +54,40 @@ WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 10
 # stage's gradient bytes (2) and bandwidth (2), the exact ratio comparison
 # of two 64x64->128-bit products (20): 36.  Together 65.
 OPS_PER_UNIT = {1: 16, 2: 65}
+# Screen (decode, validate, DP degree, memory screen), per candidate, in
+# 32-bit lane operations: the depth and M checks (2) and the status decision
+# (3); per stage the admissibility bit (1), its units added to its type's
+# demand word (2), the in-flight count min(S - s, M) (2), the run-table row
+# offset (1) and the running sum and minimum of the runs (2): 8; per type
+# used, its demand fields unpacked (2), and per (type, degree) used the
+# cumulative demand (1), the quotient capacity / demand as a multiply-high
+# and shift (2) and the running minimum (1): 4.  Top-k, per searched
+# candidate: its throughput key and the threshold comparison (4).
+SCREEN_OPS = {"candidate": 5, "stage": 8, "type": 2, "pair": 4}
+TOPK_OPS_PER_SEARCHED = 4
+
+
+def screen_ops(cands) -> int:
+    """Algorithmic lane operations of the screen over a candidate set."""
+    S = cands["S"].astype(np.int64)
+    code = cands["code"]
+    pairs = np.zeros(S.shape[0], np.uint64)
+    types = np.zeros(S.shape[0], np.uint32)
+    for s_ in range(code.shape[0]):
+        live = S > s_
+        b = code[s_].astype(np.uint64) & 31
+        pairs |= np.where(live, np.uint64(1) << b, np.uint64(0))
+        types |= np.where(live, np.uint32(1) << (code[s_].astype(np.uint32) & 7), np.uint32(0))
+    npairs = sum(int(((pairs >> np.uint64(i)) & np.uint64(1)).sum()) for i in range(32))
+    ntypes = sum(int(((types >> np.uint32(i)) & np.uint32(1)).sum()) for i in range(8))
+    return (SCREEN_OPS["candidate"] * S.shape[0] + SCREEN_OPS["stage"] * int(S.sum()) +
+            SCREEN_OPS["type"] * ntypes + SCREEN_OPS["pair"] * npairs)
+
+
 SEARCH_NAMES = {1: "general interval search", 2: "equal-layer closed form"}
 SEARCH_KERNELS = {1: "wsearch_kernel (general threshold search, one warp per entry)",
                   2: "eq_search_kernel (equal-layer closed form)"}
-SMS, LANES_PER_SM = 152, 128  # 4 SM sub-partitions x 32 lanes issue per clock
+LANES_PER_SM = 128  # 4 SM sub-partitions x 32 lanes issue per clock; the SM count comes from the device
 
 # DRAM bytes (read + write) of one search launch on a 1e6-candidate batch of
 # the stress workload, from an ncu capture, with the SHA-256 of the kernel
@@ -78,6 +108,59 @@ def traffic_per_launch(search, batch):
         with open(os.path.join(ROOT, "paper_2609_34244_gb300", "csrc", f), "rb") as fh:
             hs.update(fh.read())
     return rec["bytes"] if hs.hexdigest() == rec["sha256"] else None
+
+
+def gpu_numa(dev):
+    """NUMA node and local CPUs of the GPU from sysfs (empty when unknown)."""
+    import torch
+    p = torch.cuda.get_device_properties(dev)
+    try:
+        bus = "%04x:%02x:%02x.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+    except AttributeError:
+        return {}
+    out = {"pci": bus}
+    base = "/sys/bus/pci/devices/" + bus
+    try:
+        with open(base + "/numa_node") as f:
+            out["gpu_numa_node"] = int(f.read().strip())
+    except (OSError, ValueError):
+        pass
+    try:
+        with open(base + "/local_cpulist") as f:
+            txt = f.read().strip()
+        cpus = set()
+        for part in txt.split(","):
+            if "-" in part:
+                a, b = part.split("-")
+                cpus.update(range(int(a), int(b) + 1))
+            elif part:
+                cpus.add(int(part))
+        out["local_cpulist"] = txt
+        out["cpus"] = sorted(cpus)
+    except (OSError, ValueError):
+        pass
+    return out
+
+
+def h2d_copy_gbs(nbytes):
+    """Host-to-device copy rate from pinned memory, GB/s (best of 5)."""
+    import torch
+    src = torch.empty(nbytes, dtype=torch.uint8, pin_memory=True)
+    src.numpy()[...] = 1
+    dst = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    dst.copy_(src, non_blocking=True)
+    torch.cuda.synchronize()
+    best = None
+    for _ in range(5):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        dst.copy_(src, non_blocking=True)
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1)
+        best = ms if best is None else min(best, ms)
+    del src, dst
+    return nbytes / (best / 1e3) / 1e9
 
 
 def load_peaks():
@@ -184,6 +267,109 @@ def run_reference(args, w):
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+# The five workloads of the benchmark suite, each measured on its own in
+# the default run (the headline line stays stress128).
+PER_CONFIG = ("tiny", "dense32", "dense80", "moe48", "stress128")
+
+
+def measure_config(h, name, peaks, sms, steps=20, cpu_seconds=3.0, main=None):
+    """Candidates/s, per-candidate and single-batch latency, the dominant
+    kernel's own launch time and roofline fraction, and the oracle's rate on
+    the host cores in the same run, for one workload at its defining size
+    (one pricing call over all candidates, chunks of 1e6).  Inputs smaller
+    than L2 are preceded by an L2 flush outside each timed step."""
+    import torch
+    from paper_2609_34244_gb300 import workloads as W
+    w = W.make_workload(name, seed=0)
+    n = w.n
+    batch = min(1_000_000, n)
+    stream = torch.cuda.current_stream()
+    ctx = h.heddle_create(torch.cuda.current_device())
+    try:
+        h.heddle_load_cluster(ctx, w.cluster)
+        h.heddle_load_model(ctx, w.model)
+        h.heddle_set_chunk(ctx, batch)
+        search = h.heddle_get_search(ctx)
+        dc = h.cands_to_device(w.cands)
+        res = h.alloc_results(n)
+        state = h.alloc_topk_state()
+        bat = [(h.make_candidates(dc, lo, min(n, lo + batch)), h.make_results(res, lo, min(n, lo + batch)))
+               for lo in range(0, n, batch)]
+        for c, r in bat:
+            h.heddle_count_next(ctx, True)
+            h.heddle_price_candidates(ctx, c, r, stream)
+        work = h.heddle_work_counters(ctx)
+        allc, allr = h.make_candidates(dc), h.make_results(res)
+        in_bytes = sum(int(v.numel() * v.element_size()) for v in dc.values())
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda") if in_bytes < (200 << 20) else None
+
+        def step():
+            h.heddle_topk_reset(ctx, state, 16, stream)
+            h.heddle_price_topk(ctx, allc, allr, state, stream)
+
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+        evs = []
+        for _ in range(steps):
+            if flush is not None:
+                flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            step()
+            e1.record(stream)
+            evs.append((e0, e1))
+        torch.cuda.synchronize()
+        per = [a.elapsed_time(b) for a, b in evs]
+        ms = float(np.mean(per))
+        lat = []
+        c0, r0 = bat[0]
+        for _ in range(10):
+            t0 = time.perf_counter()
+            h.heddle_topk_reset(ctx, state, 16, stream)
+            h.heddle_price_topk(ctx, c0, r0, state, stream)
+            torch.cuda.synchronize()
+            lat.append((time.perf_counter() - t0) * 1e3)
+        # the search kernel's own launches: one call per batch, no overlap
+        h.heddle_time_phases(ctx, True)
+        for _ in range(3):
+            h.heddle_topk_reset(ctx, state, 16, stream)
+            for c, r in bat:
+                h.heddle_price_topk(ctx, c, r, state, stream)
+        torch.cuda.synchronize()
+        h.heddle_time_phases(ctx, False)
+        ph = h.heddle_phase_times(ctx)
+        errors = h.heddle_device_errors(ctx)
+    finally:
+        h.heddle_destroy(ctx)
+    peak = sms * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+    s_ms, s_launches = ph["search"]
+    ops = work["checks"] * OPS_PER_UNIT.get(search, 0)
+    tops = ops * 3 / (s_ms / 1e3) / 1e12 if s_ms > 0 else None
+    threads = os.cpu_count() or 1
+    rate, ncpu, used, dt = oracle_rate(w, cpu_seconds, threads)
+    out = {"workload": name, "candidates": n, "search": SEARCH_NAMES.get(search, search),
+           "value": n / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "per_candidate_ns": 1e6 * ms / n,
+           "step_ms": {"median": float(np.median(per)), "best": float(np.min(per)), "runs": len(per)},
+           "single_batch_latency_ms": {"median": float(np.median(lat)), "best": float(np.min(lat)),
+                                       "batch": batch},
+           "l2": ("inputs %.1f MB; L2 flushed (256 MB write) before each timed step" % (in_bytes / 1e6)
+                  if flush is not None else "inputs %.0f MB, larger than L2" % (in_bytes / 1e6)),
+           "dominant_kernel": SEARCH_KERNELS.get(search, "search"),
+           "roofline": {"bound": "alu", "achieved": tops, "peak": peak, "unit": "Tops/s",
+                        "frac": tops / peak if tops else None,
+                        "launch_us": 1e3 * s_ms / max(1, s_launches),
+                        "phases_us_per_batch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in ph.items()},
+                        "ops_per_unit": OPS_PER_UNIT.get(search), "units_per_candidate": work["checks"] / n,
+                        "searched_fraction": work["priced"] / n,
+                        "upper_bound": search == 1},
+           "device_errors": errors,
+           "cpu_baseline": {"value": rate, "unit": UNIT, "cores": used, "kind": "oracle",
+                            "sample": "first %d candidates (%.1f s, %d host threads)" % (ncpu, dt, used)},
+           "gpu_over_oracle": (n / (ms / 1e3)) / rate}
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -198,6 +384,7 @@ def main():
     ap.add_argument("--mbs-levels", type=int, default=4, help="micro-batch sizes of the fill figure (0: skip)")
     ap.add_argument("--no-distribute", action="store_true", help="skip the paper's-split comparison figure")
     ap.add_argument("--plans", type=int, default=1_000_000, help="multi-template plans of the plan figure (0: skip)")
+    ap.add_argument("--no-per-config", action="store_true", help="skip the per-workload measurements")
     ap.add_argument("--tiling", type=int, default=1_000_000,
                     help="moe48 candidates of the expert-tiling figure (0: skip)")
     args = ap.parse_args()
@@ -223,6 +410,7 @@ def main():
     from paper_2609_34244_gb300 import shard
 
     torch.cuda.set_device(local)
+    sms = torch.cuda.get_device_properties(local).multi_processor_count
     group = shard.init(world)
     n, batch = args.n, min(args.batch, args.n)
     # weak scaling: rank r prices its own n candidates (seed r), global indices r*n + c
@@ -385,7 +573,7 @@ def main():
                    "checks_per_candidate": gwork["checks"] / n,
                    "probes_per_searched": gwork["probes"] / max(1, gwork["priced"]),
                    "alu_frac": gwork["checks"] * OPS_PER_UNIT[1] / (gsearch_ms / 1e3) / 1e12 /
-                   (SMS * LANES_PER_SM * 2070.0 * 1e6 / 1e12),
+                   (sms * LANES_PER_SM * 2070.0 * 1e6 / 1e12),
                    "same_topk": gtopk["idx"].tolist() == local_topk["idx"].tolist()}
         h.heddle_set_search(ctx, h.SEARCH_AUTO)
 
@@ -505,9 +693,26 @@ def main():
         finally:
             h.heddle_destroy(ctx2)
 
-    # end to end through the public host-buffer call (pinned host memory)
-    pinned = {k: torch.from_numpy(v.view(np.int16) if v.dtype == np.uint16 else v).pin_memory()
+    # end to end through the public host-buffer call (pinned host memory,
+    # placed on the GPU's own NUMA node: the process runs on the GPU's local
+    # CPUs while the pages are pinned and first written)
+    numa = gpu_numa(local)
+    old_aff = os.sched_getaffinity(0) if hasattr(os, "sched_getaffinity") else None
+    if numa.get("cpus") and old_aff is not None:
+        try:
+            os.sched_setaffinity(0, numa["cpus"])
+        except OSError:
+            pass
+    pinned = {k: torch.empty(v.shape, dtype=torch.int16 if v.dtype == np.uint16 else torch.uint8, pin_memory=True)
               for k, v in w.cands.items()}
+    for k, v in w.cands.items():
+        pinned[k].numpy()[...] = v.view(np.int16) if v.dtype == np.uint16 else v
+    copy_peak = h2d_copy_gbs(1 << 30)
+    if old_aff is not None:
+        try:
+            os.sched_setaffinity(0, old_aff)
+        except OSError:
+            pass
     h2d = int(sum(v.numel() * v.element_size() for v in pinned.values()))
     st = h.new_topk_state(16)
     e2e_steps = max(1, args.e2e_steps)
@@ -525,9 +730,12 @@ def main():
     if rank != 0:
         return
     peaks, peak_kind = load_peaks()
+    per_config = None
+    if not args.no_per_config:
+        per_config = [measure_config(h, name, peaks, sms) for name in PER_CONFIG]
     value = n * world * args.steps / (ms_all / 1e3)
     ops_step = work["checks"] * OPS_PER_UNIT[search]
-    peak_tops = SMS * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
+    peak_tops = sms * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
     # the dominant kernel is the search: its average launch duration from
     # the events around it, its algorithmic ops per launch from the counters
     search_ms, search_launches = phases["search"]
@@ -536,6 +744,16 @@ def main():
     iso_ms, iso_launches = iso_phases["search"]
     iso_tops = ops_step * 3 / (iso_ms / 1e3) / 1e12 if iso_ms > 0 else None
     total_phase_ms = sum(v[0] for v in phases.values())
+    # the whole step against the same issue-slot peak: the screen's,
+    # the search's and the top-k's algorithmic operations over the step time
+    scr_ops = screen_ops(w.cands)
+    tk_ops = TOPK_OPS_PER_SEARCHED * work["priced"]
+    step_s = ms_all / args.steps / 1e3
+    step_roofline = {"achieved": (scr_ops + ops_step + tk_ops) / step_s / 1e12, "peak": peak_tops,
+                     "unit": "Tops/s", "frac": (scr_ops + ops_step + tk_ops) / step_s / 1e12 / peak_tops,
+                     "ops_per_step": {"screen": scr_ops, "search": ops_step, "topk": tk_ops},
+                     "screen_ops_basis": SCREEN_OPS, "topk_ops_per_searched": TOPK_OPS_PER_SEARCHED,
+                     "how": "algorithmic lane operations of one step / the mean step time of the K timed steps"}
     cpu = None
     if not args.no_cpu_baseline:
         rate, ncpu, used, dt = oracle_rate(w, args.cpu_seconds, os.cpu_count() or 1)
@@ -558,36 +776,49 @@ def main():
         "single_batch_latency_ms": {"median": float(np.median(lat)), "best": float(np.min(lat)),
                                     "batch": batch, "how": "wall time of one heddle_price_topk call on one batch, "
                                                            "synchronised, 20 runs after a warm call"},
-        "roofline": {"bound": "alu", "achieved": achieved_tops, "peak": peak_tops, "unit": "Tops/s",
-                     "frac": achieved_tops / peak_tops,
+        # the dominant kernel's own launch duration: one call per batch right
+        # after the timed region, so no other chunk's kernel shares the GPU
+        # with it; the overlapped launch time of the timed steps is under "live"
+        "roofline": {"bound": "alu", "achieved": iso_tops, "peak": peak_tops, "unit": "Tops/s",
+                     "frac": iso_tops / peak_tops if iso_tops else None,
                      "traffic": traffic_per_launch(search, batch),
                      "kernel": SEARCH_KERNELS[search], "search": SEARCH_NAMES[search],
-                     "launch_us": search_us, "launches_timed": search_launches,
+                     "launch_us": 1e3 * iso_ms / max(1, iso_launches), "launches_timed": iso_launches,
+                     "duration_basis": "CUDA events around each search launch on its stream, one pricing call "
+                                       "per batch (no overlap), 3 steps after the timed region",
                      "ops_per_unit": OPS_PER_UNIT[search],
                      "ops_per_launch": ops_step / n_batches,
                      "units_per_candidate": work["checks"] / n,
                      "probes_per_searched": work["probes"] / max(1, work["priced"]),
                      "searched_fraction": work["priced"] / n,
-                     "phases_us_per_batch": {k: 1e3 * v[0] / max(1, search_launches) for k, v in phases.items()},
-                     "phase_share": {k: v[0] / total_phase_ms for k, v in phases.items()},
-                     "overlap": "chunks pipelined over two work streams: each launch's event-timed "
-                                "duration includes sharing the GPU with the neighbouring chunks' kernels",
-                     "isolated": {"launch_us": 1e3 * iso_ms / max(1, iso_launches),
-                                  "achieved": iso_tops,
-                                  "frac": iso_tops / peak_tops if iso_tops else None,
-                                  "phases_us_per_batch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in iso_phases.items()},
-                                  "how": "one call per batch (no overlap), 3 steps after the timed region"},
+                     "phases_us_per_batch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in iso_phases.items()},
+                     "live": {"launch_us": search_us, "launches_timed": search_launches,
+                              "achieved": achieved_tops, "frac": achieved_tops / peak_tops,
+                              "phases_us_per_batch": {k: 1e3 * v[0] / max(1, search_launches)
+                                                      for k, v in phases.items()},
+                              "phase_share": {k: v[0] / total_phase_ms for k, v in phases.items()},
+                              "how": "inside the timed steps (every 8th step): chunks pipelined over two work "
+                                     "streams, so each launch shares the GPU with the neighbouring chunks' "
+                                     "kernels"},
+                     "step": step_roofline,
                      "peak_basis": "%s: %d SMs x %d lanes x %.0f MHz (%s sm_max)" % (
-                         "issue slots", SMS, LANES_PER_SM, float(peaks.get("sm_max_mhz", 2070.0)), peak_kind)},
+                         "issue slots", sms, LANES_PER_SM, float(peaks.get("sm_max_mhz", 2070.0)), peak_kind)},
         "clocks": clocks,
         "e2e": {"value": n * world / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d * world,
-                "d2h_bytes_per_step": h.TOPK_STATE_BYTES * world},
+                "d2h_bytes_per_step": h.TOPK_STATE_BYTES * world,
+                "d2h_contents": "the merged top-16 state (index, T and n*M of the 16 best plans); the per-candidate "
+                                "T / n_dp / status planes stay on the device",
+                "h2d_gbs_achieved": h2d / e2e_s / 1e9,
+                "h2d_copy_peak_gbs": copy_peak,
+                "copy_peak_how": "plain cudaMemcpyAsync of 1 GiB from pinned host memory, best of 5, CUDA events",
+                "pinned_memory": {k: v for k, v in numa.items() if k != "cpus"}},
         "device_errors": errors,
         "general_search": general,
         "distribute_split": distribute,
         "mbs_fill": mbs_fig,
         "plans": plans_fig,
         "expert_tiling": tiling_fig,
+        "per_config": per_config,
         "topk_head": merged["idx"][:4].tolist() if merged["count"] else [],
         "e2e_topk_matches": e2e_topk["idx"].tolist() == local_topk["idx"].tolist(),
     }
