@@ -266,8 +266,11 @@ heddle_status heddle_price_topk(heddle_ctx* ctx, const heddle_candidates* cands,
  * the library's device code is loaded until the process exits: 64 lists of
  * 64 entries, one per slice of 65,536 candidates, so a call handles at most
  * HEDDLE_TOPK_NOALLOC_MAX_N = 4,194,304 candidates (E_LIMIT beyond).
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * Every call looks up the array's device address on the current device
+ * (cudaGetSymbolAddress; a device reset reloads the library's device code,
+ * so an address kept from before it would be stale).  The first call on a
+ * device also loads the library's device code there: make that first call
+ * before any stream capture.
  * Every call on a device shares the array and overwrites it, so calls whose
  * kernels overlap on the GPU race: serialise them (one stream).
  *

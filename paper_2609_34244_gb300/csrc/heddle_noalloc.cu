@@ -11,9 +11,9 @@
 // bounds the batch size instead of the call allocating for it.
 //
 // The array's name is only a host-side stand-in: host code passes the
-// device address obtained from cudaGetSymbolAddress, once per device.
-
-#include <mutex>
+// device address obtained from cudaGetSymbolAddress on the current device,
+// looked up again on every call (a device reset reloads the module and can
+// move the array, so an address kept from an earlier call could be stale).
 
 #include "heddle_rank.cuh"
 
@@ -47,12 +47,20 @@ struct NaArgs {
 
 // CTA b scans candidates [b * kNaSlice, (b + 1) * kNaSlice) and writes one
 // list and its length (every CTA writes its count, so nothing has to be
-// cleared between calls).
+// cleared between calls).  A candidate that does not beat the incoming
+// state's k-th entry (when the state is full) cannot enter the result and
+// is not offered.
 __global__ void __launch_bounds__(kNaBlock) noalloc_block_kernel(NaArgs a) {
     const int k = state_k(a.state);
     __shared__ TopkEntry lists[kNaWarps][kMaxTopK];
     __shared__ int counts[kNaWarps];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool full = a.state->count >= k;
+    TopkEntry bar;
+    bar.idx = full ? a.state->idx[k - 1] : 0;
+    bar.T = full ? a.state->T[k - 1] : 0;
+    bar.nM = full ? a.state->nM[k - 1] : 0;
+    bar.pad = 0;
     int cnt = 0;
     const int64_t lo = (int64_t)blockIdx.x * kNaSlice;
     const int64_t hi = min(a.n, lo + kNaSlice);
@@ -65,7 +73,7 @@ __global__ void __launch_bounds__(kNaBlock) noalloc_block_kernel(NaArgs a) {
             e.T = a.T[c];
             e.nM = (uint32_t)a.ndp[c] * (uint32_t)a.M[c];
             e.pad = 0;
-            valid = true;
+            valid = !full || better(e, bar);
         }
         warp_offer(&lists[warp][0], cnt, k, valid, e);
     }
@@ -119,24 +127,14 @@ __global__ void __launch_bounds__(kNaMergeBlock) noalloc_merge_kernel(NaArgs a, 
     if (threadIdx.x == 0) a.state->count = merged_count;
 }
 
-// Device address of g_topk_scratch per device, resolved on first use.
-constexpr int kMaxDevices = 64;
-std::mutex g_setup_mutex;
-unsigned char* g_scratch_ptr[kMaxDevices] = {};
-
+// Device address of g_topk_scratch on the current device, looked up on
+// every call: cheap once the module is loaded, and never stale after a
+// device reset.
 cudaError_t scratch_for_current_device(unsigned char** out) {
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
+    unsigned char* ptr = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress((void**)&ptr, g_topk_scratch);
     if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (!g_scratch_ptr[dev]) {
-        unsigned char* ptr = nullptr;
-        e = cudaGetSymbolAddress((void**)&ptr, g_topk_scratch);
-        if (e != cudaSuccess) return e;
-        g_scratch_ptr[dev] = ptr;
-    }
-    *out = g_scratch_ptr[dev];
+    *out = ptr;
     return cudaSuccess;
 }
 
