@@ -33,7 +33,11 @@ namespace wp {
 
 constexpr int kSetWords = 8;  // 256-bit position sets (L <= 255)
 constexpr unsigned kFull = 0xffffffffu;
-constexpr long long kWaitSpins = 1 << 22;
+// Bounds of the image wait, in global-timer nanoseconds: the copy's own
+// wait, then (after raising the error flag) a second wait for the copies
+// still in flight.
+constexpr uint64_t kWaitNs = 1000000000ull;
+constexpr uint64_t kDrainNs = 1000000000ull;
 
 // per-warp shared state: sets C[0..32], forward bounds U, the split A
 struct WarpArea {
@@ -47,10 +51,40 @@ __device__ __forceinline__ uint32_t saddr(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Wait on phase 0 of bar for at most `limit` ns; true once it completed.
+__device__ __forceinline__ bool wait_phase0(uint64_t* bar, uint64_t limit) {
+    const uint64_t t0 = global_ns();
+    for (;;) {
+        uint32_t done;
+        asm volatile(
+            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0; selp.u32 %0, 1, 0, p; }"
+            : "=r"(done)
+            : "r"(saddr(bar))
+            : "memory");
+        if (done) return true;
+        if (global_ns() - t0 > limit) return false;
+    }
+}
+
 // A table image into shared memory: one thread arms an mbarrier with the
-// byte count (a multiple of 16) and issues bulk asynchronous copies; all
-// wait on phase 0 with a bounded spin.  False (and the error flag) if the
-// wait gave up.
+// byte count (a multiple of 16) and issues bulk asynchronous copies that
+// together move exactly that count; all threads wait on phase 0.
+//
+// No copy outlives this function while the device works: the armed count
+// equals the bytes issued, so the phase completes exactly when the last
+// copy lands, and the copies depend on nothing but device memory (no other
+// thread, CTA or kernel), so they land within microseconds.  The wait is
+// still bounded (global timer, kWaitNs): if it runs out the CTA raises the
+// error flag and waits once more, again bounded (kDrainNs), for the copies
+// in flight before it returns; only a memory system that has stopped
+// altogether -- a lost context, where no CTA runs again -- gets past both.
+// False (error flag raised) if the first wait ran out.
 __device__ inline bool load_image(unsigned char* dst, const unsigned char* src, uint32_t bytes, uint64_t* bar,
                                   uint32_t* err) {
     if (threadIdx.x == 0) {
@@ -69,17 +103,14 @@ __device__ inline bool load_image(unsigned char* dst, const unsigned char* src, 
         }
     }
     __syncthreads();
-    uint32_t done = 0;
-    for (long long spin = 0; spin < kWaitSpins; ++spin) {
-        asm volatile(
-            "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0; selp.u32 %0, 1, 0, p; }"
-            : "=r"(done)
-            : "r"(saddr(bar))
-            : "memory");
-        if (done) break;
+    const bool done = wait_phase0(bar, kWaitNs);
+    const int all = __syncthreads_and(done);
+    if (!all) {
+        if (threadIdx.x == 0) atomicOr(err, kErrStageWait);
+        // the copies in flight land before the CTA leaves its shared memory
+        if (threadIdx.x == 0) (void)wait_phase0(bar, kDrainNs);
+        __syncthreads();
     }
-    const int all = __syncthreads_and(done != 0);
-    if (!all && threadIdx.x == 0) atomicOr(err, kErrStageWait);
     return all != 0;
 }
 
