@@ -19,7 +19,9 @@ import numpy as np
 HERE = os.path.dirname(os.path.abspath(__file__))
 SRC = os.path.join(HERE, "heddle_oracle.c")
 HDR = os.path.join(HERE, "heddle_oracle.h")
-LIB = os.path.join(HERE, "liboracle.so")
+# HEDDLE_ORACLE_LIB names a prebuilt library to load instead (the sanitizer
+# test's instrumented build); it is then not rebuilt here
+LIB = os.environ.get("HEDDLE_ORACLE_LIB") or os.path.join(HERE, "liboracle.so")
 
 OK, OOM, NO_FIT, INVALID, SKIPPED = 0, 1, 2, 3, 4
 
@@ -28,6 +30,8 @@ _lib = None
 
 def build(force: bool = False) -> str:
     """Compile ``liboracle.so`` with gcc (no fused multiply-add)."""
+    if os.environ.get("HEDDLE_ORACLE_LIB"):
+        return LIB
     newest = max(os.path.getmtime(SRC), os.path.getmtime(HDR))
     if force or not os.path.exists(LIB) or os.path.getmtime(LIB) < newest:
         tmp = LIB + ".tmp%d" % os.getpid()

@@ -42,23 +42,45 @@ def _deps():
         + [os.path.abspath(__file__)]
 
 
-def stale() -> bool:
-    if not os.path.exists(LIB):
+# Variants of the library beside the product build, for the tests:
+# "checked" adds device-side bounds checks that raise an error flag instead of
+# reading or writing out of range, and shrinks the equal-layer search's queue
+# of open searches so its fallback path runs often; "asan" instruments the
+# host code with AddressSanitizer and UndefinedBehaviorSanitizer.
+VARIANTS = {
+    "checked": ["-DHEDDLE_CHECKED=1"],
+    "asan": ["-Xcompiler", "-fsanitize=address", "-Xcompiler", "-fsanitize=undefined", "-Xcompiler",
+             "-fno-omit-frame-pointer", "-Xcompiler", "-fno-sanitize-recover=all"],
+}
+
+VARIANT_LINK = {"asan": ["-Xcompiler", "-fsanitize=address", "-Xcompiler", "-fsanitize=undefined"]}
+
+
+def lib_path(variant: str | None = None) -> str:
+    return LIB if not variant else os.path.join(PKG, "libheddle_%s.so" % variant)
+
+
+def stale(variant: str | None = None) -> bool:
+    path = lib_path(variant)
+    if not os.path.exists(path):
         return True
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(path)
     return any(os.path.getmtime(p) > t for p in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, extra: list | None = None) -> str:
-    """Compile and link; returns the library path."""
-    if not force and not stale():
-        return LIB
-    os.makedirs(BUILD, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, extra: list | None = None, variant: str | None = None) -> str:
+    """Compile and link; returns the library path (``variant``: one of
+    VARIANTS, built beside the product library)."""
+    target = lib_path(variant)
+    if not force and not stale(variant):
+        return target
+    objdir = BUILD if not variant else os.path.join(BUILD, variant)
+    os.makedirs(objdir, exist_ok=True)
     cc = nvcc()
-    extra = list(extra or [])
+    extra = list(extra or []) + (VARIANTS[variant] if variant else [])
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src) + ".o")
+        obj = os.path.join(objdir, os.path.basename(src) + ".o")
         cmd = [cc, *ARCH, *NVCC_FLAGS, *extra, "-c", src, "-o", obj]
         p = subprocess.run(cmd, capture_output=True, text=True)
         if p.returncode != 0:
@@ -71,13 +93,14 @@ def build(force: bool = False, verbose: bool = False, extra: list | None = None)
         for obj, err in results:
             if err.strip():
                 print(err)
-    tmp = LIB + ".tmp%d" % os.getpid()
-    cmd = [cc, *ARCH, "-shared", "-o", tmp, *[o for o, _ in results], "-cudart", "static"]
+    tmp = target + ".tmp%d" % os.getpid()
+    link_extra = VARIANT_LINK.get(variant, [])
+    cmd = [cc, *ARCH, "-shared", "-o", tmp, *[o for o, _ in results], "-cudart", "static", *link_extra]
     p = subprocess.run(cmd, capture_output=True, text=True)
     if p.returncode != 0:
         raise RuntimeError("link failed:\n%s\n%s" % (" ".join(cmd), p.stderr))
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, target)
+    return target
 
 
 if __name__ == "__main__":

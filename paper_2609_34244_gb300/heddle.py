@@ -14,7 +14,9 @@ import os
 
 import numpy as np
 
-LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libheddle.so")
+# HEDDLE_LIB names another build of the library to load (the sanitizer and
+# bounds-checked builds of the tests)
+LIB_PATH = os.environ.get("HEDDLE_LIB") or os.path.join(os.path.dirname(os.path.abspath(__file__)), "libheddle.so")
 
 MAX_TYPES, MAX_STAGES, MAX_LAYERS, MAX_TOPK = 8, 32, 255, 64
 BOUND_PLANES = MAX_STAGES + 1
