@@ -13,33 +13,32 @@
 // First guess, in float only: the continuous balance
 // sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2 (the
 // floors lose half a layer per such stage on average), solved by at most
-// three Newton steps from the unsaturated balance.  Exact probes then decide and snap
-// the bracket to breakpoints: a feasible probe keeps its caps down to
-// hi = max_s (c_s + cap_s q_s); an infeasible one keeps them up to the next
-// breakpoint lo = min_s c_s + (cap_s + 1) q_s.  Two exact stop rules end
-// most searches after one probe:
-//   feasible, and dropping the stages that attain hi (each loses one layer
-//   just below hi) leaves fewer than L layers or an empty stage -> B* = hi;
-//   infeasible, and at lo every stage holds a layer and the stages that
-//   attain lo (each gains exactly one) bring the total to L -> B* = lo.
-// Otherwise the next bound interpolates the cap count between the bracket's
-// probes (a Newton step while one side is missing), else bisects.  The caps
-// at B* give the componentwise smallest split -- hence the lexicographically
+// three Newton steps from the unsaturated balance.  One exact probe then
+// decides the bracket, and exact stop rules name B* from that probe alone
+// in almost every case:
+//   feasible, and the stages at the largest stage time hi cannot all lose
+//   a layer (one of them holds a single layer, or the count would drop
+//   below L) -> B* = hi;
+//   feasible, and the same holds one level down, at hi2 = the largest stage
+//   time once the stages at hi have lost their top layer -> B* = hi2;
+//   infeasible, and at the next breakpoint lo every stage holds a layer and
+//   the stages that gain one there bring the total to L -> B* = lo.
+// Every probe leaves each stage's cap in that stage's word, so the caps at
+// B* follow from the last probe (the same, one fewer for the stages at hi,
+// or one more for the stages gaining at lo) and Evaluate needs no division.
+// A search still open after the first probe continues in its own thread:
+// the next bound interpolates the cap count between the bracket's probes (a
+// Newton step while one side is missing), else bisects.  The caps at B*
+// give the componentwise smallest split -- hence the lexicographically
 // smallest -- a_{s+1} = max(a_s + 1, L - sum_{t > s} cap_t).
 //
-// Scheduling: the screen files every entry in a bucket per depth S; CTA b
-// takes entries [128 b, 128 b + 128) of the buckets read in order of
-// decreasing S, so the lanes of a warp run stage loops of equal length and
-// the warps of a CTA carry equal work (the search runs in one wave: a deep
-// warp would otherwise hold its whole CTA at the barrier).  Small CTAs
-// (eight per SM) spread the deep slices over more SMs.  Every
-// thread packs its candidate's stages once into 32-bit words (cost index |
-// P2P index | memory run) held in shared memory interleaved by thread, runs
-// the float guess and one exact probe; the few searches still open are
-// queued in shared memory and finished by the first threads of the CTA
-// (reading the owner's words), so that they fill whole warps instead of
-// holding every warp that has one; then every thread evaluates its own
-// candidate.
+// Scheduling: the screen files every entry in a bucket per depth S; warp w
+// takes entries [32 w, 32 w + 32) of the buckets read in order of
+// decreasing S, so its lanes run stage loops of equal length.  Warps work
+// independently (no CTA barrier after the tables are staged): every thread
+// packs its candidate's stages once into 32-bit words (cost index | P2P
+// index | memory run | cap) held in shared memory interleaved by thread,
+// runs the float guess, the exact probe and Evaluate.
 
 #include <algorithm>
 
@@ -49,25 +48,25 @@ namespace hd {
 namespace {
 
 constexpr int kEqBlock = 128;
+constexpr int kEqWarps = kEqBlock / 32;
 constexpr int kZeroP2P = 128;  // a zero entry after the 8 x 8 x 2 P2P table
 constexpr int kMaxIters = 256;
 
-constexpr int kTailCap = 48;  // open searches queued per slice
+// How the caps at B* follow from the caps the last probe stored.
+enum CapMode : int { kCapsAsStored = 0, kCapsLessAtHi = 1, kCapsMoreAtLo = 2 };
 
-// State of one threshold search.
+// State of one threshold search (registers of the thread that owns it).
 struct Search {
     int64_t lo, hi, B;  // B* lies in [lo, hi]; B is the next bound to probe
     int64_t Blo, Bhi;   // last infeasible / feasible bound probed (-1: none)
-    int64_t fhi;        // hi of the last feasible probe (-1: none); chi is its layer count
-    int32_t clo, chi;   // layer counts of those probes
-    int16_t owner, S;   // thread whose shared-memory column holds the stages; depth
+    int64_t anchor;     // hi (kCapsLessAtHi) or lo (kCapsMoreAtLo) of the last probe
+    int32_t clo, chi;   // layer counts of those probes; chi is the count at hi
     int32_t probes;
-    int32_t p;          // worklist entry
-    uint16_t M, n;      // its microbatches and DP degree
+    int32_t mode;       // CapMode of the stored caps relative to q.hi, -1: not at B* (yet)
 };
 
 struct EqLayout {
-    uint32_t q, rq, p2p, cf, inter, maxn, PB, win, sw, tail, bytes;
+    uint32_t q, rq, p2p, cf, inter, maxn, PB, win, sw, bytes;
 };
 
 __host__ __device__ inline uint32_t al16(uint32_t x) { return (x + 15u) & ~15u; }
@@ -84,7 +83,6 @@ __host__ __device__ inline EqLayout eq_layout(int L) {
     e.PB = o;    o = al16(o + 8 * (L + 1));        // int64 gradient-byte prefix
     e.win = o;   o = al16(o + 8 * 4 * 33);         // uint8 [(g * 4 + j) * 33 + f]
     e.sw = o;    o = al16(o + 4 * kMaxStages * kEqBlock);  // uint32 [s][thread]
-    e.tail = o;  o = al16(o + sizeof(struct Search) * kTailCap);  // open searches
     e.bytes = o;
     return e;
 }
@@ -99,12 +97,15 @@ struct EqTabs {
     const int64_t* PB;
     const uint8_t* win;
     int64_t pbytes;  // gradient bytes of every layer when they are all equal, else -1
-    uint32_t* sw;   // stage words of thread 0; thread o's element s at [s * kEqBlock + o]
     int L;
 };
 
 // Stage word: bits 0-4 cost index (the stage byte's type | degree bits),
-// bits 5-12 P2P index, bits 13-20 memory run m.
+// bits 5-12 P2P index, bits 13-20 memory run m, bits 21-28 the cap the last
+// probe found.
+constexpr int kCapShift = 21;
+constexpr uint32_t kNoCap = 0x1fffffu;
+
 __device__ __forceinline__ uint32_t stage_word(int code, int next, bool last, int f, const EqTabs& t) {
     const int g = code & 7, j = (code >> 3) & 3;
     int pidx = kZeroP2P;
@@ -115,34 +116,6 @@ __device__ __forceinline__ uint32_t stage_word(int code, int next, bool last, in
     }
     const int m = t.win[(g * 4 + j) * 33 + f];
     return (uint32_t)(code & 31) | ((uint32_t)pidx << 5) | ((uint32_t)m << 13);
-}
-
-struct Cap {
-    int k;          // layers held within B (-1: not even one)
-    int64_t q, c;
-    int m;
-};
-
-__device__ __forceinline__ Cap stage_cap(const EqTabs& t, uint32_t w, int64_t B) {
-    Cap r;
-    r.q = t.q[w & 31];
-    r.c = t.p2p[(w >> 5) & 255];
-    r.m = (int)(w >> 13) & 255;
-    if (B < r.c + r.q || r.m < 1) {
-        r.k = -1;
-        return r;
-    }
-    const int64_t x = B - r.c;
-    if (r.q == 0 || x >= (int64_t)r.m * r.q) {
-        r.k = r.m;
-        return r;
-    }
-    // x < m q with m <= 255: the float estimate is off by at most one
-    int k = (int)(u64_to_float((uint64_t)x) * t.rq[w & 31]);
-    if ((int64_t)k * r.q > x) --k;
-    if ((int64_t)(k + 1) * r.q <= x) ++k;
-    r.k = k;
-    return r;
 }
 
 // Continuous count at Bf (float): sum_s min(m_s, (Bf - c_s) / q_s), with
@@ -173,33 +146,53 @@ struct Probe {
     int64_t hi;    // largest stage time c + k q over stages holding a layer
     int64_t lo;    // next breakpoint above B: min c + (k + 1) q over stages below their run
     int64_t zmax;  // largest c + q over stages holding no layer (-1: none)
+    int64_t P;     // largest c + (k - 1) q over the stages at hi
+    int64_t R;     // largest stage time below hi
     int tot;       // layers the stages hold
     int nhi, nlo;  // stages attaining hi / lo
+    int nP, nR;    // stages attaining P / R
     bool hi1;      // a stage attaining hi holds a single layer
+    bool P1, R1;   // a stage attaining P / R would hold a single layer there
     float slope;   // sum of 1/q over stages below their run
 };
 
-// Exact probe of bound B for the stages in column sw.
-__device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, int S, int64_t B, Probe& p) {
+// Exact probe of bound B for the stages in column sw; stores each stage's
+// cap in its word.
+__device__ bool eq_probe(const EqTabs& t, uint32_t* sw, int S, int64_t B, Probe& p) {
     p.hi = -1;
     p.lo = kInf;
     p.zmax = -1;
+    p.P = -1;
+    p.R = -1;
     p.tot = 0;
-    p.nhi = 0;
-    p.nlo = 0;
-    p.hi1 = false;
+    p.nhi = p.nlo = p.nP = p.nR = 0;
+    p.hi1 = p.P1 = p.R1 = false;
     p.slope = 0.f;
     for (int s = 0; s < S; ++s) {
         const uint32_t w = sw[s * kEqBlock];
-        const Cap r = stage_cap(t, w, B);
-        const int k = max(r.k, 0);
-        if (r.m < 1) {
+        const int64_t q = t.q[w & 31];
+        const int64_t c = t.p2p[(w >> 5) & 255];
+        const int m = (int)(w >> 13) & 255;
+        int k;
+        const int64_t x = B - c;
+        if (m < 1 || x < q) {
+            k = 0;
+        } else if (q == 0 || x >= (int64_t)m * q) {
+            k = m;
+        } else {
+            // x < m q with m <= 255: the float estimate is off by at most one
+            k = (int)(u64_to_float((uint64_t)x) * t.rq[w & 31]);
+            if ((int64_t)k * q > x) --k;
+            if ((int64_t)(k + 1) * q <= x) ++k;
+        }
+        sw[s * kEqBlock] = (w & kNoCap) | ((uint32_t)k << kCapShift);
+        if (m < 1) {
             p.zmax = kInf;  // never holds a layer
             continue;
         }
-        if (k < r.m) {
+        if (k < m) {
             p.slope += t.rq[w & 31];
-            const int64_t nb = r.c + (int64_t)(k + 1) * r.q;
+            const int64_t nb = c + (int64_t)(k + 1) * q;
             if (nb < p.lo) {
                 p.lo = nb;
                 p.nlo = 1;
@@ -208,44 +201,90 @@ __device__ bool eq_probe(const EqTabs& t, const uint32_t* sw, int S, int64_t B, 
             }
         }
         if (k < 1) {
-            p.zmax = max(p.zmax, r.c + r.q);
+            p.zmax = max(p.zmax, c + q);
             continue;
         }
         p.tot += k;
-        const int64_t v = r.c + (int64_t)k * r.q;
+        const int64_t v = c + (int64_t)k * q;
         if (v > p.hi) {
+            // the stages at the old hi drop to the level below
+            if (p.hi > p.R) {
+                p.R = p.hi;
+                p.nR = p.nhi;
+                p.R1 = p.hi1;
+            } else if (p.hi == p.R) {
+                p.nR += p.nhi;
+                p.R1 |= p.hi1;
+            }
             p.hi = v;
             p.nhi = 1;
             p.hi1 = k == 1;
+            p.P = v - q;
+            p.nP = 1;
+            p.P1 = k == 2;
         } else if (v == p.hi) {
             ++p.nhi;
             p.hi1 |= k == 1;
+            const int64_t u = v - q;
+            if (u > p.P) {
+                p.P = u;
+                p.nP = 1;
+                p.P1 = k == 2;
+            } else if (u == p.P) {
+                ++p.nP;
+                p.P1 |= k == 2;
+            }
+        } else if (v > p.R) {
+            p.R = v;
+            p.nR = 1;
+            p.R1 = k == 1;
+        } else if (v == p.R) {
+            ++p.nR;
+            p.R1 |= k == 1;
         }
     }
     return p.zmax < 0 && p.tot >= t.L;
 }
 
 // One exact probe of search q at q.B and the bracket update; returns true
-// when B* = q.hi is known.
-__device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
-    const uint32_t* sw = t.sw + q.owner;
+// when B* = q.hi is known (q.mode then says how the stored caps give the
+// caps at B*, or -1 if they do not).
+__device__ bool eq_step(const EqTabs& t, uint32_t* sw, int S, Search& q, uint32_t* err) {
     q.B = min(max(q.B, q.lo), q.hi - 1);
     ++q.probes;
     Probe p;
-    const bool feas = eq_probe(t, sw, q.S, q.B, p);
+    const bool feas = eq_probe(t, sw, S, q.B, p);
+    q.mode = -1;
     if (feas) {
         q.hi = p.hi;
         q.Bhi = q.B;
         q.chi = p.tot;
-        q.fhi = p.hi;
+        q.mode = kCapsAsStored;
         // just below hi every stage attaining hi loses a layer
-        if (p.tot - p.nhi < t.L || p.hi1) q.lo = q.hi;
+        if (p.tot - p.nhi < t.L || p.hi1) {
+            q.lo = q.hi;
+        } else {
+            // the next level down, hi2, is feasible with tot - nhi layers
+            const int64_t hi2 = max(p.P, p.R);
+            const int n2 = (p.P == hi2 ? p.nP : 0) + (p.R == hi2 ? p.nR : 0);
+            const bool one2 = (p.P == hi2 && p.P1) || (p.R == hi2 && p.R1);
+            q.anchor = p.hi;
+            q.hi = hi2;
+            q.chi = p.tot - p.nhi;
+            q.mode = kCapsLessAtHi;
+            if (p.tot - p.nhi - n2 < t.L || one2) q.lo = hi2;
+        }
     } else {
         q.lo = min(max(q.lo, p.lo), q.hi);
         q.Blo = q.B;
         q.clo = p.tot;
         // at lo every stage attaining lo gains exactly one layer
-        if (p.zmax <= p.lo && p.tot + p.nlo >= t.L) q.hi = q.lo;
+        if (p.zmax <= p.lo && p.tot + p.nlo >= t.L && p.lo < kInf) {
+            q.hi = q.lo;
+            q.chi = p.tot + p.nlo;
+            q.anchor = p.lo;
+            q.mode = kCapsMoreAtLo;
+        }
     }
     if (q.lo >= q.hi) return true;
     // next bound: interpolate the cap count between the bracket's probes,
@@ -266,36 +305,21 @@ __device__ bool eq_step(const EqTabs& t, Search& q, uint32_t* err) {
     if (q.probes > kMaxIters) {
         atomicOr(err, kErrSearchBound);
         q.lo = q.hi;
+        q.mode = -1;
         return true;
     }
     return false;
 }
 
-// Finish search q: probe until B* = q.hi is known, then make sure q.chi is
-// the layer count at B*.  (A feasible probe at B keeps every cap of its hi:
-// no stage time lies in (hi, B].)
-__device__ void eq_finish(const EqTabs& t, Search& q, uint32_t* err) {
-    while (q.lo < q.hi)
-        if (eq_step(t, q, err)) break;
-    if (q.fhi != q.hi) {
-        // B* was reached from below (or never probed): its layer count
-        ++q.probes;
-        Probe p;
-        if (!eq_probe(t, t.sw + q.owner, q.S, q.hi, p)) atomicOr(err, kErrInternal);
-        q.fhi = q.hi;
-        q.chi = p.tot;
-    }
-}
-
-// The smallest boundaries from the caps at B* (recomputed stage by stage
-// from the stage words of column `owner`; `total` layers in all), then
-// Evaluate: T = (M-1) max t_s + sum t_s + max g_s; writes entry p and
-// returns T.
-__device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, int64_t p, int S, int M, int64_t n,
-                               int64_t Bstar, int total) {
+// The smallest boundaries from the caps at B* (the stored caps, adjusted by
+// q.mode), then Evaluate: T = (M-1) max t_s + sum t_s + max g_s; writes
+// entry p and returns T.
+__device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, const uint32_t* sw, int64_t p, int S, int M,
+                               int64_t n, const Search& q) {
     const int L = t.L;
+    const int64_t Bstar = q.hi;
+    const int total = q.chi;
     const int64_t c = a.wl_idx[p];
-    const uint32_t* sw = t.sw + owner;
     int64_t tmax = 0, tsum = 0;
     int sg = -1;
     // the stage with the largest G_s / (k_s bw_s), compared exactly: with
@@ -306,13 +330,19 @@ __device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, i
     int64_t pb_at = t.PB[0];
     for (int s = 0; s < S; ++s) {
         const uint32_t w = sw[s * kEqBlock];
-        const Cap r = stage_cap(t, w, Bstar);
-        const int k = r.k;
+        const int64_t qq = t.q[w & 31];
+        const int64_t cc = t.p2p[(w >> 5) & 255];
+        int k = (int)(w >> kCapShift) & 255;
+        if (q.mode == kCapsLessAtHi) {
+            if (cc + (int64_t)k * qq == q.anchor) --k;
+        } else if (q.mode == kCapsMoreAtLo) {
+            if (k < (int)((w >> 13) & 255) && cc + (int64_t)(k + 1) * qq == q.anchor) ++k;
+        }
         if (k < 1) atomicOr(a.err, kErrInternal);
         pre += k;
         const int nxt = s + 1 == S ? L : max(at + 1, L - (total - pre));
         if (a.bounds) a.bounds[(int64_t)(s + 1) * a.bstride + c] = (uint8_t)nxt;
-        const int64_t ts = (int64_t)(nxt - at) * r.q + r.c;
+        const int64_t ts = (int64_t)(nxt - at) * qq + cc;
         tmax = max(tmax, ts);
         tsum += ts;
         if (n > 1) {
@@ -366,7 +396,6 @@ __device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, int owner, i
 template <bool kCount>
 __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(PriceArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
-    __shared__ int tail_n;
     __shared__ int end_of[kMaxStages + 2];  // entries of depths >= S, [S]
     const Layout& y = a.lay;
     const int L = y.L;
@@ -401,24 +430,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
         for (int i = threadIdx.x; i <= L; i += blockDim.x)
             PB[i] = reinterpret_cast<const int64_t*>(a.img + y.offPB)[i];
     }
-    __syncthreads();
-    EqTabs t;
-    t.q = reinterpret_cast<const int64_t*>(smem + el.q);
-    t.rq = reinterpret_cast<const float*>(smem + el.rq);
-    t.p2p = reinterpret_cast<const int64_t*>(smem + el.p2p);
-    t.cf = reinterpret_cast<const float*>(smem + el.cf);
-    t.inter = reinterpret_cast<const int64_t*>(smem + el.inter);
-    t.maxn = reinterpret_cast<const int32_t*>(smem + el.maxn);
-    t.PB = reinterpret_cast<const int64_t*>(smem + el.PB);
-    t.win = smem + el.win;
-    t.pbytes = reinterpret_cast<const int32_t*>(a.img + y.offModel)[2]
-                   ? t.PB[1] - t.PB[0]
-                   : -1;
-    t.sw = reinterpret_cast<uint32_t*>(smem + el.sw);
-    t.L = L;
-    Search* tail = reinterpret_cast<Search*>(smem + el.tail);
-    uint32_t* mysw = t.sw + threadIdx.x;
-
     if (threadIdx.x < 32) {
         // end_of[S] = entries of depths >= S: an inclusive scan of depths
         // 32 .. 1 in lanes 0 .. 31
@@ -433,18 +444,35 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
         if (lane == 0) end_of[kMaxStages + 1] = 0;
     }
     __syncthreads();
+    EqTabs t;
+    t.q = reinterpret_cast<const int64_t*>(smem + el.q);
+    t.rq = reinterpret_cast<const float*>(smem + el.rq);
+    t.p2p = reinterpret_cast<const int64_t*>(smem + el.p2p);
+    t.cf = reinterpret_cast<const float*>(smem + el.cf);
+    t.inter = reinterpret_cast<const int64_t*>(smem + el.inter);
+    t.maxn = reinterpret_cast<const int32_t*>(smem + el.maxn);
+    t.PB = reinterpret_cast<const int64_t*>(smem + el.PB);
+    t.win = smem + el.win;
+    t.pbytes = reinterpret_cast<const int32_t*>(a.img + y.offModel)[2]
+                   ? t.PB[1] - t.PB[0]
+                   : -1;
+    t.L = L;
+    uint32_t* mysw = reinterpret_cast<uint32_t*>(smem + el.sw) + threadIdx.x;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
     unsigned long long units = 0, probes = 0, searched = 0;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t count_r = (count + kEqBlock - 1) / kEqBlock * kEqBlock;
     const int64_t stride = (int64_t)gridDim.x * kEqBlock;
-    for (int64_t base = (int64_t)blockIdx.x * kEqBlock; base < count_r; base += stride) {
-        // ---- this CTA's 256 entries of the order by decreasing S, so the
-        //      lanes of a warp (and the warps of a CTA) have nearly equal S
-        if (threadIdx.x == 0) tail_n = 0;
-        __syncthreads();
-        const int64_t g = base + threadIdx.x;
+    // warp w of CTA b takes entries [32 (4 b + w), +32) of the order by
+    // decreasing S, so its lanes have nearly equal S; warps never wait on
+    // one another
+    for (int64_t base = ((int64_t)blockIdx.x * kEqWarps + warp) * 32; base < count; base += stride) {
+        const int64_t g = base + lane;
         const bool have = g < count;
         int64_t p = 0;
+        int S = 0, M = 0;
+        int64_t n = 0;
+        int64_t T = -1;
         if (have) {
             // its depth: the largest S with end_of[S] > g (end_of falls with S)
             int lo = 1, hi = kMaxStages;
@@ -453,14 +481,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                 if (end_of[mid] > g) lo = mid; else hi = mid - 1;
             }
             p = a.wl_bucket[(int64_t)(lo - 1) * a.wl_cap + (g - end_of[lo + 1])];
-        }
-
-        int S = 0, M = 0;
-        int64_t n = 0;
-        int64_t Bstar = 0;  // with its layer count, unless queued
-        int btot = 0, slot = -1;
-        bool queued = false;
-        if (have) {
             S = a.wl_S[p];
             M = a.wl_M[p];
             n = a.wl_n[p];
@@ -512,48 +532,27 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                 Bf += (tgt - cnt) / sl;
             }
             q.B = (int64_t)float_to_u64(fminf(Bf, fhi));
-            q.Blo = q.Bhi = q.fhi = -1;
+            q.Blo = q.Bhi = -1;
             q.clo = q.chi = 0;
-            q.owner = (int16_t)threadIdx.x;
-            q.S = (int16_t)S;
             q.probes = 0;
-            q.p = (int32_t)p;
-            q.M = (uint16_t)M;
-            q.n = (uint16_t)n;
-            // one exact probe here; open searches go to the CTA's queue
-            const bool done = q.lo >= q.hi || eq_step(t, q, a.err);
-            if (!(done && q.fhi == q.hi)) {
-                slot = atomicAdd(&tail_n, 1);
-                if (slot < kTailCap) {
-                    tail[slot] = q;
-                    q.probes = 0;  // counted by the thread that finishes it
-                    queued = true;
-                } else {
-                    eq_finish(t, q, a.err);
+            q.mode = -1;
+            q.anchor = 0;
+            // exact probes until B* is known (one in almost every case),
+            // then one more at B* itself if the stored caps are not its own
+            if (q.lo < q.hi) {
+                while (!eq_step(t, mysw, S, q, a.err)) {
                 }
             }
-            Bstar = q.hi;
-            btot = q.chi;
+            if (q.mode < 0) {
+                Probe pr;
+                ++q.probes;
+                if (!eq_probe(t, mysw, S, q.hi, pr) || pr.hi != q.hi) atomicOr(a.err, kErrInternal);
+                q.chi = pr.tot;
+                q.mode = kCapsAsStored;
+            }
             if (kCount) probes += q.probes;
+            T = eq_evaluate(a, t, mysw, p, S, M, n, q);
         }
-        __syncthreads();
-        // ---- the open searches, one per thread
-        const int nt = min(tail_n, kTailCap);
-        for (int i = threadIdx.x; i < nt; i += kEqBlock) {
-            Search q = tail[i];
-            eq_finish(t, q, a.err);
-            tail[i].hi = q.hi;
-            tail[i].chi = q.chi;
-            if (kCount) probes += q.probes;
-        }
-        __syncthreads();
-        if (queued) {
-            const Search& q = tail[slot];
-            Bstar = q.hi;
-            btot = q.chi;
-        }
-        int64_t T = -1;
-        if (have) T = eq_evaluate(a, t, threadIdx.x, p, S, M, n, Bstar, btot);
         if (a.sv_count) {
             // inside a top-k pricing: the entries whose n*M / T reaches the
             // running threshold (float, below the k-th key by a margin that
@@ -563,7 +562,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
             // final k-th, so the raised value keeps the filter exact
             const uint32_t nM = (uint32_t)n * (uint32_t)M;
             const float key = have && T > 0 ? (float)nM / (float)T : -1.0f;
-            const int lane = threadIdx.x & 31;
             const int kk = min(max(__ldg(a.topk_k), 1), kMaxTopK);
             float own = 0.f;
             if (kk <= 32) {
@@ -571,10 +569,10 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
 #pragma unroll
                 for (int size = 2; size <= 32; size <<= 1)
 #pragma unroll
-                    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-                        const float o = __shfl_xor_sync(0xffffffffu, v, stride);
+                    for (int stride2 = size >> 1; stride2 > 0; stride2 >>= 1) {
+                        const float o = __shfl_xor_sync(0xffffffffu, v, stride2);
                         const bool desc = (lane & size) == 0 || size == 32;
-                        v = (((lane & stride) == 0) == desc) ? fmaxf(v, o) : fminf(v, o);
+                        v = (((lane & stride2) == 0) == desc) ? fmaxf(v, o) : fminf(v, o);
                     }
                 const float kth = __shfl_sync(0xffffffffu, v, kk - 1);
                 if (kth > 0.f) {
@@ -586,7 +584,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
             const bool keep = key > 0.f && key >= thr;
             const unsigned mask = __ballot_sync(0xffffffffu, keep);
             if (mask) {
-                const int lane = threadIdx.x & 31;
                 int base0 = 0;
                 if (lane == __ffs(mask) - 1) base0 = atomicAdd(a.sv_count, __popc(mask));
                 const int pos = __shfl_sync(0xffffffffu, base0, __ffs(mask) - 1) + __popc(mask & ((1u << lane) - 1));
@@ -597,7 +594,6 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                 }
             }
         }
-        __syncthreads();  // columns and queue are reused by the next slice
     }
     if (kCount) {
         unsigned long long v0 = units, v1 = probes, v2 = searched;
@@ -606,7 +602,7 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
             v1 += __shfl_down_sync(0xffffffffu, v1, o);
             v2 += __shfl_down_sync(0xffffffffu, v2, o);
         }
-        if ((threadIdx.x & 31) == 0) {
+        if (lane == 0) {
             atomicAdd(&a.counters[0], v0);
             atomicAdd(&a.counters[1], v1);
             atomicAdd(&a.counters[2], v2);
