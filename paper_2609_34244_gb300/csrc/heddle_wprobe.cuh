@@ -250,6 +250,70 @@ __device__ bool probe(const J& check, int S, int L, int64_t B, WarpArea& wa, int
     return feasible;
 }
 
+// The forward pass alone, for a bound B at which every stage could hold any
+// single layer of the model (its most expensive layer's time plus its P2P
+// within B, and the largest single-layer state and activation within its
+// memory; the caller checks this).  Then, by induction, the feasible
+// stage-s ends form the interval [s, U_s]: positions up to U_{s-1} + 1 are
+// reached one layer after their predecessor, those beyond only from U_{s-1}
+// (the largest predecessor dominates), so B is feasible iff the last stage
+// fits [U_{S-1}, L), and the chain of U_s is a split attaining every
+// accepted stage time.  The snap values therefore mean what they mean for
+// probe(): every bound in [hi, B] is feasible, every bound in [B, lo) is
+// not (the interval property holds at any bound >= B).  No sets are built:
+// the canonical split needs probe() at B*.
+template <class J>
+__device__ bool forward_probe(const J& check, int S, int L, int64_t B, int64_t& hi_out, int64_t& lo_out,
+                              unsigned long long& checks) {
+    const int lane = threadIdx.x & 31;
+    int64_t hi = -1, lo = kInf;
+    bool ok = true;
+    int u = 0;
+    for (int s = 0; s + 1 < S && ok; ++s) {
+        const typename J::Stage st = check.stage(s);
+        const int lim = L - (S - 1 - s);
+        int reach = u;
+        for (int base = u + 1; base <= lim; base += 32) {
+            const int j = base + lane;
+            int r = 1;
+            int64_t v = 0;
+            if (j <= lim) {
+                r = check.eval(st, u, j, B, &v);
+                ++checks;
+                if (r == 0) hi = max(hi, v);
+                else if (r == 1) lo = min(lo, v);
+            }
+            const unsigned rej = __ballot_sync(kFull, r != 0);
+            if (rej) {
+                reach = base + __ffs(rej) - 2;
+                break;
+            }
+            reach = base + 31;
+        }
+        if (reach < s + 1) ok = false;
+        u = reach;
+    }
+    bool feasible = false;
+    if (ok) {
+        const typename J::Stage st = check.stage(S - 1);
+        if (lane == 0) {
+            int64_t v = 0;
+            const int r = check.eval(st, u, L, B, &v);
+            ++checks;
+            if (r == 0) {
+                hi = max(hi, v);
+                feasible = true;
+            } else if (r == 1) {
+                lo = min(lo, v);
+            }
+        }
+        feasible = __shfl_sync(kFull, feasible, 0);
+    }
+    hi_out = wmax64(hi);
+    lo_out = wmin64(lo);
+    return feasible;
+}
+
 // The first guess of B* (warp-uniform): the saturating continuous balance
 // sum_s min(m_s, (B - c_s) / q_s) = L + (stages below their run) / 2, with
 // each lane's stage given by 1 / q_s (rq, its average layer cost), c_s (cf)

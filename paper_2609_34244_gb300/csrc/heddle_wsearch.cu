@@ -32,6 +32,8 @@ constexpr int kWarps = kWBlock / 32;
 constexpr int kMaxIters = 256;
 
 struct WTabs {
+    const int64_t* qmax;  // [NT * 4] the most expensive single layer per (type, degree)
+    int64_t smax, amax;   // the largest single-layer state and activation bytes
     const int64_t* P;
     const longlong2* SA;
     const int64_t* PB;
@@ -96,12 +98,46 @@ __device__ __noinline__ int64_t plain_guess(const int64_t* P, const longlong2* S
 }
 
 template <bool kCount>
-__global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
+__global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
+    __shared__ int64_t qmax[4 * kMaxTypes], single[2];
     if (!wp::load_image(smem, a.img, a.lay.bytes, &bar, a.err)) return;
     const Layout& y = a.lay;
+    {
+        // the most expensive single layer per (type, degree), and the
+        // largest single-layer state and activation, for the forward-only
+        // probe's condition
+        const int64_t* P = reinterpret_cast<const int64_t*>(smem + y.offP);
+        const longlong2* SA = reinterpret_cast<const longlong2*>(smem + y.offSA);
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        for (int r = warp; r <= 4 * y.NT; r += kWarps) {
+            int64_t m0 = 0, m1 = 0;
+            for (int l = lane; l < y.L; l += 32) {
+                if (r < 4 * y.NT) {
+                    m0 = max(m0, P[r * (y.L + 1) + l + 1] - P[r * (y.L + 1) + l]);
+                } else {
+                    m0 = max(m0, (int64_t)(SA[l + 1].x - SA[l].x));
+                    m1 = max(m1, (int64_t)(SA[l + 1].y - SA[l].y));
+                }
+            }
+            m0 = wp::wmax64(m0);
+            m1 = wp::wmax64(m1);
+            if (lane == 0) {
+                if (r < 4 * y.NT) {
+                    qmax[r] = m0;
+                } else {
+                    single[0] = m0;
+                    single[1] = m1;
+                }
+            }
+        }
+        __syncthreads();
+    }
     WTabs t;
+    t.qmax = qmax;
+    t.smax = single[0];
+    t.amax = single[1];
     t.P = reinterpret_cast<const int64_t*>(smem + y.offP);
     t.SA = reinterpret_cast<const longlong2*>(smem + y.offSA);
     t.PB = reinterpret_cast<const int64_t*>(smem + y.offPB);
@@ -120,6 +156,7 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
     for (int64_t p = (int64_t)blockIdx.x * kWarps + warp; p < count; p += nwarps) {
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
+        if (!in_range(c, a.n, a.err) || !in_range(S - 1, kMaxStages, a.err)) continue;
         const int M = a.wl_M[p];
         const int64_t n = a.wl_n[p];
         const bool memok = a.wl_memok[p] != 0;
@@ -139,6 +176,10 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
             const int same = (g == h) && ((1 << j) + (1 << jn) <= t.maxn[g]);
             mine.c = t.p2p[(g * 8 + h) * 2 + same];
         }
+        // the forward-only probe is exact at bounds where every stage could
+        // hold any single layer (time and memory)
+        const int64_t qmc = live ? t.qmax[g * 4 + j] + mine.c : -1;
+        const bool memfit = !live || t.smax + mine.f * t.amax <= mine.capk;
         // a bound feasible whenever memory is
         int64_t hi = live ? t.P[mine.row + L] + mine.c : 0;
         hi = wp::wmax64(hi);
@@ -161,7 +202,9 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
         while (true) {
             int64_t shi, slo;
             if (kCount && lane == 0) ++probes;
-            const bool feas = wp::probe(check, S, L, B, wa, shi, slo, checks);
+            const bool fast = phase != 2 && __all_sync(kFull, qmc <= B && memfit);
+            const bool feas = fast ? wp::forward_probe(check, S, L, B, shi, slo, checks)
+                                   : wp::probe(check, S, L, B, wa, shi, slo, checks);
             if (phase == 0) {
                 if (!feas) {
                     oom = true;
@@ -191,8 +234,8 @@ __global__ void __launch_bounds__(kWBlock) wsearch_kernel(PriceArgs a) {
                     if (lane == 0) atomicOr(a.err, kErrSearchBound);
                     lo = hi;
                 }
-                // closed by a feasible probe: its sets are those of B* = hi
-                if (lo >= hi && feas && it <= kMaxIters) break;
+                // closed by a feasible full probe: its sets are those of B* = hi
+                if (lo >= hi && feas && !fast && it <= kMaxIters) break;
             } else {
                 if (!feas && lane == 0) atomicOr(a.err, kErrInternal);
                 break;
