@@ -445,7 +445,8 @@ heddle_status heddle_get_tables(heddle_ctx* ctx, int64_t* q, int64_t* p2p);
 /* Device-side error flags raised since the last call (synchronises the
  * device first, then clears them): bit 0 a table-staging wait timed out,
  * bit 1 a search exceeded its iteration bound, bit 2 an internal
- * consistency check failed.  0 in normal operation. */
+ * consistency check failed, bit 3 (bounds-checked builds only) an index
+ * test failed and the access was skipped.  0 in normal operation. */
 heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
 
 /* PartitionLayers search.  AUTO (default) uses the equal-layer closed form

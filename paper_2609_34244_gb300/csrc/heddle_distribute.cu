@@ -96,6 +96,7 @@ __global__ void __launch_bounds__(kDistBlock) distribute_kernel(PriceArgs a) {
     for (int64_t p = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); p < count; p += warps) {
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
+        if (!in_range(c, a.n, a.err) || !in_range(S - 1, kMaxStages, a.err)) continue;
         const int M = a.wl_M[p];
         const int64_t n = a.wl_n[p];
         const bool live = lane < S;

@@ -320,6 +320,7 @@ __device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, const uint32
     const int64_t Bstar = q.hi;
     const int total = q.chi;
     const int64_t c = a.wl_idx[p];
+    if (!in_range(c, a.n, a.err)) return -1;
     int64_t tmax = 0, tsum = 0;
     int sg = -1;
     // the stage with the largest G_s / (k_s bw_s), compared exactly: with
@@ -356,7 +357,7 @@ __device__ int64_t eq_evaluate(const PriceArgs& a, const EqTabs& t, const uint32
                     bestD = D;
                 }
             } else {
-                const int64_t pb_nxt = t.PB[nxt];
+                const int64_t pb_nxt = in_range(nxt, L + 1, a.err) ? t.PB[nxt] : pb_at;
                 const uint64_t G = (uint64_t)(pb_nxt - pb_at);
                 pb_at = pb_nxt;
                 if (sg < 0 || (u128)G * bestD > (u128)bestG * D) {
@@ -468,7 +469,7 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
     // one another
     for (int64_t base = ((int64_t)blockIdx.x * kEqWarps + warp) * 32; base < count; base += stride) {
         const int64_t g = base + lane;
-        const bool have = g < count;
+        bool have = g < count;
         int64_t p = 0;
         int S = 0, M = 0;
         int64_t n = 0;
@@ -480,7 +481,12 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                 const int mid = (lo + hi + 1) >> 1;
                 if (end_of[mid] > g) lo = mid; else hi = mid - 1;
             }
-            p = a.wl_bucket[(int64_t)(lo - 1) * a.wl_cap + (g - end_of[lo + 1])];
+            const int64_t off = g - end_of[lo + 1];
+            if (!in_range(off, a.wl_cap, a.err)) have = false;
+            else p = a.wl_bucket[(int64_t)(lo - 1) * a.wl_cap + off];
+            if (have && !in_range(p, count, a.err)) have = false;
+        }
+        if (have) {
             S = a.wl_S[p];
             M = a.wl_M[p];
             n = a.wl_n[p];

@@ -21,6 +21,23 @@ typedef unsigned __int128 u128;
 constexpr uint32_t kErrStageWait = 1u;
 constexpr uint32_t kErrSearchBound = 2u;
 constexpr uint32_t kErrInternal = 4u;
+constexpr uint32_t kErrBounds = 8u;  // a bounds check of the checked build failed
+
+// The bounds-checked build (HEDDLE_CHECKED) tests the data-dependent
+// indices -- worklist entries, candidate indices, table rows -- before it
+// uses them; a failed test raises kErrBounds and the access is skipped (no
+// trap, no out-of-range access).  The product build compiles the tests away.
+#ifdef HEDDLE_CHECKED
+constexpr bool kChecked = true;
+#else
+constexpr bool kChecked = false;
+#endif
+__device__ __forceinline__ bool in_range(int64_t i, int64_t n, uint32_t* err) {
+    if (!kChecked) return true;
+    if (i >= 0 && i < n) return true;
+    atomicOr(err, kErrBounds);
+    return false;
+}
 // Table-build flags (checked by the host at load time).
 constexpr uint32_t kTabBadValue = 1u;   // non-finite or negative per-layer cost
 constexpr uint32_t kTabTooLarge = 2u;   // a table total or P2P term above its limit
