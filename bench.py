@@ -344,6 +344,7 @@ def measure_config(h, name, peaks, sms, steps=20, cpu_seconds=3.0, main=None):
         h.heddle_destroy(ctx)
     peak = sms * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
     s_ms, s_launches = ph["search"]
+    chunks = max(1, ph["screen"][1])
     ops = work["checks"] * OPS_PER_UNIT.get(search, 0)
     tops = ops * 3 / (s_ms / 1e3) / 1e12 if s_ms > 0 else None
     threads = os.cpu_count() or 1
@@ -358,8 +359,8 @@ def measure_config(h, name, peaks, sms, steps=20, cpu_seconds=3.0, main=None):
            "dominant_kernel": SEARCH_KERNELS.get(search, "search"),
            "roofline": {"bound": "alu", "achieved": tops, "peak": peak, "unit": "Tops/s",
                         "frac": tops / peak if tops else None,
-                        "launch_us": 1e3 * s_ms / max(1, s_launches),
-                        "phases_us_per_batch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in ph.items()},
+                        "launch_us": 1e3 * s_ms / chunks, "launches_per_chunk": s_launches / chunks,
+                        "phases_us_per_batch": {k: 1e3 * v[0] / chunks for k, v in ph.items()},
                         "ops_per_unit": OPS_PER_UNIT.get(search), "units_per_candidate": work["checks"] / n,
                         "searched_fraction": work["priced"] / n,
                         "upper_bound": search == 1},
@@ -738,10 +739,14 @@ def main():
     peak_tops = sms * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
     # the dominant kernel is the search: its average launch duration from
     # the events around it, its algorithmic ops per launch from the counters
+    # per chunk: one screen launch per chunk (the equal-layer search is two
+    # launches, its worklist pass and the pass over the entries it left open)
     search_ms, search_launches = phases["search"]
-    search_us = 1e3 * search_ms / max(1, search_launches)
+    chunks_timed = max(1, phases["screen"][1])
+    search_us = 1e3 * search_ms / chunks_timed
     achieved_tops = ops_step * sampled / (search_ms / 1e3) / 1e12
     iso_ms, iso_launches = iso_phases["search"]
+    iso_chunks = max(1, iso_phases["screen"][1])
     iso_tops = ops_step * 3 / (iso_ms / 1e3) / 1e12 if iso_ms > 0 else None
     total_phase_ms = sum(v[0] for v in phases.values())
     # the whole step against the same issue-slot peak: the screen's,
@@ -783,19 +788,19 @@ def main():
                      "frac": iso_tops / peak_tops if iso_tops else None,
                      "traffic": traffic_per_launch(search, batch),
                      "kernel": SEARCH_KERNELS[search], "search": SEARCH_NAMES[search],
-                     "launch_us": 1e3 * iso_ms / max(1, iso_launches), "launches_timed": iso_launches,
-                     "duration_basis": "CUDA events around each search launch on its stream, one pricing call "
-                                       "per batch (no overlap), 3 steps after the timed region",
+                     "launch_us": 1e3 * iso_ms / iso_chunks, "chunks_timed": iso_chunks,
+                     "launches_per_chunk": iso_launches / iso_chunks,
+                     "duration_basis": "CUDA events around each chunk's search launches on their stream, one "
+                                       "pricing call per batch (no overlap), 3 steps after the timed region",
                      "ops_per_unit": OPS_PER_UNIT[search],
                      "ops_per_launch": ops_step / n_batches,
                      "units_per_candidate": work["checks"] / n,
                      "probes_per_searched": work["probes"] / max(1, work["priced"]),
                      "searched_fraction": work["priced"] / n,
-                     "phases_us_per_batch": {k: 1e3 * v[0] / max(1, v[1]) for k, v in iso_phases.items()},
-                     "live": {"launch_us": search_us, "launches_timed": search_launches,
+                     "phases_us_per_batch": {k: 1e3 * v[0] / iso_chunks for k, v in iso_phases.items()},
+                     "live": {"launch_us": search_us, "chunks_timed": chunks_timed,
                               "achieved": achieved_tops, "frac": achieved_tops / peak_tops,
-                              "phases_us_per_batch": {k: 1e3 * v[0] / max(1, search_launches)
-                                                      for k, v in phases.items()},
+                              "phases_us_per_batch": {k: 1e3 * v[0] / chunks_timed for k, v in phases.items()},
                               "phase_share": {k: v[0] / total_phase_ms for k, v in phases.items()},
                               "how": "inside the timed steps (every 8th step): chunks pipelined over two work "
                                      "streams, so each launch shares the GPU with the neighbouring chunks' "
