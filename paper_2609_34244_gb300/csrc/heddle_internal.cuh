@@ -207,6 +207,7 @@ cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st);
 cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
 constexpr int kWlMeta = 1 + kMaxStages + 1 + 1;  // ints of a.wl_count
+constexpr int kWlGeneral = 1;  // entries the thread-per-entry general search left to the warp search
 constexpr int kWlSurv = kWlMeta - 1;             // the survivor count (see PriceArgs::sv_count)
 
 

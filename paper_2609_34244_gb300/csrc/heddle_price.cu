@@ -13,7 +13,9 @@
 // which one of the searches then prices: the equal-layer closed form
 // (heddle_eqsearch.cu) when every layer costs the same, the paper's split
 // rule in that mode (heddle_distribute.cu), else the general exact
-// threshold search with one warp per entry (heddle_wsearch.cu).
+// threshold search: one thread per entry while every stage fits any single
+// layer (heddle_gsearch.cu), one warp per entry for the rest
+// (heddle_wsearch.cu).
 
 #include <algorithm>
 
@@ -223,9 +225,9 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                     atomicOr(a.err, kErrInternal);
                 }
             }
-            if (a.uniform && take) {
-                // the entry in its depth's bucket, for the equal-layer
-                // search's order by decreasing depth
+            if (take) {
+                // the entry in its depth's bucket, for the searches' order
+                // by decreasing depth
                 const unsigned same = __match_any_sync(mask, S);
                 const int leader = __ffs(same) - 1;
                 int b0 = 0;
@@ -250,8 +252,10 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
 
 }  // namespace
 
-// The general search with one warp per worklist entry (heddle_wsearch.cu).
-cudaError_t launch_warp_search(const PriceArgs& a, int num_sms, cudaStream_t st);
+// The general search: one thread per entry where every stage fits any single
+// layer (heddle_gsearch.cu), then one warp per entry it left (heddle_wsearch.cu).
+cudaError_t launch_thread_search(const PriceArgs& a, int num_sms, cudaStream_t st);
+cudaError_t launch_warp_search(const PriceArgs& a, int num_sms, cudaStream_t st, bool listed);
 
 cudaError_t launch_screen(const PriceArgs& a, int num_sms, cudaStream_t st, cudaEvent_t mid, int64_t* launches) {
     if (a.n <= 0) return cudaSuccess;
@@ -282,7 +286,8 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
     if (launches) launches[1] += 1;
     if (a.split_mode) return launch_distribute(a, num_sms, st);
     if (a.uniform) return launch_eq_search(a, num_sms, st);
-    return launch_warp_search(a, num_sms, st);
+    if ((e = launch_thread_search(a, num_sms, st)) != cudaSuccess) return e;
+    return launch_warp_search(a, num_sms, st, true);
 }
 
 }  // namespace hd

@@ -97,8 +97,10 @@ __device__ __noinline__ int64_t plain_guess(const int64_t* P, const longlong2* S
     return wp::first_guess(rq, cf, mr, S, L, hi);
 }
 
+// listed: the entries of the list the thread-per-entry search left
+// (a.sv_idx, count at wl_count[kWlGeneral]); else every worklist entry.
 template <bool kCount>
-__global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a) {
+__global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a, int listed) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     __shared__ int64_t qmax[4 * kMaxTypes], single[2];
@@ -151,9 +153,11 @@ __global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a) {
     WarpArea& wa = reinterpret_cast<WarpArea*>(smem + ((y.bytes + 127u) & ~127u))[warp];
 
     unsigned long long checks = 0, probes = 0, priced = 0;
-    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    const int64_t count = min((int64_t)(listed ? a.wl_count[kWlGeneral] : *a.wl_count), (int64_t)a.wl_cap);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-    for (int64_t p = (int64_t)blockIdx.x * kWarps + warp; p < count; p += nwarps) {
+    for (int64_t e = (int64_t)blockIdx.x * kWarps + warp; e < count; e += nwarps) {
+        const int64_t p = listed ? a.sv_idx[e] : e;
+        if (!in_range(p, a.wl_cap, a.err)) continue;
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
         if (!in_range(c, a.n, a.err) || !in_range(S - 1, kMaxStages, a.err)) continue;
@@ -326,7 +330,7 @@ __global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a) {
 }
 
 template <bool kCount>
-cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
+cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st, bool listed) {
     const size_t smem = ((a.lay.bytes + 127u) & ~127u) + sizeof(WarpArea) * kWarps;
     cudaError_t e = cudaFuncSetAttribute(wsearch_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -338,14 +342,14 @@ cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
     // at most one wave
     const int64_t need = (a.n + kWarps - 1) / kWarps;
     const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
-    wsearch_kernel<kCount><<<grid, kWBlock, smem, st>>>(a);
+    wsearch_kernel<kCount><<<grid, kWBlock, smem, st>>>(a, listed ? 1 : 0);
     return cudaGetLastError();
 }
 
 }  // namespace
 
-cudaError_t launch_warp_search(const PriceArgs& a, int num_sms, cudaStream_t st) {
-    return a.counters ? launch<true>(a, num_sms, st) : launch<false>(a, num_sms, st);
+cudaError_t launch_warp_search(const PriceArgs& a, int num_sms, cudaStream_t st, bool listed) {
+    return a.counters ? launch<true>(a, num_sms, st, listed) : launch<false>(a, num_sms, st, listed);
 }
 
 }  // namespace hd
