@@ -462,7 +462,9 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     unsigned long long units = 0, probes = 0, searched = 0;
-    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    // the entries filed in the depth buckets (every worklist entry here)
+    const int64_t entries = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    const int64_t count = min((int64_t)end_of[1], entries);
     const int64_t stride = (int64_t)gridDim.x * kEqBlock;
     // warp w of CTA b takes entries [32 (4 b + w), +32) of the order by
     // decreasing S, so its lanes have nearly equal S; warps never wait on
@@ -482,9 +484,9 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
                 if (end_of[mid] > g) lo = mid; else hi = mid - 1;
             }
             const int64_t off = g - end_of[lo + 1];
-            if (!in_range(off, a.wl_cap, a.err)) have = false;
+            if (!in_range(off, end_of[lo] - end_of[lo + 1], a.err)) have = false;
             else p = a.wl_bucket[(int64_t)(lo - 1) * a.wl_cap + off];
-            if (have && !in_range(p, count, a.err)) have = false;
+            if (have && !in_range(p, entries, a.err)) have = false;
         }
         if (have) {
             S = a.wl_S[p];

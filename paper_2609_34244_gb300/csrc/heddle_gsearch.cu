@@ -212,7 +212,10 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
     uint32_t* sw = reinterpret_cast<uint32_t*>(smem + ((y.bytes + 127u) & ~127u)) + threadIdx.x;
 
     unsigned long long checks = 0, probes = 0, priced = 0;
-    const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    // the entries filed in the depth buckets (the screen lists the others
+    // for the warp kernel directly)
+    const int64_t entries = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
+    const int64_t count = min((int64_t)end_of[1], entries);
     const int64_t stride = (int64_t)gridDim.x * kGBlock;
     for (int64_t base = ((int64_t)blockIdx.x * kGWarps + warp) * 32; base < count; base += stride) {
         const int64_t g = base + lane;
@@ -223,9 +226,9 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
             if (end_of[mid] > g) lo_d = mid; else hi_d = mid - 1;
         }
         const int64_t off = g - end_of[lo_d + 1];
-        if (!in_range(off, a.wl_cap, a.err)) continue;
+        if (!in_range(off, end_of[lo_d] - end_of[lo_d + 1], a.err)) continue;
         const int64_t p = a.wl_bucket[(int64_t)(lo_d - 1) * a.wl_cap + off];
-        if (!in_range(p, count, a.err)) continue;
+        if (!in_range(p, entries, a.err)) continue;
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p], M = a.wl_M[p];
         const int64_t n = a.wl_n[p];

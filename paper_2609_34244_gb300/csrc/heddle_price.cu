@@ -66,6 +66,8 @@ __device__ __forceinline__ uint32_t stage_desc(int b, const Layout& y, const uns
 // (16-byte vector copies when the planes are aligned), the candidates are
 // counting-sorted by S, and thread i screens the i-th of that order, so the
 // lanes of a warp run stage loops of nearly equal length.
+// kGen: the general search follows (the single-fit routing below is live).
+template <bool kGen>
 __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
     __shared__ uint32_t desc[256];
     __shared__ uint8_t win[8 * 4 * 33];
@@ -78,8 +80,40 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
     __shared__ uint8_t order[kScreenBlock];
     __shared__ int bins[kMaxStages + 3];
     __shared__ int smax;
+    // general search only: per (type, degree, in-flight count) whether any
+    // single layer of the model fits the stage's memory; entries with a
+    // stage where not go straight to the warp-per-entry search's list
+    __shared__ uint8_t sfit[8 * 4 * 33];
+    __shared__ long long single[2];
     const Layout& y = a.lay;
     const int L = y.L;
+    constexpr bool gen = kGen;
+    if (gen) {
+        if (threadIdx.x < 32) {
+            const longlong2* SA = reinterpret_cast<const longlong2*>(a.img + y.offSA);
+            long long m0 = 0, m1 = 0;
+            for (int l = threadIdx.x; l < L; l += 32) {
+                const longlong2 u = SA[l], v = SA[l + 1];
+                m0 = max(m0, v.x - u.x);
+                m1 = max(m1, v.y - u.y);
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                m0 = max(m0, __shfl_xor_sync(0xffffffffu, m0, o));
+                m1 = max(m1, __shfl_xor_sync(0xffffffffu, m1, o));
+            }
+            if (threadIdx.x == 0) {
+                single[0] = m0;
+                single[1] = m1;
+            }
+        }
+        __syncthreads();
+        const int64_t* gmem = reinterpret_cast<const int64_t*>(a.img + y.offMem);
+        for (int i = threadIdx.x; i < 8 * 4 * 33; i += blockDim.x) {
+            const int g = i / 132, j = (i / 33) & 3, f = i % 33;
+            sfit[i] = g < y.NT && single[0] + (long long)f * single[1] <= (long long)(gmem[g] << j);
+        }
+    }
     {
         const int32_t* gcap = reinterpret_cast<const int32_t*>(a.img + y.offCap);
         for (int i = threadIdx.x; i < 256; i += blockDim.x) desc[i] = stage_desc(i, y, a.img, a.moe);
@@ -154,6 +188,7 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
         const bool live = threadIdx.x < nloc;  // padding sorts last
         const int64_t c = c0 + ci;
         int S = 0, M = 0, status = HEDDLE_CAND_INVALID;
+        uint32_t fits1 = 1;  // every stage could hold any single layer (general search)
         int64_t n = 0;
         if (live) {
             S = sS[ci];
@@ -169,9 +204,11 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                     bad |= d;
                     const int g = (d >> 24) & 7;
                     mydem[g * kScreenBlock] += 1u << ((d >> 16) & 31);
-                    const int w = win[(d & 0x7ff) + min(S - s, M)];
+                    const int wi = (d & 0x7ff) + min(S - s, M);
+                    const int w = win[wi];
                     run_sum += w;
                     run_min = min(run_min, w);
+                    if (gen) fits1 &= sfit[wi];
                 }
                 if (bad >> 31) {
                     status = HEDDLE_CAND_INVALID;
@@ -225,10 +262,21 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
                     atomicOr(a.err, kErrInternal);
                 }
             }
-            if (take) {
-                // the entry in its depth's bucket, for the searches' order
-                // by decreasing depth
-                const unsigned same = __match_any_sync(mask, S);
+            // the entry in its depth's bucket, for the searches' order by
+            // decreasing depth -- or, for the general search when some
+            // stage cannot hold every single layer, in the list of the
+            // warp-per-entry search
+            const bool listed = gen && take && !fits1;
+            const unsigned bmask = __ballot_sync(0xffffffffu, take && !listed);
+            const unsigned lmask = __ballot_sync(0xffffffffu, listed);
+            if (lmask) {
+                int l0 = 0;
+                if (lane == __ffs(lmask) - 1) l0 = atomicAdd(a.wl_count + kWlGeneral, __popc(lmask));
+                l0 = __shfl_sync(0xffffffffu, l0, __ffs(lmask) - 1) + __popc(lmask & ((1u << lane) - 1));
+                if (listed && p < a.wl_cap && l0 < a.wl_cap) a.sv_idx[l0] = p;
+            }
+            if (take && !listed) {
+                const unsigned same = __match_any_sync(bmask, S);
                 const int leader = __ffs(same) - 1;
                 int b0 = 0;
                 if (lane == leader) b0 = atomicAdd(a.wl_count + 1 + S, __popc(same));
@@ -266,13 +314,14 @@ cudaError_t launch_screen(const PriceArgs& a, int num_sms, cudaStream_t st, cuda
     static int screen_per_sm = 0;
     if (screen_per_sm == 0) {
         int v = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, screen_kernel, kScreenBlock, 0);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, screen_kernel<false>, kScreenBlock, 0);
         if (e != cudaSuccess) return e;
         screen_per_sm = v > 0 ? v : 1;
     }
     const int grid =
         (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * screen_per_sm);
-    screen_kernel<<<grid, kScreenBlock, 0, st>>>(a);
+    if (!a.uniform && !a.split_mode) screen_kernel<true><<<grid, kScreenBlock, 0, st>>>(a);
+    else screen_kernel<false><<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (launches) launches[0] += 1;
     if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
