@@ -38,7 +38,7 @@ __host__ __device__ inline size_t plan_smem(int NT, int vmax) {
     return (size_t)kPlanBlock * (2 * (size_t)NT * (vmax + 1) + 8 * kMaxTypes);
 }
 
-__global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
+__global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
     const Layout& y = a.lay;
     const int L = y.L, NT = y.NT, V = a.vmax;
     const int64_t* P = reinterpret_cast<const int64_t*>(a.img + y.offP);
@@ -62,16 +62,20 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
     }
     __syncthreads();
     auto H = [&](int g, int v) -> uint16_t& { return hist[(size_t)(g * (V + 1) + v) * kPlanBlock]; };
-    // whole warps step together (lanes past n idle), so the warp can
-    // reconverge before each slot's stores and every store covers whole
-    // 32-byte sectors (a partial sector costs a DRAM read-modify-write)
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t c0 = (int64_t)blockIdx.x * blockDim.x; c0 < a.n; c0 += stride) {
-        const int64_t c = c0 + threadIdx.x;
-        const bool valid = c < a.n;
+    // Most plans end at their first template, whose standalone price is
+    // already what the walk would give it (the whole cluster is free, so
+    // its degree, split and T are the standalone ones): a quick pass writes
+    // such plans' later slots as SKIPPED, and the others are queued in
+    // shared memory and walked 128 at a time, one per thread, so the lanes
+    // that walk are dense.
+    __shared__ int32_t queue[2 * kPlanBlock];
+    __shared__ int queued;
+    if (threadIdx.x == 0) queued = 0;
+    __syncthreads();
+    auto walk = [&](int64_t c) {
         for (int g = 0; g < NT; ++g)
             for (int v = 0; v <= V; ++v) H(g, v) = init[g][v];
-        const int nt = valid ? min((int)a.n_tmpl[c], a.slots) : 0;
+        const int nt = min((int)a.n_tmpl[c], a.slots);
         bool ended = false;
         int placed = 0;
         double thr = 0.0;
@@ -80,8 +84,8 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
             uint8_t st = HEDDLE_CAND_SKIPPED;
             int64_t T = -1, B = -1;
             int64_t n = 0;
-            const int S = valid ? sl.S[c] : 0;
-            const int M = valid ? sl.M[c] : 0;
+            const int S = sl.S[c];
+            const int M = sl.M[c];
             if (!ended && t < nt) {
                 const uint8_t st0 = sl.status[c];
                 if (st0 == HEDDLE_CAND_INVALID) {
@@ -199,8 +203,7 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
                 }
                 if (st != HEDDLE_CAND_OK) ended = true;
             }
-            __syncwarp();
-            if (valid) {
+            {
                 sl.T[c] = T;
                 sl.B[c] = B;
                 sl.ndp[c] = (uint16_t)(st == HEDDLE_CAND_OK || st == HEDDLE_CAND_OOM ? n : 0);
@@ -212,11 +215,56 @@ __global__ void __launch_bounds__(kPlanBlock) plan_kernel(PlanArgs a) {
                 }
             }
         }
-        __syncwarp();
-        if (valid) {
-            a.placed[c] = (uint8_t)placed;
-            a.thr[c] = thr;
+        a.placed[c] = (uint8_t)placed;
+        a.thr[c] = thr;
+    };
+    const int lane = threadIdx.x & 31;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    int64_t c0 = (int64_t)blockIdx.x * blockDim.x;
+    while (true) {
+        const bool more = c0 < a.n;  // uniform over the CTA
+        if (more) {
+            const int64_t c = c0 + threadIdx.x;
+            bool walks = false;
+            if (c < a.n) {
+                const int nt = min((int)a.n_tmpl[c], a.slots);
+                walks = nt >= 1 && a.slot[0].status[c] == HEDDLE_CAND_OK;
+                if (!walks) {
+                    // the first template (if any) keeps its standalone
+                    // price; a walking plan's slots stay untouched here,
+                    // since its walk reads their standalone prices
+                    // (so these stores leave partial sectors: measured
+                    // 710 MB of DRAM traffic per 1e6 plans, 480 us)
+                    for (int t = nt >= 1 ? 1 : 0; t < a.slots; ++t) {
+                        const PlanSlot& sl = a.slot[t];
+                        sl.T[c] = -1;
+                        sl.B[c] = -1;
+                        sl.ndp[c] = 0;
+                        sl.status[c] = HEDDLE_CAND_SKIPPED;
+                        for (int s2 = 0; s2 <= kMaxStages; ++s2) sl.bounds[(int64_t)s2 * sl.bstride + c] = 0;
+                    }
+                    a.placed[c] = 0;
+                    a.thr[c] = 0.0;
+                }
+            }
+            const unsigned wm = __ballot_sync(0xffffffffu, walks);
+            if (wm) {
+                int q0 = 0;
+                if (lane == __ffs(wm) - 1) q0 = atomicAdd(&queued, __popc(wm));
+                q0 = __shfl_sync(0xffffffffu, q0, __ffs(wm) - 1);
+                if (walks) queue[q0 + __popc(wm & ((1u << lane) - 1))] = (int32_t)(c0 + threadIdx.x);
+            }
         }
+        __syncthreads();
+        const int have = queued;
+        const int take = more ? (have >= kPlanBlock ? kPlanBlock : 0) : min(have, kPlanBlock);
+        const int64_t mine = threadIdx.x < take ? (int64_t)queue[have - take + threadIdx.x] : -1;
+        __syncthreads();
+        if (threadIdx.x == 0) queued = have - take;
+        if (mine >= 0) walk(mine);
+        __syncthreads();
+        if (!more && have - take == 0) break;
+        if (more) c0 += stride;
     }
 }
 
