@@ -46,7 +46,9 @@ struct GTabs {
     const int64_t* mem;    // [8]
     const int64_t* inter;  // [8]
     const int64_t* qmax;   // [NT * 4] the most expensive single layer
+    const float* rqavg;    // [NT * 4] 1 / the average layer time
     int64_t smax, amax;    // the largest single-layer state and activation
+    float avs, ava;        // the average layer state and activation bytes
     int L;
 };
 
@@ -83,20 +85,72 @@ __device__ __forceinline__ int64_t cost(const GTabs& t, const GStage& st, int i,
     return t.P[st.row + j] - t.P[st.row + i] + st.c;
 }
 
-// The furthest end j in (u, lim] of a stage starting at u within B and its
-// memory (u if none), by binary search.  acc: the stage time at that end
-// (-1 if none); rej: the stage time at the next end if memory admits it
-// there and its time is above B (kInf otherwise).  checks counts the
-// interval tests.
-__device__ __forceinline__ int reach_of(const GTabs& t, const GStage& st, int u, int lim, int64_t B, int64_t& acc,
-                                        int64_t& rej, unsigned long long& checks) {
-    int lo = u, hi = lim;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        ++checks;
-        if (cost(t, st, u, mid) <= B && fits_mem(t, st, u, mid)) lo = mid;
-        else hi = mid - 1;
+// The largest x in [lo, hi] with ok(x), for a test that holds up to some
+// point and fails beyond it (ok(lo) taken as true), searched from an
+// estimate x0: gallop away from x0 (1, 2, 4, ... positions) until the
+// boundary is bracketed, then bisect.  With a good estimate -- the prefix
+// sums are nearly linear, exactly so for equal layers -- that is two tests
+// instead of a bisection's eight.
+template <class F>
+__device__ __forceinline__ int last_ok(int lo, int hi, int x0, F ok) {
+    x0 = min(max(x0, lo), hi);
+    int a, b;
+    if (x0 == lo || ok(x0)) {
+        int good = x0, step = 1;
+        b = hi;
+        while (true) {
+            const int k = good + step;
+            if (k > hi) break;
+            if (!ok(k)) {
+                b = k - 1;
+                break;
+            }
+            good = k;
+            step <<= 1;
+        }
+        a = good;
+    } else {
+        int fail = x0, step = 1;
+        a = lo;
+        while (true) {
+            const int k = fail - step;
+            if (k <= lo) break;
+            if (ok(k)) {
+                a = k;
+                break;
+            }
+            fail = k;
+            step <<= 1;
+        }
+        b = fail - 1;
     }
+    while (a < b) {
+        const int mid = (a + b + 1) >> 1;
+        if (ok(mid)) a = mid;
+        else b = mid - 1;
+    }
+    return a;
+}
+
+// Layers of stage st that a bound B and its memory admit, estimated from
+// the average layer time and footprint (for the searches' first guesses).
+__device__ __forceinline__ float layers_est(const GTabs& t, const GStage& st, int row_idx, int64_t room) {
+    const float by_time = room > 0 ? u64_to_float((uint64_t)room) * t.rqavg[row_idx] : 0.f;
+    const float by_mem = u64_to_float((uint64_t)st.capk) / fmaxf(t.avs + (float)st.f * t.ava, 1.f);
+    return fminf(fminf(by_time, by_mem), (float)t.L);
+}
+
+// The furthest end j in (u, lim] of a stage starting at u within B and its
+// memory (u if none).  acc: the stage time at that end (-1 if none); rej:
+// the stage time at the next end if memory admits it there and its time is
+// above B (kInf otherwise).  checks counts the interval tests.
+__device__ __forceinline__ int reach_of(const GTabs& t, const GStage& st, int row_idx, int u, int lim, int64_t B,
+                                        int64_t& acc, int64_t& rej, unsigned long long& checks) {
+    const int x0 = u + (int)layers_est(t, st, row_idx, B - st.c);
+    const int lo = last_ok(u, lim, x0, [&](int j) {
+        ++checks;
+        return cost(t, st, u, j) <= B && fits_mem(t, st, u, j);
+    });
     acc = lo > u ? cost(t, st, u, lo) : -1;
     rej = kInf;
     if (lo < lim && fits_mem(t, st, u, lo + 1)) {
@@ -116,9 +170,10 @@ __device__ bool gprobe(const GTabs& t, const uint32_t* sw, int S, int64_t B, int
     lo = kInf;
     int u = 0;
     for (int s = 0; s + 1 < S; ++s) {
-        const GStage st = unpack(sw[s * kGBlock], t);
+        const uint32_t w = sw[s * kGBlock];
+        const GStage st = unpack(w, t);
         int64_t acc, rej;
-        const int r = reach_of(t, st, u, L - (S - 1 - s), B, acc, rej, checks);
+        const int r = reach_of(t, st, (w & 7) * 4 + ((w >> 3) & 3), u, L - (S - 1 - s), B, acc, rej, checks);
         lo = min(lo, rej);
         if (r < s + 1) return false;
         hi = max(hi, acc);
@@ -204,8 +259,14 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
     t.mem = reinterpret_cast<const int64_t*>(smem + y.offMem);
     t.inter = reinterpret_cast<const int64_t*>(smem + y.offInter);
     t.qmax = qmax;
+    t.rqavg = rqavg;
     t.smax = single[0];
     t.amax = single[1];
+    {
+        const longlong2 all = t.SA[L];
+        t.avs = u64_to_float((uint64_t)all.x) / (float)L;
+        t.ava = u64_to_float((uint64_t)all.y) / (float)L;
+    }
     t.L = L;
     const int32_t* maxn = reinterpret_cast<const int32_t*>(smem + y.offMaxN);
     const int64_t* minq = reinterpret_cast<const int64_t*>(smem + y.offMinQ);
@@ -265,11 +326,8 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
             hiB = max(hiB, t.P[st.row + L] + st.c);
             memall &= t.smax + st.f * t.amax <= st.capk;
             // the longest run [0, r) within memory (for the guess)
-            int r0 = 0, r1 = L;
-            while (r0 < r1) {
-                const int mid = (r0 + r1 + 1) >> 1;
-                if (fits_mem(t, st, 0, mid)) r0 = mid; else r1 = mid - 1;
-            }
+            const int r0 = last_ok(0, L, (int)layers_est(t, st, gg * 4 + jj, kInf),
+                                   [&](int r) { return fits_mem(t, st, 0, r); });
             w |= (uint32_t)r0 << kVShift;
             sw[s * kGBlock] = w;
         }
@@ -383,14 +441,15 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
             for (int s = S - 1; s >= 1; --s) {
                 const uint32_t w = sw[s * kGBlock];
                 const GStage st = unpack(w, t);
-                int l0 = s, l1 = v - 1;  // l1 holds a single layer
-                while (l0 < l1) {
-                    const int mid = (l0 + l1) >> 1;
+                // the most layers y + 1 ending at v that stage s holds
+                // within B* (v - 1 holds a single layer), from the estimate
+                const int vv = v;
+                const int y0 = (int)layers_est(t, st, (w & 7) * 4 + ((w >> 3) & 3), Bstar - st.c) - 1;
+                const int y = last_ok(0, vv - 1 - s, y0, [&](int yy) {
                     ++checks;
-                    if (cost(t, st, mid, v) <= Bstar && fits_mem(t, st, mid, v)) l1 = mid;
-                    else l0 = mid + 1;
-                }
-                v = l0;
+                    return cost(t, st, vv - 1 - yy, vv) <= Bstar && fits_mem(t, st, vv - 1 - yy, vv);
+                });
+                v = vv - 1 - y;
                 sw[s * kGBlock] = (w & kNoV) | ((uint32_t)v << kVShift);
             }
         }
