@@ -478,6 +478,17 @@ heddle_status heddle_device_errors(heddle_ctx* ctx, uint32_t* flags);
 heddle_status heddle_set_search(heddle_ctx* ctx, int32_t mode);
 heddle_status heddle_get_search(heddle_ctx* ctx, int32_t* in_use);
 
+/* Routing of the general search (models whose layers differ, §3.1
+ * PartitionLayers) between its two kernels.  The thread-per-entry search
+ * takes the worklist entries whose stages could each hold any single layer
+ * when there are at least min_entries of them, and the warp-per-entry
+ * search prices the rest; with fewer, the warp search prices every entry
+ * (a thread search with too few entries runs as long as its longest serial
+ * chain).  min_entries < 0 restores the default, 32 x the device's SM
+ * count; 0 always runs the thread search.  Both routes return identical
+ * results.  Errors: E_ARG (ctx NULL). */
+heddle_status heddle_set_thread_search_min(heddle_ctx* ctx, int32_t min_entries);
+
 /* Work counters of the next heddle_price_candidates call on ctx, for the
  * roofline report: when enabled, that call runs the counting variant of the
  * pricing kernel and accumulates, in device memory owned by ctx,

@@ -30,6 +30,7 @@ struct heddle_ctx {
     bool tables_ready = false;
     int32_t model_flags[4] = {0, 0, 0, 0};  // copy of the image's model flags
     int32_t search_mode = HEDDLE_SEARCH_AUTO;
+    int32_t thread_min = -1;  // heddle_set_thread_search_min (< 0: the default)
     unsigned char* d_img = nullptr;
     size_t img_cap = 0;
     int64_t* d_q = nullptr;
@@ -734,6 +735,7 @@ void fill_price_args(heddle_ctx* x, const heddle_candidates* c, const heddle_ctx
     a.wl_cap = hd::kWorklistCap;
     a.uniform = !tiled && equal_layer_search(x, lvl ? lvl->flags : x->model_flags) ? 1 : 0;
     a.split_mode = x->search_mode == HEDDLE_SEARCH_DISTRIBUTE ? 1 : 0;
+    a.thread_min = x->thread_min < 0 ? hd::thread_search_min(x->num_sms) : x->thread_min;
 }
 
 // One chunk [lo, lo + nb) of cands into r: screen and search on `ws` with
@@ -1134,6 +1136,12 @@ heddle_status heddle_set_search(heddle_ctx* x, int32_t mode) {
     if (mode != HEDDLE_SEARCH_AUTO && mode != HEDDLE_SEARCH_GENERAL && mode != HEDDLE_SEARCH_DISTRIBUTE)
         return fail(x, HEDDLE_E_ARG, "unknown search mode %d", mode);
     x->search_mode = mode;
+    return ok(x);
+}
+
+heddle_status heddle_set_thread_search_min(heddle_ctx* x, int32_t min_entries) {
+    if (!x) return HEDDLE_E_ARG;
+    x->thread_min = min_entries < 0 ? -1 : min_entries;
     return ok(x);
 }
 

@@ -197,6 +197,8 @@ __device__ __forceinline__ void defer(const PriceArgs& a, int64_t p) {
     if (in_range(pos, a.wl_cap, a.err)) a.sv_idx[pos] = (int32_t)p;
 }
 
+// Below a.thread_min bucketed entries the kernel returns at once and the
+// warp kernel prices the whole worklist.
 template <bool kCount>
 __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -206,8 +208,21 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
     __shared__ int end_of[kMaxStages + 2];
     const Layout& y = a.lay;
     const int L = y.L;
-    if (!wp::load_image(smem, a.img, y.bytes, &bar, a.err)) return;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (threadIdx.x < 32) {
+        // end_of[S] = entries of depths >= S (see eq_search_kernel)
+        int x = a.wl_count[1 + (kMaxStages - lane)];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y2 = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y2;
+        }
+        end_of[kMaxStages - lane] = x;
+        if (lane == 0) end_of[kMaxStages + 1] = 0;
+    }
+    __syncthreads();
+    if (end_of[1] < a.thread_min) return;
+    if (!wp::load_image(smem, a.img, y.bytes, &bar, a.err)) return;
     {
         const int64_t* P = reinterpret_cast<const int64_t*>(smem + y.offP);
         const longlong2* SA = reinterpret_cast<const longlong2*>(smem + y.offSA);
@@ -238,17 +253,6 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
         }
         const int64_t* p2p = reinterpret_cast<const int64_t*>(smem + y.offP2P);
         for (int i = threadIdx.x; i < 129; i += blockDim.x) cfl[i] = i < 128 ? u64_to_float((uint64_t)p2p[i]) : 0.f;
-        if (threadIdx.x < 32) {
-            // end_of[S] = entries of depths >= S (see eq_search_kernel)
-            int x = a.wl_count[1 + (kMaxStages - lane)];
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int y2 = __shfl_up_sync(0xffffffffu, x, o);
-                if (lane >= o) x += y2;
-            }
-            end_of[kMaxStages - lane] = x;
-            if (lane == 0) end_of[kMaxStages + 1] = 0;
-        }
         __syncthreads();
     }
     GTabs t;

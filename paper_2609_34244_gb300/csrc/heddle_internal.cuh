@@ -11,6 +11,7 @@ namespace hd {
 
 constexpr int kMaxTypes = HEDDLE_MAX_TYPES;
 constexpr int kMaxStages = HEDDLE_MAX_STAGES;
+static_assert(kMaxStages == 32, "the searches hold one stage (or one depth) per lane");
 constexpr int kMaxLayers = HEDDLE_MAX_LAYERS;
 constexpr int kMaxTopK = HEDDLE_MAX_TOPK;
 constexpr int64_t kInf = INT64_MAX;
@@ -146,6 +147,7 @@ struct PriceArgs {
     int32_t uniform;     // search with the equal-layer closed form (model flags [0] and [1])
     int32_t mbs_shift;   // micro-batch size 2^shift: M >> shift micro-batches (invalid unless 2^shift | M)
     int32_t split_mode;  // 1: the paper's own split rule (distribute_kernel) instead of PartitionLayers
+    int32_t thread_min;  // general search: the bucketed entries below which only the warp search runs
     // per worklist entry, written by the search: T (-1 unless OK) and n * M,
     // so a top-k can run over the searched candidates only
     int64_t* wl_T;
@@ -208,6 +210,11 @@ cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
 constexpr int kWlMeta = 1 + kMaxStages + 1 + 1;  // ints of a.wl_count
 constexpr int kWlGeneral = 1;  // entries the thread-per-entry general search left to the warp search
+// The thread-per-entry general search runs when the depth buckets hold at
+// least one warp of entries per SM; with fewer it would run one warp or less
+// per SM, its time the latency of its longest serial chain, and the warp
+// search (whose probes spread over 32 lanes) prices every entry instead.
+inline int thread_search_min(int num_sms) { return num_sms * 32; }
 constexpr int kWlSurv = kWlMeta - 1;             // the survivor count (see PriceArgs::sv_count)
 
 

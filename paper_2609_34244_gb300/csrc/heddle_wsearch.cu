@@ -19,6 +19,8 @@
 // ceiling division for the gradient term.  The table image is staged into
 // shared memory with bulk asynchronous copies.
 
+#include <climits>
+
 #include "heddle_wprobe.cuh"
 
 namespace hd {
@@ -97,10 +99,12 @@ __device__ __noinline__ int64_t plain_guess(const int64_t* P, const longlong2* S
     return wp::first_guess(rq, cf, mr, S, L, hi);
 }
 
-// listed: the entries of the list the thread-per-entry search left
-// (a.sv_idx, count at wl_count[kWlGeneral]); else every worklist entry.
+// The entries of the list the thread-per-entry search left (a.sv_idx,
+// count at wl_count[kWlGeneral]) -- or every worklist entry when the depth
+// buckets hold fewer than thread_min entries (that search then ran none;
+// thread_min is a.thread_min, or INT_MAX for the whole worklist).
 template <bool kCount>
-__global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a, int listed) {
+__global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a, int thread_min) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     __shared__ int64_t qmax[4 * kMaxTypes], single[2];
@@ -153,6 +157,10 @@ __global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a, int li
     WarpArea& wa = reinterpret_cast<WarpArea*>(smem + ((y.bytes + 127u) & ~127u))[warp];
 
     unsigned long long checks = 0, probes = 0, priced = 0;
+    int bucketed = a.wl_count[1 + 1 + lane];  // depth 1 + lane
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) bucketed += __shfl_xor_sync(kFull, bucketed, o);
+    const bool listed = bucketed >= thread_min;
     const int64_t count = min((int64_t)(listed ? a.wl_count[kWlGeneral] : *a.wl_count), (int64_t)a.wl_cap);
     const int64_t nwarps = (int64_t)gridDim.x * kWarps;
     for (int64_t e = (int64_t)blockIdx.x * kWarps + warp; e < count; e += nwarps) {
@@ -342,7 +350,7 @@ cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st, bool listed
     // at most one wave
     const int64_t need = (a.n + kWarps - 1) / kWarps;
     const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
-    wsearch_kernel<kCount><<<grid, kWBlock, smem, st>>>(a, listed ? 1 : 0);
+    wsearch_kernel<kCount><<<grid, kWBlock, smem, st>>>(a, listed ? a.thread_min : INT_MAX);
     return cudaGetLastError();
 }
 

@@ -79,7 +79,7 @@ TOPK_STATE_BYTES = C.sizeof(heddle_topk_state)
 EXPORTS = ["heddle_create", "heddle_destroy", "heddle_last_error", "heddle_load_cluster",
            "heddle_load_model", "heddle_price_candidates", "heddle_topk_reset", "heddle_topk",
            "heddle_price_topk_host", "heddle_get_tables", "heddle_device_errors",
-           "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search",
+           "heddle_count_next", "heddle_work_counters", "heddle_set_search", "heddle_get_search", "heddle_set_thread_search_min",
            "heddle_price_topk", "heddle_topk_noalloc", "heddle_time_phases", "heddle_phase_times",
            "heddle_load_mbs", "heddle_price_mbs", "heddle_price_plans", "heddle_load_experts",
            "heddle_price_tiled", "heddle_set_chunk"]
@@ -117,6 +117,7 @@ def load_library(path: str = LIB_PATH):
         "heddle_count_next": (i32, [p, i32]),
         "heddle_work_counters": (i32, [p, C.POINTER(C.c_uint64)]),
         "heddle_set_search": (i32, [p, i32]),
+        "heddle_set_thread_search_min": (i32, [p, i32]),
         "heddle_get_search": (i32, [p, C.POINTER(C.c_int32)]),
         "heddle_time_phases": (i32, [p, i32]),
         "heddle_load_mbs": (i32, [p, i32, p]),
@@ -390,6 +391,12 @@ def heddle_phase_times(ctx):
 
 def heddle_set_search(ctx, mode: int):
     _check(ctx, load_library().heddle_set_search(ctx, int(mode)))
+
+
+def heddle_set_thread_search_min(ctx, min_entries: int):
+    """Bucketed entries from which the general search runs its
+    thread-per-entry kernel (< 0: the default, 32 x the SM count)."""
+    _check(ctx, load_library().heddle_set_thread_search_min(ctx, int(min_entries)))
 
 
 def heddle_get_search(ctx) -> int:

@@ -20,10 +20,12 @@ def main():
     cases = (("tiny_ext", None), ("dense32", 30011), ("dense80", 20011), ("moe48", 30011), ("stress128", 150001))
     for name, n in cases:
         w = W.make_workload(name, seed=3, n=n)
-        for mode, split in ((h.SEARCH_AUTO, "minmax"), (h.SEARCH_GENERAL, "minmax"), (h.SEARCH_DISTRIBUTE, "distribute")):
+        for mode, split, tmin in ((h.SEARCH_AUTO, "minmax", None), (h.SEARCH_GENERAL, "minmax", None),
+                                  (h.SEARCH_GENERAL, "minmax", 0), (h.SEARCH_DISTRIBUTE, "distribute", None)):
             ref = O.Oracle(w.cluster, w.model).set_split(split).price(w.cands, threads=8)
             for fused in (False, True):
-                got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, search=mode, fused=fused, chunk=65536)
+                got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, search=mode, fused=fused, chunk=65536,
+                                  thread_min=tmin)
                 assert got["errors"] == 0, "%s mode %d: device flags %#x" % (name, mode, got["errors"])
                 G.assert_same(got, ref, what="%s mode %d fused %s" % (name, mode, fused))
                 exp = O.topk(ref, w.cands["M"], 16)

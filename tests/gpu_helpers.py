@@ -9,14 +9,16 @@ import numpy as np
 
 
 def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count=False, search=None,
-              fused=False, phases=False, chunk=None):
+              fused=False, phases=False, chunk=None, thread_min=None):
     """Price on the GPU through the C ABI; returns numpy results, the top-k
     and (optionally) the work counters.  ``batch`` splits the candidates into
     consecutive launches merged into one top-k state; ``fused`` prices and
     merges in one call (heddle_price_topk); ``phases`` times the pricing
     phases with the library's events and returns them under "phases";
     ``chunk`` sets the library's chunk size (calls of several chunks are
-    pipelined over its work streams)."""
+    pipelined over its work streams); ``thread_min`` sets the general
+    search's routing threshold (0: thread kernel whenever it has entries,
+    2**31 - 1: warp kernel only)."""
     import torch
     ctx = h.heddle_create(0)
     try:
@@ -26,6 +28,8 @@ def price_gpu(h, w_cluster, w_model, cands, k=16, bounds=True, batch=None, count
             h.heddle_set_search(ctx, search)
         if chunk is not None:
             h.heddle_set_chunk(ctx, chunk)
+        if thread_min is not None:
+            h.heddle_set_thread_search_min(ctx, thread_min)
         n = int(cands["S"].shape[0])
         dc = h.cands_to_device(cands)
         res = h.alloc_results(n, bounds=False)

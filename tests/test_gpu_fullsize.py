@@ -76,6 +76,20 @@ def test_full_size(heddle_lib, oracle_mod, name, n, search, path):
     assert tk["nM"].tolist() == top["nM"].tolist()
 
 
+@pytest.mark.parametrize("thread_min", [0, 2**31 - 1], ids=["thread", "warp"])
+def test_full_size_general_routes(heddle_lib, oracle_mod, thread_min):
+    """moe48 at full size with the general search's routing forced each way
+    (by default its few single-fit entries go to the warp kernel)."""
+    h = heddle_lib
+    name, n = "moe48", 1_000_000
+    w, ref, top = _oracle_full(oracle_mod, name, n)
+    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=F.TOPK, bounds=False, search=h.SEARCH_GENERAL,
+                      fused=True, chunk=1_000_000, thread_min=thread_min)
+    assert got["errors"] == 0
+    G.assert_same(got, ref, what="moe48 thread_min %d" % thread_min)
+    assert got["topk"]["idx"].tolist() == top["idx"].tolist()
+
+
 def test_one_call_larger_than_the_worklist(heddle_lib, oracle_mod):
     """A single pricing call of 1.2e6 candidates (more than one 2^20-candidate
     worklist chunk) with bounds, checked on a sample."""

@@ -35,14 +35,20 @@ SMALL = [("tiny", None), ("tiny_ext", None), ("dense32", 6007), ("dense80", 1531
 EQUAL = {"dense32", "dense80", "stress128"}
 
 
+# the general search's two routes forced: the thread-per-entry kernel
+# wherever it has entries, or the warp-per-entry kernel for every entry
+ROUTES = {"auto": (0, None), "general": (1, None), "thread": (1, 0), "warp": (1, 2**31 - 1)}
+
+
 @pytest.mark.parametrize("name,n", SMALL)
 @pytest.mark.parametrize("seed", [0, 1])
-@pytest.mark.parametrize("search", [0, 1], ids=["auto", "general"])
-def test_parity_small(h, W, oracle_mod, name, n, seed, search):
+@pytest.mark.parametrize("route", list(ROUTES))
+def test_parity_small(h, W, oracle_mod, name, n, seed, route):
+    search, thread_min = ROUTES[route]
     w = W.make_workload(name, seed=seed, n=n)
     orc = oracle_mod.Oracle(w.cluster, w.model)
     ref = orc.price(w.cands, threads=8)
-    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, search=search)
+    got = G.price_gpu(h, w.cluster, w.model, w.cands, k=16, search=search, thread_min=thread_min)
     assert got["errors"] == 0
     assert got["search"] == (2 if (search == 0 and name in EQUAL) else 1)
     G.assert_same(got, ref, what=name)
