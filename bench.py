@@ -85,7 +85,8 @@ def screen_ops(cands) -> int:
 
 
 SEARCH_NAMES = {1: "general interval search", 2: "equal-layer closed form"}
-SEARCH_KERNELS = {1: "wsearch_kernel (general threshold search, one warp per entry)",
+SEARCH_KERNELS = {1: "gsearch_kernel + wsearch_kernel (general threshold search: one thread per single-fit "
+                     "entry when there are at least 32 per SM, one warp per entry for the rest)",
                   2: "eq_search_kernel (equal-layer closed form)"}
 LANES_PER_SM = 128  # 4 SM sub-partitions x 32 lanes issue per clock; the SM count comes from the device
 
@@ -94,7 +95,7 @@ LANES_PER_SM = 128  # 4 SM sub-partitions x 32 lanes issue per clock; the SM cou
 # sources it was taken on; reported as null once those sources change.
 TRAFFIC = {2: {"bytes": 15309824, "batch": 1000000,
               "sha256": "80e96c99741dac1063e4533d8627886bbd8862ce4db740e2bced451141e957cb"}}
-TRAFFIC_SOURCES = {1: ["heddle_price.cu", "heddle_internal.cuh"],
+TRAFFIC_SOURCES = {1: ["heddle_gsearch.cu", "heddle_wsearch.cu", "heddle_wprobe.cuh", "heddle_internal.cuh"],
                    2: ["heddle_eqsearch.cu", "heddle_internal.cuh"]}
 
 
@@ -386,6 +387,8 @@ def main():
     ap.add_argument("--no-distribute", action="store_true", help="skip the paper's-split comparison figure")
     ap.add_argument("--plans", type=int, default=1_000_000, help="multi-template plans of the plan figure (0: skip)")
     ap.add_argument("--no-per-config", action="store_true", help="skip the per-workload measurements")
+    ap.add_argument("--configs", default=",".join(PER_CONFIG),
+                    help="comma-separated workloads of the per-workload measurements")
     ap.add_argument("--tiling", type=int, default=1_000_000,
                     help="moe48 candidates of the expert-tiling figure (0: skip)")
     args = ap.parse_args()
@@ -733,7 +736,11 @@ def main():
     peaks, peak_kind = load_peaks()
     per_config = None
     if not args.no_per_config:
-        per_config = [measure_config(h, name, peaks, sms) for name in PER_CONFIG]
+        names = [x for x in args.configs.split(",") if x]
+        unknown = sorted(set(names) - set(PER_CONFIG))
+        if unknown:
+            raise SystemExit("unknown workloads in --configs: %s" % ", ".join(unknown))
+        per_config = [measure_config(h, name, peaks, sms) for name in names]
     value = n * world * args.steps / (ms_all / 1e3)
     ops_step = work["checks"] * OPS_PER_UNIT[search]
     peak_tops = sms * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12
