@@ -281,8 +281,15 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
     // for the warp kernel directly)
     const int64_t entries = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const int64_t count = min((int64_t)end_of[1], entries);
-    const int64_t stride = (int64_t)gridDim.x * kGBlock;
-    for (int64_t base = ((int64_t)blockIdx.x * kGWarps + warp) * 32; base < count; base += stride) {
+    // each warp prices 32 entries (deepest first): its own first, then the
+    // next untaken ones whenever it is free
+    const int64_t first = (int64_t)gridDim.x * kGBlock;
+    auto take = [&]() {
+        int b = 0;
+        if (lane == 0) b = atomicAdd(a.wl_count + kWlTakeThread, 32);
+        return first + __shfl_sync(0xffffffffu, b, 0);
+    };
+    for (int64_t base = ((int64_t)blockIdx.x * kGWarps + warp) * 32; base < count; base = take()) {
         const int64_t g = base + lane;
         if (g >= count) continue;
         int lo_d = 1, hi_d = kMaxStages;
@@ -303,19 +310,15 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
         // pack the stages; the single-fit threshold QC (no bound below it
         // is single-fit), the memory test, a bound feasible whenever
         // memory is, and each stage's memory run from layer 0 for the guess
-        uint32_t cw4[8];
-        {
-            const uint4* row = reinterpret_cast<const uint4*>(a.wl_code + p * kMaxStages);
-            const uint4 v0 = __ldg(row);
-            const uint4 v1 = S > 16 ? __ldg(row + 1) : make_uint4(0, 0, 0, 0);
-            cw4[0] = v0.x; cw4[1] = v0.y; cw4[2] = v0.z; cw4[3] = v0.w;
-            cw4[4] = v1.x; cw4[5] = v1.y; cw4[6] = v1.z; cw4[7] = v1.w;
-        }
+        // (the entry's 32-byte row of stage bytes, read a byte per stage:
+        // an array indexed by the stage would live in local memory)
+        const uint8_t* row = a.wl_code + p * kMaxStages;
         int64_t QC = 0, hiB = 0, LB = 0;
         bool memall = true;
+        int next = __ldg(row);
         for (int s = 0; s < S; ++s) {
-            const int code = (cw4[s >> 2] >> ((s & 3) * 8)) & 0xff;
-            const int next = s + 1 < kMaxStages ? (cw4[(s + 1) >> 2] >> (((s + 1) & 3) * 8)) & 0xff : 0;
+            const int code = next;
+            next = s + 1 < S ? __ldg(row + s + 1) : 0;
             const int gg = code & 7, jj = (code >> 3) & 3;
             int pidx = kGZeroP2P;
             if (s + 1 < S) {

@@ -133,8 +133,8 @@ struct PriceArgs {
     unsigned long long* counters;  // non-null selects the counting variant
     // worklist of the candidates that need the threshold search (device
     // scratch owned by the context, capacity wl_cap candidates)
-    int32_t* wl_count;   // [1 + kMaxStages + 1]: entries, then per depth S the entries of
-                         // that depth (equal-layer search; cleared per chunk)
+    int32_t* wl_count;   // [kWlMeta]: entries, the general list, per depth S the entries
+                         // of that depth, two take counters, survivors (cleared per chunk)
     int32_t* wl_idx;
     uint16_t* wl_n;
     uint16_t* wl_M;
@@ -208,8 +208,12 @@ cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st);
 // The paper's own layer split over the worklist (comparison mode).
 cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);
 constexpr int32_t kWorklistCap = 1 << 20;
-constexpr int kWlMeta = 1 + kMaxStages + 1 + 1;  // ints of a.wl_count
+constexpr int kWlMeta = 1 + kMaxStages + 1 + 2 + 1;  // ints of a.wl_count
 constexpr int kWlGeneral = 1;  // entries the thread-per-entry general search left to the warp search
+// the next entries the general searches take (each warp of the thread
+// search takes 32 at a time, each warp of the warp search one)
+constexpr int kWlTakeThread = kWlMeta - 3;
+constexpr int kWlTakeWarp = kWlMeta - 2;
 // The thread-per-entry general search runs when the depth buckets hold at
 // least one warp of entries per SM; with fewer it would run one warp or less
 // per SM, its time the latency of its longest serial chain, and the warp

@@ -162,8 +162,15 @@ __global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a, int th
     for (int o = 16; o > 0; o >>= 1) bucketed += __shfl_xor_sync(kFull, bucketed, o);
     const bool listed = bucketed >= thread_min;
     const int64_t count = min((int64_t)(listed ? a.wl_count[kWlGeneral] : *a.wl_count), (int64_t)a.wl_cap);
-    const int64_t nwarps = (int64_t)gridDim.x * kWarps;
-    for (int64_t e = (int64_t)blockIdx.x * kWarps + warp; e < count; e += nwarps) {
+    // each warp prices its own first entry, then the next untaken one
+    // whenever it is free
+    const int64_t first = (int64_t)gridDim.x * kWarps;
+    auto take = [&]() {
+        int e = 0;
+        if (lane == 0) e = atomicAdd(a.wl_count + kWlTakeWarp, 1);
+        return first + __shfl_sync(kFull, e, 0);
+    };
+    for (int64_t e = (int64_t)blockIdx.x * kWarps + warp; e < count; e = take()) {
         const int64_t p = listed ? a.sv_idx[e] : e;
         if (!in_range(p, a.wl_cap, a.err)) continue;
         const int64_t c = a.wl_idx[p];
