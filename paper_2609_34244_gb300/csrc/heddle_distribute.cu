@@ -92,8 +92,15 @@ __global__ void __launch_bounds__(kDistBlock) distribute_kernel(PriceArgs a) {
     const uint8_t* win = a.img + y.offWin;
     const int lane = threadIdx.x & 31;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t warps = (int64_t)gridDim.x * (blockDim.x >> 5);
-    for (int64_t p = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); p < count; p += warps) {
+    // each warp prices its own first entry, then the next untaken one
+    // whenever it is free
+    const int64_t first = (int64_t)gridDim.x * (blockDim.x >> 5);
+    auto take = [&]() {
+        int e = 0;
+        if (lane == 0) e = atomicAdd(a.wl_count + kWlTakeWarp, 1);
+        return first + __shfl_sync(kFull, e, 0);
+    };
+    for (int64_t p = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); p < count; p = take()) {
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
         if (!in_range(c, a.n, a.err) || !in_range(S - 1, kMaxStages, a.err)) continue;

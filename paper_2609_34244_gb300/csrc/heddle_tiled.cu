@@ -321,8 +321,15 @@ __global__ void __launch_bounds__(kTBlock, 3) tiled_search_kernel(PriceArgs a, T
     wp::WarpArea& wa = reinterpret_cast<wp::WarpArea*>(smem + ((y.bytes + 127u) & ~127u))[warp];
     unsigned long long checks = 0;
     const int64_t count = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
-    const int64_t nwarps = (int64_t)gridDim.x * kTWarps;
-    for (int64_t p = (int64_t)blockIdx.x * kTWarps + warp; p < count; p += nwarps) {
+    // each warp prices its own first entry, then the next untaken one
+    // whenever it is free
+    const int64_t first = (int64_t)gridDim.x * kTWarps;
+    auto take = [&]() {
+        int e = 0;
+        if (lane == 0) e = atomicAdd(a.wl_count + kWlTakeWarp, 1);
+        return first + __shfl_sync(wp::kFull, e, 0);
+    };
+    for (int64_t p = (int64_t)blockIdx.x * kTWarps + warp; p < count; p = take()) {
         const int64_t c = a.wl_idx[p];
         const int S = a.wl_S[p];
         if (!in_range(c, a.n, a.err) || !in_range(S - 1, kMaxStages, a.err)) continue;
