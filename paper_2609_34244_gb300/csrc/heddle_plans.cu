@@ -136,11 +136,12 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
                         int64_t tmax = 0, tsum = 0;
                         uint64_t bestG = 0, bestD = 1;
                         int sg = -1;
+                        int hi = sl.bounds[c];
                         for (int s = 0; s < S; ++s) {
                             const int b = sl.code[(int64_t)s * sl.stride + c];
                             const int g = b & 7, j = (b >> 3) & 3;
-                            const int lo = sl.bounds[(int64_t)s * sl.bstride + c];
-                            const int hi = sl.bounds[(int64_t)(s + 1) * sl.bstride + c];
+                            const int lo = hi;
+                            hi = sl.bounds[(int64_t)(s + 1) * sl.bstride + c];
                             int64_t cs = 0;
                             if (s + 1 < S) {
                                 const int bn = sl.code[(int64_t)(s + 1) * sl.stride + c];
@@ -208,11 +209,10 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
                 sl.B[c] = B;
                 sl.ndp[c] = (uint16_t)(st == HEDDLE_CAND_OK || st == HEDDLE_CAND_OOM ? n : 0);
                 sl.status[c] = st;
-                // every lane rewrites all planes (its split, or zeros unless OK)
-                for (int s = 0; s <= kMaxStages; ++s) {
-                    uint8_t* bp = sl.bounds + (int64_t)s * sl.bstride + c;
-                    *bp = st == HEDDLE_CAND_OK ? *bp : (uint8_t)0;
-                }
+                // an OK template keeps its standalone split; any other
+                // status clears the planes
+                if (st != HEDDLE_CAND_OK)
+                    for (int s = 0; s <= kMaxStages; ++s) sl.bounds[(int64_t)s * sl.bstride + c] = 0;
             }
         }
         a.placed[c] = (uint8_t)placed;
