@@ -415,6 +415,7 @@ def main():
 
     torch.cuda.set_device(local)
     sms = torch.cuda.get_device_properties(local).multi_processor_count
+    peaks, peak_kind = load_peaks()
     group = shard.init(world)
     n, batch = args.n, min(args.batch, args.n)
     # weak scaling: rank r prices its own n candidates (seed r), global indices r*n + c
@@ -573,11 +574,22 @@ def main():
         gph = h.heddle_phase_times(ctx)
         gsearch_ms = gph["search"][0] / 2
         gtopk = h.read_topk_state(state)
+        # the search kernels' own time: one call per batch, no overlap
+        h.heddle_time_phases(ctx, True)
+        h.heddle_topk_reset(ctx, state, 16, stream)
+        for c, r in cbatches:
+            h.heddle_price_topk(ctx, c, r, state, stream)
+        torch.cuda.synchronize()
+        h.heddle_time_phases(ctx, False)
+        giso_ms = h.heddle_phase_times(ctx)["search"][0]
         general = {"value": n / (gms / 1e3), "ms_per_step": gms, "search_ms_per_step": gsearch_ms,
+                   "search_us_per_batch_isolated": 1e3 * giso_ms / n_batches,
                    "checks_per_candidate": gwork["checks"] / n,
                    "probes_per_searched": gwork["probes"] / max(1, gwork["priced"]),
-                   "alu_frac": gwork["checks"] * OPS_PER_UNIT[1] / (gsearch_ms / 1e3) / 1e12 /
-                   (sms * LANES_PER_SM * 2070.0 * 1e6 / 1e12),
+                   "alu_frac": gwork["checks"] * OPS_PER_UNIT[1] / (giso_ms / 1e3) / 1e12 /
+                   (sms * LANES_PER_SM * float(peaks.get("sm_max_mhz", 2070.0)) * 1e6 / 1e12),
+                   "alu_frac_basis": "interval tests x 16 lane operations over the search kernels' "
+                                     "isolated time (one call per batch)",
                    "same_topk": gtopk["idx"].tolist() == local_topk["idx"].tolist()}
         h.heddle_set_search(ctx, h.SEARCH_AUTO)
 
@@ -733,7 +745,6 @@ def main():
 
     if rank != 0:
         return
-    peaks, peak_kind = load_peaks()
     per_config = None
     if not args.no_per_config:
         names = [x for x in args.configs.split(",") if x]
