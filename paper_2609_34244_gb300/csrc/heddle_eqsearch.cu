@@ -621,11 +621,8 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
 template <bool kCount>
 cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const size_t smem = eq_layout(a.lay.L).bytes;
-    cudaError_t e = cudaFuncSetAttribute(eq_search_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
-    if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, eq_search_kernel<kCount>, kEqBlock, smem);
+    const cudaError_t e = resident_blocks(reinterpret_cast<const void*>(&eq_search_kernel<kCount>), kEqBlock, smem, &per_sm);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     // the worklist length is only known on the device: size for the batch

@@ -524,10 +524,8 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
 template <bool kCount>
 cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const size_t smem = ((a.lay.bytes + 127u) & ~127u) + sizeof(uint32_t) * kMaxStages * kGBlock;
-    cudaError_t e = cudaFuncSetAttribute(gsearch_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gsearch_kernel<kCount>, kGBlock, smem);
+    const cudaError_t e = resident_blocks(reinterpret_cast<const void*>(&gsearch_kernel<kCount>), kGBlock, smem, &per_sm);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     // the worklist length is only known on the device: one wave at most

@@ -113,6 +113,13 @@ struct TableArgs {
 };
 cudaError_t launch_tables(const TableArgs& a, cudaStream_t st);
 
+// Blocks of `func` (a kernel) resident per SM at `block` threads and `smem`
+// bytes of dynamic shared memory, after raising the kernel's dynamic
+// shared-memory limit to smem.  The answer is cached per (kernel, block,
+// smem, device): the two runtime queries cost microseconds of host time,
+// which a small pricing call would otherwise pay on every launch.
+cudaError_t resident_blocks(const void* func, int block, size_t smem, int* per_sm);
+
 struct PriceArgs {
     Layout lay;
     const unsigned char* img;

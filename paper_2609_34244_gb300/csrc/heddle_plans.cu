@@ -274,10 +274,8 @@ cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;
     if (a.vmax < 1 || a.vmax > kPlanMaxNode) return cudaErrorInvalidValue;
     const size_t smem = plan_smem(a.lay.NT, a.vmax);
-    cudaError_t e = cudaFuncSetAttribute(plan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, plan_kernel, kPlanBlock, smem);
+    const cudaError_t e = resident_blocks(reinterpret_cast<const void*>(&plan_kernel), kPlanBlock, smem, &per_sm);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     const int grid = (int)std::min<int64_t>((a.n + kPlanBlock - 1) / kPlanBlock, (int64_t)num_sms * per_sm);

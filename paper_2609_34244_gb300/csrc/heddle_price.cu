@@ -18,6 +18,7 @@
 // (heddle_wsearch.cu).
 
 #include <algorithm>
+#include <mutex>
 
 #include "heddle_tiled.cuh"
 
@@ -311,20 +312,66 @@ cudaError_t launch_screen(const PriceArgs& a, int num_sms, cudaStream_t st, cuda
     cudaError_t e = cudaMemsetAsync(a.wl_count, 0, sizeof(int32_t) * kWlMeta, st);
     if (e != cudaSuccess) return e;
     // one wave of resident CTAs, each looping over slices
-    static int screen_per_sm = 0;
-    if (screen_per_sm == 0) {
-        int v = 0;
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, screen_kernel<false>, kScreenBlock, 0);
-        if (e != cudaSuccess) return e;
-        screen_per_sm = v > 0 ? v : 1;
-    }
-    const int grid =
-        (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock, (int64_t)num_sms * screen_per_sm);
+    int screen_per_sm = 0;
+    e = resident_blocks(reinterpret_cast<const void*>(&screen_kernel<false>), kScreenBlock, 0, &screen_per_sm);
+    if (e != cudaSuccess) return e;
+    const int grid = (int)std::min<int64_t>((a.n + kScreenBlock - 1) / kScreenBlock,
+                                            (int64_t)num_sms * std::max(screen_per_sm, 1));
     if (!a.uniform && !a.split_mode) screen_kernel<true><<<grid, kScreenBlock, 0, st>>>(a);
     else screen_kernel<false><<<grid, kScreenBlock, 0, st>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     if (launches) launches[0] += 1;
     if (mid && (e = cudaEventRecord(mid, st)) != cudaSuccess) return e;
+    return cudaSuccess;
+}
+
+cudaError_t resident_blocks(const void* func, int block, size_t smem, int* per_sm) {
+    struct Limit {  // the largest dynamic shared memory a kernel was allowed so far
+        const void* func;
+        int device;
+        size_t smem;
+    };
+    struct Answer {
+        const void* func;
+        int device, block;
+        size_t smem;
+        int per_sm;
+    };
+    static std::mutex mu;
+    static Limit limits[32];
+    static Answer answers[128];
+    static int n_limits = 0, n_answers = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < n_answers; ++i) {
+        const Answer& x = answers[i];
+        if (x.func == func && x.device == dev && x.block == block && x.smem == smem) {
+            *per_sm = x.per_sm;
+            return cudaSuccess;
+        }
+    }
+    // raise (never lower) the kernel's limit: cached launches of larger
+    // sizes rely on it.  Past the tables' capacity nothing is cached and
+    // the limit is set on every call.
+    int li = -1;
+    for (int i = 0; i < n_limits; ++i)
+        if (limits[i].func == func && limits[i].device == dev) li = i;
+    if (li < 0 && n_limits < 32) {
+        li = n_limits++;
+        limits[li] = Limit{func, dev, 0};
+    }
+    if (li < 0 || limits[li].smem < smem) {
+        e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        if (li >= 0) limits[li].smem = smem;
+    }
+    int v = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, func, block, smem);
+    if (e != cudaSuccess) return e;
+    if (li >= 0 && n_answers < 128) answers[n_answers++] = Answer{func, dev, block, smem, v};
+    *per_sm = v;
     return cudaSuccess;
 }
 
@@ -335,7 +382,9 @@ cudaError_t launch_price(const PriceArgs& a, int num_sms, cudaStream_t st, cudaE
     if (launches) launches[1] += 1;
     if (a.split_mode) return launch_distribute(a, num_sms, st);
     if (a.uniform) return launch_eq_search(a, num_sms, st);
-    if ((e = launch_thread_search(a, num_sms, st)) != cudaSuccess) return e;
+    // a batch smaller than the thread search's threshold cannot fill its
+    // buckets up to it: that kernel would return at once, so it is not launched
+    if (a.n >= a.thread_min && (e = launch_thread_search(a, num_sms, st)) != cudaSuccess) return e;
     return launch_warp_search(a, num_sms, st, true);
 }
 

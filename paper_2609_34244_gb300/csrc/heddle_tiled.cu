@@ -521,10 +521,8 @@ cudaError_t launch_tiled_tables(const TiledTableArgs& a, cudaStream_t st) {
 
 cudaError_t launch_tiled_search(const PriceArgs& a, const TiledArgs& t, int num_sms, cudaStream_t st) {
     const size_t smem = ((t.tl.bytes + 127u) & ~127u) + sizeof(wp::WarpArea) * kTWarps;
-    cudaError_t e = cudaFuncSetAttribute(tiled_search_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, tiled_search_kernel, kTBlock, smem);
+    const cudaError_t e = resident_blocks(reinterpret_cast<const void*>(&tiled_search_kernel), kTBlock, smem, &per_sm);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     // the worklist length is only known on the device: one warp per entry,

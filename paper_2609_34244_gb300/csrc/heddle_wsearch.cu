@@ -347,10 +347,8 @@ __global__ void __launch_bounds__(kWBlock, 3) wsearch_kernel(PriceArgs a, int th
 template <bool kCount>
 cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st, bool listed) {
     const size_t smem = ((a.lay.bytes + 127u) & ~127u) + sizeof(WarpArea) * kWarps;
-    cudaError_t e = cudaFuncSetAttribute(wsearch_kernel<kCount>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, wsearch_kernel<kCount>, kWBlock, smem);
+    const cudaError_t e = resident_blocks(reinterpret_cast<const void*>(&wsearch_kernel<kCount>), kWBlock, smem, &per_sm);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
     // the worklist length is only known on the device: one warp per entry,
