@@ -350,6 +350,8 @@ def measure_config(h, name, peaks, sms, steps=20, cpu_seconds=3.0, main=None):
     tops = ops * 3 / (s_ms / 1e3) / 1e12 if s_ms > 0 else None
     threads = os.cpu_count() or 1
     rate, ncpu, used, dt = oracle_rate(w, cpu_seconds, threads)
+    # one host thread on the first 1e4 candidates (at most ~2 s of work)
+    rate1, n1, _, dt1 = oracle_rate(w, 2.0, 1, max_n=10_000)
     out = {"workload": name, "candidates": n, "search": SEARCH_NAMES.get(search, search),
            "value": n / (ms / 1e3), "unit": UNIT, "ms_per_step": ms, "per_candidate_ns": 1e6 * ms / n,
            "step_ms": {"median": float(np.median(per)), "best": float(np.min(per)), "runs": len(per)},
@@ -368,6 +370,8 @@ def measure_config(h, name, peaks, sms, steps=20, cpu_seconds=3.0, main=None):
            "device_errors": errors,
            "cpu_baseline": {"value": rate, "unit": UNIT, "cores": used, "kind": "oracle",
                             "sample": "first %d candidates (%.1f s, %d host threads)" % (ncpu, dt, used)},
+           "cpu_single_thread": {"value": rate1, "unit": UNIT, "cores": 1, "kind": "oracle",
+                                 "sample": "first %d candidates (%.2f s, one host thread)" % (n1, dt1)},
            "gpu_over_oracle": (n / (ms / 1e3)) / rate}
     return out
 
