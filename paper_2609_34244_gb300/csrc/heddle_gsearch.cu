@@ -332,9 +332,9 @@ __global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
             LB = max(LB, minq[gg * 4 + jj] + st.c);
             hiB = max(hiB, t.P[st.row + L] + st.c);
             memall &= t.smax + st.f * t.amax <= st.capk;
-            // the longest run [0, r) within memory (for the guess)
-            const int r0 = last_ok(0, L, (int)layers_est(t, st, gg * 4 + jj, kInf),
-                                   [&](int r) { return fits_mem(t, st, 0, r); });
+            // the run of layers memory admits, estimated from the average
+            // layer footprint (for the guess only)
+            const int r0 = min(L, (int)layers_est(t, st, gg * 4 + jj, kInf));
             w |= (uint32_t)r0 << kVShift;
             sw[s * kGBlock] = w;
         }
