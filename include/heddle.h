@@ -336,9 +336,11 @@ heddle_status heddle_price_mbs(heddle_ctx* ctx, const heddle_candidates* cands,
  * (§5.1: a node whose size equals the degree first, else GPUs from a larger
  * node).  The layer split, the bottleneck and OOM do not depend on the DP
  * degree, so each slot is first priced as standalone candidates with the
- * context's search mode, then re-evaluated with the plan's degree.  The
- * first template that is not OK (INVALID, NO_FIT on the GPUs left, OOM)
- * ends the plan; later templates are SKIPPED.  The plan's throughput is
+ * context's search mode, then re-evaluated with the plan's degree (slot t
+ * is priced only for the plans whose templates 0 .. t-1 are each OK on
+ * their own: no other plan reaches it).  The first template that is not OK
+ * (INVALID, NO_FIT on the GPUs left, OOM) ends the plan; later templates
+ * are SKIPPED.  The plan's throughput is
  * the sum over its placed templates of n * M * 1e9 / T base micro-batches
  * per second, each term rounded in IEEE double, in template order (so the
  * step rewards are those terms).

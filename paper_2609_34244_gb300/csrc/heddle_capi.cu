@@ -136,6 +136,8 @@ struct heddle_ctx {
     bool nodes_on_device = false;  // d_node_* hold the loaded cluster's nodes
     uint8_t* plan_bounds[HEDDLE_MAX_TEMPLATES] = {nullptr, nullptr, nullptr, nullptr};
     size_t plan_bounds_cap[HEDDLE_MAX_TEMPLATES] = {0, 0, 0, 0};
+    uint8_t* plan_skip = nullptr;  // the SKIPPED mask of the slot being priced
+    size_t plan_skip_cap = 0;
     // expert tiling: the experts' byte counts and the tiled image
     bool have_experts = false, tiled_ready = false;
     std::vector<int64_t> expert_state, expert_param;
@@ -550,6 +552,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_node_type);
     cudaFree(x->d_node_gpus);
     for (auto* b : x->plan_bounds) cudaFree(b);
+    cudaFree(x->plan_skip);
     for (auto& r : x->phase_recs)
         for (cudaEvent_t ev : r.e) x->ev_pool.push_back(ev);
     for (cudaEvent_t ev : x->ev_pool) cudaEventDestroy(ev);
@@ -884,6 +887,7 @@ struct PriceUnit {
     const heddle_ctx::Level* lvl;
     int shift;
     int64_t lo, nb;
+    const uint8_t* skip = nullptr;  // per candidate of c: price it SKIPPED (nullable)
 };
 
 // Independent chunk pricings (no top-k, no tiling output) as one pipeline:
@@ -915,6 +919,7 @@ heddle_status price_units(heddle_ctx* x, const PriceUnit* u, int nu, void* strea
         const bool t = tiled && !u[k].lvl;
         hd::PriceArgs a{};
         fill_price_args(x, u[k].c, u[k].lvl, u[k].shift, t, a);
+        a.skip = u[k].skip ? u[k].skip + u[k].lo : nullptr;
         if ((st = price_chunk(x, a, u[k].c, u[k].r, u[k].lo, u[k].nb, b, ws, nullptr, cs, t, nullptr)) != HEDDLE_OK)
             return st;
         if (pipe) CU(cudaEventRecord(x->ev_wl_free[b], ws));
@@ -1307,23 +1312,27 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     a.placed = pr->placed;
     a.thr = pr->thr;
     a.err = x->d_flags + 1;
-    // every slot priced as standalone candidates (the split needs bounds),
-    // the slots pipelined over the work streams
+    // the slots priced as standalone candidates, slot by slot: slot t only
+    // for the plans whose templates 0 .. t-1 are each OK alone (the mask
+    // reads slot t - 1's statuses), the chunks of a slot pipelined over the
+    // work streams.  The walk re-evaluates templates after the first from
+    // their splits, so those slots need bounds
     heddle_results rs[HEDDLE_MAX_TEMPLATES];
-    const heddle_candidates* cs_[HEDDLE_MAX_TEMPLATES];
+    CU(grow(&x->plan_skip, &x->plan_skip_cap, (size_t)pl->n));
     for (int t = 0; t < pl->slots; ++t) {
         rs[t] = pr->t[t];
-        if (!rs[t].bounds) {
+        if (!rs[t].bounds && t > 0) {
             CU(grow(&x->plan_bounds[t], &x->plan_bounds_cap[t], (size_t)(HEDDLE_MAX_STAGES + 1) * pl->n));
             rs[t].bounds = x->plan_bounds[t];
         }
-        cs_[t] = &pl->t[t];
-    }
-    {
+        CU(hd::launch_plan_mask(pl->n_templates, pl->slots, t, t > 0 ? rs[t - 1].status : nullptr, x->plan_skip,
+                                pl->n, x->num_sms, sm));
         std::vector<PriceUnit> units;
-        for (int t = 0; t < pl->slots; ++t)
-            for (int64_t lo = 0; lo < pl->n; lo += x->chunk)
-                units.push_back(PriceUnit{cs_[t], &rs[t], nullptr, 0, lo, std::min<int64_t>(x->chunk, pl->n - lo)});
+        for (int64_t lo = 0; lo < pl->n; lo += x->chunk) {
+            PriceUnit u{&pl->t[t], &rs[t], nullptr, 0, lo, std::min<int64_t>(x->chunk, pl->n - lo)};
+            u.skip = x->plan_skip;
+            units.push_back(u);
+        }
         if ((st = price_units(x, units.data(), (int)units.size(), stream)) != HEDDLE_OK) return st;
     }
     for (int t = 0; t < pl->slots; ++t) {

@@ -127,6 +127,7 @@ struct PriceArgs {
     const uint8_t* S;
     const uint16_t* M;
     const uint8_t* code;
+    const uint8_t* skip;  // nullable: nonzero prices the candidate SKIPPED (a template its plan does not reach)
     int64_t n;
     int64_t stride;
     int32_t s_max;
@@ -211,6 +212,9 @@ struct PlanArgs {
     uint32_t* err;
 };
 cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st);
+// The SKIPPED mask of slot t of a plan batch (see plan_mask_kernel).
+cudaError_t launch_plan_mask(const uint8_t* n_tmpl, int slots, int t, const uint8_t* prev_status, uint8_t* skip,
+                             int64_t n, int num_sms, cudaStream_t st);
 
 // The paper's own layer split over the worklist (comparison mode).
 cudaError_t launch_distribute(const PriceArgs& a, int num_sms, cudaStream_t st);

@@ -2,10 +2,14 @@
 // sequence of structural templates, each holding its own GPUs; the reward
 // of a step is the throughput the new template adds).
 //
-// The library first prices every template slot of every plan as a
-// standalone candidate (screen + search, unchanged): PartitionLayers and
-// the memory decision do not depend on the DP degree n, so the split, the
-// bottleneck and OOM carry over.  This kernel then walks each plan in
+// The library first prices the template slots as standalone candidates
+// (screen + search, unchanged): PartitionLayers and the memory decision do
+// not depend on the DP degree n, so the split, the bottleneck and OOM carry
+// over.  Slot t is priced only for the plans whose templates 0 .. t-1 are
+// each OK alone (a walk ends at its first template that is not OK, and a
+// template is OK in the walk only if it is OK alone); for the others the
+// screen writes SKIPPED.  The first template, on the whole free cluster,
+// keeps its standalone price.  This kernel then walks each plan in
 // order against the GPUs the earlier templates left: the template's n
 // comes from the free GPUs per node -- n = min over (type, size class e) of
 // floor(cap / demand), cap = sum over nodes of floor(free / 2^e) 2^e, exact
@@ -79,14 +83,15 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
         bool ended = false;
         int placed = 0;
         double thr = 0.0;
-        for (int t = 0; t < a.slots; ++t) {
+        // (the slots past the plan's templates were priced SKIPPED)
+        for (int t = 0; t < nt; ++t) {
             const PlanSlot& sl = a.slot[t];
             uint8_t st = HEDDLE_CAND_SKIPPED;
             int64_t T = -1, B = -1;
             int64_t n = 0;
             const int S = sl.S[c];
             const int M = sl.M[c];
-            if (!ended && t < nt) {
+            if (!ended) {
                 const uint8_t st0 = sl.status[c];
                 if (st0 == HEDDLE_CAND_INVALID) {
                     st = HEDDLE_CAND_INVALID;
@@ -131,6 +136,12 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
                         st = HEDDLE_CAND_NO_FIT;
                     } else if (st0 == HEDDLE_CAND_OOM) {
                         st = HEDDLE_CAND_OOM;
+                    } else if (t == 0) {
+                        // the whole cluster is free: n, T and B are the standalone ones
+                        T = sl.T[c];
+                        B = sl.B[c];
+                        st = HEDDLE_CAND_OK;
+                        if (n != (int64_t)sl.ndp[c]) atomicOr(a.err, kErrInternal);
                     } else {
                         // Evaluate with this n: T = (M-1) max t_s + sum t_s + max g_s
                         int64_t tmax = 0, tsum = 0;
@@ -171,6 +182,8 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
                         T = (int64_t)(M - 1) * tmax + tsum + gmax;
                         B = tmax;
                         st = HEDDLE_CAND_OK;
+                    }
+                    if (st == HEDDLE_CAND_OK) {
                         thr = __dadd_rn(thr, __ddiv_rn(__dmul_rn((double)(n * (int64_t)M), 1e9), (double)T));
                         placed = t + 1;
                         // place n copies of the groups, largest first
@@ -204,7 +217,7 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
                 }
                 if (st != HEDDLE_CAND_OK) ended = true;
             }
-            {
+            if (t > 0) {  // the first template keeps its standalone results
                 sl.T[c] = T;
                 sl.B[c] = B;
                 sl.ndp[c] = (uint16_t)(st == HEDDLE_CAND_OK || st == HEDDLE_CAND_OOM ? n : 0);
@@ -227,24 +240,22 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
             const int64_t c = c0 + threadIdx.x;
             bool walks = false;
             if (c < a.n) {
+                // a plan walks from its second template on; the others keep
+                // their slots as priced (templates past the first OK-alone
+                // prefix were priced SKIPPED) and take the first template's
+                // throughput if it is OK
                 const int nt = min((int)a.n_tmpl[c], a.slots);
-                walks = nt >= 1 && a.slot[0].status[c] == HEDDLE_CAND_OK;
+                const bool ok0 = nt >= 1 && a.slot[0].status[c] == HEDDLE_CAND_OK;
+                walks = ok0 && nt >= 2;
                 if (!walks) {
-                    // the first template (if any) keeps its standalone
-                    // price; a walking plan's slots stay untouched here,
-                    // since its walk reads their standalone prices
-                    // (so these stores leave partial sectors: measured
-                    // 710 MB of DRAM traffic per 1e6 plans, 480 us)
-                    for (int t = nt >= 1 ? 1 : 0; t < a.slots; ++t) {
-                        const PlanSlot& sl = a.slot[t];
-                        sl.T[c] = -1;
-                        sl.B[c] = -1;
-                        sl.ndp[c] = 0;
-                        sl.status[c] = HEDDLE_CAND_SKIPPED;
-                        for (int s2 = 0; s2 <= kMaxStages; ++s2) sl.bounds[(int64_t)s2 * sl.bstride + c] = 0;
+                    double thr = 0.0;
+                    if (ok0) {
+                        const PlanSlot& s0 = a.slot[0];
+                        const int64_t n0 = s0.ndp[c];
+                        thr = __ddiv_rn(__dmul_rn((double)(n0 * (int64_t)s0.M[c]), 1e9), (double)s0.T[c]);
                     }
-                    a.placed[c] = 0;
-                    a.thr[c] = 0.0;
+                    a.placed[c] = ok0 ? 1 : 0;
+                    a.thr[c] = thr;
                 }
             }
             const unsigned wm = __ballot_sync(0xffffffffu, walks);
@@ -268,7 +279,29 @@ __global__ void __launch_bounds__(kPlanBlock, 8) plan_kernel(PlanArgs a) {
     }
 }
 
+// skip[i] = plan i does not reach template t on its templates' own prices:
+// it has at most t templates, or template t - 1 is not OK alone (a
+// template priced SKIPPED is not OK either, so the mask of t covers every
+// earlier template).
+__global__ void plan_mask_kernel(const uint8_t* n_tmpl, int slots, int t, const uint8_t* prev_status,
+                                 uint8_t* skip, int64_t n) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        const int nt = min((int)n_tmpl[i], slots);
+        const bool reach = nt > t && (t == 0 || prev_status[i] == HEDDLE_CAND_OK);
+        skip[i] = reach ? 0 : 1;
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_plan_mask(const uint8_t* n_tmpl, int slots, int t, const uint8_t* prev_status, uint8_t* skip,
+                             int64_t n, int num_sms, cudaStream_t st) {
+    if (n <= 0) return cudaSuccess;
+    const int grid = (int)std::min<int64_t>((n + 255) / 256, (int64_t)num_sms * 8);
+    plan_mask_kernel<<<grid, 256, 0, st>>>(n_tmpl, slots, t, prev_status, skip, n);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_plans(const PlanArgs& a, int num_sms, cudaStream_t st) {
     if (a.n <= 0) return cudaSuccess;

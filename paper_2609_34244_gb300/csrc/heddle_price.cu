@@ -140,7 +140,11 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
             const int M = Mraw >> a.mbs_shift;
             const bool whole = (Mraw & ((1 << a.mbs_shift) - 1)) == 0;
             key = (S >= 1 && S <= s_lim && M >= 1 && whole) ? S : 0;
-            sS[threadIdx.x] = (uint8_t)key;
+            // a plan's template that the plan cannot reach is priced SKIPPED
+            // (bit 7 of its S byte; it sorts with the invalid ones)
+            const bool skipped = a.skip && a.skip[c0 + threadIdx.x];
+            if (skipped) key = 0;
+            sS[threadIdx.x] = (uint8_t)(key | (skipped ? 0x80 : 0));
             sM[threadIdx.x] = (uint16_t)M;
         }
         if (threadIdx.x < kMaxStages + 3) bins[threadIdx.x] = 0;
@@ -192,8 +196,9 @@ __global__ void __launch_bounds__(kScreenBlock) screen_kernel(PriceArgs a) {
         uint32_t fits1 = 1;  // every stage could hold any single layer (general search)
         int64_t n = 0;
         if (live) {
-            S = sS[ci];
+            S = sS[ci] & 0x3f;
             M = sM[ci];
+            if (sS[ci] & 0x80) status = HEDDLE_CAND_SKIPPED;
             if (S > 0) {
 #pragma unroll
                 for (int g = 0; g < 8; ++g) mydem[g * kScreenBlock] = 0;
