@@ -136,8 +136,8 @@ struct heddle_ctx {
     bool nodes_on_device = false;  // d_node_* hold the loaded cluster's nodes
     uint8_t* plan_bounds[HEDDLE_MAX_TEMPLATES] = {nullptr, nullptr, nullptr, nullptr};
     size_t plan_bounds_cap[HEDDLE_MAX_TEMPLATES] = {0, 0, 0, 0};
-    uint8_t* plan_skip = nullptr;  // the SKIPPED mask of the slot being priced
-    size_t plan_skip_cap = 0;
+    uint8_t* skip_mask = nullptr;  // the plan slot being priced: candidates priced SKIPPED
+    size_t skip_mask_cap = 0;
     // expert tiling: the experts' byte counts and the tiled image
     bool have_experts = false, tiled_ready = false;
     std::vector<int64_t> expert_state, expert_param;
@@ -552,7 +552,7 @@ void heddle_destroy(heddle_ctx* x) {
     cudaFree(x->d_node_type);
     cudaFree(x->d_node_gpus);
     for (auto* b : x->plan_bounds) cudaFree(b);
-    cudaFree(x->plan_skip);
+    cudaFree(x->skip_mask);
     for (auto& r : x->phase_recs)
         for (cudaEvent_t ev : r.e) x->ev_pool.push_back(ev);
     for (cudaEvent_t ev : x->ev_pool) cudaEventDestroy(ev);
@@ -1318,19 +1318,19 @@ heddle_status heddle_price_plans(heddle_ctx* x, const heddle_plans* pl, const he
     // work streams.  The walk re-evaluates templates after the first from
     // their splits, so those slots need bounds
     heddle_results rs[HEDDLE_MAX_TEMPLATES];
-    CU(grow(&x->plan_skip, &x->plan_skip_cap, (size_t)pl->n));
+    CU(grow(&x->skip_mask, &x->skip_mask_cap, (size_t)pl->n));
     for (int t = 0; t < pl->slots; ++t) {
         rs[t] = pr->t[t];
         if (!rs[t].bounds && t > 0) {
             CU(grow(&x->plan_bounds[t], &x->plan_bounds_cap[t], (size_t)(HEDDLE_MAX_STAGES + 1) * pl->n));
             rs[t].bounds = x->plan_bounds[t];
         }
-        CU(hd::launch_plan_mask(pl->n_templates, pl->slots, t, t > 0 ? rs[t - 1].status : nullptr, x->plan_skip,
+        CU(hd::launch_plan_mask(pl->n_templates, pl->slots, t, t > 0 ? rs[t - 1].status : nullptr, x->skip_mask,
                                 pl->n, x->num_sms, sm));
         std::vector<PriceUnit> units;
         for (int64_t lo = 0; lo < pl->n; lo += x->chunk) {
             PriceUnit u{&pl->t[t], &rs[t], nullptr, 0, lo, std::min<int64_t>(x->chunk, pl->n - lo)};
-            u.skip = x->plan_skip;
+            u.skip = x->skip_mask;
             units.push_back(u);
         }
         if ((st = price_units(x, units.data(), (int)units.size(), stream)) != HEDDLE_OK) return st;

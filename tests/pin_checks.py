@@ -372,6 +372,16 @@ def check_mbs_properties(O, seed=11):
             assert (one[k] == plain[k]).all(), (name, k)
         r = O.price_mbs(w.cluster, w.model, w.cands, 3, prof)
         assert not ((plain["status"] == O.OOM) & (r["status"] == O.OK)).any(), name
+        # each larger size on its own: a candidate that is not OK at the
+        # base size is OK at none (the library prices only the base size's
+        # OK candidates at the larger sizes)
+        M0 = np.asarray(w.cands["M"], np.int64)
+        for i in (1, 2):
+            ci = dict(w.cands)
+            ci["M"] = np.where(M0 % (1 << i) == 0, M0 >> i, 0).astype(np.uint16)
+            li = O.Oracle(w.cluster, O.level_model(w.model, i, prof[i])).price(ci)
+            assert not ((plain["status"] != O.OK) & (li["status"] == O.OK)).any(), (name, i)
+            assert (li["status"][plain["status"] == O.OOM] != O.OK).all(), (name, i)
         assert ((r["status"] == O.OK) | (r["status"] == plain["status"])).all(), name
         M = np.asarray(w.cands["M"], np.int64)
         assert ((M % (1 << r["mbs"].astype(np.int64))) == 0).all(), name
