@@ -200,7 +200,7 @@ __device__ __forceinline__ void defer(const PriceArgs& a, int64_t p) {
 // Below a.thread_min bucketed entries the kernel returns at once and the
 // warp kernel prices the whole worklist.
 template <bool kCount>
-__global__ void __launch_bounds__(kGBlock) gsearch_kernel(PriceArgs a) {
+__global__ void __launch_bounds__(kGBlock, 4) gsearch_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ uint64_t bar;
     __shared__ int64_t qmax[4 * kMaxTypes], single[2];
