@@ -198,7 +198,9 @@ __device__ __forceinline__ void defer(const PriceArgs& a, int64_t p) {
 }
 
 // Below a.thread_min bucketed entries the kernel returns at once and the
-// warp kernel prices the whole worklist.
+// warp kernel prices the whole worklist.  Four CTAs per SM (the table
+// image and the stage words fill shared memory there), so up to 128
+// registers a thread.
 template <bool kCount>
 __global__ void __launch_bounds__(kGBlock, 4) gsearch_kernel(PriceArgs a) {
     extern __shared__ __align__(128) unsigned char smem[];
