@@ -30,6 +30,15 @@ def main():
                 G.assert_same(got, ref, what="%s mode %d fused %s" % (name, mode, fused))
                 exp = O.topk(ref, w.cands["M"], 16)
                 assert got["topk"]["idx"].tolist() == exp["idx"].tolist(), (name, mode)
+    # plans: the per-slot SKIPPED mask and the walk
+    import test_gpu_plans as TP
+    for name in ("dense32", "stress128"):
+        w = W.make_workload(name, seed=4, n=3001)
+        plans = W.make_plans(w, 3001, 4, seed=4)
+        ref = O.Oracle(w.cluster, w.model).price_plans(plans)
+        got = TP.price_plans_gpu(h, w.cluster, w.model, plans, bounds=True)
+        assert got["errors"] == 0, "%s plans: device flags %#x" % (name, got["errors"])
+        TP._same(got, ref, "%s plans" % name)
     w = W.make_workload("moe16", seed=2, n=20011)
     ref = O.Oracle(w.cluster, w.model).set_experts(w.model["expert_state_bytes"], w.model["expert_param_bytes"]) \
         .price(w.cands, threads=8)

@@ -86,6 +86,26 @@ def test_plans_other_split_modes(h, W, oracle_mod, search):
     _same(got, ref, "dense32 search %d" % search)
 
 
+def test_plans_bounds(h, W, oracle_mod):
+    """With bound planes requested: an OK template keeps the split of its
+    standalone price (the oracle's, slot by slot), every other template's
+    planes are zero (slots that no plan reaches included)."""
+    w = W.make_workload("dense32", seed=3, n=3001)
+    plans = W.make_plans(w, 3001, 3, seed=3)
+    ref = oracle_mod.Oracle(w.cluster, w.model).price_plans(plans)
+    got = price_plans_gpu(h, w.cluster, w.model, plans, bounds=True)
+    _same(got, ref, "dense32 plans with bounds")
+    orc = oracle_mod.Oracle(w.cluster, w.model)
+    for t in range(3):
+        alone = orc.price({"S": np.ascontiguousarray(plans["S"][t]), "M": np.ascontiguousarray(plans["M"][t]),
+                           "code": np.ascontiguousarray(plans["code"][t])}, bounds=True)
+        b = got["bounds"][t]
+        ok = got["status"][t] == 0
+        assert ok.any() and (~ok).any(), t
+        assert (b[:, ok] == alone["bounds"][:, ok]).all(), t
+        assert (b[:, ~ok] == 0).all(), t
+
+
 def test_plans_hand_cases(h, W):
     path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "hand_plans.json")
     d = json.load(open(path))
