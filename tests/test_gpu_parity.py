@@ -28,7 +28,7 @@ def W():
 
 # sizes span many CTAs (128 threads each) and end on a ragged tail
 SMALL = [("tiny", None), ("tiny_ext", None), ("dense32", 6007), ("dense80", 1531),
-         ("moe48", 6011), ("stress128", 613)]
+         ("moe48", 6011), ("moe16", 4001), ("stress128", 613)]
 
 
 # the equal-layer search runs on models whose layers all cost the same
@@ -57,6 +57,21 @@ def test_parity_small(h, W, oracle_mod, name, n, seed, route):
     assert got["topk"]["idx"].tolist() == tk["idx"].tolist()
     assert got["topk"]["T"].tolist() == tk["T"].tolist()
     assert got["topk"]["nM"].tolist() == tk["nM"].tolist()
+
+
+def test_thread_search_defers_to_warp_search(h, W, oracle_mod):
+    """moe16 through the thread-per-entry search: entries whose bracket
+    falls below the single-fit threshold are handed to the warp search
+    (counted twice: the interval-test counters see both kernels), and the
+    results still equal the oracle's."""
+    w = W.make_workload("moe16", seed=0, n=4001)
+    ref = oracle_mod.Oracle(w.cluster, w.model).price(w.cands, threads=8)
+    both = G.price_gpu(h, w.cluster, w.model, w.cands, search=1, thread_min=0, count=True)
+    warp = G.price_gpu(h, w.cluster, w.model, w.cands, search=1, thread_min=2**31 - 1, count=True)
+    for got in (both, warp):
+        assert got["errors"] == 0
+        G.assert_same(got, ref, what="moe16")
+    assert both["counters"]["priced"] > warp["counters"]["priced"], "no entry was handed on"
 
 
 @pytest.mark.parametrize("name", ["tiny", "dense32", "dense80", "moe48", "stress128"])
