@@ -24,7 +24,10 @@
 // largest accepted or smallest rejected stage time (every bound in [hi, B]
 // or [B, lo) decides alike), galloping, then bisecting.  An entry that meets
 // a bound that is not single-fit is left to the warp kernel, which runs the
-// general set-based probe; it gets the list of those entries.
+// general set-based probe; it gets the list of those entries.  The kernel
+// runs only when the depth buckets hold at least PriceArgs::thread_min
+// entries (a few entries would leave it as long as its longest serial
+// chain); each warp takes 32 entries at a time, deepest first.
 
 #include <algorithm>
 

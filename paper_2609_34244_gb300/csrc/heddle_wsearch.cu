@@ -11,13 +11,17 @@
 // (1, 2, 4, ... away) until both sides are known, then bisects.  The sets
 // of the probe at B* give the canonical split; a feasible probe that closes
 // the bracket already holds them (every bound in [hi, B] takes the same
-// decisions), so only a bracket closed from below costs a final probe.  The probe (heddle_wprobe.cuh) checks 32
-// positions per round with the interval test of this file: stage time
+// decisions), so only a bracket closed from below costs a final probe.
+// The probe (heddle_wprobe.cuh) checks 32 positions per round with the
+// interval test of this file: stage time
 // P[j] - P[i] + c and memory against k times the GPU memory.  Evaluate runs
 // one lane per stage: the stage times' maximum and sum, the stage with the
 // largest G / (k bw) by exact cross-multiplication, and one 128/64-bit
 // ceiling division for the gradient term.  The table image is staged into
-// shared memory with bulk asynchronous copies.
+// shared memory with bulk asynchronous copies.  The kernel prices the
+// entries the thread-per-entry search (heddle_gsearch.cu) left, or every
+// worklist entry when that search had too few to run; each warp takes its
+// own first entry, then the next untaken one from a counter.
 
 #include <climits>
 
