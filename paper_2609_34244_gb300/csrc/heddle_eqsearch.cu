@@ -34,7 +34,8 @@
 //
 // Scheduling: the screen files every entry in a bucket per depth S; warp w
 // takes entries [32 w, 32 w + 32) of the buckets read in order of
-// decreasing S, so its lanes run stage loops of equal length.  Warps work
+// decreasing S, so its lanes run stage loops of equal length, and then the
+// next 32 untaken entries from a counter whenever it is free.  Warps work
 // independently (no CTA barrier after the tables are staged): every thread
 // packs its candidate's stages once into 32-bit words (cost index | P2P
 // index | memory run | cap) held in shared memory interleaved by thread,
@@ -465,11 +466,16 @@ __global__ void __launch_bounds__(kEqBlock, 1024 / kEqBlock) eq_search_kernel(Pr
     // the entries filed in the depth buckets (every worklist entry here)
     const int64_t entries = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const int64_t count = min((int64_t)end_of[1], entries);
-    const int64_t stride = (int64_t)gridDim.x * kEqBlock;
     // warp w of CTA b takes entries [32 (4 b + w), +32) of the order by
-    // decreasing S, so its lanes have nearly equal S; warps never wait on
-    // one another
-    for (int64_t base = ((int64_t)blockIdx.x * kEqWarps + warp) * 32; base < count; base += stride) {
+    // decreasing S, so its lanes have nearly equal S, then the next 32
+    // untaken ones whenever it is free; warps never wait on one another
+    const int64_t first = (int64_t)gridDim.x * kEqBlock;
+    auto take = [&]() {
+        int b = 0;
+        if (lane == 0) b = atomicAdd(a.wl_count + kWlTakeThread, 32);
+        return first + __shfl_sync(0xffffffffu, b, 0);
+    };
+    for (int64_t base = ((int64_t)blockIdx.x * kEqWarps + warp) * 32; base < count; base = take()) {
         const int64_t g = base + lane;
         bool have = g < count;
         int64_t p = 0;
@@ -625,9 +631,12 @@ cudaError_t launch(const PriceArgs& a, int num_sms, cudaStream_t st) {
     const cudaError_t e = resident_blocks(reinterpret_cast<const void*>(&eq_search_kernel<kCount>), kEqBlock, smem, &per_sm);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorInvalidConfiguration;
-    // the worklist length is only known on the device: size for the batch
+    // the worklist length is only known on the device: size for the batch,
+    // at most seven of the eight CTAs that fit an SM -- warps fetch further
+    // entries when free, and the free slot lets the next chunk's screen
+    // start beside this search's last warps
     const int64_t need = (a.n + kEqBlock - 1) / kEqBlock;
-    const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * per_sm);
+    const int grid = (int)std::min<int64_t>(need, (int64_t)num_sms * std::min(per_sm, 7));
     eq_search_kernel<kCount><<<grid, kEqBlock, smem, st>>>(a);
     return cudaGetLastError();
 }
