@@ -248,7 +248,10 @@ struct TiledCheck {
         r.f = __shfl_sync(wp::kFull, mine.f, s);
         return r;
     }
-    __device__ __forceinline__ int eval(const TLane& st, int i, int e, int64_t B, int64_t* cost) const {
+    // not inlined: the probe calls it from several places, and inlined
+    // copies of its loop over the tilings made the kernel wait on
+    // instruction fetch
+    __device__ __noinline__ int eval(const TLane& st, int i, int e, int64_t B, int64_t* cost) const {
         const int base = tile_base(st.j), cnt = (st.j + 1) * (st.j + 2) / 2;
         int64_t best = kInf;
         for (int o = 0; o < cnt; ++o) {
