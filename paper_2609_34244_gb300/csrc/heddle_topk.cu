@@ -233,6 +233,59 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     const int64_t n = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const bool few = n <= kFewEntries;
     if (few && blockIdx.x != 0) return;
+    if (n <= 32) {
+        // at most one entry per lane: warp 0 ranks them against each other
+        // (the order is strict, so the ranks are distinct), places them,
+        // and merges them with the state -- no CTA barrier
+        if (warp != 0) return;
+        TopkEntry e;
+        e.idx = 0;
+        e.T = 0;
+        e.nM = 0;
+        e.pad = 0;
+        bool valid = lane < n && fetch<true>(a, lane, e);
+        if (valid && full) valid = better(e, bar);
+        int rank = 0;
+        for (int j = 0; j < 32; ++j) {
+            TopkEntry o;
+            o.idx = __shfl_sync(0xffffffffu, e.idx, j);
+            o.T = __shfl_sync(0xffffffffu, e.T, j);
+            o.nM = __shfl_sync(0xffffffffu, e.nM, j);
+            o.pad = 0;
+            const bool ov = __shfl_sync(0xffffffffu, valid, j);
+            rank += (valid && ov && better(o, e)) ? 1 : 0;
+        }
+        const int nv = min(__popc(__ballot_sync(0xffffffffu, valid)), k);
+        TopkEntry* mine = lists + kMaxTopK;
+        if (valid && rank < k) mine[rank] = e;
+        const int c = min(max(a.state->count, 0), k);
+        for (int i = lane; i < c; i += 32) {
+            TopkEntry x;
+            x.idx = a.state->idx[i];
+            x.T = a.state->T[i];
+            x.nM = a.state->nM[i];
+            x.pad = 0;
+            lists[i] = x;
+        }
+        __syncwarp();
+        const int total = warp_merge(lists, c, mine, nv, tmp, k);
+        for (int i = lane; i < kMaxTopK; i += 32) {
+            const bool live = i < total;
+            a.state->idx[i] = live ? tmp[i].idx : -1;
+            a.state->T[i] = live ? tmp[i].T : -1;
+            a.state->nM[i] = live ? tmp[i].nM : 0;
+        }
+        if (lane == 0) {
+            a.state->count = total;
+            if (a.thr && total >= k) {
+                // the new k-th key, rounded and lowered by 2^-16 (see TopkArgs::thr)
+                const TopkEntry x = tmp[k - 1];
+                const float r = (float)x.nM / (float)x.T * (1.0f - 1.0f / 65536.0f);
+                atomicMax(a.thr, __float_as_uint(r));
+            }
+        }
+        return;
+    }
     const int64_t step = few ? (int64_t)W * 32 : (int64_t)gridDim.x * W * 32;
     const int64_t start = few ? (int64_t)warp * 32 : ((int64_t)blockIdx.x * W + warp) * 32;
     constexpr int U = 4;
