@@ -33,7 +33,7 @@ METRIC = "candidate plans priced/sec on 1 GB300 (and % of ALU/HBM roofline)"
 UNIT = "candidates/s"
 WORKLOAD = "stress128"
 WORKLOAD_DESC = ("stress128: 128-layer dense model (h 12288, seq 4096, bf16), 1024 GPUs of 8 types in "
-                 "nodes of 2/4/8, 1e7 candidates per step in one call, priced in 10 chunks of 1e6 pipelined over two "
+                 "nodes of 2/4/8, 1e7 candidates per step in one call, priced in 10 chunks of 1e6 pipelined over four "
                  "work streams, S<=32, "
                  "TP in {1,2,4,8}, M=256, global top-16")
 # Algorithmic integer work per counted unit, in 32-bit lane operations.
@@ -442,7 +442,7 @@ def main():
     def step():
         """One pass of the hot path: one heddle_price_topk call over all n
         candidates -- the library prices them in chunks of `batch` (screen,
-        search) pipelined over two work streams and merges each chunk into
+        search) pipelined over four work streams and merges each chunk into
         the running top-16 in order."""
         h.heddle_topk_reset(ctx, state, 16, stream)
         h.heddle_price_topk(ctx, call_all, res_all, state, stream)
@@ -824,7 +824,7 @@ def main():
                               "achieved": achieved_tops, "frac": achieved_tops / peak_tops,
                               "phases_us_per_batch": {k: 1e3 * v[0] / chunks_timed for k, v in phases.items()},
                               "phase_share": {k: v[0] / total_phase_ms for k, v in phases.items()},
-                              "how": "inside the timed steps (every 8th step): chunks pipelined over two work "
+                              "how": "inside the timed steps (every 8th step): chunks pipelined over four work "
                                      "streams, so each launch shares the GPU with the neighbouring chunks' "
                                      "kernels"},
                      "step": step_roofline,

@@ -187,12 +187,12 @@ typedef struct {
  * candidates needing the threshold search into a worklist owned by the
  * context, then the search over that worklist.  A batch of one chunk runs
  * on `stream` and allocates nothing.  A batch of several chunks
- * rotates three worklist sets over two context-owned work streams, so
- * chunk i + 1 is screened and searched while chunk i finishes: each work
+ * rotates five worklist sets over four context-owned work streams, so
+ * the next chunks are screened and searched while chunk i finishes: each work
  * stream first waits for the work queued on `stream` before the call, any
  * top-k merge runs on `stream` in chunk order, and `stream` waits for every
  * chunk before work queued after the call runs (stream-ordered as a single
- * launch would be).  The first such call allocates the other two sets
+ * launch would be).  The first such call allocates the other four sets
  * (~210 MB each) and the streams (E_NOMEM if that fails).  Calls on one context
  * must not overlap on the GPU (use one stream per context, or one context
  * per stream).
@@ -425,7 +425,7 @@ heddle_status heddle_price_tiled(heddle_ctx* ctx, const heddle_candidates* cands
  * `results` (host arrays of cands->n entries; bounds uses plane stride
  * cands->n).  Batch k is copied in on a copy stream into staging set k % 3
  * (free once batch k - 3 is copied out), screened and searched
- * on work stream k % 2 with worklist set k % 3, merged on `stream` in batch
+ * on work stream k % 2 with worklist set k % 5, merged on `stream` in batch
  * order and copied out on a second copy stream, so copies, the search of
  * one batch and the screen of the next overlap.  *state is host memory,
  * read on entry (k, and any entries already held) and written on return.
