@@ -301,5 +301,9 @@ def test_call_errors(h, W):
         with pytest.raises(h.HeddleError) as e:
             h.heddle_topk_reset(ctx, h.alloc_topk_state(), 65)
         assert e.value.status == 3
+        # the routing setting: a NULL context is refused; any value is taken
+        assert h.load_library().heddle_set_thread_search_min(None, 0) == 1
+        for v in (-5, 0, 2**31 - 1):
+            h.heddle_set_thread_search_min(ctx, v)
     finally:
         h.heddle_destroy(ctx)
