@@ -61,6 +61,29 @@ __device__ inline void warp_offer(TopkEntry* list, int& cnt, int k, bool valid, 
     }
 }
 
+// One round of a warp's running top-32 of float keys: lane l holds the
+// (l+1)-th largest key so far (run); the round's 32 keys (one per lane) are
+// sorted by a bitonic network, reversed against run (the larger of each
+// pair is a bitonic sequence holding the 32 largest of both) and merged.
+__device__ __forceinline__ float warp_keep_top32(float run, float key) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const float o = __shfl_xor_sync(0xffffffffu, key, stride);
+            const bool desc = (lane & size) == 0 || size == 32;
+            key = (((lane & stride) == 0) == desc) ? fmaxf(key, o) : fminf(key, o);
+        }
+    float c = fmaxf(run, __shfl_sync(0xffffffffu, key, 31 - lane));
+#pragma unroll
+    for (int stride = 16; stride > 0; stride >>= 1) {
+        const float o = __shfl_xor_sync(0xffffffffu, c, stride);
+        c = (lane & stride) == 0 ? fmaxf(c, o) : fminf(c, o);
+    }
+    return c;
+}
+
 // Merge the sorted lists of the CTA's warps (lists[w], counts[w]) into
 // lists[0] with warp 0, then write it and its length to out / out_count.
 // Every thread of the CTA must call it (it synchronises the CTA).

@@ -7,7 +7,12 @@
 // the incoming state's k-th is dropped at once, the others are offered to
 // the warp's sorted list in shared memory (inserted only if they beat its
 // current k-th), the CTA merges its warps' lists (a tree of parallel
-// two-list merges) and writes one list to scratch.  Then the per-CTA lists are folded into the state by merge
+// two-list merges) and writes one list to scratch.  While the state is not
+// yet full, a first pass over the same slice finds each warp's k-th largest
+// float key (a running top-32 per warp, merged by a bitonic network); the
+// CTA's largest, lowered by a margin, drops the entries that k others beat
+// before any is offered, so a warp inserts a handful of entries instead of
+// every new best of an unsorted slice.  Then the per-CTA lists are folded into the state by merge
 // levels of 16 lists per CTA: one level for up to 16 lists, else two.  No
 // CTA waits on another.
 
@@ -67,6 +72,29 @@ __global__ void __launch_bounds__(kBlock) topk_block_kernel(TopkArgs a) {
     // four rounds of 32 entries per warp are loaded before any is offered
     constexpr int U = 4;
     const int64_t step = nwarps * 32;
+    // first pass (k <= 32, while the state is not full): the k-th largest
+    // float key n*M / T among the entries each warp visits; k of them reach
+    // it, so the CTA's largest such key, lowered by 2^-16 (more than the
+    // rounding of two keys computed the same way), is a floor below which
+    // no entry can enter the top-k
+    __shared__ unsigned floor_bits;
+    float floor_cta = 0.0f;
+    if (k <= 32 && !full) {
+        if (threadIdx.x == 0) floor_bits = 0;
+        __syncthreads();
+        float run = -1.0f;
+        for (int64_t base = gw * 32; base < n; base += step) {
+            const int64_t i = base + lane;
+            float key = -1.0f;
+            TopkEntry e;
+            if (i < n && fetch<kWorklist>(a, i, e) && e.T > 0) key = (float)e.nM / (float)e.T;
+            run = warp_keep_top32(run, key);
+        }
+        const float kth = __shfl_sync(0xffffffffu, run, k - 1);
+        if (lane == 0 && kth > 0.0f) atomicMax(&floor_bits, __float_as_uint(kth * (1.0f - 1.0f / 65536.0f)));
+        __syncthreads();
+        floor_cta = __uint_as_float(floor_bits);
+    }
     for (int64_t base = gw * 32; base < n; base += step * U) {
         TopkEntry e[U];
         bool valid[U];
@@ -81,7 +109,10 @@ __global__ void __launch_bounds__(kBlock) topk_block_kernel(TopkArgs a) {
             if (i < n) valid[u] = fetch<kWorklist>(a, i, e[u]);
         }
 #pragma unroll
-        for (int u = 0; u < U; ++u) warp_offer(list, cnt, k, valid[u] && (!full || better(e[u], bar)), e[u]);
+        for (int u = 0; u < U; ++u) {
+            const bool above = valid[u] && (float)e[u].nM / (float)e[u].T >= floor_cta;
+            warp_offer(list, cnt, k, above && (!full || better(e[u], bar)), e[u]);
+        }
     }
     if (lane == 0) counts[warp] = cnt;
     cta_tree_merge(lists, counts, tmp, tmp_counts, W, k);
@@ -220,6 +251,7 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     __shared__ TopkEntry tmp[((kFan + 2) / 2) * kMaxTopK];
     __shared__ int counts[kFan + 1], tmp_counts[(kFan + 2) / 2];
     __shared__ int last_flag;
+    __shared__ unsigned floor_bits;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const bool full = a.state->count >= k;
     TopkEntry bar;
@@ -227,6 +259,11 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     bar.T = full ? a.state->T[k - 1] : 0;
     bar.nM = full ? a.state->nM[k - 1] : 0;
     bar.pad = 0;
+    // the running threshold of the call (a float lower bound, lowered by a
+    // margin that covers the rounding, on the k-th key of the candidates
+    // priced so far): an entry whose key n*M / T, computed the same way,
+    // falls below it has k entries of the call that rank before it
+    const float floor_key = a.thr ? __uint_as_float(__ldcg(a.thr)) : 0.0f;
     // ---- this CTA's share of the worklist (all of it when it is short)
     int cnt = 0;
     TopkEntry* list = lists + warp * kMaxTopK;
@@ -288,6 +325,33 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     }
     const int64_t step = few ? (int64_t)W * 32 : (int64_t)gridDim.x * W * 32;
     const int64_t start = few ? (int64_t)warp * 32 : ((int64_t)blockIdx.x * W + warp) * 32;
+    // ---- first pass (k <= 32, while the state is not full: once it is,
+    //      its k-th entry stops almost every entry): the k-th largest float
+    //      key among the entries each warp visits; k of them reach it, so
+    //      the CTA's largest such key, lowered by the margin, is a floor for
+    //      every entry that can enter the top-k, and it raises the call's
+    //      threshold for the other CTAs
+    float floor_cta = floor_key;
+    if (k <= 32 && !full) {
+        if (threadIdx.x == 0) floor_bits = 0;
+        __syncthreads();
+        float run = -1.0f;
+        for (int64_t base = start; base < n; base += step) {
+            const int64_t i = base + lane;
+            float key = -1.0f;
+            if (i < n) {
+                const int64_t T = a.wl_T[i];
+                if (T > 0) key = (float)a.wl_nM[i] / (float)T;
+            }
+            run = warp_keep_top32(run, key);
+        }
+        const float kth = __shfl_sync(0xffffffffu, run, k - 1);
+        if (lane == 0 && kth > 0.0f) atomicMax(&floor_bits, __float_as_uint(kth * (1.0f - 1.0f / 65536.0f)));
+        __syncthreads();
+        floor_cta = fmaxf(floor_cta, __uint_as_float(floor_bits));
+        if (threadIdx.x == 0 && a.thr && floor_cta > floor_key) atomicMax(a.thr, __float_as_uint(floor_cta));
+        if (a.thr) floor_cta = fmaxf(floor_cta, __uint_as_float(__ldcg(a.thr)));
+    }
     constexpr int U = 4;
     for (int64_t base = start; base < n; base += step * U) {
         TopkEntry e[U];
@@ -303,7 +367,10 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
             if (i < n) valid[u] = fetch<true>(a, i, e[u]);
         }
 #pragma unroll
-        for (int u = 0; u < U; ++u) warp_offer(list, cnt, k, valid[u] && (!full || better(e[u], bar)), e[u]);
+        for (int u = 0; u < U; ++u) {
+            const bool above = valid[u] && (float)e[u].nM / (float)e[u].T >= floor_cta;
+            warp_offer(list, cnt, k, above && (!full || better(e[u], bar)), e[u]);
+        }
     }
     if (lane == 0) counts[warp] = cnt;
     cta_tree_merge(lists, counts, tmp, tmp_counts, W, k);
