@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kBlock) topk_block_kernel(TopkArgs a) {
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const bool above = valid[u] && (float)e[u].nM / (float)e[u].T >= floor_cta;
+            const bool above = valid[u] && (floor_cta <= 0.0f || (float)e[u].nM / (float)e[u].T >= floor_cta);
             warp_offer(list, cnt, k, above && (!full || better(e[u], bar)), e[u]);
         }
     }
@@ -368,7 +368,7 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
-            const bool above = valid[u] && (float)e[u].nM / (float)e[u].T >= floor_cta;
+            const bool above = valid[u] && (floor_cta <= 0.0f || (float)e[u].nM / (float)e[u].T >= floor_cta);
             warp_offer(list, cnt, k, above && (!full || better(e[u], bar)), e[u]);
         }
     }
