@@ -193,13 +193,19 @@ cudaError_t merge_lists(const TopkArgs& a, int blocks, cudaStream_t st, int64_t*
 // CTA of a group to finish (a ticket counter after a memory fence, no
 // waiting) merges the group's lists, and the last group to finish folds
 // the group lists and the incoming state into the state, then clears the
-// tickets for the next launch.
+// tickets for the next launch.  Shorter worklists take fewer CTAs: up to
+// kOneGroupEntries one group (its last CTA folds the state at once), up to
+// kFewEntries CTA 0 alone.
 constexpr int kFusedBlock = 256;
 constexpr int kFusedGroups = 4;
 // at most this many entries (typically the survivors of the threshold once
 // a pricing's first chunks have filled the state): CTA 0 alone merges them
 // with the state and the other CTAs leave at once
 constexpr int kFewEntries = 4096;
+// at most this many (and more than kFewEntries): the first kFan CTAs scan
+// them as one group, whose last CTA folds the group's lists and the state
+// directly -- one ticket level instead of two
+constexpr int kOneGroupEntries = 32768;
 
 // Stage lists [first, first + nl) of src into lists[0 ..), one warp per
 // list; the entries were written by other CTAs, so they are read past L1.
@@ -269,7 +275,10 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     TopkEntry* list = lists + warp * kMaxTopK;
     const int64_t n = min((int64_t)*a.wl_count, (int64_t)a.wl_cap);
     const bool few = n <= kFewEntries;
+    const bool one_group = !few && n <= kOneGroupEntries;
     if (few && blockIdx.x != 0) return;
+    if (one_group && blockIdx.x >= kFan) return;
+    const int ncta = one_group ? min((int)gridDim.x, kFan) : (int)gridDim.x;  // CTAs that scan
     if (n <= 32) {
         // at most one entry per lane: warp 0 ranks them against each other
         // (the order is strict, so the ranks are distinct), places them,
@@ -323,7 +332,7 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
         }
         return;
     }
-    const int64_t step = few ? (int64_t)W * 32 : (int64_t)gridDim.x * W * 32;
+    const int64_t step = few ? (int64_t)W * 32 : (int64_t)ncta * W * 32;
     const int64_t start = few ? (int64_t)warp * 32 : ((int64_t)blockIdx.x * W + warp) * 32;
     // ---- first pass (k <= 32, while the state is not full: once it is,
     //      its k-th entry stops almost every entry): the k-th largest float
@@ -377,18 +386,21 @@ __global__ void __launch_bounds__(kFusedBlock) topk_fused_kernel(TopkArgs a) {
     int nl = 1;  // lists to fold with the incoming state
     if (!few) {
         // ---- the last CTA of its group merges the group's lists
-        const int group = blockIdx.x / kFan, ngroups = (gridDim.x + kFan - 1) / kFan;
-        const int first = group * kFan, gsize = min(kFan, (int)gridDim.x - first);
+        const int group = blockIdx.x / kFan, ngroups = (ncta + kFan - 1) / kFan;
+        const int first = group * kFan, gsize = min(kFan, ncta - first);
         if (!publish(lists, counts, a.scratch + (size_t)blockIdx.x * kMaxTopK, a.scratch_count + blockIdx.x,
                      a.tickets + group, gsize, &last_flag))
             return;
         stage_lists<W>(lists, counts, a.scratch, a.scratch_count, first, gsize, k);
         cta_tree_merge(lists, counts, tmp, tmp_counts, gsize, k);
         // ---- the last group folds the group lists and the incoming state
-        if (!publish(lists, counts, a.scratch2 + (size_t)group * kMaxTopK, a.scratch2_count + group,
-                     a.tickets + kFan, ngroups, &last_flag))
-            return;
-        stage_lists<W>(lists, counts, a.scratch2, a.scratch2_count, 0, ngroups, k);
+        //      (a single group's list is already in lists[0])
+        if (ngroups > 1) {
+            if (!publish(lists, counts, a.scratch2 + (size_t)group * kMaxTopK, a.scratch2_count + group,
+                         a.tickets + kFan, ngroups, &last_flag))
+                return;
+            stage_lists<W>(lists, counts, a.scratch2, a.scratch2_count, 0, ngroups, k);
+        }
         nl = ngroups;
     }
     const int ngroups = nl;
