@@ -12,9 +12,9 @@
 // float key (a running top-32 per warp, merged by a bitonic network); the
 // CTA's largest, lowered by a margin, drops the entries that k others beat
 // before any is offered, so a warp inserts a handful of entries instead of
-// every new best of an unsorted slice.  Then the per-CTA lists are folded into the state by merge
-// levels of 16 lists per CTA: one level for up to 16 lists, else two.  No
-// CTA waits on another.
+// every new best of an unsorted slice.  Then the per-CTA lists are folded
+// into the state by merge levels of 16 lists per CTA: one level for up to
+// 16 lists, else two.  No CTA waits on another.
 
 #include <algorithm>
 
