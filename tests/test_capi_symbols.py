@@ -66,3 +66,19 @@ def test_create_without_gpu_fails_loudly(heddle_lib):
         pytest.skip("a GPU is present")
     with pytest.raises(heddle_lib.HeddleError):
         heddle_lib.heddle_create(0)
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    # the binding has no fallback: without the built library every entry
+    # point raises instead of computing anything
+    import sys
+    code = ("from paper_2609_34244_gb300 import heddle as h\n"
+            "try:\n"
+            "    h.heddle_create(0)\n"
+            "except RuntimeError as e:\n"
+            "    print('raised:', e)\n")
+    env = dict(os.environ, HEDDLE_LIB=str(tmp_path / "libheddle.so"))
+    p = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True,
+                       timeout=300)
+    assert p.returncode == 0, p.stderr[-2000:]
+    assert "raised:" in p.stdout and "not built" in p.stdout
