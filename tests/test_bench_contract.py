@@ -1,7 +1,9 @@
-"""bench.py's reference arm (the CPU oracle on a bounded sample per step),
-run here without a GPU: one JSON line carrying the benchmark contract's
-keys, an e2e object with no copied bytes, and no output from a rank other
-than 0."""
+"""bench.py's host side, run here without a GPU: the reference arm (the CPU
+oracle on a bounded sample per step) prints one JSON line carrying the
+benchmark contract's keys and an e2e object with no copied bytes, and
+nothing on a rank other than 0; the screen's algorithmic operation count
+and the clock record's parsing (median, maximum, active throttle reasons)
+are recomputed by hand."""
 
 import json
 import os
@@ -44,3 +46,42 @@ def test_reference_arm_other_ranks_print_nothing():
              {"RANK": "1", "WORLD_SIZE": "2", "LOCAL_RANK": "1"})
     assert p.returncode == 0, p.stderr[-2000:]
     assert not p.stdout.strip()
+
+
+def _bench_module():
+    import importlib.util
+    spec = importlib.util.spec_from_file_location("bench_under_test", os.path.join(ROOT, "bench.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def test_screen_ops_counts_per_candidate_stage_type_and_pair():
+    # the screen's algorithmic count, recounted candidate by candidate
+    from paper_2609_34244_gb300 import workloads as W
+    b = _bench_module()
+    cands = W.make_workload("dense80", seed=3, n=500).cands
+    exp = 0
+    for c in range(cands["S"].shape[0]):
+        S = int(cands["S"][c])
+        codes = [int(cands["code"][s, c]) for s in range(S)]
+        exp += (b.SCREEN_OPS["candidate"] + b.SCREEN_OPS["stage"] * S
+                + b.SCREEN_OPS["type"] * len({x & 7 for x in codes})
+                + b.SCREEN_OPS["pair"] * len({x & 31 for x in codes}))
+    assert b.screen_ops(cands) == exp
+
+
+def test_clock_summary_reads_median_max_and_active_reasons(tmp_path):
+    b = _bench_module()
+    csv = tmp_path / "clocks.csv"
+    csv.write_text("0, 2070, 2070, 900.1, 0x4, Not Active, Not Active, Not Active, Active\n"
+                   "0, 1980, 2070, 950.3, 0x4, Not Active, Not Active, Not Active, Active\n"
+                   "0, 2055, 2070, 910.0, 0x0, Not Active, Active, Not Active, Not Active\n"
+                   "garbled line\n")
+    s = b.ClockSampler(0)
+    s.path = str(csv)
+    out = s.summary()
+    assert out == {"sm_mhz": 2055.0, "sm_max_mhz": 2070.0,
+                   "reasons": ["hw_thermal_slowdown", "sw_power_cap"], "samples": 3}
+    empty = b.ClockSampler(0)
+    assert empty.summary() == {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
